@@ -1,0 +1,432 @@
+#!/usr/bin/env python3
+"""Benchmark of the GB300 Frac scan (one JSON line on rank 0).
+
+Headline: the training-shaped layer step (forward + backward of the chunked scan) on
+B8 L4096 H64 P64 N128 K8 bf16 inputs, in tokens/s (whole job, all ranks).  Also
+reported: the decode step (B128 H64 P64 N128 K8, float32 state, 512-token prefill then
+1024 single-token steps) in tokens/s, per-kernel device times, the roofline fraction of
+the dominant kernel, an end-to-end number through host buffers, and the fp64 CPU oracle
+timed on a bounded sample of the same workload.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl {gb300,reference}]
+Under torchrun (N > 1) every rank runs an independent replica of the workload (the scan
+shards over batch with no exchange) and rank 0 prints the line.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "Frac scan tokens/s (prefill, fwd+bwd) and % of GB300 roofline; decode tok/s"
+TRAIN = "train_bf16_b8_l4096"
+DECODE = "decode_b128"
+FALLBACK_PEAKS = dict(hbm_gbs=6800.0, bf16_tflops=1900.0, bf16_tflops_sustained=1700.0,
+                      sm_max_mhz=2070.0)
+NUM_SMS = 152
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
+    ap.add_argument("--decode-steps", type=int, default=1024)
+    ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        p["source"] = "measured"
+        return p
+    p = dict(FALLBACK_PEAKS)
+    p["source"] = "fallback"
+    return p
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(prefix="frac_clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-i", self.gpu_id], stdout=self.out, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.out.close()
+        sm, mx, reasons = [], [], set()
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for name, v in zip(self.NAMES, parts[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(name)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def gpu_id_for(dev_index: int) -> str:
+    import torch
+    try:
+        u = str(torch.cuda.get_device_properties(dev_index).uuid)
+        return u if u.startswith("GPU-") else "GPU-" + u
+    except Exception:
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+        if vis:
+            return vis.split(",")[dev_index]
+        return str(dev_index)
+
+
+# ----------------------------------------------------------------------------- helpers
+def shape_of(name):
+    from paper_2609_36314_gb300 import synth
+    return synth.WORKLOADS[name]
+
+
+def kpn(s):
+    return s.nmodes * s.headdim * s.dstate
+
+
+def algorithmic_work(kernel: str, s, per_launch_units: float):
+    """Algorithmic flops or bytes of one launch of `kernel` (see the measurement section of
+    the design notes): state contractions count 2 K P N flops per token-head each."""
+    per_th = {
+        "state_pass_fwd_simt": 2, "state_pass_rev_simt": 2, "chunk_fwd_simt": 2,
+        "chunk_bwd_simt": 8,
+    }
+    if kernel in per_th:
+        return "flops", per_th[kernel] * kpn(s) * per_launch_units
+    if kernel == "decode_step":
+        return "bytes", 2.0 * 4 * kpn(s) * per_launch_units
+    return None, None
+
+
+def run_reference(args, rank):
+    """The fp64 CPU oracle on a bounded sample of the training workload, per step."""
+    if rank != 0:
+        return
+    from oracle import oracle
+    from paper_2609_36314_gb300 import synth
+    s = shape_of(TRAIN)
+    heads = 4
+    sub = s.replace(batch=1, nheads=heads)
+    host = synth.make_scan_inputs(sub, seed=0, with_dy=True)
+    d = {k: synth.to_f64(v) for k, v in host.items()}
+
+    def step():
+        oracle.fwd(d["x"], d["dt"], d["alpha"], d["lam"], d["tau"], d["B"], d["C"],
+                   d["w_read"], d["w_write"], d["D"])
+        oracle.bwd(d["x"], d["dt"], d["alpha"], d["lam"], d["tau"], d["B"], d["C"],
+                   d["w_read"], d["w_write"], d["D"], d["dy"])
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = time.perf_counter() - t0
+    tokens = sub.seqlen * heads / s.nheads  # token-heads of the sample in full-layer tokens
+    value = tokens * args.steps / dt
+    cores = oracle.max_threads()
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"{TRAIN} sample: batch row 0, heads 0-{heads - 1}, L={s.seqlen}, "
+                               "fwd+bwd", "global_batch": 1, "seq_len": s.seqlen},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                         "sample": f"1 x {s.seqlen} tokens x {heads}/{s.nheads} heads per step"},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def cpu_baseline(heads=16):
+    from oracle import oracle
+    from paper_2609_36314_gb300 import synth
+    s = shape_of(TRAIN)
+    sub = s.replace(batch=1, nheads=heads)
+    host = synth.make_scan_inputs(sub, seed=1, with_dy=True)
+    d = {k: synth.to_f64(v) for k, v in host.items()}
+    t0 = time.perf_counter()
+    oracle.fwd(d["x"], d["dt"], d["alpha"], d["lam"], d["tau"], d["B"], d["C"], d["w_read"],
+               d["w_write"], d["D"])
+    oracle.bwd(d["x"], d["dt"], d["alpha"], d["lam"], d["tau"], d["B"], d["C"], d["w_read"],
+               d["w_write"], d["D"], d["dy"])
+    dt = time.perf_counter() - t0
+    tokens = sub.seqlen * heads / s.nheads
+    return {"value": tokens / dt, "unit": "tokens/s", "cores": oracle.max_threads(),
+            "kind": "oracle",
+            "sample": f"fwd+bwd of batch row 0, heads 0-{heads - 1}, L={s.seqlen} "
+                      f"({heads}/{s.nheads * s.batch} of the (batch, head) streams), "
+                      f"{dt:.1f} s"}
+
+
+# ----------------------------------------------------------------------------- GPU arm
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank)
+        return
+
+    import torch
+    import torch.distributed as dist
+
+    from paper_2609_36314_gb300 import _lib, scan_bwd, scan_fwd, synth
+    from paper_2609_36314_gb300.api import bwd_workspace_size, fwd_workspace_size, make_dims
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", rank=rank, world_size=world, device_id=dev)
+    peaks = load_peaks()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    def max_over_ranks(v):
+        if world == 1:
+            return v
+        t = torch.tensor([v], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    s = shape_of(TRAIN)
+    inp = synth.make_scan_inputs_torch(s, seed=1000 + rank, device=dev, with_dy=True)
+    dims = make_dims(s.batch, s.seqlen, s.nheads, s.headdim, s.ngroups, s.dstate, s.nmodes,
+                     torch.bfloat16)
+    ws_f = torch.empty(fwd_workspace_size(dims), dtype=torch.uint8, device=dev)
+    ws_b = torch.empty(bwd_workspace_size(dims), dtype=torch.uint8, device=dev)
+    y = torch.empty_like(inp["x"])
+    grads = dict(dx=torch.empty_like(inp["x"]), ddt=torch.empty_like(inp["dt"]),
+                 dalpha=torch.empty_like(inp["alpha"]), dlam=torch.empty_like(inp["lam"]),
+                 dB=torch.empty_like(inp["B"]), dC=torch.empty_like(inp["C"]),
+                 dw_read=torch.empty_like(inp["w_read"]), dw_write=torch.empty_like(inp["w_write"]),
+                 dD=torch.empty_like(inp["D"]), dh0=None)
+    a = inp
+
+    def train_step():
+        scan_fwd(a["x"], a["dt"], a["alpha"], a["lam"], a["tau"], a["B"], a["C"], a["w_read"],
+                 a["w_write"], a["D"], want_final_state=False, y=y, workspace=ws_f)
+        scan_bwd(a["x"], a["dt"], a["alpha"], a["lam"], a["tau"], a["B"], a["C"], a["w_read"],
+                 a["w_write"], a["D"], a["dy"], workspace=ws_b, out=grads)
+
+    for _ in range(max(args.warmup, 3)):
+        train_step()
+    torch.cuda.synchronize()
+
+    clocks = ClockSampler(gpu_id_for(local)) if rank == 0 else None
+    if clocks:
+        clocks.start()
+    _lib.trace_reset()
+    _lib.trace_enable(True)
+    barrier()
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        train_step()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    _lib.trace_enable(False)
+    ms = ev0.elapsed_time(ev1) / args.steps
+    trace = _lib.trace_collect()
+    clk = clocks.stop() if clocks else None
+    ms_max = max_over_ranks(ms)
+    tokens_per_step = s.batch * s.seqlen
+    value = world * tokens_per_step / (ms_max / 1e3)
+
+    # per-kernel device time and the dominant kernel's roofline
+    kern = {k: {"launches": n, "avg_ms": t / max(n, 1), "share": 0.0} for k, (n, t) in trace.items()}
+    tot = sum(t for _, t in trace.values()) or 1.0
+    for k, (n, t) in trace.items():
+        kern[k]["share"] = t / tot
+    launches = sum(n for n, _ in trace.values())
+    dom = max(trace.items(), key=lambda kv: kv[1][1])[0] if trace else None
+    roofline = None
+    if dom:
+        kind, work = algorithmic_work(dom, s, s.batch * s.seqlen * s.nheads)
+        avg_s = kern[dom]["avg_ms"] / 1e3
+        if kind == "flops":
+            # CUDA-core float32 FMA peak: SMs x 128 lanes x 2 flops x max SM clock
+            peak = NUM_SMS * 128 * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+            ach = work / avg_s / 1e12
+            roofline = {"kernel": dom, "bound": "alu", "achieved": ach, "peak": peak,
+                        "unit": "TFLOP/s", "frac": ach / peak, "traffic": None,
+                        "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 x max SM clock"}
+        elif kind == "bytes":
+            ach = work / avg_s / 1e9
+            roofline = {"kernel": dom, "bound": "hbm", "achieved": ach,
+                        "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                        "frac": ach / peaks["hbm_gbs"], "traffic": None,
+                        "peak_source": peaks["source"]}
+
+    # end to end through host buffers (pinned), copies inside the timed region
+    e2e = None
+    if not args.no_e2e:
+        hin = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True).copy_(v)
+               for k, v in inp.items()}
+        hout = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True)
+                for k, v in grads.items() if v is not None}
+        hout["y"] = torch.empty(y.shape, dtype=y.dtype, pin_memory=True)
+        h2d = sum(v.numel() * v.element_size() for v in hin.values())
+        d2h = sum(v.numel() * v.element_size() for v in hout.values())
+
+        def e2e_step():
+            for k, v in hin.items():
+                inp[k].copy_(v, non_blocking=True)
+            train_step()
+            for k, v in hout.items():
+                v.copy_(grads[k] if k != "y" else y, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize()
+        barrier()
+        ev0.record(stream)
+        n_e2e = max(2, args.steps // 2)
+        for _ in range(n_e2e):
+            e2e_step()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        ms_e2e = max_over_ranks(ev0.elapsed_time(ev1) / n_e2e)
+        e2e = {"value": world * tokens_per_step / (ms_e2e / 1e3), "unit": "tokens/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e}
+        del hin, hout
+
+    decode = None
+    if not args.no_decode:
+        decode = bench_decode(args, dev, peaks, world, max_over_ranks, barrier)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f32", "data": "synthetic",
+            "config": {"workload": f"{TRAIN}: forward + backward of the chunked scan, B{s.batch} "
+                                   f"L{s.seqlen} H{s.nheads} P{s.headdim} N{s.dstate} "
+                                   f"K{s.nmodes} G{s.ngroups}, bf16 inputs, float32 arithmetic",
+                       "global_batch": s.batch * world, "seq_len": s.seqlen,
+                       "parallelism": f"replicas{world}" if world > 1 else "single",
+                       "l2": "inputs larger than L2 (0.78 GB per step), no flush"},
+            "roofline": roofline, "kernels": kern, "gpu_launches": launches,
+            "e2e": e2e, "decode": decode, "clocks": clk, "peaks_source": peaks["source"],
+        }
+        if world == 1 and not args.no_cpu_baseline:
+            line["cpu_baseline"] = cpu_baseline()
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def bench_decode(args, dev, peaks, world, max_over_ranks, barrier):
+    import torch
+
+    from paper_2609_36314_gb300 import decode_step, scan_fwd, synth
+    s = shape_of(DECODE)
+    pre = synth.make_scan_inputs_torch(s, seed=7, device=dev)
+    _, state = scan_fwd(pre["x"], pre["dt"], pre["alpha"], pre["lam"], pre["tau"], pre["B"],
+                        pre["C"], pre["w_read"], pre["w_write"], pre["D"])
+    del pre
+    T = args.decode_steps
+    stp = synth.make_scan_inputs_torch(s.replace(seqlen=T), seed=8, device=dev)
+    # [B, T, ...] -> [T, B, ...] so that every step reads contiguous inputs
+    stp = {k: (v.transpose(0, 1).contiguous() if k not in ("tau", "D") else v)
+           for k, v in stp.items()}
+    ybuf = torch.empty((T, s.batch, s.nheads, s.headdim), dtype=torch.bfloat16, device=dev)
+
+    def steps():
+        for t in range(T):
+            decode_step(stp["x"][t], stp["dt"][t], stp["alpha"][t], stp["lam"][t], stp["tau"],
+                        stp["B"][t], stp["C"][t], stp["w_read"][t], stp["w_write"][t],
+                        stp["D"], state, y_t=ybuf[t])
+
+    steps()  # warm-up
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        steps()
+    g.replay()
+    torch.cuda.synchronize()
+    barrier()
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = 2
+    e0.record(stream)
+    for _ in range(reps):
+        g.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    ms_step = max_over_ranks(e0.elapsed_time(e1) / (reps * T))
+    state_bytes = 2.0 * 4 * s.batch * s.nheads * kpn(s)
+    gbs = state_bytes / (ms_step / 1e3) / 1e9
+    return {"workload": f"{DECODE}: B{s.batch} H{s.nheads} P{s.headdim} N{s.dstate} K{s.nmodes}, "
+                        f"float32 state, 512-token prefill then {T} steps in one CUDA graph",
+            "value": world * s.batch / (ms_step / 1e3), "unit": "tokens/s",
+            "us_per_step": 1e3 * ms_step,
+            "roofline": {"kernel": "decode_step", "bound": "hbm", "achieved": gbs,
+                         "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                         "frac": gbs / peaks["hbm_gbs"], "traffic": None,
+                         "peak_source": peaks["source"]}}
+
+
+if __name__ == "__main__":
+    main()

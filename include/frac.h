@@ -1,0 +1,179 @@
+/*
+ * frac.h -- C ABI of the GB300 (sm_103a) Frac selective fractional state-space scan.
+ *
+ * The layer (arXiv 2609.36314, Sec. 3.2 and Algorithm 1 of App. D), with the mode
+ * state lifted to an N-dimensional outer product per head (N = 1, B = C = 1 is
+ * Algorithm 1 itself):
+ *
+ *   e_t        = Delta_t * lambda_t^(1/alpha_t)                (Eq. tau-eff: tau~ = tau / lambda^(1/alpha))
+ *   rho_{t,m}  = exp(-e_t / tau_m)                             (Eq. rho-beta-def-frac)
+ *   kappa_{t,m}= (1 - rho_{t,m}) * w_write_{t,m}               (Algorithm 1 steps 3 and 6; the remark after it)
+ *   S_{t,m}    = rho_{t,m} S_{t-1,m} + kappa_{t,m} x_t B_t^T   (Eq. frac-selective-update; S_{t,m} is P x N)
+ *   y_t        = sum_m w_read_{t,m} S_{t,m} C_t + D x_t        (Eq. frac-readout; skip D u_t of Sec. 3.3)
+ *
+ * w_read / w_write are the already-normalised read and write mode weights of
+ * Eq. read-softmax (computed upstream).  Head h reads B/C group g = h / (H / G).
+ *
+ * Conventions shared by every entry point
+ *   - Tensor arguments are device pointers owned by the caller, row-major and contiguous,
+ *     16-byte aligned, and must not alias each other (except where stated).  The library
+ *     never allocates device memory and keeps no state between calls apart from a
+ *     thread-local error message.
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream).  Every call only
+ *     enqueues work on `stream`; results are valid once the stream has completed.
+ *   - Element types: x, B, C, w_read, w_write, y and their gradients use `dims->dtype`
+ *     (FRAC_DTYPE_F32 or FRAC_DTYPE_BF16).  Delta, alpha, lambda, tau, D, all mode states
+ *     (h0, h_final, state, dh_final, dh0) and the gradients of Delta, alpha, lambda, D are
+ *     always float32.  Arithmetic is float32 (tensor-core products take bf16 operands with
+ *     float32 accumulation on the bf16 path).
+ *   - Controls must satisfy Delta > 0, 0 < alpha <= 1, lambda > 0, tau > 0.  e_t is clamped
+ *     to 64 * max_m tau_{h,m} (every mode's retention is then <= e^-64); the gradient of a
+ *     clamped e_t is zero.
+ *   - Return values: FRAC_OK, or FRAC_ERR_INVALID_ARGUMENT (bad dims, NULL or misaligned
+ *     pointer, workspace too small) and FRAC_ERR_UNSUPPORTED (a shape the kernels do not
+ *     handle) before anything is enqueued, or FRAC_ERR_CUDA if a launch failed.
+ *     frac_last_error() then holds a readable reason for the calling thread.
+ *
+ * Layouts
+ *   x, y, dy, dx             [batch, seqlen, nheads, headdim]
+ *   dt, alpha, lam (+grads)  [batch, seqlen, nheads]               float32
+ *   Bm, Cm (+grads)          [batch, seqlen, ngroups, dstate]
+ *   w_read, w_write (+grads) [batch, seqlen, nheads, nmodes]
+ *   tau                      [nheads, nmodes]                       float32
+ *   D, dD                    [nheads]                               float32
+ *   h0, h_final, dh_final, dh0, state   [batch, nheads, nmodes, headdim, dstate]   float32
+ */
+#ifndef FRAC_H_
+#define FRAC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    FRAC_OK = 0,
+    FRAC_ERR_INVALID_ARGUMENT = 1,
+    FRAC_ERR_UNSUPPORTED = 2,
+    FRAC_ERR_CUDA = 3,
+    FRAC_ERR_TIMEOUT = 4
+} frac_status;
+
+typedef enum { FRAC_DTYPE_F32 = 0, FRAC_DTYPE_BF16 = 1 } frac_dtype;
+
+/* Bits of frac_dims.flags. */
+enum {
+    FRAC_FLAG_FORCE_SIMT = 1 /* use the CUDA-core chunked kernels even where tensor-core ones exist */
+};
+
+typedef struct {
+    int64_t batch;   /* B >= 1 */
+    int64_t seqlen;  /* L >= 0 (ignored by frac_decode_step) */
+    int64_t nheads;  /* H >= 1 */
+    int64_t headdim; /* P >= 1 */
+    int64_t ngroups; /* G >= 1, H % G == 0 */
+    int64_t dstate;  /* N >= 1 */
+    int64_t nmodes;  /* K, 1 <= K <= 32 */
+    int64_t chunk;   /* Q: 0 = implementation's choice; otherwise one of the sizes the selected
+                        path supports (16, 32 or 64 on CUDA cores, 128 on tensor cores).
+                        Results do not depend on Q beyond rounding. */
+    int32_t dtype;   /* frac_dtype */
+    int32_t flags;   /* FRAC_FLAG_* */
+} frac_dims;
+
+/*
+ * Bytes of scratch device memory frac_scan_fwd needs for these dims (per-chunk mode states
+ * handed from the chunk-serial state pass to the chunk-parallel output kernel).
+ */
+frac_status frac_scan_fwd_workspace_size(const frac_dims *dims, size_t *bytes);
+
+/*
+ * Chunked parallel forward scan (training / prefill), the Remark after Eq. read-softmax:
+ * the affine recurrence evaluated chunk by chunk with chunk-local cumulative log-decays,
+ * the stable intra-chunk coefficient Gamma of App. E, cross-chunk state passing, and the
+ * skip D fused into the output.
+ *   x, dt, alpha, lam, tau, Bm, Cm, w_read, w_write, D : inputs (layouts above)
+ *   h0       : initial mode state, or NULL for zeros
+ *   y        : output [B, L, H, P] (dtype)
+ *   h_final  : final mode state S_L (float32), or NULL; it is the decode cache
+ *   workspace: >= frac_scan_fwd_workspace_size bytes, 256-byte aligned; contents undefined on
+ *              entry and exit; must not be used concurrently by another call.
+ */
+frac_status frac_scan_fwd(const frac_dims *dims, const void *x, const float *dt,
+                          const float *alpha, const float *lam, const float *tau,
+                          const void *Bm, const void *Cm, const void *w_read,
+                          const void *w_write, const float *D, const float *h0, void *y,
+                          float *h_final, void *workspace, size_t workspace_bytes,
+                          void *stream);
+
+/* Bytes of scratch device memory frac_scan_bwd needs for these dims. */
+frac_status frac_scan_bwd_workspace_size(const frac_dims *dims, size_t *bytes);
+
+/*
+ * Backward of frac_scan_fwd (the adjoint of the recurrence; the paper trains through it but
+ * prints no formulas).  Recomputes the forward mode states from the inputs, then walks the
+ * chunks in reverse carrying dS, and forms every gradient chunk-locally.  The gradient through
+ * the decay, rho_t <dS_t, S_{t-1}>, is evaluated per position from terms that each carry their
+ * own decay factor, so it stays accurate when lambda^(1/alpha) is large.
+ *   dy       : upstream gradient of y (dtype)
+ *   dh_final : upstream gradient of h_final (float32), or NULL for zeros
+ *   dx, dB, dC, dw_read, dw_write : gradients (dtype, layouts of their inputs)
+ *   ddt, dalpha, dlam : gradients (float32)
+ *   dD       : gradient of D (float32 [H]), summed over batch and sequence
+ *   dh0      : gradient of h0 (float32), or NULL if not wanted
+ * dB / dC sum over the heads of each group.  All outputs are overwritten (not accumulated).
+ */
+frac_status frac_scan_bwd(const frac_dims *dims, const void *x, const float *dt,
+                          const float *alpha, const float *lam, const float *tau,
+                          const void *Bm, const void *Cm, const void *w_read,
+                          const void *w_write, const float *D, const float *h0,
+                          const void *dy, const float *dh_final, void *dx, float *ddt,
+                          float *dalpha, float *dlam, void *dB, void *dC, void *dw_read,
+                          void *dw_write, float *dD, float *dh0, void *workspace,
+                          size_t workspace_bytes, void *stream);
+
+/*
+ * One decode step (Algorithm 1: a single token, recurrent form with the cached state):
+ * updates every mode of `state` in place and writes y_t.  One pass over the state.
+ *   x_t [B, H, P], B_t/C_t [B, G, N], w_read/w_write [B, H, K] : dtype
+ *   dt, alpha, lam [B, H], tau [H, K], D [H] : float32
+ *   state [B, H, K, P, N] float32, read and written (may not alias any other argument)
+ *   y_t   [B, H, P] : dtype
+ * dims->seqlen and dims->chunk are ignored.
+ */
+frac_status frac_decode_step(const frac_dims *dims, const void *x_t, const float *dt,
+                             const float *alpha, const float *lam, const float *tau,
+                             const void *B_t, const void *C_t, const void *w_read,
+                             const void *w_write, const float *D, float *state, void *y_t,
+                             void *stream);
+
+/*
+ * Kernel tracing (a profiling aid, off by default).  While enabled, every kernel the library
+ * launches is bracketed by two CUDA events recorded on its launch stream (do not enable it
+ * while a stream is being captured into a CUDA graph).  frac_trace_collect waits for the
+ * recorded events and returns, per kernel name, the launch count and summed device time since
+ * the last frac_trace_reset; it writes at most `capacity` entries and the total in *count.
+ */
+typedef struct {
+    char name[64];
+    int32_t launches;
+    double total_ms;
+} frac_trace_entry;
+
+frac_status frac_trace_enable(int on);
+frac_status frac_trace_collect(frac_trace_entry *out, int capacity, int *count);
+frac_status frac_trace_reset(void);
+
+/* Static description of a status code. */
+const char *frac_status_string(frac_status status);
+
+/* Detail of the last failure on the calling thread ("" if none). */
+const char *frac_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FRAC_H_ */

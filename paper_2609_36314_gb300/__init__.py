@@ -1,0 +1,11 @@
+"""GB300-native (sm_103a) Frac selective fractional state-space scan (arXiv 2609.36314).
+
+The scan runs in hand-written CUDA kernels behind the C ABI of include/frac.h
+(libfrac.so, built in-tree); this package only marshals torch tensors to it.
+"""
+from .api import (bwd_workspace_size, decode_step, fwd_workspace_size, make_dims, scan_bwd,
+                  scan_fwd)
+from ._lib import FracError
+
+__all__ = ["scan_fwd", "scan_bwd", "decode_step", "fwd_workspace_size", "bwd_workspace_size",
+           "make_dims", "FracError"]

@@ -1,0 +1,169 @@
+"""Python binding of the Frac scan C ABI (argument marshalling only).
+
+PyTorch provides device memory and the current CUDA stream; every step of the scan
+runs in libfrac.so.  Tensors must be CUDA, contiguous, in the dtypes include/frac.h
+states (x, B, C, w_read, w_write, y and their gradients in one dtype: float32 or
+bfloat16; controls, tau, D and mode states float32).
+"""
+from __future__ import annotations
+
+import ctypes
+
+import torch
+
+from . import _lib
+
+_DT = {torch.float32: _lib.FRAC_DTYPE_F32, torch.bfloat16: _lib.FRAC_DTYPE_BF16}
+
+
+def make_dims(batch, seqlen, nheads, headdim, ngroups, dstate, nmodes, dtype, chunk=0,
+              force_simt=False) -> _lib.FracDims:
+    return _lib.FracDims(batch, seqlen, nheads, headdim, ngroups, dstate, nmodes, chunk,
+                         _DT[dtype], _lib.FRAC_FLAG_FORCE_SIMT if force_simt else 0)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _need(t, name, dtype, shape=None):
+    if t is None:
+        raise ValueError(f"{name} is required")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+    return t
+
+
+def _scan_dims(x, B, tau, chunk, force_simt):
+    if x.dim() != 4 or B.dim() != 4 or tau.dim() != 2:
+        raise ValueError("x [B,L,H,P], B/C [B,L,G,N], tau [H,K] expected")
+    Bz, L, H, P = x.shape
+    G, N = B.shape[2], B.shape[3]
+    K = tau.shape[1]
+    return make_dims(Bz, L, H, P, G, N, K, x.dtype, chunk, force_simt), (Bz, L, H, P, G, N, K)
+
+
+def fwd_workspace_size(dims: _lib.FracDims) -> int:
+    n = ctypes.c_size_t(0)
+    _lib.check(_lib.load().frac_scan_fwd_workspace_size(ctypes.byref(dims), ctypes.byref(n)),
+               "frac_scan_fwd_workspace_size")
+    return int(n.value)
+
+
+def bwd_workspace_size(dims: _lib.FracDims) -> int:
+    n = ctypes.c_size_t(0)
+    _lib.check(_lib.load().frac_scan_bwd_workspace_size(ctypes.byref(dims), ctypes.byref(n)),
+               "frac_scan_bwd_workspace_size")
+    return int(n.value)
+
+
+def _workspace(nbytes, device, given):
+    if given is not None:
+        if given.numel() * given.element_size() < nbytes:
+            raise ValueError("workspace too small")
+        return given
+    return torch.empty(max(nbytes, 1), dtype=torch.uint8, device=device)
+
+
+def scan_fwd(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, h0=None, *, chunk=0,
+             force_simt=False, want_final_state=True, y=None, h_final=None, workspace=None,
+             stream=None):
+    """Chunked forward scan.  Returns (y [B,L,H,P], h_final [B,H,K,P,N] or None)."""
+    dims, (Bz, L, H, P, G, N, K) = _scan_dims(x, B, tau, chunk, force_simt)
+    dt_ = x.dtype
+    f32 = torch.float32
+    _need(x, "x", dt_, (Bz, L, H, P))
+    for name, t in (("dt", dt), ("alpha", alpha), ("lam", lam)):
+        _need(t, name, f32, (Bz, L, H))
+    _need(tau, "tau", f32, (H, K))
+    _need(B, "B", dt_, (Bz, L, G, N))
+    _need(C, "C", dt_, (Bz, L, G, N))
+    _need(w_read, "w_read", dt_, (Bz, L, H, K))
+    _need(w_write, "w_write", dt_, (Bz, L, H, K))
+    _need(D, "D", f32, (H,))
+    if h0 is not None:
+        _need(h0, "h0", f32, (Bz, H, K, P, N))
+    if y is None:
+        y = torch.empty_like(x)
+    if want_final_state and h_final is None:
+        h_final = torch.empty((Bz, H, K, P, N), dtype=f32, device=x.device)
+    ws = _workspace(fwd_workspace_size(dims), x.device, workspace)
+    _lib.check(_lib.load().frac_scan_fwd(
+        ctypes.byref(dims), _ptr(x), _ptr(dt), _ptr(alpha), _ptr(lam), _ptr(tau), _ptr(B),
+        _ptr(C), _ptr(w_read), _ptr(w_write), _ptr(D), _ptr(h0), _ptr(y),
+        _ptr(h_final if want_final_state else None), _ptr(ws), ws.numel(), _stream(stream)),
+        "frac_scan_fwd")
+    return y, (h_final if want_final_state else None)
+
+
+def scan_bwd(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, dy, h0=None, dh_final=None, *,
+             chunk=0, force_simt=False, want_dh0=True, workspace=None, out=None, stream=None):
+    """Backward of scan_fwd.  Returns a dict of gradients (dx, ddt, dalpha, dlam, dB, dC,
+    dw_read, dw_write, dD, dh0)."""
+    dims, (Bz, L, H, P, G, N, K) = _scan_dims(x, B, tau, chunk, force_simt)
+    dt_ = x.dtype
+    f32 = torch.float32
+    _need(dy, "dy", dt_, (Bz, L, H, P))
+    if dh_final is not None:
+        _need(dh_final, "dh_final", f32, (Bz, H, K, P, N))
+    if h0 is not None:
+        _need(h0, "h0", f32, (Bz, H, K, P, N))
+    for name, t in (("x", x), ("B", B), ("C", C), ("w_read", w_read), ("w_write", w_write)):
+        _need(t, name, dt_)
+    for name, t in (("dt", dt), ("alpha", alpha), ("lam", lam), ("tau", tau), ("D", D)):
+        _need(t, name, f32)
+    g = out if out is not None else dict(
+        dx=torch.empty_like(x), ddt=torch.empty_like(dt), dalpha=torch.empty_like(alpha),
+        dlam=torch.empty_like(lam), dB=torch.empty_like(B), dC=torch.empty_like(C),
+        dw_read=torch.empty_like(w_read), dw_write=torch.empty_like(w_write),
+        dD=torch.empty_like(D),
+        dh0=torch.empty((Bz, H, K, P, N), dtype=f32, device=x.device) if want_dh0 else None)
+    ws = _workspace(bwd_workspace_size(dims), x.device, workspace)
+    _lib.check(_lib.load().frac_scan_bwd(
+        ctypes.byref(dims), _ptr(x), _ptr(dt), _ptr(alpha), _ptr(lam), _ptr(tau), _ptr(B),
+        _ptr(C), _ptr(w_read), _ptr(w_write), _ptr(D), _ptr(h0), _ptr(dy), _ptr(dh_final),
+        _ptr(g["dx"]), _ptr(g["ddt"]), _ptr(g["dalpha"]), _ptr(g["dlam"]), _ptr(g["dB"]),
+        _ptr(g["dC"]), _ptr(g["dw_read"]), _ptr(g["dw_write"]), _ptr(g["dD"]),
+        _ptr(g.get("dh0")), _ptr(ws), ws.numel(), _stream(stream)), "frac_scan_bwd")
+    return g
+
+
+def decode_step(x_t, dt, alpha, lam, tau, B_t, C_t, w_read, w_write, D, state, y_t=None,
+                stream=None):
+    """One decode step: updates `state` in place and returns y_t [B,H,P]."""
+    if x_t.dim() != 3 or B_t.dim() != 3:
+        raise ValueError("x_t [B,H,P], B_t/C_t [B,G,N] expected")
+    Bz, H, P = x_t.shape
+    G, N = B_t.shape[1], B_t.shape[2]
+    K = tau.shape[1]
+    dt_ = x_t.dtype
+    f32 = torch.float32
+    _need(x_t, "x_t", dt_)
+    _need(B_t, "B_t", dt_, (Bz, G, N))
+    _need(C_t, "C_t", dt_, (Bz, G, N))
+    _need(w_read, "w_read", dt_, (Bz, H, K))
+    _need(w_write, "w_write", dt_, (Bz, H, K))
+    for name, t in (("dt", dt), ("alpha", alpha), ("lam", lam)):
+        _need(t, name, f32, (Bz, H))
+    _need(tau, "tau", f32, (H, K))
+    _need(D, "D", f32, (H,))
+    _need(state, "state", f32, (Bz, H, K, P, N))
+    if y_t is None:
+        y_t = torch.empty_like(x_t)
+    dims = make_dims(Bz, 1, H, P, G, N, K, dt_)
+    _lib.check(_lib.load().frac_decode_step(
+        ctypes.byref(dims), _ptr(x_t), _ptr(dt), _ptr(alpha), _ptr(lam), _ptr(tau), _ptr(B_t),
+        _ptr(C_t), _ptr(w_read), _ptr(w_write), _ptr(D), _ptr(state), _ptr(y_t),
+        _stream(stream)), "frac_decode_step")
+    return y_t

@@ -1,0 +1,47 @@
+// Internal interface between the C-ABI layer and the kernels (not installed).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace frac {
+
+// Tracing hooks (no-ops unless frac_trace_enable(1)); bracket each kernel launch.
+void trace_begin(const char *name, cudaStream_t st);
+void trace_end(cudaStream_t st);
+
+struct DecodeArgs {
+    int B, H, P, G, N, K;
+    const float *dt, *alpha, *lam, *tau, *D;
+    float *state;
+};
+
+cudaError_t launch_decode(const DecodeArgs &a, int dtype, const void *x, const void *Bt,
+                          const void *Ct, const void *wr, const void *ww, void *y,
+                          cudaStream_t st);
+
+// Problem dimensions as the chunked kernels see them.
+struct ScanDims {
+    int B, L, H, P, G, N, K;
+    int Q;   // chunk length
+    int nc;  // number of chunks = ceil(L / Q)
+};
+
+// Pointers of one scan call.  Element types follow the dtype of the call.
+struct ScanPtrs {
+    const void *x, *Bm, *Cm, *wr, *ww, *dy;
+    const float *dt, *alpha, *lam, *tau, *D, *h0, *dh_final;
+    void *y, *dx, *dB, *dC, *dwr, *dww;
+    float *h_final, *ddt, *dalpha, *dlam, *dD, *dh0;
+};
+
+// CUDA-core (SIMT) chunked path; works for float32 and bf16 I/O.
+int simt_pick_chunk(const ScanDims &d, int requested);     // 0 if the shape is unsupported
+size_t simt_state_elems(const ScanDims &d);                 // per-chunk state workspace elements
+cudaError_t simt_scan_fwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in,
+                          cudaStream_t st);
+cudaError_t simt_scan_bwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in,
+                          void *dS_out, float *dB_acc, float *dC_acc, cudaStream_t st);
+
+}  // namespace frac

@@ -1,0 +1,939 @@
+// CUDA-core (SIMT) chunked Frac scan: forward and backward, float32 arithmetic.
+//
+// The chunked evaluation order (App. E of the paper; the Remark after Eq. read-softmax):
+// per chunk of Q positions, E_t = sum of e_j = Delta_j lambda_j^(1/alpha_j) from the chunk
+// start through t (kept in double so that differences E_t - E_k are exact to float
+// precision even when e_j is huge), so that the log of the product of retentions from k+1
+// to t in mode m is -(E_t - E_k) / tau_m.
+//
+//   state pass (chunk-serial per (b, h, p-slice)):  S_out,m = d_m S_in,m + sum_k s_{k,m} x_k B_k^T
+//        d_m = exp(-E_end / tau_m),  s_{k,m} = kappa_{k,m} exp(-(E_end - E_k) / tau_m)
+//        emits S_in of every chunk into the workspace; the same kernel run over the chunks in
+//        reverse with (dy, C, f_{t,m} = w_read_{t,m} exp(-E_t / tau_m)) carries dS backwards.
+//   chunk output (chunk-parallel per (b, h, c)):
+//        y_t = sum_m f_{t,m} S_in,m C_t + sum_{k<=t} Gamma_{t,k} (C_t . B_k) x_k + D x_t
+//        Gamma_{t,k} = sum_m w_read_{t,m} kappa_{k,m} exp(-(E_t - E_k) / tau_m)   (App. E)
+//   chunk backward (chunk-parallel per (b, h, c)): every gradient from x, dy, B, C, the mode
+//        weights, S_in and dS_out of the chunk (see the comments in simt_chunk_bwd).
+//
+// Threads own register tiles of the small per-chunk contractions; shared-memory rows are
+// padded by one float so that both row and column walks are free of bank conflicts.
+#include <algorithm>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace frac {
+namespace {
+
+constexpr int kQMax = 64;
+constexpr int kThreads = 256;
+
+template <typename TS> __device__ __forceinline__ TS cvt_state(float v);
+template <> __device__ __forceinline__ float cvt_state<float>(float v) { return v; }
+template <> __device__ __forceinline__ __nv_bfloat16 cvt_state<__nv_bfloat16>(float v) {
+    return __float2bfloat16_rn(v);
+}
+
+__device__ __forceinline__ size_t blh(const ScanDims &d, int b, int t, int h) {
+    return (size_t(b) * d.L + t) * d.H + h;
+}
+
+// e_t of positions [c0, c0 + n) of head h and their in-chunk inclusive prefix sums (double).
+// Executed by warp 0.
+__device__ void chunk_rates(const ScanDims &d, int b, int h, int c0, int n, float log_cap,
+                            const float *__restrict__ dt, const float *__restrict__ alpha,
+                            const float *__restrict__ lam, float *e_s, double *E_s,
+                            float *clamp_s) {
+    if (threadIdx.x >= 32) return;
+    const int lane = threadIdx.x;
+    double carry = 0.0;
+    for (int base = 0; base < n; base += 32) {
+        const int t = base + lane;
+        float e = 0.f;
+        bool cl = false;
+        if (t < n) {
+            const size_t i = blh(d, b, c0 + t, h);
+            e = token_rate(dt[i], alpha[i], lam[i], log_cap, &cl);
+        }
+        double v = warp_inclusive_scan_d(double(e)) + carry;
+        if (t < n) {
+            e_s[t] = e;
+            E_s[t] = v;
+            if (clamp_s) clamp_s[t] = cl ? 1.f : 0.f;
+        }
+        carry = __shfl_sync(0xffffffffu, v, 31);
+    }
+}
+
+__device__ __forceinline__ float head_log_cap(const float *__restrict__ tau, int h, int K) {
+    float tmax = 0.f;
+    for (int j = 0; j < K; ++j) tmax = fmaxf(tmax, tau[h * K + j]);
+    return logf(64.f * tmax);
+}
+
+__device__ float block_sum(float v, float *red) {
+    v = warp_sum(v);
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    __syncthreads();
+    if (lane == 0) red[w] = v;
+    __syncthreads();
+    float s = 0.f;
+    if (threadIdx.x < 32) {
+        s = (lane < int(blockDim.x >> 5)) ? red[lane] : 0.f;
+        s = warp_sum(s);
+        if (lane == 0) red[0] = s;
+    }
+    __syncthreads();
+    s = red[0];
+    __syncthreads();
+    return s;
+}
+
+// ---------------------------------------------------------------------------------------------
+// State pass.  REV = false: forward (U = x, V = B, W = w_write, coefficient s).
+//              REV = true : backward (U = dy, V = C, W = w_read, coefficient f), chunks reversed.
+// Thread tile: one mode m, 8 consecutive p, 4 consecutive n of the CTA's p-slice.
+template <typename T, typename TS, bool REV>
+__global__ void __launch_bounds__(512) simt_state_pass(
+    ScanDims d, int Ps, const T *__restrict__ U, const T *__restrict__ V,
+    const T *__restrict__ W, const float *__restrict__ dt, const float *__restrict__ alpha,
+    const float *__restrict__ lam, const float *__restrict__ tau, const float *__restrict__ init,
+    TS *__restrict__ emit, float *__restrict__ fin) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int b = blockIdx.z, h = blockIdx.y, pbase = blockIdx.x * Ps;
+    const int g = h / (d.H / d.G);
+    const int K = d.K, N = d.N, P = d.P;
+    const int nnt = (N + 3) >> 2, npt = Ps >> 3, Npad = nnt * 4;
+    const int ntiles = K * npt * nnt;
+    const int tid = threadIdx.x;
+    const bool active = tid < ntiles;
+    const int nt = tid % nnt, pt = (tid / nnt) % npt, m = active ? tid / (nnt * npt) : 0;
+    const int p0 = pbase + pt * 8, n0 = nt * 4;
+
+    double *E_s = reinterpret_cast<double *>(smem_raw);  // [kQMax]
+    float *e_s = reinterpret_cast<float *>(E_s + kQMax);  // [kQMax]
+    float *itau = e_s + kQMax;                            // [32]
+    float *dec = itau + 32;                               // [32]
+    float *coef = dec + 32;                               // [kQMax][K]
+    float *u_s = coef + kQMax * K;                        // [kQMax][Ps]
+    float *v_s = u_s + kQMax * Ps;                        // [kQMax][Npad]
+
+    if (tid < K) itau[tid] = 1.f / tau[h * K + tid];
+    const float log_cap = head_log_cap(tau, h, K);
+    const size_t PN = size_t(P) * N;
+    const size_t bh = size_t(b) * d.H + h;
+
+    float S[8][4];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int p = p0 + i, nn = n0 + j;
+            S[i][j] = (active && init && p < P && nn < N)
+                          ? init[(bh * K + m) * PN + size_t(p) * N + nn]
+                          : 0.f;
+        }
+
+    for (int ci = 0; ci < d.nc; ++ci) {
+        const int c = REV ? d.nc - 1 - ci : ci;
+        const int c0 = c * d.Q, n = min(d.Q, d.L - c0);
+        __syncthreads();  // the previous chunk's shared-memory reads are done
+        chunk_rates(d, b, h, c0, n, log_cap, dt, alpha, lam, e_s, E_s, nullptr);
+        for (int idx = tid; idx < n * Ps; idx += blockDim.x) {
+            const int k = idx / Ps, pp = idx - k * Ps, p = pbase + pp;
+            u_s[k * Ps + pp] = p < P ? to_f(U[blh(d, b, c0 + k, h) * P + p]) : 0.f;
+        }
+        for (int idx = tid; idx < n * Npad; idx += blockDim.x) {
+            const int k = idx / Npad, nn = idx - k * Npad;
+            v_s[k * Npad + nn] =
+                nn < N ? to_f(V[((size_t(b) * d.L + c0 + k) * d.G + g) * N + nn]) : 0.f;
+        }
+        __syncthreads();  // E_s, e_s ready
+        const double Eend = E_s[n - 1];
+        for (int idx = tid; idx < n * K; idx += blockDim.x) {
+            const int k = idx / K, mm = idx - k * K;
+            const float w = to_f(W[blh(d, b, c0 + k, h) * K + mm]);
+            float cval;
+            if (!REV) {
+                const float kap = -expm1f(-e_s[k] * itau[mm]) * w;
+                cval = kap * expf(-float(Eend - E_s[k]) * itau[mm]);
+            } else {
+                cval = w * expf(-float(E_s[k]) * itau[mm]);
+            }
+            coef[k * K + mm] = cval;
+        }
+        if (tid < K) dec[tid] = expf(-float(Eend) * itau[tid]);
+        if (active) {  // emit the state entering this chunk (before its update)
+            TS *dst = emit + ((bh * d.nc + c) * K + m) * PN;
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    if (p0 + i < P && n0 + j < N)
+                        dst[size_t(p0 + i) * N + n0 + j] = cvt_state<TS>(S[i][j]);
+        }
+        __syncthreads();  // coef, dec ready
+        if (active) {
+            const float dm = dec[m];
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) S[i][j] *= dm;
+            for (int k = 0; k < n; ++k) {
+                const float cf = coef[k * K + m];
+                const float4 ua = *reinterpret_cast<const float4 *>(u_s + k * Ps + pt * 8);
+                const float4 ub = *reinterpret_cast<const float4 *>(u_s + k * Ps + pt * 8 + 4);
+                const float4 vv = *reinterpret_cast<const float4 *>(v_s + k * Npad + n0);
+                const float cu[8] = {cf * ua.x, cf * ua.y, cf * ua.z, cf * ua.w,
+                                     cf * ub.x, cf * ub.y, cf * ub.z, cf * ub.w};
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    S[i][0] = fmaf(cu[i], vv.x, S[i][0]);
+                    S[i][1] = fmaf(cu[i], vv.y, S[i][1]);
+                    S[i][2] = fmaf(cu[i], vv.z, S[i][2]);
+                    S[i][3] = fmaf(cu[i], vv.w, S[i][3]);
+                }
+            }
+        }
+    }
+    if (active && fin) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+                if (p0 + i < P && n0 + j < N)
+                    fin[(bh * K + m) * PN + size_t(p0 + i) * N + n0 + j] = S[i][j];
+    }
+}
+
+size_t state_pass_smem(const ScanDims &d, int Ps) {
+    const int Npad = ((d.N + 3) >> 2) * 4;
+    return sizeof(double) * kQMax + sizeof(float) * (kQMax + 64 + size_t(kQMax) * d.K +
+                                                     size_t(kQMax) * Ps + size_t(kQMax) * Npad);
+}
+
+// ---------------------------------------------------------------------------------------------
+// Chunk output: y for one (b, h, chunk).  Thread tiles: 4x4 over (t, k) for Gamma o G,
+// 4 t x 4 p for y (at most two tiles per thread).
+template <typename T, typename TS>
+__global__ void __launch_bounds__(kThreads) simt_chunk_fwd(
+    ScanDims d, const T *__restrict__ x, const T *__restrict__ Bm, const T *__restrict__ Cm,
+    const T *__restrict__ wr, const T *__restrict__ ww, const float *__restrict__ dt,
+    const float *__restrict__ alpha, const float *__restrict__ lam,
+    const float *__restrict__ tau, const float *__restrict__ Dv, const TS *__restrict__ S_in,
+    T *__restrict__ y) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+    const int g = h / (d.H / d.G);
+    const int K = d.K, N = d.N, P = d.P, Q = d.Q;
+    const int c0 = c * Q, n = min(Q, d.L - c0);
+    const int P1 = P + 1, N1 = N + 1, Q1 = Q + 1;
+    const int tid = threadIdx.x;
+
+    double *E_s = reinterpret_cast<double *>(smem_raw);
+    float *e_s = reinterpret_cast<float *>(E_s + kQMax);
+    float *itau = e_s + kQMax;
+    float *wr_s = itau + 32;            // [Q][K]
+    float *kap_s = wr_s + Q * K;        // [Q][K]
+    float *f_s = kap_s + Q * K;         // [Q][K]
+    float *xs = f_s + Q * K;            // [Q][P1]
+    float *Cs = xs + Q * P1;            // [Q][N1]
+    float *Bs = Cs + Q * N1;            // [Q][N1]
+    float *Ms = Bs + Q * N1;            // [Q][Q1]
+    float *Ss = Ms + Q * Q1;            // [P][N1]
+
+    if (tid < K) itau[tid] = 1.f / tau[h * K + tid];
+    const float log_cap = head_log_cap(tau, h, K);
+    chunk_rates(d, b, h, c0, n, log_cap, dt, alpha, lam, e_s, E_s, nullptr);
+    for (int idx = tid; idx < Q * P; idx += blockDim.x) {
+        const int t = idx / P, p = idx - t * P;
+        xs[t * P1 + p] = t < n ? to_f(x[blh(d, b, c0 + t, h) * P + p]) : 0.f;
+    }
+    for (int idx = tid; idx < Q * N; idx += blockDim.x) {
+        const int t = idx / N, nn = idx - t * N;
+        const size_t gi = ((size_t(b) * d.L + c0 + t) * d.G + g) * N + nn;
+        Cs[t * N1 + nn] = t < n ? to_f(Cm[gi]) : 0.f;
+        Bs[t * N1 + nn] = t < n ? to_f(Bm[gi]) : 0.f;
+    }
+    __syncthreads();
+    for (int idx = tid; idx < Q * K; idx += blockDim.x) {
+        const int t = idx / K, mm = idx - t * K;
+        float w = 0.f, kp = 0.f, f = 0.f;
+        if (t < n) {
+            const size_t wi = blh(d, b, c0 + t, h) * K + mm;
+            w = to_f(wr[wi]);
+            kp = -expm1f(-e_s[t] * itau[mm]) * to_f(ww[wi]);
+            f = w * expf(-float(E_s[t]) * itau[mm]);
+        }
+        wr_s[idx] = w;
+        kap_s[idx] = kp;
+        f_s[idx] = f;
+    }
+    __syncthreads();
+    // Gamma o (C B^T), lower triangle
+    const int qt = Q >> 2;
+    for (int tile = tid; tile < qt * qt; tile += blockDim.x) {
+        const int t0 = 4 * (tile / qt), k0 = 4 * (tile % qt);
+        float G[4][4] = {};
+        if (k0 <= t0 + 3) {
+            for (int nn = 0; nn < N; ++nn) {
+                float cv[4], bv[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    cv[i] = Cs[(t0 + i) * N1 + nn];
+                    bv[i] = Bs[(k0 + i) * N1 + nn];
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) G[i][j] = fmaf(cv[i], bv[j], G[i][j]);
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int t = t0 + i, k = k0 + j;
+                float v = 0.f;
+                if (k <= t && t < n) {
+                    const float dE = float(E_s[t] - E_s[k]);
+                    float gam = 0.f;
+                    for (int mm = 0; mm < K; ++mm)
+                        gam = fmaf(wr_s[t * K + mm] * kap_s[k * K + mm], expf(-dE * itau[mm]), gam);
+                    v = gam * G[i][j];
+                }
+                Ms[t * Q1 + k] = v;
+            }
+    }
+    __syncthreads();
+    // y tiles
+    const int npt4 = (P + 3) >> 2;
+    const int ytiles = qt * npt4;
+    float acc[2][4][4] = {};
+    int tt0[2], pp0[2];
+#pragma unroll
+    for (int s = 0; s < 2; ++s) {
+        const int tile = tid + s * blockDim.x;
+        tt0[s] = 4 * (tile / npt4);
+        pp0[s] = 4 * (tile % npt4);
+        if (tile < ytiles) {
+            const int kend = min(tt0[s] + 4, n);
+            for (int k = 0; k < kend; ++k) {
+                float mv[4], xv[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    mv[i] = Ms[(tt0[s] + i) * Q1 + k];
+                    xv[i] = (pp0[s] + i < P) ? xs[k * P1 + pp0[s] + i] : 0.f;
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) acc[s][i][j] = fmaf(mv[i], xv[j], acc[s][i][j]);
+            }
+        }
+    }
+    const size_t PN = size_t(P) * N;
+    const TS *Sbase = S_in + ((size_t(b) * d.H + h) * d.nc + c) * K * PN;
+    for (int mm = 0; mm < K; ++mm) {
+        __syncthreads();
+        for (int idx = tid; idx < P * N; idx += blockDim.x) {
+            const int p = idx / N, nn = idx - p * N;
+            Ss[p * N1 + nn] = to_f(Sbase[mm * PN + idx]);
+        }
+        __syncthreads();
+#pragma unroll
+        for (int s = 0; s < 2; ++s) {
+            const int tile = tid + s * blockDim.x;
+            if (tile >= ytiles) continue;
+            float z[4][4] = {};
+            for (int nn = 0; nn < N; ++nn) {
+                float cv[4], sv[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    cv[i] = Cs[(tt0[s] + i) * N1 + nn];
+                    sv[i] = (pp0[s] + i < P) ? Ss[(pp0[s] + i) * N1 + nn] : 0.f;
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) z[i][j] = fmaf(cv[i], sv[j], z[i][j]);
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float f = f_s[(tt0[s] + i) * K + mm];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[s][i][j] = fmaf(f, z[i][j], acc[s][i][j]);
+            }
+        }
+    }
+    const float Dh = Dv[h];
+#pragma unroll
+    for (int s = 0; s < 2; ++s) {
+        const int tile = tid + s * blockDim.x;
+        if (tile >= ytiles) continue;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int t = tt0[s] + i;
+            if (t >= n) continue;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int p = pp0[s] + j;
+                if (p < P)
+                    y[blh(d, b, c0 + t, h) * P + p] =
+                        from_f<T>(acc[s][i][j] + Dh * xs[t * P1 + p]);
+            }
+        }
+    }
+}
+
+size_t chunk_fwd_smem(const ScanDims &d) {
+    const int Q = d.Q;
+    return sizeof(double) * kQMax +
+           sizeof(float) * (kQMax + 32 + 3 * size_t(Q) * d.K + size_t(Q) * (d.P + 1) +
+                            2 * size_t(Q) * (d.N + 1) + size_t(Q) * (Q + 1) +
+                            size_t(d.P) * (d.N + 1));
+}
+
+// ---------------------------------------------------------------------------------------------
+// Chunk backward for one (b, h, chunk).  With G[t,k] = C_t . B_k, H[t,k] = dy_t . x_k,
+// W_{t,k,m} = exp(-(E_t - E_k)/tau_m) (t >= k), u_{k,m} = exp(-(E_end - E_k)/tau_m),
+// s = kappa u, f = w_read exp(-E_t/tau), U_m = B dS_out,m^T, Z_m = C S_in,m^T:
+//   dx_k      = sum_m s_{k,m} U_m[k] + sum_{t>=k} Gamma_{t,k} G_{t,k} dy_t + D dy_k
+//   dkappa_km = u_{k,m} x_k . U_m[k] + sum_{t>=k} w_read_{t,m} W_{t,k,m} G_{t,k} H_{t,k}
+//   dw_read_tm= exp(-E_t/tau_m) dy_t . Z_m[t] + sum_{k<=t} kappa_{k,m} W_{t,k,m} G_{t,k} H_{t,k}
+//   dC_t     += sum_m f_{t,m} S_in,m^T dy_t + sum_{k<=t} Gamma_{t,k} H_{t,k} B_k
+//   dB_k     += sum_m s_{k,m} dS_out,m^T x_k + sum_{t>=k} Gamma_{t,k} H_{t,k} C_t
+//   sum_m rho_t <dS_t, S_{t-1}>_m / tau_m = sum_{t'>=t} a_t' + sum_{k<t} b_k + c
+//                                           + sum_{t'>=t, k<t} Gamma'_{t',k} G_{t',k} H_{t',k}
+//        a_t = sum_m f_{t,m} dy_t.Z_m[t] / tau_m,  b_k = sum_m s_{k,m} x_k.U_m[k] / tau_m,
+//        c = sum_m d_m <dS_out,m, S_in,m> / tau_m,  Gamma' = Gamma with kappa / tau
+//   (every term carries its own decay, so this stays accurate when e_t is large)
+//   de_t = -(that) + sum_m dkappa_{t,m} rho_{t,m} w_write_{t,m} / tau_m   (0 if e_t was clamped)
+template <typename T, typename TS>
+__global__ void __launch_bounds__(kThreads) simt_chunk_bwd(
+    ScanDims d, const T *__restrict__ x, const T *__restrict__ Bm, const T *__restrict__ Cm,
+    const T *__restrict__ wr, const T *__restrict__ ww, const T *__restrict__ dy,
+    const float *__restrict__ dt, const float *__restrict__ alpha, const float *__restrict__ lam,
+    const float *__restrict__ tau, const float *__restrict__ Dv, const TS *__restrict__ S_in,
+    const TS *__restrict__ dS_out, T *__restrict__ dx, T *__restrict__ dwr_o,
+    T *__restrict__ dww_o, float *__restrict__ ddt, float *__restrict__ dalpha,
+    float *__restrict__ dlam, float *__restrict__ dD, float *__restrict__ dB_acc,
+    float *__restrict__ dC_acc) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+    const int g = h / (d.H / d.G);
+    const int K = d.K, N = d.N, P = d.P, Q = d.Q;
+    const int c0 = c * Q, n = min(Q, d.L - c0);
+    const int P1 = P + 1, N1 = N + 1, Q1 = Q + 1;
+    const int tid = threadIdx.x;
+    const int QK = Q * K;
+
+    double *E_s = reinterpret_cast<double *>(smem_raw);
+    float *e_s = reinterpret_cast<float *>(E_s + kQMax);
+    float *cl_s = e_s + kQMax;
+    float *itau = cl_s + kQMax;     // [32]
+    float *dec = itau + 32;         // [32]
+    float *red = dec + 32;          // [32]
+    float *a_s = red + 32;          // [kQMax]
+    float *b_s = a_s + kQMax;       // [kQMax]
+    float *rp_s = b_s + kQMax;      // [kQMax]
+    float *wr_s = rp_s + kQMax;     // [Q][K] x 11
+    float *ww_s = wr_s + QK;
+    float *kap_s = ww_s + QK;
+    float *rho_s = kap_s + QK;
+    float *omr_s = rho_s + QK;
+    float *fd_s = omr_s + QK;       // exp(-E_t/tau)
+    float *u_s = fd_s + QK;         // exp(-(E_end - E_k)/tau)
+    float *dwri = u_s + QK;         // intra part of dw_read
+    float *dkpi = dwri + QK;        // intra part of dkappa
+    float *xU = dkpi + QK;          // x_k . U_m[k]
+    float *dyZ = xU + QK;           // dy_t . Z_m[t]
+    float *xs = dyZ + QK;           // [Q][P1]
+    float *dys = xs + Q * P1;       // [Q][P1]
+    float *Bs = dys + Q * P1;       // [Q][N1]
+    float *Cs = Bs + Q * N1;        // [Q][N1]
+    float *un = Cs + Q * N1;        // union
+    float *MG = un;                 // [Q][Q1]  Gamma o G
+    float *MH = MG + Q * Q1;        // [Q][Q1]  Gamma o H
+    float *XX = MH + Q * Q1;        // [Q][Q1]  Gamma' o G o H
+    float *Ss = un;                 // [P][N1]
+    float *dSs = Ss + P * N1;       // [P][N1]
+
+    // ---- loads
+    if (tid < K) itau[tid] = 1.f / tau[h * K + tid];
+    const float log_cap = head_log_cap(tau, h, K);
+    chunk_rates(d, b, h, c0, n, log_cap, dt, alpha, lam, e_s, E_s, cl_s);
+    for (int idx = tid; idx < Q * P; idx += blockDim.x) {
+        const int t = idx / P, p = idx - t * P;
+        const size_t gi = blh(d, b, c0 + t, h) * P + p;
+        xs[t * P1 + p] = t < n ? to_f(x[gi]) : 0.f;
+        dys[t * P1 + p] = t < n ? to_f(dy[gi]) : 0.f;
+    }
+    for (int idx = tid; idx < Q * N; idx += blockDim.x) {
+        const int t = idx / N, nn = idx - t * N;
+        const size_t gi = ((size_t(b) * d.L + c0 + t) * d.G + g) * N + nn;
+        Cs[t * N1 + nn] = t < n ? to_f(Cm[gi]) : 0.f;
+        Bs[t * N1 + nn] = t < n ? to_f(Bm[gi]) : 0.f;
+    }
+    __syncthreads();
+    const double Eend = E_s[n - 1];
+    for (int idx = tid; idx < QK; idx += blockDim.x) {
+        const int t = idx / K, mm = idx - t * K;
+        float w_r = 0.f, w_w = 0.f, rho = 0.f, omr = 0.f, fd = 0.f, uu = 0.f;
+        if (t < n) {
+            const size_t wi = blh(d, b, c0 + t, h) * K + mm;
+            w_r = to_f(wr[wi]);
+            w_w = to_f(ww[wi]);
+            const float z = e_s[t] * itau[mm];
+            rho = expf(-z);
+            omr = -expm1f(-z);
+            fd = expf(-float(E_s[t]) * itau[mm]);
+            uu = expf(-float(Eend - E_s[t]) * itau[mm]);
+        }
+        wr_s[idx] = w_r;
+        ww_s[idx] = w_w;
+        kap_s[idx] = omr * w_w;
+        rho_s[idx] = rho;
+        omr_s[idx] = omr;
+        fd_s[idx] = fd;
+        u_s[idx] = uu;
+        dwri[idx] = 0.f;
+        dkpi[idx] = 0.f;
+        xU[idx] = 0.f;
+        dyZ[idx] = 0.f;
+    }
+    if (tid < K) dec[tid] = expf(-float(Eend) * itau[tid]);
+    __syncthreads();
+
+    // ---- intra-chunk pairs: 4 t x 4 k tiles
+    const int qt = Q >> 2;
+    for (int tile = tid; tile < qt * qt; tile += blockDim.x) {
+        const int t0 = 4 * (tile / qt), k0 = 4 * (tile % qt);
+        float G[4][4] = {}, Hm[4][4] = {};
+        if (k0 <= t0 + 3) {
+            for (int nn = 0; nn < N; ++nn) {
+                float cv[4], bv[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    cv[i] = Cs[(t0 + i) * N1 + nn];
+                    bv[i] = Bs[(k0 + i) * N1 + nn];
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) G[i][j] = fmaf(cv[i], bv[j], G[i][j]);
+            }
+            for (int p = 0; p < P; ++p) {
+                float dv[4], xv[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    dv[i] = dys[(t0 + i) * P1 + p];
+                    xv[i] = xs[(k0 + i) * P1 + p];
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) Hm[i][j] = fmaf(dv[i], xv[j], Hm[i][j]);
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int t = t0 + i, k = k0 + j;
+                float mg = 0.f, mh = 0.f, xx = 0.f;
+                if (k <= t && t < n) {
+                    const float dE = float(E_s[t] - E_s[k]);
+                    const float gh = G[i][j] * Hm[i][j];
+                    float gam = 0.f, gamt = 0.f;
+                    for (int mm = 0; mm < K; ++mm) {
+                        const float Wm = expf(-dE * itau[mm]);
+                        const float a = wr_s[t * K + mm] * kap_s[k * K + mm] * Wm;
+                        gam += a;
+                        gamt = fmaf(a, itau[mm], gamt);
+                        const float cw = Wm * gh;
+                        atomicAdd(&dwri[t * K + mm], kap_s[k * K + mm] * cw);
+                        atomicAdd(&dkpi[k * K + mm], wr_s[t * K + mm] * cw);
+                    }
+                    mg = gam * G[i][j];
+                    mh = gam * Hm[i][j];
+                    xx = gamt * gh;
+                }
+                MG[t * Q1 + k] = mg;
+                MH[t * Q1 + k] = mh;
+                XX[t * Q1 + k] = xx;
+            }
+    }
+    __syncthreads();
+    // exclusive row prefix of XX, then column suffix -> pair rectangle sums
+    if (tid < Q) {
+        float run = 0.f;
+        for (int j = 0; j < Q; ++j) {
+            const float v = XX[tid * Q1 + j];
+            XX[tid * Q1 + j] = run;
+            run += v;
+        }
+    }
+    __syncthreads();
+    if (tid < Q) {
+        float s = 0.f;
+        for (int tp = tid; tp < n; ++tp) s += XX[tp * Q1 + tid];
+        rp_s[tid] = s;
+    }
+
+    // ---- register tiles: dx (4 k x 4 p), dC / dB (4 rows x 8 n)
+    const int npt4 = (P + 3) >> 2, nnt8 = (N + 7) >> 3;
+    const bool has_x = tid < qt * npt4, has_cb = tid < qt * nnt8;
+    const int xr0 = 4 * (tid / npt4), xp0 = 4 * (tid % npt4);
+    const int cr0 = 4 * (tid / nnt8), cn0 = 8 * (tid % nnt8);
+    float adx[4][4] = {}, adC[4][8] = {}, adB[4][8] = {};
+    if (has_x) {
+        for (int t = xr0; t < n; ++t) {
+            float mv[4], dv[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                mv[i] = MG[t * Q1 + xr0 + i];
+                dv[i] = (xp0 + i < P) ? dys[t * P1 + xp0 + i] : 0.f;
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) adx[i][j] = fmaf(mv[i], dv[j], adx[i][j]);
+        }
+    }
+    if (has_cb) {
+        for (int k = 0; k < min(cr0 + 4, n); ++k) {  // dC_t += sum_{k<=t} (Gamma o H)[t,k] B_k
+            float mv[4], bv[8];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) mv[i] = MH[(cr0 + i) * Q1 + k];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) bv[j] = (cn0 + j < N) ? Bs[k * N1 + cn0 + j] : 0.f;
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 8; ++j) adC[i][j] = fmaf(mv[i], bv[j], adC[i][j]);
+        }
+        for (int t = cr0; t < n; ++t) {  // dB_k += sum_{t>=k} (Gamma o H)[t,k] C_t
+            float mv[4], cv[8];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) mv[i] = MH[t * Q1 + cr0 + i];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) cv[j] = (cn0 + j < N) ? Cs[t * N1 + cn0 + j] : 0.f;
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 8; ++j) adB[i][j] = fmaf(mv[i], cv[j], adB[i][j]);
+        }
+    }
+
+    // ---- inter-chunk terms, mode by mode
+    const size_t PN = size_t(P) * N;
+    const size_t sbase = ((size_t(b) * d.H + h) * d.nc + c) * K * PN;
+    float cpart = 0.f;
+    for (int mm = 0; mm < K; ++mm) {
+        __syncthreads();  // the union region / previous mode is no longer read
+        float dot = 0.f;
+        for (int idx = tid; idx < P * N; idx += blockDim.x) {
+            const int p = idx / N, nn = idx - p * N;
+            const float sv = to_f(S_in[sbase + mm * PN + idx]);
+            const float dv = to_f(dS_out[sbase + mm * PN + idx]);
+            Ss[p * N1 + nn] = sv;
+            dSs[p * N1 + nn] = dv;
+            dot = fmaf(sv, dv, dot);
+        }
+        cpart = fmaf(dec[mm] * itau[mm], dot, cpart);
+        __syncthreads();
+        if (has_x) {
+            float Uq[4][4] = {}, Zq[4][4] = {};
+            for (int nn = 0; nn < N; ++nn) {
+                float bv[4], cv[4], dsv[4], sv[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    bv[i] = Bs[(xr0 + i) * N1 + nn];
+                    cv[i] = Cs[(xr0 + i) * N1 + nn];
+                    const bool ok = xp0 + i < P;
+                    dsv[i] = ok ? dSs[(xp0 + i) * N1 + nn] : 0.f;
+                    sv[i] = ok ? Ss[(xp0 + i) * N1 + nn] : 0.f;
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        Uq[i][j] = fmaf(bv[i], dsv[j], Uq[i][j]);
+                        Zq[i][j] = fmaf(cv[i], sv[j], Zq[i][j]);
+                    }
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int r = xr0 + i;
+                const float sk = kap_s[r * K + mm] * u_s[r * K + mm];
+                float xu = 0.f, dz = 0.f;
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    adx[i][j] = fmaf(sk, Uq[i][j], adx[i][j]);
+                    if (xp0 + j < P) {
+                        xu = fmaf(xs[r * P1 + xp0 + j], Uq[i][j], xu);
+                        dz = fmaf(dys[r * P1 + xp0 + j], Zq[i][j], dz);
+                    }
+                }
+                if (r < n) {
+                    atomicAdd(&xU[r * K + mm], xu);
+                    atomicAdd(&dyZ[r * K + mm], dz);
+                }
+            }
+        }
+        if (has_cb) {
+            float fr[4], sr[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int r = cr0 + i;
+                fr[i] = wr_s[r * K + mm] * fd_s[r * K + mm];
+                sr[i] = kap_s[r * K + mm] * u_s[r * K + mm];
+            }
+            for (int p = 0; p < P; ++p) {
+                float fy[4], sx[4], sv[8], dsv[8];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    fy[i] = fr[i] * dys[(cr0 + i) * P1 + p];
+                    sx[i] = sr[i] * xs[(cr0 + i) * P1 + p];
+                }
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    const bool ok = cn0 + j < N;
+                    sv[j] = ok ? Ss[p * N1 + cn0 + j] : 0.f;
+                    dsv[j] = ok ? dSs[p * N1 + cn0 + j] : 0.f;
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        adC[i][j] = fmaf(fy[i], sv[j], adC[i][j]);
+                        adB[i][j] = fmaf(sx[i], dsv[j], adB[i][j]);
+                    }
+            }
+        }
+    }
+    const float cprime = block_sum(cpart, red);  // contains __syncthreads
+
+    // ---- dD partial
+    float dd = 0.f;
+    for (int idx = tid; idx < n * P; idx += blockDim.x) {
+        const int t = idx / P, p = idx - t * P;
+        dd = fmaf(dys[t * P1 + p], xs[t * P1 + p], dd);
+    }
+    dd = block_sum(dd, red);
+    if (tid == 0) atomicAdd(&dD[h], dd);
+
+    // ---- stores of the tiles
+    const float Dh = Dv[h];
+    if (has_x) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int t = xr0 + i;
+            if (t >= n) continue;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int p = xp0 + j;
+                if (p < P)
+                    dx[blh(d, b, c0 + t, h) * P + p] =
+                        from_f<T>(adx[i][j] + Dh * dys[t * P1 + p]);
+            }
+        }
+    }
+    if (has_cb) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int t = cr0 + i;
+            if (t >= n) continue;
+            const size_t gi = ((size_t(b) * d.L + c0 + t) * d.G + g) * N;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int nn = cn0 + j;
+                if (nn < N) {
+                    atomicAdd(&dC_acc[gi + nn], adC[i][j]);
+                    atomicAdd(&dB_acc[gi + nn], adB[i][j]);
+                }
+            }
+        }
+    }
+    // ---- per-position scalars
+    if (tid < n) {
+        const int t = tid;
+        float a = 0.f, bb = 0.f;
+        for (int mm = 0; mm < K; ++mm) {
+            a = fmaf(wr_s[t * K + mm] * fd_s[t * K + mm] * dyZ[t * K + mm], itau[mm], a);
+            bb = fmaf(kap_s[t * K + mm] * u_s[t * K + mm] * xU[t * K + mm], itau[mm], bb);
+        }
+        a_s[t] = a;
+        b_s[t] = bb;
+    }
+    __syncthreads();
+    if (tid < n) {
+        const int t = tid;
+        float suf = 0.f, pre = 0.f;
+        for (int j = t; j < n; ++j) suf += a_s[j];
+        for (int j = 0; j < t; ++j) pre += b_s[j];
+        const float R = suf + pre + cprime + rp_s[t];
+        float de = -R;
+        const size_t wi0 = blh(d, b, c0 + t, h) * K;
+        for (int mm = 0; mm < K; ++mm) {
+            const int q = t * K + mm;
+            const float dk = u_s[q] * xU[q] + dkpi[q];
+            const float dw = fd_s[q] * dyZ[q] + dwri[q];
+            de = fmaf(dk * rho_s[q] * ww_s[q], itau[mm], de);
+            dwr_o[wi0 + mm] = from_f<T>(dw);
+            dww_o[wi0 + mm] = from_f<T>(dk * omr_s[q]);
+        }
+        const size_t i = blh(d, b, c0 + t, h);
+        const float e = e_s[t];
+        const bool cl = cl_s[t] != 0.f;
+        const float al = alpha[i], lm = lam[i], dtv = dt[i];
+        const float ge = cl ? 0.f : de * e;
+        ddt[i] = ge / dtv;
+        dlam[i] = ge / (al * lm);
+        dalpha[i] = -ge * logf(lm) / (al * al);
+    }
+}
+
+size_t chunk_bwd_smem(const ScanDims &d) {
+    const size_t Q = d.Q, P1 = d.P + 1, N1 = d.N + 1;
+    const size_t uni = std::max(3 * Q * (Q + 1), 2 * size_t(d.P) * N1);
+    return sizeof(double) * kQMax +
+           sizeof(float) * (2 * kQMax + 3 * 32 + 3 * kQMax + 11 * Q * d.K + 2 * Q * P1 +
+                            2 * Q * N1 + uni);
+}
+
+__global__ void f32_to_bf16_kernel(const float *__restrict__ in, __nv_bfloat16 *__restrict__ out,
+                                   size_t n) {
+    for (size_t i = blockIdx.x * size_t(blockDim.x) + threadIdx.x; i < n;
+         i += size_t(gridDim.x) * blockDim.x)
+        out[i] = __float2bfloat16_rn(in[i]);
+}
+
+int state_pass_ps(const ScanDims &d) {
+    const int nnt = (d.N + 3) >> 2;
+    const int per8 = d.K * nnt;  // tiles per 8 p-rows
+    if (per8 > 512) return 0;
+    int npt = std::max(1, 256 / per8);
+    npt = std::min(npt, (d.P + 7) / 8);
+    npt = std::max(1, std::min(npt, 512 / per8));
+    return npt * 8;
+}
+
+template <typename T, typename TS>
+cudaError_t run_state_pass(const ScanDims &d, bool rev, const void *U, const void *V,
+                           const void *W, const ScanPtrs &p, const float *init, void *emit,
+                           float *fin, cudaStream_t st) {
+    const int Ps = state_pass_ps(d);
+    const int ntiles = d.K * (Ps / 8) * ((d.N + 3) >> 2);
+    const int threads = ((ntiles + 31) / 32) * 32;
+    const size_t smem = state_pass_smem(d, Ps);
+    dim3 grid((d.P + Ps - 1) / Ps, d.H, d.B);
+    if (rev) {
+        auto k = simt_state_pass<T, TS, true>;
+        cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+        trace_begin("state_pass_rev_simt", st);
+        k<<<grid, threads, smem, st>>>(d, Ps, (const T *)U, (const T *)V, (const T *)W, p.dt,
+                                       p.alpha, p.lam, p.tau, init, (TS *)emit, fin);
+        trace_end(st);
+    } else {
+        auto k = simt_state_pass<T, TS, false>;
+        cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+        trace_begin("state_pass_fwd_simt", st);
+        k<<<grid, threads, smem, st>>>(d, Ps, (const T *)U, (const T *)V, (const T *)W, p.dt,
+                                       p.alpha, p.lam, p.tau, init, (TS *)emit, fin);
+        trace_end(st);
+    }
+    return cudaGetLastError();
+}
+
+template <typename T, typename TS>
+cudaError_t fwd_t(const ScanDims &d, const ScanPtrs &p, void *S_in, cudaStream_t st) {
+    cudaError_t e = run_state_pass<T, TS>(d, false, p.x, p.Bm, p.ww, p, p.h0, S_in, p.h_final, st);
+    if (e != cudaSuccess || d.nc == 0) return e;  // L = 0: h_final = h0 was written
+    const size_t smem = chunk_fwd_smem(d);
+    auto k = simt_chunk_fwd<T, TS>;
+    cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    trace_begin("chunk_fwd_simt", st);
+    k<<<dim3(d.nc, d.H, d.B), kThreads, smem, st>>>(
+        d, (const T *)p.x, (const T *)p.Bm, (const T *)p.Cm, (const T *)p.wr, (const T *)p.ww,
+        p.dt, p.alpha, p.lam, p.tau, p.D, (const TS *)S_in, (T *)p.y);
+    trace_end(st);
+    return cudaGetLastError();
+}
+
+template <typename T, typename TS>
+cudaError_t bwd_t(const ScanDims &d, const ScanPtrs &p, void *S_in, void *dS_out, float *dB_acc,
+                  float *dC_acc, cudaStream_t st) {
+    cudaError_t e = run_state_pass<T, TS>(d, false, p.x, p.Bm, p.ww, p, p.h0, S_in, nullptr, st);
+    if (e != cudaSuccess) return e;
+    e = run_state_pass<T, TS>(d, true, p.dy, p.Cm, p.wr, p, p.dh_final, dS_out, p.dh0, st);
+    if (e != cudaSuccess) return e;
+    const size_t ngn = size_t(d.B) * d.L * d.G * d.N;
+    if ((e = cudaMemsetAsync(p.dD, 0, sizeof(float) * d.H, st)) != cudaSuccess) return e;
+    if ((e = cudaMemsetAsync(dB_acc, 0, sizeof(float) * ngn, st)) != cudaSuccess) return e;
+    if ((e = cudaMemsetAsync(dC_acc, 0, sizeof(float) * ngn, st)) != cudaSuccess) return e;
+    if (d.nc == 0) return cudaSuccess;  // L = 0: dh0 = dh_final was written, dD = 0
+    const size_t smem = chunk_bwd_smem(d);
+    auto k = simt_chunk_bwd<T, TS>;
+    cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    trace_begin("chunk_bwd_simt", st);
+    k<<<dim3(d.nc, d.H, d.B), kThreads, smem, st>>>(
+        d, (const T *)p.x, (const T *)p.Bm, (const T *)p.Cm, (const T *)p.wr, (const T *)p.ww,
+        (const T *)p.dy, p.dt, p.alpha, p.lam, p.tau, p.D, (const TS *)S_in,
+        (const TS *)dS_out, (T *)p.dx, (T *)p.dwr, (T *)p.dww, p.ddt, p.dalpha, p.dlam, p.dD,
+        dB_acc, dC_acc);
+    trace_end(st);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (sizeof(T) == 2 && ngn > 0) {
+        const unsigned blocks = unsigned(std::min<size_t>((ngn + 255) / 256, 4096));
+        trace_begin("f32_to_bf16", st);
+        f32_to_bf16_kernel<<<blocks, 256, 0, st>>>(dB_acc, (__nv_bfloat16 *)p.dB, ngn);
+        trace_end(st);
+        trace_begin("f32_to_bf16", st);
+        f32_to_bf16_kernel<<<blocks, 256, 0, st>>>(dC_acc, (__nv_bfloat16 *)p.dC, ngn);
+        trace_end(st);
+        e = cudaGetLastError();
+    }
+    return e;
+}
+
+}  // namespace
+
+int simt_pick_chunk(const ScanDims &d0, int requested) {
+    const int cands[3] = {64, 32, 16};
+    for (int qi = 0; qi < 3; ++qi) {
+        const int Q = cands[qi];
+        if (requested && requested != Q) continue;
+        ScanDims d = d0;
+        d.Q = Q;
+        const int qt = Q / 4;
+        if (state_pass_ps(d) == 0) continue;
+        if (qt * ((d.P + 3) / 4) > kThreads) continue;     // dx tiles (and <= 2 y tiles per thread)
+        if (qt * ((d.N + 7) / 8) > kThreads) continue;     // dB / dC tiles
+        if (chunk_fwd_smem(d) > 227 * 1024) continue;
+        if (chunk_bwd_smem(d) > 227 * 1024) continue;
+        if (state_pass_smem(d, state_pass_ps(d)) > 227 * 1024) continue;
+        return Q;
+    }
+    return 0;
+}
+
+size_t simt_state_elems(const ScanDims &d) {
+    return size_t(d.B) * d.H * d.nc * d.K * d.P * d.N;
+}
+
+cudaError_t simt_scan_fwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in,
+                          cudaStream_t st) {
+    if (dtype == 0) return fwd_t<float, float>(d, p, S_in, st);
+    return fwd_t<__nv_bfloat16, __nv_bfloat16>(d, p, S_in, st);
+}
+
+cudaError_t simt_scan_bwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in,
+                          void *dS_out, float *dB_acc, float *dC_acc, cudaStream_t st) {
+    if (dtype == 0) return bwd_t<float, float>(d, p, S_in, dS_out, dB_acc, dC_acc, st);
+    return bwd_t<__nv_bfloat16, __nv_bfloat16>(d, p, S_in, dS_out, dB_acc, dC_acc, st);
+}
+
+}  // namespace frac

@@ -186,3 +186,33 @@ def algorithmic_flops_per_token_head(s: Shape) -> float:
     return 4.0 * s.nmodes * s.headdim * s.dstate
 
 
+
+
+def make_scan_inputs_torch(s: Shape, seed: int, device, with_dy: bool = False) -> dict:
+    """The same recipe drawn with torch's generator on `device` (fast inputs for timing runs;
+    the parity tests use the numpy recipe above so that the oracle reads identical bytes)."""
+    import torch
+    import torch.nn.functional as F
+    g = torch.Generator(device=device)
+    g.manual_seed(int(seed))
+    Bz, L, H, P, G, N, K = s.batch, s.seqlen, s.nheads, s.headdim, s.ngroups, s.dstate, s.nmodes
+    dty = torch.bfloat16 if s.dtype == "bf16" else torch.float32
+
+    def n(*shape):
+        return torch.randn(shape, generator=g, device=device, dtype=torch.float32)
+
+    dt = torch.clamp(F.softplus(n(Bz, L, H) - s.dt_shift), 1e-4, 1.0)
+    alpha = torch.sigmoid(n(Bz, L, H))
+    lam = torch.clamp(F.softplus(n(Bz, L, H)), 0.25, 4.0)
+    tau = torch.from_numpy(timescales(K, H)).to(device)
+    ltau = torch.log(tau)
+
+    def weights():
+        return torch.softmax(-alpha[..., None] * ltau + 0.5 * n(Bz, L, H, K), dim=-1).to(dty)
+
+    out = dict(x=n(Bz, L, H, P).to(dty), dt=dt, alpha=alpha, lam=lam, tau=tau,
+               B=n(Bz, L, G, N).to(dty), C=n(Bz, L, G, N).to(dty), w_read=weights(),
+               w_write=weights(), D=n(H))
+    if with_dy:
+        out["dy"] = n(Bz, L, H, P).to(dty)
+    return out

@@ -1,0 +1,110 @@
+"""The C-ABI library loads, exports every symbol include/frac.h declares, and rejects bad
+arguments before anything is enqueued (CPU only: none of these calls reaches the GPU)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2609_36314_gb300 import _lib
+from paper_2609_36314_gb300.api import make_dims
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "frac.h")
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(frac_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    fns = declared_functions()
+    for f in ("frac_scan_fwd", "frac_scan_bwd", "frac_decode_step", "frac_scan_fwd_workspace_size",
+              "frac_scan_bwd_workspace_size", "frac_status_string", "frac_last_error"):
+        assert f in fns
+    assert set(fns) == set(_lib.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol():
+    lib = _lib.load()
+    for f in declared_functions():
+        assert hasattr(lib, f), f
+
+
+def _fwd_call(lib, dims, ptr=ctypes.c_void_p(0x1000), **over):
+    args = dict(x=ptr, dt=ptr, alpha=ptr, lam=ptr, tau=ptr, Bm=ptr, Cm=ptr, wr=ptr, ww=ptr,
+                D=ptr, h0=None, y=ptr, hf=None, ws=ptr, wsb=1 << 40, stream=None)
+    args.update(over)
+    return lib.frac_scan_fwd(ctypes.byref(dims), args["x"], args["dt"], args["alpha"],
+                             args["lam"], args["tau"], args["Bm"], args["Cm"], args["wr"],
+                             args["ww"], args["D"], args["h0"], args["y"], args["hf"],
+                             args["ws"], args["wsb"], args["stream"])
+
+
+@pytest.mark.parametrize("bad", [
+    dict(nheads=6, ngroups=4),
+    dict(nmodes=0),
+    dict(nmodes=33),
+    dict(headdim=0),
+    dict(seqlen=-1),
+    dict(chunk=-2),
+])
+def test_invalid_dims_are_rejected(bad):
+    import torch
+    kw = dict(batch=2, seqlen=64, nheads=4, headdim=32, ngroups=1, dstate=16, nmodes=4,
+              dtype=torch.bfloat16)
+    kw.update(bad)
+    dims = make_dims(**kw)
+    lib = _lib.load()
+    st = _fwd_call(lib, dims)
+    assert st == 1, lib.frac_last_error()
+    assert lib.frac_last_error().decode()
+
+
+def test_unknown_dtype_and_null_pointers():
+    import torch
+    lib = _lib.load()
+    dims = make_dims(2, 64, 4, 32, 1, 16, 4, torch.float32)
+    dims.dtype = 7
+    assert _fwd_call(lib, dims) == 1
+    dims = make_dims(2, 64, 4, 32, 1, 16, 4, torch.float32)
+    assert _fwd_call(lib, dims, tau=None) == 1
+    assert b"tau" in lib.frac_last_error()
+    assert _fwd_call(lib, dims, x=ctypes.c_void_p(0x1004)) == 1
+    assert b"aligned" in lib.frac_last_error()
+    assert _fwd_call(lib, dims, ws=ctypes.c_void_p(0x1010)) == 1
+    assert b"workspace" in lib.frac_last_error()
+    assert _fwd_call(lib, dims, wsb=16) == 1
+    assert b"too small" in lib.frac_last_error()
+
+
+def test_unsupported_chunk_is_reported():
+    import torch
+    lib = _lib.load()
+    dims = make_dims(1, 64, 2, 32, 1, 16, 4, torch.float32, chunk=48)
+    assert _fwd_call(lib, dims) == 2
+    assert lib.frac_status_string(2) == b"unsupported"
+
+
+def test_workspace_queries():
+    import torch
+    from paper_2609_36314_gb300 import bwd_workspace_size, fwd_workspace_size
+    d = make_dims(2, 100, 4, 32, 1, 16, 4, torch.float32, chunk=32)
+    # per-chunk mode states: B * H * ceil(L / Q) * K * P * N float32
+    states = 2 * 4 * 4 * 4 * 32 * 16 * 4
+    assert fwd_workspace_size(d) >= states
+    assert bwd_workspace_size(d) >= 2 * states
+    with pytest.raises(_lib.FracError):
+        fwd_workspace_size(make_dims(2, 100, 4, 32, 3, 16, 4, torch.float32))
+
+
+def test_decode_rejects_null_state():
+    import torch
+    lib = _lib.load()
+    dims = make_dims(2, 1, 4, 32, 1, 16, 4, torch.bfloat16)
+    p = ctypes.c_void_p(0x1000)
+    st = lib.frac_decode_step(ctypes.byref(dims), p, p, p, p, p, p, p, p, p, p, None, p, None)
+    assert st == 1
+    assert b"state" in lib.frac_last_error()

@@ -1,0 +1,208 @@
+"""GPU parity of the chunked scan (forward and backward) against the fp64 oracle.
+
+Inputs are the seeded synthetic workloads; the CUDA path runs through the C ABI
+(libfrac.so via the thin binding) and is compared element by element with the
+oracle on the same bytes.  Tolerances (relative L2 per output tensor): 1e-5 on the
+float32 path, 1e-2 for bf16 inputs with float32 accumulation.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle
+from paper_2609_36314_gb300 import scan_bwd, scan_fwd, synth
+from tests.gpu_util import assert_close, dev_inputs, f64_inputs, to_host64, tol
+
+pytestmark = pytest.mark.gpu
+
+GRADS = ["dx", "ddt", "dalpha", "dlam", "dB", "dC", "dw_read", "dw_write", "dD", "dh0"]
+
+
+def _gpu_fwd(dv, **kw):
+    return scan_fwd(dv["x"], dv["dt"], dv["alpha"], dv["lam"], dv["tau"], dv["B"], dv["C"],
+                    dv["w_read"], dv["w_write"], dv["D"], dv.get("h0"), **kw)
+
+
+def _gpu_bwd(dv, **kw):
+    return scan_bwd(dv["x"], dv["dt"], dv["alpha"], dv["lam"], dv["tau"], dv["B"], dv["C"],
+                    dv["w_read"], dv["w_write"], dv["D"], dv["dy"], dv.get("h0"),
+                    dv.get("dh_final"), **kw)
+
+
+def _ora_fwd(d):
+    return oracle.fwd(d["x"], d["dt"], d["alpha"], d["lam"], d["tau"], d["B"], d["C"],
+                      d["w_read"], d["w_write"], d["D"], d.get("h0"))
+
+
+def _ora_bwd(d):
+    return oracle.bwd(d["x"], d["dt"], d["alpha"], d["lam"], d["tau"], d["B"], d["C"],
+                      d["w_read"], d["w_write"], d["D"], d["dy"], h0=d.get("h0"),
+                      dh_final=d.get("dh_final"))
+
+
+def _check_fwd(shape, seed=0, h0=False, **kw):
+    host = synth.make_scan_inputs(shape, seed=seed, with_h0=h0)
+    dv = dev_inputs(host)
+    y, hf = _gpu_fwd(dv, **kw)
+    torch.cuda.synchronize()
+    yr, hfr = _ora_fwd(f64_inputs(host))
+    t = tol(shape.dtype)
+    assert_close("y", to_host64(y), yr, t)
+    assert_close("h_final", to_host64(hf), hfr, t)
+
+
+def _check_bwd(shape, seed=0, h0=False, dhf=False, **kw):
+    host = synth.make_scan_inputs(shape, seed=seed, with_dy=True, with_h0=h0, with_dh_final=dhf)
+    dv = dev_inputs(host)
+    g = _gpu_bwd(dv, **kw)
+    torch.cuda.synchronize()
+    gr = _ora_bwd(f64_inputs(host))
+    t = tol(shape.dtype)
+    for k in GRADS:
+        assert_close(k, to_host64(g[k]), gr[k], t)
+
+
+# ------------------------------------------------------------------ float32 path (1e-5)
+def test_fwd_f32_small_workload():
+    """B1 L256 H2 P32 N16 K4, chunk 64, float32."""
+    _check_fwd(synth.WORKLOADS["fwd_f32_small"], chunk=64)
+
+
+@pytest.mark.parametrize("chunk", [16, 32, 64])
+@pytest.mark.parametrize("L", [1, 37, 100, 128])
+def test_fwd_f32_chunks_and_ragged_lengths(chunk, L):
+    s = synth.Shape(2, L, 4, 24, 2, 12, 3, chunk, "f32")
+    _check_fwd(s, seed=L, h0=True, chunk=chunk)
+
+
+@pytest.mark.parametrize("chunk", [16, 64])
+def test_bwd_f32(chunk):
+    s = synth.Shape(2, 150, 4, 16, 2, 12, 3, chunk, "f32")
+    _check_bwd(s, seed=3, h0=True, dhf=True, chunk=chunk)
+
+
+def test_bwd_f32_small_workload_shape():
+    s = synth.WORKLOADS["fwd_f32_small"]
+    _check_bwd(s, seed=1, chunk=64)
+
+
+def test_odd_sizes_f32():
+    """N not a multiple of 4, P not a multiple of 8, one head, K = 1."""
+    _check_fwd(synth.Shape(1, 45, 1, 5, 1, 5, 1, 0, "f32"), seed=9, h0=True)
+    _check_bwd(synth.Shape(1, 45, 1, 5, 1, 5, 1, 0, "f32"), seed=9, h0=True, dhf=True)
+
+
+def test_empty_sequence():
+    s = synth.Shape(2, 0, 3, 8, 1, 4, 2, 0, "f32")
+    host = synth.make_scan_inputs(s, with_h0=True, with_dy=True, with_dh_final=True)
+    dv = dev_inputs(host)
+    y, hf = _gpu_fwd(dv)
+    assert y.numel() == 0
+    assert torch.equal(hf, dv["h0"])
+    g = _gpu_bwd(dv)
+    assert torch.equal(g["dh0"], dv["dh_final"])
+    assert torch.count_nonzero(g["dD"]) == 0
+
+
+# ------------------------------------------------------------------ bf16 path (1e-2)
+def test_fwd_bf16_b4_l2048_workload():
+    """B4 L2048 H16 P64 N64 K8, chunk 128 requested by the workload: full-size parity."""
+    s = synth.WORKLOADS["fwd_bf16_b4_l2048"]
+    _check_fwd(s)
+
+
+@pytest.mark.parametrize("L", [1, 63, 200])
+def test_fwd_bf16_ragged(L):
+    _check_fwd(synth.Shape(2, L, 4, 64, 1, 64, 8, 0, "bf16"), seed=L, h0=True)
+
+
+def test_bwd_bf16_medium():
+    _check_bwd(synth.Shape(2, 300, 4, 64, 1, 64, 8, 0, "bf16"), seed=5, h0=True, dhf=True)
+
+
+def test_bwd_bf16_groups():
+    _check_bwd(synth.Shape(1, 130, 4, 32, 2, 32, 4, 0, "bf16"), seed=6)
+
+
+def test_force_simt_matches_default_path():
+    s = synth.Shape(2, 260, 4, 64, 1, 128, 8, 0, "bf16")
+    host = synth.make_scan_inputs(s, seed=12, with_dy=True)
+    dv = dev_inputs(host)
+    y0, h0 = _gpu_fwd(dv)
+    y1, h1 = _gpu_fwd(dv, force_simt=True)
+    torch.cuda.synchronize()
+    yr, hr = _ora_fwd(f64_inputs(host))
+    assert_close("y default", to_host64(y0), yr, 1e-2)
+    assert_close("y simt", to_host64(y1), yr, 1e-2)
+    assert_close("h default", to_host64(h0), hr, 1e-2)
+    assert_close("h simt", to_host64(h1), hr, 1e-2)
+
+
+# ------------------------------------------------------------------ full-size workloads, sampled
+def _slice_streams(host, b, heads):
+    """Oracle inputs for batch row b and a subset of heads (B/C groups kept whole; G = 1)."""
+    out = {}
+    for k, v in host.items():
+        a = synth.to_f64(v)
+        if k in ("x", "dy", "w_read", "w_write", "dt", "alpha", "lam"):
+            out[k] = a[b:b + 1][:, :, heads]
+        elif k in ("B", "C"):
+            out[k] = a[b:b + 1]
+        elif k in ("tau",):
+            out[k] = a[heads]
+        elif k == "D":
+            out[k] = a[heads]
+        else:
+            out[k] = a
+    return out
+
+
+@pytest.mark.slow
+def test_train_workload_fwd_bwd_sampled():
+    """B8 L4096 H64 P64 N128 K8 bf16 at full size, in the configuration the benchmark times.
+    y, h_final and every per-stream gradient are compared on two (batch, head) streams; dy is
+    zero outside those streams so that dB, dC (sums over all heads) and dD are exactly the
+    sampled streams' contributions, which the oracle computes."""
+    s = synth.WORKLOADS["train_bf16_b8_l4096"]
+    host = synth.make_scan_inputs(s, seed=0, with_dy=True)
+    b, heads = 3, [5, 37]
+    mask = np.zeros((s.batch, 1, s.nheads, 1), dtype=bool)
+    mask[b, 0, heads] = True
+    dy = synth.bf16_bits_to_f32(host["dy"]) * mask
+    host["dy"] = synth.f32_to_bf16_bits(dy)
+    dv = dev_inputs(host)
+    y, hf = _gpu_fwd(dv)
+    g = _gpu_bwd(dv)
+    torch.cuda.synchronize()
+    sub = _slice_streams(host, b, heads)
+    yr, hfr = _ora_fwd(sub)
+    gr = _ora_bwd(sub)
+    assert_close("y", to_host64(y[b:b + 1][:, :, heads]), yr, 1e-2)
+    assert_close("h_final", to_host64(hf[b:b + 1][:, heads]), hfr, 1e-2)
+    for k in ("dx", "dw_read", "dw_write"):
+        assert_close(k, to_host64(g[k][b:b + 1][:, :, heads]), gr[k], 1e-2)
+    for k in ("ddt", "dalpha", "dlam"):
+        assert_close(k, to_host64(g[k][b:b + 1][:, :, heads]), gr[k], 1e-2)
+    assert_close("dh0", to_host64(g["dh0"][b:b + 1][:, heads]), gr["dh0"], 1e-2)
+    assert_close("dB", to_host64(g["dB"][b:b + 1]), gr["dB"], 1e-2)
+    assert_close("dC", to_host64(g["dC"][b:b + 1]), gr["dC"], 1e-2)
+    assert_close("dD", to_host64(g["dD"][heads]), gr["dD"], 1e-2)
+    # streams outside the sample got no upstream gradient
+    other = torch.ones(s.batch, dtype=torch.bool)
+    other[b] = False
+    assert torch.count_nonzero(g["dB"][other]) == 0
+
+
+@pytest.mark.slow
+def test_long_prefill_workload_sampled():
+    """B1 L65536 H64 P64 N128 K8 bf16, Delta skewed small: y and h_final of two heads."""
+    s = synth.WORKLOADS["prefill_bf16_l65536"]
+    host = synth.make_scan_inputs(s, seed=0)
+    dv = dev_inputs(host)
+    y, hf = _gpu_fwd(dv)
+    torch.cuda.synchronize()
+    heads = [0, 50]
+    sub = _slice_streams(host, 0, heads)
+    yr, hfr = _ora_fwd(sub)
+    assert_close("y", to_host64(y[:, :, heads]), yr, 1e-2)
+    assert_close("h_final", to_host64(hf[:, heads]), hfr, 1e-2)
