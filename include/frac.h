@@ -16,7 +16,9 @@
  *
  * Conventions shared by every entry point
  *   - Tensor arguments are device pointers owned by the caller, row-major and contiguous,
- *     16-byte aligned, and must not alias each other (except where stated).  The library
+ *     aligned at least to their element size, and must not alias each other (except where
+ *     stated).  16-byte alignment of every tensor lets the library pick its vectorised and
+ *     TMA-fed kernels; otherwise it uses kernels with scalar accesses.  The library
  *     never allocates device memory and keeps no state between calls apart from a
  *     thread-local error message.
  *   - `stream` is a cudaStream_t (NULL = the legacy default stream).  Every call only

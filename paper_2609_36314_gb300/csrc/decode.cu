@@ -118,9 +118,13 @@ cudaError_t launch_decode_t(const DecodeArgs &a, const void *x, const void *Bt, 
     const int64_t rows = int64_t(a.B) * a.H * a.P;
     const int64_t blocks = (rows * 32 + 255) / 256;
     // vector path: N a multiple of 128 so that every lane runs the same number of iterations
-    // (the mode broadcasts use full-warp shuffles)
+    // (the mode broadcasts use full-warp shuffles), the state 16-byte aligned and B/C aligned
+    // to four elements
+    const bool vec = a.N % 128 == 0 && (reinterpret_cast<uintptr_t>(a.state) & 15u) == 0 &&
+                     (reinterpret_cast<uintptr_t>(Bt) % (4 * sizeof(T))) == 0 &&
+                     (reinterpret_cast<uintptr_t>(Ct) % (4 * sizeof(T))) == 0;
     trace_begin("decode_step", st);
-    if (a.N % 128 == 0)
+    if (vec)
         decode_step_kernel<T, true><<<dim3(unsigned(blocks)), 256, 0, st>>>(
             a, (const T *)x, (const T *)Bt, (const T *)Ct, (const T *)wr, (const T *)ww, (T *)y);
     else

@@ -24,21 +24,27 @@ frac_status cuda_status(cudaError_t e, const char *where) {
     return fail(FRAC_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
 }
 
-bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+bool aligned_to(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 constexpr size_t kAlign = 256;
 size_t round_up(size_t v) { return (v + kAlign - 1) / kAlign * kAlign; }
 
-#define REQUIRE_PTR(p)                                                                         \
+// Every tensor must be aligned to its element size (float32 tensors: 4 bytes; dtype tensors:
+// 2 or 4 bytes).  Stronger alignment only selects faster kernels.
+#define REQUIRE_PTR_A(p, a)                                                                    \
     do {                                                                                       \
         if (!(p)) return fail(FRAC_ERR_INVALID_ARGUMENT, "%s must not be NULL", #p);           \
-        if (!aligned16(p)) return fail(FRAC_ERR_INVALID_ARGUMENT, "%s is not 16-byte aligned", #p); \
+        if (!aligned_to(p, a))                                                                 \
+            return fail(FRAC_ERR_INVALID_ARGUMENT, "%s is not aligned to %d bytes", #p, int(a)); \
     } while (0)
-#define OPTIONAL_PTR(p)                                                                        \
+#define OPTIONAL_PTR_A(p, a)                                                                   \
     do {                                                                                       \
-        if ((p) && !aligned16(p))                                                              \
-            return fail(FRAC_ERR_INVALID_ARGUMENT, "%s is not 16-byte aligned", #p);           \
+        if ((p) && !aligned_to(p, a))                                                          \
+            return fail(FRAC_ERR_INVALID_ARGUMENT, "%s is not aligned to %d bytes", #p, int(a)); \
     } while (0)
+#define REQUIRE_PTR(p) REQUIRE_PTR_A(p, sizeof(*(p)))
+#define OPTIONAL_PTR(p) OPTIONAL_PTR_A(p, sizeof(*(p)))
+#define REQUIRE_T(p) REQUIRE_PTR_A(p, elem(d))
 
 frac_status check_dims(const frac_dims *d, bool need_seq) {
     if (!d) return fail(FRAC_ERR_INVALID_ARGUMENT, "dims must not be NULL");
@@ -159,15 +165,15 @@ frac_status frac_scan_fwd(const frac_dims *d, const void *x, const float *dt, co
     OPTIONAL_PTR(h0);
     OPTIONAL_PTR(h_final);
     if (d->seqlen > 0) {
-        REQUIRE_PTR(x);
+        REQUIRE_T(x);
         REQUIRE_PTR(dt);
         REQUIRE_PTR(alpha);
         REQUIRE_PTR(lam);
-        REQUIRE_PTR(Bm);
-        REQUIRE_PTR(Cm);
-        REQUIRE_PTR(w_read);
-        REQUIRE_PTR(w_write);
-        REQUIRE_PTR(y);
+        REQUIRE_T(Bm);
+        REQUIRE_T(Cm);
+        REQUIRE_T(w_read);
+        REQUIRE_T(w_write);
+        REQUIRE_T(y);
     }
     frac::ScanDims sd;
     if ((s = plan(d, &sd))) return s;
@@ -206,11 +212,11 @@ frac_status frac_scan_bwd(const frac_dims *d, const void *x, const float *dt, co
     OPTIONAL_PTR(dh_final);
     OPTIONAL_PTR(dh0);
     if (d->seqlen > 0) {
-        REQUIRE_PTR(x); REQUIRE_PTR(dt); REQUIRE_PTR(alpha); REQUIRE_PTR(lam);
-        REQUIRE_PTR(Bm); REQUIRE_PTR(Cm); REQUIRE_PTR(w_read); REQUIRE_PTR(w_write);
-        REQUIRE_PTR(dy); REQUIRE_PTR(dx); REQUIRE_PTR(ddt); REQUIRE_PTR(dalpha);
-        REQUIRE_PTR(dlam); REQUIRE_PTR(dB); REQUIRE_PTR(dC); REQUIRE_PTR(dw_read);
-        REQUIRE_PTR(dw_write);
+        REQUIRE_T(x); REQUIRE_PTR(dt); REQUIRE_PTR(alpha); REQUIRE_PTR(lam);
+        REQUIRE_T(Bm); REQUIRE_T(Cm); REQUIRE_T(w_read); REQUIRE_T(w_write);
+        REQUIRE_T(dy); REQUIRE_T(dx); REQUIRE_PTR(ddt); REQUIRE_PTR(dalpha);
+        REQUIRE_PTR(dlam); REQUIRE_T(dB); REQUIRE_T(dC); REQUIRE_T(dw_read);
+        REQUIRE_T(dw_write);
     }
     frac::ScanDims sd;
     if ((s = plan(d, &sd))) return s;
@@ -247,9 +253,9 @@ frac_status frac_decode_step(const frac_dims *d, const void *x_t, const float *d
     g_err[0] = 0;
     frac_status s = check_dims(d, false);
     if (s) return s;
-    REQUIRE_PTR(x_t); REQUIRE_PTR(dt); REQUIRE_PTR(alpha); REQUIRE_PTR(lam); REQUIRE_PTR(tau);
-    REQUIRE_PTR(B_t); REQUIRE_PTR(C_t); REQUIRE_PTR(w_read); REQUIRE_PTR(w_write);
-    REQUIRE_PTR(D); REQUIRE_PTR(state); REQUIRE_PTR(y_t);
+    REQUIRE_T(x_t); REQUIRE_PTR(dt); REQUIRE_PTR(alpha); REQUIRE_PTR(lam); REQUIRE_PTR(tau);
+    REQUIRE_T(B_t); REQUIRE_T(C_t); REQUIRE_T(w_read); REQUIRE_T(w_write);
+    REQUIRE_PTR(D); REQUIRE_PTR(state); REQUIRE_T(y_t);
     frac::DecodeArgs a;
     a.B = int(d->batch); a.H = int(d->nheads); a.P = int(d->headdim); a.G = int(d->ngroups);
     a.N = int(d->dstate); a.K = int(d->nmodes);

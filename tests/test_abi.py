@@ -72,7 +72,7 @@ def test_unknown_dtype_and_null_pointers():
     dims = make_dims(2, 64, 4, 32, 1, 16, 4, torch.float32)
     assert _fwd_call(lib, dims, tau=None) == 1
     assert b"tau" in lib.frac_last_error()
-    assert _fwd_call(lib, dims, x=ctypes.c_void_p(0x1004)) == 1
+    assert _fwd_call(lib, dims, x=ctypes.c_void_p(0x1002)) == 1
     assert b"aligned" in lib.frac_last_error()
     assert _fwd_call(lib, dims, ws=ctypes.c_void_p(0x1010)) == 1
     assert b"workspace" in lib.frac_last_error()
