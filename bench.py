@@ -44,6 +44,8 @@ def parse():
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--batch", type=int, default=0,
+                    help="override the training workload's batch (small profiling captures)")
     return ap.parse_args()
 
 
@@ -246,6 +248,8 @@ def main():
         return float(t.item())
 
     s = shape_of(TRAIN)
+    if args.batch:
+        s = s.replace(batch=args.batch)
     inp = synth.make_scan_inputs_torch(s, seed=1000 + rank, device=dev, with_dy=True)
     dims = make_dims(s.batch, s.seqlen, s.nheads, s.headdim, s.ngroups, s.dstate, s.nmodes,
                      torch.bfloat16)
@@ -369,6 +373,8 @@ def main():
             "roofline": roofline, "kernels": kern, "gpu_launches": launches,
             "e2e": e2e, "decode": decode, "clocks": clk, "peaks_source": peaks["source"],
         }
+        if args.batch:
+            line["config"]["workload"] += f" (batch overridden to {args.batch})"
         if world == 1 and not args.no_cpu_baseline:
             line["cpu_baseline"] = cpu_baseline()
         print(json.dumps(line), flush=True)
