@@ -152,6 +152,29 @@ frac_status frac_decode_step(const frac_dims *dims, const void *x_t, const float
                              void *stream);
 
 /*
+ * Allocation-free forward scan.  The paper has no counterpart; this exists for callers that
+ * cannot hand the library scratch memory: for example code running inside a host application
+ * that owns the whole device-memory budget and gives its plug-ins no allocator, or code that
+ * may only touch the buffers it was given once it is running.  Same arguments and results as
+ * frac_scan_fwd without the workspace: the per-chunk mode states go to a fixed device array
+ * of FRAC_SCAN_FWD_STATIC_SCRATCH_BYTES that the library owns on every GPU that loads it, held
+ * until the process exits.  No device memory is allocated by the call.
+ *   - Problems whose frac_scan_fwd_workspace_size exceeds that size are rejected with
+ *     FRAC_ERR_UNSUPPORTED (frac_last_error() says how much they need); nothing is enqueued.
+ *   - The first call on a device looks up the array's address on that device (a CUDA runtime
+ *     query, made with that device current); make the first call before any stream capture.
+ *   - All calls share the array.  Calls whose GPU work overlaps (other streams, other host
+ *     threads on the same device) race on it and must be serialised by the caller.  Nothing in
+ *     it needs to start at zero: every per-chunk state is written before it is read.
+ */
+#define FRAC_SCAN_FWD_STATIC_SCRATCH_BYTES ((size_t)64 << 20)
+frac_status frac_scan_fwd_static(const frac_dims *dims, const void *x, const float *dt,
+                                 const float *alpha, const float *lam, const float *tau,
+                                 const void *Bm, const void *Cm, const void *w_read,
+                                 const void *w_write, const float *D, const float *h0, void *y,
+                                 float *h_final, void *stream);
+
+/*
  * Kernel tracing (a profiling aid, off by default).  While enabled, every kernel the library
  * launches is bracketed by two CUDA events recorded on its launch stream (do not enable it
  * while a stream is being captured into a CUDA graph).  frac_trace_collect waits for the

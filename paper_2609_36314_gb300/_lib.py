@@ -20,6 +20,7 @@ EXPORTS = (
     "frac_scan_bwd_workspace_size",
     "frac_scan_bwd",
     "frac_decode_step",
+    "frac_scan_fwd_static",
     "frac_trace_enable",
     "frac_trace_collect",
     "frac_trace_reset",
@@ -31,6 +32,7 @@ FRAC_OK = 0
 FRAC_DTYPE_F32 = 0
 FRAC_DTYPE_BF16 = 1
 FRAC_FLAG_FORCE_SIMT = 1
+FRAC_SCAN_FWD_STATIC_SCRATCH_BYTES = 64 << 20
 
 
 class FracDims(ctypes.Structure):
@@ -81,6 +83,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.frac_scan_bwd.restype = st
         lib.frac_decode_step.argtypes = [dims_p] + [P] * 12 + [P]
         lib.frac_decode_step.restype = st
+        lib.frac_scan_fwd_static.argtypes = [dims_p] + [P] * 13 + [P]
+        lib.frac_scan_fwd_static.restype = st
         lib.frac_trace_enable.argtypes = [ctypes.c_int]
         lib.frac_trace_enable.restype = st
         lib.frac_trace_collect.argtypes = [ctypes.POINTER(FracTraceEntry), ctypes.c_int,

@@ -107,6 +107,24 @@ def scan_fwd(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, h0=None, *, chunk
     return y, (h_final if want_final_state else None)
 
 
+def scan_fwd_static(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, h0=None, *, chunk=0,
+                    force_simt=False, want_final_state=True, y=None, h_final=None, stream=None):
+    """scan_fwd for callers that cannot provide scratch memory: the library's own fixed device
+    array (FRAC_SCAN_FWD_STATIC_SCRATCH_BYTES) holds the per-chunk states, so this call
+    allocates nothing besides the outputs it is not given.  Calls that overlap on the GPU
+    race on that array."""
+    dims, (Bz, L, H, P, G, N, K) = _scan_dims(x, B, tau, chunk, force_simt)
+    if y is None:
+        y = torch.empty_like(x)
+    if want_final_state and h_final is None:
+        h_final = torch.empty((Bz, H, K, P, N), dtype=torch.float32, device=x.device)
+    _lib.check(_lib.load().frac_scan_fwd_static(
+        ctypes.byref(dims), _ptr(x), _ptr(dt), _ptr(alpha), _ptr(lam), _ptr(tau), _ptr(B),
+        _ptr(C), _ptr(w_read), _ptr(w_write), _ptr(D), _ptr(h0), _ptr(y),
+        _ptr(h_final if want_final_state else None), _stream(stream)), "frac_scan_fwd_static")
+    return y, (h_final if want_final_state else None)
+
+
 def scan_bwd(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, dy, h0=None, dh_final=None, *,
              chunk=0, force_simt=False, want_dh0=True, workspace=None, out=None, stream=None):
     """Backward of scan_fwd.  Returns a dict of gradients (dx, ddt, dalpha, dlam, dB, dC,

@@ -115,6 +115,10 @@ BwdLayout bwd_layout(const frac_dims *d, const frac::ScanDims &sd) {
 
 }  // namespace
 
+namespace frac {
+void set_last_error(const char *msg) { snprintf(g_err, sizeof(g_err), "%s", msg); }
+}  // namespace frac
+
 extern "C" {
 
 const char *frac_status_string(frac_status s) {

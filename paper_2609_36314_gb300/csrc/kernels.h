@@ -7,6 +7,9 @@
 
 namespace frac {
 
+// Sets the message frac_last_error() returns on the calling thread.
+void set_last_error(const char *msg);
+
 // Tracing hooks (no-ops unless frac_trace_enable(1)); bracket each kernel launch.
 void trace_begin(const char *name, cudaStream_t st);
 void trace_end(cudaStream_t st);
