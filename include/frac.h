@@ -67,7 +67,11 @@ typedef enum { FRAC_DTYPE_F32 = 0, FRAC_DTYPE_BF16 = 1 } frac_dtype;
 
 /* Bits of frac_dims.flags. */
 enum {
-    FRAC_FLAG_FORCE_SIMT = 1 /* use the CUDA-core chunked kernels even where tensor-core ones exist */
+    /* Use the CUDA-core chunked kernels even where tensor-core ones exist.  Without it, bf16
+       calls with headdim % 32 == 0, dstate in {64, 128} and nmodes in {4, 8} run the forward on
+       the tensor cores (TMA-fed tcgen05 MMAs, chunk 128); they need x, Bm, Cm, y (and h_final)
+       16-byte aligned. */
+    FRAC_FLAG_FORCE_SIMT = 1
 };
 
 typedef struct {
@@ -79,8 +83,8 @@ typedef struct {
     int64_t dstate;  /* N >= 1 */
     int64_t nmodes;  /* K, 1 <= K <= 32 */
     int64_t chunk;   /* Q: 0 = implementation's choice; otherwise one of the sizes the selected
-                        path supports (16, 32 or 64 on CUDA cores, 128 on tensor cores).
-                        Results do not depend on Q beyond rounding. */
+                        path supports (128 on the tensor-core forward; 16, 32 or 64 on the
+                        CUDA-core kernels).  Results do not depend on Q beyond rounding. */
     int32_t dtype;   /* frac_dtype */
     int32_t flags;   /* FRAC_FLAG_* */
 } frac_dims;
@@ -190,6 +194,13 @@ typedef struct {
 frac_status frac_trace_enable(int on);
 frac_status frac_trace_collect(frac_trace_entry *out, int capacity, int *count);
 frac_status frac_trace_reset(void);
+
+/*
+ * Waits for `stream` and reports the device status word of a scan call's workspace:
+ * FRAC_ERR_TIMEOUT if one of the call's kernels gave up on a bounded device-side wait (its
+ * outputs are then incomplete), FRAC_OK otherwise.  The word is reset by every scan call.
+ */
+frac_status frac_workspace_status(const void *workspace, void *stream);
 
 /* Static description of a status code. */
 const char *frac_status_string(frac_status status);

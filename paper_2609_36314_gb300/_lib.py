@@ -21,6 +21,7 @@ EXPORTS = (
     "frac_scan_bwd",
     "frac_decode_step",
     "frac_scan_fwd_static",
+    "frac_workspace_status",
     "frac_trace_enable",
     "frac_trace_collect",
     "frac_trace_reset",
@@ -85,6 +86,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.frac_decode_step.restype = st
         lib.frac_scan_fwd_static.argtypes = [dims_p] + [P] * 13 + [P]
         lib.frac_scan_fwd_static.restype = st
+        lib.frac_workspace_status.argtypes = [P, P]
+        lib.frac_workspace_status.restype = st
         lib.frac_trace_enable.argtypes = [ctypes.c_int]
         lib.frac_trace_enable.restype = st
         lib.frac_trace_collect.argtypes = [ctypes.POINTER(FracTraceEntry), ctypes.c_int,

@@ -67,8 +67,12 @@ frac_status check_dims(const frac_dims *d, bool need_seq) {
 
 size_t elem(const frac_dims *d) { return d->dtype == FRAC_DTYPE_BF16 ? 2 : 4; }
 
-// Path selection and the dims the kernels see.
-frac_status plan(const frac_dims *d, frac::ScanDims *sd) {
+// Path selection and the dims the kernels see.  The forward uses the tensor-core kernels
+// for bf16 shapes they support (unless FRAC_FLAG_FORCE_SIMT); everything else, and the
+// backward, runs on the CUDA-core kernels.
+enum Path { PATH_SIMT = 0, PATH_TC = 1 };
+
+frac_status plan(const frac_dims *d, frac::ScanDims *sd, int *path, bool backward) {
     sd->B = int(d->batch);
     sd->L = int(d->seqlen);
     sd->H = int(d->nheads);
@@ -76,15 +80,28 @@ frac_status plan(const frac_dims *d, frac::ScanDims *sd) {
     sd->G = int(d->ngroups);
     sd->N = int(d->dstate);
     sd->K = int(d->nmodes);
-    const int Q = frac::simt_pick_chunk(*sd, int(d->chunk));
-    if (Q == 0)
-        return fail(FRAC_ERR_UNSUPPORTED,
-                    "no chunk size fits these dims on the CUDA-core path (chunk=%lld, P=%d, N=%d, K=%d)",
-                    (long long)d->chunk, sd->P, sd->N, sd->K);
-    sd->Q = Q;
-    sd->nc = (sd->L + Q - 1) / Q;
+    const bool tc = !backward && !(d->flags & FRAC_FLAG_FORCE_SIMT) &&
+                    frac::tc_supported(*sd, d->dtype) && (d->chunk == 0 || d->chunk == 128);
+    if (tc) {
+        sd->Q = 128;
+        *path = PATH_TC;
+    } else {
+        const int Q = frac::simt_pick_chunk(*sd, int(d->chunk));
+        if (Q == 0)
+            return fail(FRAC_ERR_UNSUPPORTED,
+                        "chunk=%lld is not supported for these dims (P=%d, N=%d, K=%d, dtype=%d); "
+                        "use 0 to let the library choose",
+                        (long long)d->chunk, sd->P, sd->N, sd->K, d->dtype);
+        sd->Q = Q;
+        *path = PATH_SIMT;
+    }
+    sd->nc = (sd->L + sd->Q - 1) / sd->Q;
     return FRAC_OK;
 }
+
+// Workspace layout: [0, 256) device status word (FRAC_OK or FRAC_ERR_TIMEOUT written by
+// kernels with bounded waits), then the per-chunk states and accumulators.
+constexpr size_t kStatusBytes = kAlign;
 
 struct FwdLayout {
     size_t s_in, total;
@@ -93,10 +110,12 @@ struct BwdLayout {
     size_t s_in, ds_out, db, dc, total;
 };
 
-FwdLayout fwd_layout(const frac_dims *d, const frac::ScanDims &sd) {
+FwdLayout fwd_layout(const frac_dims *d, const frac::ScanDims &sd, int path) {
     FwdLayout l;
-    l.s_in = 0;
-    l.total = round_up(frac::simt_state_elems(sd) * elem(d));
+    l.s_in = kStatusBytes;
+    const size_t elems = path == PATH_TC ? frac::tc_state_elems(sd) : frac::simt_state_elems(sd);
+    const size_t esz = path == PATH_TC ? 2 : elem(d);
+    l.total = kStatusBytes + round_up(elems * esz);
     return l;
 }
 
@@ -104,9 +123,9 @@ BwdLayout bwd_layout(const frac_dims *d, const frac::ScanDims &sd) {
     BwdLayout l;
     const size_t st = round_up(frac::simt_state_elems(sd) * elem(d));
     const size_t ngn = size_t(sd.B) * sd.L * sd.G * sd.N;
-    l.s_in = 0;
-    l.ds_out = st;
-    l.db = 2 * st;
+    l.s_in = kStatusBytes;
+    l.ds_out = l.s_in + st;
+    l.db = l.ds_out + st;
     const size_t acc = (d->dtype == FRAC_DTYPE_BF16) ? round_up(ngn * sizeof(float)) : 0;
     l.dc = l.db + acc;
     l.total = l.dc + acc;
@@ -134,14 +153,28 @@ const char *frac_status_string(frac_status s) {
 
 const char *frac_last_error(void) { return g_err; }
 
+frac_status frac_workspace_status(const void *workspace, void *stream) {
+    g_err[0] = 0;
+    if (!workspace || !aligned_to(workspace, kAlign))
+        return fail(FRAC_ERR_INVALID_ARGUMENT, "workspace must be the 256-byte aligned workspace of a call");
+    int word = 0;
+    cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e == cudaSuccess) e = cudaMemcpy(&word, workspace, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_status(e, "frac_workspace_status");
+    if (word == FRAC_ERR_TIMEOUT)
+        return fail(FRAC_ERR_TIMEOUT, "a device-side wait gave up (work of that call is incomplete)");
+    return word == 0 ? FRAC_OK : fail(FRAC_ERR_CUDA, "device status word %d", word);
+}
+
 frac_status frac_scan_fwd_workspace_size(const frac_dims *d, size_t *bytes) {
     g_err[0] = 0;
     frac_status s = check_dims(d, true);
     if (s) return s;
     if (!bytes) return fail(FRAC_ERR_INVALID_ARGUMENT, "bytes must not be NULL");
     frac::ScanDims sd;
-    if ((s = plan(d, &sd))) return s;
-    *bytes = fwd_layout(d, sd).total;
+    int path;
+    if ((s = plan(d, &sd, &path, false))) return s;
+    *bytes = fwd_layout(d, sd, path).total;
     return FRAC_OK;
 }
 
@@ -151,7 +184,8 @@ frac_status frac_scan_bwd_workspace_size(const frac_dims *d, size_t *bytes) {
     if (s) return s;
     if (!bytes) return fail(FRAC_ERR_INVALID_ARGUMENT, "bytes must not be NULL");
     frac::ScanDims sd;
-    if ((s = plan(d, &sd))) return s;
+    int path;
+    if ((s = plan(d, &sd, &path, true))) return s;
     *bytes = bwd_layout(d, sd).total;
     return FRAC_OK;
 }
@@ -180,9 +214,20 @@ frac_status frac_scan_fwd(const frac_dims *d, const void *x, const float *dt, co
         REQUIRE_T(y);
     }
     frac::ScanDims sd;
-    if ((s = plan(d, &sd))) return s;
-    const FwdLayout l = fwd_layout(d, sd);
-    if (l.total > 0) {
+    int path;
+    if ((s = plan(d, &sd, &path, false))) return s;
+    const FwdLayout l = fwd_layout(d, sd, path);
+    if (path == PATH_TC && d->seqlen > 0) {
+        const void *need16[] = {x, Bm, Cm, y};
+        for (const void *q : need16)
+            if (!aligned_to(q, 16))
+                return fail(FRAC_ERR_INVALID_ARGUMENT,
+                            "the tensor-core path needs x, Bm, Cm and y 16-byte aligned "
+                            "(or set FRAC_FLAG_FORCE_SIMT)");
+        if (h_final && !aligned_to(h_final, 16))
+            return fail(FRAC_ERR_INVALID_ARGUMENT, "h_final is not 16-byte aligned");
+    }
+    {
         if (!workspace) return fail(FRAC_ERR_INVALID_ARGUMENT, "workspace must not be NULL");
         if (reinterpret_cast<uintptr_t>(workspace) % kAlign)
             return fail(FRAC_ERR_INVALID_ARGUMENT, "workspace is not 256-byte aligned");
@@ -195,8 +240,15 @@ frac_status frac_scan_fwd(const frac_dims *d, const void *x, const float *dt, co
     p.dt = dt; p.alpha = alpha; p.lam = lam; p.tau = tau; p.D = D; p.h0 = h0;
     p.y = y; p.h_final = h_final;
     char *ws = static_cast<char *>(workspace);
-    return cuda_status(frac::simt_scan_fwd(sd, d->dtype, p, ws + l.s_in, (cudaStream_t)stream),
-                       "frac_scan_fwd");
+    cudaStream_t st = (cudaStream_t)stream;
+    cudaError_t e = cudaMemsetAsync(ws, 0, sizeof(int), st);
+    if (e == cudaSuccess) {
+        if (path == PATH_TC)
+            e = frac::tc_scan_fwd(sd, p, ws + l.s_in, reinterpret_cast<int *>(ws), st);
+        else
+            e = frac::simt_scan_fwd(sd, d->dtype, p, ws + l.s_in, st);
+    }
+    return cuda_status(e, "frac_scan_fwd");
 }
 
 frac_status frac_scan_bwd(const frac_dims *d, const void *x, const float *dt, const float *alpha,
@@ -223,9 +275,10 @@ frac_status frac_scan_bwd(const frac_dims *d, const void *x, const float *dt, co
         REQUIRE_T(dw_write);
     }
     frac::ScanDims sd;
-    if ((s = plan(d, &sd))) return s;
+    int path;
+    if ((s = plan(d, &sd, &path, true))) return s;
     const BwdLayout l = bwd_layout(d, sd);
-    if (l.total > 0) {
+    {
         if (!workspace) return fail(FRAC_ERR_INVALID_ARGUMENT, "workspace must not be NULL");
         if (reinterpret_cast<uintptr_t>(workspace) % kAlign)
             return fail(FRAC_ERR_INVALID_ARGUMENT, "workspace is not 256-byte aligned");
@@ -244,9 +297,11 @@ frac_status frac_scan_bwd(const frac_dims *d, const void *x, const float *dt, co
                                                 : static_cast<float *>(dB);
     float *dC_acc = d->dtype == FRAC_DTYPE_BF16 ? reinterpret_cast<float *>(ws + l.dc)
                                                 : static_cast<float *>(dC);
-    return cuda_status(frac::simt_scan_bwd(sd, d->dtype, p, ws + l.s_in, ws + l.ds_out, dB_acc,
-                                           dC_acc, (cudaStream_t)stream),
-                       "frac_scan_bwd");
+    cudaStream_t st = (cudaStream_t)stream;
+    cudaError_t e = cudaMemsetAsync(ws, 0, sizeof(int), st);
+    if (e == cudaSuccess)
+        e = frac::simt_scan_bwd(sd, d->dtype, p, ws + l.s_in, ws + l.ds_out, dB_acc, dC_acc, st);
+    return cuda_status(e, "frac_scan_bwd");
 }
 
 frac_status frac_decode_step(const frac_dims *d, const void *x_t, const float *dt,

@@ -47,4 +47,10 @@ cudaError_t simt_scan_fwd(const ScanDims &d, int dtype, const ScanPtrs &p, void 
 cudaError_t simt_scan_bwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in,
                           void *dS_out, float *dB_acc, float *dC_acc, cudaStream_t st);
 
+// Tensor-core (tcgen05) path: bf16 inputs, chunk 128, P % 32 == 0, N in {64, 128}, K in {4, 8}.
+bool tc_supported(const ScanDims &d, int dtype);
+size_t tc_state_elems(const ScanDims &d);  // bf16 elements of the per-chunk state workspace
+cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, int *err,
+                        cudaStream_t st);
+
 }  // namespace frac

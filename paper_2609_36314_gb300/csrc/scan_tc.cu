@@ -1,0 +1,619 @@
+// Tensor-core (tcgen05 / TMEM / TMA) chunked Frac scan for bf16 inputs, sm_103a.
+//
+// Same chunked evaluation order as the CUDA-core kernels (App. E of the paper), with chunk
+// Q = 128 and the two state contractions of every chunk on the tensor cores:
+//
+//   tc_state_pass  (chunk-serial; one CTA per (b, h, 32-wide slice of P)):
+//        the P-slice of every mode's state lives in tensor memory as fp32, lanes = (mode%4, p),
+//        columns = (mode/4, n).  Per chunk: emit the entering state (bf16) for the output
+//        kernel, scale it by d_m = exp(-E_end/tau_m) in place, then accumulate
+//        S_m += sum_k s_{k,m} x_k B_k^T  as  D[(m,p), n] += A[(m,p), k] * B[k, n]
+//        (A = s o x generated in shared memory, B = the chunk of B loaded by TMA).
+//        Run over the chunks in reverse with (dy, C, f) it carries dS for the backward.
+//   tc_chunk_fwd   (chunk-parallel; one CTA per (b, c, h, 32-wide slice of P)):
+//        G = C B^T and Z = C S_in^T on the tensor cores (TMA-fed), then each thread owns one
+//        position t: Gamma_{t,k} G_{t,k} -> bf16 tile, Y_intra = (Gamma o G) X on the tensor
+//        cores, and y_t = sum_m f_{t,m} Z[t, (m, p)] + Y_intra + D x_t.
+//
+// All mbarrier waits are bounded (a few seconds); on a timeout the kernel records
+// FRAC_ERR_TIMEOUT in the error word, stops issuing work, frees its tensor memory and exits.
+#include <cuda.h>
+
+#include <algorithm>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "tc.cuh"
+
+namespace frac {
+namespace {
+
+using namespace tc;
+using bf16 = __nv_bfloat16;
+
+constexpr int TQ = 128;   // chunk length on the tensor path
+constexpr int TPS = 32;   // P-slice per CTA
+constexpr int kThreads = 128;
+constexpr int KMAX = 8;          // modes handled by the tensor path (4 or 8)
+constexpr int kTimeoutCode = 4;  // FRAC_ERR_TIMEOUT
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<const uint32_t *>(&v);
+}
+
+__device__ __forceinline__ size_t blh(const ScanDims &d, int b, int t, int h) {
+    return (size_t(b) * d.L + t) * d.H + h;
+}
+
+// Inclusive prefix sum (double) of one value per thread over a 128-thread block.
+__device__ __forceinline__ double block_scan128(double v, double *wsum) {
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    v = warp_inclusive_scan_d(v);
+    if (lane == 31) wsum[w] = v;
+    __syncthreads();
+    double off = 0.0;
+    for (int i = 0; i < w; ++i) off += wsum[i];
+    __syncthreads();
+    return v + off;
+}
+
+struct StateArgs {
+    ScanDims d;
+    const bf16 *U;    // x or dy      [B, L, H, P]
+    const bf16 *W;    // w_write or w_read [B, L, H, K]
+    const float *dt, *alpha, *lam, *tau;
+    const float *init;  // h0 or dh_final [B, H, K, P, N] or null
+    bf16 *emit;         // per-chunk entering states [B, H, nc, K, P, N]
+    float *fin;         // h_final or dh0, or null
+    int *err;
+};
+
+// Shared-memory plan of tc_state_pass (offsets from a 1024-aligned base).
+struct StateSmem {
+    int a_bytes, v_bytes, total;
+    __host__ __device__ StateSmem(int K, int N) {
+        a_bytes = (K / 4) * 2 * 16384;     // K/4 M-tiles x 2 k-atoms x (128 rows x 128 B)
+        v_bytes = (N / 64) * 16384;        // N/64 boxes of [128 t][64 n]
+        total = a_bytes + v_bytes + TQ * TPS * 2 /*x*/ + TQ * KMAX * 4 /*coef*/ +
+                TQ * 8 /*E*/ + TQ * 4 /*e*/ + 64 * 4 /*itau, dec*/ + 64 /*wsum*/ + 64 /*bars*/;
+    }
+};
+
+template <bool REV>
+__global__ void __launch_bounds__(kThreads, 2)
+    tc_state_pass(const __grid_constant__ CUtensorMap mapV, StateArgs a) {
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char *base =
+        reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const ScanDims &d = a.d;
+    const int K = d.K, N = d.N, P = d.P;
+    const StateSmem plan(K, N);
+    unsigned char *sA = base;
+    unsigned char *sV = sA + plan.a_bytes;
+    bf16 *xs = reinterpret_cast<bf16 *>(sV + plan.v_bytes);          // [128][32]
+    float *coef = reinterpret_cast<float *>(xs + TQ * TPS);           // [128][K]
+    double *E_s = reinterpret_cast<double *>(coef + TQ * KMAX);       // [128]
+    float *e_s = reinterpret_cast<float *>(E_s + TQ);                 // [128]
+    float *itau = e_s + TQ;                                           // [32]
+    float *dec = itau + 32;                                           // [32]
+    double *wsum = reinterpret_cast<double *>(dec + 32);              // [4]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);          // tma, mma
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 2);
+    volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
+
+    const int tid = threadIdx.x, w = tid >> 5, j = tid & 31;
+    const int h = blockIdx.y, b = blockIdx.z, p0 = blockIdx.x * TPS;
+    const int g = h / (d.H / d.G);
+    const int mtiles = K / 4;
+    const uint32_t ncols = uint32_t(mtiles * N);  // power of two >= 32 (checked by the host)
+    const size_t PN = size_t(P) * N;
+    const size_t bh = size_t(b) * d.H + h;
+
+    if (tid == 0) {
+        mbar_init(&bars[0], 1);
+        mbar_init(&bars[1], 1);
+        *abort_s = 0;
+        fence_barrier_init();
+    }
+    if (tid < K) itau[tid] = 1.f / a.tau[h * K + tid];
+    if (w == 0) tmem_alloc(tslot, ncols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tslot;
+    const uint32_t lane_base = tmem + (uint32_t(w * 32) << 16);
+    float tmax = 0.f;
+    for (int m = 0; m < K; ++m) tmax = fmaxf(tmax, a.tau[h * K + m]);
+    const float log_cap = logf(64.f * tmax);
+
+    // initial state into tensor memory
+    for (int mt = 0; mt < mtiles; ++mt) {
+        const int m = mt * 4 + w;
+        const float *src = a.init ? a.init + (bh * K + m) * PN + size_t(p0 + j) * N : nullptr;
+        for (int c8 = 0; c8 < N; c8 += 8) {
+            float v[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) v[i] = src ? src[c8 + i] : 0.f;
+            tmem_st8(lane_base + mt * N + c8, v);
+        }
+    }
+    tmem_st_wait();
+
+    int phase = 0;
+    for (int ci = 0; ci < d.nc; ++ci, phase ^= 1) {
+        const int c = REV ? d.nc - 1 - ci : ci;
+        const int c0 = c * TQ, n = min(TQ, d.L - c0);
+        if (ci > 0) {  // previous chunk's MMAs done: tensor memory, sA and sV are free
+            if (!mbar_wait(&bars[1], phase ^ 1)) *abort_s = 1;
+        }
+        __syncthreads();
+        if (*abort_s) break;
+        tc_fence_after();
+        if (tid == 0) {
+            mbar_arrive_expect_tx(&bars[0], uint32_t(N * TQ * 2));
+            for (int jb = 0; jb < N / 64; ++jb)
+                tma_load_3d(sV + jb * 16384, &mapV, &bars[0], g * N + 64 * jb, c0, b);
+        }
+        // chunk inputs: x / dy rows of the P-slice, rates, weights
+        {
+            const int t = tid;
+            float e = 0.f;
+            if (t < n) {
+                const uint4 *src = reinterpret_cast<const uint4 *>(a.U + blh(d, b, c0 + t, h) * P + p0);
+                uint4 *dst = reinterpret_cast<uint4 *>(xs + t * TPS);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) dst[q] = src[q];
+                bool cl;
+                const size_t i = blh(d, b, c0 + t, h);
+                e = token_rate(a.dt[i], a.alpha[i], a.lam[i], log_cap, &cl);
+            } else {
+                uint4 *dst = reinterpret_cast<uint4 *>(xs + t * TPS);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) dst[q] = make_uint4(0, 0, 0, 0);
+            }
+            e_s[t] = e;
+            E_s[t] = block_scan128(double(e), wsum);
+        }
+        __syncthreads();
+        {
+            const int t = tid;
+            const double Eend = E_s[n - 1];
+            for (int m = 0; m < K; ++m) {
+                float cv = 0.f;
+                if (t < n) {
+                    const float wv = to_f(a.W[blh(d, b, c0 + t, h) * K + m]);
+                    if (!REV)
+                        cv = -expm1f(-e_s[t] * itau[m]) * wv * expf(-float(Eend - E_s[t]) * itau[m]);
+                    else
+                        cv = wv * expf(-float(E_s[t]) * itau[m]);
+                }
+                coef[t * K + m] = cv;
+            }
+            if (t < K) dec[t] = expf(-float(Eend) * itau[t]);
+        }
+        __syncthreads();
+        // emit the entering state (bf16) and apply the chunk's decay in place
+        for (int mt = 0; mt < mtiles; ++mt) {
+            const int m = mt * 4 + w;
+            const float dm = dec[m];
+            bf16 *dst = a.emit + ((bh * d.nc + c) * K + m) * PN + size_t(p0 + j) * N;
+            for (int c32 = 0; c32 < N; c32 += 32) {
+                float v[32];
+                tmem_ld32(lane_base + mt * N + c32, v);
+                tmem_ld_wait();
+                uint4 *o = reinterpret_cast<uint4 *>(dst + c32);
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    o[q] = make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                                      pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+#pragma unroll
+                for (int i = 0; i < 32; ++i) v[i] *= dm;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) tmem_st8(lane_base + mt * N + c32 + 8 * q, v + 8 * q);
+            }
+        }
+        tmem_st_wait();
+        // A[(m%4, p), k] = s_{k,m} x_{k,p} (or f dy) as bf16, K-major, 128-byte swizzle
+        for (int mt = 0; mt < mtiles; ++mt) {
+            const int m = mt * 4 + w;
+            const int r = w * 32 + j;
+            for (int ka = 0; ka < 2; ++ka) {
+                unsigned char *tile = sA + (mt * 2 + ka) * 16384;
+#pragma unroll
+                for (int c8 = 0; c8 < 8; ++c8) {
+                    const int k0 = ka * 64 + c8 * 8;
+                    float v[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i)
+                        v[i] = coef[(k0 + i) * K + m] * __bfloat162float(xs[(k0 + i) * TPS + j]);
+                    *reinterpret_cast<uint4 *>(tile + r * 128 + ((c8 ^ (r & 7)) * 16)) =
+                        make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
+                                   pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
+                }
+            }
+        }
+        fence_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+        if (tid == 0) {
+            if (!mbar_wait(&bars[0], phase)) {
+                *abort_s = 1;
+            } else {
+                const uint32_t idesc = idesc_bf16(128, N, false, true);
+                for (int mt = 0; mt < mtiles; ++mt)
+                    for (int ks = 0; ks < TQ / 16; ++ks) {
+                        const uint64_t ad = desc_sw128(smem_u32(sA + (mt * 2 + ks / 4) * 16384) + (ks % 4) * 32, 16, 1024);
+                        const uint64_t bd = desc_sw128(smem_u32(sV) + ks * 2048, 16384, 1024);
+                        mma_bf16(tmem + mt * N, ad, bd, idesc, 1);
+                    }
+                mma_commit(&bars[1]);
+            }
+        }
+    }
+    // drain: last chunk's MMAs
+    __syncthreads();
+    if (!*abort_s && d.nc > 0) {
+        if (!mbar_wait(&bars[1], phase ^ 1)) *abort_s = 1;
+    }
+    __syncthreads();
+    tc_fence_after();
+    if (!*abort_s && a.fin) {
+        for (int mt = 0; mt < mtiles; ++mt) {
+            const int m = mt * 4 + w;
+            float *dst = a.fin + (bh * K + m) * PN + size_t(p0 + j) * N;
+            for (int c32 = 0; c32 < N; c32 += 32) {
+                float v[32];
+                tmem_ld32(lane_base + mt * N + c32, v);
+                tmem_ld_wait();
+                float4 *o = reinterpret_cast<float4 *>(dst + c32);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) o[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            }
+        }
+    }
+    if (*abort_s && tid == 0) atomicExch(a.err, kTimeoutCode);
+    tc_fence_before();
+    __syncthreads();
+    if (w == 0) tmem_dealloc(tmem, ncols);
+}
+
+// ---------------------------------------------------------------------------------------------
+struct OutArgs {
+    ScanDims d;
+    const bf16 *x, *wr, *ww;
+    const float *dt, *alpha, *lam, *tau, *D;
+    bf16 *y;
+    int *err;
+};
+
+struct OutSmem {
+    int c_bytes, b_bytes, s_bytes, total;
+    __host__ __device__ OutSmem(int K, int N) {
+        c_bytes = (N / 64) * 16384;            // C chunk, K-major over n
+        b_bytes = (N / 64) * 16384;            // B chunk
+        s_bytes = (N / 64) * (K * TPS * 128);  // S_in rows (m, p), K-major over n
+        total = c_bytes + b_bytes + s_bytes + 2 * 16384 /*Gamma o G*/ + 2 * 4096 /*X^T*/ +
+                TQ * TPS * 2 /*x*/ + TQ * 32 * 4 /*kappa*/ + TQ * 8 /*E*/ + 32 * 4 + 64 + 64;
+    }
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_chunk_fwd(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapB,
+                 const __grid_constant__ CUtensorMap mapS, OutArgs a) {
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char *base =
+        reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const ScanDims &d = a.d;
+    const int K = d.K, N = d.N, P = d.P;
+    const OutSmem plan(K, N);
+    unsigned char *sC = base;
+    unsigned char *sB = sC + plan.c_bytes;
+    unsigned char *sS = sB + plan.b_bytes;
+    unsigned char *sM = sS + plan.s_bytes;          // Gamma o G, [t][k] K-major, 2 atoms
+    unsigned char *sX = sM + 2 * 16384;             // X^T, [p][k] K-major, 2 atoms of 32 rows
+    bf16 *xs = reinterpret_cast<bf16 *>(sX + 2 * 4096);         // [128][32]
+    float *kap_s = reinterpret_cast<float *>(xs + TQ * TPS);     // [128][32]
+    double *E_s = reinterpret_cast<double *>(kap_s + TQ * 32);   // [128]
+    float *itau = reinterpret_cast<float *>(E_s + TQ);           // [32]
+    double *wsum = reinterpret_cast<double *>(itau + 32);        // [4] (+pad)
+    uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);     // tma, mma1, mma2
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 3);
+    volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
+
+    const int tid = threadIdx.x, w = tid >> 5;
+    const int npart = P / TPS;
+    const int h = blockIdx.x / npart, p0 = (blockIdx.x % npart) * TPS;
+    const int c = blockIdx.y, b = blockIdx.z;
+    const int g = h / (d.H / d.G);
+    const int c0 = c * TQ, n = min(TQ, d.L - c0);
+    const int t = tid;
+    const uint32_t ZN = uint32_t(K * TPS);  // Z columns: (m, p)
+
+    if (tid == 0) {
+        for (int i = 0; i < 3; ++i) mbar_init(&bars[i], 1);
+        *abort_s = 0;
+        fence_barrier_init();
+    }
+    if (tid < K) itau[tid] = 1.f / a.tau[h * K + tid];
+    if (w == 0) tmem_alloc(tslot, 512);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tslot;
+    const uint32_t lane_base = tmem + (uint32_t(w * 32) << 16);
+    const uint32_t colG = 0, colZ = 128, colY = 128 + ZN;
+
+    if (tid == 0) {
+        const uint32_t bytes = uint32_t(plan.c_bytes + plan.b_bytes + plan.s_bytes);
+        mbar_arrive_expect_tx(&bars[0], bytes);
+        for (int jb = 0; jb < N / 64; ++jb) {
+            tma_load_3d(sC + jb * 16384, &mapC, &bars[0], g * N + 64 * jb, c0, b);
+            tma_load_3d(sB + jb * 16384, &mapB, &bars[0], g * N + 64 * jb, c0, b);
+            tma_load_3d(sS + jb * (K * TPS * 128), &mapS, &bars[0], 64 * jb, p0,
+                        int(((size_t(b) * d.H + h) * d.nc + c) * K));
+        }
+    }
+    // per-position data of row t
+    float tmax = 0.f;
+    for (int m = 0; m < K; ++m) tmax = fmaxf(tmax, a.tau[h * K + m]);
+    const float log_cap = logf(64.f * tmax);
+    float e = 0.f;
+    float wr_t[KMAX], f_t[KMAX];
+    if (t < n) {
+        const size_t i = blh(d, b, c0 + t, h);
+        bool cl;
+        e = token_rate(a.dt[i], a.alpha[i], a.lam[i], log_cap, &cl);
+        const uint4 *src = reinterpret_cast<const uint4 *>(a.x + i * P + p0);
+        uint4 *dst = reinterpret_cast<uint4 *>(xs + t * TPS);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) dst[q] = src[q];
+    } else {
+        uint4 *dst = reinterpret_cast<uint4 *>(xs + t * TPS);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) dst[q] = make_uint4(0, 0, 0, 0);
+    }
+    const double Et = block_scan128(double(e), wsum);
+    E_s[t] = Et;
+#pragma unroll
+    for (int m = 0; m < KMAX; ++m) {
+        wr_t[m] = 0.f;
+        f_t[m] = 0.f;
+        if (m < K) {
+            float kp = 0.f;
+            if (t < n) {
+                const size_t wi = blh(d, b, c0 + t, h) * K + m;
+                wr_t[m] = to_f(a.wr[wi]);
+                kp = -expm1f(-e * itau[m]) * to_f(a.ww[wi]);
+                f_t[m] = wr_t[m] * expf(-float(Et) * itau[m]);
+            }
+            kap_s[t * 32 + m] = kp;
+        }
+    }
+    __syncthreads();
+    // X^T tile: row p, column k = t (K-major, 128-byte swizzle, 32 rows per k-atom)
+    {
+        unsigned char *tile = sX + (t >> 6) * 4096;
+        const int kk = t & 63;
+#pragma unroll
+        for (int p = 0; p < TPS; ++p)
+            *reinterpret_cast<bf16 *>(tile + sw128_offset(p, kk)) = xs[t * TPS + p];
+    }
+    fence_async_smem();
+    __syncthreads();
+    // G = C B^T and Z = C S_in^T
+    if (tid == 0) {
+        if (!mbar_wait(&bars[0], 0)) {
+            *abort_s = 1;
+        } else {
+            tc_fence_after();
+            const uint32_t idG = idesc_bf16(128, 128, false, false);
+            const uint32_t idZ = idesc_bf16(128, int(ZN), false, false);
+            for (int ks = 0; ks < N / 16; ++ks) {
+                const uint32_t koff = (ks / 4) * 16384 + (ks % 4) * 32;
+                const uint64_t ad = desc_sw128(smem_u32(sC) + koff, 16, 1024);
+                const uint64_t bdB = desc_sw128(smem_u32(sB) + koff, 16, 1024);
+                const uint64_t bdS =
+                    desc_sw128(smem_u32(sS) + (ks / 4) * (K * TPS * 128) + (ks % 4) * 32, 16, 1024);
+                mma_bf16(tmem + colG, ad, bdB, idG, ks > 0);
+                mma_bf16(tmem + colZ, ad, bdS, idZ, ks > 0);
+            }
+            mma_commit(&bars[1]);
+        }
+    }
+    __syncthreads();
+    if (!*abort_s && !mbar_wait(&bars[1], 0)) *abort_s = 1;
+    __syncthreads();
+    tc_fence_after();
+    if (!*abort_s) {
+        // row t of Gamma o G -> bf16, K-major [t][k]
+        for (int k32 = 0; k32 < TQ; k32 += 32) {
+            float gv[32];
+            tmem_ld32(lane_base + colG + k32, gv);
+            tmem_ld_wait();
+#pragma unroll
+            for (int kk = 0; kk < 32; ++kk) {
+                const int k = k32 + kk;
+                float v = 0.f;
+                if (k <= t && t < n) {
+                    const float dE = float(Et - E_s[k]);
+                    float gam = 0.f;
+#pragma unroll
+                    for (int m = 0; m < KMAX; ++m)
+                        if (m < K) gam = fmaf(wr_t[m] * kap_s[k * 32 + m], expf(-dE * itau[m]), gam);
+                    v = gam * gv[kk];
+                }
+                gv[kk] = v;
+            }
+            unsigned char *tile = sM + (k32 >> 6) * 16384;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int c8 = ((k32 & 63) >> 3) + q;
+                *reinterpret_cast<uint4 *>(tile + t * 128 + ((c8 ^ (t & 7)) * 16)) =
+                    make_uint4(pack_bf16x2(gv[8 * q], gv[8 * q + 1]), pack_bf16x2(gv[8 * q + 2], gv[8 * q + 3]),
+                               pack_bf16x2(gv[8 * q + 4], gv[8 * q + 5]), pack_bf16x2(gv[8 * q + 6], gv[8 * q + 7]));
+            }
+        }
+    }
+    fence_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (tid == 0 && !*abort_s) {
+        const uint32_t idY = idesc_bf16(128, TPS, false, false);
+        for (int ks = 0; ks < TQ / 16; ++ks) {
+            const uint64_t ad = desc_sw128(smem_u32(sM) + (ks / 4) * 16384 + (ks % 4) * 32, 16, 1024);
+            const uint64_t bd = desc_sw128(smem_u32(sX) + (ks / 4) * 4096 + (ks % 4) * 32, 16, 1024);
+            mma_bf16(tmem + colY, ad, bd, idY, ks > 0);
+        }
+        mma_commit(&bars[2]);
+    }
+    __syncthreads();
+    if (!*abort_s && !mbar_wait(&bars[2], 0)) *abort_s = 1;
+    __syncthreads();
+    tc_fence_after();
+    if (!*abort_s) {
+        float acc[32];
+        tmem_ld32(lane_base + colY, acc);
+        tmem_ld_wait();
+#pragma unroll
+        for (int m = 0; m < KMAX; ++m) {
+            if (m >= K) break;
+            float z[32];
+            tmem_ld32(lane_base + colZ + m * TPS, z);
+            tmem_ld_wait();
+            const float fm = f_t[m];
+#pragma unroll
+            for (int p = 0; p < 32; ++p) acc[p] = fmaf(fm, z[p], acc[p]);
+        }
+        if (t < n) {
+            const float Dh = a.D[h];
+            uint4 *o = reinterpret_cast<uint4 *>(a.y + blh(d, b, c0 + t, h) * P + p0);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                float v[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) v[i] = acc[8 * q + i] + Dh * __bfloat162float(xs[t * TPS + 8 * q + i]);
+                o[q] = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]),
+                                  pack_bf16x2(v[6], v[7]));
+            }
+        }
+    }
+    if (*abort_s && tid == 0) atomicExch(a.err, kTimeoutCode);
+    tc_fence_before();
+    __syncthreads();
+    if (w == 0) tmem_dealloc(tmem, 512);
+}
+
+// ------------------------------------------------------------------------------------- host
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    return fn;
+}
+
+// 3-D bf16 tensor map, innermost dimension first; 128-byte swizzle.
+bool make_map3(CUtensorMap *m, const void *ptr, uint64_t d0, uint64_t d1, uint64_t d2,
+               uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1,
+               uint32_t b2) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[3] = {d0, d1, d2};
+    const cuuint64_t strides[2] = {stride1_bytes, stride2_bytes};
+    const cuuint32_t box[3] = {b0, b1, b2};
+    const cuuint32_t es[3] = {1, 1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), dims, strides, box,
+              es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+bool tc_supported(const ScanDims &d, int dtype) {
+    if (dtype != 1) return false;
+    if (d.P % TPS || (d.N != 64 && d.N != 128) || (d.K != 4 && d.K != 8)) return false;
+    return true;
+}
+
+size_t tc_state_elems(const ScanDims &d) {
+    return size_t(d.B) * d.H * d.nc * d.K * d.P * d.N;
+}
+
+cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, const void *V,
+                                 const void *W, const float *dt, const float *alpha,
+                                 const float *lam, const float *tau, const float *init,
+                                 void *emit, float *fin, int *err, cudaStream_t st) {
+    CUtensorMap mapV;
+    if (!make_map3(&mapV, V, uint64_t(d.G) * d.N, d.L, d.B, uint64_t(d.G) * d.N * 2,
+                   uint64_t(d.L) * d.G * d.N * 2, 64, TQ, 1))
+        return cudaErrorInvalidValue;
+    StateArgs a;
+    a.d = d;
+    a.U = (const bf16 *)U;
+    a.W = (const bf16 *)W;
+    a.dt = dt; a.alpha = alpha; a.lam = lam; a.tau = tau;
+    a.init = init;
+    a.emit = (bf16 *)emit;
+    a.fin = fin;
+    a.err = err;
+    const size_t smem = StateSmem(d.K, d.N).total + 1024;
+    dim3 grid(d.P / TPS, d.H, d.B);
+    if (rev) {
+        auto k = tc_state_pass<true>;
+        cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+        trace_begin("state_pass_rev_tc", st);
+        k<<<grid, kThreads, smem, st>>>(mapV, a);
+        trace_end(st);
+    } else {
+        auto k = tc_state_pass<false>;
+        cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+        trace_begin("state_pass_fwd_tc", st);
+        k<<<grid, kThreads, smem, st>>>(mapV, a);
+        trace_end(st);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, int *err,
+                        cudaStream_t st) {
+    cudaError_t e = tc_state_pass_launch(d, false, p.x, p.Bm, p.ww, p.dt, p.alpha, p.lam, p.tau,
+                                         p.h0, S_in, p.h_final, err, st);
+    if (e != cudaSuccess || d.nc == 0) return e;
+    CUtensorMap mapC, mapB, mapS;
+    const uint64_t GN = uint64_t(d.G) * d.N;
+    if (!make_map3(&mapC, p.Cm, GN, d.L, d.B, GN * 2, uint64_t(d.L) * GN * 2, 64, TQ, 1) ||
+        !make_map3(&mapB, p.Bm, GN, d.L, d.B, GN * 2, uint64_t(d.L) * GN * 2, 64, TQ, 1) ||
+        !make_map3(&mapS, S_in, d.N, d.P, uint64_t(d.B) * d.H * d.nc * d.K, uint64_t(d.N) * 2,
+                   uint64_t(d.P) * d.N * 2, 64, TPS, d.K))
+        return cudaErrorInvalidValue;
+    OutArgs a;
+    a.d = d;
+    a.x = (const bf16 *)p.x;
+    a.wr = (const bf16 *)p.wr;
+    a.ww = (const bf16 *)p.ww;
+    a.dt = p.dt; a.alpha = p.alpha; a.lam = p.lam; a.tau = p.tau; a.D = p.D;
+    a.y = (bf16 *)p.y;
+    a.err = err;
+    const size_t smem = OutSmem(d.K, d.N).total + 1024;
+    cudaFuncSetAttribute(tc_chunk_fwd, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    dim3 grid(d.H * (d.P / TPS), d.nc, d.B);
+    trace_begin("chunk_fwd_tc", st);
+    tc_chunk_fwd<<<grid, kThreads, smem, st>>>(mapC, mapB, mapS, a);
+    trace_end(st);
+    return cudaGetLastError();
+}
+
+}  // namespace frac
