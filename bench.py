@@ -142,10 +142,18 @@ def algorithmic_work(kernel: str, s, per_launch_units: float):
     the design notes): state contractions count 2 K P N flops per token-head each."""
     per_th = {
         "state_pass_fwd_simt": 2, "state_pass_rev_simt": 2, "chunk_fwd_simt": 2,
-        "chunk_bwd_simt": 8,
+        "chunk_bwd_simt": 8, "state_pass_fwd_tc": 2, "state_pass_rev_tc": 2,
+        "bwd_inter_tc": 4, "bwd_dcdb_tc": 4,
     }
     if kernel in per_th:
         return "flops", per_th[kernel] * kpn(s) * per_launch_units
+    # kernels with the intra-chunk terms: the readout (2 K P N) plus the causal intra-chunk
+    # products (Q P per token-head, and Q N per token for the C B^T shared by the heads of a group)
+    q = 128
+    if kernel == "chunk_fwd_tc":
+        return "flops", (2 * kpn(s) + q * s.headdim + q * s.dstate * s.ngroups / s.nheads) * per_launch_units
+    if kernel == "bwd_intra_tc":
+        return "flops", (2 * q * s.headdim + q * s.dstate * s.ngroups / s.nheads) * per_launch_units
     if kernel == "decode_step":
         return "bytes", 2.0 * 4 * kpn(s) * per_launch_units
     return None, None
@@ -307,7 +315,14 @@ def main():
     if dom:
         kind, work = algorithmic_work(dom, s, s.batch * s.seqlen * s.nheads)
         avg_s = kern[dom]["avg_ms"] / 1e3
-        if kind == "flops":
+        if kind == "flops" and dom.endswith("_tc"):
+            # tensor-core kernel timed inside a long step: sustained bf16 peak
+            peak = peaks.get("bf16_tflops_sustained", peaks.get("bf16_tflops"))
+            ach = work / avg_s / 1e12
+            roofline = {"kernel": dom, "bound": "tensor", "achieved": ach, "peak": peak,
+                        "unit": "TFLOP/s", "frac": ach / peak, "traffic": None,
+                        "peak_source": peaks["source"] + " (bf16, sustained)"}
+        elif kind == "flops":
             # CUDA-core float32 FMA peak: SMs x 128 lanes x 2 flops x max SM clock
             peak = NUM_SMS * 128 * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
             ach = work / avg_s / 1e12
@@ -363,10 +378,13 @@ def main():
             "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": "f32", "data": "synthetic",
+            "dtype": "bf16" if any(k.endswith("_tc") for k in trace) else "f32",
+            "data": "synthetic",
             "config": {"workload": f"{TRAIN}: forward + backward of the chunked scan, B{s.batch} "
                                    f"L{s.seqlen} H{s.nheads} P{s.headdim} N{s.dstate} "
-                                   f"K{s.nmodes} G{s.ngroups}, bf16 inputs, float32 arithmetic",
+                                   f"K{s.nmodes} G{s.ngroups}, bf16 inputs; tensor-core products "
+                                   "take bf16 operands with float32 accumulation, the rest is "
+                                   "float32",
                        "global_batch": s.batch * world, "seq_len": s.seqlen,
                        "parallelism": f"replicas{world}" if world > 1 else "single",
                        "l2": "inputs larger than L2 (0.78 GB per step), no flush"},

@@ -73,6 +73,7 @@ size_t elem(const frac_dims *d) { return d->dtype == FRAC_DTYPE_BF16 ? 2 : 4; }
 enum Path { PATH_SIMT = 0, PATH_TC = 1 };
 
 frac_status plan(const frac_dims *d, frac::ScanDims *sd, int *path, bool backward) {
+    // (the backward runs on the tensor cores when headdim is 64 as well)
     sd->B = int(d->batch);
     sd->L = int(d->seqlen);
     sd->H = int(d->nheads);
@@ -80,8 +81,10 @@ frac_status plan(const frac_dims *d, frac::ScanDims *sd, int *path, bool backwar
     sd->G = int(d->ngroups);
     sd->N = int(d->dstate);
     sd->K = int(d->nmodes);
-    const bool tc = !backward && !(d->flags & FRAC_FLAG_FORCE_SIMT) &&
-                    frac::tc_supported(*sd, d->dtype) && (d->chunk == 0 || d->chunk == 128);
+    const bool tc = !(d->flags & FRAC_FLAG_FORCE_SIMT) &&
+                    (backward ? frac::tc_bwd_supported(*sd, d->dtype)
+                              : frac::tc_supported(*sd, d->dtype)) &&
+                    (d->chunk == 0 || d->chunk == 128);
     if (tc) {
         sd->Q = 128;
         *path = PATH_TC;
@@ -119,8 +122,14 @@ FwdLayout fwd_layout(const frac_dims *d, const frac::ScanDims &sd, int path) {
     return l;
 }
 
-BwdLayout bwd_layout(const frac_dims *d, const frac::ScanDims &sd) {
+BwdLayout bwd_layout(const frac_dims *d, const frac::ScanDims &sd, int path) {
     BwdLayout l;
+    if (path == PATH_TC) {
+        frac::TcBwdWorkspace t;
+        l.s_in = l.ds_out = l.db = l.dc = 0;
+        l.total = kStatusBytes + frac::tc_bwd_workspace_bytes(sd, &t, nullptr);
+        return l;
+    }
     const size_t st = round_up(frac::simt_state_elems(sd) * elem(d));
     const size_t ngn = size_t(sd.B) * sd.L * sd.G * sd.N;
     l.s_in = kStatusBytes;
@@ -186,7 +195,7 @@ frac_status frac_scan_bwd_workspace_size(const frac_dims *d, size_t *bytes) {
     frac::ScanDims sd;
     int path;
     if ((s = plan(d, &sd, &path, true))) return s;
-    *bytes = bwd_layout(d, sd).total;
+    *bytes = bwd_layout(d, sd, path).total;
     return FRAC_OK;
 }
 
@@ -277,7 +286,18 @@ frac_status frac_scan_bwd(const frac_dims *d, const void *x, const float *dt, co
     frac::ScanDims sd;
     int path;
     if ((s = plan(d, &sd, &path, true))) return s;
-    const BwdLayout l = bwd_layout(d, sd);
+    const BwdLayout l = bwd_layout(d, sd, path);
+    if (path == PATH_TC && d->seqlen > 0) {
+        const void *need16[] = {x, Bm, Cm, dy, dx, dB, dC, dw_read, dw_write};
+        for (const void *q : need16)
+            if (!aligned_to(q, 16))
+                return fail(FRAC_ERR_INVALID_ARGUMENT,
+                            "the tensor-core backward needs x, Bm, Cm, dy, dx, dB, dC, dw_read and "
+                            "dw_write 16-byte aligned (or set FRAC_FLAG_FORCE_SIMT)");
+        if ((h0 && !aligned_to(h0, 16)) || (dh_final && !aligned_to(dh_final, 16)) ||
+            (dh0 && !aligned_to(dh0, 16)))
+            return fail(FRAC_ERR_INVALID_ARGUMENT, "state tensors must be 16-byte aligned");
+    }
     {
         if (!workspace) return fail(FRAC_ERR_INVALID_ARGUMENT, "workspace must not be NULL");
         if (reinterpret_cast<uintptr_t>(workspace) % kAlign)
@@ -299,8 +319,15 @@ frac_status frac_scan_bwd(const frac_dims *d, const void *x, const float *dt, co
                                                 : static_cast<float *>(dC);
     cudaStream_t st = (cudaStream_t)stream;
     cudaError_t e = cudaMemsetAsync(ws, 0, sizeof(int), st);
-    if (e == cudaSuccess)
-        e = frac::simt_scan_bwd(sd, d->dtype, p, ws + l.s_in, ws + l.ds_out, dB_acc, dC_acc, st);
+    if (e == cudaSuccess) {
+        if (path == PATH_TC) {
+            frac::TcBwdWorkspace t;
+            frac::tc_bwd_workspace_bytes(sd, &t, ws + kStatusBytes);
+            e = frac::tc_scan_bwd(sd, p, t, reinterpret_cast<int *>(ws), st);
+        } else {
+            e = frac::simt_scan_bwd(sd, d->dtype, p, ws + l.s_in, ws + l.ds_out, dB_acc, dC_acc, st);
+        }
+    }
     return cuda_status(e, "frac_scan_bwd");
 }
 

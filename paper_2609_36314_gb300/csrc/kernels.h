@@ -1,6 +1,7 @@
 // Internal interface between the C-ABI layer and the kernels (not installed).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -51,6 +52,27 @@ cudaError_t simt_scan_bwd(const ScanDims &d, int dtype, const ScanPtrs &p, void 
 bool tc_supported(const ScanDims &d, int dtype);
 size_t tc_state_elems(const ScanDims &d);  // bf16 elements of the per-chunk state workspace
 cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, int *err,
+                        cudaStream_t st);
+// Chunk-serial state pass on the tensor cores (forward: U = x, V = B, W = w_write; reverse:
+// U = dy, V = C, W = w_read, optionally accumulating <dS_out, S_in> per chunk and mode).
+cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, const void *V,
+                                 const void *W, const float *dt, const float *alpha,
+                                 const float *lam, const float *tau, const float *init,
+                                 void *emit, float *fin, const void *dot_src, float *dot_out,
+                                 int *err, cudaStream_t st);
+bool tc_make_map3(CUtensorMap *m, const void *ptr, uint64_t d0, uint64_t d1, uint64_t d2,
+                  uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1,
+                  uint32_t b2);
+// Tensor-core backward (headdim 64 in addition to the forward's conditions).
+bool tc_bwd_supported(const ScanDims &d, int dtype);
+struct TcBwdWorkspace {
+    void *S_in, *dS_out;                     // bf16 per-chunk states
+    float *dx_acc, *dwr_acc, *dkap_acc;      // [B,L,H,P], [B,L,H,K] x 2
+    float *ab_acc, *rect, *cdot, *mh_total;  // [B,L,H,2], [B,L,H], [B,H,nc,K], [B,nc,Q,Q]
+    float *dB_acc, *dC_acc;                  // [B,L,G,N] x 2
+};
+size_t tc_bwd_workspace_bytes(const ScanDims &d, TcBwdWorkspace *layout, char *base);
+cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspace &ws, int *err,
                         cudaStream_t st);
 
 }  // namespace frac

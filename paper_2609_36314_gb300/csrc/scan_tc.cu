@@ -24,6 +24,7 @@
 #include "common.cuh"
 #include "kernels.h"
 #include "tc.cuh"
+#include "tc_util.cuh"
 
 namespace frac {
 namespace {
@@ -31,32 +32,7 @@ namespace {
 using namespace tc;
 using bf16 = __nv_bfloat16;
 
-constexpr int TQ = 128;   // chunk length on the tensor path
-constexpr int TPS = 32;   // P-slice per CTA
 constexpr int kThreads = 128;
-constexpr int KMAX = 8;          // modes handled by the tensor path (4 or 8)
-constexpr int kTimeoutCode = 4;  // FRAC_ERR_TIMEOUT
-
-__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
-    const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
-    return *reinterpret_cast<const uint32_t *>(&v);
-}
-
-__device__ __forceinline__ size_t blh(const ScanDims &d, int b, int t, int h) {
-    return (size_t(b) * d.L + t) * d.H + h;
-}
-
-// Inclusive prefix sum (double) of one value per thread over a 128-thread block.
-__device__ __forceinline__ double block_scan128(double v, double *wsum) {
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    v = warp_inclusive_scan_d(v);
-    if (lane == 31) wsum[w] = v;
-    __syncthreads();
-    double off = 0.0;
-    for (int i = 0; i < w; ++i) off += wsum[i];
-    __syncthreads();
-    return v + off;
-}
 
 struct StateArgs {
     ScanDims d;
@@ -66,6 +42,8 @@ struct StateArgs {
     const float *init;  // h0 or dh_final [B, H, K, P, N] or null
     bf16 *emit;         // per-chunk entering states [B, H, nc, K, P, N]
     float *fin;         // h_final or dh0, or null
+    const bf16 *dot_src;  // reverse pass only: S_in of every chunk (same layout as emit), or null
+    float *dot_out;       // reverse pass only: <emitted dS, S_in> per (b, h, chunk, mode) [B,H,nc,K]
     int *err;
 };
 
@@ -197,11 +175,27 @@ __global__ void __launch_bounds__(kThreads, 2)
         for (int mt = 0; mt < mtiles; ++mt) {
             const int m = mt * 4 + w;
             const float dm = dec[m];
-            bf16 *dst = a.emit + ((bh * d.nc + c) * K + m) * PN + size_t(p0 + j) * N;
+            const size_t row = ((bh * d.nc + c) * K + m) * PN + size_t(p0 + j) * N;
+            bf16 *dst = a.emit + row;
+            float dsum = 0.f;
             for (int c32 = 0; c32 < N; c32 += 32) {
                 float v[32];
                 tmem_ld32(lane_base + mt * N + c32, v);
                 tmem_ld_wait();
+                if (REV && a.dot_out) {
+                    const uint4 *sp = reinterpret_cast<const uint4 *>(a.dot_src + row + c32);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const uint4 u4 = sp[q];
+                        const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&u4);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            const float2 f2 = __bfloat1622float2(h2[i]);
+                            dsum = fmaf(v[8 * q + 2 * i], f2.x, dsum);
+                            dsum = fmaf(v[8 * q + 2 * i + 1], f2.y, dsum);
+                        }
+                    }
+                }
                 uint4 *o = reinterpret_cast<uint4 *>(dst + c32);
 #pragma unroll
                 for (int q = 0; q < 4; ++q)
@@ -211,6 +205,10 @@ __global__ void __launch_bounds__(kThreads, 2)
                 for (int i = 0; i < 32; ++i) v[i] *= dm;
 #pragma unroll
                 for (int q = 0; q < 4; ++q) tmem_st8(lane_base + mt * N + c32 + 8 * q, v + 8 * q);
+            }
+            if (REV && a.dot_out) {
+                dsum = warp_sum(dsum);  // the 32 lanes of warp w are the 32 p of mode m
+                if (j == 0) atomicAdd(a.dot_out + (bh * d.nc + c) * K + m, dsum);
             }
         }
         tmem_st_wait();
@@ -525,8 +523,10 @@ EncodeTiledFn encode_fn() {
     return fn;
 }
 
+}  // namespace
+
 // 3-D bf16 tensor map, innermost dimension first; 128-byte swizzle.
-bool make_map3(CUtensorMap *m, const void *ptr, uint64_t d0, uint64_t d1, uint64_t d2,
+bool tc_make_map3(CUtensorMap *m, const void *ptr, uint64_t d0, uint64_t d1, uint64_t d2,
                uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1,
                uint32_t b2) {
     EncodeTiledFn fn = encode_fn();
@@ -539,8 +539,6 @@ bool make_map3(CUtensorMap *m, const void *ptr, uint64_t d0, uint64_t d1, uint64
               es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
-
-}  // namespace
 
 bool tc_supported(const ScanDims &d, int dtype) {
     if (dtype != 1) return false;
@@ -555,9 +553,10 @@ size_t tc_state_elems(const ScanDims &d) {
 cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, const void *V,
                                  const void *W, const float *dt, const float *alpha,
                                  const float *lam, const float *tau, const float *init,
-                                 void *emit, float *fin, int *err, cudaStream_t st) {
+                                 void *emit, float *fin, const void *dot_src, float *dot_out,
+                                 int *err, cudaStream_t st) {
     CUtensorMap mapV;
-    if (!make_map3(&mapV, V, uint64_t(d.G) * d.N, d.L, d.B, uint64_t(d.G) * d.N * 2,
+    if (!tc_make_map3(&mapV, V, uint64_t(d.G) * d.N, d.L, d.B, uint64_t(d.G) * d.N * 2,
                    uint64_t(d.L) * d.G * d.N * 2, 64, TQ, 1))
         return cudaErrorInvalidValue;
     StateArgs a;
@@ -568,6 +567,8 @@ cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, con
     a.init = init;
     a.emit = (bf16 *)emit;
     a.fin = fin;
+    a.dot_src = (const bf16 *)dot_src;
+    a.dot_out = dot_out;
     a.err = err;
     const size_t smem = StateSmem(d.K, d.N).total + 1024;
     dim3 grid(d.P / TPS, d.H, d.B);
@@ -590,13 +591,13 @@ cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, con
 cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, int *err,
                         cudaStream_t st) {
     cudaError_t e = tc_state_pass_launch(d, false, p.x, p.Bm, p.ww, p.dt, p.alpha, p.lam, p.tau,
-                                         p.h0, S_in, p.h_final, err, st);
+                                         p.h0, S_in, p.h_final, nullptr, nullptr, err, st);
     if (e != cudaSuccess || d.nc == 0) return e;
     CUtensorMap mapC, mapB, mapS;
     const uint64_t GN = uint64_t(d.G) * d.N;
-    if (!make_map3(&mapC, p.Cm, GN, d.L, d.B, GN * 2, uint64_t(d.L) * GN * 2, 64, TQ, 1) ||
-        !make_map3(&mapB, p.Bm, GN, d.L, d.B, GN * 2, uint64_t(d.L) * GN * 2, 64, TQ, 1) ||
-        !make_map3(&mapS, S_in, d.N, d.P, uint64_t(d.B) * d.H * d.nc * d.K, uint64_t(d.N) * 2,
+    if (!tc_make_map3(&mapC, p.Cm, GN, d.L, d.B, GN * 2, uint64_t(d.L) * GN * 2, 64, TQ, 1) ||
+        !tc_make_map3(&mapB, p.Bm, GN, d.L, d.B, GN * 2, uint64_t(d.L) * GN * 2, 64, TQ, 1) ||
+        !tc_make_map3(&mapS, S_in, d.N, d.P, uint64_t(d.B) * d.H * d.nc * d.K, uint64_t(d.N) * 2,
                    uint64_t(d.P) * d.N * 2, 64, TPS, d.K))
         return cudaErrorInvalidValue;
     OutArgs a;

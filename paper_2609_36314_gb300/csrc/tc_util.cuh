@@ -1,0 +1,38 @@
+// Small device helpers shared by the tensor-core kernels.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace frac {
+
+constexpr int TQ = 128;          // chunk length on the tensor path
+constexpr int TPS = 32;          // P-slice of the state pass / output kernels
+constexpr int KMAX = 8;          // modes handled by the tensor path (4 or 8)
+constexpr int kTimeoutCode = 4;  // FRAC_ERR_TIMEOUT
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<const uint32_t *>(&v);
+}
+
+__device__ __forceinline__ size_t blh(const ScanDims &d, int b, int t, int h) {
+    return (size_t(b) * d.L + t) * d.H + h;
+}
+
+// Inclusive prefix sum (double) of one value per thread over a 128-thread block.
+__device__ __forceinline__ double block_scan128(double v, double *wsum) {
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    v = warp_inclusive_scan_d(v);
+    if (lane == 31) wsum[w] = v;
+    __syncthreads();
+    double off = 0.0;
+    for (int i = 0; i < w; ++i) off += wsum[i];
+    __syncthreads();
+    return v + off;
+}
+
+}  // namespace frac

@@ -206,3 +206,35 @@ def test_long_prefill_workload_sampled():
     yr, hfr = _ora_fwd(sub)
     assert_close("y", to_host64(y[:, :, heads]), yr, 1e-2)
     assert_close("h_final", to_host64(hf[:, heads]), hfr, 1e-2)
+
+
+def test_bwd_tensor_core_path_matches_cuda_core_path():
+    """bf16, P = 64: the default (tensor-core) backward and the CUDA-core backward against the
+    oracle, with h0 and dh_final, a ragged last chunk and several chunks."""
+    s = synth.Shape(2, 300, 4, 64, 1, 128, 8, 0, "bf16")
+    host = synth.make_scan_inputs(s, seed=21, with_dy=True, with_h0=True, with_dh_final=True)
+    dv = dev_inputs(host)
+    g_tc = _gpu_bwd(dv)
+    g_simt = _gpu_bwd(dv, force_simt=True)
+    torch.cuda.synchronize()
+    gr = _ora_bwd(f64_inputs(host))
+    for k in GRADS:
+        assert_close(k + " (tensor cores)", to_host64(g_tc[k]), gr[k], 1e-2)
+        assert_close(k + " (CUDA cores)", to_host64(g_simt[k]), gr[k], 1e-2)
+
+
+def test_bwd_bf16_paper_like_lambda_alpha_extremes():
+    """Small alpha and large lambda make e = Delta lambda^(1/alpha) huge (clamped) on some
+    positions; the decay gradient must stay accurate there (per-position decayed terms)."""
+    s = synth.Shape(1, 256, 4, 64, 1, 64, 8, 0, "bf16")
+    host = synth.make_scan_inputs(s, seed=33, with_dy=True)
+    host["alpha"] = (host["alpha"] * 0.25).astype(np.float32)   # alpha in (0, 0.25)
+    host["lam"] = np.full_like(host["lam"], 3.5)
+    host["w_read"] = synth.cast(synth.mode_weights(host["alpha"], host["tau"], synth.normal(33, "w_read", (1, 256, 4, 8))), "bf16")
+    host["w_write"] = synth.cast(synth.mode_weights(host["alpha"], host["tau"], synth.normal(33, "w_write", (1, 256, 4, 8))), "bf16")
+    dv = dev_inputs(host)
+    g = _gpu_bwd(dv)
+    torch.cuda.synchronize()
+    gr = _ora_bwd(f64_inputs(host))
+    for k in GRADS:
+        assert_close(k, to_host64(g[k]), gr[k], 1e-2)
