@@ -293,11 +293,13 @@ struct OutSmem {
         b_bytes = (N / 64) * 16384;            // B chunk
         s_bytes = (N / 64) * (K * TPS * 128);  // S_in rows (m, p), K-major over n
         total = c_bytes + b_bytes + s_bytes + 2 * 16384 /*Gamma o G*/ + 2 * 4096 /*X^T*/ +
-                TQ * TPS * 2 /*x*/ + TQ * 32 * 4 /*kappa*/ + TQ * 8 /*E*/ + 32 * 4 + 64 + 64;
+                TQ * TPS * 2 /*x*/ + TQ * 32 * 4 /*kappa*/ + TQ * 8 /*E*/ + 32 * 4 + 64 + 64 + 64;
     }
 };
 
-__global__ void __launch_bounds__(kThreads, 1)
+constexpr int kOutThreads = 256;  // two groups of four warps share the 128 TMEM lanes
+
+__global__ void __launch_bounds__(kOutThreads, 1)
     tc_chunk_fwd(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapB,
                  const __grid_constant__ CUtensorMap mapS, OutArgs a) {
     extern __shared__ unsigned char smem_raw[];
@@ -312,21 +314,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     unsigned char *sM = sS + plan.s_bytes;          // Gamma o G, [t][k] K-major, 2 atoms
     unsigned char *sX = sM + 2 * 16384;             // X^T, [p][k] K-major, 2 atoms of 32 rows
     bf16 *xs = reinterpret_cast<bf16 *>(sX + 2 * 4096);         // [128][32]
-    float *kap_s = reinterpret_cast<float *>(xs + TQ * TPS);     // [128][32]
+    float *kap_s = reinterpret_cast<float *>(xs + TQ * TPS);     // [128][32]; later partial y
     double *E_s = reinterpret_cast<double *>(kap_s + TQ * 32);   // [128]
-    float *itau = reinterpret_cast<float *>(E_s + TQ);           // [32]
-    double *wsum = reinterpret_cast<double *>(itau + 32);        // [4] (+pad)
+    float *l2t = reinterpret_cast<float *>(E_s + TQ);            // [32] log2(e) / tau
+    double *wsum = reinterpret_cast<double *>(l2t + 32);         // [8]
     uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);     // tma, mma1, mma2
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 3);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
 
-    const int tid = threadIdx.x, w = tid >> 5;
+    const int tid = threadIdx.x, grp = tid >> 7, t = tid & 127, w4 = (tid >> 5) & 3;
     const int npart = P / TPS;
     const int h = blockIdx.x / npart, p0 = (blockIdx.x % npart) * TPS;
     const int c = blockIdx.y, b = blockIdx.z;
     const int g = h / (d.H / d.G);
     const int c0 = c * TQ, n = min(TQ, d.L - c0);
-    const int t = tid;
     const uint32_t ZN = uint32_t(K * TPS);  // Z columns: (m, p)
 
     if (tid == 0) {
@@ -334,13 +335,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         *abort_s = 0;
         fence_barrier_init();
     }
-    if (tid < K) itau[tid] = 1.f / a.tau[h * K + tid];
-    if (w == 0) tmem_alloc(tslot, 512);
+    if (tid < K) l2t[tid] = kLog2e / a.tau[h * K + tid];
+    if (tid < 32) tmem_alloc(tslot, 512);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tslot;
-    const uint32_t lane_base = tmem + (uint32_t(w * 32) << 16);
+    const uint32_t lane_base = tmem + (uint32_t(w4 * 32) << 16);
     const uint32_t colG = 0, colZ = 128, colY = 128 + ZN;
 
     if (tid == 0) {
@@ -353,7 +354,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         int(((size_t(b) * d.H + h) * d.nc + c) * K));
         }
     }
-    // per-position data of row t
+    // per-position data of row t (both groups hold it)
     float tmax = 0.f;
     for (int m = 0; m < K; ++m) tmax = fmaxf(tmax, a.tau[h * K + m]);
     const float log_cap = logf(64.f * tmax);
@@ -363,17 +364,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         const size_t i = blh(d, b, c0 + t, h);
         bool cl;
         e = token_rate(a.dt[i], a.alpha[i], a.lam[i], log_cap, &cl);
-        const uint4 *src = reinterpret_cast<const uint4 *>(a.x + i * P + p0);
-        uint4 *dst = reinterpret_cast<uint4 *>(xs + t * TPS);
+        if (grp == 0) {
+            const uint4 *src = reinterpret_cast<const uint4 *>(a.x + i * P + p0);
+            uint4 *dst = reinterpret_cast<uint4 *>(xs + t * TPS);
 #pragma unroll
-        for (int q = 0; q < 4; ++q) dst[q] = src[q];
-    } else {
+            for (int q = 0; q < 4; ++q) dst[q] = src[q];
+        }
+    } else if (grp == 0) {
         uint4 *dst = reinterpret_cast<uint4 *>(xs + t * TPS);
 #pragma unroll
         for (int q = 0; q < 4; ++q) dst[q] = make_uint4(0, 0, 0, 0);
     }
-    const double Et = block_scan128(double(e), wsum);
-    E_s[t] = Et;
+    const double Et = group_scan128(double(e), wsum);
+    if (grp == 0) E_s[t] = Et;
 #pragma unroll
     for (int m = 0; m < KMAX; ++m) {
         wr_t[m] = 0.f;
@@ -383,15 +386,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (t < n) {
                 const size_t wi = blh(d, b, c0 + t, h) * K + m;
                 wr_t[m] = to_f(a.wr[wi]);
-                kp = -expm1f(-e * itau[m]) * to_f(a.ww[wi]);
-                f_t[m] = wr_t[m] * expf(-float(Et) * itau[m]);
+                kp = -expm1f(-e * (l2t[m] / kLog2e)) * to_f(a.ww[wi]);
+                f_t[m] = wr_t[m] * ex2_approx(-float(Et) * l2t[m]);
             }
-            kap_s[t * 32 + m] = kp;
+            if (grp == 0) kap_s[t * 32 + m] = kp;
         }
     }
     __syncthreads();
     // X^T tile: row p, column k = t (K-major, 128-byte swizzle, 32 rows per k-atom)
-    {
+    if (grp == 0) {
         unsigned char *tile = sX + (t >> 6) * 4096;
         const int kk = t & 63;
 #pragma unroll
@@ -425,8 +428,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
     if (!*abort_s) {
-        // row t of Gamma o G -> bf16, K-major [t][k]
-        for (int k32 = 0; k32 < TQ; k32 += 32) {
+        // row t of Gamma o G -> bf16, K-major [t][k]; group 0 takes k in [0,32) and [96,128),
+        // group 1 takes [32,96) (the causal triangle splits about evenly)
+        for (int half = 0; half < 2; ++half) {
+            const int k32 = grp == 0 ? (half == 0 ? 0 : 96) : (half == 0 ? 32 : 64);
             float gv[32];
             tmem_ld32(lane_base + colG + k32, gv);
             tmem_ld_wait();
@@ -439,7 +444,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     float gam = 0.f;
 #pragma unroll
                     for (int m = 0; m < KMAX; ++m)
-                        if (m < K) gam = fmaf(wr_t[m] * kap_s[k * 32 + m], expf(-dE * itau[m]), gam);
+                        if (m < K) gam = fmaf(wr_t[m] * kap_s[k * 32 + m], ex2_approx(-dE * l2t[m]), gam);
                     v = gam * gv[kk];
                 }
                 gv[kk] = v;
@@ -467,24 +472,41 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         mma_commit(&bars[2]);
     }
+    // mode-weighted readout of Z: group g takes modes [g K/2, (g+1) K/2)
+    float acc[32];
+#pragma unroll
+    for (int p = 0; p < 32; ++p) acc[p] = 0.f;
+    if (!*abort_s) {
+        const int m0 = grp * (K / 2);
+#pragma unroll
+        for (int mm = 0; mm < KMAX / 2; ++mm) {
+            if (mm >= K / 2) break;
+            const int m = m0 + mm;
+            float z[32];
+            tmem_ld32(lane_base + colZ + m * TPS, z);
+            tmem_ld_wait();
+            float fm = 0.f;
+#pragma unroll
+            for (int q = 0; q < KMAX; ++q)
+                if (q == m) fm = f_t[q];
+#pragma unroll
+            for (int p = 0; p < 32; ++p) acc[p] = fmaf(fm, z[p], acc[p]);
+        }
+    }
+    __syncthreads();  // kap_s is no longer read: reuse it for group 1's partial sums
+    float *part = kap_s;  // [32][128], column-major in t
+    if (grp == 1) {
+#pragma unroll
+        for (int p = 0; p < 32; ++p) part[p * TQ + t] = acc[p];
+    }
     __syncthreads();
     if (!*abort_s && !mbar_wait(&bars[2], 0)) *abort_s = 1;
     __syncthreads();
     tc_fence_after();
-    if (!*abort_s) {
-        float acc[32];
-        tmem_ld32(lane_base + colY, acc);
+    if (!*abort_s && grp == 0) {
+        float yi[32];
+        tmem_ld32(lane_base + colY, yi);
         tmem_ld_wait();
-#pragma unroll
-        for (int m = 0; m < KMAX; ++m) {
-            if (m >= K) break;
-            float z[32];
-            tmem_ld32(lane_base + colZ + m * TPS, z);
-            tmem_ld_wait();
-            const float fm = f_t[m];
-#pragma unroll
-            for (int p = 0; p < 32; ++p) acc[p] = fmaf(fm, z[p], acc[p]);
-        }
         if (t < n) {
             const float Dh = a.D[h];
             uint4 *o = reinterpret_cast<uint4 *>(a.y + blh(d, b, c0 + t, h) * P + p0);
@@ -492,7 +514,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int q = 0; q < 4; ++q) {
                 float v[8];
 #pragma unroll
-                for (int i = 0; i < 8; ++i) v[i] = acc[8 * q + i] + Dh * __bfloat162float(xs[t * TPS + 8 * q + i]);
+                for (int i = 0; i < 8; ++i) {
+                    const int p = 8 * q + i;
+                    v[i] = acc[p] + part[p * TQ + t] + yi[p] + Dh * __bfloat162float(xs[t * TPS + p]);
+                }
                 o[q] = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]),
                                   pack_bf16x2(v[6], v[7]));
             }
@@ -501,7 +526,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (*abort_s && tid == 0) atomicExch(a.err, kTimeoutCode);
     tc_fence_before();
     __syncthreads();
-    if (w == 0) tmem_dealloc(tmem, 512);
+    if (tid < 32) tmem_dealloc(tmem, 512);
 }
 
 // ------------------------------------------------------------------------------------- host
@@ -612,7 +637,7 @@ cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, int *e
     cudaFuncSetAttribute(tc_chunk_fwd, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
     dim3 grid(d.H * (d.P / TPS), d.nc, d.B);
     trace_begin("chunk_fwd_tc", st);
-    tc_chunk_fwd<<<grid, kThreads, smem, st>>>(mapC, mapB, mapS, a);
+    tc_chunk_fwd<<<grid, kOutThreads, smem, st>>>(mapC, mapB, mapS, a);
     trace_end(st);
     return cudaGetLastError();
 }

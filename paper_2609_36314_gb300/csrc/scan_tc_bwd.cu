@@ -82,6 +82,8 @@ __device__ __forceinline__ unsigned char *align1024(unsigned char *p) {
 }
 
 // ============================================================================= intra
+constexpr int kIntraThreads = 256;  // two groups of four warps share the 128 TMEM lanes
+
 struct IntraSmem {
     int rcb, x, dy, mg, xx, total;
     __host__ __device__ IntraSmem() {
@@ -90,11 +92,11 @@ struct IntraSmem {
         dy = 16384;                // dy chunk
         mg = 2 * 16384;            // Gamma o G, [t][k] K-major
         xx = TQ * XS * 4;          // fp32 Gamma' G H, then its row prefix sums
-        total = rcb + x + dy + mg + xx + 2 * TQ * KMAX * 4 + TQ * 8 + 64 * 4 + 64 + 64;
+        total = rcb + x + dy + mg + xx + 3 * TQ * KMAX * 4 + TQ * 8 + 64 * 4 + 64 + 64 + 64;
     }
 };
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kIntraThreads, 1)
     tc_bwd_intra(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapB,
                  const __grid_constant__ CUtensorMap mapX, const __grid_constant__ CUtensorMap mapDY,
                  BwdArgs a) {
@@ -112,14 +114,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     float *XX = reinterpret_cast<float *>(sMG + L.mg);
     float *wr_s = XX + TQ * XS;                              // [128][KMAX]
     float *kap_s = wr_s + TQ * KMAX;                         // [128][KMAX]
-    double *E_s = reinterpret_cast<double *>(kap_s + TQ * KMAX);
-    float *itau = reinterpret_cast<float *>(E_s + TQ);
-    double *wsum = reinterpret_cast<double *>(itau + 32);
+    float *part = kap_s + TQ * KMAX;                         // [128][KMAX] partial sums of group 1
+    double *E_s = reinterpret_cast<double *>(part + TQ * KMAX);
+    float *l2t = reinterpret_cast<float *>(E_s + TQ);
+    double *wsum = reinterpret_cast<double *>(l2t + 32);
     uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 3);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
 
-    const int tid = threadIdx.x, w = tid >> 5, t = tid;
+    const int tid = threadIdx.x, grp = tid >> 7, t = tid & 127, w4 = (tid >> 5) & 3;
     const int h = blockIdx.x, c = blockIdx.y, b = blockIdx.z;
     const int g = h / (d.H / d.G);
     const int c0 = c * TQ, n = min(TQ, d.L - c0);
@@ -129,13 +132,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         *abort_s = 0;
         fence_barrier_init();
     }
-    if (tid < K) itau[tid] = 1.f / a.tau[h * K + tid];
-    if (w == 0) tmem_alloc(tslot, 512);
+    if (tid < K) l2t[tid] = kLog2e / a.tau[h * K + tid];
+    if (tid < 32) tmem_alloc(tslot, 512);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tslot;
-    const uint32_t lane_base = tmem + (uint32_t(w * 32) << 16);
+    const uint32_t lane_base = tmem + (uint32_t(w4 * 32) << 16);
     const uint32_t colG = 0, colH = 128, colX = 256;
 
     if (tid == 0) {
@@ -155,19 +158,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool cl;
         e = token_rate(a.dt[i], a.alpha[i], a.lam[i], log_cap, &cl);
     }
-    const double Et = block_scan128(double(e), wsum);
-    E_s[t] = Et;
+    const double Et = group_scan128(double(e), wsum);
+    if (grp == 0) E_s[t] = Et;
 #pragma unroll
     for (int m = 0; m < KMAX; ++m) {
         float wv = 0.f, kp = 0.f;
         if (m < K && t < n) {
             const size_t wi = blh(d, b, c0 + t, h) * K + m;
             wv = to_f(a.wr[wi]);
-            kp = -expm1f(-e * itau[m]) * to_f(a.ww[wi]);
+            kp = -expm1f(-e * (l2t[m] / kLog2e)) * to_f(a.ww[wi]);
         }
         wr_t[m] = wv;
-        wr_s[t * KMAX + m] = wv;
-        kap_s[t * KMAX + m] = kp;
+        if (grp == 0) {
+            wr_s[t * KMAX + m] = wv;
+            kap_s[t * KMAX + m] = kp;
+        }
     }
     __syncthreads();
     if (tid == 0) {
@@ -192,19 +197,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (!*abort_s && !mbar_wait(&bars[1], 0)) *abort_s = 1;
     __syncthreads();
     tc_fence_after();
-    // ---- row pass (thread t): Gamma, Gamma', intra dw_read, Gamma o G tile, Gamma o H (summed
-    // over heads in L2), Gamma' G H and G H pair tiles
+    // ---- row pass (row t; group 0 takes k in [0,32) and [96,128), group 1 takes [32,96)):
+    // Gamma, Gamma', intra dw_read, Gamma o G tile, Gamma o H summed over heads in L2, Gamma' G H
+    // and G H pair tiles
     float dwr_i[KMAX];
 #pragma unroll
     for (int m = 0; m < KMAX; ++m) dwr_i[m] = 0.f;
     if (!*abort_s) {
         float *mh_row = a.mh_total + ((size_t(b) * d.nc + c) * TQ + t) * TQ;
-        for (int k32 = 0; k32 < TQ; k32 += 32) {
+        for (int half = 0; half < 2; ++half) {
+            const int k32 = grp == 0 ? (half == 0 ? 0 : 96) : (half == 0 ? 32 : 64);
             float gv[32], hv[32];
             tmem_ld32(lane_base + colG + k32, gv);
             tmem_ld32(lane_base + colH + k32, hv);
             tmem_ld_wait();
-            float mg[32];
 #pragma unroll
             for (int kk = 0; kk < 32; ++kk) {
                 const int k = k32 + kk;
@@ -215,25 +221,27 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int m = 0; m < KMAX; ++m) {
                         if (m < K) {
-                            const float W = expf(-dE * itau[m]);
+                            const float W = ex2_approx(-dE * l2t[m]);
                             const float kp = kap_s[k * KMAX + m];
                             const float aa = wr_t[m] * kp * W;
                             gam += aa;
-                            gamt = fmaf(aa, itau[m], gamt);
+                            gamt = fmaf(aa, l2t[m], gamt);  // times log2(e) / tau
                             dwr_i[m] = fmaf(kp * W, gh, dwr_i[m]);
                         }
                     }
                 }
-                mg[kk] = gam * gv[kk];
+                gv[kk] = gam * gv[kk];  // Gamma o G
                 hv[kk] = gam * hv[kk];  // Gamma o H
-                XX[t * XS + k] = gamt * gh;
+                XX[t * XS + k] = gamt * (1.f / kLog2e) * gh;
                 GHs[t * XS + k] = gh;
             }
             unsigned char *tile = sMG + (k32 >> 6) * 16384;
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 const int c8 = ((k32 & 63) >> 3) + q;
-                store_bf16x8(tile + t * 128 + ((c8 ^ (t & 7)) * 16), mg + 8 * q);
+                *reinterpret_cast<uint4 *>(tile + t * 128 + ((c8 ^ (t & 7)) * 16)) =
+                    make_uint4(pack_bf16x2(gv[8 * q], gv[8 * q + 1]), pack_bf16x2(gv[8 * q + 2], gv[8 * q + 3]),
+                               pack_bf16x2(gv[8 * q + 4], gv[8 * q + 5]), pack_bf16x2(gv[8 * q + 6], gv[8 * q + 7]));
             }
             if (t < n && k32 <= t) {
 #pragma unroll
@@ -243,15 +251,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                                   make_float4(hv[4 * q], hv[4 * q + 1], hv[4 * q + 2], hv[4 * q + 3]));
             }
         }
-        if (t < n) {
-            float *o = a.dwr_acc + blh(d, b, c0 + t, h) * K;
-            for (int m = 0; m < K; ++m) o[m] = dwr_i[m];
+        if (grp == 1) {
+#pragma unroll
+            for (int m = 0; m < KMAX; ++m) part[t * KMAX + m] = dwr_i[m];
         }
     }
     fence_async_smem();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    if (!*abort_s && grp == 0 && t < n) {
+        float *o = a.dwr_acc + blh(d, b, c0 + t, h) * K;
+#pragma unroll
+        for (int m = 0; m < KMAX; ++m)
+            if (m < K) o[m] = dwr_i[m] + part[t * KMAX + m];
+    }
     if (tid == 0 && !*abort_s) {  // dx_intra = (Gamma o G)^T dY: M = k, N = p, K = t
         const uint32_t idX = idesc_bf16(128, BP, true, true);
         for (int ks = 0; ks < TQ / 16; ++ks)
@@ -259,25 +273,28 @@ __global__ void __launch_bounds__(kThreads, 1)
                      desc_sw128(smem_u32(sDY) + ks * 2048, 16384, 1024), idX, ks > 0);
         mma_commit(&bars[2]);
     }
-    // ---- column pass (thread k): intra dkappa; pair rectangle sums
-    if (!*abort_s) {
+    __syncthreads();  // part[] is reused below
+    // ---- column pass (column k = t; group g takes rows t' = k + g, k + g + 2, ...): intra dkappa
+    float dk[KMAX];
+#pragma unroll
+    for (int m = 0; m < KMAX; ++m) dk[m] = 0.f;
+    if (!*abort_s && t < n) {
         const int k = t;
-        float dk[KMAX];
+        const double Ek = E_s[k];
+        for (int tt = k + grp; tt < n; tt += 2) {
+            const float dE = float(E_s[tt] - Ek);
+            const float gh = GHs[tt * XS + k];
 #pragma unroll
-        for (int m = 0; m < KMAX; ++m) dk[m] = 0.f;
-        if (k < n) {
-            const double Ek = E_s[k];
-            for (int tt = k; tt < n; ++tt) {
-                const float dE = float(E_s[tt] - Ek);
-                const float gh = GHs[tt * XS + k];
-#pragma unroll
-                for (int m = 0; m < KMAX; ++m)
-                    if (m < K) dk[m] = fmaf(wr_s[tt * KMAX + m] * expf(-dE * itau[m]), gh, dk[m]);
-            }
-            float *o = a.dkap_acc + blh(d, b, c0 + k, h) * K;
-            for (int m = 0; m < K; ++m) o[m] = dk[m];
+            for (int m = 0; m < KMAX; ++m)
+                if (m < K) dk[m] = fmaf(wr_s[tt * KMAX + m] * ex2_approx(-dE * l2t[m]), gh, dk[m]);
         }
-        // exclusive row prefix of XX (row t)
+        if (grp == 1) {
+#pragma unroll
+            for (int m = 0; m < KMAX; ++m) part[k * KMAX + m] = dk[m];
+        }
+    }
+    // exclusive row prefix of XX (row t, group 0)
+    if (!*abort_s && grp == 0) {
         float run = 0.f;
         for (int j = 0; j < TQ; ++j) {
             const float v = XX[t * XS + j];
@@ -286,31 +303,33 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     }
     __syncthreads();
-    if (!*abort_s && t < n) {
-        float s = 0.f;
-        for (int tp = t; tp < n; ++tp) s += XX[tp * XS + t];
-        a.rect[blh(d, b, c0 + t, h)] = s;
+    if (!*abort_s && grp == 0 && t < n) {
+        float *o = a.dkap_acc + blh(d, b, c0 + t, h) * K;
+#pragma unroll
+        for (int m = 0; m < KMAX; ++m)
+            if (m < K) o[m] = dk[m] + part[t * KMAX + m];
+        float sr = 0.f;
+        for (int tp = t; tp < n; ++tp) sr += XX[tp * XS + t];
+        a.rect[blh(d, b, c0 + t, h)] = sr;
     }
     __syncthreads();
     if (!*abort_s && !mbar_wait(&bars[2], 0)) *abort_s = 1;
     __syncthreads();
     tc_fence_after();
-    if (!*abort_s) {
+    if (!*abort_s) {  // dx_intra row: group g takes columns [32 g, 32 g + 32)
         float v[32];
-        for (int p32 = 0; p32 < BP; p32 += 32) {
-            tmem_ld32(lane_base + colX + p32, v);
-            tmem_ld_wait();
-            if (t < n) {
-                float4 *o = reinterpret_cast<float4 *>(a.dx_acc + blh(d, b, c0 + t, h) * P + p32);
+        tmem_ld32(lane_base + colX + grp * 32, v);
+        tmem_ld_wait();
+        if (t < n) {
+            float4 *o = reinterpret_cast<float4 *>(a.dx_acc + blh(d, b, c0 + t, h) * P + grp * 32);
 #pragma unroll
-                for (int q = 0; q < 8; ++q) o[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-            }
+            for (int q = 0; q < 8; ++q) o[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
         }
     }
     if (*abort_s && tid == 0) atomicExch(a.err, kTimeoutCode);
     tc_fence_before();
     __syncthreads();
-    if (w == 0) tmem_dealloc(tmem, 512);
+    if (tid < 32) tmem_dealloc(tmem, 512);
 }
 
 // ============================================================================= inter
@@ -855,7 +874,7 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
         const size_t smem = IntraSmem().total + 1024;
         cudaFuncSetAttribute(tc_bwd_intra, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
         trace_begin("bwd_intra_tc", st);
-        tc_bwd_intra<<<dim3(d.H, d.nc, d.B), kThreads, smem, st>>>(mapC, mapB, mapX, mapDY, a);
+        tc_bwd_intra<<<dim3(d.H, d.nc, d.B), kIntraThreads, smem, st>>>(mapC, mapB, mapX, mapDY, a);
         trace_end(st);
         if ((e = cudaGetLastError())) return e;
     }

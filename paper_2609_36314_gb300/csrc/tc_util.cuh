@@ -35,4 +35,27 @@ __device__ __forceinline__ double block_scan128(double v, double *wsum) {
     return v + off;
 }
 
+// 2^x with the hardware approximation (relative error ~2^-22); exp(-d / tau) is evaluated as
+// 2^(-d * l2t) with l2t = log2(e) / tau precomputed.
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+constexpr float kLog2e = 1.4426950408889634f;
+
+// Inclusive prefix sum (double) of one value per thread within groups of four warps (threads
+// 128 g .. 128 g + 127 scan independently); wsum holds one slot per warp.
+__device__ __forceinline__ double group_scan128(double v, double *wsum) {
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    v = warp_inclusive_scan_d(v);
+    if (lane == 31) wsum[w] = v;
+    __syncthreads();
+    double off = 0.0;
+    const int g0 = w & ~3;
+    for (int i = g0; i < w; ++i) off += wsum[i];
+    __syncthreads();
+    return v + off;
+}
+
 }  // namespace frac
