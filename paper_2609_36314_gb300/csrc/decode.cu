@@ -30,7 +30,7 @@ template <> struct Vec4<__nv_bfloat16> {
 constexpr int kDecodeModeGroup = 8;
 
 template <typename T, bool VEC>
-__global__ void __launch_bounds__(256) decode_step_kernel(
+__global__ void __launch_bounds__(256, 4) decode_step_kernel(
     DecodeArgs a, const T *__restrict__ x, const T *__restrict__ Bt, const T *__restrict__ Ct,
     const T *__restrict__ wr, const T *__restrict__ ww, T *__restrict__ y) {
     const int64_t row = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;

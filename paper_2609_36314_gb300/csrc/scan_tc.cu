@@ -122,18 +122,8 @@ __global__ void __launch_bounds__(kThreads, 2)
     for (int ci = 0; ci < d.nc; ++ci, phase ^= 1) {
         const int c = REV ? d.nc - 1 - ci : ci;
         const int c0 = c * TQ, n = min(TQ, d.L - c0);
-        if (ci > 0) {  // previous chunk's MMAs done: tensor memory, sA and sV are free
-            if (!mbar_wait(&bars[1], phase ^ 1)) *abort_s = 1;
-        }
-        __syncthreads();
-        if (*abort_s) break;
-        tc_fence_after();
-        if (tid == 0) {
-            mbar_arrive_expect_tx(&bars[0], uint32_t(N * TQ * 2));
-            for (int jb = 0; jb < N / 64; ++jb)
-                tma_load_3d(sV + jb * 16384, &mapV, &bars[0], g * N + 64 * jb, c0, b);
-        }
-        // chunk inputs: x / dy rows of the P-slice, rates, weights
+        // chunk inputs (x / dy rows of the P-slice, rates, weights) and coefficients: xs and coef
+        // were last read before the previous chunk's MMAs were issued, so this overlaps them
         {
             const int t = tid;
             float e = 0.f;
@@ -170,7 +160,17 @@ __global__ void __launch_bounds__(kThreads, 2)
             }
             if (t < K) dec[t] = expf(-float(Eend) * itau[t]);
         }
+        if (ci > 0) {  // previous chunk's MMAs done: tensor memory, sA and sV are free
+            if (!mbar_wait(&bars[1], phase ^ 1)) *abort_s = 1;
+        }
         __syncthreads();
+        if (*abort_s) break;
+        tc_fence_after();
+        if (tid == 0) {
+            mbar_arrive_expect_tx(&bars[0], uint32_t(N * TQ * 2));
+            for (int jb = 0; jb < N / 64; ++jb)
+                tma_load_3d(sV + jb * 16384, &mapV, &bars[0], g * N + 64 * jb, c0, b);
+        }
         // emit the entering state (bf16) and apply the chunk's decay in place
         for (int mt = 0; mt < mtiles; ++mt) {
             const int m = mt * 4 + w;
@@ -315,7 +315,7 @@ __global__ void __launch_bounds__(kOutThreads, 1)
     unsigned char *sX = sM + 2 * 16384;             // X^T, [p][k] K-major, 2 atoms of 32 rows
     bf16 *xs = reinterpret_cast<bf16 *>(sX + 2 * 4096);         // [128][32]
     float *kap_s = reinterpret_cast<float *>(xs + TQ * TPS);     // [128][32]; later partial y
-    double *E_s = reinterpret_cast<double *>(kap_s + TQ * 32);   // [128]
+    float2 *E_s = reinterpret_cast<float2 *>(kap_s + TQ * 32);   // [128] hi / lo pairs
     float *l2t = reinterpret_cast<float *>(E_s + TQ);            // [32] log2(e) / tau
     double *wsum = reinterpret_cast<double *>(l2t + 32);         // [8]
     uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);     // tma, mma1, mma2
@@ -376,7 +376,8 @@ __global__ void __launch_bounds__(kOutThreads, 1)
         for (int q = 0; q < 4; ++q) dst[q] = make_uint4(0, 0, 0, 0);
     }
     const double Et = group_scan128(double(e), wsum);
-    if (grp == 0) E_s[t] = Et;
+    const float2 Et2 = split_f2(Et);
+    if (grp == 0) E_s[t] = Et2;
 #pragma unroll
     for (int m = 0; m < KMAX; ++m) {
         wr_t[m] = 0.f;
@@ -440,7 +441,7 @@ __global__ void __launch_bounds__(kOutThreads, 1)
                 const int k = k32 + kk;
                 float v = 0.f;
                 if (k <= t && t < n) {
-                    const float dE = float(Et - E_s[k]);
+                    const float dE = diff_f2(Et2, E_s[k]);
                     float gam = 0.f;
 #pragma unroll
                     for (int m = 0; m < KMAX; ++m)

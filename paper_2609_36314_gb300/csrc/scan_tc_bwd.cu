@@ -115,7 +115,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     float *wr_s = XX + TQ * XS;                              // [128][KMAX]
     float *kap_s = wr_s + TQ * KMAX;                         // [128][KMAX]
     float *part = kap_s + TQ * KMAX;                         // [128][KMAX] partial sums of group 1
-    double *E_s = reinterpret_cast<double *>(part + TQ * KMAX);
+    float2 *E_s = reinterpret_cast<float2 *>(part + TQ * KMAX);  // hi / lo pairs
     float *l2t = reinterpret_cast<float *>(E_s + TQ);
     double *wsum = reinterpret_cast<double *>(l2t + 32);
     uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);
@@ -159,7 +159,8 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         e = token_rate(a.dt[i], a.alpha[i], a.lam[i], log_cap, &cl);
     }
     const double Et = group_scan128(double(e), wsum);
-    if (grp == 0) E_s[t] = Et;
+    const float2 Et2 = split_f2(Et);
+    if (grp == 0) E_s[t] = Et2;
 #pragma unroll
     for (int m = 0; m < KMAX; ++m) {
         float wv = 0.f, kp = 0.f;
@@ -216,7 +217,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
                 const int k = k32 + kk;
                 float gam = 0.f, gamt = 0.f, gh = 0.f;
                 if (k <= t && t < n) {
-                    const float dE = float(Et - E_s[k]);
+                    const float dE = diff_f2(Et2, E_s[k]);
                     gh = gv[kk] * hv[kk];
 #pragma unroll
                     for (int m = 0; m < KMAX; ++m) {
@@ -280,9 +281,9 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     for (int m = 0; m < KMAX; ++m) dk[m] = 0.f;
     if (!*abort_s && t < n) {
         const int k = t;
-        const double Ek = E_s[k];
+        const float2 Ek = E_s[k];
         for (int tt = k + grp; tt < n; tt += 2) {
-            const float dE = float(E_s[tt] - Ek);
+            const float dE = diff_f2(E_s[tt], Ek);
             const float gh = GHs[tt * XS + k];
 #pragma unroll
             for (int m = 0; m < KMAX; ++m)

@@ -44,6 +44,15 @@ __device__ __forceinline__ float ex2_approx(float x) {
 }
 constexpr float kLog2e = 1.4426950408889634f;
 
+// A cumulative log-decay kept as an unevaluated float pair hi + lo (hi = E rounded to float):
+// the difference of two such values is accurate to float precision of the difference itself,
+// without a double-precision subtraction per pair.
+__device__ __forceinline__ float2 split_f2(double E) {
+    const float hi = float(E);
+    return make_float2(hi, float(E - double(hi)));
+}
+__device__ __forceinline__ float diff_f2(float2 a, float2 b) { return (a.x - b.x) + (a.y - b.y); }
+
 // Inclusive prefix sum (double) of one value per thread within groups of four warps (threads
 // 128 g .. 128 g + 127 scan independently); wsum holds one slot per warp.
 __device__ __forceinline__ double group_scan128(double v, double *wsum) {
