@@ -261,8 +261,10 @@ def main():
     inp = synth.make_scan_inputs_torch(s, seed=1000 + rank, device=dev, with_dy=True)
     dims = make_dims(s.batch, s.seqlen, s.nheads, s.headdim, s.ngroups, s.dstate, s.nmodes,
                      torch.bfloat16)
-    ws_f = torch.empty(fwd_workspace_size(dims), dtype=torch.uint8, device=dev)
-    ws_b = torch.empty(bwd_workspace_size(dims), dtype=torch.uint8, device=dev)
+    # one workspace for both calls: the backward reuses the per-chunk states of the forward
+    ws_b = torch.empty(max(bwd_workspace_size(dims), fwd_workspace_size(dims)), dtype=torch.uint8,
+                       device=dev)
+    ws_f = ws_b
     y = torch.empty_like(inp["x"])
     grads = dict(dx=torch.empty_like(inp["x"]), ddt=torch.empty_like(inp["dt"]),
                  dalpha=torch.empty_like(inp["alpha"]), dlam=torch.empty_like(inp["lam"]),
@@ -275,7 +277,7 @@ def main():
         scan_fwd(a["x"], a["dt"], a["alpha"], a["lam"], a["tau"], a["B"], a["C"], a["w_read"],
                  a["w_write"], a["D"], want_final_state=False, y=y, workspace=ws_f)
         scan_bwd(a["x"], a["dt"], a["alpha"], a["lam"], a["tau"], a["B"], a["C"], a["w_read"],
-                 a["w_write"], a["D"], a["dy"], workspace=ws_b, out=grads)
+                 a["w_write"], a["D"], a["dy"], workspace=ws_b, out=grads, reuse_fwd_states=True)
 
     for _ in range(max(args.warmup, 3)):
         train_step()

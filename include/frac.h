@@ -68,10 +68,16 @@ typedef enum { FRAC_DTYPE_F32 = 0, FRAC_DTYPE_BF16 = 1 } frac_dtype;
 /* Bits of frac_dims.flags. */
 enum {
     /* Use the CUDA-core chunked kernels even where tensor-core ones exist.  Without it, bf16
-       calls with headdim % 32 == 0, dstate in {64, 128} and nmodes in {4, 8} run the forward on
-       the tensor cores (TMA-fed tcgen05 MMAs, chunk 128); they need x, Bm, Cm, y (and h_final)
-       16-byte aligned. */
-    FRAC_FLAG_FORCE_SIMT = 1
+       calls with headdim 32 or 64, dstate in {64, 128} and nmodes in {4, 8} run the forward on
+       the tensor cores (TMA-fed tcgen05 MMAs, chunk 128), and with headdim 64 the backward too;
+       they need the dtype tensors and the states 16-byte aligned. */
+    FRAC_FLAG_FORCE_SIMT = 1,
+    /* frac_scan_bwd only: the workspace already holds the per-chunk states that a frac_scan_fwd
+       call with the same inputs, h0 and dims left in this same workspace (give both calls one
+       buffer of frac_scan_bwd_workspace_size bytes), so the backward does not recompute them.
+       Rejected with FRAC_ERR_INVALID_ARGUMENT when the forward and backward would run on
+       different paths (then the states are not compatible). */
+    FRAC_FLAG_BWD_REUSE_FWD_STATES = 2
 };
 
 typedef struct {
@@ -105,7 +111,8 @@ frac_status frac_scan_fwd_workspace_size(const frac_dims *dims, size_t *bytes);
  *   y        : output [B, L, H, P] (dtype)
  *   h_final  : final mode state S_L (float32), or NULL; it is the decode cache
  *   workspace: >= frac_scan_fwd_workspace_size bytes, 256-byte aligned; contents undefined on
- *              entry and exit; must not be used concurrently by another call.
+ *              entry; on exit it holds the per-chunk states (see FRAC_FLAG_BWD_REUSE_FWD_STATES);
+ *              must not be used concurrently by another call.
  */
 frac_status frac_scan_fwd(const frac_dims *dims, const void *x, const float *dt,
                           const float *alpha, const float *lam, const float *tau,

@@ -33,6 +33,7 @@ FRAC_OK = 0
 FRAC_DTYPE_F32 = 0
 FRAC_DTYPE_BF16 = 1
 FRAC_FLAG_FORCE_SIMT = 1
+FRAC_FLAG_BWD_REUSE_FWD_STATES = 2
 FRAC_SCAN_FWD_STATIC_SCRATCH_BYTES = 64 << 20
 
 

@@ -17,9 +17,11 @@ _DT = {torch.float32: _lib.FRAC_DTYPE_F32, torch.bfloat16: _lib.FRAC_DTYPE_BF16}
 
 
 def make_dims(batch, seqlen, nheads, headdim, ngroups, dstate, nmodes, dtype, chunk=0,
-              force_simt=False) -> _lib.FracDims:
+              force_simt=False, reuse_fwd_states=False) -> _lib.FracDims:
+    flags = (_lib.FRAC_FLAG_FORCE_SIMT if force_simt else 0) | (
+        _lib.FRAC_FLAG_BWD_REUSE_FWD_STATES if reuse_fwd_states else 0)
     return _lib.FracDims(batch, seqlen, nheads, headdim, ngroups, dstate, nmodes, chunk,
-                         _DT[dtype], _lib.FRAC_FLAG_FORCE_SIMT if force_simt else 0)
+                         _DT[dtype], flags)
 
 
 def _ptr(t):
@@ -45,13 +47,14 @@ def _need(t, name, dtype, shape=None):
     return t
 
 
-def _scan_dims(x, B, tau, chunk, force_simt):
+def _scan_dims(x, B, tau, chunk, force_simt, reuse_fwd_states=False):
     if x.dim() != 4 or B.dim() != 4 or tau.dim() != 2:
         raise ValueError("x [B,L,H,P], B/C [B,L,G,N], tau [H,K] expected")
     Bz, L, H, P = x.shape
     G, N = B.shape[2], B.shape[3]
     K = tau.shape[1]
-    return make_dims(Bz, L, H, P, G, N, K, x.dtype, chunk, force_simt), (Bz, L, H, P, G, N, K)
+    return (make_dims(Bz, L, H, P, G, N, K, x.dtype, chunk, force_simt, reuse_fwd_states),
+            (Bz, L, H, P, G, N, K))
 
 
 def fwd_workspace_size(dims: _lib.FracDims) -> int:
@@ -126,10 +129,14 @@ def scan_fwd_static(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, h0=None, *
 
 
 def scan_bwd(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, dy, h0=None, dh_final=None, *,
-             chunk=0, force_simt=False, want_dh0=True, workspace=None, out=None, stream=None):
+             chunk=0, force_simt=False, want_dh0=True, workspace=None, out=None, stream=None,
+             reuse_fwd_states=False):
     """Backward of scan_fwd.  Returns a dict of gradients (dx, ddt, dalpha, dlam, dB, dC,
-    dw_read, dw_write, dD, dh0)."""
-    dims, (Bz, L, H, P, G, N, K) = _scan_dims(x, B, tau, chunk, force_simt)
+    dw_read, dw_write, dD, dh0).  With reuse_fwd_states, `workspace` must be the buffer a
+    scan_fwd call on the same inputs just used (sized with bwd_workspace_size)."""
+    if reuse_fwd_states and workspace is None:
+        raise ValueError("reuse_fwd_states needs the workspace of the forward call")
+    dims, (Bz, L, H, P, G, N, K) = _scan_dims(x, B, tau, chunk, force_simt, reuse_fwd_states)
     dt_ = x.dtype
     f32 = torch.float32
     _need(dy, "dy", dt_, (Bz, L, H, P))

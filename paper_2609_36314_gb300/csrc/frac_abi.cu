@@ -287,6 +287,17 @@ frac_status frac_scan_bwd(const frac_dims *d, const void *x, const float *dt, co
     int path;
     if ((s = plan(d, &sd, &path, true))) return s;
     const BwdLayout l = bwd_layout(d, sd, path);
+    const bool reuse = (d->flags & FRAC_FLAG_BWD_REUSE_FWD_STATES) != 0;
+    if (reuse) {
+        frac::ScanDims sf;
+        int fpath;
+        if ((s = plan(d, &sf, &fpath, false))) return s;
+        if (fpath != path || sf.Q != sd.Q)
+            return fail(FRAC_ERR_INVALID_ARGUMENT,
+                        "FRAC_FLAG_BWD_REUSE_FWD_STATES: the forward of these dims runs on another "
+                        "path (chunk %d) than the backward (chunk %d); its states cannot be reused",
+                        sf.Q, sd.Q);
+    }
     if (path == PATH_TC && d->seqlen > 0) {
         const void *need16[] = {x, Bm, Cm, dy, dx, dB, dC, dw_read, dw_write};
         for (const void *q : need16)
@@ -323,9 +334,10 @@ frac_status frac_scan_bwd(const frac_dims *d, const void *x, const float *dt, co
         if (path == PATH_TC) {
             frac::TcBwdWorkspace t;
             frac::tc_bwd_workspace_bytes(sd, &t, ws + kStatusBytes);
-            e = frac::tc_scan_bwd(sd, p, t, reinterpret_cast<int *>(ws), st);
+            e = frac::tc_scan_bwd(sd, p, t, reinterpret_cast<int *>(ws), reuse, st);
         } else {
-            e = frac::simt_scan_bwd(sd, d->dtype, p, ws + l.s_in, ws + l.ds_out, dB_acc, dC_acc, st);
+            e = frac::simt_scan_bwd(sd, d->dtype, p, ws + l.s_in, ws + l.ds_out, dB_acc, dC_acc,
+                                    reuse, st);
         }
     }
     return cuda_status(e, "frac_scan_bwd");

@@ -45,10 +45,12 @@ int simt_pick_chunk(const ScanDims &d, int requested);     // 0 if the shape is 
 size_t simt_state_elems(const ScanDims &d);                 // per-chunk state workspace elements
 cudaError_t simt_scan_fwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in,
                           cudaStream_t st);
+// reuse_states: S_in already holds the forward's per-chunk states (no recompute)
 cudaError_t simt_scan_bwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in,
-                          void *dS_out, float *dB_acc, float *dC_acc, cudaStream_t st);
+                          void *dS_out, float *dB_acc, float *dC_acc, bool reuse_states,
+                          cudaStream_t st);
 
-// Tensor-core (tcgen05) path: bf16 inputs, chunk 128, P % 32 == 0, N in {64, 128}, K in {4, 8}.
+// Tensor-core (tcgen05) path: bf16 inputs, chunk 128, P in {32, 64}, N in {64, 128}, K in {4, 8}.
 bool tc_supported(const ScanDims &d, int dtype);
 size_t tc_state_elems(const ScanDims &d);  // bf16 elements of the per-chunk state workspace
 cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, int *err,
@@ -73,6 +75,6 @@ struct TcBwdWorkspace {
 };
 size_t tc_bwd_workspace_bytes(const ScanDims &d, TcBwdWorkspace *layout, char *base);
 cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspace &ws, int *err,
-                        cudaStream_t st);
+                        bool reuse_states, cudaStream_t st);
 
 }  // namespace frac

@@ -865,8 +865,9 @@ cudaError_t fwd_t(const ScanDims &d, const ScanPtrs &p, void *S_in, cudaStream_t
 
 template <typename T, typename TS>
 cudaError_t bwd_t(const ScanDims &d, const ScanPtrs &p, void *S_in, void *dS_out, float *dB_acc,
-                  float *dC_acc, cudaStream_t st) {
-    cudaError_t e = run_state_pass<T, TS>(d, false, p.x, p.Bm, p.ww, p, p.h0, S_in, nullptr, st);
+                  float *dC_acc, bool reuse, cudaStream_t st) {
+    cudaError_t e = cudaSuccess;
+    if (!reuse) e = run_state_pass<T, TS>(d, false, p.x, p.Bm, p.ww, p, p.h0, S_in, nullptr, st);
     if (e != cudaSuccess) return e;
     e = run_state_pass<T, TS>(d, true, p.dy, p.Cm, p.wr, p, p.dh_final, dS_out, p.dh0, st);
     if (e != cudaSuccess) return e;
@@ -931,9 +932,9 @@ cudaError_t simt_scan_fwd(const ScanDims &d, int dtype, const ScanPtrs &p, void 
 }
 
 cudaError_t simt_scan_bwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in,
-                          void *dS_out, float *dB_acc, float *dC_acc, cudaStream_t st) {
-    if (dtype == 0) return bwd_t<float, float>(d, p, S_in, dS_out, dB_acc, dC_acc, st);
-    return bwd_t<__nv_bfloat16, __nv_bfloat16>(d, p, S_in, dS_out, dB_acc, dC_acc, st);
+                          void *dS_out, float *dB_acc, float *dC_acc, bool reuse, cudaStream_t st) {
+    if (dtype == 0) return bwd_t<float, float>(d, p, S_in, dS_out, dB_acc, dC_acc, reuse, st);
+    return bwd_t<__nv_bfloat16, __nv_bfloat16>(d, p, S_in, dS_out, dB_acc, dC_acc, reuse, st);
 }
 
 }  // namespace frac

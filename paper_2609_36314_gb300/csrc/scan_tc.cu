@@ -118,43 +118,81 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
     tmem_st_wait();
 
+    // Inputs of chunk ci + 1 are fetched into registers while chunk ci is processed, so the
+    // global-load latency is off the chunk-serial critical path.
+    uint4 nx[4];
+    float ndt = 1.f, nal = 1.f, nlm = 1.f;
+    float nw[KMAX];
+    auto fetch = [&](int ci_) {
+        const int c_ = REV ? d.nc - 1 - ci_ : ci_;
+        const int c0_ = c_ * TQ, n_ = min(TQ, d.L - c0_);
+        const int t = tid;
+        if (t < n_) {
+            const size_t i = blh(d, b, c0_ + t, h);
+            const uint4 *src = reinterpret_cast<const uint4 *>(a.U + i * P + p0);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) nx[q] = src[q];
+            ndt = a.dt[i];
+            nal = a.alpha[i];
+            nlm = a.lam[i];
+            if (K == 8) {
+                const uint4 wv = *reinterpret_cast<const uint4 *>(a.W + i * K);
+                const __nv_bfloat162 *w2 = reinterpret_cast<const __nv_bfloat162 *>(&wv);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float2 f = __bfloat1622float2(w2[q]);
+                    nw[2 * q] = f.x;
+                    nw[2 * q + 1] = f.y;
+                }
+            } else {
+#pragma unroll
+                for (int m = 0; m < KMAX; ++m) nw[m] = m < K ? to_f(a.W[i * K + m]) : 0.f;
+            }
+        } else {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) nx[q] = make_uint4(0, 0, 0, 0);
+#pragma unroll
+            for (int m = 0; m < KMAX; ++m) nw[m] = 0.f;
+        }
+    };
+    if (d.nc > 0) fetch(0);
+
     int phase = 0;
     for (int ci = 0; ci < d.nc; ++ci, phase ^= 1) {
         const int c = REV ? d.nc - 1 - ci : ci;
         const int c0 = c * TQ, n = min(TQ, d.L - c0);
-        // chunk inputs (x / dy rows of the P-slice, rates, weights) and coefficients: xs and coef
-        // were last read before the previous chunk's MMAs were issued, so this overlaps them
+        // this chunk's inputs (fetched one iteration earlier) and coefficients: xs and coef were
+        // last read before the previous chunk's MMAs were issued, so this overlaps them
+        float wcur[KMAX];
         {
             const int t = tid;
+            uint4 *dst = reinterpret_cast<uint4 *>(xs + t * TPS);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) dst[q] = nx[q];
+#pragma unroll
+            for (int m = 0; m < KMAX; ++m) wcur[m] = nw[m];
             float e = 0.f;
             if (t < n) {
-                const uint4 *src = reinterpret_cast<const uint4 *>(a.U + blh(d, b, c0 + t, h) * P + p0);
-                uint4 *dst = reinterpret_cast<uint4 *>(xs + t * TPS);
-#pragma unroll
-                for (int q = 0; q < 4; ++q) dst[q] = src[q];
                 bool cl;
-                const size_t i = blh(d, b, c0 + t, h);
-                e = token_rate(a.dt[i], a.alpha[i], a.lam[i], log_cap, &cl);
-            } else {
-                uint4 *dst = reinterpret_cast<uint4 *>(xs + t * TPS);
-#pragma unroll
-                for (int q = 0; q < 4; ++q) dst[q] = make_uint4(0, 0, 0, 0);
+                e = token_rate(ndt, nal, nlm, log_cap, &cl);
             }
             e_s[t] = e;
             E_s[t] = block_scan128(double(e), wsum);
         }
+        if (ci + 1 < d.nc) fetch(ci + 1);
         __syncthreads();
         {
             const int t = tid;
             const double Eend = E_s[n - 1];
-            for (int m = 0; m < K; ++m) {
+#pragma unroll
+            for (int m = 0; m < KMAX; ++m) {
+                if (m >= K) break;
                 float cv = 0.f;
                 if (t < n) {
-                    const float wv = to_f(a.W[blh(d, b, c0 + t, h) * K + m]);
                     if (!REV)
-                        cv = -expm1f(-e_s[t] * itau[m]) * wv * expf(-float(Eend - E_s[t]) * itau[m]);
+                        cv = -expm1f(-e_s[t] * itau[m]) * wcur[m] * expf(-float(Eend - E_s[t]) * itau[m]);
                     else
-                        cv = wv * expf(-float(E_s[t]) * itau[m]);
+                        cv = wcur[m] * expf(-float(E_s[t]) * itau[m]);
                 }
                 coef[t * K + m] = cv;
             }
@@ -291,14 +329,17 @@ struct OutSmem {
     __host__ __device__ OutSmem(int K, int N) {
         c_bytes = (N / 64) * 16384;            // C chunk, K-major over n
         b_bytes = (N / 64) * 16384;            // B chunk
-        s_bytes = (N / 64) * (K * TPS * 128);  // S_in rows (m, p), K-major over n
-        total = c_bytes + b_bytes + s_bytes + 2 * 16384 /*Gamma o G*/ + 2 * 4096 /*X^T*/ +
-                TQ * TPS * 2 /*x*/ + TQ * 32 * 4 /*kappa*/ + TQ * 8 /*E*/ + 32 * 4 + 64 + 64 + 64;
+        s_bytes = (N / 64) * (K * TPS * 128);  // S_in rows (m, p) of one P-slice, K-major over n
+        total = c_bytes + b_bytes + s_bytes + 2 * 16384 /*Gamma o G*/ + 2 * 2 * 4096 /*X^T x2*/ +
+                TQ * 64 * 2 /*x*/ + TQ * 32 * 4 /*partial y*/ + TQ * KMAX * 4 /*kappa*/ +
+                TQ * 8 /*E*/ + 32 * 4 + 64 + 64 + 64;
     }
 };
 
 constexpr int kOutThreads = 256;  // two groups of four warps share the 128 TMEM lanes
 
+// One CTA per (b, h, chunk) with headdim 64 = two 32-wide P-slices: Gamma and C B^T are formed
+// once and serve both slices; the second slice's S_in tile is loaded while Gamma is built.
 __global__ void __launch_bounds__(kOutThreads, 1)
     tc_chunk_fwd(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapB,
                  const __grid_constant__ CUtensorMap mapS, OutArgs a) {
@@ -307,31 +348,32 @@ __global__ void __launch_bounds__(kOutThreads, 1)
         reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const ScanDims &d = a.d;
     const int K = d.K, N = d.N, P = d.P;
+    const int nsl = P / TPS;  // P-slices of this head (1 or 2)
     const OutSmem plan(K, N);
     unsigned char *sC = base;
     unsigned char *sB = sC + plan.c_bytes;
     unsigned char *sS = sB + plan.b_bytes;
     unsigned char *sM = sS + plan.s_bytes;          // Gamma o G, [t][k] K-major, 2 atoms
-    unsigned char *sX = sM + 2 * 16384;             // X^T, [p][k] K-major, 2 atoms of 32 rows
-    bf16 *xs = reinterpret_cast<bf16 *>(sX + 2 * 4096);         // [128][32]
-    float *kap_s = reinterpret_cast<float *>(xs + TQ * TPS);     // [128][32]; later partial y
-    float2 *E_s = reinterpret_cast<float2 *>(kap_s + TQ * 32);   // [128] hi / lo pairs
+    unsigned char *sX = sM + 2 * 16384;             // X^T per slice: [p][k] K-major, 2 atoms of 32 rows
+    bf16 *xs = reinterpret_cast<bf16 *>(sX + 2 * 2 * 4096);      // [128][64]
+    float *part = reinterpret_cast<float *>(xs + TQ * 64);       // [32][128] partial y of group 1
+    float *kap_s = part + TQ * 32;                               // [128][KMAX]
+    float2 *E_s = reinterpret_cast<float2 *>(kap_s + TQ * KMAX); // [128] hi / lo pairs
     float *l2t = reinterpret_cast<float *>(E_s + TQ);            // [32] log2(e) / tau
     double *wsum = reinterpret_cast<double *>(l2t + 32);         // [8]
-    uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);     // tma, mma1, mma2
-    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 3);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);     // tma0, tma1, mma G/Z0, Y, Z1
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 5);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
 
     const int tid = threadIdx.x, grp = tid >> 7, t = tid & 127, w4 = (tid >> 5) & 3;
-    const int npart = P / TPS;
-    const int h = blockIdx.x / npart, p0 = (blockIdx.x % npart) * TPS;
-    const int c = blockIdx.y, b = blockIdx.z;
+    const int h = blockIdx.x, c = blockIdx.y, b = blockIdx.z;
     const int g = h / (d.H / d.G);
     const int c0 = c * TQ, n = min(TQ, d.L - c0);
     const uint32_t ZN = uint32_t(K * TPS);  // Z columns: (m, p)
+    const int srow = int(((size_t(b) * d.H + h) * d.nc + c) * K);
 
     if (tid == 0) {
-        for (int i = 0; i < 3; ++i) mbar_init(&bars[i], 1);
+        for (int i = 0; i < 5; ++i) mbar_init(&bars[i], 1);
         *abort_s = 0;
         fence_barrier_init();
     }
@@ -342,16 +384,14 @@ __global__ void __launch_bounds__(kOutThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *tslot;
     const uint32_t lane_base = tmem + (uint32_t(w4 * 32) << 16);
-    const uint32_t colG = 0, colZ = 128, colY = 128 + ZN;
+    const uint32_t colG = 0, colZ = 128, colY = 128 + ZN;  // Y of slice s at colY + 32 s
 
     if (tid == 0) {
-        const uint32_t bytes = uint32_t(plan.c_bytes + plan.b_bytes + plan.s_bytes);
-        mbar_arrive_expect_tx(&bars[0], bytes);
+        mbar_arrive_expect_tx(&bars[0], uint32_t(plan.c_bytes + plan.b_bytes + plan.s_bytes));
         for (int jb = 0; jb < N / 64; ++jb) {
             tma_load_3d(sC + jb * 16384, &mapC, &bars[0], g * N + 64 * jb, c0, b);
             tma_load_3d(sB + jb * 16384, &mapB, &bars[0], g * N + 64 * jb, c0, b);
-            tma_load_3d(sS + jb * (K * TPS * 128), &mapS, &bars[0], 64 * jb, p0,
-                        int(((size_t(b) * d.H + h) * d.nc + c) * K));
+            tma_load_3d(sS + jb * (K * TPS * 128), &mapS, &bars[0], 64 * jb, 0, srow);
         }
     }
     // per-position data of row t (both groups hold it)
@@ -365,15 +405,13 @@ __global__ void __launch_bounds__(kOutThreads, 1)
         bool cl;
         e = token_rate(a.dt[i], a.alpha[i], a.lam[i], log_cap, &cl);
         if (grp == 0) {
-            const uint4 *src = reinterpret_cast<const uint4 *>(a.x + i * P + p0);
-            uint4 *dst = reinterpret_cast<uint4 *>(xs + t * TPS);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) dst[q] = src[q];
+            const uint4 *src = reinterpret_cast<const uint4 *>(a.x + i * P);
+            uint4 *dst = reinterpret_cast<uint4 *>(xs + t * 64);
+            for (int q = 0; q < nsl * 4; ++q) dst[q] = src[q];
         }
     } else if (grp == 0) {
-        uint4 *dst = reinterpret_cast<uint4 *>(xs + t * TPS);
-#pragma unroll
-        for (int q = 0; q < 4; ++q) dst[q] = make_uint4(0, 0, 0, 0);
+        uint4 *dst = reinterpret_cast<uint4 *>(xs + t * 64);
+        for (int q = 0; q < 8; ++q) dst[q] = make_uint4(0, 0, 0, 0);
     }
     const double Et = group_scan128(double(e), wsum);
     const float2 Et2 = split_f2(Et);
@@ -390,44 +428,49 @@ __global__ void __launch_bounds__(kOutThreads, 1)
                 kp = -expm1f(-e * (l2t[m] / kLog2e)) * to_f(a.ww[wi]);
                 f_t[m] = wr_t[m] * ex2_approx(-float(Et) * l2t[m]);
             }
-            if (grp == 0) kap_s[t * 32 + m] = kp;
+            if (grp == 0) kap_s[t * KMAX + m] = kp;
         }
     }
     __syncthreads();
-    // X^T tile: row p, column k = t (K-major, 128-byte swizzle, 32 rows per k-atom)
-    if (grp == 0) {
-        unsigned char *tile = sX + (t >> 6) * 4096;
+    // X^T tiles, one per slice: row p, column k = t (K-major, 128-byte swizzle)
+    if (grp < nsl) {
+        unsigned char *tile = sX + grp * 8192 + (t >> 6) * 4096;
         const int kk = t & 63;
 #pragma unroll
         for (int p = 0; p < TPS; ++p)
-            *reinterpret_cast<bf16 *>(tile + sw128_offset(p, kk)) = xs[t * TPS + p];
+            *reinterpret_cast<bf16 *>(tile + sw128_offset(p, kk)) = xs[t * 64 + grp * TPS + p];
     }
     fence_async_smem();
     __syncthreads();
-    // G = C B^T and Z = C S_in^T
+    const uint32_t idZ = idesc_bf16(128, int(ZN), false, false);
+    // G = C B^T and Z = C S_in^T (slice 0)
     if (tid == 0) {
         if (!mbar_wait(&bars[0], 0)) {
             *abort_s = 1;
         } else {
             tc_fence_after();
             const uint32_t idG = idesc_bf16(128, 128, false, false);
-            const uint32_t idZ = idesc_bf16(128, int(ZN), false, false);
             for (int ks = 0; ks < N / 16; ++ks) {
                 const uint32_t koff = (ks / 4) * 16384 + (ks % 4) * 32;
                 const uint64_t ad = desc_sw128(smem_u32(sC) + koff, 16, 1024);
-                const uint64_t bdB = desc_sw128(smem_u32(sB) + koff, 16, 1024);
-                const uint64_t bdS =
-                    desc_sw128(smem_u32(sS) + (ks / 4) * (K * TPS * 128) + (ks % 4) * 32, 16, 1024);
-                mma_bf16(tmem + colG, ad, bdB, idG, ks > 0);
-                mma_bf16(tmem + colZ, ad, bdS, idZ, ks > 0);
+                mma_bf16(tmem + colG, ad, desc_sw128(smem_u32(sB) + koff, 16, 1024), idG, ks > 0);
+                mma_bf16(tmem + colZ, ad,
+                         desc_sw128(smem_u32(sS) + (ks / 4) * (K * TPS * 128) + (ks % 4) * 32, 16, 1024),
+                         idZ, ks > 0);
             }
-            mma_commit(&bars[1]);
+            mma_commit(&bars[2]);
         }
     }
     __syncthreads();
-    if (!*abort_s && !mbar_wait(&bars[1], 0)) *abort_s = 1;
+    if (!*abort_s && !mbar_wait(&bars[2], 0)) *abort_s = 1;
     __syncthreads();
     tc_fence_after();
+    // the S_in tile of slice 1 streams in while Gamma is formed
+    if (tid == 0 && !*abort_s && nsl > 1) {
+        mbar_arrive_expect_tx(&bars[1], uint32_t(plan.s_bytes));
+        for (int jb = 0; jb < N / 64; ++jb)
+            tma_load_3d(sS + jb * (K * TPS * 128), &mapS, &bars[1], 64 * jb, TPS, srow);
+    }
     if (!*abort_s) {
         // row t of Gamma o G -> bf16, K-major [t][k]; group 0 takes k in [0,32) and [96,128),
         // group 1 takes [32,96) (the causal triangle splits about evenly)
@@ -445,7 +488,7 @@ __global__ void __launch_bounds__(kOutThreads, 1)
                     float gam = 0.f;
 #pragma unroll
                     for (int m = 0; m < KMAX; ++m)
-                        if (m < K) gam = fmaf(wr_t[m] * kap_s[k * 32 + m], ex2_approx(-dE * l2t[m]), gam);
+                        if (m < K) gam = fmaf(wr_t[m] * kap_s[k * KMAX + m], ex2_approx(-dE * l2t[m]), gam);
                     v = gam * gv[kk];
                 }
                 gv[kk] = v;
@@ -464,63 +507,88 @@ __global__ void __launch_bounds__(kOutThreads, 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (tid == 0 && !*abort_s) {
+    if (tid == 0 && !*abort_s) {  // Y_s = (Gamma o G) X_s for every slice
         const uint32_t idY = idesc_bf16(128, TPS, false, false);
-        for (int ks = 0; ks < TQ / 16; ++ks) {
-            const uint64_t ad = desc_sw128(smem_u32(sM) + (ks / 4) * 16384 + (ks % 4) * 32, 16, 1024);
-            const uint64_t bd = desc_sw128(smem_u32(sX) + (ks / 4) * 4096 + (ks % 4) * 32, 16, 1024);
-            mma_bf16(tmem + colY, ad, bd, idY, ks > 0);
-        }
-        mma_commit(&bars[2]);
+        for (int sl = 0; sl < nsl; ++sl)
+            for (int ks = 0; ks < TQ / 16; ++ks) {
+                const uint64_t ad = desc_sw128(smem_u32(sM) + (ks / 4) * 16384 + (ks % 4) * 32, 16, 1024);
+                const uint64_t bd = desc_sw128(smem_u32(sX) + sl * 8192 + (ks / 4) * 4096 + (ks % 4) * 32, 16, 1024);
+                mma_bf16(tmem + colY + 32 * sl, ad, bd, idY, ks > 0);
+            }
+        mma_commit(&bars[3]);
     }
-    // mode-weighted readout of Z: group g takes modes [g K/2, (g+1) K/2)
-    float acc[32];
-#pragma unroll
-    for (int p = 0; p < 32; ++p) acc[p] = 0.f;
-    if (!*abort_s) {
-        const int m0 = grp * (K / 2);
-#pragma unroll
-        for (int mm = 0; mm < KMAX / 2; ++mm) {
-            if (mm >= K / 2) break;
-            const int m = m0 + mm;
-            float z[32];
-            tmem_ld32(lane_base + colZ + m * TPS, z);
-            tmem_ld_wait();
-            float fm = 0.f;
-#pragma unroll
-            for (int q = 0; q < KMAX; ++q)
-                if (q == m) fm = f_t[q];
-#pragma unroll
-            for (int p = 0; p < 32; ++p) acc[p] = fmaf(fm, z[p], acc[p]);
-        }
-    }
-    __syncthreads();  // kap_s is no longer read: reuse it for group 1's partial sums
-    float *part = kap_s;  // [32][128], column-major in t
-    if (grp == 1) {
-#pragma unroll
-        for (int p = 0; p < 32; ++p) part[p * TQ + t] = acc[p];
-    }
-    __syncthreads();
-    if (!*abort_s && !mbar_wait(&bars[2], 0)) *abort_s = 1;
-    __syncthreads();
-    tc_fence_after();
-    if (!*abort_s && grp == 0) {
-        float yi[32];
-        tmem_ld32(lane_base + colY, yi);
-        tmem_ld_wait();
-        if (t < n) {
-            const float Dh = a.D[h];
-            uint4 *o = reinterpret_cast<uint4 *>(a.y + blh(d, b, c0 + t, h) * P + p0);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                float v[8];
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int p = 8 * q + i;
-                    v[i] = acc[p] + part[p * TQ + t] + yi[p] + Dh * __bfloat162float(xs[t * TPS + p]);
+    const float Dh = a.D[h];
+    for (int sl = 0; sl < nsl; ++sl) {
+        if (sl == 1) {  // Z of slice 1 once its tile has arrived and Z of slice 0 has been read
+            tc_fence_before();
+            __syncthreads();
+            tc_fence_after();
+            if (tid == 0 && !*abort_s) {
+                if (!mbar_wait(&bars[1], 0)) {
+                    *abort_s = 1;
+                } else {
+                    tc_fence_after();
+                    for (int ks = 0; ks < N / 16; ++ks) {
+                        const uint32_t koff = (ks / 4) * 16384 + (ks % 4) * 32;
+                        mma_bf16(tmem + colZ, desc_sw128(smem_u32(sC) + koff, 16, 1024),
+                                 desc_sw128(smem_u32(sS) + (ks / 4) * (K * TPS * 128) + (ks % 4) * 32, 16, 1024),
+                                 idZ, ks > 0);
+                    }
+                    mma_commit(&bars[4]);
                 }
-                o[q] = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]),
-                                  pack_bf16x2(v[6], v[7]));
+            }
+            __syncthreads();
+            if (!*abort_s && !mbar_wait(&bars[4], 0)) *abort_s = 1;
+            __syncthreads();
+            tc_fence_after();
+        }
+        // mode-weighted readout of Z: group g takes modes [g K/2, (g+1) K/2)
+        float acc[32];
+#pragma unroll
+        for (int p = 0; p < 32; ++p) acc[p] = 0.f;
+        if (!*abort_s) {
+            const int m0 = grp * (K / 2);
+#pragma unroll
+            for (int mm = 0; mm < KMAX / 2; ++mm) {
+                if (mm >= K / 2) break;
+                const int m = m0 + mm;
+                float z[32];
+                tmem_ld32(lane_base + colZ + m * TPS, z);
+                tmem_ld_wait();
+                float fm = 0.f;
+#pragma unroll
+                for (int q = 0; q < KMAX; ++q)
+                    if (q == m) fm = f_t[q];
+#pragma unroll
+                for (int p = 0; p < 32; ++p) acc[p] = fmaf(fm, z[p], acc[p]);
+            }
+        }
+        if (grp == 1) {
+#pragma unroll
+            for (int p = 0; p < 32; ++p) part[p * TQ + t] = acc[p];
+        }
+        __syncthreads();
+        if (sl == 0 && !*abort_s && !mbar_wait(&bars[3], 0)) *abort_s = 1;
+        __syncthreads();
+        tc_fence_after();
+        if (!*abort_s && grp == 0) {
+            float yi[32];
+            tmem_ld32(lane_base + colY + 32 * sl, yi);
+            tmem_ld_wait();
+            if (t < n) {
+                uint4 *o = reinterpret_cast<uint4 *>(a.y + blh(d, b, c0 + t, h) * P + sl * TPS);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    float v[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const int p = 8 * q + i;
+                        v[i] = acc[p] + part[p * TQ + t] + yi[p] +
+                               Dh * __bfloat162float(xs[t * 64 + sl * TPS + p]);
+                    }
+                    o[q] = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]),
+                                      pack_bf16x2(v[6], v[7]));
+                }
             }
         }
     }
@@ -568,7 +636,7 @@ bool tc_make_map3(CUtensorMap *m, const void *ptr, uint64_t d0, uint64_t d1, uin
 
 bool tc_supported(const ScanDims &d, int dtype) {
     if (dtype != 1) return false;
-    if (d.P % TPS || (d.N != 64 && d.N != 128) || (d.K != 4 && d.K != 8)) return false;
+    if ((d.P != 32 && d.P != 64) || (d.N != 64 && d.N != 128) || (d.K != 4 && d.K != 8)) return false;
     return true;
 }
 
@@ -636,7 +704,7 @@ cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, int *e
     a.err = err;
     const size_t smem = OutSmem(d.K, d.N).total + 1024;
     cudaFuncSetAttribute(tc_chunk_fwd, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-    dim3 grid(d.H * (d.P / TPS), d.nc, d.B);
+    dim3 grid(d.H, d.nc, d.B);
     trace_begin("chunk_fwd_tc", st);
     tc_chunk_fwd<<<grid, kOutThreads, smem, st>>>(mapC, mapB, mapS, a);
     trace_end(st);

@@ -279,10 +279,14 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     float dk[KMAX];
 #pragma unroll
     for (int m = 0; m < KMAX; ++m) dk[m] = 0.f;
-    if (!*abort_s && t < n) {
+    if (!*abort_s) {
+        // all lanes of a warp walk the same rows tt (broadcast loads of E, w_read); rows above the
+        // diagonal (tt < k) contribute nothing
         const int k = t;
         const float2 Ek = E_s[k];
-        for (int tt = k + grp; tt < n; tt += 2) {
+        // group grp takes the rows of parity grp, starting at this warp's first column
+        for (int tt = (t & ~31) + grp; tt < n; tt += 2) {
+            if (tt < k) continue;
             const float dE = diff_f2(E_s[tt], Ek);
             const float gh = GHs[tt * XS + k];
 #pragma unroll
@@ -440,6 +444,32 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             mma_commit(&bars[1]);
         }
+    }
+    // <dS_out, S_in> of this P-slice per mode, straight from the two tiles in shared memory (both
+    // carry the same swizzle, so the byte-for-byte dot product is the element dot product);
+    // it runs while the tensor cores work
+    if (mbar_wait(&bars[0], 0)) {
+        const int tpm = kThreads / K;  // threads per mode
+        const int m = tid / tpm, jl = tid % tpm;
+        float acc = 0.f;
+        for (int jb = 0; jb < N / 64; ++jb) {
+            const uint4 *ps = reinterpret_cast<const uint4 *>(sS + jb * (K * TPS * 128) + m * 4096);
+            const uint4 *pd = reinterpret_cast<const uint4 *>(sD + jb * (K * TPS * 128) + m * 4096);
+            for (int q = jl; q < 256; q += tpm) {
+                const uint4 u = ps[q], v = pd[q];
+                const __nv_bfloat162 *a2 = reinterpret_cast<const __nv_bfloat162 *>(&u);
+                const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(&v);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const float2 fa = __bfloat1622float2(a2[i]), fb = __bfloat1622float2(b2[i]);
+                    acc = fmaf(fa.x, fb.x, fmaf(fa.y, fb.y, acc));
+                }
+            }
+        }
+        for (int o = tpm >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        if (jl == 0) atomicAdd(a.cdot + ((size_t(b) * d.H + h) * d.nc + c) * K + m, acc);
+    } else {
+        *abort_s = 1;
     }
     __syncthreads();
     if (!*abort_s && !mbar_wait(&bars[1], 0)) *abort_s = 1;
@@ -828,7 +858,7 @@ size_t tc_bwd_workspace_bytes(const ScanDims &d, TcBwdWorkspace *l, char *base) 
 }
 
 cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspace &ws, int *err,
-                        cudaStream_t st) {
+                        bool reuse_states, cudaStream_t st) {
     cudaError_t e;
     const size_t ngn = size_t(d.B) * d.L * d.G * d.N;
     const size_t blh_ = size_t(d.B) * d.L * d.H;
@@ -838,11 +868,12 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
     if ((e = cudaMemsetAsync(ws.cdot, 0, sizeof(float) * d.B * d.H * d.nc * d.K, st))) return e;
     if ((e = cudaMemsetAsync(ws.ab_acc, 0, sizeof(float) * blh_ * 2, st))) return e;
     if ((e = cudaMemsetAsync(ws.mh_total, 0, sizeof(float) * d.B * d.nc * TQ * TQ, st))) return e;
-    if ((e = tc_state_pass_launch(d, false, p.x, p.Bm, p.ww, p.dt, p.alpha, p.lam, p.tau, p.h0,
+    if (!reuse_states &&
+        (e = tc_state_pass_launch(d, false, p.x, p.Bm, p.ww, p.dt, p.alpha, p.lam, p.tau, p.h0,
                                   ws.S_in, nullptr, nullptr, nullptr, err, st)))
         return e;
     if ((e = tc_state_pass_launch(d, true, p.dy, p.Cm, p.wr, p.dt, p.alpha, p.lam, p.tau,
-                                  p.dh_final, ws.dS_out, p.dh0, ws.S_in, ws.cdot, err, st)))
+                                  p.dh_final, ws.dS_out, p.dh0, nullptr, nullptr, err, st)))
         return e;
     if (d.nc == 0) return cudaSuccess;
     const uint64_t GN = uint64_t(d.G) * d.N, HP = uint64_t(d.H) * d.P;

@@ -238,3 +238,22 @@ def test_bwd_bf16_paper_like_lambda_alpha_extremes():
     gr = _ora_bwd(f64_inputs(host))
     for k in GRADS:
         assert_close(k, to_host64(g[k]), gr[k], 1e-2)
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_bwd_reusing_forward_states(dtype):
+    """The backward may take the per-chunk states the forward left in a shared workspace."""
+    from paper_2609_36314_gb300 import bwd_workspace_size, fwd_workspace_size, make_dims
+    s = synth.Shape(2, 260, 4, 64, 1, 64, 8, 0, dtype)
+    host = synth.make_scan_inputs(s, seed=44, with_dy=True, with_h0=True)
+    dv = dev_inputs(host)
+    tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
+    dims = make_dims(2, 260, 4, 64, 1, 64, 8, tdt)
+    ws = torch.empty(max(bwd_workspace_size(dims), fwd_workspace_size(dims)), dtype=torch.uint8,
+                     device="cuda")
+    _gpu_fwd(dv, workspace=ws)
+    g = _gpu_bwd(dv, workspace=ws, reuse_fwd_states=True)
+    g_ref = _gpu_bwd(dv)
+    torch.cuda.synchronize()
+    for k in GRADS:
+        assert torch.equal(g[k], g_ref[k]) or synth.rel_l2(to_host64(g[k]), to_host64(g_ref[k])) < 1e-6, k
