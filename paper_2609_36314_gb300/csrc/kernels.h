@@ -50,7 +50,7 @@ cudaError_t simt_scan_bwd(const ScanDims &d, int dtype, const ScanPtrs &p, void 
                           void *dS_out, float *dB_acc, float *dC_acc, bool reuse_states,
                           cudaStream_t st);
 
-// Tensor-core (tcgen05) path: bf16 inputs, chunk 128, P in {32, 64}, N in {64, 128}, K in {4, 8}.
+// Tensor-core (tcgen05) path: bf16 inputs, chunk 128, P = 64, N in {64, 128}, K in {4, 8}.
 bool tc_supported(const ScanDims &d, int dtype);
 size_t tc_state_elems(const ScanDims &d);  // bf16 elements of the per-chunk state workspace
 cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, int *err,
@@ -70,7 +70,7 @@ bool tc_bwd_supported(const ScanDims &d, int dtype);
 struct TcBwdWorkspace {
     void *S_in, *dS_out;                     // bf16 per-chunk states
     float *dx_acc, *dwr_acc, *dkap_acc;      // [B,L,H,P], [B,L,H,K] x 2
-    float *ab_acc, *rect, *cdot, *mh_total;  // [B,L,H,2], [B,L,H], [B,H,nc,K], [B,nc,Q,Q]
+    float *ab_acc, *rect, *cdot, *mh_total;  // [B,L,H,2], [B,L,H], [B,H,nc,K], [B,nc,G,Q,Q]
     float *dB_acc, *dC_acc;                  // [B,L,G,N] x 2
 };
 size_t tc_bwd_workspace_bytes(const ScanDims &d, TcBwdWorkspace *layout, char *base);

@@ -10,10 +10,11 @@
 //        S_m += sum_k s_{k,m} x_k B_k^T  as  D[(m,p), n] += A[(m,p), k] * B[k, n]
 //        (A = s o x generated in shared memory, B = the chunk of B loaded by TMA).
 //        Run over the chunks in reverse with (dy, C, f) it carries dS for the backward.
-//   tc_chunk_fwd   (chunk-parallel; one CTA per (b, c, h, 32-wide slice of P)):
-//        G = C B^T and Z = C S_in^T on the tensor cores (TMA-fed), then each thread owns one
-//        position t: Gamma_{t,k} G_{t,k} -> bf16 tile, Y_intra = (Gamma o G) X on the tensor
-//        cores, and y_t = sum_m f_{t,m} Z[t, (m, p)] + Y_intra + D x_t.
+//   tc_chunk_fwd   (chunk-parallel; one CTA per (b, c, h), headdim 64):
+//        G = C B^T on the tensor cores, Gamma_{t,k} G_{t,k} per position pair -> bf16 tile,
+//        then one TMEM accumulator Y[t, p] collects (Gamma o G) X and sum_m (f_m o C) S_in,m^T
+//        (K = (mode, n) in 64-wide steps, S_in tiles by TMA, f o C tiles written by the
+//        threads), and y = Y + D x.
 //
 // All mbarrier waits are bounded (a few seconds); on a timeout the kernel records
 // FRAC_ERR_TIMEOUT in the error word, stops issuing work, frees its tensor memory and exits.
@@ -95,7 +96,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         fence_barrier_init();
     }
     if (tid < K) itau[tid] = 1.f / a.tau[h * K + tid];
-    if (w == 0) tmem_alloc(tslot, ncols);
+    if (w == 0) tmem_alloc_once(tslot, ncols);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -318,132 +319,161 @@ __global__ void __launch_bounds__(kThreads, 2)
 // ---------------------------------------------------------------------------------------------
 struct OutArgs {
     ScanDims d;
-    const bf16 *x, *wr, *ww;
+    const bf16 *wr, *ww;
     const float *dt, *alpha, *lam, *tau, *D;
     bf16 *y;
     int *err;
 };
 
+constexpr int kOutThreads = 256;  // two groups of four warps share the 128 TMEM lanes
+constexpr int kSBuf = 3;          // S_in tiles in flight
+
+// Shared-memory plan of tc_chunk_fwd (offsets from a 1024-aligned base): about 110 KB at
+// N = 128, so that two CTAs share an SM.
 struct OutSmem {
-    int c_bytes, b_bytes, s_bytes, total;
-    __host__ __device__ OutSmem(int K, int N) {
-        c_bytes = (N / 64) * 16384;            // C chunk, K-major over n
-        b_bytes = (N / 64) * 16384;            // B chunk
-        s_bytes = (N / 64) * (K * TPS * 128);  // S_in rows (m, p) of one P-slice, K-major over n
-        total = c_bytes + b_bytes + s_bytes + 2 * 16384 /*Gamma o G*/ + 2 * 2 * 4096 /*X^T x2*/ +
-                TQ * 64 * 2 /*x*/ + TQ * 32 * 4 /*partial y*/ + TQ * KMAX * 4 /*kappa*/ +
-                TQ * 8 /*E*/ + 32 * 4 + 64 + 64 + 64;
+    int c, m, x, s, total;
+    __host__ __device__ explicit OutSmem(int N) {
+        c = (N / 64) * 16384;  // C chunk [t][n], K-major, 64-wide n atoms
+        m = 2 * 16384;         // B chunk, then Gamma o G [t][k], then two (f o C) tiles
+        x = 16384;             // x chunk [t][p]: the MN-major operand of the intra MMA
+        s = kSBuf * 8192;      // S_in tiles, one (mode, 64-wide n half) each: [p][n]
+        total = c + m + x + s + TQ * KMAX * 4 /*kappa*/ + TQ * 8 /*E*/ + 64 * 4 /*tau, l2t*/ +
+                64 /*wsum*/ + 8 * 8 /*bars*/ + 16;
     }
 };
 
-constexpr int kOutThreads = 256;  // two groups of four warps share the 128 TMEM lanes
+__device__ __forceinline__ void load_weights(const bf16 *src, int K, float *w) {
+    if (K == 8) {
+        const uint4 u = *reinterpret_cast<const uint4 *>(src);
+        const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&u);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float2 f = __bfloat1622float2(h2[q]);
+            w[2 * q] = f.x;
+            w[2 * q + 1] = f.y;
+        }
+    } else {  // K == 4
+        const uint2 u = *reinterpret_cast<const uint2 *>(src);
+        const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&u);
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const float2 f = __bfloat1622float2(h2[q]);
+            w[2 * q] = f.x;
+            w[2 * q + 1] = f.y;
+        }
+#pragma unroll
+        for (int m = 4; m < KMAX; ++m) w[m] = 0.f;
+    }
+}
 
-// One CTA per (b, h, chunk) with headdim 64 = two 32-wide P-slices: Gamma and C B^T are formed
-// once and serve both slices; the second slice's S_in tile is loaded while Gamma is built.
-__global__ void __launch_bounds__(kOutThreads, 1)
+// One CTA per (b, h, chunk), headdim 64, all in one TMEM accumulator Y[t, p]:
+//   Y  = (Gamma o C B^T) X                      (intra-chunk pairs, K = t)
+//   Y += sum_m (f_m o C) S_in,m^T               (entering state, K = (m, n), 64-wide n steps)
+//   y  = Y + D x
+// G = C B^T comes from the tensor cores; Gamma is formed per position pair; the scaled copies
+// f_m o C are written by the threads into two alternating tiles while the tensor cores consume
+// the previous one, and the S_in tiles stream in by TMA three steps ahead.
+__global__ void __launch_bounds__(kOutThreads, 2)
     tc_chunk_fwd(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapB,
-                 const __grid_constant__ CUtensorMap mapS, OutArgs a) {
+                 const __grid_constant__ CUtensorMap mapX, const __grid_constant__ CUtensorMap mapS,
+                 OutArgs a) {
     extern __shared__ unsigned char smem_raw[];
     unsigned char *base =
         reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const ScanDims &d = a.d;
     const int K = d.K, N = d.N, P = d.P;
-    const int nsl = P / TPS;  // P-slices of this head (1 or 2)
-    const OutSmem plan(K, N);
+    const OutSmem plan(N);
     unsigned char *sC = base;
-    unsigned char *sB = sC + plan.c_bytes;
-    unsigned char *sS = sB + plan.b_bytes;
-    unsigned char *sM = sS + plan.s_bytes;          // Gamma o G, [t][k] K-major, 2 atoms
-    unsigned char *sX = sM + 2 * 16384;             // X^T per slice: [p][k] K-major, 2 atoms of 32 rows
-    bf16 *xs = reinterpret_cast<bf16 *>(sX + 2 * 2 * 4096);      // [128][64]
-    float *part = reinterpret_cast<float *>(xs + TQ * 64);       // [32][128] partial y of group 1
-    float *kap_s = part + TQ * 32;                               // [128][KMAX]
-    float2 *E_s = reinterpret_cast<float2 *>(kap_s + TQ * KMAX); // [128] hi / lo pairs
-    float *l2t = reinterpret_cast<float *>(E_s + TQ);            // [32] log2(e) / tau
-    double *wsum = reinterpret_cast<double *>(l2t + 32);         // [8]
-    uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);     // tma0, tma1, mma G/Z0, Y, Z1
-    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 5);
+    unsigned char *sM = sC + plan.c;
+    unsigned char *sX = sM + plan.m;
+    unsigned char *sS = sX + plan.x;
+    float *kap_s = reinterpret_cast<float *>(sS + plan.s);      // [128][KMAX]
+    float2 *E_s = reinterpret_cast<float2 *>(kap_s + TQ * KMAX);  // [128] hi / lo pairs
+    float *tau_s = reinterpret_cast<float *>(E_s + TQ);           // [32]
+    float *l2t = tau_s + 32;                                      // [32] log2(e) / tau
+    double *wsum = reinterpret_cast<double *>(l2t + 32);          // [8]
+    // bars: 0 C, B, x loaded | 1 G done | 2 intra Y done | 3..5 S tile loaded | 6, 7 (f o C) tile consumed
+    uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 8);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
 
     const int tid = threadIdx.x, grp = tid >> 7, t = tid & 127, w4 = (tid >> 5) & 3;
     const int h = blockIdx.x, c = blockIdx.y, b = blockIdx.z;
     const int g = h / (d.H / d.G);
     const int c0 = c * TQ, n = min(TQ, d.L - c0);
-    const uint32_t ZN = uint32_t(K * TPS);  // Z columns: (m, p)
+    const int nhalf = N / 64, niter = K * nhalf;
     const int srow = int(((size_t(b) * d.H + h) * d.nc + c) * K);
 
     if (tid == 0) {
-        for (int i = 0; i < 5; ++i) mbar_init(&bars[i], 1);
+        for (int i = 0; i < 8; ++i) mbar_init(&bars[i], 1);
         *abort_s = 0;
         fence_barrier_init();
     }
-    if (tid < K) l2t[tid] = kLog2e / a.tau[h * K + tid];
-    if (tid < 32) tmem_alloc(tslot, 512);
+    if (tid < K) {
+        const float tv = a.tau[h * K + tid];
+        tau_s[tid] = tv;
+        l2t[tid] = kLog2e / tv;
+    }
+    if (tid < 32) tmem_alloc_once(tslot, 256);
+    // per-position inputs of row t, all loads issued before anything waits on them
+    float dtv = 1.f, alv = 1.f, lmv = 1.f;
+    float wr_t[KMAX], ww_t[KMAX];
+    if (t < n) {
+        const size_t i = blh(d, b, c0 + t, h);
+        dtv = a.dt[i];
+        alv = a.alpha[i];
+        lmv = a.lam[i];
+        load_weights(a.wr + i * K, K, wr_t);
+        load_weights(a.ww + i * K, K, ww_t);
+    } else {
+#pragma unroll
+        for (int m = 0; m < KMAX; ++m) wr_t[m] = ww_t[m] = 0.f;
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tslot;
     const uint32_t lane_base = tmem + (uint32_t(w4 * 32) << 16);
-    const uint32_t colG = 0, colZ = 128, colY = 128 + ZN;  // Y of slice s at colY + 32 s
+    constexpr uint32_t colG = 0, colY = 128;
 
     if (tid == 0) {
-        mbar_arrive_expect_tx(&bars[0], uint32_t(plan.c_bytes + plan.b_bytes + plan.s_bytes));
-        for (int jb = 0; jb < N / 64; ++jb) {
+        mbar_arrive_expect_tx(&bars[0], uint32_t(2 * plan.c + plan.x));
+        for (int jb = 0; jb < nhalf; ++jb) {
             tma_load_3d(sC + jb * 16384, &mapC, &bars[0], g * N + 64 * jb, c0, b);
-            tma_load_3d(sB + jb * 16384, &mapB, &bars[0], g * N + 64 * jb, c0, b);
-            tma_load_3d(sS + jb * (K * TPS * 128), &mapS, &bars[0], 64 * jb, 0, srow);
+            tma_load_3d(sM + jb * 16384, &mapB, &bars[0], g * N + 64 * jb, c0, b);
+        }
+        tma_load_3d(sX, &mapX, &bars[0], h * P, c0, b);
+        for (int j = 0; j < min(kSBuf, niter); ++j) {
+            mbar_arrive_expect_tx(&bars[3 + j], 8192u);
+            tma_load_3d(sS + j * 8192, &mapS, &bars[3 + j], (j % nhalf) * 64, 0, srow + j / nhalf);
         }
     }
-    // per-position data of row t (both groups hold it)
     float tmax = 0.f;
-    for (int m = 0; m < K; ++m) tmax = fmaxf(tmax, a.tau[h * K + m]);
+    for (int m = 0; m < K; ++m) tmax = fmaxf(tmax, tau_s[m]);
     const float log_cap = logf(64.f * tmax);
     float e = 0.f;
-    float wr_t[KMAX], f_t[KMAX];
     if (t < n) {
-        const size_t i = blh(d, b, c0 + t, h);
         bool cl;
-        e = token_rate(a.dt[i], a.alpha[i], a.lam[i], log_cap, &cl);
-        if (grp == 0) {
-            const uint4 *src = reinterpret_cast<const uint4 *>(a.x + i * P);
-            uint4 *dst = reinterpret_cast<uint4 *>(xs + t * 64);
-            for (int q = 0; q < nsl * 4; ++q) dst[q] = src[q];
-        }
-    } else if (grp == 0) {
-        uint4 *dst = reinterpret_cast<uint4 *>(xs + t * 64);
-        for (int q = 0; q < 8; ++q) dst[q] = make_uint4(0, 0, 0, 0);
+        e = token_rate(dtv, alv, lmv, log_cap, &cl);
     }
     const double Et = group_scan128(double(e), wsum);
     const float2 Et2 = split_f2(Et);
     if (grp == 0) E_s[t] = Et2;
+    float f_t[KMAX];
 #pragma unroll
     for (int m = 0; m < KMAX; ++m) {
-        wr_t[m] = 0.f;
         f_t[m] = 0.f;
         if (m < K) {
             float kp = 0.f;
             if (t < n) {
-                const size_t wi = blh(d, b, c0 + t, h) * K + m;
-                wr_t[m] = to_f(a.wr[wi]);
-                kp = -expm1f(-e * (l2t[m] / kLog2e)) * to_f(a.ww[wi]);
+                kp = -expm1f(-e / tau_s[m]) * ww_t[m];
                 f_t[m] = wr_t[m] * ex2_approx(-float(Et) * l2t[m]);
             }
             if (grp == 0) kap_s[t * KMAX + m] = kp;
         }
     }
     __syncthreads();
-    // X^T tiles, one per slice: row p, column k = t (K-major, 128-byte swizzle)
-    if (grp < nsl) {
-        unsigned char *tile = sX + grp * 8192 + (t >> 6) * 4096;
-        const int kk = t & 63;
-#pragma unroll
-        for (int p = 0; p < TPS; ++p)
-            *reinterpret_cast<bf16 *>(tile + sw128_offset(p, kk)) = xs[t * 64 + grp * TPS + p];
-    }
-    fence_async_smem();
-    __syncthreads();
-    const uint32_t idZ = idesc_bf16(128, int(ZN), false, false);
-    // G = C B^T and Z = C S_in^T (slice 0)
+    // G = C B^T
     if (tid == 0) {
         if (!mbar_wait(&bars[0], 0)) {
             *abort_s = 1;
@@ -452,28 +482,19 @@ __global__ void __launch_bounds__(kOutThreads, 1)
             const uint32_t idG = idesc_bf16(128, 128, false, false);
             for (int ks = 0; ks < N / 16; ++ks) {
                 const uint32_t koff = (ks / 4) * 16384 + (ks % 4) * 32;
-                const uint64_t ad = desc_sw128(smem_u32(sC) + koff, 16, 1024);
-                mma_bf16(tmem + colG, ad, desc_sw128(smem_u32(sB) + koff, 16, 1024), idG, ks > 0);
-                mma_bf16(tmem + colZ, ad,
-                         desc_sw128(smem_u32(sS) + (ks / 4) * (K * TPS * 128) + (ks % 4) * 32, 16, 1024),
-                         idZ, ks > 0);
+                mma_bf16(tmem + colG, desc_sw128(smem_u32(sC) + koff, 16, 1024),
+                         desc_sw128(smem_u32(sM) + koff, 16, 1024), idG, ks > 0);
             }
-            mma_commit(&bars[2]);
+            mma_commit(&bars[1]);
         }
     }
     __syncthreads();
-    if (!*abort_s && !mbar_wait(&bars[2], 0)) *abort_s = 1;
+    if (!*abort_s && !mbar_wait(&bars[1], 0)) *abort_s = 1;
     __syncthreads();
     tc_fence_after();
-    // the S_in tile of slice 1 streams in while Gamma is formed
-    if (tid == 0 && !*abort_s && nsl > 1) {
-        mbar_arrive_expect_tx(&bars[1], uint32_t(plan.s_bytes));
-        for (int jb = 0; jb < N / 64; ++jb)
-            tma_load_3d(sS + jb * (K * TPS * 128), &mapS, &bars[1], 64 * jb, TPS, srow);
-    }
     if (!*abort_s) {
-        // row t of Gamma o G -> bf16, K-major [t][k]; group 0 takes k in [0,32) and [96,128),
-        // group 1 takes [32,96) (the causal triangle splits about evenly)
+        // row t of Gamma o G -> bf16, K-major [t][k] over the B tile; group 0 takes k in [0,32)
+        // and [96,128), group 1 takes [32,96) (the causal triangle splits about evenly)
         for (int half = 0; half < 2; ++half) {
             const int k32 = grp == 0 ? (half == 0 ? 0 : 96) : (half == 0 ? 32 : 64);
             float gv[32];
@@ -507,95 +528,95 @@ __global__ void __launch_bounds__(kOutThreads, 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (tid == 0 && !*abort_s) {  // Y_s = (Gamma o G) X_s for every slice
-        const uint32_t idY = idesc_bf16(128, TPS, false, false);
-        for (int sl = 0; sl < nsl; ++sl)
-            for (int ks = 0; ks < TQ / 16; ++ks) {
-                const uint64_t ad = desc_sw128(smem_u32(sM) + (ks / 4) * 16384 + (ks % 4) * 32, 16, 1024);
-                const uint64_t bd = desc_sw128(smem_u32(sX) + sl * 8192 + (ks / 4) * 4096 + (ks % 4) * 32, 16, 1024);
-                mma_bf16(tmem + colY + 32 * sl, ad, bd, idY, ks > 0);
-            }
-        mma_commit(&bars[3]);
+    if (tid == 0 && !*abort_s) {  // Y = (Gamma o G) X: M = t, N = p, K = k
+        const uint32_t idY = idesc_bf16(128, 64, false, true);
+        for (int ks = 0; ks < TQ / 16; ++ks)
+            mma_bf16(tmem + colY, desc_sw128(smem_u32(sM) + (ks / 4) * 16384 + (ks % 4) * 32, 16, 1024),
+                     desc_sw128(smem_u32(sX) + ks * 2048, 16384, 1024), idY, ks > 0);
+        mma_commit(&bars[2]);
     }
-    const float Dh = a.D[h];
-    for (int sl = 0; sl < nsl; ++sl) {
-        if (sl == 1) {  // Z of slice 1 once its tile has arrived and Z of slice 0 has been read
-            tc_fence_before();
-            __syncthreads();
-            tc_fence_after();
-            if (tid == 0 && !*abort_s) {
-                if (!mbar_wait(&bars[1], 0)) {
-                    *abort_s = 1;
-                } else {
-                    tc_fence_after();
-                    for (int ks = 0; ks < N / 16; ++ks) {
-                        const uint32_t koff = (ks / 4) * 16384 + (ks % 4) * 32;
-                        mma_bf16(tmem + colZ, desc_sw128(smem_u32(sC) + koff, 16, 1024),
-                                 desc_sw128(smem_u32(sS) + (ks / 4) * (K * TPS * 128) + (ks % 4) * 32, 16, 1024),
-                                 idZ, ks > 0);
-                    }
-                    mma_commit(&bars[4]);
-                }
-            }
-            __syncthreads();
-            if (!*abort_s && !mbar_wait(&bars[4], 0)) *abort_s = 1;
-            __syncthreads();
-            tc_fence_after();
-        }
-        // mode-weighted readout of Z: group g takes modes [g K/2, (g+1) K/2)
-        float acc[32];
-#pragma unroll
-        for (int p = 0; p < 32; ++p) acc[p] = 0.f;
-        if (!*abort_s) {
-            const int m0 = grp * (K / 2);
-#pragma unroll
-            for (int mm = 0; mm < KMAX / 2; ++mm) {
-                if (mm >= K / 2) break;
-                const int m = m0 + mm;
-                float z[32];
-                tmem_ld32(lane_base + colZ + m * TPS, z);
-                tmem_ld_wait();
-                float fm = 0.f;
-#pragma unroll
-                for (int q = 0; q < KMAX; ++q)
-                    if (q == m) fm = f_t[q];
-#pragma unroll
-                for (int p = 0; p < 32; ++p) acc[p] = fmaf(fm, z[p], acc[p]);
+    // the (f o C) tiles take the place of Gamma o G once the intra MMA has read it
+    if (!*abort_s && !mbar_wait(&bars[2], 0)) *abort_s = 1;
+    __syncthreads();
+    const uint32_t idS = idesc_bf16(128, 64, false, false);
+    for (int it = 0; it < niter; ++it) {
+        const int m = it / nhalf, hn = it % nhalf, buf = it & 1;
+        if (it >= 2 && !*abort_s) {
+            // the MMA of step it - 2 has released tile buffer `buf` and S buffer (it + 1) % 3
+            if (!mbar_wait(&bars[6 + buf], ((it - 2) >> 1) & 1)) *abort_s = 1;
+            const int j = it + 1;
+            if (tid == 0 && j < niter && !*abort_s) {
+                mbar_arrive_expect_tx(&bars[3 + j % kSBuf], 8192u);
+                tma_load_3d(sS + (j % kSBuf) * 8192, &mapS, &bars[3 + j % kSBuf], (j % nhalf) * 64, 0,
+                            srow + j / nhalf);
             }
         }
-        if (grp == 1) {
+        // (f_m o C)[t, n] for this 64-wide n half; group g writes n in [32 g, 32 g + 32)
+        float fm = 0.f;
 #pragma unroll
-            for (int p = 0; p < 32; ++p) part[p * TQ + t] = acc[p];
+        for (int q = 0; q < KMAX; ++q)
+            if (q == m) fm = f_t[q];
+        const unsigned char *crow = sC + hn * 16384 + t * 128;
+        unsigned char *drow = sM + buf * 16384 + t * 128;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int off = (((grp * 4 + q) ^ (t & 7)) * 16);
+            uint4 u = *reinterpret_cast<const uint4 *>(crow + off);
+            const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&u);
+            uint32_t r[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float2 f = __bfloat1622float2(h2[i]);
+                r[i] = pack_bf16x2(f.x * fm, f.y * fm);
+            }
+            *reinterpret_cast<uint4 *>(drow + off) = make_uint4(r[0], r[1], r[2], r[3]);
         }
+        fence_async_smem();
+        tc_fence_before();
         __syncthreads();
-        if (sl == 0 && !*abort_s && !mbar_wait(&bars[3], 0)) *abort_s = 1;
-        __syncthreads();
-        tc_fence_after();
-        if (!*abort_s && grp == 0) {
-            float yi[32];
-            tmem_ld32(lane_base + colY + 32 * sl, yi);
-            tmem_ld_wait();
-            if (t < n) {
-                uint4 *o = reinterpret_cast<uint4 *>(a.y + blh(d, b, c0 + t, h) * P + sl * TPS);
+        if (tid == 0 && !*abort_s) {
+            const int sb = it % kSBuf;
+            if (!mbar_wait(&bars[3 + sb], (it / kSBuf) & 1)) {
+                *abort_s = 1;
+            } else {
+                tc_fence_after();
+                for (int ks = 0; ks < 4; ++ks)
+                    mma_bf16(tmem + colY, desc_sw128(smem_u32(sM + buf * 16384) + ks * 32, 16, 1024),
+                             desc_sw128(smem_u32(sS + sb * 8192) + ks * 32, 16, 1024), idS, 1);
+                mma_commit(&bars[6 + buf]);
+            }
+        }
+    }
+    if (!*abort_s && niter > 0 && !mbar_wait(&bars[6 + ((niter - 1) & 1)], ((niter - 1) >> 1) & 1))
+        *abort_s = 1;
+    __syncthreads();
+    tc_fence_after();
+    if (!*abort_s) {  // y = Y + D x; group g takes p in [32 g, 32 g + 32)
+        float v[32];
+        tmem_ld32(lane_base + colY + grp * 32, v);
+        tmem_ld_wait();
+        if (t < n) {
+            const float Dh = a.D[h];
+            const unsigned char *xrow = sX + t * 128;
+            uint4 *o = reinterpret_cast<uint4 *>(a.y + blh(d, b, c0 + t, h) * P + grp * 32);
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    float v[8];
+            for (int q = 0; q < 4; ++q) {
+                const uint4 u = *reinterpret_cast<const uint4 *>(xrow + (((grp * 4 + q) ^ (t & 7)) * 16));
+                const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&u);
+                uint32_t r[4];
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) {
-                        const int p = 8 * q + i;
-                        v[i] = acc[p] + part[p * TQ + t] + yi[p] +
-                               Dh * __bfloat162float(xs[t * 64 + sl * TPS + p]);
-                    }
-                    o[q] = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]),
-                                      pack_bf16x2(v[6], v[7]));
+                for (int i = 0; i < 4; ++i) {
+                    const float2 f = __bfloat1622float2(h2[i]);
+                    r[i] = pack_bf16x2(fmaf(Dh, f.x, v[8 * q + 2 * i]), fmaf(Dh, f.y, v[8 * q + 2 * i + 1]));
                 }
+                o[q] = make_uint4(r[0], r[1], r[2], r[3]);
             }
         }
     }
     if (*abort_s && tid == 0) atomicExch(a.err, kTimeoutCode);
     tc_fence_before();
     __syncthreads();
-    if (tid < 32) tmem_dealloc(tmem, 512);
+    if (tid < 32) tmem_dealloc(tmem, 256);
 }
 
 // ------------------------------------------------------------------------------------- host
@@ -636,7 +657,7 @@ bool tc_make_map3(CUtensorMap *m, const void *ptr, uint64_t d0, uint64_t d1, uin
 
 bool tc_supported(const ScanDims &d, int dtype) {
     if (dtype != 1) return false;
-    if ((d.P != 32 && d.P != 64) || (d.N != 64 && d.N != 128) || (d.K != 4 && d.K != 8)) return false;
+    if (d.P != 64 || (d.N != 64 && d.N != 128) || (d.K != 4 && d.K != 8)) return false;
     return true;
 }
 
@@ -687,26 +708,26 @@ cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, int *e
     cudaError_t e = tc_state_pass_launch(d, false, p.x, p.Bm, p.ww, p.dt, p.alpha, p.lam, p.tau,
                                          p.h0, S_in, p.h_final, nullptr, nullptr, err, st);
     if (e != cudaSuccess || d.nc == 0) return e;
-    CUtensorMap mapC, mapB, mapS;
-    const uint64_t GN = uint64_t(d.G) * d.N;
+    CUtensorMap mapC, mapB, mapX, mapS;
+    const uint64_t GN = uint64_t(d.G) * d.N, HP = uint64_t(d.H) * d.P;
     if (!tc_make_map3(&mapC, p.Cm, GN, d.L, d.B, GN * 2, uint64_t(d.L) * GN * 2, 64, TQ, 1) ||
         !tc_make_map3(&mapB, p.Bm, GN, d.L, d.B, GN * 2, uint64_t(d.L) * GN * 2, 64, TQ, 1) ||
+        !tc_make_map3(&mapX, p.x, HP, d.L, d.B, HP * 2, uint64_t(d.L) * HP * 2, 64, TQ, 1) ||
         !tc_make_map3(&mapS, S_in, d.N, d.P, uint64_t(d.B) * d.H * d.nc * d.K, uint64_t(d.N) * 2,
-                   uint64_t(d.P) * d.N * 2, 64, TPS, d.K))
+                      uint64_t(d.P) * d.N * 2, 64, 64, 1))
         return cudaErrorInvalidValue;
     OutArgs a;
     a.d = d;
-    a.x = (const bf16 *)p.x;
     a.wr = (const bf16 *)p.wr;
     a.ww = (const bf16 *)p.ww;
     a.dt = p.dt; a.alpha = p.alpha; a.lam = p.lam; a.tau = p.tau; a.D = p.D;
     a.y = (bf16 *)p.y;
     a.err = err;
-    const size_t smem = OutSmem(d.K, d.N).total + 1024;
+    const size_t smem = OutSmem(d.N).total + 1024;
     cudaFuncSetAttribute(tc_chunk_fwd, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
     dim3 grid(d.H, d.nc, d.B);
     trace_begin("chunk_fwd_tc", st);
-    tc_chunk_fwd<<<grid, kOutThreads, smem, st>>>(mapC, mapB, mapS, a);
+    tc_chunk_fwd<<<grid, kOutThreads, smem, st>>>(mapC, mapB, mapX, mapS, a);
     trace_end(st);
     return cudaGetLastError();
 }

@@ -133,7 +133,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         fence_barrier_init();
     }
     if (tid < K) l2t[tid] = kLog2e / a.tau[h * K + tid];
-    if (tid < 32) tmem_alloc(tslot, 512);
+    if (tid < 32) tmem_alloc_once(tslot, 512);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -205,7 +205,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
 #pragma unroll
     for (int m = 0; m < KMAX; ++m) dwr_i[m] = 0.f;
     if (!*abort_s) {
-        float *mh_row = a.mh_total + ((size_t(b) * d.nc + c) * TQ + t) * TQ;
+        float *mh_row = a.mh_total + (((size_t(b) * d.nc + c) * d.G + g) * TQ + t) * TQ;
         for (int half = 0; half < 2; ++half) {
             const int k32 = grp == 0 ? (half == 0 ? 0 : 96) : (half == 0 ? 32 : 64);
             float gv[32], hv[32];
@@ -378,7 +378,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         fence_barrier_init();
     }
     if (tid < K) itau[tid] = 1.f / a.tau[h * K + tid];
-    if (w == 0) tmem_alloc(tslot, 512);
+    if (w == 0) tmem_alloc_once(tslot, 512);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -564,7 +564,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         *abort_s = 0;
         fence_barrier_init();
     }
-    if (w == 0) tmem_alloc(tslot, 256);
+    if (w == 0) tmem_alloc_once(tslot, 256);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -579,8 +579,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         mma_phase ^= 1;
     };
 
-    // head-summed intra term, once per chunk (group 0): dC = M_H B, dB = M_H^T C
-    if (hg == 0) {
+    // head-summed intra term, once per chunk and B/C group (by the group's first block):
+    // dC = M_H B, dB = M_H^T C
+    if (h_first % (d.H / d.G) == 0) {
         if (tid == 0) {
             mbar_arrive_expect_tx(&bars[0], uint32_t(2 * (N / 64) * 16384));
             for (int jb = 0; jb < N / 64; ++jb) {
@@ -588,7 +589,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tma_load_3d(sD + jb * 16384, &mapC, &bars[0], g * N + 64 * jb, c0, b);
             }
         }
-        const float *mrow = a.mh_total + ((size_t(b) * d.nc + c) * TQ + t) * TQ;
+        const float *mrow = a.mh_total + (((size_t(b) * d.nc + c) * d.G + g) * TQ + t) * TQ;
         for (int k8 = 0; k8 < TQ; k8 += 8) {
             float v[8];
 #pragma unroll
@@ -851,7 +852,7 @@ size_t tc_bwd_workspace_bytes(const ScanDims &d, TcBwdWorkspace *l, char *base) 
     l->ab_acc = (float *)take(blh_ * 2 * 4);
     l->rect = (float *)take(blh_ * 4);
     l->cdot = (float *)take(size_t(d.B) * d.H * d.nc * d.K * 4);
-    l->mh_total = (float *)take(size_t(d.B) * d.nc * TQ * TQ * 4);
+    l->mh_total = (float *)take(size_t(d.B) * d.nc * d.G * TQ * TQ * 4);
     l->dB_acc = (float *)take(size_t(d.B) * d.L * d.G * d.N * 4);
     l->dC_acc = (float *)take(size_t(d.B) * d.L * d.G * d.N * 4);
     return off;
@@ -867,7 +868,7 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
     if ((e = cudaMemsetAsync(ws.dC_acc, 0, sizeof(float) * ngn, st))) return e;
     if ((e = cudaMemsetAsync(ws.cdot, 0, sizeof(float) * d.B * d.H * d.nc * d.K, st))) return e;
     if ((e = cudaMemsetAsync(ws.ab_acc, 0, sizeof(float) * blh_ * 2, st))) return e;
-    if ((e = cudaMemsetAsync(ws.mh_total, 0, sizeof(float) * d.B * d.nc * TQ * TQ, st))) return e;
+    if ((e = cudaMemsetAsync(ws.mh_total, 0, sizeof(float) * d.B * d.nc * d.G * TQ * TQ, st))) return e;
     if (!reuse_states &&
         (e = tc_state_pass_launch(d, false, p.x, p.Bm, p.ww, p.dt, p.alpha, p.lam, p.tau, p.h0,
                                   ws.S_in, nullptr, nullptr, nullptr, err, st)))

@@ -92,6 +92,13 @@ __device__ __forceinline__ void tmem_alloc(uint32_t *slot, uint32_t ncols) {
 __device__ __forceinline__ void tmem_relinquish() {
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
 }
+// Allocation followed by giving up this CTA's allocation permit (the CTA allocates once).  A CTA
+// that keeps its permit holds the SM's tensor memory allocator for its whole lifetime, and the
+// SM then runs no second CTA of the kernel, whatever the shared memory would allow.
+__device__ __forceinline__ void tmem_alloc_once(uint32_t *slot, uint32_t ncols) {
+    tmem_alloc(slot, ncols);
+    tmem_relinquish();
+}
 __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
                  : "memory");

@@ -124,6 +124,23 @@ def test_bwd_bf16_groups():
     _check_bwd(synth.Shape(1, 130, 4, 32, 2, 32, 4, 0, "bf16"), seed=6)
 
 
+@pytest.mark.parametrize("N,K,G", [(128, 4, 1), (64, 4, 2), (128, 8, 2)])
+def test_tensor_path_modes_and_groups(N, K, G):
+    """bf16, headdim 64: every (N, K) the tensor-core kernels take, with B/C groups; the trace
+    shows that the tensor-core kernels ran."""
+    from paper_2609_36314_gb300 import _lib
+    s = synth.Shape(2, 200, 4, 64, G, N, K, 0, "bf16")
+    _lib.trace_reset()
+    _lib.trace_enable(True)
+    try:
+        _check_fwd(s, seed=20 + N + K, h0=True)
+        _check_bwd(s, seed=30 + N + K, h0=True, dhf=True)
+        names = set(_lib.trace_collect())
+    finally:
+        _lib.trace_enable(False)
+    assert {"state_pass_fwd_tc", "chunk_fwd_tc", "state_pass_rev_tc", "bwd_intra_tc"} <= names
+
+
 def test_force_simt_matches_default_path():
     s = synth.Shape(2, 260, 4, 64, 1, 128, 8, 0, "bf16")
     host = synth.make_scan_inputs(s, seed=12, with_dy=True)
