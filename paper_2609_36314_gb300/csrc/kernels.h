@@ -56,12 +56,11 @@ size_t tc_state_elems(const ScanDims &d);  // bf16 elements of the per-chunk sta
 cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, int *err,
                         cudaStream_t st);
 // Chunk-serial state pass on the tensor cores (forward: U = x, V = B, W = w_write; reverse:
-// U = dy, V = C, W = w_read, optionally accumulating <dS_out, S_in> per chunk and mode).
+// U = dy, V = C, W = w_read).
 cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, const void *V,
                                  const void *W, const float *dt, const float *alpha,
                                  const float *lam, const float *tau, const float *init,
-                                 void *emit, float *fin, const void *dot_src, float *dot_out,
-                                 int *err, cudaStream_t st);
+                                 void *emit, float *fin, int *err, cudaStream_t st);
 bool tc_make_map3(CUtensorMap *m, const void *ptr, uint64_t d0, uint64_t d1, uint64_t d2,
                   uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1,
                   uint32_t b2);

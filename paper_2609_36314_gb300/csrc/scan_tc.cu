@@ -43,8 +43,6 @@ struct StateArgs {
     const float *init;  // h0 or dh_final [B, H, K, P, N] or null
     bf16 *emit;         // per-chunk entering states [B, H, nc, K, P, N]
     float *fin;         // h_final or dh0, or null
-    const bf16 *dot_src;  // reverse pass only: S_in of every chunk (same layout as emit), or null
-    float *dot_out;       // reverse pass only: <emitted dS, S_in> per (b, h, chunk, mode) [B,H,nc,K]
     int *err;
 };
 
@@ -52,10 +50,9 @@ struct StateArgs {
 struct StateSmem {
     int a_bytes, v_bytes, total;
     __host__ __device__ StateSmem(int K, int N) {
-        a_bytes = (K / 4) * 2 * 16384;     // K/4 M-tiles x 2 k-atoms x (128 rows x 128 B)
-        v_bytes = (N / 64) * 16384;        // N/64 boxes of [128 t][64 n]
-        total = a_bytes + v_bytes + TQ * TPS * 2 /*x*/ + TQ * KMAX * 4 /*coef*/ +
-                TQ * 8 /*E*/ + TQ * 4 /*e*/ + 64 * 4 /*itau, dec*/ + 64 /*wsum*/ + 64 /*bars*/;
+        a_bytes = (K / 4) * 2 * 16384;  // K/4 M-tiles x 2 M-atoms x (128 k rows x 128 B), MN-major
+        v_bytes = (N / 64) * 16384;     // N/64 boxes of [128 t][64 n]
+        total = a_bytes + v_bytes + 64 * 4 /*itau, dec*/ + 64 /*wsum*/ + 16 /*E_end*/ + 64 /*bars*/;
     }
 };
 
@@ -70,14 +67,11 @@ __global__ void __launch_bounds__(kThreads, 2)
     const StateSmem plan(K, N);
     unsigned char *sA = base;
     unsigned char *sV = sA + plan.a_bytes;
-    bf16 *xs = reinterpret_cast<bf16 *>(sV + plan.v_bytes);          // [128][32]
-    float *coef = reinterpret_cast<float *>(xs + TQ * TPS);           // [128][K]
-    double *E_s = reinterpret_cast<double *>(coef + TQ * KMAX);       // [128]
-    float *e_s = reinterpret_cast<float *>(E_s + TQ);                 // [128]
-    float *itau = e_s + TQ;                                           // [32]
-    float *dec = itau + 32;                                           // [32]
-    double *wsum = reinterpret_cast<double *>(dec + 32);              // [4]
-    uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);          // tma, mma
+    float *itau = reinterpret_cast<float *>(sV + plan.v_bytes);  // [32]
+    float *dec = itau + 32;                                       // [32]
+    double *wsum = reinterpret_cast<double *>(dec + 32);          // [4]
+    double *Eend_s = wsum + 8;                                    // [1]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(Eend_s + 2);    // tma, mma
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 2);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
 
@@ -106,7 +100,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     for (int m = 0; m < K; ++m) tmax = fmaxf(tmax, a.tau[h * K + m]);
     const float log_cap = logf(64.f * tmax);
 
-    // initial state into tensor memory
+    // initial state into tensor memory: lane (m % 4, p), columns (m / 4, n)
     for (int mt = 0; mt < mtiles; ++mt) {
         const int m = mt * 4 + w;
         const float *src = a.init ? a.init + (bh * K + m) * PN + size_t(p0 + j) * N : nullptr;
@@ -119,8 +113,8 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
     tmem_st_wait();
 
-    // Inputs of chunk ci + 1 are fetched into registers while chunk ci is processed, so the
-    // global-load latency is off the chunk-serial critical path.
+    // Thread t owns chunk position t: its row of x (or dy) and its mode coefficients stay in
+    // registers, and the inputs of chunk ci + 1 are fetched while chunk ci is processed.
     uint4 nx[4];
     float ndt = 1.f, nal = 1.f, nlm = 1.f;
     float nw[KMAX];
@@ -162,43 +156,37 @@ __global__ void __launch_bounds__(kThreads, 2)
     for (int ci = 0; ci < d.nc; ++ci, phase ^= 1) {
         const int c = REV ? d.nc - 1 - ci : ci;
         const int c0 = c * TQ, n = min(TQ, d.L - c0);
-        // this chunk's inputs (fetched one iteration earlier) and coefficients: xs and coef were
-        // last read before the previous chunk's MMAs were issued, so this overlaps them
+        const int t = tid;
+        uint4 xr[4];
         float wcur[KMAX];
-        {
-            const int t = tid;
-            uint4 *dst = reinterpret_cast<uint4 *>(xs + t * TPS);
 #pragma unroll
-            for (int q = 0; q < 4; ++q) dst[q] = nx[q];
+        for (int q = 0; q < 4; ++q) xr[q] = nx[q];
 #pragma unroll
-            for (int m = 0; m < KMAX; ++m) wcur[m] = nw[m];
-            float e = 0.f;
-            if (t < n) {
-                bool cl;
-                e = token_rate(ndt, nal, nlm, log_cap, &cl);
-            }
-            e_s[t] = e;
-            E_s[t] = block_scan128(double(e), wsum);
+        for (int m = 0; m < KMAX; ++m) wcur[m] = nw[m];
+        float e = 0.f;
+        if (t < n) {
+            bool cl;
+            e = token_rate(ndt, nal, nlm, log_cap, &cl);
         }
+        const double Et = block_scan128(double(e), wsum);
+        if (t == n - 1) *Eend_s = Et;
         if (ci + 1 < d.nc) fetch(ci + 1);
         __syncthreads();
-        {
-            const int t = tid;
-            const double Eend = E_s[n - 1];
+        // this position's coefficient per mode: s = kappa exp(-(E_end - E_t)/tau) (forward) or
+        // f = w_read exp(-E_t/tau) (reverse)
+        const double Eend = *Eend_s;
+        float cv[KMAX];
 #pragma unroll
-            for (int m = 0; m < KMAX; ++m) {
-                if (m >= K) break;
-                float cv = 0.f;
-                if (t < n) {
-                    if (!REV)
-                        cv = -expm1f(-e_s[t] * itau[m]) * wcur[m] * expf(-float(Eend - E_s[t]) * itau[m]);
-                    else
-                        cv = wcur[m] * expf(-float(E_s[t]) * itau[m]);
-                }
-                coef[t * K + m] = cv;
+        for (int m = 0; m < KMAX; ++m) {
+            cv[m] = 0.f;
+            if (m < K && t < n) {
+                if (!REV)
+                    cv[m] = -expm1f(-e * itau[m]) * wcur[m] * expf(-float(Eend - Et) * itau[m]);
+                else
+                    cv[m] = wcur[m] * expf(-float(Et) * itau[m]);
             }
-            if (t < K) dec[t] = expf(-float(Eend) * itau[t]);
         }
+        if (t < K) dec[t] = expf(-float(Eend) * itau[t]);
         if (ci > 0) {  // previous chunk's MMAs done: tensor memory, sA and sV are free
             if (!mbar_wait(&bars[1], phase ^ 1)) *abort_s = 1;
         }
@@ -210,31 +198,39 @@ __global__ void __launch_bounds__(kThreads, 2)
             for (int jb = 0; jb < N / 64; ++jb)
                 tma_load_3d(sV + jb * 16384, &mapV, &bars[0], g * N + 64 * jb, c0, b);
         }
+        // A[(m%4, p), k] = s_{k,m} x_{k,p} as bf16, MN-major: row k = this thread's position,
+        // 64-element M-atoms (modes 2a, 2a+1 of the tile x 32 p), 128-byte swizzle
+#pragma unroll
+        for (int mt = 0; mt < KMAX / 4; ++mt) {
+            if (mt >= mtiles) break;
+#pragma unroll
+            for (int at = 0; at < 2; ++at) {
+                unsigned char *row = sA + (mt * 2 + at) * 16384 + t * 128;
+#pragma unroll
+                for (int c8 = 0; c8 < 8; ++c8) {
+                    const float s = cv[mt * 4 + 2 * at + (c8 >> 2)];  // mode of this 8-element run
+                    const uint4 xv = xr[c8 & 3];
+                    const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
+                    uint32_t r[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const float2 f = bf16x2_to_float2(xw[i]);
+                        r[i] = pack_bf16x2(s * f.x, s * f.y);
+                    }
+                    *reinterpret_cast<uint4 *>(row + ((c8 ^ (t & 7)) * 16)) = make_uint4(r[0], r[1], r[2], r[3]);
+                }
+            }
+        }
         // emit the entering state (bf16) and apply the chunk's decay in place
         for (int mt = 0; mt < mtiles; ++mt) {
             const int m = mt * 4 + w;
             const float dm = dec[m];
             const size_t row = ((bh * d.nc + c) * K + m) * PN + size_t(p0 + j) * N;
             bf16 *dst = a.emit + row;
-            float dsum = 0.f;
             for (int c32 = 0; c32 < N; c32 += 32) {
                 float v[32];
                 tmem_ld32(lane_base + mt * N + c32, v);
                 tmem_ld_wait();
-                if (REV && a.dot_out) {
-                    const uint4 *sp = reinterpret_cast<const uint4 *>(a.dot_src + row + c32);
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const uint4 u4 = sp[q];
-                        const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&u4);
-#pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            const float2 f2 = __bfloat1622float2(h2[i]);
-                            dsum = fmaf(v[8 * q + 2 * i], f2.x, dsum);
-                            dsum = fmaf(v[8 * q + 2 * i + 1], f2.y, dsum);
-                        }
-                    }
-                }
                 uint4 *o = reinterpret_cast<uint4 *>(dst + c32);
 #pragma unroll
                 for (int q = 0; q < 4; ++q)
@@ -245,31 +241,8 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
                 for (int q = 0; q < 4; ++q) tmem_st8(lane_base + mt * N + c32 + 8 * q, v + 8 * q);
             }
-            if (REV && a.dot_out) {
-                dsum = warp_sum(dsum);  // the 32 lanes of warp w are the 32 p of mode m
-                if (j == 0) atomicAdd(a.dot_out + (bh * d.nc + c) * K + m, dsum);
-            }
         }
         tmem_st_wait();
-        // A[(m%4, p), k] = s_{k,m} x_{k,p} (or f dy) as bf16, K-major, 128-byte swizzle
-        for (int mt = 0; mt < mtiles; ++mt) {
-            const int m = mt * 4 + w;
-            const int r = w * 32 + j;
-            for (int ka = 0; ka < 2; ++ka) {
-                unsigned char *tile = sA + (mt * 2 + ka) * 16384;
-#pragma unroll
-                for (int c8 = 0; c8 < 8; ++c8) {
-                    const int k0 = ka * 64 + c8 * 8;
-                    float v[8];
-#pragma unroll
-                    for (int i = 0; i < 8; ++i)
-                        v[i] = coef[(k0 + i) * K + m] * __bfloat162float(xs[(k0 + i) * TPS + j]);
-                    *reinterpret_cast<uint4 *>(tile + r * 128 + ((c8 ^ (r & 7)) * 16)) =
-                        make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
-                                   pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
-                }
-            }
-        }
         fence_async_smem();
         tc_fence_before();
         __syncthreads();
@@ -278,10 +251,10 @@ __global__ void __launch_bounds__(kThreads, 2)
             if (!mbar_wait(&bars[0], phase)) {
                 *abort_s = 1;
             } else {
-                const uint32_t idesc = idesc_bf16(128, N, false, true);
+                const uint32_t idesc = idesc_bf16(128, N, true, true);
                 for (int mt = 0; mt < mtiles; ++mt)
                     for (int ks = 0; ks < TQ / 16; ++ks) {
-                        const uint64_t ad = desc_sw128(smem_u32(sA + (mt * 2 + ks / 4) * 16384) + (ks % 4) * 32, 16, 1024);
+                        const uint64_t ad = desc_sw128(smem_u32(sA + mt * 32768) + ks * 2048, 16384, 1024);
                         const uint64_t bd = desc_sw128(smem_u32(sV) + ks * 2048, 16384, 1024);
                         mma_bf16(tmem + mt * N, ad, bd, idesc, 1);
                     }
@@ -668,8 +641,7 @@ size_t tc_state_elems(const ScanDims &d) {
 cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, const void *V,
                                  const void *W, const float *dt, const float *alpha,
                                  const float *lam, const float *tau, const float *init,
-                                 void *emit, float *fin, const void *dot_src, float *dot_out,
-                                 int *err, cudaStream_t st) {
+                                 void *emit, float *fin, int *err, cudaStream_t st) {
     CUtensorMap mapV;
     if (!tc_make_map3(&mapV, V, uint64_t(d.G) * d.N, d.L, d.B, uint64_t(d.G) * d.N * 2,
                    uint64_t(d.L) * d.G * d.N * 2, 64, TQ, 1))
@@ -682,8 +654,6 @@ cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, con
     a.init = init;
     a.emit = (bf16 *)emit;
     a.fin = fin;
-    a.dot_src = (const bf16 *)dot_src;
-    a.dot_out = dot_out;
     a.err = err;
     const size_t smem = StateSmem(d.K, d.N).total + 1024;
     dim3 grid(d.P / TPS, d.H, d.B);
@@ -706,7 +676,7 @@ cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, con
 cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, int *err,
                         cudaStream_t st) {
     cudaError_t e = tc_state_pass_launch(d, false, p.x, p.Bm, p.ww, p.dt, p.alpha, p.lam, p.tau,
-                                         p.h0, S_in, p.h_final, nullptr, nullptr, err, st);
+                                         p.h0, S_in, p.h_final, err, st);
     if (e != cudaSuccess || d.nc == 0) return e;
     CUtensorMap mapC, mapB, mapX, mapS;
     const uint64_t GN = uint64_t(d.G) * d.N, HP = uint64_t(d.H) * d.P;

@@ -871,10 +871,10 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
     if ((e = cudaMemsetAsync(ws.mh_total, 0, sizeof(float) * d.B * d.nc * d.G * TQ * TQ, st))) return e;
     if (!reuse_states &&
         (e = tc_state_pass_launch(d, false, p.x, p.Bm, p.ww, p.dt, p.alpha, p.lam, p.tau, p.h0,
-                                  ws.S_in, nullptr, nullptr, nullptr, err, st)))
+                                  ws.S_in, nullptr, err, st)))
         return e;
     if ((e = tc_state_pass_launch(d, true, p.dy, p.Cm, p.wr, p.dt, p.alpha, p.lam, p.tau,
-                                  p.dh_final, ws.dS_out, p.dh0, nullptr, nullptr, err, st)))
+                                  p.dh_final, ws.dS_out, p.dh0, err, st)))
         return e;
     if (d.nc == 0) return cudaSuccess;
     const uint64_t GN = uint64_t(d.G) * d.N, HP = uint64_t(d.H) * d.P;

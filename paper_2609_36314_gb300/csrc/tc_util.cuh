@@ -19,6 +19,11 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
     return *reinterpret_cast<const uint32_t *>(&v);
 }
 
+// The two bf16 halves of a 32-bit word as floats (low half first); exact.
+__device__ __forceinline__ float2 bf16x2_to_float2(uint32_t v) {
+    return make_float2(__uint_as_float(v << 16), __uint_as_float(v & 0xffff0000u));
+}
+
 __device__ __forceinline__ size_t blh(const ScanDims &d, int b, int t, int h) {
     return (size_t(b) * d.L + t) * d.H + h;
 }
