@@ -315,30 +315,6 @@ struct OutSmem {
     }
 };
 
-__device__ __forceinline__ void load_weights(const bf16 *src, int K, float *w) {
-    if (K == 8) {
-        const uint4 u = *reinterpret_cast<const uint4 *>(src);
-        const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&u);
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const float2 f = __bfloat1622float2(h2[q]);
-            w[2 * q] = f.x;
-            w[2 * q + 1] = f.y;
-        }
-    } else {  // K == 4
-        const uint2 u = *reinterpret_cast<const uint2 *>(src);
-        const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&u);
-#pragma unroll
-        for (int q = 0; q < 2; ++q) {
-            const float2 f = __bfloat1622float2(h2[q]);
-            w[2 * q] = f.x;
-            w[2 * q + 1] = f.y;
-        }
-#pragma unroll
-        for (int m = 4; m < KMAX; ++m) w[m] = 0.f;
-    }
-}
-
 // One CTA per (b, h, chunk), headdim 64, all in one TMEM accumulator Y[t, p]:
 //   Y  = (Gamma o C B^T) X                      (intra-chunk pairs, K = t)
 //   Y += sum_m (f_m o C) S_in,m^T               (entering state, K = (m, n), 64-wide n steps)

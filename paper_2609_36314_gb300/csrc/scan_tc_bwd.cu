@@ -117,7 +117,8 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     float *part = kap_s + TQ * KMAX;                         // [128][KMAX] partial sums of group 1
     float2 *E_s = reinterpret_cast<float2 *>(part + TQ * KMAX);  // hi / lo pairs
     float *l2t = reinterpret_cast<float *>(E_s + TQ);
-    double *wsum = reinterpret_cast<double *>(l2t + 32);
+    float *tau_s = l2t + 32;
+    double *wsum = reinterpret_cast<double *>(tau_s + 32);
     uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 3);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
@@ -132,8 +133,26 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         *abort_s = 0;
         fence_barrier_init();
     }
-    if (tid < K) l2t[tid] = kLog2e / a.tau[h * K + tid];
+    if (tid < K) {
+        const float tv = a.tau[h * K + tid];
+        tau_s[tid] = tv;
+        l2t[tid] = kLog2e / tv;
+    }
     if (tid < 32) tmem_alloc_once(tslot, 512);
+    // per-position inputs of row t, all loads issued before anything waits on them
+    float dtv = 1.f, alv = 1.f, lmv = 1.f;
+    float wr_t[KMAX], ww_t[KMAX];
+    if (t < n) {
+        const size_t i = blh(d, b, c0 + t, h);
+        dtv = a.dt[i];
+        alv = a.alpha[i];
+        lmv = a.lam[i];
+        load_weights(a.wr + i * K, K, wr_t);
+        load_weights(a.ww + i * K, K, ww_t);
+    } else {
+#pragma unroll
+        for (int m = 0; m < KMAX; ++m) wr_t[m] = ww_t[m] = 0.f;
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -150,28 +169,25 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         tma_load_3d(sX, &mapX, &bars[0], h * P, c0, b);
         tma_load_3d(sDY, &mapDY, &bars[0], h * P, c0, b);
     }
-    const float log_cap = head_log_cap(a.tau, h, K);
+    float tmax = 0.f;
+    for (int m = 0; m < K; ++m) tmax = fmaxf(tmax, tau_s[m]);
+    const float log_cap = logf(64.f * tmax);
     float e = 0.f;
-    float wr_t[KMAX];
     if (t < n) {
-        const size_t i = blh(d, b, c0 + t, h);
         bool cl;
-        e = token_rate(a.dt[i], a.alpha[i], a.lam[i], log_cap, &cl);
+        e = token_rate(dtv, alv, lmv, log_cap, &cl);
     }
     const double Et = group_scan128(double(e), wsum);
     const float2 Et2 = split_f2(Et);
     if (grp == 0) E_s[t] = Et2;
+    float l2r[KMAX];  // log2(e) / tau per mode, in registers
 #pragma unroll
     for (int m = 0; m < KMAX; ++m) {
-        float wv = 0.f, kp = 0.f;
-        if (m < K && t < n) {
-            const size_t wi = blh(d, b, c0 + t, h) * K + m;
-            wv = to_f(a.wr[wi]);
-            kp = -expm1f(-e * (l2t[m] / kLog2e)) * to_f(a.ww[wi]);
-        }
-        wr_t[m] = wv;
+        l2r[m] = m < K ? l2t[m] : 0.f;
+        float kp = 0.f;
+        if (m < K && t < n) kp = -expm1f(-e / tau_s[m]) * ww_t[m];
         if (grp == 0) {
-            wr_s[t * KMAX + m] = wv;
+            wr_s[t * KMAX + m] = wr_t[m];
             kap_s[t * KMAX + m] = kp;
         }
     }
@@ -222,11 +238,11 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
 #pragma unroll
                     for (int m = 0; m < KMAX; ++m) {
                         if (m < K) {
-                            const float W = ex2_approx(-dE * l2t[m]);
+                            const float W = ex2_approx(-dE * l2r[m]);
                             const float kp = kap_s[k * KMAX + m];
                             const float aa = wr_t[m] * kp * W;
                             gam += aa;
-                            gamt = fmaf(aa, l2t[m], gamt);  // times log2(e) / tau
+                            gamt = fmaf(aa, l2r[m], gamt);  // times log2(e) / tau
                             dwr_i[m] = fmaf(kp * W, gh, dwr_i[m]);
                         }
                     }
@@ -284,15 +300,33 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         // diagonal (tt < k) contribute nothing
         const int k = t;
         const float2 Ek = E_s[k];
-        // group grp takes the rows of parity grp, starting at this warp's first column
-        for (int tt = (t & ~31) + grp; tt < n; tt += 2) {
-            if (tt < k) continue;
-            const float dE = diff_f2(E_s[tt], Ek);
-            const float gh = GHs[tt * XS + k];
+        float dk2[KMAX];
 #pragma unroll
-            for (int m = 0; m < KMAX; ++m)
-                if (m < K) dk[m] = fmaf(wr_s[tt * KMAX + m] * ex2_approx(-dE * l2t[m]), gh, dk[m]);
+        for (int m = 0; m < KMAX; ++m) dk2[m] = 0.f;
+        // group grp takes the rows of parity grp, starting at this warp's first column; four
+        // rows per step (two accumulator sets) keep several exponentials in flight
+        for (int tt0 = (t & ~31) + grp; tt0 < n; tt0 += 8) {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int tt = tt0 + 2 * u;
+                if (tt < n && tt >= k) {
+                    const float dE = diff_f2(E_s[tt], Ek);
+                    const float gh = GHs[tt * XS + k];
+#pragma unroll
+                    for (int m = 0; m < KMAX; ++m) {
+                        if (m < K) {
+                            const float v = wr_s[tt * KMAX + m] * ex2_approx(-dE * l2r[m]);
+                            if (u & 1)
+                                dk2[m] = fmaf(v, gh, dk2[m]);
+                            else
+                                dk[m] = fmaf(v, gh, dk[m]);
+                        }
+                    }
+                }
+            }
         }
+#pragma unroll
+        for (int m = 0; m < KMAX; ++m) dk[m] += dk2[m];
         if (grp == 1) {
 #pragma unroll
             for (int m = 0; m < KMAX; ++m) part[k * KMAX + m] = dk[m];

@@ -28,6 +28,32 @@ __device__ __forceinline__ size_t blh(const ScanDims &d, int b, int t, int h) {
     return (size_t(b) * d.L + t) * d.H + h;
 }
 
+// The K (4 or 8) bf16 mode weights of one position as floats (16- or 8-byte load); modes
+// beyond K are zero.
+__device__ __forceinline__ void load_weights(const __nv_bfloat16 *src, int K, float *w) {
+    if (K == 8) {
+        const uint4 v = *reinterpret_cast<const uint4 *>(src);
+        const uint32_t r[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float2 f = bf16x2_to_float2(r[q]);
+            w[2 * q] = f.x;
+            w[2 * q + 1] = f.y;
+        }
+    } else {  // K == 4
+        const uint2 v = *reinterpret_cast<const uint2 *>(src);
+        const uint32_t r[2] = {v.x, v.y};
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const float2 f = bf16x2_to_float2(r[q]);
+            w[2 * q] = f.x;
+            w[2 * q + 1] = f.y;
+        }
+#pragma unroll
+        for (int m = 4; m < KMAX; ++m) w[m] = 0.f;
+    }
+}
+
 // Inclusive prefix sum (double) of one value per thread over a 128-thread block.
 __device__ __forceinline__ double block_scan128(double v, double *wsum) {
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
