@@ -143,7 +143,6 @@ def algorithmic_work(kernel: str, s, per_launch_units: float):
     per_th = {
         "state_pass_fwd_simt": 2, "state_pass_rev_simt": 2, "chunk_fwd_simt": 2,
         "chunk_bwd_simt": 8, "state_pass_fwd_tc": 2, "state_pass_rev_tc": 2,
-        "bwd_inter_tc": 4, "bwd_dcdb_tc": 4,
     }
     if kernel in per_th:
         return "flops", per_th[kernel] * kpn(s) * per_launch_units
@@ -152,6 +151,8 @@ def algorithmic_work(kernel: str, s, per_launch_units: float):
     q = 128
     if kernel == "chunk_fwd_tc":
         return "flops", (2 * kpn(s) + q * s.headdim + q * s.dstate * s.ngroups / s.nheads) * per_launch_units
+    if kernel == "bwd_state_tc":  # Z, U, dC, dB contractions + the head-summed intra dC, dB
+        return "flops", (8 * kpn(s) + 4 * q * s.dstate * s.ngroups / s.nheads) * per_launch_units
     if kernel == "bwd_intra_tc":
         return "flops", (2 * q * s.headdim + q * s.dstate * s.ngroups / s.nheads) * per_launch_units
     if kernel == "decode_step":

@@ -15,10 +15,10 @@
 //   tc_bwd_intra  (b, c, h): G, H on the tensor cores; per-position passes for Gamma, Gamma',
 //                 the intra parts of dw_read / dkappa and the pair rectangle sums; dx_intra =
 //                 (Gamma o G)^T dy on the tensor cores; Gamma o H added over heads (fp32, L2).
-//   tc_bwd_inter  (b, c, h, 32-wide P-slice): Z = C S_in^T and U = B dS_out^T on the tensor
-//                 cores; epilogue to dx, dw_read, dkappa and the a, b terms.
-//   tc_bwd_dcdb   (b, c, group of heads): dC and dB accumulated in tensor memory over the heads
-//                 of the group (and the head-summed intra term, once per chunk).
+//   tc_bwd_state  (b, c, group of heads): per (head, mode) Z = C S_in^T and U = B dS_out^T,
+//                 dx += (s o B) dS_out^T, dC += (f o dY) S_in and dB += (s o X) dS_out on the
+//                 tensor cores (dC, dB summed over the group's heads in TMEM); epilogue to
+//                 dw_read, dkappa, the a, b terms and <dS_out, S_in>; the head-summed intra term.
 //   tc_bwd_final  (b, h, c): per-position gradients of Delta, alpha, lambda, w_write, bf16 casts.
 // All mbarrier waits are bounded; a timeout sets FRAC_ERR_TIMEOUT in the status word.
 #include <cuda.h>
@@ -371,181 +371,353 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     if (tid < 32) tmem_dealloc(tmem, 512);
 }
 
-// ============================================================================= inter
-struct InterSmem {
-    int cb, s, total;
-    __host__ __device__ InterSmem(int K, int N) {
-        cb = (N / 64) * 16384;           // one of C / B
-        s = (N / 64) * (K * TPS * 128);  // one of S_in / dS_out slices
-        total = 2 * cb + 2 * s + 64 + 64;
+// ============================================================================= state terms
+// One CTA per (b, c, group of hg heads of one B/C group), 256 threads, software-pipelined over
+// the (head, mode) steps.  Step i, with the mode's S_in and dS_out tiles [p][n] streamed in by
+// TMA (three buffers):
+//   Z_m = C S_in,m^T,  U_m = B dS_out,m^T                  (TMEM, two buffers of 2 x 64 columns)
+//   dC += (f_m o dY) S_in,m,  dB += (s_m o X) dS_out,m       (TMEM, summed over modes and heads)
+// While the tensor cores run step i, the threads read out step i - 1: group 0 contracts Z_m with
+// its dY row (dw_read, the a term), group 1 contracts U_m with its X row (dkappa, the b term) and
+// accumulates dx = sum_m s_m U_m in registers.  <dS_out,m, S_in,m> comes from the two tiles in
+// shared memory.  The head-summed intra tile Gamma o H adds M_H B to dC and M_H^T C to dB once
+// per (b, c, B/C group).
+constexpr int kStThreads = 256;
+constexpr int kStBuf = 3;  // S_in / dS_out tile buffers
+
+struct StSmem {
+    int cb, tile, gen, total;
+    __host__ __device__ explicit StSmem(int N) {
+        cb = (N / 64) * 16384;   // one of C / B: [t][n]
+        tile = (N / 64) * 8192;  // one S_in or dS_out mode tile: [p = 64][n], 64-wide n atoms
+        gen = 2 * 16384;         // f o dY and s o X: [t][p] each; two buffers (the first holds M_H)
+        total = 2 * cb + kStBuf * 2 * tile + 2 * gen + 256;
     }
 };
 
-__global__ void __launch_bounds__(kThreads, 1)
-    tc_bwd_inter(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapB,
+__device__ __forceinline__ float dot_bf16x8(uint4 a, uint4 b, float acc) {
+    const uint32_t ra[4] = {a.x, a.y, a.z, a.w}, rb[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 fa = bf16x2_to_float2(ra[i]), fb = bf16x2_to_float2(rb[i]);
+        acc = fmaf(fa.x, fb.x, fmaf(fa.y, fb.y, acc));
+    }
+    return acc;
+}
+
+__device__ __forceinline__ uint4 scale_bf16x8(uint4 a, float s) {
+    const uint32_t ra[4] = {a.x, a.y, a.z, a.w};
+    uint32_t r[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 f = bf16x2_to_float2(ra[i]);
+        r[i] = pack_bf16x2(s * f.x, s * f.y);
+    }
+    return make_uint4(r[0], r[1], r[2], r[3]);
+}
+
+__global__ void __launch_bounds__(kStThreads, 1)
+    tc_bwd_state(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapB,
                  const __grid_constant__ CUtensorMap mapS, const __grid_constant__ CUtensorMap mapD,
                  BwdArgs a) {
     extern __shared__ unsigned char smem_raw[];
     unsigned char *base = align1024(smem_raw);
     const ScanDims &d = a.d;
     const int K = d.K, N = d.N, P = d.P;
-    const InterSmem L(K, N);
-    unsigned char *sC = base, *sB = sC + L.cb, *sS = sB + L.cb, *sD = sS + L.s;
-    double *wsum = reinterpret_cast<double *>(sD + L.s);
-    uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 4);
-    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 2);
+    const StSmem L(N);
+    unsigned char *sC = base, *sB = sC + L.cb, *sT = sB + L.cb;
+    unsigned char *sG = sT + kStBuf * 2 * L.tile;             // [buf][f o dY | s o X]
+    // per-warp partial dots of steps i mod 3: step i - 1 is summed by thread 0 after the
+    // barrier of step i, while other warps may already write step i + 1
+    float *red = reinterpret_cast<float *>(sG + 2 * L.gen);   // [3][8]
+    double *wsum = reinterpret_cast<double *>(red + 24);      // [8]
+    double *Eend_s = wsum + 8;                                // [1]
+    // bars: 0..2 tile buffers | 3, 4 MMA of step parity | 5 C, B | 6 intra MMA
+    uint64_t *bars = reinterpret_cast<uint64_t *>(Eend_s + 2);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 7);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
-    __shared__ float itau[32];
 
-    const int tid = threadIdx.x, w = tid >> 5, r = tid;
-    const int npart = P / TPS;
-    const int h = blockIdx.x / npart, p0 = (blockIdx.x % npart) * TPS;
-    const int c = blockIdx.y, b = blockIdx.z;
-    const int g = h / (d.H / d.G);
+    const int tid = threadIdx.x, grp = tid >> 7, t = tid & 127, w = tid >> 5, w4 = w & 3;
+    const int hgi = blockIdx.x, c = blockIdx.y, b = blockIdx.z;
+    const int h_first = hgi * a.hg;
+    const int g = h_first / (d.H / d.G);
     const int c0 = c * TQ, n = min(TQ, d.L - c0);
-    const uint32_t ZN = uint32_t(K * TPS);
+    const int nsteps = a.hg * K;
+    const bool intra = (h_first % (d.H / d.G)) == 0;
+    constexpr uint32_t colC = 0, colB = 128, colZU = 256;  // Z / U of buffer q at 256 + 128 q (+ 64)
 
     if (tid == 0) {
-        mbar_init(&bars[0], 1);
-        mbar_init(&bars[1], 1);
+        for (int i = 0; i < 7; ++i) mbar_init(&bars[i], 1);
         *abort_s = 0;
         fence_barrier_init();
     }
-    if (tid < K) itau[tid] = 1.f / a.tau[h * K + tid];
     if (w == 0) tmem_alloc_once(tslot, 512);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tslot;
-    const uint32_t lane_base = tmem + (uint32_t(w * 32) << 16);
-    if (tid == 0) {
-        mbar_arrive_expect_tx(&bars[0], uint32_t(2 * L.cb + 2 * L.s));
-        const int srow = int(((size_t(b) * d.H + h) * d.nc + c) * K);
+    const uint32_t lane_base = tmem + (uint32_t(w4 * 32) << 16);
+
+    auto issue_tiles = [&](int i) {  // thread 0: S_in / dS_out tiles of step i into buffer i % 3
+        const int q = i % kStBuf;
+        const int srow = int(((size_t(b) * d.H + h_first + i / K) * d.nc + c) * K + i % K);
+        mbar_arrive_expect_tx(&bars[q], uint32_t(2 * L.tile));
         for (int jb = 0; jb < N / 64; ++jb) {
-            tma_load_3d(sC + jb * 16384, &mapC, &bars[0], g * N + 64 * jb, c0, b);
-            tma_load_3d(sB + jb * 16384, &mapB, &bars[0], g * N + 64 * jb, c0, b);
-            tma_load_3d(sS + jb * (K * TPS * 128), &mapS, &bars[0], 64 * jb, p0, srow);
-            tma_load_3d(sD + jb * (K * TPS * 128), &mapD, &bars[0], 64 * jb, p0, srow);
+            tma_load_3d(sT + (2 * q) * L.tile + jb * 8192, &mapS, &bars[q], 64 * jb, 0, srow);
+            tma_load_3d(sT + (2 * q + 1) * L.tile + jb * 8192, &mapD, &bars[q], 64 * jb, 0, srow);
         }
-    }
-    // per-position coefficients of row r
-    const float log_cap = head_log_cap(a.tau, h, K);
-    float e = 0.f;
-    if (r < n) {
-        const size_t i = blh(d, b, c0 + r, h);
-        bool cl;
-        e = token_rate(a.dt[i], a.alpha[i], a.lam[i], log_cap, &cl);
-    }
-    const double Er = block_scan128(double(e), wsum);
-    __shared__ double Eend_s;
-    if (r == n - 1) Eend_s = Er;
-    __syncthreads();
-    const double Eend = Eend_s;
-    float s_r[KMAX], u_r[KMAX], fd_r[KMAX], f_r[KMAX];
-#pragma unroll
-    for (int m = 0; m < KMAX; ++m) {
-        s_r[m] = u_r[m] = fd_r[m] = f_r[m] = 0.f;
-        if (m < K && r < n) {
-            const size_t wi = blh(d, b, c0 + r, h) * K + m;
-            const float kp = -expm1f(-e * itau[m]) * to_f(a.ww[wi]);
-            u_r[m] = expf(-float(Eend - Er) * itau[m]);
-            s_r[m] = kp * u_r[m];
-            fd_r[m] = expf(-float(Er) * itau[m]);
-            f_r[m] = to_f(a.wr[wi]) * fd_r[m];
-        }
-    }
-    float xr[32], dyr[32];
-    if (r < n) {
-        load_bf16x32(a.x + blh(d, b, c0 + r, h) * P + p0, xr);
-        load_bf16x32(a.dy + blh(d, b, c0 + r, h) * P + p0, dyr);
-    } else {
-#pragma unroll
-        for (int p = 0; p < 32; ++p) xr[p] = dyr[p] = 0.f;
-    }
+    };
     if (tid == 0) {
-        if (!mbar_wait(&bars[0], 0)) {
-            *abort_s = 1;
-        } else {
-            tc_fence_after();
-            const uint32_t idZ = idesc_bf16(128, int(ZN), false, false);
-            for (int ks = 0; ks < N / 16; ++ks) {
-                const uint32_t koff = (ks / 4) * 16384 + (ks % 4) * 32;
-                const uint32_t soff = (ks / 4) * (K * TPS * 128) + (ks % 4) * 32;
-                mma_bf16(tmem, desc_sw128(smem_u32(sC) + koff, 16, 1024),
-                         desc_sw128(smem_u32(sS) + soff, 16, 1024), idZ, ks > 0);
-                mma_bf16(tmem + ZN, desc_sw128(smem_u32(sB) + koff, 16, 1024),
-                         desc_sw128(smem_u32(sD) + soff, 16, 1024), idZ, ks > 0);
+        mbar_arrive_expect_tx(&bars[5], uint32_t(2 * L.cb));
+        for (int jb = 0; jb < N / 64; ++jb) {
+            tma_load_3d(sC + jb * 16384, &mapC, &bars[5], g * N + 64 * jb, c0, b);
+            tma_load_3d(sB + jb * 16384, &mapB, &bars[5], g * N + 64 * jb, c0, b);
+        }
+        for (int i = 0; i < min(kStBuf, nsteps); ++i) issue_tiles(i);
+    }
+
+    // head-summed intra term: dC = M_H B, dB = M_H^T C (M_H as bf16 [t][k] in generator buffer 0)
+    if (intra) {
+        const float *mrow = a.mh_total + (((size_t(b) * d.nc + c) * d.G + g) * TQ + t) * TQ + grp * 64;
+#pragma unroll
+        for (int k8 = 0; k8 < 64; k8 += 8) {
+            const float4 u0 = *reinterpret_cast<const float4 *>(mrow + k8);
+            const float4 u1 = *reinterpret_cast<const float4 *>(mrow + k8 + 4);
+            const float v[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+            store_bf16x8(sG + grp * 16384 + t * 128 + (((k8 >> 3) ^ (t & 7)) * 16), v);
+        }
+        fence_async_smem();
+        __syncthreads();
+        if (tid == 0) {
+            if (!mbar_wait(&bars[5], 0)) {
+                *abort_s = 1;
+            } else {
+                tc_fence_after();
+                const uint32_t idC = idesc_bf16(128, N, false, true);
+                const uint32_t idB = idesc_bf16(128, N, true, true);
+                for (int ks = 0; ks < TQ / 16; ++ks) {
+                    mma_bf16(tmem + colC, desc_sw128(smem_u32(sG) + (ks / 4) * 16384 + (ks % 4) * 32, 16, 1024),
+                             desc_sw128(smem_u32(sB) + ks * 2048, 16384, 1024), idC, ks > 0);
+                    mma_bf16(tmem + colB, desc_sw128(smem_u32(sG) + ks * 2048, 16384, 1024),
+                             desc_sw128(smem_u32(sC) + ks * 2048, 16384, 1024), idB, ks > 0);
+                }
+                mma_commit(&bars[6]);
             }
-            mma_commit(&bars[1]);
         }
+        __syncthreads();
+        if (!*abort_s && !mbar_wait(&bars[6], 0)) *abort_s = 1;  // generator buffer 0 is rewritten
     }
-    // <dS_out, S_in> of this P-slice per mode, straight from the two tiles in shared memory (both
-    // carry the same swizzle, so the byte-for-byte dot product is the element dot product);
-    // it runs while the tensor cores work
-    if (mbar_wait(&bars[0], 0)) {
-        const int tpm = kThreads / K;  // threads per mode
-        const int m = tid / tpm, jl = tid % tpm;
-        float acc = 0.f;
-        for (int jb = 0; jb < N / 64; ++jb) {
-            const uint4 *ps = reinterpret_cast<const uint4 *>(sS + jb * (K * TPS * 128) + m * 4096);
-            const uint4 *pd = reinterpret_cast<const uint4 *>(sD + jb * (K * TPS * 128) + m * 4096);
-            for (int q = jl; q < 256; q += tpm) {
-                const uint4 u = ps[q], v = pd[q];
-                const __nv_bfloat162 *a2 = reinterpret_cast<const __nv_bfloat162 *>(&u);
-                const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(&v);
+    if (!*abort_s && !mbar_wait(&bars[5], 0)) *abort_s = 1;      // C and B are read below
+
+    float f_t[KMAX], s_t[KMAX], u_t[KMAX], fd_t[KMAX], itr[KMAX];
+    uint4 row[8];     // group 0: dY row (64 p), group 1: X row
+    float dxr[64];    // group 1: inter-chunk dx of this row, current head
+    float acc_h[KMAX], ab_h = 0.f;  // group 0: dw_read and a; group 1: dkappa and b
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const float2 fa = __bfloat1622float2(a2[i]), fb = __bfloat1622float2(b2[i]);
-                    acc = fmaf(fa.x, fb.x, fmaf(fa.y, fb.y, acc));
+    for (int m = 0; m < KMAX; ++m) f_t[m] = s_t[m] = u_t[m] = fd_t[m] = itr[m] = acc_h[m] = 0.f;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) row[q] = make_uint4(0, 0, 0, 0);
+#pragma unroll
+    for (int p = 0; p < 64; ++p) dxr[p] = 0.f;
+
+    // read out step j (its MMAs complete): Z (group 0) or U (group 1) against this row
+    auto readout = [&](int j) {
+        if (!*abort_s && !mbar_wait(&bars[3 + (j & 1)], (j >> 1) & 1)) *abort_s = 1;
+        tc_fence_after();
+        if (tid == 0 && j + kStBuf < nsteps && !*abort_s) issue_tiles(j + kStBuf);  // buffer of step j
+        const int mj = j % K, hj = h_first + j / K;
+        if (!*abort_s) {
+            const uint32_t col = colZU + 128 * (j & 1) + 64 * grp;
+            float sj = 0.f;
+#pragma unroll
+            for (int m = 0; m < KMAX; ++m)
+                if (m == mj) sj = s_t[m];
+            float dotv = 0.f;
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                float zv[32];
+                tmem_ld32(lane_base + col + half * 32, zv);
+                tmem_ld_wait();
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const uint4 rv = row[half * 4 + q];
+                    const uint32_t rr[4] = {rv.x, rv.y, rv.z, rv.w};
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const float2 f = bf16x2_to_float2(rr[k]);
+                        dotv = fmaf(f.x, zv[8 * q + 2 * k], fmaf(f.y, zv[8 * q + 2 * k + 1], dotv));
+                    }
+                }
+                if (grp == 1) {
+#pragma unroll
+                    for (int p = 0; p < 32; ++p) dxr[half * 32 + p] = fmaf(sj, zv[p], dxr[half * 32 + p]);
+                }
+            }
+#pragma unroll
+            for (int m = 0; m < KMAX; ++m) {
+                if (m == mj) {
+                    if (grp == 0) {
+                        acc_h[m] = fd_t[m] * dotv;                 // dw_read (inter)
+                        ab_h = fmaf(f_t[m] * dotv, itr[m], ab_h);  // a
+                    } else {
+                        acc_h[m] = u_t[m] * dotv;                  // dkappa (inter)
+                        ab_h = fmaf(s_t[m] * dotv, itr[m], ab_h);  // b
+                    }
                 }
             }
         }
-        for (int o = tpm >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-        if (jl == 0) atomicAdd(a.cdot + ((size_t(b) * d.H + h) * d.nc + c) * K + m, acc);
-    } else {
-        *abort_s = 1;
-    }
-    __syncthreads();
-    if (!*abort_s && !mbar_wait(&bars[1], 0)) *abort_s = 1;
-    __syncthreads();
-    tc_fence_after();
-    if (!*abort_s) {
-        float dx[32];
-#pragma unroll
-        for (int p = 0; p < 32; ++p) dx[p] = 0.f;
-        float aa = 0.f, bb = 0.f;
-        float *dwr = a.dwr_acc + blh(d, b, c0 + r, h) * K;
-        float *dkp = a.dkap_acc + blh(d, b, c0 + r, h) * K;
-#pragma unroll
-        for (int m = 0; m < KMAX; ++m) {
-            if (m >= K) break;
-            float z[32], u[32];
-            tmem_ld32(lane_base + m * TPS, z);
-            tmem_ld32(lane_base + ZN + m * TPS, u);
-            tmem_ld_wait();
-            float dyz = 0.f, xu = 0.f;
-#pragma unroll
-            for (int p = 0; p < 32; ++p) {
-                dyz = fmaf(dyr[p], z[p], dyz);
-                xu = fmaf(xr[p], u[p], xu);
-                dx[p] = fmaf(s_r[m], u[p], dx[p]);
-            }
-            if (r < n) {
-                atomicAdd(dwr + m, fd_r[m] * dyz);
-                atomicAdd(dkp + m, u_r[m] * xu);
-            }
-            aa = fmaf(f_r[m] * dyz, itau[m], aa);
-            bb = fmaf(s_r[m] * xu, itau[m], bb);
+        if (tid == 0) {
+            const float *r2 = red + (j % 3) * 8;
+            a.cdot[((size_t(b) * d.H + hj) * d.nc + c) * K + mj] =
+                ((r2[0] + r2[1]) + (r2[2] + r2[3])) + ((r2[4] + r2[5]) + (r2[6] + r2[7]));
         }
-        if (r < n) {
-            atomicAdd(a.ab_acc + blh(d, b, c0 + r, h) * 2, aa);
-            atomicAdd(a.ab_acc + blh(d, b, c0 + r, h) * 2 + 1, bb);
-            float4 *o = reinterpret_cast<float4 *>(a.dx_acc + blh(d, b, c0 + r, h) * P + p0);
+        if (mj == K - 1 && !*abort_s && t < n) {  // head hj complete
+            const size_t i0 = blh(d, b, c0 + t, hj);
+            float *acc_dst = (grp == 0 ? a.dwr_acc : a.dkap_acc) + i0 * K;
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                float4 v = o[q];
-                v.x += dx[4 * q]; v.y += dx[4 * q + 1]; v.z += dx[4 * q + 2]; v.w += dx[4 * q + 3];
-                o[q] = v;
+            for (int m = 0; m < KMAX; ++m)
+                if (m < K) acc_dst[m] += acc_h[m];
+            a.ab_acc[i0 * 2 + grp] = ab_h;
+            if (grp == 1) {
+                float4 *o = reinterpret_cast<float4 *>(a.dx_acc + i0 * P);
+#pragma unroll
+                for (int q = 0; q < 16; ++q) {
+                    float4 x4 = o[q];
+                    x4.x += dxr[4 * q]; x4.y += dxr[4 * q + 1]; x4.z += dxr[4 * q + 2]; x4.w += dxr[4 * q + 3];
+                    o[q] = x4;
+                }
+            }
+        }
+    };
+
+    for (int i = 0; i < nsteps; ++i) {
+        const int hh = i / K, m = i % K, h = h_first + hh, gb = i & 1, q = i % kStBuf;
+        bool prev_done = i == 0;
+        if (m == 0) {
+            // a new head: step i - 1 (the previous head's last) is read out with that head's
+            // coefficients first, then the coefficients of row t and its row of dY / X change
+            if (i > 0) {
+                readout(i - 1);
+                prev_done = true;
+            }
+            float dtv = 1.f, alv = 1.f, lmv = 1.f, wr[KMAX], ww[KMAX];
+            float tmax = 0.f;
+#pragma unroll
+            for (int k = 0; k < KMAX; ++k) {
+                const float tv = k < K ? a.tau[h * K + k] : 1.f;
+                itr[k] = k < K ? 1.f / tv : 0.f;
+                if (k < K) tmax = fmaxf(tmax, tv);
+            }
+            if (t < n) {
+                const size_t i0 = blh(d, b, c0 + t, h);
+                dtv = a.dt[i0];
+                alv = a.alpha[i0];
+                lmv = a.lam[i0];
+                load_weights(a.wr + i0 * K, K, wr);
+                load_weights(a.ww + i0 * K, K, ww);
+                const uint4 *src = reinterpret_cast<const uint4 *>((grp == 0 ? a.dy : a.x) + i0 * P);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) row[k] = src[k];
+            } else {
+#pragma unroll
+                for (int k = 0; k < KMAX; ++k) wr[k] = ww[k] = 0.f;
+#pragma unroll
+                for (int k = 0; k < 8; ++k) row[k] = make_uint4(0, 0, 0, 0);
+            }
+            const float log_cap = logf(64.f * tmax);
+            float e = 0.f;
+            if (t < n) {
+                bool cl;
+                e = token_rate(dtv, alv, lmv, log_cap, &cl);
+            }
+            const double Et = group_scan128(double(e), wsum);
+            if (grp == 0 && t == n - 1) *Eend_s = Et;
+            __syncthreads();
+            const double Eend = *Eend_s;
+#pragma unroll
+            for (int k = 0; k < KMAX; ++k) {
+                f_t[k] = s_t[k] = u_t[k] = fd_t[k] = 0.f;
+                if (k < K && t < n) {
+                    const float kp = -expm1f(-e * itr[k]) * ww[k];
+                    u_t[k] = expf(-float(Eend - Et) * itr[k]);
+                    s_t[k] = kp * u_t[k];
+                    fd_t[k] = expf(-float(Et) * itr[k]);
+                    f_t[k] = wr[k] * fd_t[k];
+                }
+                acc_h[k] = 0.f;
+            }
+            ab_h = 0.f;
+#pragma unroll
+            for (int p = 0; p < 64; ++p) dxr[p] = 0.f;
+        }
+        // generated operands of step i into buffer gb (step i - 2 has finished reading it)
+        {
+            float sc = 0.f;
+#pragma unroll
+            for (int k = 0; k < KMAX; ++k)
+                if (k == m) sc = grp == 0 ? f_t[k] : s_t[k];
+            unsigned char *dst = sG + gb * L.gen + grp * 16384 + t * 128;
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+                *reinterpret_cast<uint4 *>(dst + ((k ^ (t & 7)) * 16)) = scale_bf16x8(row[k], sc);
+        }
+        // this step's tiles: <dS_out,m, S_in,m> partials (the same swizzle in both tiles)
+        if (!*abort_s && !mbar_wait(&bars[q], (i / kStBuf) & 1)) *abort_s = 1;
+        {
+            const uint4 *ps = reinterpret_cast<const uint4 *>(sT + (2 * q) * L.tile);
+            const uint4 *pd = reinterpret_cast<const uint4 *>(sT + (2 * q + 1) * L.tile);
+            float acc = 0.f;
+            for (int k = tid; k < L.tile / 16; k += kStThreads) acc = dot_bf16x8(ps[k], pd[k], acc);
+            acc = warp_sum(acc);
+            if ((tid & 31) == 0) red[(i % 3) * 8 + w] = acc;
+        }
+        fence_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+        if (tid == 0 && !*abort_s) {
+            const uint32_t sS = smem_u32(sT + (2 * q) * L.tile), sD = smem_u32(sT + (2 * q + 1) * L.tile);
+            const uint32_t g1 = smem_u32(sG + gb * L.gen), g2 = g1 + 16384;
+            const uint32_t id64 = idesc_bf16(128, 64, false, false);
+            const uint32_t idN = idesc_bf16(128, N, false, true);
+            const uint32_t zc = colZU + 128 * gb;
+            for (int ks = 0; ks < N / 16; ++ks) {
+                const uint32_t ko = (ks / 4) * 16384 + (ks % 4) * 32, to = (ks / 4) * 8192 + (ks % 4) * 32;
+                mma_bf16(tmem + zc, desc_sw128(smem_u32(sC) + ko, 16, 1024), desc_sw128(sS + to, 16, 1024),
+                         id64, ks > 0);
+                mma_bf16(tmem + zc + 64, desc_sw128(smem_u32(sB) + ko, 16, 1024),
+                         desc_sw128(sD + to, 16, 1024), id64, ks > 0);
+            }
+            const bool acc0 = intra || i > 0;
+            for (int ks = 0; ks < 4; ++ks) {  // K = p
+                mma_bf16(tmem + colC, desc_sw128(g1 + ks * 32, 16, 1024), desc_sw128(sS + ks * 2048, 8192, 1024),
+                         idN, (acc0 || ks > 0) ? 1u : 0u);
+                mma_bf16(tmem + colB, desc_sw128(g2 + ks * 32, 16, 1024), desc_sw128(sD + ks * 2048, 8192, 1024),
+                         idN, (acc0 || ks > 0) ? 1u : 0u);
+            }
+            mma_commit(&bars[3 + gb]);
+        }
+        // step i - 1 is read out while the tensor cores run step i
+        if (!prev_done) readout(i - 1);
+    }
+    if (nsteps > 0) readout(nsteps - 1);
+    // the group's dC / dB into the float32 accumulators (group g takes n in [64 g, 64 g + 64))
+    tc_fence_after();
+    if (!*abort_s && grp < N / 64) {
+        const size_t gi = ((size_t(b) * d.L + c0 + min(t, n - 1)) * d.G + g) * N + grp * 64;
+        for (int n32 = 0; n32 < 64; n32 += 32) {
+            float vc[32], vb[32];
+            tmem_ld32(lane_base + colC + grp * 64 + n32, vc);
+            tmem_ld32(lane_base + colB + grp * 64 + n32, vb);
+            tmem_ld_wait();
+            if (t < n) {
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    atomicAdd(reinterpret_cast<float4 *>(a.dC_acc + gi + n32 + 4 * k),
+                              make_float4(vc[4 * k], vc[4 * k + 1], vc[4 * k + 2], vc[4 * k + 3]));
+                    atomicAdd(reinterpret_cast<float4 *>(a.dB_acc + gi + n32 + 4 * k),
+                              make_float4(vb[4 * k], vb[4 * k + 1], vb[4 * k + 2], vb[4 * k + 3]));
+                }
             }
         }
     }
@@ -555,301 +727,139 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (w == 0) tmem_dealloc(tmem, 512);
 }
 
-// ============================================================================= dC / dB
-struct DcdbSmem {
-    int s, gen, total;
-    __host__ __device__ DcdbSmem(int K, int N) {
-        s = (N / 64) * (K * TPS * 128);  // S_in / dS_out slice; also holds the B / C chunk
-        if (s < (N / 64) * 16384) s = (N / 64) * 16384;
-        gen = (K * TPS / 64) * 16384;    // generated [128][(m, p)] operand; also Gamma o H
-        if (gen < 2 * 16384) gen = 2 * 16384;
-        total = 2 * s + gen + 64 + 64;
+// ============================================================================= final
+// Float block scans of one value per thread over 128 threads: inclusive prefix, inclusive suffix
+// and total (no difference of two sums is ever formed).
+__device__ __forceinline__ void block_scans128(float v, float *pre, float *suf, float *tot,
+                                               float *sh /* [3][4] */) {
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    float p = v, q = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const float up = __shfl_up_sync(0xffffffffu, p, o);
+        const float dn = __shfl_down_sync(0xffffffffu, q, o);
+        if (lane >= o) p += up;
+        if (lane + o < 32) q += dn;
     }
-};
-
-__global__ void __launch_bounds__(kThreads, 1)
-    tc_bwd_dcdb(const __grid_constant__ CUtensorMap mapS, const __grid_constant__ CUtensorMap mapD,
-                const __grid_constant__ CUtensorMap mapB, const __grid_constant__ CUtensorMap mapC,
-                BwdArgs a) {
-    extern __shared__ unsigned char smem_raw[];
-    unsigned char *base = align1024(smem_raw);
-    const ScanDims &d = a.d;
-    const int K = d.K, N = d.N, P = d.P;
-    const DcdbSmem L(K, N);
-    unsigned char *sS = base, *sD = sS + L.s, *sG = sD + L.s;
-    double *wsum = reinterpret_cast<double *>(sG + L.gen);
-    uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 4);  // tma, mma
-    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 2);
-    volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
-    __shared__ float itau[32];
-    __shared__ double Eend_s;
-
-    const int tid = threadIdx.x, w = tid >> 5, t = tid;
-    const int hg = blockIdx.x, c = blockIdx.y, b = blockIdx.z;
-    const int h_first = hg * a.hg;
-    const int g = h_first / (d.H / d.G);
-    const int c0 = c * TQ, n = min(TQ, d.L - c0);
-    const uint32_t KP = uint32_t(K * TPS);  // contraction length per P-slice
-    const uint32_t colC = 0, colB = 128;
-
-    if (tid == 0) {
-        mbar_init(&bars[0], 1);
-        mbar_init(&bars[1], 1);
-        *abort_s = 0;
-        fence_barrier_init();
-    }
-    if (w == 0) tmem_alloc_once(tslot, 256);
-    tc_fence_before();
+    if (lane == 31) sh[w] = p;  // warp totals
     __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem = *tslot;
-    const uint32_t lane_base = tmem + (uint32_t(w * 32) << 16);
-    uint32_t tma_phase = 0, mma_phase = 0;
-    bool first = true;  // first MMA into the accumulators overwrites them
-
-    // helpers ---------------------------------------------------------------
-    auto wait_mma = [&]() {
-        if (!mbar_wait(&bars[1], mma_phase)) *abort_s = 1;
-        mma_phase ^= 1;
-    };
-
-    // head-summed intra term, once per chunk and B/C group (by the group's first block):
-    // dC = M_H B, dB = M_H^T C
-    if (h_first % (d.H / d.G) == 0) {
-        if (tid == 0) {
-            mbar_arrive_expect_tx(&bars[0], uint32_t(2 * (N / 64) * 16384));
-            for (int jb = 0; jb < N / 64; ++jb) {
-                tma_load_3d(sS + jb * 16384, &mapB, &bars[0], g * N + 64 * jb, c0, b);
-                tma_load_3d(sD + jb * 16384, &mapC, &bars[0], g * N + 64 * jb, c0, b);
-            }
-        }
-        const float *mrow = a.mh_total + (((size_t(b) * d.nc + c) * d.G + g) * TQ + t) * TQ;
-        for (int k8 = 0; k8 < TQ; k8 += 8) {
-            float v[8];
+    float before = 0.f, after = 0.f;
 #pragma unroll
-            for (int i = 0; i < 8; ++i) v[i] = mrow[k8 + i];
-            const int c8 = (k8 & 63) >> 3;
-            store_bf16x8(sG + (k8 >> 6) * 16384 + t * 128 + ((c8 ^ (t & 7)) * 16), v);
-        }
-        fence_async_smem();
-        __syncthreads();
-        if (tid == 0) {
-            if (!mbar_wait(&bars[0], tma_phase)) {
-                *abort_s = 1;
-            } else {
-                tc_fence_after();
-                const uint32_t idC = idesc_bf16(128, N, false, true);
-                const uint32_t idB = idesc_bf16(128, N, true, true);
-                for (int ks = 0; ks < TQ / 16; ++ks) {
-                    // dC[t, n] += sum_k M[t, k] B[k, n]
-                    mma_bf16(tmem + colC,
-                             desc_sw128(smem_u32(sG) + (ks / 4) * 16384 + (ks % 4) * 32, 16, 1024),
-                             desc_sw128(smem_u32(sS) + ks * 2048, 16384, 1024), idC, ks > 0);
-                    // dB[k, n] += sum_t M[t, k] C[t, n]
-                    mma_bf16(tmem + colB, desc_sw128(smem_u32(sG) + ks * 2048, 16384, 1024),
-                             desc_sw128(smem_u32(sD) + ks * 2048, 16384, 1024), idB, ks > 0);
-                }
-                mma_commit(&bars[1]);
-            }
-        }
-        tma_phase ^= 1;
-        __syncthreads();
-        if (!*abort_s) wait_mma();
-        __syncthreads();
-        first = false;
+    for (int i = 0; i < 4; ++i) {
+        if (i < w) before += sh[i];
+        if (i > w) after += sh[i];
     }
-
-    for (int hh = 0; hh < a.hg && !*abort_s; ++hh) {
-        const int h = h_first + hh;
-        if (tid < K) itau[tid] = 1.f / a.tau[h * K + tid];
-        __syncthreads();
-        const float log_cap = head_log_cap(a.tau, h, K);
-        float e = 0.f;
-        if (t < n) {
-            const size_t i = blh(d, b, c0 + t, h);
-            bool cl;
-            e = token_rate(a.dt[i], a.alpha[i], a.lam[i], log_cap, &cl);
-        }
-        const double Et = block_scan128(double(e), wsum);
-        if (t == n - 1) Eend_s = Et;
-        __syncthreads();
-        const double Eend = Eend_s;
-        float f_t[KMAX], s_t[KMAX];
-#pragma unroll
-        for (int m = 0; m < KMAX; ++m) {
-            f_t[m] = s_t[m] = 0.f;
-            if (m < K && t < n) {
-                const size_t wi = blh(d, b, c0 + t, h) * K + m;
-                f_t[m] = to_f(a.wr[wi]) * expf(-float(Et) * itau[m]);
-                s_t[m] = -expm1f(-e * itau[m]) * to_f(a.ww[wi]) * expf(-float(Eend - Et) * itau[m]);
-            }
-        }
-        const int srow = int(((size_t(b) * d.H + h) * d.nc + c) * K);
-        for (int ps = 0; ps < P / TPS && !*abort_s; ++ps) {
-            const int p0 = ps * TPS;
-            if (tid == 0) {
-                mbar_arrive_expect_tx(&bars[0], uint32_t(2 * (N / 64) * (K * TPS * 128)));
-                for (int jb = 0; jb < N / 64; ++jb) {
-                    tma_load_3d(sS + jb * (K * TPS * 128), &mapS, &bars[0], 64 * jb, p0, srow);
-                    tma_load_3d(sD + jb * (K * TPS * 128), &mapD, &bars[0], 64 * jb, p0, srow);
-                }
-            }
-            // dC += (f o dy)[t, (m, p)] S_in[(m, p), n]
-            for (int pass = 0; pass < 2; ++pass) {
-                float src[32];
-                if (t < n)
-                    load_bf16x32((pass == 0 ? a.dy : a.x) + blh(d, b, c0 + t, h) * P + p0, src);
-                else
-#pragma unroll
-                    for (int p = 0; p < 32; ++p) src[p] = 0.f;
-#pragma unroll
-                for (int m = 0; m < KMAX; ++m) {
-                    if (m >= K) break;
-                    const float cm = pass == 0 ? f_t[m] : s_t[m];
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        float v[8];
-#pragma unroll
-                        for (int i = 0; i < 8; ++i) v[i] = cm * src[8 * q + i];
-                        const int kidx = m * TPS + 8 * q;  // (m, p) index of the first element
-                        const int c8 = (kidx & 63) >> 3;
-                        store_bf16x8(sG + (kidx >> 6) * 16384 + t * 128 + ((c8 ^ (t & 7)) * 16), v);
-                    }
-                }
-                fence_async_smem();
-                tc_fence_before();
-                __syncthreads();
-                tc_fence_after();
-                if (tid == 0) {
-                    bool ok = true;
-                    if (pass == 0 && !mbar_wait(&bars[0], tma_phase)) ok = false;
-                    if (!ok) {
-                        *abort_s = 1;
-                    } else {
-                        tc_fence_after();
-                        const uint32_t id = idesc_bf16(128, N, false, true);
-                        unsigned char *bt = pass == 0 ? sS : sD;
-                        for (int ks = 0; ks < int(KP) / 16; ++ks)
-                            mma_bf16(tmem + (pass == 0 ? colC : colB),
-                                     desc_sw128(smem_u32(sG) + (ks / 4) * 16384 + (ks % 4) * 32, 16, 1024),
-                                     desc_sw128(smem_u32(bt) + ks * 2048, K * TPS * 128, 1024), id,
-                                     (first && ks == 0) ? 0u : 1u);
-                        mma_commit(&bars[1]);
-                    }
-                }
-                __syncthreads();
-                if (!*abort_s) wait_mma();  // the generated operand buffer is reused next
-                __syncthreads();
-                if (pass == 1) first = false;  // both accumulators now hold data
-            }
-            tma_phase ^= 1;
-        }
-    }
-    // accumulate the group's dC / dB into the fp32 outputs (every lane takes part in the
-    // warp-collective tensor-memory loads; rows beyond the sequence end store nothing)
-    tc_fence_after();
-    if (!*abort_s) {
-        const size_t gi = ((size_t(b) * d.L + c0 + min(t, n - 1)) * d.G + g) * N;
-        for (int n32 = 0; n32 < N; n32 += 32) {
-            float vc[32], vb[32];
-            tmem_ld32(lane_base + colC + n32, vc);
-            tmem_ld32(lane_base + colB + n32, vb);
-            tmem_ld_wait();
-            if (t < n) {
-#pragma unroll
-                for (int q = 0; q < 8; ++q) {
-                    atomicAdd(reinterpret_cast<float4 *>(a.dC_acc + gi + n32 + 4 * q),
-                              make_float4(vc[4 * q], vc[4 * q + 1], vc[4 * q + 2], vc[4 * q + 3]));
-                    atomicAdd(reinterpret_cast<float4 *>(a.dB_acc + gi + n32 + 4 * q),
-                              make_float4(vb[4 * q], vb[4 * q + 1], vb[4 * q + 2], vb[4 * q + 3]));
-                }
-            }
-        }
-    }
-    if (*abort_s && tid == 0) atomicExch(a.err, kTimeoutCode);
-    tc_fence_before();
+    *pre = p + before;
+    *suf = q + after;
+    *tot = (sh[0] + sh[1]) + (sh[2] + sh[3]);
     __syncthreads();
-    if (w == 0) tmem_dealloc(tmem, 256);
 }
 
-// ============================================================================= final
+// One CTA per (b, h, chunk): per-position gradients of Delta, alpha, lambda, w_write, w_read
+// (from the accumulated mode terms and rho <dS_t, S_{t-1}>), then dx = dx_acc + D dy as bf16 and
+// the dD partial, one warp per row so that every access is a contiguous row segment.
 __global__ void __launch_bounds__(kThreads) tc_bwd_final(BwdArgs a) {
     const ScanDims &d = a.d;
     const int K = d.K, P = d.P;
     const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z, t = threadIdx.x;
+    const int lane = t & 31, w = t >> 5;
     const int c0 = c * TQ, n = min(TQ, d.L - c0);
-    __shared__ double wsum[4];
-    __shared__ float itau[32];
-    __shared__ double tot_s[2];
+    __shared__ float itau[32], tau_sh[32];
+    __shared__ float sh[4];
     __shared__ float red[4];
-    if (t < K) itau[t] = 1.f / a.tau[h * K + t];
-    __syncthreads();
-    const float log_cap = head_log_cap(a.tau, h, K);
-    float e = 0.f;
-    bool cl = false;
-    const size_t i = (t < n) ? blh(d, b, c0 + t, h) : 0;
-    if (t < n) e = token_rate(a.dt[i], a.alpha[i], a.lam[i], log_cap, &cl);
-    const double Et = block_scan128(double(e), wsum);
-    const float av = t < n ? a.ab_acc[i * 2] : 0.f;
-    const float bv = t < n ? a.ab_acc[i * 2 + 1] : 0.f;
-    const double pa = block_scan128(double(av), wsum);  // inclusive prefix of a
-    const double pb = block_scan128(double(bv), wsum);  // inclusive prefix of b
-    if (t == n - 1) {
-        tot_s[0] = pa;
-        tot_s[1] = Et;
+    if (t < K) {
+        const float tv = a.tau[h * K + t];
+        tau_sh[t] = tv;
+        itau[t] = 1.f / tv;
     }
-    __syncthreads();
-    const double Eend = tot_s[1];
-    float cprime = 0.f;
-    for (int m = 0; m < K; ++m)
-        cprime = fmaf(expf(-float(Eend) * itau[m]) * itau[m],
-                      a.cdot[((size_t(b) * d.H + h) * d.nc + c) * K + m], cprime);
-    float dd = 0.f;
+    const size_t i = (t < n) ? blh(d, b, c0 + t, h) : 0;
+    float dtv = 1.f, alv = 1.f, lmv = 1.f, av = 0.f, bv = 0.f, rc = 0.f;
+    float ww[KMAX], dkv[KMAX], dwv[KMAX];
+#pragma unroll
+    for (int m = 0; m < KMAX; ++m) ww[m] = dkv[m] = dwv[m] = 0.f;
     if (t < n) {
-        const double suf_a = tot_s[0] - (pa - av);
-        const double pre_b = pb - bv;
-        const float R = float(suf_a + pre_b) + cprime + a.rect[i];
-        float de = -R;
-        for (int m = 0; m < K; ++m) {
-            const float z = e * itau[m];
-            const float rho = expf(-z), omr = -expm1f(-z);
-            const float ww = to_f(a.ww[i * K + m]);
-            const float dk = a.dkap_acc[i * K + m];
-            de = fmaf(dk * rho * ww, itau[m], de);
-            a.dwr[i * K + m] = from_f<bf16>(a.dwr_acc[i * K + m]);
-            a.dww[i * K + m] = from_f<bf16>(dk * omr);
-        }
-        const float al = a.alpha[i], lm = a.lam[i], dtv = a.dt[i];
-        const float ge = cl ? 0.f : de * e;
-        a.ddt[i] = ge / dtv;
-        a.dlam[i] = ge / (al * lm);
-        a.dalpha[i] = -ge * logf(lm) / (al * al);
-        const float Dh = a.D[h];
-        for (int p32 = 0; p32 < P; p32 += 32) {
-            float dyv[32], xv[32];
-            load_bf16x32(a.dy + i * P + p32, dyv);
-            load_bf16x32(a.x + i * P + p32, xv);
-            const float4 *src = reinterpret_cast<const float4 *>(a.dx_acc + i * P + p32);
-            uint4 *o = reinterpret_cast<uint4 *>(a.dx + i * P + p32);
+        dtv = a.dt[i];
+        alv = a.alpha[i];
+        lmv = a.lam[i];
+        const float2 ab = *reinterpret_cast<const float2 *>(a.ab_acc + i * 2);
+        av = ab.x;
+        bv = ab.y;
+        rc = a.rect[i];
+        load_weights(a.ww + i * K, K, ww);
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const float4 u0 = src[2 * q], u1 = src[2 * q + 1];
-                const float v[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
-                float r8[8];
-#pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    r8[k] = v[k] + Dh * dyv[8 * q + k];
-                    dd = fmaf(dyv[8 * q + k], xv[8 * q + k], dd);
-                }
-                o[q] = make_uint4(pack_bf16x2(r8[0], r8[1]), pack_bf16x2(r8[2], r8[3]),
-                                  pack_bf16x2(r8[4], r8[5]), pack_bf16x2(r8[6], r8[7]));
+        for (int q = 0; q < KMAX / 4; ++q) {
+            if (4 * q < K) {
+                const float4 u = *reinterpret_cast<const float4 *>(a.dkap_acc + i * K + 4 * q);
+                const float4 v = *reinterpret_cast<const float4 *>(a.dwr_acc + i * K + 4 * q);
+                dkv[4 * q] = u.x; dkv[4 * q + 1] = u.y; dkv[4 * q + 2] = u.z; dkv[4 * q + 3] = u.w;
+                dwv[4 * q] = v.x; dwv[4 * q + 1] = v.y; dwv[4 * q + 2] = v.z; dwv[4 * q + 3] = v.w;
             }
         }
     }
-    dd = warp_sum(dd);
-    if ((t & 31) == 0) red[t >> 5] = dd;
     __syncthreads();
-    if (t == 0) atomicAdd(a.dD + h, red[0] + red[1] + red[2] + red[3]);
+    float tmax = 0.f;
+    for (int m = 0; m < K; ++m) tmax = fmaxf(tmax, tau_sh[m]);
+    const float log_cap = logf(64.f * tmax);
+    float e = 0.f;
+    bool cl = false;
+    if (t < n) e = token_rate(dtv, alv, lmv, log_cap, &cl);
+    float pe, se, Eend;  // chunk total of e (the log-decay across the chunk)
+    block_scans128(e, &pe, &se, &Eend, sh);
+    float pa, suf_a, ta, pb, sb, tb;
+    block_scans128(av, &pa, &suf_a, &ta, sh);  // suffix of a, inclusive
+    block_scans128(bv, &pb, &sb, &tb, sh);     // prefix of b, exclusive = inclusive - own
+    float cprime = 0.f;
+    for (int m = 0; m < K; ++m)
+        cprime = fmaf(expf(-Eend * itau[m]) * itau[m], a.cdot[((size_t(b) * d.H + h) * d.nc + c) * K + m], cprime);
+    if (t < n) {
+        const float pre_b = pb - bv;
+        const float R = (suf_a + pre_b) + cprime + rc;
+        float de = -R;
+        float dww[KMAX];
+#pragma unroll
+        for (int m = 0; m < KMAX; ++m) {
+            dww[m] = 0.f;
+            if (m < K) {
+                const float z = e * itau[m];
+                const float rho = expf(-z), omr = -expm1f(-z);
+                de = fmaf(dkv[m] * rho * ww[m], itau[m], de);
+                dww[m] = dkv[m] * omr;
+            }
+        }
+        if (K == 8) {
+            *reinterpret_cast<uint4 *>(a.dwr + i * K) =
+                make_uint4(pack_bf16x2(dwv[0], dwv[1]), pack_bf16x2(dwv[2], dwv[3]), pack_bf16x2(dwv[4], dwv[5]),
+                           pack_bf16x2(dwv[6], dwv[7]));
+            *reinterpret_cast<uint4 *>(a.dww + i * K) =
+                make_uint4(pack_bf16x2(dww[0], dww[1]), pack_bf16x2(dww[2], dww[3]), pack_bf16x2(dww[4], dww[5]),
+                           pack_bf16x2(dww[6], dww[7]));
+        } else {
+            *reinterpret_cast<uint2 *>(a.dwr + i * K) = make_uint2(pack_bf16x2(dwv[0], dwv[1]), pack_bf16x2(dwv[2], dwv[3]));
+            *reinterpret_cast<uint2 *>(a.dww + i * K) = make_uint2(pack_bf16x2(dww[0], dww[1]), pack_bf16x2(dww[2], dww[3]));
+        }
+        const float ge = cl ? 0.f : de * e;
+        a.ddt[i] = ge / dtv;
+        a.dlam[i] = ge / (alv * lmv);
+        a.dalpha[i] = -ge * logf(lmv) / (alv * alv);
+    }
+    // dx = dx_acc + D dy (bf16) and sum dy x, one warp per row, two p per lane
+    const float Dh = a.D[h];
+    float dd = 0.f;
+#pragma unroll 4
+    for (int r = w; r < n; r += 4) {
+        const size_t i0 = blh(d, b, c0 + r, h) * P;
+        for (int p = 2 * lane; p < P; p += 64) {
+            const float2 acc = *reinterpret_cast<const float2 *>(a.dx_acc + i0 + p);
+            const float2 dyv = bf16x2_to_float2(*reinterpret_cast<const uint32_t *>(a.dy + i0 + p));
+            const float2 xv = bf16x2_to_float2(*reinterpret_cast<const uint32_t *>(a.x + i0 + p));
+            *reinterpret_cast<uint32_t *>(a.dx + i0 + p) = pack_bf16x2(fmaf(Dh, dyv.x, acc.x), fmaf(Dh, dyv.y, acc.y));
+            dd = fmaf(dyv.x, xv.x, fmaf(dyv.y, xv.y, dd));
+        }
+    }
+    dd = warp_sum(dd);
+    if (lane == 0) red[w] = dd;
+    __syncthreads();
+    if (t == 0) atomicAdd(a.dD + h, (red[0] + red[1]) + (red[2] + red[3]));
 }
 
 __global__ void f32_to_bf16_tc(const float *__restrict__ in, bf16 *__restrict__ out, size_t n) {
@@ -857,9 +867,10 @@ __global__ void f32_to_bf16_tc(const float *__restrict__ in, bf16 *__restrict__ 
         out[i] = __float2bfloat16_rn(in[i]);
 }
 
+// Heads per CTA of tc_bwd_state: a divisor of the heads of one B/C group, at most 4.
 int pick_hg(const ScanDims &d) {
     const int hpg = d.H / d.G;
-    for (int hg = 16; hg >= 1; --hg)
+    for (int hg = 4; hg >= 1; --hg)
         if (hpg % hg == 0) return hg;
     return 1;
 }
@@ -896,12 +907,9 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
                         bool reuse_states, cudaStream_t st) {
     cudaError_t e;
     const size_t ngn = size_t(d.B) * d.L * d.G * d.N;
-    const size_t blh_ = size_t(d.B) * d.L * d.H;
     if ((e = cudaMemsetAsync(p.dD, 0, sizeof(float) * d.H, st))) return e;
     if ((e = cudaMemsetAsync(ws.dB_acc, 0, sizeof(float) * ngn, st))) return e;
     if ((e = cudaMemsetAsync(ws.dC_acc, 0, sizeof(float) * ngn, st))) return e;
-    if ((e = cudaMemsetAsync(ws.cdot, 0, sizeof(float) * d.B * d.H * d.nc * d.K, st))) return e;
-    if ((e = cudaMemsetAsync(ws.ab_acc, 0, sizeof(float) * blh_ * 2, st))) return e;
     if ((e = cudaMemsetAsync(ws.mh_total, 0, sizeof(float) * d.B * d.nc * d.G * TQ * TQ, st))) return e;
     if (!reuse_states &&
         (e = tc_state_pass_launch(d, false, p.x, p.Bm, p.ww, p.dt, p.alpha, p.lam, p.tau, p.h0,
@@ -919,9 +927,9 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
         !tc_make_map3(&mapX, p.x, HP, d.L, d.B, HP * 2, uint64_t(d.L) * HP * 2, 64, TQ, 1) ||
         !tc_make_map3(&mapDY, p.dy, HP, d.L, d.B, HP * 2, uint64_t(d.L) * HP * 2, 64, TQ, 1) ||
         !tc_make_map3(&mapS, ws.S_in, d.N, d.P, srows, uint64_t(d.N) * 2, uint64_t(d.P) * d.N * 2, 64,
-                      TPS, d.K) ||
+                      64, 1) ||
         !tc_make_map3(&mapD, ws.dS_out, d.N, d.P, srows, uint64_t(d.N) * 2, uint64_t(d.P) * d.N * 2, 64,
-                      TPS, d.K))
+                      64, 1))
         return cudaErrorInvalidValue;
     BwdArgs a;
     a.d = d;
@@ -946,18 +954,10 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
         if ((e = cudaGetLastError())) return e;
     }
     {
-        const size_t smem = InterSmem(d.K, d.N).total + 1024;
-        cudaFuncSetAttribute(tc_bwd_inter, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-        trace_begin("bwd_inter_tc", st);
-        tc_bwd_inter<<<dim3(d.H * (d.P / TPS), d.nc, d.B), kThreads, smem, st>>>(mapC, mapB, mapS, mapD, a);
-        trace_end(st);
-        if ((e = cudaGetLastError())) return e;
-    }
-    {
-        const size_t smem = DcdbSmem(d.K, d.N).total + 1024;
-        cudaFuncSetAttribute(tc_bwd_dcdb, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-        trace_begin("bwd_dcdb_tc", st);
-        tc_bwd_dcdb<<<dim3(d.H / a.hg, d.nc, d.B), kThreads, smem, st>>>(mapS, mapD, mapB, mapC, a);
+        const size_t smem = StSmem(d.N).total + 1024;
+        cudaFuncSetAttribute(tc_bwd_state, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+        trace_begin("bwd_state_tc", st);
+        tc_bwd_state<<<dim3(d.H / a.hg, d.nc, d.B), kStThreads, smem, st>>>(mapC, mapB, mapS, mapD, a);
         trace_end(st);
         if ((e = cudaGetLastError())) return e;
     }
