@@ -70,6 +70,7 @@ struct TcBwdWorkspace {
     void *S_in, *dS_out;                     // bf16 per-chunk states
     float *dx_acc, *dwr_acc, *dkap_acc;      // [B,L,H,P], [B,L,H,K] x 2
     float *ab_acc, *rect, *cdot, *mh_total;  // [B,L,H,2], [B,L,H], [B,H,nc,K], [B,nc,G,Q,Q]
+    float *coef;                             // [B,L,H,4,K]: f, s, u, exp(-E/tau)
     float *dB_acc, *dC_acc;                  // [B,L,G,N] x 2
 };
 size_t tc_bwd_workspace_bytes(const ScanDims &d, TcBwdWorkspace *layout, char *base);

@@ -45,6 +45,7 @@ struct BwdArgs {
     const float *dt, *alpha, *lam, *tau, *D;
     const bf16 *S_in, *dS_out;
     float *dx_acc, *dwr_acc, *dkap_acc, *ab_acc, *rect, *cdot, *mh_total, *dB_acc, *dC_acc;
+    float *coef;  // per position: f, s, u, exp(-E/tau) for every mode [B, L, H, 4, K]
     bf16 *dx, *dwr, *dww;
     float *ddt, *dalpha, *dlam, *dD;
     int *err;
@@ -182,16 +183,42 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     if (grp == 0) E_s[t] = Et2;
     float l2r[KMAX];  // log2(e) / tau per mode, in registers
 #pragma unroll
+    float kap_t[KMAX];
     for (int m = 0; m < KMAX; ++m) {
         l2r[m] = m < K ? l2t[m] : 0.f;
         float kp = 0.f;
         if (m < K && t < n) kp = -expm1f(-e / tau_s[m]) * ww_t[m];
+        kap_t[m] = kp;
         if (grp == 0) {
             wr_s[t * KMAX + m] = wr_t[m];
             kap_s[t * KMAX + m] = kp;
         }
     }
     __syncthreads();
+    if (grp == 1 && t < n) {
+        // the per-position mode coefficients of the state terms, for tc_bwd_state:
+        // f = w_read exp(-E/tau), s = kappa u, u = exp(-(E_end - E)/tau), exp(-E/tau)
+        const float dEnd = diff_f2(E_s[n - 1], Et2);
+        float fv[KMAX], sv[KMAX], uv[KMAX], dv[KMAX];
+#pragma unroll
+        for (int m = 0; m < KMAX; ++m) {
+            const float it = m < K ? 1.f / tau_s[m] : 0.f;
+            dv[m] = expf(-Et2.x * it);
+            uv[m] = expf(-dEnd * it);
+            fv[m] = wr_t[m] * dv[m];
+            sv[m] = kap_t[m] * uv[m];
+        }
+        float4 *o = reinterpret_cast<float4 *>(a.coef + blh(d, b, c0 + t, h) * 4 * K);
+#pragma unroll
+        for (int q = 0; q < KMAX / 4; ++q) {
+            if (4 * q < K) {
+                o[q] = make_float4(fv[4 * q], fv[4 * q + 1], fv[4 * q + 2], fv[4 * q + 3]);
+                o[K / 4 + q] = make_float4(sv[4 * q], sv[4 * q + 1], sv[4 * q + 2], sv[4 * q + 3]);
+                o[2 * K / 4 + q] = make_float4(uv[4 * q], uv[4 * q + 1], uv[4 * q + 2], uv[4 * q + 3]);
+                o[3 * K / 4 + q] = make_float4(dv[4 * q], dv[4 * q + 1], dv[4 * q + 2], dv[4 * q + 3]);
+            }
+        }
+    }
     if (tid == 0) {
         if (!mbar_wait(&bars[0], 0)) {
             *abort_s = 1;
@@ -391,7 +418,7 @@ struct StSmem {
         cb = (N / 64) * 16384;   // one of C / B: [t][n]
         tile = (N / 64) * 8192;  // one S_in or dS_out mode tile: [p = 64][n], 64-wide n atoms
         gen = 2 * 16384;         // f o dY and s o X: [t][p] each; two buffers (the first holds M_H)
-        total = 2 * cb + kStBuf * 2 * tile + 2 * gen + 256;
+        total = 2 * cb + kStBuf * 2 * tile + 2 * gen + 384;
     }
 };
 
@@ -427,14 +454,13 @@ __global__ void __launch_bounds__(kStThreads, 1)
     const StSmem L(N);
     unsigned char *sC = base, *sB = sC + L.cb, *sT = sB + L.cb;
     unsigned char *sG = sT + kStBuf * 2 * L.tile;             // [buf][f o dY | s o X]
-    // per-warp partial dots of steps i mod 3: step i - 1 is summed by thread 0 after the
-    // barrier of step i, while other warps may already write step i + 1
-    float *red = reinterpret_cast<float *>(sG + 2 * L.gen);   // [3][8]
-    double *wsum = reinterpret_cast<double *>(red + 24);      // [8]
-    double *Eend_s = wsum + 8;                                // [1]
-    // bars: 0..2 tile buffers | 3, 4 MMA of step parity | 5 C, B | 6 intra MMA
+    float *itau_s = reinterpret_cast<float *>(sG + 2 * L.gen);  // [hg][K] 1 / tau
+    double *wsum = reinterpret_cast<double *>(itau_s + 32);     // [8]
+    double *Eend_s = wsum + 8;                                  // [1]
+    // bars: 0..2 tile buffers | 3, 4 MMA of step parity | 5 C, B | 6 intra MMA |
+    //       7, 8 generated operands of step parity written (all 256 threads arrive)
     uint64_t *bars = reinterpret_cast<uint64_t *>(Eend_s + 2);
-    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 7);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 9);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
 
     const int tid = threadIdx.x, grp = tid >> 7, t = tid & 127, w = tid >> 5, w4 = w & 3;
@@ -448,10 +474,13 @@ __global__ void __launch_bounds__(kStThreads, 1)
 
     if (tid == 0) {
         for (int i = 0; i < 7; ++i) mbar_init(&bars[i], 1);
+        mbar_init(&bars[7], kStThreads);
+        mbar_init(&bars[8], kStThreads);
         *abort_s = 0;
         fence_barrier_init();
     }
     if (w == 0) tmem_alloc_once(tslot, 512);
+    if (tid < a.hg * K) itau_s[tid] = 1.f / a.tau[h_first * K + tid];
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -509,12 +538,13 @@ __global__ void __launch_bounds__(kStThreads, 1)
     }
     if (!*abort_s && !mbar_wait(&bars[5], 0)) *abort_s = 1;      // C and B are read below
 
-    float f_t[KMAX], s_t[KMAX], u_t[KMAX], fd_t[KMAX], itr[KMAX];
+    // mode coefficients of row t: group 0 cA = f, cB = exp(-E/tau); group 1 cA = s, cB = u
+    float cA[KMAX], cB[KMAX];
     uint4 row[8];     // group 0: dY row (64 p), group 1: X row
     float dxr[64];    // group 1: inter-chunk dx of this row, current head
     float acc_h[KMAX], ab_h = 0.f;  // group 0: dw_read and a; group 1: dkappa and b
 #pragma unroll
-    for (int m = 0; m < KMAX; ++m) f_t[m] = s_t[m] = u_t[m] = fd_t[m] = itr[m] = acc_h[m] = 0.f;
+    for (int m = 0; m < KMAX; ++m) cA[m] = cB[m] = acc_h[m] = 0.f;
 #pragma unroll
     for (int q = 0; q < 8; ++q) row[q] = make_uint4(0, 0, 0, 0);
 #pragma unroll
@@ -531,8 +561,8 @@ __global__ void __launch_bounds__(kStThreads, 1)
             float sj = 0.f;
 #pragma unroll
             for (int m = 0; m < KMAX; ++m)
-                if (m == mj) sj = s_t[m];
-            float dotv = 0.f;
+                if (m == mj) sj = cA[m];
+            float dp[4] = {0.f, 0.f, 0.f, 0.f};  // independent partial sums
 #pragma unroll
             for (int half = 0; half < 2; ++half) {
                 float zv[32];
@@ -545,7 +575,7 @@ __global__ void __launch_bounds__(kStThreads, 1)
 #pragma unroll
                     for (int k = 0; k < 4; ++k) {
                         const float2 f = bf16x2_to_float2(rr[k]);
-                        dotv = fmaf(f.x, zv[8 * q + 2 * k], fmaf(f.y, zv[8 * q + 2 * k + 1], dotv));
+                        dp[k] = fmaf(f.x, zv[8 * q + 2 * k], fmaf(f.y, zv[8 * q + 2 * k + 1], dp[k]));
                     }
                 }
                 if (grp == 1) {
@@ -553,39 +583,28 @@ __global__ void __launch_bounds__(kStThreads, 1)
                     for (int p = 0; p < 32; ++p) dxr[half * 32 + p] = fmaf(sj, zv[p], dxr[half * 32 + p]);
                 }
             }
+            const float dotv = (dp[0] + dp[1]) + (dp[2] + dp[3]);
 #pragma unroll
             for (int m = 0; m < KMAX; ++m) {
-                if (m == mj) {
-                    if (grp == 0) {
-                        acc_h[m] = fd_t[m] * dotv;                 // dw_read (inter)
-                        ab_h = fmaf(f_t[m] * dotv, itr[m], ab_h);  // a
-                    } else {
-                        acc_h[m] = u_t[m] * dotv;                  // dkappa (inter)
-                        ab_h = fmaf(s_t[m] * dotv, itr[m], ab_h);  // b
-                    }
+                if (m == mj) {  // group 0: dw_read (inter) and a; group 1: dkappa (inter) and b
+                    acc_h[m] = cB[m] * dotv;
+                    ab_h = fmaf(cA[m] * dotv, itau_s[(j / K) * K + m], ab_h);
                 }
             }
         }
-        if (tid == 0) {
-            const float *r2 = red + (j % 3) * 8;
-            a.cdot[((size_t(b) * d.H + hj) * d.nc + c) * K + mj] =
-                ((r2[0] + r2[1]) + (r2[2] + r2[3])) + ((r2[4] + r2[5]) + (r2[6] + r2[7]));
-        }
-        if (mj == K - 1 && !*abort_s && t < n) {  // head hj complete
+        if (mj == K - 1 && !*abort_s && t < n) {  // head hj complete: reductions, nothing waits
             const size_t i0 = blh(d, b, c0 + t, hj);
-            float *acc_dst = (grp == 0 ? a.dwr_acc : a.dkap_acc) + i0 * K;
+            float4 *acc_dst = reinterpret_cast<float4 *>((grp == 0 ? a.dwr_acc : a.dkap_acc) + i0 * K);
 #pragma unroll
-            for (int m = 0; m < KMAX; ++m)
-                if (m < K) acc_dst[m] += acc_h[m];
+            for (int q = 0; q < KMAX / 4; ++q)
+                if (4 * q < K)
+                    atomicAdd(acc_dst + q, make_float4(acc_h[4 * q], acc_h[4 * q + 1], acc_h[4 * q + 2], acc_h[4 * q + 3]));
             a.ab_acc[i0 * 2 + grp] = ab_h;
             if (grp == 1) {
                 float4 *o = reinterpret_cast<float4 *>(a.dx_acc + i0 * P);
 #pragma unroll
-                for (int q = 0; q < 16; ++q) {
-                    float4 x4 = o[q];
-                    x4.x += dxr[4 * q]; x4.y += dxr[4 * q + 1]; x4.z += dxr[4 * q + 2]; x4.w += dxr[4 * q + 3];
-                    o[q] = x4;
-                }
+                for (int q = 0; q < 16; ++q)
+                    atomicAdd(o + q, make_float4(dxr[4 * q], dxr[4 * q + 1], dxr[4 * q + 2], dxr[4 * q + 3]));
             }
         }
     };
@@ -600,51 +619,29 @@ __global__ void __launch_bounds__(kStThreads, 1)
                 readout(i - 1);
                 prev_done = true;
             }
-            float dtv = 1.f, alv = 1.f, lmv = 1.f, wr[KMAX], ww[KMAX];
-            float tmax = 0.f;
 #pragma unroll
             for (int k = 0; k < KMAX; ++k) {
-                const float tv = k < K ? a.tau[h * K + k] : 1.f;
-                itr[k] = k < K ? 1.f / tv : 0.f;
-                if (k < K) tmax = fmaxf(tmax, tv);
+                cA[k] = cB[k] = 0.f;
+                acc_h[k] = 0.f;
             }
-            if (t < n) {
+            if (t < n) {  // coefficients of this row from tc_bwd_intra; group 0: f, exp(-E/tau); 1: s, u
                 const size_t i0 = blh(d, b, c0 + t, h);
-                dtv = a.dt[i0];
-                alv = a.alpha[i0];
-                lmv = a.lam[i0];
-                load_weights(a.wr + i0 * K, K, wr);
-                load_weights(a.ww + i0 * K, K, ww);
+                const float4 *cf = reinterpret_cast<const float4 *>(a.coef + i0 * 4 * K);
+#pragma unroll
+                for (int q = 0; q < KMAX / 4; ++q) {
+                    if (4 * q < K) {
+                        const float4 v0 = cf[(grp == 0 ? 0 : 1) * (K / 4) + q];
+                        const float4 v1 = cf[(grp == 0 ? 3 : 2) * (K / 4) + q];
+                        cA[4 * q] = v0.x; cA[4 * q + 1] = v0.y; cA[4 * q + 2] = v0.z; cA[4 * q + 3] = v0.w;
+                        cB[4 * q] = v1.x; cB[4 * q + 1] = v1.y; cB[4 * q + 2] = v1.z; cB[4 * q + 3] = v1.w;
+                    }
+                }
                 const uint4 *src = reinterpret_cast<const uint4 *>((grp == 0 ? a.dy : a.x) + i0 * P);
 #pragma unroll
                 for (int k = 0; k < 8; ++k) row[k] = src[k];
             } else {
 #pragma unroll
-                for (int k = 0; k < KMAX; ++k) wr[k] = ww[k] = 0.f;
-#pragma unroll
                 for (int k = 0; k < 8; ++k) row[k] = make_uint4(0, 0, 0, 0);
-            }
-            const float log_cap = logf(64.f * tmax);
-            float e = 0.f;
-            if (t < n) {
-                bool cl;
-                e = token_rate(dtv, alv, lmv, log_cap, &cl);
-            }
-            const double Et = group_scan128(double(e), wsum);
-            if (grp == 0 && t == n - 1) *Eend_s = Et;
-            __syncthreads();
-            const double Eend = *Eend_s;
-#pragma unroll
-            for (int k = 0; k < KMAX; ++k) {
-                f_t[k] = s_t[k] = u_t[k] = fd_t[k] = 0.f;
-                if (k < K && t < n) {
-                    const float kp = -expm1f(-e * itr[k]) * ww[k];
-                    u_t[k] = expf(-float(Eend - Et) * itr[k]);
-                    s_t[k] = kp * u_t[k];
-                    fd_t[k] = expf(-float(Et) * itr[k]);
-                    f_t[k] = wr[k] * fd_t[k];
-                }
-                acc_h[k] = 0.f;
             }
             ab_h = 0.f;
 #pragma unroll
@@ -655,7 +652,7 @@ __global__ void __launch_bounds__(kStThreads, 1)
             float sc = 0.f;
 #pragma unroll
             for (int k = 0; k < KMAX; ++k)
-                if (k == m) sc = grp == 0 ? f_t[k] : s_t[k];
+                if (k == m) sc = cA[k];
             unsigned char *dst = sG + gb * L.gen + grp * 16384 + t * 128;
 #pragma unroll
             for (int k = 0; k < 8; ++k)
@@ -666,15 +663,22 @@ __global__ void __launch_bounds__(kStThreads, 1)
         {
             const uint4 *ps = reinterpret_cast<const uint4 *>(sT + (2 * q) * L.tile);
             const uint4 *pd = reinterpret_cast<const uint4 *>(sT + (2 * q + 1) * L.tile);
-            float acc = 0.f;
-            for (int k = tid; k < L.tile / 16; k += kStThreads) acc = dot_bf16x8(ps[k], pd[k], acc);
-            acc = warp_sum(acc);
-            if ((tid & 31) == 0) red[(i % 3) * 8 + w] = acc;
+            float acc0 = 0.f, acc1 = 0.f;  // L.tile / 16 is a multiple of 2 * kStThreads
+            for (int k = tid; k < L.tile / 16; k += 2 * kStThreads) {
+                acc0 = dot_bf16x8(ps[k], pd[k], acc0);
+                acc1 = dot_bf16x8(ps[k + kStThreads], pd[k + kStThreads], acc1);
+            }
+            const float v = warp_sum(acc0 + acc1);
+            if ((tid & 31) == 0) atomicAdd(a.cdot + ((size_t(b) * d.H + h) * d.nc + c) * K + m, v);
         }
+        // hand the generated operands to the MMA issuer (no CTA-wide barrier in the loop)
         fence_async_smem();
         tc_fence_before();
-        __syncthreads();
-        tc_fence_after();
+        mbar_arrive(&bars[7 + gb]);
+        if (tid == 0 && !*abort_s) {
+            if (!mbar_wait(&bars[7 + gb], (i >> 1) & 1)) *abort_s = 1;
+            tc_fence_after();
+        }
         if (tid == 0 && !*abort_s) {
             const uint32_t sS = smem_u32(sT + (2 * q) * L.tile), sD = smem_u32(sT + (2 * q + 1) * L.tile);
             const uint32_t g1 = smem_u32(sG + gb * L.gen), g2 = g1 + 16384;
@@ -898,6 +902,7 @@ size_t tc_bwd_workspace_bytes(const ScanDims &d, TcBwdWorkspace *l, char *base) 
     l->rect = (float *)take(blh_ * 4);
     l->cdot = (float *)take(size_t(d.B) * d.H * d.nc * d.K * 4);
     l->mh_total = (float *)take(size_t(d.B) * d.nc * d.G * TQ * TQ * 4);
+    l->coef = (float *)take(blh_ * 4 * d.K * 4);
     l->dB_acc = (float *)take(size_t(d.B) * d.L * d.G * d.N * 4);
     l->dC_acc = (float *)take(size_t(d.B) * d.L * d.G * d.N * 4);
     return off;
@@ -910,6 +915,7 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
     if ((e = cudaMemsetAsync(p.dD, 0, sizeof(float) * d.H, st))) return e;
     if ((e = cudaMemsetAsync(ws.dB_acc, 0, sizeof(float) * ngn, st))) return e;
     if ((e = cudaMemsetAsync(ws.dC_acc, 0, sizeof(float) * ngn, st))) return e;
+    if ((e = cudaMemsetAsync(ws.cdot, 0, sizeof(float) * d.B * d.H * d.nc * d.K, st))) return e;
     if ((e = cudaMemsetAsync(ws.mh_total, 0, sizeof(float) * d.B * d.nc * d.G * TQ * TQ, st))) return e;
     if (!reuse_states &&
         (e = tc_state_pass_launch(d, false, p.x, p.Bm, p.ww, p.dt, p.alpha, p.lam, p.tau, p.h0,
@@ -938,7 +944,7 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
     a.dt = p.dt; a.alpha = p.alpha; a.lam = p.lam; a.tau = p.tau; a.D = p.D;
     a.S_in = (const bf16 *)ws.S_in; a.dS_out = (const bf16 *)ws.dS_out;
     a.dx_acc = ws.dx_acc; a.dwr_acc = ws.dwr_acc; a.dkap_acc = ws.dkap_acc; a.ab_acc = ws.ab_acc;
-    a.rect = ws.rect; a.cdot = ws.cdot; a.mh_total = ws.mh_total;
+    a.rect = ws.rect; a.cdot = ws.cdot; a.mh_total = ws.mh_total; a.coef = ws.coef;
     a.dB_acc = ws.dB_acc; a.dC_acc = ws.dC_acc;
     a.dx = (bf16 *)p.dx; a.dwr = (bf16 *)p.dwr; a.dww = (bf16 *)p.dww;
     a.ddt = p.ddt; a.dalpha = p.dalpha; a.dlam = p.dlam; a.dD = p.dD;
