@@ -383,7 +383,8 @@ __global__ void __launch_bounds__(kOutThreads, 2)
     tc_fence_after();
     const uint32_t tmem = *tslot;
     const uint32_t lane_base = tmem + (uint32_t(w4 * 32) << 16);
-    constexpr uint32_t colG = 0, colY = 128;
+    // TMEM: G = C B^T at [0, 128), the factored Gamma blocks at [128, 256); Y replaces G
+    constexpr uint32_t colG = 0, colGam = 128, colY = 0;
 
     if (tid == 0) {
         mbar_arrive_expect_tx(&bars[0], uint32_t(2 * plan.c + plan.x));
@@ -392,10 +393,6 @@ __global__ void __launch_bounds__(kOutThreads, 2)
             tma_load_3d(sM + jb * 16384, &mapB, &bars[0], g * N + 64 * jb, c0, b);
         }
         tma_load_3d(sX, &mapX, &bars[0], h * P, c0, b);
-        for (int j = 0; j < min(kSBuf, niter); ++j) {
-            mbar_arrive_expect_tx(&bars[3 + j], 8192u);
-            tma_load_3d(sS + j * 8192, &mapS, &bars[3 + j], (j % nhalf) * 64, 0, srow + j / nhalf);
-        }
     }
     float tmax = 0.f;
     for (int m = 0; m < K; ++m) tmax = fmaxf(tmax, tau_s[m]);
@@ -408,21 +405,52 @@ __global__ void __launch_bounds__(kOutThreads, 2)
     const double Et = group_scan128(double(e), wsum);
     const float2 Et2 = split_f2(Et);
     if (grp == 0) E_s[t] = Et2;
-    float f_t[KMAX];
+    float f_t[KMAX], kap_t[KMAX];
 #pragma unroll
     for (int m = 0; m < KMAX; ++m) {
-        f_t[m] = 0.f;
+        f_t[m] = kap_t[m] = 0.f;
         if (m < K) {
-            float kp = 0.f;
             if (t < n) {
-                kp = -expm1f(-e / tau_s[m]) * ww_t[m];
+                kap_t[m] = -expm1f(-e / tau_s[m]) * ww_t[m];
                 f_t[m] = wr_t[m] * ex2_approx(-float(Et) * l2t[m]);
             }
-            if (grp == 0) kap_s[t * KMAX + m] = kp;
+            if (grp == 0) kap_s[t * KMAX + m] = kap_t[m];
         }
     }
     __syncthreads();
-    // G = C B^T
+    // Gamma below the diagonal 32 x 32 blocks, factored through the log-decay E_a at the end of
+    // the column block J: exp(-(E_t - E_k)/tau) = exp(-(E_t - E_a)/tau) exp(-(E_a - E_k)/tau),
+    // both factors <= 1, so Gamma[t, k in J] = sum_m U_J[t, m] V[k, m] (a K = 8 tf32 product):
+    //   U_J[t, m] = w_read[t, m] exp(-(E_t - E_a)/tau_m)   (rows t of later blocks, else 0)
+    //   V[k, m]   = kappa[k, m] exp(-(E_a - E_k)/tau_m)
+    // U: [128 t][4 J x 8 m] and V: [32 k mod 32][4 J x 8 m], 128-byte swizzled, in the S ring.
+    unsigned char *sU = sS, *sVt = sS + 16384;
+    if (grp == 0) {
+        const int I = t >> 5;
+        unsigned char *row = sU + t * 128;
+#pragma unroll
+        for (int J = 0; J < 4; ++J) {
+            uint32_t u[8];
+            const float dE = diff_f2(Et2, E_s[32 * J + 31]);
+#pragma unroll
+            for (int m = 0; m < KMAX; ++m)
+                u[m] = (J < I && m < K && t < n) ? to_tf32(wr_t[m] * ex2_approx(-dE * l2t[m])) : 0u;
+            *reinterpret_cast<uint4 *>(row + (((2 * J) ^ (t & 7)) * 16)) = make_uint4(u[0], u[1], u[2], u[3]);
+            *reinterpret_cast<uint4 *>(row + (((2 * J + 1) ^ (t & 7)) * 16)) = make_uint4(u[4], u[5], u[6], u[7]);
+        }
+    } else {
+        const int J = t >> 5, r = t & 31;
+        const float dE = diff_f2(E_s[32 * J + 31], Et2);
+        uint32_t v[8];
+#pragma unroll
+        for (int m = 0; m < KMAX; ++m) v[m] = m < K ? to_tf32(kap_t[m] * ex2_approx(-dE * l2t[m])) : 0u;
+        unsigned char *row = sVt + r * 128;
+        *reinterpret_cast<uint4 *>(row + (((2 * J) ^ (r & 7)) * 16)) = make_uint4(v[0], v[1], v[2], v[3]);
+        *reinterpret_cast<uint4 *>(row + (((2 * J + 1) ^ (r & 7)) * 16)) = make_uint4(v[4], v[5], v[6], v[7]);
+    }
+    fence_async_smem();
+    __syncthreads();
+    // G = C B^T (bf16) and the four Gamma column blocks (tf32)
     if (tid == 0) {
         if (!mbar_wait(&bars[0], 0)) {
             *abort_s = 1;
@@ -434,6 +462,10 @@ __global__ void __launch_bounds__(kOutThreads, 2)
                 mma_bf16(tmem + colG, desc_sw128(smem_u32(sC) + koff, 16, 1024),
                          desc_sw128(smem_u32(sM) + koff, 16, 1024), idG, ks > 0);
             }
+            const uint32_t idT = idesc_tf32(128, 32);
+            for (int J = 0; J < 4; ++J)
+                mma_tf32(tmem + colGam + 32 * J, desc_sw128(smem_u32(sU) + 32 * J, 16, 1024),
+                         desc_sw128(smem_u32(sVt) + 32 * J, 16, 1024), idT, 0);
             mma_commit(&bars[1]);
         }
     }
@@ -441,32 +473,55 @@ __global__ void __launch_bounds__(kOutThreads, 2)
     if (!*abort_s && !mbar_wait(&bars[1], 0)) *abort_s = 1;
     __syncthreads();
     tc_fence_after();
+    // the S ring is free again: first S_in tiles
+    if (tid == 0 && !*abort_s) {
+        for (int j = 0; j < min(kSBuf, niter); ++j) {
+            mbar_arrive_expect_tx(&bars[3 + j], 8192u);
+            tma_load_3d(sS + j * 8192, &mapS, &bars[3 + j], (j % nhalf) * 64, 0, srow + j / nhalf);
+        }
+    }
     if (!*abort_s) {
-        // row t of Gamma o G -> bf16, K-major [t][k] over the B tile; group 0 takes k in [0,32)
-        // and [96,128), group 1 takes [32,96) (the causal triangle splits about evenly)
-        for (int half = 0; half < 2; ++half) {
-            const int k32 = grp == 0 ? (half == 0 ? 0 : 96) : (half == 0 ? 32 : 64);
+        // row t of Gamma o G -> bf16, K-major [t][k] over the B tile.  Warp rows are one 32-block
+        // I; column block kc < I takes the factored Gamma, kc == I the direct sum (pairs k <= t),
+        // kc > I is zero.  Group 0 takes kc = 0, 1, group 1 kc = 2, 3.
+        const int I = t >> 5;
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+            const int kc = grp * 2 + h2;
             float gv[32];
-            tmem_ld32(lane_base + colG + k32, gv);
-            tmem_ld_wait();
+            tmem_ld32(lane_base + colG + 32 * kc, gv);
+            if (kc < I) {
+                float gm[32];
+                tmem_ld32(lane_base + colGam + 32 * kc, gm);
+                tmem_ld_wait();
 #pragma unroll
-            for (int kk = 0; kk < 32; ++kk) {
-                const int k = k32 + kk;
-                float v = 0.f;
-                if (k <= t && t < n) {
-                    const float dE = diff_f2(Et2, E_s[k]);
-                    float gam = 0.f;
+                for (int kk = 0; kk < 32; ++kk) gv[kk] *= gm[kk];
+            } else {
+                tmem_ld_wait();
+                if (kc == I) {
 #pragma unroll
-                    for (int m = 0; m < KMAX; ++m)
-                        if (m < K) gam = fmaf(wr_t[m] * kap_s[k * KMAX + m], ex2_approx(-dE * l2t[m]), gam);
-                    v = gam * gv[kk];
+                    for (int kk = 0; kk < 32; ++kk) {
+                        const int k = 32 * kc + kk;
+                        float v = 0.f;
+                        if (k <= t && t < n) {
+                            const float dE = diff_f2(Et2, E_s[k]);
+                            float gam = 0.f;
+#pragma unroll
+                            for (int m = 0; m < KMAX; ++m)
+                                if (m < K) gam = fmaf(wr_t[m] * kap_s[k * KMAX + m], ex2_approx(-dE * l2t[m]), gam);
+                            v = gam * gv[kk];
+                        }
+                        gv[kk] = v;
+                    }
+                } else {
+#pragma unroll
+                    for (int kk = 0; kk < 32; ++kk) gv[kk] = 0.f;
                 }
-                gv[kk] = v;
             }
-            unsigned char *tile = sM + (k32 >> 6) * 16384;
+            unsigned char *tile = sM + (kc >> 1) * 16384;
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
-                const int c8 = ((k32 & 63) >> 3) + q;
+                const int c8 = (kc & 1) * 4 + q;
                 *reinterpret_cast<uint4 *>(tile + t * 128 + ((c8 ^ (t & 7)) * 16)) =
                     make_uint4(pack_bf16x2(gv[8 * q], gv[8 * q + 1]), pack_bf16x2(gv[8 * q + 2], gv[8 * q + 3]),
                                pack_bf16x2(gv[8 * q + 4], gv[8 * q + 5]), pack_bf16x2(gv[8 * q + 6], gv[8 * q + 7]));
@@ -477,7 +532,7 @@ __global__ void __launch_bounds__(kOutThreads, 2)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (tid == 0 && !*abort_s) {  // Y = (Gamma o G) X: M = t, N = p, K = k
+    if (tid == 0 && !*abort_s) {  // Y = (Gamma o G) X: M = t, N = p, K = k (over G's columns)
         const uint32_t idY = idesc_bf16(128, 64, false, true);
         for (int ks = 0; ks < TQ / 16; ++ks)
             mma_bf16(tmem + colY, desc_sw128(smem_u32(sM) + (ks / 4) * 16384 + (ks % 4) * 32, 16, 1024),
