@@ -93,7 +93,7 @@ struct IntraSmem {
         dy = 16384;                // dy chunk
         mg = 2 * 16384;            // Gamma o G, [t][k] K-major
         xx = TQ * XS * 4;          // fp32 Gamma' G H, then its row prefix sums
-        total = rcb + x + dy + mg + xx + 3 * TQ * KMAX * 4 + TQ * 8 + 64 * 4 + 64 + 64 + 64;
+        total = rcb + x + dy + mg + xx + 4 * TQ * KMAX * 4 + TQ * 8 + 64 * 4 + 64 + 64 + 64;
     }
 };
 
@@ -116,7 +116,8 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     float *wr_s = XX + TQ * XS;                              // [128][KMAX]
     float *kap_s = wr_s + TQ * KMAX;                         // [128][KMAX]
     float *part = kap_s + TQ * KMAX;                         // [128][KMAX] partial sums of group 1
-    float2 *E_s = reinterpret_cast<float2 *>(part + TQ * KMAX);  // hi / lo pairs
+    float *Vs = part + TQ * KMAX;                            // [128][KMAX] kappa exp(-(E_a - E_k)/tau)
+    float2 *E_s = reinterpret_cast<float2 *>(Vs + TQ * KMAX);  // hi / lo pairs
     float *l2t = reinterpret_cast<float *>(E_s + TQ);
     float *tau_s = l2t + 32;
     double *wsum = reinterpret_cast<double *>(tau_s + 32);
@@ -159,7 +160,8 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *tslot;
     const uint32_t lane_base = tmem + (uint32_t(w4 * 32) << 16);
-    const uint32_t colG = 0, colH = 128, colX = 256;
+    // TMEM: G, H, the factored Gamma and Gamma' blocks; dx_intra replaces G after the row pass
+    const uint32_t colG = 0, colH = 128, colGam = 256, colGamP = 384, colX = 0;
 
     if (tid == 0) {
         mbar_arrive_expect_tx(&bars[0], uint32_t(2 * (N / 64) * 16384 + 2 * 16384));
@@ -219,6 +221,44 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
             }
         }
     }
+    // ---- Gamma below the diagonal 32 x 32 blocks, factored through the log-decay E_a at the end
+    // of the column block J (as in the forward output kernel): Gamma[t, k in J] =
+    // sum_m U_J[t, m] V[k, m] and Gamma'[t, k] = sum_m U_J[t, m] V[k, m] / tau_m, tf32 products.
+    // Operand tiles (128-byte swizzled) in the XX region: U [128 t][4 J x 8 m],
+    // V and V / tau [32 k mod 32][4 J x 8 m]; V also as fp32 in Vs for the intra dw_read.
+    unsigned char *sU = reinterpret_cast<unsigned char *>(XX), *sV = sU + 16384, *sVp = sV + 4096;
+    if (grp == 0) {
+        const int I = t >> 5;
+        unsigned char *row = sU + t * 128;
+#pragma unroll
+        for (int J = 0; J < 4; ++J) {
+            uint32_t u[8];
+            const float dE = diff_f2(Et2, E_s[32 * J + 31]);
+#pragma unroll
+            for (int m = 0; m < KMAX; ++m)
+                u[m] = (J < I && m < K && t < n) ? to_tf32(wr_t[m] * ex2_approx(-dE * l2r[m])) : 0u;
+            *reinterpret_cast<uint4 *>(row + (((2 * J) ^ (t & 7)) * 16)) = make_uint4(u[0], u[1], u[2], u[3]);
+            *reinterpret_cast<uint4 *>(row + (((2 * J + 1) ^ (t & 7)) * 16)) = make_uint4(u[4], u[5], u[6], u[7]);
+        }
+    } else {
+        const int J = t >> 5, r = t & 31;
+        const float dE = diff_f2(E_s[32 * J + 31], Et2);
+        uint32_t v[8], vp[8];
+#pragma unroll
+        for (int m = 0; m < KMAX; ++m) {
+            const float vv = m < K ? kap_t[m] * ex2_approx(-dE * l2r[m]) : 0.f;
+            Vs[t * KMAX + m] = vv;
+            v[m] = to_tf32(vv);
+            vp[m] = m < K ? to_tf32(vv / tau_s[m]) : 0u;
+        }
+        unsigned char *row = sV + r * 128, *rowp = sVp + r * 128;
+        *reinterpret_cast<uint4 *>(row + (((2 * J) ^ (r & 7)) * 16)) = make_uint4(v[0], v[1], v[2], v[3]);
+        *reinterpret_cast<uint4 *>(row + (((2 * J + 1) ^ (r & 7)) * 16)) = make_uint4(v[4], v[5], v[6], v[7]);
+        *reinterpret_cast<uint4 *>(rowp + (((2 * J) ^ (r & 7)) * 16)) = make_uint4(vp[0], vp[1], vp[2], vp[3]);
+        *reinterpret_cast<uint4 *>(rowp + (((2 * J + 1) ^ (r & 7)) * 16)) = make_uint4(vp[4], vp[5], vp[6], vp[7]);
+    }
+    fence_async_smem();
+    __syncthreads();
     if (tid == 0) {
         if (!mbar_wait(&bars[0], 0)) {
             *abort_s = 1;
@@ -234,6 +274,13 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
                 mma_bf16(tmem + colH, desc_sw128(smem_u32(sDY) + ks * 32, 16, 1024),
                          desc_sw128(smem_u32(sX) + ks * 32, 16, 1024), idG, ks > 0);
             }
+            const uint32_t idT = idesc_tf32(128, 32);
+            for (int J = 0; J < 4; ++J) {
+                mma_tf32(tmem + colGam + 32 * J, desc_sw128(smem_u32(sU) + 32 * J, 16, 1024),
+                         desc_sw128(smem_u32(sV) + 32 * J, 16, 1024), idT, 0);
+                mma_tf32(tmem + colGamP + 32 * J, desc_sw128(smem_u32(sU) + 32 * J, 16, 1024),
+                         desc_sw128(smem_u32(sVp) + 32 * J, 16, 1024), idT, 0);
+            }
             mma_commit(&bars[1]);
         }
     }
@@ -241,58 +288,110 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     if (!*abort_s && !mbar_wait(&bars[1], 0)) *abort_s = 1;
     __syncthreads();
     tc_fence_after();
-    // ---- row pass (row t; group 0 takes k in [0,32) and [96,128), group 1 takes [32,96)):
-    // Gamma, Gamma', intra dw_read, Gamma o G tile, Gamma o H summed over heads in L2, Gamma' G H
-    // and G H pair tiles
+    // U rows as fp32 [128 t][4 J][8 m] in the x tile (free now) for the column pass, before the
+    // row pass overwrites the operand tiles with XX
+    float *Ufp = reinterpret_cast<float *>(sX);
+    if (grp == 0) {
+        const unsigned char *row = sU + t * 128;
+#pragma unroll
+        for (int c8 = 0; c8 < 8; ++c8)
+            *reinterpret_cast<uint4 *>(Ufp + t * 32 + 4 * c8) =
+                *reinterpret_cast<const uint4 *>(row + ((c8 ^ (t & 7)) * 16));
+    }
+    __syncthreads();
+    // ---- row pass (row t = this warp's row block I; group 0 takes column blocks 0, 1, group 1
+    // blocks 2, 3): Gamma o G tile, Gamma o H summed over heads in L2, Gamma' G H and G H tiles,
+    // intra dw_read.  Blocks below the diagonal take the factored Gamma from TMEM, the diagonal
+    // block sums its pairs k <= t directly, blocks above it are zero.
     float dwr_i[KMAX];
 #pragma unroll
     for (int m = 0; m < KMAX; ++m) dwr_i[m] = 0.f;
     if (!*abort_s) {
+        const int I = t >> 5;
         float *mh_row = a.mh_total + (((size_t(b) * d.nc + c) * d.G + g) * TQ + t) * TQ;
-        for (int half = 0; half < 2; ++half) {
-            const int k32 = grp == 0 ? (half == 0 ? 0 : 96) : (half == 0 ? 32 : 64);
-            float gv[32], hv[32];
-            tmem_ld32(lane_base + colG + k32, gv);
-            tmem_ld32(lane_base + colH + k32, hv);
-            tmem_ld_wait();
+        // outer loops stay rolled: the fully unrolled pass overflowed the instruction cache
+#pragma unroll 1
+        for (int h2 = 0; h2 < 2; ++h2) {
+            const int kc = grp * 2 + h2;
+            unsigned char *tile = sMG + (kc >> 1) * 16384 + t * 128;
+            if (kc > I) {
+#pragma unroll 1
+                for (int q = 0; q < 4; ++q) {
+                    *reinterpret_cast<uint4 *>(tile + ((((kc & 1) * 4 + q) ^ (t & 7)) * 16)) = make_uint4(0, 0, 0, 0);
 #pragma unroll
-            for (int kk = 0; kk < 32; ++kk) {
-                const int k = k32 + kk;
-                float gam = 0.f, gamt = 0.f, gh = 0.f;
-                if (k <= t && t < n) {
-                    const float dE = diff_f2(Et2, E_s[k]);
-                    gh = gv[kk] * hv[kk];
+                    for (int kk = 0; kk < 8; ++kk) XX[t * XS + 32 * kc + 8 * q + kk] = 0.f;  // rows are 129 floats apart
+                }
+                continue;
+            }
+            float acc[KMAX];
 #pragma unroll
-                    for (int m = 0; m < KMAX; ++m) {
-                        if (m < K) {
-                            const float W = ex2_approx(-dE * l2r[m]);
-                            const float kp = kap_s[k * KMAX + m];
-                            const float aa = wr_t[m] * kp * W;
-                            gam += aa;
-                            gamt = fmaf(aa, l2r[m], gamt);  // times log2(e) / tau
-                            dwr_i[m] = fmaf(kp * W, gh, dwr_i[m]);
+            for (int m = 0; m < KMAX; ++m) acc[m] = 0.f;
+#pragma unroll 1
+            for (int q8 = 0; q8 < 4; ++q8) {  // eight columns at a time
+                const int k0 = 32 * kc + 8 * q8;
+                float gv[8], hv[8];
+                tmem_ld8(lane_base + colG + k0, gv);
+                tmem_ld8(lane_base + colH + k0, hv);
+                if (kc < I) {
+                    float gm[8], gp[8];
+                    tmem_ld8(lane_base + colGam + k0, gm);
+                    tmem_ld8(lane_base + colGamP + k0, gp);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) {
+                        const int k = k0 + kk;
+                        const float gh = gv[kk] * hv[kk];
+                        XX[t * XS + k] = gp[kk] * gh;
+                        GHs[t * XS + k] = gh;
+                        const float4 v0 = *reinterpret_cast<const float4 *>(Vs + k * KMAX);
+                        const float4 v1 = *reinterpret_cast<const float4 *>(Vs + k * KMAX + 4);
+                        const float vk[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+#pragma unroll
+                        for (int m = 0; m < KMAX; ++m) acc[m] = fmaf(vk[m], gh, acc[m]);
+                        gv[kk] *= gm[kk];  // Gamma o G
+                        hv[kk] *= gm[kk];  // Gamma o H
+                    }
+                } else {
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) {
+                        const int k = k0 + kk;
+                        float gam = 0.f, gamt = 0.f, gh = 0.f;
+                        if (k <= t && t < n) {
+                            const float dE = diff_f2(Et2, E_s[k]);
+                            gh = gv[kk] * hv[kk];
+#pragma unroll
+                            for (int m = 0; m < KMAX; ++m) {
+                                if (m < K) {
+                                    const float W = ex2_approx(-dE * l2r[m]);
+                                    const float kp = kap_s[k * KMAX + m];
+                                    const float aa = wr_t[m] * kp * W;
+                                    gam += aa;
+                                    gamt = fmaf(aa, l2r[m], gamt);  // times log2(e) / tau
+                                    dwr_i[m] = fmaf(kp * W, gh, dwr_i[m]);
+                                }
+                            }
                         }
+                        gv[kk] = gam * gv[kk];
+                        hv[kk] = gam * hv[kk];
+                        XX[t * XS + k] = gamt * (1.f / kLog2e) * gh;
+                        GHs[t * XS + k] = gh;
                     }
                 }
-                gv[kk] = gam * gv[kk];  // Gamma o G
-                hv[kk] = gam * hv[kk];  // Gamma o H
-                XX[t * XS + k] = gamt * (1.f / kLog2e) * gh;
-                GHs[t * XS + k] = gh;
+                *reinterpret_cast<uint4 *>(tile + ((((kc & 1) * 4 + q8) ^ (t & 7)) * 16)) =
+                    make_uint4(pack_bf16x2(gv[0], gv[1]), pack_bf16x2(gv[2], gv[3]), pack_bf16x2(gv[4], gv[5]),
+                               pack_bf16x2(gv[6], gv[7]));
+                if (t < n && k0 <= t) {
+                    atomicAdd(reinterpret_cast<float4 *>(mh_row + k0), make_float4(hv[0], hv[1], hv[2], hv[3]));
+                    if (k0 + 4 <= t)
+                        atomicAdd(reinterpret_cast<float4 *>(mh_row + k0 + 4), make_float4(hv[4], hv[5], hv[6], hv[7]));
+                }
             }
-            unsigned char *tile = sMG + (k32 >> 6) * 16384;
+            if (kc < I) {  // intra dw_read of the factored block: exp(-(E_t - E_a)/tau) sum_k V G H
+                const float dE = diff_f2(Et2, E_s[32 * kc + 31]);
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int c8 = ((k32 & 63) >> 3) + q;
-                *reinterpret_cast<uint4 *>(tile + t * 128 + ((c8 ^ (t & 7)) * 16)) =
-                    make_uint4(pack_bf16x2(gv[8 * q], gv[8 * q + 1]), pack_bf16x2(gv[8 * q + 2], gv[8 * q + 3]),
-                               pack_bf16x2(gv[8 * q + 4], gv[8 * q + 5]), pack_bf16x2(gv[8 * q + 6], gv[8 * q + 7]));
-            }
-            if (t < n && k32 <= t) {
-#pragma unroll
-                for (int q = 0; q < 8; ++q)
-                    if (k32 + 4 * q <= t)
-                        atomicAdd(reinterpret_cast<float4 *>(mh_row + k32 + 4 * q),
-                                  make_float4(hv[4 * q], hv[4 * q + 1], hv[4 * q + 2], hv[4 * q + 3]));
+                for (int m = 0; m < KMAX; ++m)
+                    if (m < K) dwr_i[m] = fmaf(ex2_approx(-dE * l2r[m]), acc[m], dwr_i[m]);
             }
         }
         if (grp == 1) {
@@ -318,25 +417,24 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         mma_commit(&bars[2]);
     }
     __syncthreads();  // part[] is reused below
-    // ---- column pass (column k = t; group g takes rows t' = k + g, k + g + 2, ...): intra dkappa
+    // ---- column pass (column k = t, group g takes rows of parity g): intra dkappa.  Rows of
+    // later blocks use the factored form exp(-(E_a - E_k)/tau) sum_t U_J[t, m] G H[t, k]; rows of
+    // the diagonal block (t >= k) sum directly.
     float dk[KMAX];
 #pragma unroll
     for (int m = 0; m < KMAX; ++m) dk[m] = 0.f;
     if (!*abort_s) {
-        // all lanes of a warp walk the same rows tt (broadcast loads of E, w_read); rows above the
-        // diagonal (tt < k) contribute nothing
-        const int k = t;
+        const int k = t, J = k >> 5;
         const float2 Ek = E_s[k];
         float dk2[KMAX];
 #pragma unroll
         for (int m = 0; m < KMAX; ++m) dk2[m] = 0.f;
-        // group grp takes the rows of parity grp, starting at this warp's first column; four
-        // rows per step (two accumulator sets) keep several exponentials in flight
-        for (int tt0 = (t & ~31) + grp; tt0 < n; tt0 += 8) {
+        const int dend = min(n, 32 * J + 32);
+        for (int tt0 = 32 * J + grp; tt0 < dend; tt0 += 8) {
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 const int tt = tt0 + 2 * u;
-                if (tt < n && tt >= k) {
+                if (tt < dend && tt >= k) {
                     const float dE = diff_f2(E_s[tt], Ek);
                     const float gh = GHs[tt * XS + k];
 #pragma unroll
@@ -352,8 +450,34 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
                 }
             }
         }
+        float s0[KMAX], s1[KMAX];
 #pragma unroll
-        for (int m = 0; m < KMAX; ++m) dk[m] += dk2[m];
+        for (int m = 0; m < KMAX; ++m) s0[m] = s1[m] = 0.f;
+        for (int tt0 = 32 * J + 32 + grp; tt0 < n; tt0 += 8) {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int tt = tt0 + 2 * u;
+                if (tt < n) {
+                    const float gh = GHs[tt * XS + k];
+                    const float4 u0 = *reinterpret_cast<const float4 *>(Ufp + tt * 32 + 8 * J);
+                    const float4 u1 = *reinterpret_cast<const float4 *>(Ufp + tt * 32 + 8 * J + 4);
+                    const float uu[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+#pragma unroll
+                    for (int m = 0; m < KMAX; ++m) {
+                        if (u & 1)
+                            s1[m] = fmaf(uu[m], gh, s1[m]);
+                        else
+                            s0[m] = fmaf(uu[m], gh, s0[m]);
+                    }
+                }
+            }
+        }
+        const float dEa = diff_f2(E_s[32 * J + 31], Ek);
+#pragma unroll
+        for (int m = 0; m < KMAX; ++m) {
+            dk[m] += dk2[m];
+            if (m < K) dk[m] = fmaf(ex2_approx(-dEa * l2r[m]), s0[m] + s1[m], dk[m]);
+        }
         if (grp == 1) {
 #pragma unroll
             for (int m = 0; m < KMAX; ++m) part[k * KMAX + m] = dk[m];
