@@ -52,7 +52,8 @@ struct StateSmem {
     __host__ __device__ StateSmem(int K, int N) {
         a_bytes = (K / 4) * 2 * 16384;  // K/4 M-tiles x 2 M-atoms x (128 k rows x 128 B), MN-major
         v_bytes = (N / 64) * 16384;     // N/64 boxes of [128 t][64 n]
-        total = a_bytes + v_bytes + 64 * 4 /*itau, dec*/ + 64 /*wsum*/ + 16 /*E_end*/ + 64 /*bars*/;
+        total = a_bytes + v_bytes + TQ * KMAX * 4 /*cv*/ + 64 * 4 /*itau, dec*/ + 64 /*wsum*/ +
+                16 /*E_end*/ + 64 /*bars*/;
     }
 };
 
@@ -67,7 +68,8 @@ __global__ void __launch_bounds__(kThreads, 2)
     const StateSmem plan(K, N);
     unsigned char *sA = base;
     unsigned char *sV = sA + plan.a_bytes;
-    float *itau = reinterpret_cast<float *>(sV + plan.v_bytes);  // [32]
+    float *cv_s = reinterpret_cast<float *>(sV + plan.v_bytes);  // [128][KMAX] this chunk's s or f
+    float *itau = cv_s + TQ * KMAX;                               // [32]
     float *dec = itau + 32;                                       // [32]
     double *wsum = reinterpret_cast<double *>(dec + 32);          // [4]
     double *Eend_s = wsum + 8;                                    // [1]
@@ -187,6 +189,11 @@ __global__ void __launch_bounds__(kThreads, 2)
             }
         }
         if (t < K) dec[t] = expf(-float(Eend) * itau[t]);
+        {
+            float4 *o = reinterpret_cast<float4 *>(cv_s + t * KMAX);  // this thread's own row
+            o[0] = make_float4(cv[0], cv[1], cv[2], cv[3]);
+            o[1] = make_float4(cv[4], cv[5], cv[6], cv[7]);
+        }
         if (ci > 0) {  // previous chunk's MMAs done: tensor memory, sA and sV are free
             if (!mbar_wait(&bars[1], phase ^ 1)) *abort_s = 1;
         }
@@ -200,15 +207,15 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
         // A[(m%4, p), k] = s_{k,m} x_{k,p} as bf16, MN-major: row k = this thread's position,
         // 64-element M-atoms (modes 2a, 2a+1 of the tile x 32 p), 128-byte swizzle
-#pragma unroll
-        for (int mt = 0; mt < KMAX / 4; ++mt) {
-            if (mt >= mtiles) break;
-#pragma unroll
-            for (int at = 0; at < 2; ++at) {
-                unsigned char *row = sA + (mt * 2 + at) * 16384 + t * 128;
+#pragma unroll 1
+        for (int ma = 0; ma < 2 * mtiles; ++ma) {  // (mode tile, M-atom): modes 2 ma, 2 ma + 1
+            unsigned char *row = sA + ma * 16384 + t * 128;
+            const float2 s01 = *reinterpret_cast<const float2 *>(cv_s + t * KMAX + 2 * ma);
+            const float s0 = s01.x, s1 = s01.y;
+            {
 #pragma unroll
                 for (int c8 = 0; c8 < 8; ++c8) {
-                    const float s = cv[mt * 4 + 2 * at + (c8 >> 2)];  // mode of this 8-element run
+                    const float s = c8 < 4 ? s0 : s1;  // mode of this 8-element run
                     const uint4 xv = xr[c8 & 3];
                     const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
                     uint32_t r[4];
@@ -483,25 +490,30 @@ __global__ void __launch_bounds__(kOutThreads, 2)
     if (!*abort_s) {
         // row t of Gamma o G -> bf16, K-major [t][k] over the B tile.  Warp rows are one 32-block
         // I; column block kc < I takes the factored Gamma, kc == I the direct sum (pairs k <= t),
-        // kc > I is zero.  Group 0 takes kc = 0, 1, group 1 kc = 2, 3.
+        // kc > I is zero.  Group 0 takes kc = 0, 1, group 1 kc = 2, 3; eight columns at a time
+        // with rolled outer loops (compact code: the unrolled pass overflowed the instruction cache)
         const int I = t >> 5;
-#pragma unroll
+#pragma unroll 1
         for (int h2 = 0; h2 < 2; ++h2) {
             const int kc = grp * 2 + h2;
-            float gv[32];
-            tmem_ld32(lane_base + colG + 32 * kc, gv);
-            if (kc < I) {
-                float gm[32];
-                tmem_ld32(lane_base + colGam + 32 * kc, gm);
-                tmem_ld_wait();
+            unsigned char *tile = sM + (kc >> 1) * 16384 + t * 128;
+#pragma unroll 1
+            for (int q8 = 0; q8 < 4; ++q8) {
+                const int k0 = 32 * kc + 8 * q8;
+                float gv[8];
+                if (kc < I) {
+                    float gm[8];
+                    tmem_ld8(lane_base + colG + k0, gv);
+                    tmem_ld8(lane_base + colGam + k0, gm);
+                    tmem_ld_wait();
 #pragma unroll
-                for (int kk = 0; kk < 32; ++kk) gv[kk] *= gm[kk];
-            } else {
-                tmem_ld_wait();
-                if (kc == I) {
+                    for (int kk = 0; kk < 8; ++kk) gv[kk] *= gm[kk];
+                } else if (kc == I) {
+                    tmem_ld8(lane_base + colG + k0, gv);
+                    tmem_ld_wait();
 #pragma unroll
-                    for (int kk = 0; kk < 32; ++kk) {
-                        const int k = 32 * kc + kk;
+                    for (int kk = 0; kk < 8; ++kk) {
+                        const int k = k0 + kk;
                         float v = 0.f;
                         if (k <= t && t < n) {
                             const float dE = diff_f2(Et2, E_s[k]);
@@ -515,16 +527,11 @@ __global__ void __launch_bounds__(kOutThreads, 2)
                     }
                 } else {
 #pragma unroll
-                    for (int kk = 0; kk < 32; ++kk) gv[kk] = 0.f;
+                    for (int kk = 0; kk < 8; ++kk) gv[kk] = 0.f;
                 }
-            }
-            unsigned char *tile = sM + (kc >> 1) * 16384;
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int c8 = (kc & 1) * 4 + q;
-                *reinterpret_cast<uint4 *>(tile + t * 128 + ((c8 ^ (t & 7)) * 16)) =
-                    make_uint4(pack_bf16x2(gv[8 * q], gv[8 * q + 1]), pack_bf16x2(gv[8 * q + 2], gv[8 * q + 3]),
-                               pack_bf16x2(gv[8 * q + 4], gv[8 * q + 5]), pack_bf16x2(gv[8 * q + 6], gv[8 * q + 7]));
+                *reinterpret_cast<uint4 *>(tile + ((((kc & 1) * 4 + q8) ^ (t & 7)) * 16)) =
+                    make_uint4(pack_bf16x2(gv[0], gv[1]), pack_bf16x2(gv[2], gv[3]), pack_bf16x2(gv[4], gv[5]),
+                               pack_bf16x2(gv[6], gv[7]));
             }
         }
     }
