@@ -137,6 +137,38 @@ def kpn(s):
     return s.nmodes * s.headdim * s.dstate
 
 
+# DRAM bytes (read + write) per launch of each tensor-core kernel from one ncu capture of the
+# training shape at batch 2 (profiles/tc_kernels_train_b2_l4096.md); the per-chunk state traffic
+# grows in proportion to the batch, so a run at batch B reports bytes x B / 2.  A figure is used
+# only while the kernel's sources hash to the digest they had when they were profiled.
+PROFILED_TRAFFIC_BATCH = 2
+PROFILED_TRAFFIC = {
+    "state_pass_fwd_tc": ("scan_tc.cu", "7f83405a1de4edf3", 86.132e6 + 481.253e6),
+    "chunk_fwd_tc": ("scan_tc.cu", "7f83405a1de4edf3", 631.337e6 + 59.508e6),
+    "state_pass_rev_tc": ("scan_tc.cu", "7f83405a1de4edf3", 86.476e6 + 481.268e6),
+    "bwd_intra_tc": ("scan_tc_bwd.cu", "16553d01fd1d6858", 164.203e6 + 185.403e6),
+    "bwd_state_tc": ("scan_tc_bwd.cu", "16553d01fd1d6858", 1461.356e6 + 168.297e6),
+}
+
+
+def source_digest(fname: str) -> str:
+    import hashlib
+    src = os.path.join(os.path.dirname(os.path.abspath(__file__)), "paper_2609_36314_gb300", "csrc")
+    m = hashlib.sha256()
+    for f in (fname, "tc.cuh", "tc_util.cuh", "common.cuh", "kernels.h"):
+        with open(os.path.join(src, f), "rb") as fh:
+            m.update(fh.read())
+    return m.hexdigest()[:16]
+
+
+def profiled_traffic(kernel: str, batch: int):
+    """DRAM bytes per launch at this batch from the committed ncu capture, or None."""
+    entry = PROFILED_TRAFFIC.get(kernel)
+    if entry is None or source_digest(entry[0]) != entry[1]:
+        return None
+    return entry[2] * batch / PROFILED_TRAFFIC_BATCH
+
+
 def algorithmic_work(kernel: str, s, per_launch_units: float):
     """Algorithmic flops or bytes of one launch of `kernel` (see the measurement section of
     the design notes): state contractions count 2 K P N flops per token-head each."""
@@ -202,11 +234,14 @@ def run_reference(args, rank):
     print(json.dumps(line), flush=True)
 
 
-def cpu_baseline(heads=16):
+def cpu_baseline(rows=2):
+    """The oracle (fp64, OpenMP over (batch, head) streams) on `rows` full batch rows of the
+    training workload: all heads, the full sequence, forward + backward (about 10-15 s on 16
+    cores)."""
     from oracle import oracle
     from paper_2609_36314_gb300 import synth
     s = shape_of(TRAIN)
-    sub = s.replace(batch=1, nheads=heads)
+    sub = s.replace(batch=rows)
     host = synth.make_scan_inputs(sub, seed=1, with_dy=True)
     d = {k: synth.to_f64(v) for k, v in host.items()}
     t0 = time.perf_counter()
@@ -215,12 +250,11 @@ def cpu_baseline(heads=16):
     oracle.bwd(d["x"], d["dt"], d["alpha"], d["lam"], d["tau"], d["B"], d["C"], d["w_read"],
                d["w_write"], d["D"], d["dy"])
     dt = time.perf_counter() - t0
-    tokens = sub.seqlen * heads / s.nheads
+    tokens = sub.batch * sub.seqlen
     return {"value": tokens / dt, "unit": "tokens/s", "cores": oracle.max_threads(),
             "kind": "oracle",
-            "sample": f"fwd+bwd of batch row 0, heads 0-{heads - 1}, L={s.seqlen} "
-                      f"({heads}/{s.nheads * s.batch} of the (batch, head) streams), "
-                      f"{dt:.1f} s"}
+            "sample": f"fwd+bwd of batch rows 0-{rows - 1} (all {s.nheads} heads, L={s.seqlen}; "
+                      f"{rows}/{s.batch} of the workload), {dt:.1f} s"}
 
 
 # ----------------------------------------------------------------------------- GPU arm
@@ -323,7 +357,8 @@ def main():
             peak = peaks.get("bf16_tflops_sustained", peaks.get("bf16_tflops"))
             ach = work / avg_s / 1e12
             roofline = {"kernel": dom, "bound": "tensor", "achieved": ach, "peak": peak,
-                        "unit": "TFLOP/s", "frac": ach / peak, "traffic": None,
+                        "unit": "TFLOP/s", "frac": ach / peak,
+                        "traffic": profiled_traffic(dom, s.batch),
                         "peak_source": peaks["source"] + " (bf16, sustained)"}
         elif kind == "flops":
             # CUDA-core float32 FMA peak: SMs x 128 lanes x 2 flops x max SM clock

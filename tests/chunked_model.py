@@ -68,6 +68,48 @@ def gamma_factorised(E, wr, kap, tau, sb):
     return G
 
 
+def gamma_col_anchor(E, wr, kap, tau, sb):
+    """Gamma with one anchor per column block, the form the tensor-core kernels use: below the
+    diagonal blocks exp(-(E_t - E_k)/tau) = exp(-(E_t - E_a)/tau) exp(-(E_a - E_k)/tau) with
+    E_a = E at the last position of k's block (both factors <= 1), so
+    Gamma[t, k] = sum_m U_J[t, m] V[k, m]; diagonal blocks are summed directly."""
+    Q = E.shape[0]
+    G = np.zeros((Q, Q))
+    for j0 in range(0, Q, sb):
+        j1 = min(Q, j0 + sb)
+        G[j0:j1, j0:j1] = gamma_direct(E[j0:j1], wr[j0:j1], kap[j0:j1], tau)[0]
+        Ea = E[j1 - 1]
+        V = kap[j0:j1] * np.exp(-(Ea - E[j0:j1, None]) / tau)   # [sb, K]
+        U = wr[j1:] * np.exp(-(E[j1:, None] - Ea) / tau)         # [rows after the block, K]
+        G[j1:, j0:j1] = U @ V.T
+    return G
+
+
+def intra_mode_sums_col_anchor(E, wr, kap, tau, GH, sb):
+    """The per-mode pair sums of the intra backward with the same factorisation:
+    dwr[t, m] = sum_{k<=t} kappa_{k,m} W_{t,k,m} GH[t,k] and
+    dk[k, m]  = sum_{t>=k} w_read_{t,m} W_{t,k,m} GH[t,k];
+    below the diagonal blocks dwr = exp(-(E_t - E_a)/tau) sum_k V[k] GH[t,k] and
+    dk = exp(-(E_a - E_k)/tau) sum_t U_J[t] GH[t,k]."""
+    Q, K = wr.shape
+    dwr = np.zeros((Q, K))
+    dk = np.zeros((Q, K))
+    for j0 in range(0, Q, sb):
+        j1 = min(Q, j0 + sb)
+        _, W = gamma_direct(E[j0:j1], wr[j0:j1], kap[j0:j1], tau)   # diagonal block, [q,q,K]
+        g = GH[j0:j1, j0:j1]
+        dwr[j0:j1] += np.einsum("km,tkm,tk->tm", kap[j0:j1], W, g)
+        dk[j0:j1] += np.einsum("tm,tkm,tk->km", wr[j0:j1], W, g)
+        Ea = E[j1 - 1]
+        b = np.exp(-(Ea - E[j0:j1, None]) / tau)                    # [sb, K]
+        a = np.exp(-(E[j1:, None] - Ea) / tau)                      # [rows after, K]
+        V = kap[j0:j1] * b
+        U = wr[j1:] * a
+        dwr[j1:] += a * (GH[j1:, j0:j1] @ V)
+        dk[j0:j1] += b * (GH[j1:, j0:j1].T @ U)
+    return dwr, dk
+
+
 def fwd(x, dt, alpha, lam, tau, Bm, Cm, wr, ww, D, h0=None, Q=64, sb=None, keep=False):
     Bz, L, H, P = x.shape
     G, N, K = Bm.shape[2], Bm.shape[3], tau.shape[1]

@@ -44,6 +44,39 @@ def test_subblock_factorisation_of_gamma(Q, sb):
     assert synth.rel_l2(y1, y0) < 1e-13
 
 
+def _chunk_terms(Q, seed, shift=0.0):
+    rng = np.random.default_rng(seed)
+    K = 4
+    tau = np.array([1.0, 7.0, 80.0, 2000.0])
+    e = np.exp(rng.normal(0.0, 1.5, Q) + shift)          # wide spread of decay rates
+    E = np.cumsum(e)
+    wr = rng.random((Q, K))
+    kap = rng.random((Q, K)) - 0.3
+    return E, wr, kap, tau, rng
+
+
+@pytest.mark.parametrize("Q,sb,shift", [(128, 32, 0.0), (128, 32, 3.0), (100, 32, 0.0), (37, 8, 1.0)])
+def test_column_anchored_gamma(Q, sb, shift):
+    """The kernels' factorisation (one anchor at the end of each column block) equals Gamma."""
+    E, wr, kap, tau, _ = _chunk_terms(Q, seed=Q + sb, shift=shift)
+    g0, _ = cm.gamma_direct(E, wr, kap, tau)
+    g1 = cm.gamma_col_anchor(E, wr, kap, tau, sb)
+    assert np.max(np.abs(g1 - g0)) <= 1e-13 * max(1.0, np.max(np.abs(g0)))
+
+
+@pytest.mark.parametrize("Q,sb,shift", [(128, 32, 0.0), (128, 32, 2.0), (77, 32, 0.0)])
+def test_column_anchored_intra_mode_sums(Q, sb, shift):
+    """dw_read and dkappa pair sums of the intra backward through the same factorisation."""
+    E, wr, kap, tau, rng = _chunk_terms(Q, seed=3 * Q + sb, shift=shift)
+    GH = np.tril(rng.normal(size=(Q, Q)))
+    _, W = cm.gamma_direct(E, wr, kap, tau)
+    dwr0 = np.einsum("km,tkm,tk->tm", kap, W, GH)
+    dk0 = np.einsum("tm,tkm,tk->km", wr, W, GH)
+    dwr1, dk1 = cm.intra_mode_sums_col_anchor(E, wr, kap, tau, GH, sb)
+    assert synth.rel_l2(dwr1, dwr0) < 1e-12
+    assert synth.rel_l2(dk1, dk0) < 1e-12
+
+
 @pytest.mark.parametrize("Q", [1, 5, 16, 64])
 def test_chunked_backward_equals_sequential_adjoint(Q):
     d = _inputs(h0=True, dhf=True)
