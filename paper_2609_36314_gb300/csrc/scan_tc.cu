@@ -552,15 +552,8 @@ __global__ void __launch_bounds__(kOutThreads, 2)
     const uint32_t idS = idesc_bf16(128, 64, false, false);
     for (int it = 0; it < niter; ++it) {
         const int m = it / nhalf, hn = it % nhalf, buf = it & 1;
-        if (it >= 2 && !*abort_s) {
-            // the MMA of step it - 2 has released tile buffer `buf` and S buffer (it + 1) % 3
+        if (it >= 2 && !*abort_s) {  // the MMA of step it - 2 has released tile buffer `buf`
             if (!mbar_wait(&bars[6 + buf], ((it - 2) >> 1) & 1)) *abort_s = 1;
-            const int j = it + 1;
-            if (tid == 0 && j < niter && !*abort_s) {
-                mbar_arrive_expect_tx(&bars[3 + j % kSBuf], 8192u);
-                tma_load_3d(sS + (j % kSBuf) * 8192, &mapS, &bars[3 + j % kSBuf], (j % nhalf) * 64, 0,
-                            srow + j / nhalf);
-            }
         }
         // (f_m o C)[t, n] for this 64-wide n half; group g writes n in [32 g, 32 g + 32)
         float fm = 0.f;
@@ -581,6 +574,18 @@ __global__ void __launch_bounds__(kOutThreads, 2)
                 r[i] = pack_bf16x2(f.x * fm, f.y * fm);
             }
             *reinterpret_cast<uint4 *>(drow + off) = make_uint4(r[0], r[1], r[2], r[3]);
+        }
+        // S tile it + 2 into the buffer the MMA of step it - 1 read (two steps of lead); issued
+        // by a thread of another warp than the MMA issuer, after its own tile row is written
+        if (tid == 32 && it >= 1 && it + 2 < niter && !*abort_s) {
+            if (!mbar_wait(&bars[6 + ((it - 1) & 1)], ((it - 1) >> 1) & 1)) {
+                *abort_s = 1;
+            } else {
+                const int j = it + 2;
+                mbar_arrive_expect_tx(&bars[3 + j % kSBuf], 8192u);
+                tma_load_3d(sS + (j % kSBuf) * 8192, &mapS, &bars[3 + j % kSBuf], (j % nhalf) * 64, 0,
+                            srow + j / nhalf);
+            }
         }
         fence_async_smem();
         tc_fence_before();
