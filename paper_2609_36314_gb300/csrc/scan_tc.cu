@@ -52,7 +52,7 @@ struct StateSmem {
     __host__ __device__ StateSmem(int K, int N) {
         a_bytes = (K / 4) * 2 * 16384;  // K/4 M-tiles x 2 M-atoms x (128 k rows x 128 B), MN-major
         v_bytes = (N / 64) * 16384;     // N/64 boxes of [128 t][64 n]
-        total = a_bytes + v_bytes + TQ * KMAX * 4 /*cv*/ + 64 * 4 /*itau, dec*/ + 64 /*wsum*/ +
+        total = a_bytes + v_bytes + TQ * KMAX * 4 /*cv*/ + 96 * 4 /*itau, dec, l2t*/ + 64 /*wsum*/ +
                 16 /*E_end*/ + 64 /*bars*/;
     }
 };
@@ -69,10 +69,11 @@ __global__ void __launch_bounds__(kThreads, 2)
     unsigned char *sA = base;
     unsigned char *sV = sA + plan.a_bytes;
     float *cv_s = reinterpret_cast<float *>(sV + plan.v_bytes);  // [128][KMAX] this chunk's s or f
-    float *itau = cv_s + TQ * KMAX;                               // [32]
+    float *itau = cv_s + TQ * KMAX;                               // [32] 1 / tau
     float *dec = itau + 32;                                       // [32]
-    double *wsum = reinterpret_cast<double *>(dec + 32);          // [4]
-    double *Eend_s = wsum + 8;                                    // [1]
+    float *l2t = dec + 32;                                        // [32] log2(e) / tau
+    float2 *wsum = reinterpret_cast<float2 *>(l2t + 32);          // [8]
+    float2 *Eend_s = wsum + 8;                                    // [1] E at the chunk end (hi, lo)
     uint64_t *bars = reinterpret_cast<uint64_t *>(Eend_s + 2);    // tma, mma
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 2);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
@@ -91,7 +92,11 @@ __global__ void __launch_bounds__(kThreads, 2)
         *abort_s = 0;
         fence_barrier_init();
     }
-    if (tid < K) itau[tid] = 1.f / a.tau[h * K + tid];
+    if (tid < K) {
+        const float tv = a.tau[h * K + tid];
+        itau[tid] = 1.f / tv;
+        l2t[tid] = kLog2e / tv;
+    }
     if (w == 0) tmem_alloc_once(tslot, ncols);
     tc_fence_before();
     __syncthreads();
@@ -170,25 +175,26 @@ __global__ void __launch_bounds__(kThreads, 2)
             bool cl;
             e = token_rate(ndt, nal, nlm, log_cap, &cl);
         }
-        const double Et = block_scan128(double(e), wsum);
+        const float2 Et = group_scan128_f2(e, wsum);
         if (t == n - 1) *Eend_s = Et;
         if (ci + 1 < d.nc) fetch(ci + 1);
         __syncthreads();
         // this position's coefficient per mode: s = kappa exp(-(E_end - E_t)/tau) (forward) or
         // f = w_read exp(-E_t/tau) (reverse)
-        const double Eend = *Eend_s;
+        const float2 Eend = *Eend_s;
+        const float dEnd = diff_f2(Eend, Et);  // E_end - E_t >= 0
         float cv[KMAX];
 #pragma unroll
         for (int m = 0; m < KMAX; ++m) {
             cv[m] = 0.f;
             if (m < K && t < n) {
                 if (!REV)
-                    cv[m] = -expm1f(-e * itau[m]) * wcur[m] * expf(-float(Eend - Et) * itau[m]);
+                    cv[m] = -expm1f(-e * itau[m]) * wcur[m] * ex2_approx(-dEnd * l2t[m]);
                 else
-                    cv[m] = wcur[m] * expf(-float(Et) * itau[m]);
+                    cv[m] = wcur[m] * ex2_approx(-Et.x * l2t[m]);
             }
         }
-        if (t < K) dec[t] = expf(-float(Eend) * itau[t]);
+        if (t < K) dec[t] = ex2_approx(-Eend.x * l2t[t]);
         {
             float4 *o = reinterpret_cast<float4 *>(cv_s + t * KMAX);  // this thread's own row
             o[0] = make_float4(cv[0], cv[1], cv[2], cv[3]);
@@ -229,16 +235,14 @@ __global__ void __launch_bounds__(kThreads, 2)
             }
         }
         // emit the entering state (bf16) and apply the chunk's decay in place
-        for (int mt = 0; mt < mtiles; ++mt) {
-            const int m = mt * 4 + w;
-            const float dm = dec[m];
-            const size_t row = ((bh * d.nc + c) * K + m) * PN + size_t(p0 + j) * N;
-            bf16 *dst = a.emit + row;
-            for (int c32 = 0; c32 < N; c32 += 32) {
-                float v[32];
-                tmem_ld32(lane_base + mt * N + c32, v);
-                tmem_ld_wait();
-                uint4 *o = reinterpret_cast<uint4 *>(dst + c32);
+        // (the TMEM load of the next 32 columns is in flight while the current ones are processed)
+        {
+            const int nblk = mtiles * (N / 32);
+            auto process = [&](float *v, int blk) {
+                const int mt = blk / (N / 32), c32 = (blk % (N / 32)) * 32;
+                const int m = mt * 4 + w;
+                const float dm = dec[m];
+                uint4 *o = reinterpret_cast<uint4 *>(a.emit + ((bh * d.nc + c) * K + m) * PN + size_t(p0 + j) * N + c32);
 #pragma unroll
                 for (int q = 0; q < 4; ++q)
                     o[q] = make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
@@ -247,6 +251,19 @@ __global__ void __launch_bounds__(kThreads, 2)
                 for (int i = 0; i < 32; ++i) v[i] *= dm;
 #pragma unroll
                 for (int q = 0; q < 4; ++q) tmem_st8(lane_base + mt * N + c32 + 8 * q, v + 8 * q);
+            };
+            auto col = [&](int blk) { return lane_base + (blk / (N / 32)) * N + (blk % (N / 32)) * 32; };
+            float v0[32], v1[32];
+            tmem_ld32(col(0), v0);
+            for (int blk = 0; blk < nblk; blk += 2) {
+                tmem_ld_wait();
+                if (blk + 1 < nblk) tmem_ld32(col(blk + 1), v1);
+                process(v0, blk);
+                if (blk + 1 < nblk) {
+                    tmem_ld_wait();
+                    if (blk + 2 < nblk) tmem_ld32(col(blk + 2), v0);
+                    process(v1, blk + 1);
+                }
             }
         }
         tmem_st_wait();
@@ -259,12 +276,14 @@ __global__ void __launch_bounds__(kThreads, 2)
                 *abort_s = 1;
             } else {
                 const uint32_t idesc = idesc_bf16(128, N, true, true);
+                // descriptors advance by (byte offset >> 4) in their start-address field
+                const uint64_t ad0 = desc_sw128(smem_u32(sA), 16384, 1024);
+                const uint64_t bd0 = desc_sw128(smem_u32(sV), 16384, 1024);
                 for (int mt = 0; mt < mtiles; ++mt)
-                    for (int ks = 0; ks < TQ / 16; ++ks) {
-                        const uint64_t ad = desc_sw128(smem_u32(sA + mt * 32768) + ks * 2048, 16384, 1024);
-                        const uint64_t bd = desc_sw128(smem_u32(sV) + ks * 2048, 16384, 1024);
-                        mma_bf16(tmem + mt * N, ad, bd, idesc, 1);
-                    }
+#pragma unroll
+                    for (int ks = 0; ks < TQ / 16; ++ks)
+                        mma_bf16(tmem + mt * N, ad0 + uint64_t((mt * 32768 + ks * 2048) >> 4),
+                                 bd0 + uint64_t((ks * 2048) >> 4), idesc, 1);
                 mma_commit(&bars[1]);
             }
         }

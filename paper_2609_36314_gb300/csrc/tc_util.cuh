@@ -84,6 +84,37 @@ __device__ __forceinline__ float2 split_f2(double E) {
 }
 __device__ __forceinline__ float diff_f2(float2 a, float2 b) { return (a.x - b.x) + (a.y - b.y); }
 
+// Float-pair (hi + lo) arithmetic for the cumulative log-decay: Knuth's TwoSum keeps the
+// rounding error of every addition, so a prefix sum of 128 values carries ~48 significant bits
+// (the difference of two prefixes stays accurate to float precision of the difference).
+__device__ __forceinline__ float2 f2_add(float2 a, float2 b) {
+    const float s = a.x + b.x;
+    const float bb = s - a.x;
+    const float err = (a.x - (s - bb)) + (b.x - bb);
+    const float lo = err + a.y + b.y;
+    const float hi = s + lo;
+    return make_float2(hi, lo - (hi - s));
+}
+
+// Inclusive prefix sum of one value per thread within groups of four warps (threads
+// 128 g .. 128 g + 127 scan independently), as a float pair; wsum holds one pair per warp.
+__device__ __forceinline__ float2 group_scan128_f2(float v, float2 *wsum) {
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    float2 p = make_float2(v, 0.f);
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const float2 u = make_float2(__shfl_up_sync(0xffffffffu, p.x, o), __shfl_up_sync(0xffffffffu, p.y, o));
+        if (lane >= o) p = f2_add(p, u);
+    }
+    if (lane == 31) wsum[w] = p;
+    __syncthreads();
+    float2 off = make_float2(0.f, 0.f);
+    const int g0 = w & ~3;
+    for (int i = g0; i < w; ++i) off = f2_add(off, wsum[i]);
+    __syncthreads();
+    return f2_add(p, off);
+}
+
 // Inclusive prefix sum (double) of one value per thread within groups of four warps (threads
 // 128 g .. 128 g + 127 scan independently); wsum holds one slot per warp.
 __device__ __forceinline__ double group_scan128(double v, double *wsum) {
