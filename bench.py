@@ -29,6 +29,7 @@ sys.path.insert(0, ROOT)
 METRIC = "Frac scan tokens/s (prefill, fwd+bwd) and % of GB300 roofline; decode tok/s"
 TRAIN = "train_bf16_b8_l4096"
 DECODE = "decode_b128"
+PREFILL = "prefill_bf16_l65536"
 FALLBACK_PEAKS = dict(hbm_gbs=6800.0, bf16_tflops=1900.0, bf16_tflops_sustained=1700.0,
                       sm_max_mhz=2070.0)
 NUM_SMS = 152
@@ -42,6 +43,7 @@ def parse():
     ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
     ap.add_argument("--decode-steps", type=int, default=1024)
     ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-prefill", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--batch", type=int, default=0,
@@ -346,6 +348,10 @@ def main():
     tot = sum(t for _, t in trace.values()) or 1.0
     for k, (n, t) in trace.items():
         kern[k]["share"] = t / tot
+        tb = profiled_traffic(k, s.batch)
+        if tb is not None and kern[k]["avg_ms"] > 0:  # DRAM bytes of the ncu capture / launch time
+            kern[k]["dram_gbs"] = tb / (kern[k]["avg_ms"] / 1e3) / 1e9
+            kern[k]["dram_frac_of_peak"] = kern[k]["dram_gbs"] / peaks["hbm_gbs"]
     launches = sum(n for n, _ in trace.values())
     dom = max(trace.items(), key=lambda kv: kv[1][1])[0] if trace else None
     roofline = None
@@ -410,6 +416,9 @@ def main():
     decode = None
     if not args.no_decode:
         decode = bench_decode(args, dev, peaks, world, max_over_ranks, barrier)
+    prefill = None
+    if not args.no_prefill:
+        prefill = bench_prefill(args, dev, world, max_over_ranks, barrier)
 
     if rank == 0:
         line = {
@@ -427,7 +436,8 @@ def main():
                        "parallelism": f"replicas{world}" if world > 1 else "single",
                        "l2": "inputs larger than L2 (0.78 GB per step), no flush"},
             "roofline": roofline, "kernels": kern, "gpu_launches": launches,
-            "e2e": e2e, "decode": decode, "clocks": clk, "peaks_source": peaks["source"],
+            "e2e": e2e, "decode": decode, "prefill": prefill, "clocks": clk,
+            "peaks_source": peaks["source"],
         }
         if args.batch:
             line["config"]["workload"] += f" (batch overridden to {args.batch})"
@@ -436,6 +446,52 @@ def main():
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def bench_prefill(args, dev, world, max_over_ranks, barrier):
+    """Long-context prefill: the forward scan of B1 L65536 H64 P64 N128 K8 (Delta skewed small),
+    final state kept; tokens/s over the timed forwards (inputs resident, 1.3 GB > L2)."""
+    import torch
+
+    from paper_2609_36314_gb300 import _lib, scan_fwd, synth
+    from paper_2609_36314_gb300.api import fwd_workspace_size, make_dims
+    s = shape_of(PREFILL)
+    a = synth.make_scan_inputs_torch(s, seed=11, device=dev)
+    dims = make_dims(s.batch, s.seqlen, s.nheads, s.headdim, s.ngroups, s.dstate, s.nmodes,
+                     torch.bfloat16)
+    ws = torch.empty(fwd_workspace_size(dims), dtype=torch.uint8, device=dev)
+    y = torch.empty_like(a["x"])
+    hf = torch.empty((s.batch, s.nheads, s.nmodes, s.headdim, s.dstate), dtype=torch.float32, device=dev)
+
+    def fwd():
+        scan_fwd(a["x"], a["dt"], a["alpha"], a["lam"], a["tau"], a["B"], a["C"], a["w_read"],
+                 a["w_write"], a["D"], y=y, h_final=hf, workspace=ws)
+
+    for _ in range(3):
+        fwd()
+    torch.cuda.synchronize()
+    _lib.trace_reset()
+    _lib.trace_enable(True)
+    barrier()
+    stream = torch.cuda.current_stream()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    n = 5
+    ev0.record(stream)
+    for _ in range(n):
+        fwd()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    _lib.trace_enable(False)
+    ms = max_over_ranks(ev0.elapsed_time(ev1) / n)
+    kern = {k: {"launches": c, "avg_ms": t / max(c, 1)} for k, (c, t) in _lib.trace_collect().items()}
+    del a, ws, y, hf
+    torch.cuda.empty_cache()
+    return {"workload": f"{PREFILL}: forward of B{s.batch} L{s.seqlen} H{s.nheads} P{s.headdim} "
+                        f"N{s.dstate} K{s.nmodes}, Delta = softplus(z - {s.dt_shift}), final state "
+                        "kept; chunk 128 (results are chunk-independent)",
+            "value": world * s.batch * s.seqlen / (ms / 1e3), "unit": "tokens/s", "ms_per_forward": ms,
+            "kernels": kern}
 
 
 def bench_decode(args, dev, peaks, world, max_over_ranks, barrier):
