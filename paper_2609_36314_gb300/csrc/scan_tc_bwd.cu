@@ -52,30 +52,9 @@ struct BwdArgs {
     int hg;  // heads per dC/dB group
 };
 
-__device__ __forceinline__ float head_log_cap(const float *tau, int h, int K) {
-    float tmax = 0.f;
-    for (int m = 0; m < K; ++m) tmax = fmaxf(tmax, tau[h * K + m]);
-    return logf(64.f * tmax);
-}
-
 __device__ __forceinline__ void store_bf16x8(unsigned char *p, const float *v) {
     *reinterpret_cast<uint4 *>(p) = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
                                                pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
-}
-
-__device__ __forceinline__ void load_bf16x32(const bf16 *src, float *v) {
-    const uint4 *s4 = reinterpret_cast<const uint4 *>(src);
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        const uint4 u = s4[q];
-        const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&u);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const float2 f = __bfloat1622float2(h2[i]);
-            v[8 * q + 2 * i] = f.x;
-            v[8 * q + 2 * i + 1] = f.y;
-        }
-    }
 }
 
 __device__ __forceinline__ unsigned char *align1024(unsigned char *p) {
@@ -184,8 +163,8 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     const float2 Et2 = split_f2(Et);
     if (grp == 0) E_s[t] = Et2;
     float l2r[KMAX];  // log2(e) / tau per mode, in registers
-#pragma unroll
     float kap_t[KMAX];
+#pragma unroll
     for (int m = 0; m < KMAX; ++m) {
         l2r[m] = m < K ? l2t[m] : 0.f;
         float kp = 0.f;
@@ -533,8 +512,10 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
 // accumulates dx = sum_m s_m U_m in registers.  <dS_out,m, S_in,m> comes from the two tiles in
 // shared memory.  The head-summed intra tile Gamma o H adds M_H B to dC and M_H^T C to dB once
 // per (b, c, B/C group).
-constexpr int kStThreads = 256;
-constexpr int kStBuf = 3;  // S_in / dS_out tile buffers
+constexpr int kStThreads = 256;  // compute threads (two warpgroups); a ninth warp issues the MMAs
+                                 // and TMA loads (one thread)
+constexpr int kStBuf = 2;   // S_in / dS_out tile buffers
+constexpr int kCoefStride = 3 * KMAX + 1;  // per-thread coefficient row (odd: no bank conflicts)
 
 struct StSmem {
     int cb, tile, gen, total;
@@ -542,7 +523,7 @@ struct StSmem {
         cb = (N / 64) * 16384;   // one of C / B: [t][n]
         tile = (N / 64) * 8192;  // one S_in or dS_out mode tile: [p = 64][n], 64-wide n atoms
         gen = 2 * 16384;         // f o dY and s o X: [t][p] each; two buffers (the first holds M_H)
-        total = 2 * cb + kStBuf * 2 * tile + 2 * gen + 384;
+        total = 2 * cb + kStBuf * 2 * tile + 2 * gen + kStThreads * kCoefStride * 4 + 384;
     }
 };
 
@@ -567,7 +548,7 @@ __device__ __forceinline__ uint4 scale_bf16x8(uint4 a, float s) {
     return make_uint4(r[0], r[1], r[2], r[3]);
 }
 
-__global__ void __launch_bounds__(kStThreads, 1)
+__global__ void __launch_bounds__(kStThreads + 32, 1)
     tc_bwd_state(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapB,
                  const __grid_constant__ CUtensorMap mapS, const __grid_constant__ CUtensorMap mapD,
                  BwdArgs a) {
@@ -578,7 +559,9 @@ __global__ void __launch_bounds__(kStThreads, 1)
     const StSmem L(N);
     unsigned char *sC = base, *sB = sC + L.cb, *sT = sB + L.cb;
     unsigned char *sG = sT + kStBuf * 2 * L.tile;             // [buf][f o dY | s o X]
-    float *itau_s = reinterpret_cast<float *>(sG + 2 * L.gen);  // [hg][K] 1 / tau
+    // this thread's mode coefficients for the current head: cA (f or s), cB (exp(-E/tau) or u), s
+    float *coef_s = reinterpret_cast<float *>(sG + 2 * L.gen);  // [256][kCoefStride]
+    float *itau_s = coef_s + kStThreads * kCoefStride;         // [hg][K] 1 / tau
     double *wsum = reinterpret_cast<double *>(itau_s + 32);     // [8]
     double *Eend_s = wsum + 8;                                  // [1]
     // bars: 0..2 tile buffers | 3, 4 MMA of step parity | 5 C, B | 6 intra MMA |
@@ -611,7 +594,8 @@ __global__ void __launch_bounds__(kStThreads, 1)
     const uint32_t tmem = *tslot;
     const uint32_t lane_base = tmem + (uint32_t(w4 * 32) << 16);
 
-    auto issue_tiles = [&](int i) {  // thread 0: S_in / dS_out tiles of step i into buffer i % 3
+    const bool issuer = tid == kStThreads;  // lane 0 of the ninth warp
+    auto issue_tiles = [&](int i) {  // issuer: S_in / dS_out tiles of step i into buffer i % 3
         const int q = i % kStBuf;
         const int srow = int(((size_t(b) * d.H + h_first + i / K) * d.nc + c) * K + i % K);
         mbar_arrive_expect_tx(&bars[q], uint32_t(2 * L.tile));
@@ -620,7 +604,7 @@ __global__ void __launch_bounds__(kStThreads, 1)
             tma_load_3d(sT + (2 * q + 1) * L.tile + jb * 8192, &mapD, &bars[q], 64 * jb, 0, srow);
         }
     };
-    if (tid == 0) {
+    if (issuer) {
         mbar_arrive_expect_tx(&bars[5], uint32_t(2 * L.cb));
         for (int jb = 0; jb < N / 64; ++jb) {
             tma_load_3d(sC + jb * 16384, &mapC, &bars[5], g * N + 64 * jb, c0, b);
@@ -633,7 +617,7 @@ __global__ void __launch_bounds__(kStThreads, 1)
     if (intra) {
         const float *mrow = a.mh_total + (((size_t(b) * d.nc + c) * d.G + g) * TQ + t) * TQ + grp * 64;
 #pragma unroll
-        for (int k8 = 0; k8 < 64; k8 += 8) {
+        for (int k8 = 0; k8 < 64 && tid < kStThreads; k8 += 8) {
             const float4 u0 = *reinterpret_cast<const float4 *>(mrow + k8);
             const float4 u1 = *reinterpret_cast<const float4 *>(mrow + k8 + 4);
             const float v[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
@@ -641,7 +625,7 @@ __global__ void __launch_bounds__(kStThreads, 1)
         }
         fence_async_smem();
         __syncthreads();
-        if (tid == 0) {
+        if (issuer) {
             if (!mbar_wait(&bars[5], 0)) {
                 *abort_s = 1;
             } else {
@@ -663,38 +647,35 @@ __global__ void __launch_bounds__(kStThreads, 1)
     if (!*abort_s && !mbar_wait(&bars[5], 0)) *abort_s = 1;      // C and B are read below
 
     // mode coefficients of row t: group 0 cA = f, cB = exp(-E/tau); group 1 cA = s, cB = u
-    float cA[KMAX], cB[KMAX];
+    float *my_coef = coef_s + (tid < kStThreads ? tid : 0) * kCoefStride;  // cA [0, 8), cB [8, 16), s [16, 24)
     uint4 row[8];     // group 0: dY row (64 p), group 1: X row
-    float dxr[64];    // group 1: inter-chunk dx of this row, current head
+    float dxr[32];    // inter-chunk dx of this row, p in [32 grp, 32 grp + 32), current head
     float acc_h[KMAX], ab_h = 0.f;  // group 0: dw_read and a; group 1: dkappa and b
 #pragma unroll
-    for (int m = 0; m < KMAX; ++m) cA[m] = cB[m] = acc_h[m] = 0.f;
+    for (int m = 0; m < KMAX; ++m) acc_h[m] = 0.f;
 #pragma unroll
     for (int q = 0; q < 8; ++q) row[q] = make_uint4(0, 0, 0, 0);
 #pragma unroll
-    for (int p = 0; p < 64; ++p) dxr[p] = 0.f;
+    for (int p = 0; p < 32; ++p) dxr[p] = 0.f;
 
-    // read out step j (its MMAs complete): Z (group 0) or U (group 1) against this row
+    // read out step j (its MMAs complete): Z (group 0) or U (group 1) against this row, and
+    // dx[t, p] += s_m U_m[t, p] with group g taking p in [32 g, 32 g + 32)
     auto readout = [&](int j) {
         if (!*abort_s && !mbar_wait(&bars[3 + (j & 1)], (j >> 1) & 1)) *abort_s = 1;
         tc_fence_after();
-        if (tid == 0 && j + kStBuf < nsteps && !*abort_s) issue_tiles(j + kStBuf);  // buffer of step j
         const int mj = j % K, hj = h_first + j / K;
         if (!*abort_s) {
-            const uint32_t col = colZU + 128 * (j & 1) + 64 * grp;
-            float sj = 0.f;
-#pragma unroll
-            for (int m = 0; m < KMAX; ++m)
-                if (m == mj) sj = cA[m];
+            const uint32_t zu = lane_base + colZU + 128 * (j & 1);  // Z at +0, U at +64
+            const float sj = my_coef[2 * KMAX + mj], aj = my_coef[mj], bj = my_coef[KMAX + mj];
             float dp[4] = {0.f, 0.f, 0.f, 0.f};  // independent partial sums
 #pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                float zv[32];
-                tmem_ld32(lane_base + col + half * 32, zv);
+            for (int pc = 0; pc < 4; ++pc) {
+                float zv[16];
+                tmem_ld16(zu + 64 * grp + 16 * pc, zv);
                 tmem_ld_wait();
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const uint4 rv = row[half * 4 + q];
+                for (int q = 0; q < 2; ++q) {
+                    const uint4 rv = row[2 * pc + q];
                     const uint32_t rr[4] = {rv.x, rv.y, rv.z, rv.w};
 #pragma unroll
                     for (int k = 0; k < 4; ++k) {
@@ -702,19 +683,27 @@ __global__ void __launch_bounds__(kStThreads, 1)
                         dp[k] = fmaf(f.x, zv[8 * q + 2 * k], fmaf(f.y, zv[8 * q + 2 * k + 1], dp[k]));
                     }
                 }
-                if (grp == 1) {
+                if (grp == 1 && pc >= 2) {
 #pragma unroll
-                    for (int p = 0; p < 32; ++p) dxr[half * 32 + p] = fmaf(sj, zv[p], dxr[half * 32 + p]);
+                    for (int i = 0; i < 16; ++i) dxr[16 * (pc - 2) + i] = fmaf(sj, zv[i], dxr[16 * (pc - 2) + i]);
+                }
+            }
+            if (grp == 0) {
+#pragma unroll
+                for (int pc = 0; pc < 2; ++pc) {
+                    float zv[16];
+                    tmem_ld16(zu + 64 + 16 * pc, zv);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) dxr[16 * pc + i] = fmaf(sj, zv[i], dxr[16 * pc + i]);
                 }
             }
             const float dotv = (dp[0] + dp[1]) + (dp[2] + dp[3]);
 #pragma unroll
             for (int m = 0; m < KMAX; ++m) {
-                if (m == mj) {  // group 0: dw_read (inter) and a; group 1: dkappa (inter) and b
-                    acc_h[m] = cB[m] * dotv;
-                    ab_h = fmaf(cA[m] * dotv, itau_s[(j / K) * K + m], ab_h);
-                }
+                if (m == mj) acc_h[m] = bj * dotv;  // group 0: dw_read (inter); group 1: dkappa (inter)
             }
+            ab_h = fmaf(aj * dotv, itau_s[(j / K) * K + mj], ab_h);  // group 0: a; group 1: b
         }
         if (mj == K - 1 && !*abort_s && t < n) {  // head hj complete: reductions, nothing waits
             const size_t i0 = blh(d, b, c0 + t, hj);
@@ -724,16 +713,55 @@ __global__ void __launch_bounds__(kStThreads, 1)
                 if (4 * q < K)
                     atomicAdd(acc_dst + q, make_float4(acc_h[4 * q], acc_h[4 * q + 1], acc_h[4 * q + 2], acc_h[4 * q + 3]));
             a.ab_acc[i0 * 2 + grp] = ab_h;
-            if (grp == 1) {
-                float4 *o = reinterpret_cast<float4 *>(a.dx_acc + i0 * P);
+            float4 *o = reinterpret_cast<float4 *>(a.dx_acc + i0 * P + 32 * grp);
 #pragma unroll
-                for (int q = 0; q < 16; ++q)
-                    atomicAdd(o + q, make_float4(dxr[4 * q], dxr[4 * q + 1], dxr[4 * q + 2], dxr[4 * q + 3]));
-            }
+            for (int q = 0; q < 8; ++q)
+                atomicAdd(o + q, make_float4(dxr[4 * q], dxr[4 * q + 1], dxr[4 * q + 2], dxr[4 * q + 3]));
         }
     };
 
-    for (int i = 0; i < nsteps; ++i) {
+    if (issuer) {
+        // the MMAs of step i once all compute threads have written its generated operands; then,
+        // once step i - 1 has finished, its tile buffer takes the tiles of step i + 2
+        for (int i = 0; i < nsteps && !*abort_s; ++i) {
+            const int gb = i & 1, q = i % kStBuf;
+            // step i - 1's MMAs are done (they were issued at the tensor cores' pace): its tile
+            // buffer takes the tiles of step i - 1 + kStBuf before step i's operands are awaited
+            if (i >= 1) {
+                if (!mbar_wait(&bars[3 + ((i - 1) & 1)], ((i - 1) >> 1) & 1)) {
+                    *abort_s = 1;
+                    break;
+                }
+                if (i - 1 + kStBuf < nsteps) issue_tiles(i - 1 + kStBuf);
+            }
+            if (!mbar_wait(&bars[7 + gb], (i >> 1) & 1) || !mbar_wait(&bars[q], (i / kStBuf) & 1)) {
+                *abort_s = 1;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t sS = smem_u32(sT + (2 * q) * L.tile), sD = smem_u32(sT + (2 * q + 1) * L.tile);
+            const uint32_t g1 = smem_u32(sG + gb * L.gen), g2 = g1 + 16384;
+            const uint32_t id64 = idesc_bf16(128, 64, false, false);
+            const uint32_t idN = idesc_bf16(128, N, false, true);
+            const uint32_t zc = colZU + 128 * gb;
+            for (int ks = 0; ks < N / 16; ++ks) {
+                const uint32_t ko = (ks / 4) * 16384 + (ks % 4) * 32, to = (ks / 4) * 8192 + (ks % 4) * 32;
+                mma_bf16(tmem + zc, desc_sw128(smem_u32(sC) + ko, 16, 1024), desc_sw128(sS + to, 16, 1024),
+                         id64, ks > 0);
+                mma_bf16(tmem + zc + 64, desc_sw128(smem_u32(sB) + ko, 16, 1024),
+                         desc_sw128(sD + to, 16, 1024), id64, ks > 0);
+            }
+            const bool acc0 = intra || i > 0;
+            for (int ks = 0; ks < 4; ++ks) {  // K = p
+                mma_bf16(tmem + colC, desc_sw128(g1 + ks * 32, 16, 1024), desc_sw128(sS + ks * 2048, 8192, 1024),
+                         idN, (acc0 || ks > 0) ? 1u : 0u);
+                mma_bf16(tmem + colB, desc_sw128(g2 + ks * 32, 16, 1024), desc_sw128(sD + ks * 2048, 8192, 1024),
+                         idN, (acc0 || ks > 0) ? 1u : 0u);
+            }
+            mma_commit(&bars[3 + gb]);
+        }
+    }
+    for (int i = 0; i < nsteps && tid < kStThreads; ++i) {
         const int hh = i / K, m = i % K, h = h_first + hh, gb = i & 1, q = i % kStBuf;
         bool prev_done = i == 0;
         if (m == 0) {
@@ -744,20 +772,19 @@ __global__ void __launch_bounds__(kStThreads, 1)
                 prev_done = true;
             }
 #pragma unroll
-            for (int k = 0; k < KMAX; ++k) {
-                cA[k] = cB[k] = 0.f;
-                acc_h[k] = 0.f;
-            }
+            for (int k = 0; k < KMAX; ++k) acc_h[k] = 0.f;
+            float4 c4[6];
+#pragma unroll
+            for (int k = 0; k < 6; ++k) c4[k] = make_float4(0.f, 0.f, 0.f, 0.f);
             if (t < n) {  // coefficients of this row from tc_bwd_intra; group 0: f, exp(-E/tau); 1: s, u
                 const size_t i0 = blh(d, b, c0 + t, h);
                 const float4 *cf = reinterpret_cast<const float4 *>(a.coef + i0 * 4 * K);
 #pragma unroll
                 for (int q = 0; q < KMAX / 4; ++q) {
                     if (4 * q < K) {
-                        const float4 v0 = cf[(grp == 0 ? 0 : 1) * (K / 4) + q];
-                        const float4 v1 = cf[(grp == 0 ? 3 : 2) * (K / 4) + q];
-                        cA[4 * q] = v0.x; cA[4 * q + 1] = v0.y; cA[4 * q + 2] = v0.z; cA[4 * q + 3] = v0.w;
-                        cB[4 * q] = v1.x; cB[4 * q + 1] = v1.y; cB[4 * q + 2] = v1.z; cB[4 * q + 3] = v1.w;
+                        c4[q] = cf[(grp == 0 ? 0 : 1) * (K / 4) + q];
+                        c4[2 + q] = cf[(grp == 0 ? 3 : 2) * (K / 4) + q];
+                        c4[4 + q] = cf[K / 4 + q];
                     }
                 }
                 const uint4 *src = reinterpret_cast<const uint4 *>((grp == 0 ? a.dy : a.x) + i0 * P);
@@ -767,16 +794,18 @@ __global__ void __launch_bounds__(kStThreads, 1)
 #pragma unroll
                 for (int k = 0; k < 8; ++k) row[k] = make_uint4(0, 0, 0, 0);
             }
+#pragma unroll
+            for (int k = 0; k < 6; ++k) {  // this thread's row: scalar stores (the row stride is odd)
+                float *dst = my_coef + (k >> 1) * KMAX + (k & 1) * 4;
+                dst[0] = c4[k].x; dst[1] = c4[k].y; dst[2] = c4[k].z; dst[3] = c4[k].w;
+            }
             ab_h = 0.f;
 #pragma unroll
-            for (int p = 0; p < 64; ++p) dxr[p] = 0.f;
+            for (int p = 0; p < 32; ++p) dxr[p] = 0.f;
         }
         // generated operands of step i into buffer gb (step i - 2 has finished reading it)
         {
-            float sc = 0.f;
-#pragma unroll
-            for (int k = 0; k < KMAX; ++k)
-                if (k == m) sc = cA[k];
+            const float sc = my_coef[m];
             unsigned char *dst = sG + gb * L.gen + grp * 16384 + t * 128;
 #pragma unroll
             for (int k = 0; k < 8; ++k)
@@ -799,39 +828,13 @@ __global__ void __launch_bounds__(kStThreads, 1)
         fence_async_smem();
         tc_fence_before();
         mbar_arrive(&bars[7 + gb]);
-        if (tid == 0 && !*abort_s) {
-            if (!mbar_wait(&bars[7 + gb], (i >> 1) & 1)) *abort_s = 1;
-            tc_fence_after();
-        }
-        if (tid == 0 && !*abort_s) {
-            const uint32_t sS = smem_u32(sT + (2 * q) * L.tile), sD = smem_u32(sT + (2 * q + 1) * L.tile);
-            const uint32_t g1 = smem_u32(sG + gb * L.gen), g2 = g1 + 16384;
-            const uint32_t id64 = idesc_bf16(128, 64, false, false);
-            const uint32_t idN = idesc_bf16(128, N, false, true);
-            const uint32_t zc = colZU + 128 * gb;
-            for (int ks = 0; ks < N / 16; ++ks) {
-                const uint32_t ko = (ks / 4) * 16384 + (ks % 4) * 32, to = (ks / 4) * 8192 + (ks % 4) * 32;
-                mma_bf16(tmem + zc, desc_sw128(smem_u32(sC) + ko, 16, 1024), desc_sw128(sS + to, 16, 1024),
-                         id64, ks > 0);
-                mma_bf16(tmem + zc + 64, desc_sw128(smem_u32(sB) + ko, 16, 1024),
-                         desc_sw128(sD + to, 16, 1024), id64, ks > 0);
-            }
-            const bool acc0 = intra || i > 0;
-            for (int ks = 0; ks < 4; ++ks) {  // K = p
-                mma_bf16(tmem + colC, desc_sw128(g1 + ks * 32, 16, 1024), desc_sw128(sS + ks * 2048, 8192, 1024),
-                         idN, (acc0 || ks > 0) ? 1u : 0u);
-                mma_bf16(tmem + colB, desc_sw128(g2 + ks * 32, 16, 1024), desc_sw128(sD + ks * 2048, 8192, 1024),
-                         idN, (acc0 || ks > 0) ? 1u : 0u);
-            }
-            mma_commit(&bars[3 + gb]);
-        }
         // step i - 1 is read out while the tensor cores run step i
         if (!prev_done) readout(i - 1);
     }
-    if (nsteps > 0) readout(nsteps - 1);
+    if (nsteps > 0 && tid < kStThreads) readout(nsteps - 1);
     // the group's dC / dB into the float32 accumulators (group g takes n in [64 g, 64 g + 64))
     tc_fence_after();
-    if (!*abort_s && grp < N / 64) {
+    if (!*abort_s && tid < kStThreads && grp < N / 64) {
         const size_t gi = ((size_t(b) * d.L + c0 + min(t, n - 1)) * d.G + g) * N + grp * 64;
         for (int n32 = 0; n32 < 64; n32 += 32) {
             float vc[32], vb[32];
@@ -1087,7 +1090,7 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
         const size_t smem = StSmem(d.N).total + 1024;
         cudaFuncSetAttribute(tc_bwd_state, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
         trace_begin("bwd_state_tc", st);
-        tc_bwd_state<<<dim3(d.H / a.hg, d.nc, d.B), kStThreads, smem, st>>>(mapC, mapB, mapS, mapD, a);
+        tc_bwd_state<<<dim3(d.H / a.hg, d.nc, d.B), kStThreads + 32, smem, st>>>(mapC, mapB, mapS, mapD, a);
         trace_end(st);
         if ((e = cudaGetLastError())) return e;
     }
