@@ -509,49 +509,45 @@ __global__ void __launch_bounds__(kOutThreads, 2)
     if (!*abort_s) {
         // row t of Gamma o G -> bf16, K-major [t][k] over the B tile.  Warp rows are one 32-block
         // I; column block kc < I takes the factored Gamma, kc == I the direct sum (pairs k <= t),
-        // kc > I is zero.  Group 0 takes kc = 0, 1, group 1 kc = 2, 3; eight columns at a time
-        // with rolled outer loops (compact code: the unrolled pass overflowed the instruction cache)
+        // kc > I is zero.  The 8-column items (kc, q8) alternate between the two groups, so both
+        // take half of every block (the diagonal one included); loops stay rolled (compact code)
         const int I = t >> 5;
 #pragma unroll 1
-        for (int h2 = 0; h2 < 2; ++h2) {
-            const int kc = grp * 2 + h2;
-            unsigned char *tile = sM + (kc >> 1) * 16384 + t * 128;
-#pragma unroll 1
-            for (int q8 = 0; q8 < 4; ++q8) {
-                const int k0 = 32 * kc + 8 * q8;
-                float gv[8];
-                if (kc < I) {
-                    float gm[8];
-                    tmem_ld8(lane_base + colG + k0, gv);
-                    tmem_ld8(lane_base + colGam + k0, gm);
-                    tmem_ld_wait();
+        for (int it = grp; it < 16; it += 2) {
+            const int kc = it >> 2, q8 = it & 3;
+            const int k0 = 32 * kc + 8 * q8;
+            float gv[8];
+            if (kc < I) {
+                float gm[8];
+                tmem_ld8(lane_base + colG + k0, gv);
+                tmem_ld8(lane_base + colGam + k0, gm);
+                tmem_ld_wait();
 #pragma unroll
-                    for (int kk = 0; kk < 8; ++kk) gv[kk] *= gm[kk];
-                } else if (kc == I) {
-                    tmem_ld8(lane_base + colG + k0, gv);
-                    tmem_ld_wait();
+                for (int kk = 0; kk < 8; ++kk) gv[kk] *= gm[kk];
+            } else if (kc == I) {
+                tmem_ld8(lane_base + colG + k0, gv);
+                tmem_ld_wait();
 #pragma unroll
-                    for (int kk = 0; kk < 8; ++kk) {
-                        const int k = k0 + kk;
-                        float v = 0.f;
-                        if (k <= t && t < n) {
-                            const float dE = diff_f2(Et2, E_s[k]);
-                            float gam = 0.f;
+                for (int kk = 0; kk < 8; ++kk) {
+                    const int k = k0 + kk;
+                    float v = 0.f;
+                    if (k <= t && t < n) {
+                        const float dE = diff_f2(Et2, E_s[k]);
+                        float gam = 0.f;
 #pragma unroll
-                            for (int m = 0; m < KMAX; ++m)
-                                if (m < K) gam = fmaf(wr_t[m] * kap_s[k * KMAX + m], ex2_approx(-dE * l2t[m]), gam);
-                            v = gam * gv[kk];
-                        }
-                        gv[kk] = v;
+                        for (int m = 0; m < KMAX; ++m)
+                            if (m < K) gam = fmaf(wr_t[m] * kap_s[k * KMAX + m], ex2_approx(-dE * l2t[m]), gam);
+                        v = gam * gv[kk];
                     }
-                } else {
-#pragma unroll
-                    for (int kk = 0; kk < 8; ++kk) gv[kk] = 0.f;
+                    gv[kk] = v;
                 }
-                *reinterpret_cast<uint4 *>(tile + ((((kc & 1) * 4 + q8) ^ (t & 7)) * 16)) =
-                    make_uint4(pack_bf16x2(gv[0], gv[1]), pack_bf16x2(gv[2], gv[3]), pack_bf16x2(gv[4], gv[5]),
-                               pack_bf16x2(gv[6], gv[7]));
+            } else {
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk) gv[kk] = 0.f;
             }
+            *reinterpret_cast<uint4 *>(sM + (kc >> 1) * 16384 + t * 128 + ((((kc & 1) * 4 + q8) ^ (t & 7)) * 16)) =
+                make_uint4(pack_bf16x2(gv[0], gv[1]), pack_bf16x2(gv[2], gv[3]), pack_bf16x2(gv[4], gv[5]),
+                           pack_bf16x2(gv[6], gv[7]));
         }
     }
     fence_async_smem();

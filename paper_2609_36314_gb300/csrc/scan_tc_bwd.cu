@@ -288,89 +288,86 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     if (!*abort_s) {
         const int I = t >> 5;
         float *mh_row = a.mh_total + (((size_t(b) * d.nc + c) * d.G + g) * TQ + t) * TQ;
-        // outer loops stay rolled: the fully unrolled pass overflowed the instruction cache
-#pragma unroll 1
-        for (int h2 = 0; h2 < 2; ++h2) {
-            const int kc = grp * 2 + h2;
-            unsigned char *tile = sMG + (kc >> 1) * 16384 + t * 128;
-            if (kc > I) {
-#pragma unroll 1
-                for (int q = 0; q < 4; ++q) {
-                    *reinterpret_cast<uint4 *>(tile + ((((kc & 1) * 4 + q) ^ (t & 7)) * 16)) = make_uint4(0, 0, 0, 0);
+        // 8-column work items (column block kc, eighth q8) alternate between the two groups, so
+        // that both take half of every block, the diagonal one included; loops stay rolled (the
+        // fully unrolled pass overflowed the instruction cache)
+        float acc[KMAX];
 #pragma unroll
-                    for (int kk = 0; kk < 8; ++kk) XX[t * XS + 32 * kc + 8 * q + kk] = 0.f;  // rows are 129 floats apart
-                }
+        for (int m = 0; m < KMAX; ++m) acc[m] = 0.f;
+#pragma unroll 1
+        for (int it = grp; it < 16; it += 2) {
+            const int kc = it >> 2, q8 = it & 3;
+            const int k0 = 32 * kc + 8 * q8;
+            unsigned char *mg = sMG + (kc >> 1) * 16384 + t * 128 + ((((kc & 1) * 4 + q8) ^ (t & 7)) * 16);
+            if (kc > I) {
+                *reinterpret_cast<uint4 *>(mg) = make_uint4(0, 0, 0, 0);
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk) XX[t * XS + k0 + kk] = 0.f;  // rows are 129 floats apart
                 continue;
             }
-            float acc[KMAX];
+            float gv[8], hv[8];
+            tmem_ld8(lane_base + colG + k0, gv);
+            tmem_ld8(lane_base + colH + k0, hv);
+            if (kc < I) {
+                float gm[8], gp[8];
+                tmem_ld8(lane_base + colGam + k0, gm);
+                tmem_ld8(lane_base + colGamP + k0, gp);
+                tmem_ld_wait();
 #pragma unroll
-            for (int m = 0; m < KMAX; ++m) acc[m] = 0.f;
-#pragma unroll 1
-            for (int q8 = 0; q8 < 4; ++q8) {  // eight columns at a time
-                const int k0 = 32 * kc + 8 * q8;
-                float gv[8], hv[8];
-                tmem_ld8(lane_base + colG + k0, gv);
-                tmem_ld8(lane_base + colH + k0, hv);
-                if (kc < I) {
-                    float gm[8], gp[8];
-                    tmem_ld8(lane_base + colGam + k0, gm);
-                    tmem_ld8(lane_base + colGamP + k0, gp);
-                    tmem_ld_wait();
+                for (int kk = 0; kk < 8; ++kk) {
+                    const int k = k0 + kk;
+                    const float gh = gv[kk] * hv[kk];
+                    XX[t * XS + k] = gp[kk] * gh;
+                    GHs[t * XS + k] = gh;
+                    const float4 v0 = *reinterpret_cast<const float4 *>(Vs + k * KMAX);
+                    const float4 v1 = *reinterpret_cast<const float4 *>(Vs + k * KMAX + 4);
+                    const float vk[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
 #pragma unroll
-                    for (int kk = 0; kk < 8; ++kk) {
-                        const int k = k0 + kk;
-                        const float gh = gv[kk] * hv[kk];
-                        XX[t * XS + k] = gp[kk] * gh;
-                        GHs[t * XS + k] = gh;
-                        const float4 v0 = *reinterpret_cast<const float4 *>(Vs + k * KMAX);
-                        const float4 v1 = *reinterpret_cast<const float4 *>(Vs + k * KMAX + 4);
-                        const float vk[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+                    for (int m = 0; m < KMAX; ++m) acc[m] = fmaf(vk[m], gh, acc[m]);
+                    gv[kk] *= gm[kk];  // Gamma o G
+                    hv[kk] *= gm[kk];  // Gamma o H
+                }
+            } else {
+                tmem_ld_wait();
 #pragma unroll
-                        for (int m = 0; m < KMAX; ++m) acc[m] = fmaf(vk[m], gh, acc[m]);
-                        gv[kk] *= gm[kk];  // Gamma o G
-                        hv[kk] *= gm[kk];  // Gamma o H
-                    }
-                } else {
-                    tmem_ld_wait();
+                for (int kk = 0; kk < 8; ++kk) {
+                    const int k = k0 + kk;
+                    float gam = 0.f, gamt = 0.f, gh = 0.f;
+                    if (k <= t && t < n) {
+                        const float dE = diff_f2(Et2, E_s[k]);
+                        gh = gv[kk] * hv[kk];
 #pragma unroll
-                    for (int kk = 0; kk < 8; ++kk) {
-                        const int k = k0 + kk;
-                        float gam = 0.f, gamt = 0.f, gh = 0.f;
-                        if (k <= t && t < n) {
-                            const float dE = diff_f2(Et2, E_s[k]);
-                            gh = gv[kk] * hv[kk];
-#pragma unroll
-                            for (int m = 0; m < KMAX; ++m) {
-                                if (m < K) {
-                                    const float W = ex2_approx(-dE * l2r[m]);
-                                    const float kp = kap_s[k * KMAX + m];
-                                    const float aa = wr_t[m] * kp * W;
-                                    gam += aa;
-                                    gamt = fmaf(aa, l2r[m], gamt);  // times log2(e) / tau
-                                    dwr_i[m] = fmaf(kp * W, gh, dwr_i[m]);
-                                }
+                        for (int m = 0; m < KMAX; ++m) {
+                            if (m < K) {
+                                const float W = ex2_approx(-dE * l2r[m]);
+                                const float kp = kap_s[k * KMAX + m];
+                                const float aa = wr_t[m] * kp * W;
+                                gam += aa;
+                                gamt = fmaf(aa, l2r[m], gamt);  // times log2(e) / tau
+                                dwr_i[m] = fmaf(kp * W, gh, dwr_i[m]);
                             }
                         }
-                        gv[kk] = gam * gv[kk];
-                        hv[kk] = gam * hv[kk];
-                        XX[t * XS + k] = gamt * (1.f / kLog2e) * gh;
-                        GHs[t * XS + k] = gh;
                     }
-                }
-                *reinterpret_cast<uint4 *>(tile + ((((kc & 1) * 4 + q8) ^ (t & 7)) * 16)) =
-                    make_uint4(pack_bf16x2(gv[0], gv[1]), pack_bf16x2(gv[2], gv[3]), pack_bf16x2(gv[4], gv[5]),
-                               pack_bf16x2(gv[6], gv[7]));
-                if (t < n && k0 <= t) {
-                    atomicAdd(reinterpret_cast<float4 *>(mh_row + k0), make_float4(hv[0], hv[1], hv[2], hv[3]));
-                    if (k0 + 4 <= t)
-                        atomicAdd(reinterpret_cast<float4 *>(mh_row + k0 + 4), make_float4(hv[4], hv[5], hv[6], hv[7]));
+                    gv[kk] = gam * gv[kk];
+                    hv[kk] = gam * hv[kk];
+                    XX[t * XS + k] = gamt * (1.f / kLog2e) * gh;
+                    GHs[t * XS + k] = gh;
                 }
             }
-            if (kc < I) {  // intra dw_read of the factored block: exp(-(E_t - E_a)/tau) sum_k V G H
+            *reinterpret_cast<uint4 *>(mg) = make_uint4(pack_bf16x2(gv[0], gv[1]), pack_bf16x2(gv[2], gv[3]),
+                                                        pack_bf16x2(gv[4], gv[5]), pack_bf16x2(gv[6], gv[7]));
+            if (t < n && k0 <= t) {
+                atomicAdd(reinterpret_cast<float4 *>(mh_row + k0), make_float4(hv[0], hv[1], hv[2], hv[3]));
+                if (k0 + 4 <= t)
+                    atomicAdd(reinterpret_cast<float4 *>(mh_row + k0 + 4), make_float4(hv[4], hv[5], hv[6], hv[7]));
+            }
+            if (kc < I && q8 >= 2) {  // this thread's last item of the factored block kc
                 const float dE = diff_f2(Et2, E_s[32 * kc + 31]);
 #pragma unroll
-                for (int m = 0; m < KMAX; ++m)
+                for (int m = 0; m < KMAX; ++m) {
                     if (m < K) dwr_i[m] = fmaf(ex2_approx(-dE * l2r[m]), acc[m], dwr_i[m]);
+                    acc[m] = 0.f;
+                }
             }
         }
         if (grp == 1) {
