@@ -393,14 +393,16 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         mma_commit(&bars[2]);
     }
     __syncthreads();  // part[] is reused below
-    // ---- column pass (column k = t, group g takes rows of parity g): intra dkappa.  Rows of
+    // ---- column pass (group g takes the rows of parity g of column k): intra dkappa.  Rows of
     // later blocks use the factored form exp(-(E_a - E_k)/tau) sum_t U_J[t, m] G H[t, k]; rows of
-    // the diagonal block (t >= k) sum directly.
+    // the diagonal block (t >= k) sum directly.  Column block J has 128 - 32 J rows, so group 1's
+    // warp w takes block 3 - w: every SM sub-partition gets blocks J and 3 - J.
+    const int kcol = grp == 0 ? t : (((3 - (t >> 5)) << 5) | (t & 31));
     float dk[KMAX];
 #pragma unroll
     for (int m = 0; m < KMAX; ++m) dk[m] = 0.f;
     if (!*abort_s) {
-        const int k = t, J = k >> 5;
+        const int k = kcol, J = k >> 5;
         const float2 Ek = E_s[k];
         float dk2[KMAX];
 #pragma unroll
@@ -459,24 +461,39 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
             for (int m = 0; m < KMAX; ++m) part[k * KMAX + m] = dk[m];
         }
     }
-    // exclusive row prefix of XX (row t, group 0)
-    if (!*abort_s && grp == 0) {
+    // exclusive row prefix of XX (row t): group 0 over j in [0, 64) (its total in xtot), group 1
+    // over [64, 128) starting from 0; the column sums below add the suffix sum of xtot for the
+    // columns j >= 64
+    float *xtot = Vs;  // [128], free after the row pass
+    if (!*abort_s) {
         float run = 0.f;
-        for (int j = 0; j < TQ; ++j) {
+        for (int j = 64 * grp; j < 64 * grp + 64; ++j) {
             const float v = XX[t * XS + j];
             XX[t * XS + j] = run;
             run += v;
         }
+        if (grp == 0) xtot[t] = run;
     }
+    __syncthreads();
+    // rect[j] = sum_{t' >= j} sum_{k < j} X[t', k]: column j's suffix sum of the row prefixes,
+    // rows of parity g in group g (column kcol, the column pass's balanced assignment)
+    float *rpart = Vs + TQ;  // [128] group 1's partial rect
+    float sr = 0.f;
+    if (!*abort_s) {
+        const int j = kcol;
+        for (int tp = j + ((j + grp) & 1); tp < n; tp += 2) {
+            sr += XX[tp * XS + j];
+            if (j >= 64) sr += xtot[tp];
+        }
+    }
+    if (grp == 1) rpart[kcol] = sr;
     __syncthreads();
     if (!*abort_s && grp == 0 && t < n) {
         float *o = a.dkap_acc + blh(d, b, c0 + t, h) * K;
 #pragma unroll
         for (int m = 0; m < KMAX; ++m)
             if (m < K) o[m] = dk[m] + part[t * KMAX + m];
-        float sr = 0.f;
-        for (int tp = t; tp < n; ++tp) sr += XX[tp * XS + t];
-        a.rect[blh(d, b, c0 + t, h)] = sr;
+        a.rect[blh(d, b, c0 + t, h)] = sr + rpart[t];
     }
     __syncthreads();
     if (!*abort_s && !mbar_wait(&bars[2], 0)) *abort_s = 1;
