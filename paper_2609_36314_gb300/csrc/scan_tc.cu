@@ -366,7 +366,7 @@ __global__ void __launch_bounds__(kOutThreads, 2)
     float2 *E_s = reinterpret_cast<float2 *>(kap_s + TQ * KMAX);  // [128] hi / lo pairs
     float *tau_s = reinterpret_cast<float *>(E_s + TQ);           // [32]
     float *l2t = tau_s + 32;                                      // [32] log2(e) / tau
-    double *wsum = reinterpret_cast<double *>(l2t + 32);          // [8]
+    float2 *wsum = reinterpret_cast<float2 *>(l2t + 32);          // [8]
     // bars: 0 C, B, x loaded | 1 G done | 2 intra Y done | 3..5 S tile loaded | 6, 7 (f o C) tile consumed
     uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 8);
@@ -428,8 +428,7 @@ __global__ void __launch_bounds__(kOutThreads, 2)
         bool cl;
         e = token_rate(dtv, alv, lmv, log_cap, &cl);
     }
-    const double Et = group_scan128(double(e), wsum);
-    const float2 Et2 = split_f2(Et);
+    const float2 Et2 = group_scan128_f2(e, wsum);  // in-chunk cumulative log-decay (hi, lo)
     if (grp == 0) E_s[t] = Et2;
     float f_t[KMAX], kap_t[KMAX];
 #pragma unroll
@@ -438,7 +437,7 @@ __global__ void __launch_bounds__(kOutThreads, 2)
         if (m < K) {
             if (t < n) {
                 kap_t[m] = -expm1f(-e / tau_s[m]) * ww_t[m];
-                f_t[m] = wr_t[m] * ex2_approx(-float(Et) * l2t[m]);
+                f_t[m] = wr_t[m] * ex2_approx(-Et2.x * l2t[m]);
             }
             if (grp == 0) kap_s[t * KMAX + m] = kap_t[m];
         }

@@ -99,7 +99,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     float2 *E_s = reinterpret_cast<float2 *>(Vs + TQ * KMAX);  // hi / lo pairs
     float *l2t = reinterpret_cast<float *>(E_s + TQ);
     float *tau_s = l2t + 32;
-    double *wsum = reinterpret_cast<double *>(tau_s + 32);
+    float2 *wsum = reinterpret_cast<float2 *>(tau_s + 32);
     uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 3);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
@@ -159,8 +159,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         bool cl;
         e = token_rate(dtv, alv, lmv, log_cap, &cl);
     }
-    const double Et = group_scan128(double(e), wsum);
-    const float2 Et2 = split_f2(Et);
+    const float2 Et2 = group_scan128_f2(e, wsum);  // in-chunk cumulative log-decay (hi, lo)
     if (grp == 0) E_s[t] = Et2;
     float l2r[KMAX];  // log2(e) / tau per mode, in registers
     float kap_t[KMAX];
@@ -183,9 +182,8 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         float fv[KMAX], sv[KMAX], uv[KMAX], dv[KMAX];
 #pragma unroll
         for (int m = 0; m < KMAX; ++m) {
-            const float it = m < K ? 1.f / tau_s[m] : 0.f;
-            dv[m] = expf(-Et2.x * it);
-            uv[m] = expf(-dEnd * it);
+            dv[m] = ex2_approx(-Et2.x * l2r[m]);  // l2r = 0 beyond K
+            uv[m] = ex2_approx(-dEnd * l2r[m]);
             fv[m] = wr_t[m] * dv[m];
             sv[m] = kap_t[m] * uv[m];
         }
