@@ -145,11 +145,11 @@ def kpn(s):
 # only while the kernel's sources hash to the digest they had when they were profiled.
 PROFILED_TRAFFIC_BATCH = 2
 PROFILED_TRAFFIC = {
-    "state_pass_fwd_tc": ("scan_tc.cu", "7f83405a1de4edf3", 86.132e6 + 481.253e6),
-    "chunk_fwd_tc": ("scan_tc.cu", "7f83405a1de4edf3", 631.337e6 + 59.508e6),
-    "state_pass_rev_tc": ("scan_tc.cu", "7f83405a1de4edf3", 86.476e6 + 481.268e6),
-    "bwd_intra_tc": ("scan_tc_bwd.cu", "16553d01fd1d6858", 164.203e6 + 185.403e6),
-    "bwd_state_tc": ("scan_tc_bwd.cu", "16553d01fd1d6858", 1461.356e6 + 168.297e6),
+    "state_pass_fwd_tc": ("scan_tc.cu", "3d8105d2c52b5180", 85.136e6 + 481.196e6),
+    "chunk_fwd_tc": ("scan_tc.cu", "3d8105d2c52b5180", 631.424e6 + 59.975e6),
+    "state_pass_rev_tc": ("scan_tc.cu", "3d8105d2c52b5180", 87.261e6 + 481.387e6),
+    "bwd_intra_tc": ("scan_tc_bwd.cu", "cde6c695d8150f7c", 164.243e6 + 185.976e6),
+    "bwd_state_tc": ("scan_tc_bwd.cu", "cde6c695d8150f7c", 1462.450e6 + 173.401e6),
 }
 
 
