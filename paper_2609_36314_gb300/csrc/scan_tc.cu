@@ -57,6 +57,33 @@ struct StateSmem {
     }
 };
 
+// NL x NL transpose (NL = 4 or 8) of 16-byte pieces within each group of NL lanes: on return lane
+// NL a + i holds in e[q] the piece that lane NL a + q held in e[i].  Butterfly: at stage k every
+// piece whose index differs from the lane in bit k trades places with piece q ^ k of lane ^ k.
+__device__ __forceinline__ void shfl_xor_u4(uint4 &v, int o) {
+    v.x = __shfl_xor_sync(0xffffffffu, v.x, o);
+    v.y = __shfl_xor_sync(0xffffffffu, v.y, o);
+    v.z = __shfl_xor_sync(0xffffffffu, v.z, o);
+    v.w = __shfl_xor_sync(0xffffffffu, v.w, o);
+}
+template <int NL>
+__device__ __forceinline__ void lane_transpose(uint4 (&e)[NL], int lane) {
+#pragma unroll
+    for (int k = 1; k < NL; k <<= 1) {
+        const bool b = lane & k;
+#pragma unroll
+        for (int q0 = 0; q0 < NL; ++q0) {
+            if (q0 & k) continue;
+            uint4 s = b ? e[q0] : e[q0 | k];
+            shfl_xor_u4(s, k);
+            if (b)
+                e[q0] = s;
+            else
+                e[q0 | k] = s;
+        }
+    }
+}
+
 template <bool REV>
 __global__ void __launch_bounds__(kThreads, 2)
     tc_state_pass(const __grid_constant__ CUtensorMap mapV, StateArgs a) {
@@ -238,32 +265,41 @@ __global__ void __launch_bounds__(kThreads, 2)
         // (the TMEM load of the next 32 columns is in flight while the current ones are processed)
         {
             const int nblk = mtiles * (N / 32);
-            auto process = [&](float *v, int blk) {
+            // Blocks come in pairs (blk even, blk + 1) that cover 64 columns of one mode, so lane j
+            // then holds 128 contiguous bytes of row p0 + j; an 8 x 8 transpose of 16-byte pieces
+            // within each 8-lane group lets every store instruction write 4 full rows of 128 bytes.
+            uint4 e[8];
+            auto process = [&](float *v, int blk, int hb) {
                 const int mt = blk / (N / 32), c32 = (blk % (N / 32)) * 32;
                 const int m = mt * 4 + w;
                 const float dm = dec[m];
-                uint4 *o = reinterpret_cast<uint4 *>(a.emit + ((bh * d.nc + c) * K + m) * PN + size_t(p0 + j) * N + c32);
 #pragma unroll
                 for (int q = 0; q < 4; ++q)
-                    o[q] = make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
-                                      pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+                    e[4 * hb + q] =
+                        make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                                   pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
 #pragma unroll
                 for (int i = 0; i < 32; ++i) v[i] *= dm;
 #pragma unroll
                 for (int q = 0; q < 4; ++q) tmem_st8(lane_base + mt * N + c32 + 8 * q, v + 8 * q);
+                if (hb) {
+                    lane_transpose<8>(e, j);
+                    bf16 *o = a.emit + ((bh * d.nc + c) * K + m) * PN + size_t(p0 + (j & ~7)) * N + (c32 - 32) +
+                              8 * (j & 7);
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) *reinterpret_cast<uint4 *>(o + size_t(q) * N) = e[q];
+                }
             };
             auto col = [&](int blk) { return lane_base + (blk / (N / 32)) * N + (blk % (N / 32)) * 32; };
             float v0[32], v1[32];
             tmem_ld32(col(0), v0);
-            for (int blk = 0; blk < nblk; blk += 2) {
+            for (int blk = 0; blk < nblk; blk += 2) {  // nblk = (K / 4) (N / 32) is even
                 tmem_ld_wait();
-                if (blk + 1 < nblk) tmem_ld32(col(blk + 1), v1);
-                process(v0, blk);
-                if (blk + 1 < nblk) {
-                    tmem_ld_wait();
-                    if (blk + 2 < nblk) tmem_ld32(col(blk + 2), v0);
-                    process(v1, blk + 1);
-                }
+                tmem_ld32(col(blk + 1), v1);
+                process(v0, blk, 0);
+                tmem_ld_wait();
+                if (blk + 2 < nblk) tmem_ld32(col(blk + 2), v0);
+                process(v1, blk + 1, 1);
             }
         }
         tmem_st_wait();
