@@ -57,33 +57,6 @@ struct StateSmem {
     }
 };
 
-// NL x NL transpose (NL = 4 or 8) of 16-byte pieces within each group of NL lanes: on return lane
-// NL a + i holds in e[q] the piece that lane NL a + q held in e[i].  Butterfly: at stage k every
-// piece whose index differs from the lane in bit k trades places with piece q ^ k of lane ^ k.
-__device__ __forceinline__ void shfl_xor_u4(uint4 &v, int o) {
-    v.x = __shfl_xor_sync(0xffffffffu, v.x, o);
-    v.y = __shfl_xor_sync(0xffffffffu, v.y, o);
-    v.z = __shfl_xor_sync(0xffffffffu, v.z, o);
-    v.w = __shfl_xor_sync(0xffffffffu, v.w, o);
-}
-template <int NL>
-__device__ __forceinline__ void lane_transpose(uint4 (&e)[NL], int lane) {
-#pragma unroll
-    for (int k = 1; k < NL; k <<= 1) {
-        const bool b = lane & k;
-#pragma unroll
-        for (int q0 = 0; q0 < NL; ++q0) {
-            if (q0 & k) continue;
-            uint4 s = b ? e[q0] : e[q0 | k];
-            shfl_xor_u4(s, k);
-            if (b)
-                e[q0] = s;
-            else
-                e[q0 | k] = s;
-        }
-    }
-}
-
 template <bool REV>
 __global__ void __launch_bounds__(kThreads, 2)
     tc_state_pass(const __grid_constant__ CUtensorMap mapV, StateArgs a) {
@@ -657,27 +630,28 @@ __global__ void __launch_bounds__(kOutThreads, 2)
         *abort_s = 1;
     __syncthreads();
     tc_fence_after();
-    if (!*abort_s) {  // y = Y + D x; group g takes p in [32 g, 32 g + 32)
+    {  // y = Y + D x; group g takes p in [32 g, 32 g + 32) (rows t >= n and aborted CTAs write nothing)
         float v[32];
         tmem_ld32(lane_base + colY + grp * 32, v);
         tmem_ld_wait();
-        if (t < n) {
-            const float Dh = a.D[h];
-            const unsigned char *xrow = sX + t * 128;
-            uint4 *o = reinterpret_cast<uint4 *>(a.y + blh(d, b, c0 + t, h) * P + grp * 32);
+        const float Dh = a.D[h];
+        const unsigned char *xrow = sX + t * 128;
+        uint4 e[4];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const uint4 u = *reinterpret_cast<const uint4 *>(xrow + (((grp * 4 + q) ^ (t & 7)) * 16));
-                const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&u);
-                uint32_t r[4];
+        for (int q = 0; q < 4; ++q) {
+            const uint4 u = *reinterpret_cast<const uint4 *>(xrow + (((grp * 4 + q) ^ (t & 7)) * 16));
+            const uint32_t xw[4] = {u.x, u.y, u.z, u.w};
+            uint32_t r[4];
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const float2 f = __bfloat1622float2(h2[i]);
-                    r[i] = pack_bf16x2(fmaf(Dh, f.x, v[8 * q + 2 * i]), fmaf(Dh, f.y, v[8 * q + 2 * i + 1]));
-                }
-                o[q] = make_uint4(r[0], r[1], r[2], r[3]);
+            for (int i = 0; i < 4; ++i) {
+                const float2 f = bf16x2_to_float2(xw[i]);
+                r[i] = pack_bf16x2(fmaf(Dh, f.x, v[8 * q + 2 * i]), fmaf(Dh, f.y, v[8 * q + 2 * i + 1]));
             }
+            e[q] = make_uint4(r[0], r[1], r[2], r[3]);
         }
+        const int t4 = t & ~3;
+        put_rows<4, false>(e, reinterpret_cast<unsigned char *>(a.y + blh(d, b, c0 + t4, h) * P + grp * 32),
+                           size_t(d.H) * P * 2, *abort_s ? 0 : n - t4);
     }
     if (*abort_s && tid == 0) atomicExch(a.err, kTimeoutCode);
     tc_fence_before();

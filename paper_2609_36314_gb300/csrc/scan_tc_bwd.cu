@@ -175,7 +175,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         }
     }
     __syncthreads();
-    if (grp == 1 && t < n) {
+    if (grp == 1) {
         // the per-position mode coefficients of the state terms, for tc_bwd_state:
         // f = w_read exp(-E/tau), s = kappa u, u = exp(-(E_end - E)/tau), exp(-E/tau)
         const float dEnd = diff_f2(E_s[n - 1], Et2);
@@ -187,15 +187,26 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
             fv[m] = wr_t[m] * dv[m];
             sv[m] = kap_t[m] * uv[m];
         }
-        float4 *o = reinterpret_cast<float4 *>(a.coef + blh(d, b, c0 + t, h) * 4 * K);
+        // row t: f, s, u, exp(-E/tau), K floats each (rows t >= n are not written)
+        const size_t rs = size_t(d.H) * 4 * K * 4;
+        if (K == 8) {
+            const int t8 = t & ~7;
+            uint4 e8[8];
 #pragma unroll
-        for (int q = 0; q < KMAX / 4; ++q) {
-            if (4 * q < K) {
-                o[q] = make_float4(fv[4 * q], fv[4 * q + 1], fv[4 * q + 2], fv[4 * q + 3]);
-                o[K / 4 + q] = make_float4(sv[4 * q], sv[4 * q + 1], sv[4 * q + 2], sv[4 * q + 3]);
-                o[2 * K / 4 + q] = make_float4(uv[4 * q], uv[4 * q + 1], uv[4 * q + 2], uv[4 * q + 3]);
-                o[3 * K / 4 + q] = make_float4(dv[4 * q], dv[4 * q + 1], dv[4 * q + 2], dv[4 * q + 3]);
+            for (int q = 0; q < 2; ++q) {
+                e8[q] = f4_bits(fv[4 * q], fv[4 * q + 1], fv[4 * q + 2], fv[4 * q + 3]);
+                e8[2 + q] = f4_bits(sv[4 * q], sv[4 * q + 1], sv[4 * q + 2], sv[4 * q + 3]);
+                e8[4 + q] = f4_bits(uv[4 * q], uv[4 * q + 1], uv[4 * q + 2], uv[4 * q + 3]);
+                e8[6 + q] = f4_bits(dv[4 * q], dv[4 * q + 1], dv[4 * q + 2], dv[4 * q + 3]);
             }
+            put_rows<8, false>(e8, reinterpret_cast<unsigned char *>(a.coef + blh(d, b, c0 + t8, h) * 4 * K), rs,
+                               n - t8);
+        } else {  // K == 4
+            const int t4 = t & ~3;
+            uint4 e4[4] = {f4_bits(fv[0], fv[1], fv[2], fv[3]), f4_bits(sv[0], sv[1], sv[2], sv[3]),
+                           f4_bits(uv[0], uv[1], uv[2], uv[3]), f4_bits(dv[0], dv[1], dv[2], dv[3])};
+            put_rows<4, false>(e4, reinterpret_cast<unsigned char *>(a.coef + blh(d, b, c0 + t4, h) * 4 * K), rs,
+                               n - t4);
         }
     }
     // ---- Gamma below the diagonal 32 x 32 blocks, factored through the log-decay E_a at the end
@@ -497,15 +508,16 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     if (!*abort_s && !mbar_wait(&bars[2], 0)) *abort_s = 1;
     __syncthreads();
     tc_fence_after();
-    if (!*abort_s) {  // dx_intra row: group g takes columns [32 g, 32 g + 32)
+    {  // dx_intra row: group g takes columns [32 g, 32 g + 32) (nothing written after an abort)
         float v[32];
         tmem_ld32(lane_base + colX + grp * 32, v);
         tmem_ld_wait();
-        if (t < n) {
-            float4 *o = reinterpret_cast<float4 *>(a.dx_acc + blh(d, b, c0 + t, h) * P + grp * 32);
+        uint4 e[8];
 #pragma unroll
-            for (int q = 0; q < 8; ++q) o[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-        }
+        for (int q = 0; q < 8; ++q) e[q] = f4_bits(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        const int t8 = t & ~7;
+        put_rows<8, false>(e, reinterpret_cast<unsigned char *>(a.dx_acc + blh(d, b, c0 + t8, h) * P + grp * 32),
+                           size_t(d.H) * P * 4, *abort_s ? 0 : n - t8);
     }
     if (*abort_s && tid == 0) atomicExch(a.err, kTimeoutCode);
     tc_fence_before();
@@ -717,18 +729,23 @@ __global__ void __launch_bounds__(kStThreads + 32, 1)
             }
             ab_h = fmaf(aj * dotv, itau_s[(j / K) * K + mj], ab_h);  // group 0: a; group 1: b
         }
-        if (mj == K - 1 && !*abort_s && t < n) {  // head hj complete: reductions, nothing waits
-            const size_t i0 = blh(d, b, c0 + t, hj);
-            float4 *acc_dst = reinterpret_cast<float4 *>((grp == 0 ? a.dwr_acc : a.dkap_acc) + i0 * K);
+        if (mj == K - 1) {  // head hj complete: reductions, nothing waits
+            if (!*abort_s && t < n) {
+                const size_t i0 = blh(d, b, c0 + t, hj);
+                float4 *acc_dst = reinterpret_cast<float4 *>((grp == 0 ? a.dwr_acc : a.dkap_acc) + i0 * K);
 #pragma unroll
-            for (int q = 0; q < KMAX / 4; ++q)
-                if (4 * q < K)
-                    atomicAdd(acc_dst + q, make_float4(acc_h[4 * q], acc_h[4 * q + 1], acc_h[4 * q + 2], acc_h[4 * q + 3]));
-            a.ab_acc[i0 * 2 + grp] = ab_h;
-            float4 *o = reinterpret_cast<float4 *>(a.dx_acc + i0 * P + 32 * grp);
+                for (int q = 0; q < KMAX / 4; ++q)
+                    if (4 * q < K)
+                        atomicAdd(acc_dst + q,
+                                  make_float4(acc_h[4 * q], acc_h[4 * q + 1], acc_h[4 * q + 2], acc_h[4 * q + 3]));
+                a.ab_acc[i0 * 2 + grp] = ab_h;
+            }
+            uint4 e[8];
 #pragma unroll
-            for (int q = 0; q < 8; ++q)
-                atomicAdd(o + q, make_float4(dxr[4 * q], dxr[4 * q + 1], dxr[4 * q + 2], dxr[4 * q + 3]));
+            for (int q = 0; q < 8; ++q) e[q] = f4_bits(dxr[4 * q], dxr[4 * q + 1], dxr[4 * q + 2], dxr[4 * q + 3]);
+            const int t8 = t & ~7;
+            put_rows<8, true>(e, reinterpret_cast<unsigned char *>(a.dx_acc + blh(d, b, c0 + t8, hj) * P + 32 * grp),
+                              size_t(d.H) * P * 4, *abort_s ? 0 : n - t8);
         }
     };
 
@@ -846,22 +863,23 @@ __global__ void __launch_bounds__(kStThreads + 32, 1)
     if (nsteps > 0 && tid < kStThreads) readout(nsteps - 1);
     // the group's dC / dB into the float32 accumulators (group g takes n in [64 g, 64 g + 64))
     tc_fence_after();
-    if (!*abort_s && tid < kStThreads && grp < N / 64) {
-        const size_t gi = ((size_t(b) * d.L + c0 + min(t, n - 1)) * d.G + g) * N + grp * 64;
+    if (tid < kStThreads && grp < N / 64) {
+        const int t8 = t & ~7;
+        const int nv = *abort_s ? 0 : n - t8;
+        const size_t gi = ((size_t(b) * d.L + c0 + t8) * d.G + g) * N + grp * 64;
+        const size_t rs = size_t(d.G) * N * 4;
         for (int n32 = 0; n32 < 64; n32 += 32) {
             float vc[32], vb[32];
             tmem_ld32(lane_base + colC + grp * 64 + n32, vc);
             tmem_ld32(lane_base + colB + grp * 64 + n32, vb);
             tmem_ld_wait();
-            if (t < n) {
+            uint4 e[8];
 #pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    atomicAdd(reinterpret_cast<float4 *>(a.dC_acc + gi + n32 + 4 * k),
-                              make_float4(vc[4 * k], vc[4 * k + 1], vc[4 * k + 2], vc[4 * k + 3]));
-                    atomicAdd(reinterpret_cast<float4 *>(a.dB_acc + gi + n32 + 4 * k),
-                              make_float4(vb[4 * k], vb[4 * k + 1], vb[4 * k + 2], vb[4 * k + 3]));
-                }
-            }
+            for (int k = 0; k < 8; ++k) e[k] = f4_bits(vc[4 * k], vc[4 * k + 1], vc[4 * k + 2], vc[4 * k + 3]);
+            put_rows<8, true>(e, reinterpret_cast<unsigned char *>(a.dC_acc + gi + n32), rs, nv);
+#pragma unroll
+            for (int k = 0; k < 8; ++k) e[k] = f4_bits(vb[4 * k], vb[4 * k + 1], vb[4 * k + 2], vb[4 * k + 3]);
+            put_rows<8, true>(e, reinterpret_cast<unsigned char *>(a.dB_acc + gi + n32), rs, nv);
         }
     }
     if (*abort_s && tid == 0) atomicExch(a.err, kTimeoutCode);

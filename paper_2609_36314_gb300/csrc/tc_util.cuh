@@ -54,6 +54,59 @@ __device__ __forceinline__ void load_weights(const __nv_bfloat16 *src, int K, fl
     }
 }
 
+// NL x NL transpose (NL = 4 or 8) of 16-byte pieces within each group of NL lanes: on return lane
+// NL a + i holds in e[q] the piece that lane NL a + q held in e[i].  Butterfly: at stage k every
+// piece whose index differs from the lane in bit k trades places with piece q ^ k of lane ^ k.
+__device__ __forceinline__ void shfl_xor_u4(uint4 &v, int o) {
+    v.x = __shfl_xor_sync(0xffffffffu, v.x, o);
+    v.y = __shfl_xor_sync(0xffffffffu, v.y, o);
+    v.z = __shfl_xor_sync(0xffffffffu, v.z, o);
+    v.w = __shfl_xor_sync(0xffffffffu, v.w, o);
+}
+template <int NL>
+__device__ __forceinline__ void lane_transpose(uint4 (&e)[NL], int lane) {
+#pragma unroll
+    for (int k = 1; k < NL; k <<= 1) {
+        const bool b = lane & k;
+#pragma unroll
+        for (int q0 = 0; q0 < NL; ++q0) {
+            if (q0 & k) continue;
+            uint4 s = b ? e[q0] : e[q0 | k];
+            shfl_xor_u4(s, k);
+            if (b)
+                e[q0] = s;
+            else
+                e[q0 | k] = s;
+        }
+    }
+}
+
+__device__ __forceinline__ uint4 f4_bits(float a, float b, float c, float d) {
+    return make_uint4(__float_as_uint(a), __float_as_uint(b), __float_as_uint(c), __float_as_uint(d));
+}
+
+// Every lane holds NL 16-byte pieces of its own row (lane l: row l of its NL-lane group, the
+// rows `stride` bytes apart from row0 = the group's first row).  After lane_transpose each
+// instruction writes 32 / NL whole row segments of 16 NL contiguous bytes instead of 32
+// scattered pieces; rows >= nvalid of the group are skipped.  ADD: float4 atomic add (the
+// pieces are float4), else a plain 16-byte store.  Every lane of the warp must call it.
+template <int NL, bool ADD>
+__device__ __forceinline__ void put_rows(uint4 (&e)[NL], unsigned char *row0, size_t stride, int nvalid) {
+    const int lane = threadIdx.x & 31, i = lane & (NL - 1);
+    lane_transpose<NL>(e, lane);
+#pragma unroll
+    for (int q = 0; q < NL; ++q) {
+        if (q < nvalid) {
+            unsigned char *p = row0 + size_t(q) * stride + 16 * i;
+            if (ADD)
+                atomicAdd(reinterpret_cast<float4 *>(p), make_float4(__uint_as_float(e[q].x), __uint_as_float(e[q].y),
+                                                                     __uint_as_float(e[q].z), __uint_as_float(e[q].w)));
+            else
+                *reinterpret_cast<uint4 *>(p) = e[q];
+        }
+    }
+}
+
 // Inclusive prefix sum (double) of one value per thread over a 128-thread block.
 __device__ __forceinline__ double block_scan128(double v, double *wsum) {
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
