@@ -129,11 +129,13 @@ __global__ void __launch_bounds__(kThreads, 2)
         const int c_ = REV ? d.nc - 1 - ci_ : ci_;
         const int c0_ = c_ * TQ, n_ = min(TQ, d.L - c0_);
         const int t = tid;
+        {  // this position's 32 x values (64 bytes), read row-coalesced across each 4-lane group
+            const int t4 = t & ~3;
+            get_rows<4>(nx, reinterpret_cast<const unsigned char *>(a.U + blh(d, b, c0_ + t4, h) * P + p0),
+                        size_t(d.H) * P * 2, n_ - t4);
+        }
         if (t < n_) {
             const size_t i = blh(d, b, c0_ + t, h);
-            const uint4 *src = reinterpret_cast<const uint4 *>(a.U + i * P + p0);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) nx[q] = src[q];
             ndt = a.dt[i];
             nal = a.alpha[i];
             nlm = a.lam[i];
@@ -151,8 +153,6 @@ __global__ void __launch_bounds__(kThreads, 2)
                 for (int m = 0; m < KMAX; ++m) nw[m] = m < K ? to_f(a.W[i * K + m]) : 0.f;
             }
         } else {
-#pragma unroll
-            for (int q = 0; q < 4; ++q) nx[q] = make_uint4(0, 0, 0, 0);
 #pragma unroll
             for (int m = 0; m < KMAX; ++m) nw[m] = 0.f;
         }

@@ -639,13 +639,22 @@ __global__ void __launch_bounds__(kStThreads + 32, 1)
 
     // head-summed intra term: dC = M_H B, dB = M_H^T C (M_H as bf16 [t][k] in generator buffer 0)
     if (intra) {
-        const float *mrow = a.mh_total + (((size_t(b) * d.nc + c) * d.G + g) * TQ + t) * TQ + grp * 64;
+        if (tid < kStThreads) {  // row t, k in [64 grp, 64 grp + 64), read row-coalesced in two halves
+            const float *mrow8 = a.mh_total + (((size_t(b) * d.nc + c) * d.G + g) * TQ + (t & ~7)) * TQ + grp * 64;
 #pragma unroll
-        for (int k8 = 0; k8 < 64 && tid < kStThreads; k8 += 8) {
-            const float4 u0 = *reinterpret_cast<const float4 *>(mrow + k8);
-            const float4 u1 = *reinterpret_cast<const float4 *>(mrow + k8 + 4);
-            const float v[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
-            store_bf16x8(sG + grp * 16384 + t * 128 + (((k8 >> 3) ^ (t & 7)) * 16), v);
+            for (int hf = 0; hf < 2; ++hf) {
+                uint4 e[8];
+                get_rows<8>(e, reinterpret_cast<const unsigned char *>(mrow8 + 32 * hf), TQ * 4, 8);
+#pragma unroll
+                for (int k8 = 0; k8 < 4; ++k8) {
+                    const uint4 u0 = e[2 * k8], u1 = e[2 * k8 + 1];
+                    const float v[8] = {__uint_as_float(u0.x), __uint_as_float(u0.y), __uint_as_float(u0.z),
+                                        __uint_as_float(u0.w), __uint_as_float(u1.x), __uint_as_float(u1.y),
+                                        __uint_as_float(u1.z), __uint_as_float(u1.w)};
+                    const int kb = 4 * hf + k8;  // 8-column block within the group's 64
+                    store_bf16x8(sG + grp * 16384 + t * 128 + ((kb ^ (t & 7)) * 16), v);
+                }
+            }
         }
         fence_async_smem();
         __syncthreads();
@@ -802,26 +811,44 @@ __global__ void __launch_bounds__(kStThreads + 32, 1)
             }
 #pragma unroll
             for (int k = 0; k < KMAX; ++k) acc_h[k] = 0.f;
+            // coefficients of this row from tc_bwd_intra (group 0: f, exp(-E/tau); group 1: s, u;
+            // both: s) and its row of dY / X, read row-coalesced across each 8-lane group
+            const int t8 = t & ~7;
+            const size_t r8 = blh(d, b, c0 + t8, h);
             float4 c4[6];
+            {
+                auto f4 = [](uint4 v) {
+                    return make_float4(__uint_as_float(v.x), __uint_as_float(v.y), __uint_as_float(v.z),
+                                       __uint_as_float(v.w));
+                };
+                if (K == 8) {  // pieces: f 0-1, s 2-3, u 4-5, exp(-E/tau) 6-7
+                    uint4 cr[8];
+                    get_rows<8>(cr, reinterpret_cast<const unsigned char *>(a.coef + r8 * 32), size_t(d.H) * 128,
+                                n - t8);
 #pragma unroll
-            for (int k = 0; k < 6; ++k) c4[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (t < n) {  // coefficients of this row from tc_bwd_intra; group 0: f, exp(-E/tau); 1: s, u
-                const size_t i0 = blh(d, b, c0 + t, h);
-                const float4 *cf = reinterpret_cast<const float4 *>(a.coef + i0 * 4 * K);
-#pragma unroll
-                for (int q = 0; q < KMAX / 4; ++q) {
-                    if (4 * q < K) {
-                        c4[q] = cf[(grp == 0 ? 0 : 1) * (K / 4) + q];
-                        c4[2 + q] = cf[(grp == 0 ? 3 : 2) * (K / 4) + q];
-                        c4[4 + q] = cf[K / 4 + q];
+                    for (int q = 0; q < 2; ++q) {
+                        c4[q] = f4(grp == 0 ? cr[q] : cr[2 + q]);
+                        c4[2 + q] = f4(grp == 0 ? cr[6 + q] : cr[4 + q]);
+                        c4[4 + q] = f4(cr[2 + q]);
                     }
+                } else {  // K == 4, 64-byte rows in 4-lane groups; pieces: f, s, u, exp(-E/tau)
+                    const int t4 = t & ~3;
+                    uint4 cr[4];
+                    get_rows<4>(cr, reinterpret_cast<const unsigned char *>(a.coef + blh(d, b, c0 + t4, h) * 16),
+                                size_t(d.H) * 64, n - t4);
+                    const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+                    c4[0] = f4(grp == 0 ? cr[0] : cr[1]);
+                    c4[2] = f4(grp == 0 ? cr[3] : cr[2]);
+                    c4[4] = f4(cr[1]);
+                    c4[1] = c4[3] = c4[5] = z;
                 }
-                const uint4 *src = reinterpret_cast<const uint4 *>((grp == 0 ? a.dy : a.x) + i0 * P);
+            }
+            {
+                uint4 rr[8];
+                get_rows<8>(rr, reinterpret_cast<const unsigned char *>((grp == 0 ? a.dy : a.x) + r8 * P),
+                            size_t(d.H) * P * 2, n - t8);
 #pragma unroll
-                for (int k = 0; k < 8; ++k) row[k] = src[k];
-            } else {
-#pragma unroll
-                for (int k = 0; k < 8; ++k) row[k] = make_uint4(0, 0, 0, 0);
+                for (int k = 0; k < 8; ++k) row[k] = rr[k];
             }
 #pragma unroll
             for (int k = 0; k < 6; ++k) {  // this thread's row: scalar stores (the row stride is odd)
