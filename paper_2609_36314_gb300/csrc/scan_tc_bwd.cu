@@ -526,18 +526,20 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
 }
 
 // ============================================================================= state terms
-// One CTA per (b, c, group of hg heads of one B/C group), 256 threads, software-pipelined over
-// the (head, mode) steps.  Step i, with the mode's S_in and dS_out tiles [p][n] streamed in by
-// TMA (three buffers):
+// One CTA per (b, c, group of hg heads of one B/C group), 256 compute threads plus an issuing warp
+// and three dot-product warps, software-pipelined over the (head, mode) steps.  Step i, with the
+// mode's S_in and dS_out tiles [p][n] streamed in by TMA (two buffers):
 //   Z_m = C S_in,m^T,  U_m = B dS_out,m^T                  (TMEM, two buffers of 2 x 64 columns)
 //   dC += (f_m o dY) S_in,m,  dB += (s_m o X) dS_out,m       (TMEM, summed over modes and heads)
 // While the tensor cores run step i, the threads read out step i - 1: group 0 contracts Z_m with
 // its dY row (dw_read, the a term), group 1 contracts U_m with its X row (dkappa, the b term) and
-// accumulates dx = sum_m s_m U_m in registers.  <dS_out,m, S_in,m> comes from the two tiles in
-// shared memory.  The head-summed intra tile Gamma o H adds M_H B to dC and M_H^T C to dB once
+// accumulates dx = sum_m s_m U_m in registers.  Three more warps form <dS_out,m, S_in,m> from the
+// two tiles in shared memory.  The head-summed intra tile Gamma o H adds M_H B to dC and M_H^T C to dB once
 // per (b, c, B/C group).
 constexpr int kStThreads = 256;  // compute threads (two warpgroups); a ninth warp issues the MMAs
                                  // and TMA loads (one thread)
+constexpr int kCdThreads = 96;   // three more warps form <dS_out,m, S_in,m> from each step's tiles
+constexpr int kStLaunch = kStThreads + 32 + kCdThreads;
 constexpr int kStBuf = 2;   // S_in / dS_out tile buffers
 constexpr int kCoefStride = 3 * KMAX + 1;  // per-thread coefficient row (odd: no bank conflicts)
 
@@ -572,7 +574,7 @@ __device__ __forceinline__ uint4 scale_bf16x8(uint4 a, float s) {
     return make_uint4(r[0], r[1], r[2], r[3]);
 }
 
-__global__ void __launch_bounds__(kStThreads + 32, 1)
+__global__ void __launch_bounds__(kStLaunch, 1)
     tc_bwd_state(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapB,
                  const __grid_constant__ CUtensorMap mapS, const __grid_constant__ CUtensorMap mapD,
                  BwdArgs a) {
@@ -589,9 +591,10 @@ __global__ void __launch_bounds__(kStThreads + 32, 1)
     double *wsum = reinterpret_cast<double *>(itau_s + 32);     // [8]
     double *Eend_s = wsum + 8;                                  // [1]
     // bars: 0..2 tile buffers | 3, 4 MMA of step parity | 5 C, B | 6 intra MMA |
-    //       7, 8 generated operands of step parity written (all 256 threads arrive)
+    //       7, 8 generated operands of step parity written (all 256 threads arrive) |
+    //       9, 10 tile buffer read by the <dS_out, S_in> warps (all 96 threads arrive)
     uint64_t *bars = reinterpret_cast<uint64_t *>(Eend_s + 2);
-    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 9);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 11);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
 
     const int tid = threadIdx.x, grp = tid >> 7, t = tid & 127, w = tid >> 5, w4 = w & 3;
@@ -607,6 +610,8 @@ __global__ void __launch_bounds__(kStThreads + 32, 1)
         for (int i = 0; i < 7; ++i) mbar_init(&bars[i], 1);
         mbar_init(&bars[7], kStThreads);
         mbar_init(&bars[8], kStThreads);
+        mbar_init(&bars[9], kCdThreads);
+        mbar_init(&bars[10], kCdThreads);
         *abort_s = 0;
         fence_barrier_init();
     }
@@ -766,7 +771,9 @@ __global__ void __launch_bounds__(kStThreads + 32, 1)
             // step i - 1's MMAs are done (they were issued at the tensor cores' pace): its tile
             // buffer takes the tiles of step i - 1 + kStBuf before step i's operands are awaited
             if (i >= 1) {
-                if (!mbar_wait(&bars[3 + ((i - 1) & 1)], ((i - 1) >> 1) & 1)) {
+                const int qp = (i - 1) % kStBuf;
+                if (!mbar_wait(&bars[3 + ((i - 1) & 1)], ((i - 1) >> 1) & 1) ||
+                    !mbar_wait(&bars[9 + qp], ((i - 1) / kStBuf) & 1)) {
                     *abort_s = 1;
                     break;
                 }
@@ -799,8 +806,33 @@ __global__ void __launch_bounds__(kStThreads + 32, 1)
             mma_commit(&bars[3 + gb]);
         }
     }
+    if (tid >= kStThreads + 32) {
+        // <dS_out,m, S_in,m> of every step from its two tiles (the same swizzle in both), then the
+        // tile buffer is released to the issuer
+        const int ct = tid - (kStThreads + 32);
+        for (int i = 0; i < nsteps; ++i) {
+            const int q = i % kStBuf;
+            if (*abort_s || !mbar_wait(&bars[q], (i / kStBuf) & 1)) {
+                *abort_s = 1;
+                break;
+            }
+            const uint4 *ps = reinterpret_cast<const uint4 *>(sT + (2 * q) * L.tile);
+            const uint4 *pd = reinterpret_cast<const uint4 *>(sT + (2 * q + 1) * L.tile);
+            float acc0 = 0.f, acc1 = 0.f;
+            int k = ct;
+            for (; k + kCdThreads < L.tile / 16; k += 2 * kCdThreads) {
+                acc0 = dot_bf16x8(ps[k], pd[k], acc0);
+                acc1 = dot_bf16x8(ps[k + kCdThreads], pd[k + kCdThreads], acc1);
+            }
+            if (k < L.tile / 16) acc0 = dot_bf16x8(ps[k], pd[k], acc0);
+            mbar_arrive(&bars[9 + q]);
+            const float v = warp_sum(acc0 + acc1);
+            if ((tid & 31) == 0)
+                atomicAdd(a.cdot + ((size_t(b) * d.H + h_first + i / K) * d.nc + c) * K + i % K, v);
+        }
+    }
     for (int i = 0; i < nsteps && tid < kStThreads; ++i) {
-        const int hh = i / K, m = i % K, h = h_first + hh, gb = i & 1, q = i % kStBuf;
+        const int hh = i / K, m = i % K, h = h_first + hh, gb = i & 1;
         bool prev_done = i == 0;
         if (m == 0) {
             // a new head: step i - 1 (the previous head's last) is read out with that head's
@@ -866,19 +898,6 @@ __global__ void __launch_bounds__(kStThreads + 32, 1)
 #pragma unroll
             for (int k = 0; k < 8; ++k)
                 *reinterpret_cast<uint4 *>(dst + ((k ^ (t & 7)) * 16)) = scale_bf16x8(row[k], sc);
-        }
-        // this step's tiles: <dS_out,m, S_in,m> partials (the same swizzle in both tiles)
-        if (!*abort_s && !mbar_wait(&bars[q], (i / kStBuf) & 1)) *abort_s = 1;
-        {
-            const uint4 *ps = reinterpret_cast<const uint4 *>(sT + (2 * q) * L.tile);
-            const uint4 *pd = reinterpret_cast<const uint4 *>(sT + (2 * q + 1) * L.tile);
-            float acc0 = 0.f, acc1 = 0.f;  // L.tile / 16 is a multiple of 2 * kStThreads
-            for (int k = tid; k < L.tile / 16; k += 2 * kStThreads) {
-                acc0 = dot_bf16x8(ps[k], pd[k], acc0);
-                acc1 = dot_bf16x8(ps[k + kStThreads], pd[k + kStThreads], acc1);
-            }
-            const float v = warp_sum(acc0 + acc1);
-            if ((tid & 31) == 0) atomicAdd(a.cdot + ((size_t(b) * d.H + h) * d.nc + c) * K + m, v);
         }
         // hand the generated operands to the MMA issuer (no CTA-wide barrier in the loop)
         fence_async_smem();
@@ -1147,7 +1166,7 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
         const size_t smem = StSmem(d.N).total + 1024;
         cudaFuncSetAttribute(tc_bwd_state, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
         trace_begin("bwd_state_tc", st);
-        tc_bwd_state<<<dim3(d.H / a.hg, d.nc, d.B), kStThreads + 32, smem, st>>>(mapC, mapB, mapS, mapD, a);
+        tc_bwd_state<<<dim3(d.H / a.hg, d.nc, d.B), kStLaunch, smem, st>>>(mapC, mapB, mapS, mapD, a);
         trace_end(st);
         if ((e = cudaGetLastError())) return e;
     }
