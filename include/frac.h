@@ -68,9 +68,9 @@ typedef enum { FRAC_DTYPE_F32 = 0, FRAC_DTYPE_BF16 = 1 } frac_dtype;
 /* Bits of frac_dims.flags. */
 enum {
     /* Use the CUDA-core chunked kernels even where tensor-core ones exist.  Without it, bf16
-       calls with headdim 32 or 64, dstate in {64, 128} and nmodes in {4, 8} run the forward on
-       the tensor cores (TMA-fed tcgen05 MMAs, chunk 128), and with headdim 64 the backward too;
-       they need the dtype tensors and the states 16-byte aligned. */
+       calls with headdim 64, dstate in {64, 128} and nmodes in {4, 8} run the forward and the
+       backward on the tensor cores (TMA-fed tcgen05 MMAs, chunk 128); they need the dtype
+       tensors and the states 16-byte aligned. */
     FRAC_FLAG_FORCE_SIMT = 1,
     /* frac_scan_bwd only: the workspace already holds the per-chunk states that a frac_scan_fwd
        call with the same inputs, h0 and dims left in this same workspace (give both calls one
@@ -97,7 +97,8 @@ typedef struct {
 
 /*
  * Bytes of scratch device memory frac_scan_fwd needs for these dims (per-chunk mode states
- * handed from the chunk-serial state pass to the chunk-parallel output kernel).
+ * handed from the chunk-serial state pass to the chunk-parallel output kernel; on the
+ * tensor-core path also the per-position mode coefficients).
  */
 frac_status frac_scan_fwd_workspace_size(const frac_dims *dims, size_t *bytes);
 

@@ -107,7 +107,7 @@ frac_status plan(const frac_dims *d, frac::ScanDims *sd, int *path, bool backwar
 constexpr size_t kStatusBytes = kAlign;
 
 struct FwdLayout {
-    size_t s_in, total;
+    size_t s_in, coef, total;
 };
 struct BwdLayout {
     size_t s_in, ds_out, db, dc, total;
@@ -118,7 +118,8 @@ FwdLayout fwd_layout(const frac_dims *d, const frac::ScanDims &sd, int path) {
     l.s_in = kStatusBytes;
     const size_t elems = path == PATH_TC ? frac::tc_state_elems(sd) : frac::simt_state_elems(sd);
     const size_t esz = path == PATH_TC ? 2 : elem(d);
-    l.total = kStatusBytes + round_up(elems * esz);
+    l.coef = kStatusBytes + round_up(elems * esz);  // tensor-core path: per-position coefficients
+    l.total = l.coef + (path == PATH_TC ? round_up(frac::tc_coef_elems(sd) * 4) : 0);
     return l;
 }
 
@@ -253,7 +254,8 @@ frac_status frac_scan_fwd(const frac_dims *d, const void *x, const float *dt, co
     cudaError_t e = cudaMemsetAsync(ws, 0, sizeof(int), st);
     if (e == cudaSuccess) {
         if (path == PATH_TC)
-            e = frac::tc_scan_fwd(sd, p, ws + l.s_in, reinterpret_cast<int *>(ws), st);
+            e = frac::tc_scan_fwd(sd, p, ws + l.s_in, reinterpret_cast<float *>(ws + l.coef),
+                                  reinterpret_cast<int *>(ws), st);
         else
             e = frac::simt_scan_fwd(sd, d->dtype, p, ws + l.s_in, st);
     }

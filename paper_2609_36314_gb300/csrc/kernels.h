@@ -53,20 +53,23 @@ cudaError_t simt_scan_bwd(const ScanDims &d, int dtype, const ScanPtrs &p, void 
 // Tensor-core (tcgen05) path: bf16 inputs, chunk 128, P = 64, N in {64, 128}, K in {4, 8}.
 bool tc_supported(const ScanDims &d, int dtype);
 size_t tc_state_elems(const ScanDims &d);  // bf16 elements of the per-chunk state workspace
-cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, int *err,
+size_t tc_coef_elems(const ScanDims &d);   // float elements of the per-position coefficients
+// coef: [B, L, H, 4, K] float (f, s, u, exp(-E/tau) per position), written by the forward
+cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, float *coef, int *err,
                         cudaStream_t st);
-// Chunk-serial state pass on the tensor cores (forward: U = x, V = B, W = w_write; reverse:
-// U = dy, V = C, W = w_read).
+// Per-position mode coefficients of every chunk (the first kernel of both passes).
+cudaError_t tc_coef_launch(const ScanDims &d, const ScanPtrs &p, float *coef, cudaStream_t st);
+// Chunk-serial state pass on the tensor cores (forward: U = x, V = B, coefficients s; reverse:
+// U = dy, V = C, coefficients f).
 cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, const void *V,
-                                 const void *W, const float *dt, const float *alpha,
-                                 const float *lam, const float *tau, const float *init,
-                                 void *emit, float *fin, int *err, cudaStream_t st);
+                                 const float *coef, const float *init, void *emit, float *fin,
+                                 int *err, cudaStream_t st);
 bool tc_make_map3(CUtensorMap *m, const void *ptr, uint64_t d0, uint64_t d1, uint64_t d2,
                   uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1,
                   uint32_t b2);
 // Tensor-core backward (headdim 64 in addition to the forward's conditions).
 bool tc_bwd_supported(const ScanDims &d, int dtype);
-struct TcBwdWorkspace {
+struct TcBwdWorkspace {  // S_in and coef first, at the offsets the forward uses
     void *S_in, *dS_out;                     // bf16 per-chunk states
     float *dx_acc, *dwr_acc, *dkap_acc;      // [B,L,H,P], [B,L,H,K] x 2
     float *ab_acc, *rect, *cdot, *mh_total;  // [B,L,H,2], [B,L,H], [B,H,nc,K], [B,nc,G,Q,Q]

@@ -3,10 +3,13 @@
 // Same chunked evaluation order as the CUDA-core kernels (App. E of the paper), with chunk
 // Q = 128 and the two state contractions of every chunk on the tensor cores:
 //
-//   tc_state_pass  (chunk-serial; one CTA per (b, h, 32-wide slice of P)):
-//        the P-slice of every mode's state lives in tensor memory as fp32, lanes = (mode%4, p),
-//        columns = (mode/4, n).  Per chunk: emit the entering state (bf16) for the output
-//        kernel, scale it by d_m = exp(-E_end/tau_m) in place, then accumulate
+//   tc_coef        (one CTA per (b, h, chunk)): the per-position mode coefficients of the
+//        chunk (f, s = kappa u, u, exp(-E/tau) from the float-pair cumulative log-decay E), read
+//        by the state passes and the backward instead of being recomputed per P-slice.
+//   tc_state_pass  (chunk-serial; one CTA per (b, h, 128/K-wide slice of P), three per SM):
+//        the P-slice of every mode's state lives in tensor memory as fp32, lanes = (mode, p),
+//        columns = n.  Per chunk: emit the entering state (bf16) for the output kernel, scale
+//        it by d_m = exp(-E_end/tau_m) in place, then accumulate
 //        S_m += sum_k s_{k,m} x_k B_k^T  as  D[(m,p), n] += A[(m,p), k] * B[k, n]
 //        (A = s o x generated in shared memory, B = the chunk of B loaded by TMA).
 //        Run over the chunks in reverse with (dy, C, f) it carries dS for the backward.
@@ -37,54 +40,121 @@ constexpr int kThreads = 128;
 
 struct StateArgs {
     ScanDims d;
-    const bf16 *U;    // x or dy      [B, L, H, P]
-    const bf16 *W;    // w_write or w_read [B, L, H, K]
-    const float *dt, *alpha, *lam, *tau;
+    const bf16 *U;      // x or dy      [B, L, H, P]
+    const float *coef;  // per-position mode coefficients [B, L, H, 4, K] (tc_coef)
     const float *init;  // h0 or dh_final [B, H, K, P, N] or null
     bf16 *emit;         // per-chunk entering states [B, H, nc, K, P, N]
     float *fin;         // h_final or dh0, or null
     int *err;
 };
 
-// Shared-memory plan of tc_state_pass (offsets from a 1024-aligned base).
+// ---------------------------------------------------------------------------------------------
+// Per-position mode coefficients of every chunk, computed once for all kernels that need them:
+// with E_t the in-chunk cumulative log-decay (float-pair scan of the token rates, Sec. 3.2) and
+// kappa = (1 - exp(-e_t/tau)) w_write,
+//   f = w_read exp(-E_t/tau)   s = kappa u   u = exp(-(E_end - E_t)/tau)   d = exp(-E_t/tau)
+// stored as coef[b, t, h, {f, s, u, d}, K].  d at the chunk's last position is the chunk decay.
+struct CoefArgs {
+    ScanDims d;
+    const bf16 *wr, *ww;
+    const float *dt, *alpha, *lam, *tau;
+    float *coef;
+};
+
+template <int KK>
+__global__ void __launch_bounds__(TQ) tc_coef(CoefArgs a) {
+    __shared__ float2 wsum[4];
+    __shared__ float2 Eend_s;
+    const ScanDims &d = a.d;
+    const int t = threadIdx.x, h = blockIdx.x, c = blockIdx.y, b = blockIdx.z;
+    const int c0 = c * TQ, n = min(TQ, d.L - c0);
+    float itau[KK], l2t[KK], tmax = 0.f;
+#pragma unroll
+    for (int m = 0; m < KK; ++m) {
+        const float tv = a.tau[h * KK + m];
+        itau[m] = 1.f / tv;
+        l2t[m] = kLog2e / tv;
+        tmax = fmaxf(tmax, tv);
+    }
+    float e = 0.f, wr[KMAX], ww[KMAX];
+#pragma unroll
+    for (int m = 0; m < KMAX; ++m) wr[m] = ww[m] = 0.f;
+    if (t < n) {
+        const size_t i = blh(d, b, c0 + t, h);
+        bool cl;
+        e = token_rate(a.dt[i], a.alpha[i], a.lam[i], logf(64.f * tmax), &cl);
+        load_weights(a.wr + i * KK, KK, wr);
+        load_weights(a.ww + i * KK, KK, ww);
+    }
+    const float2 Et = group_scan128_f2(e, wsum);
+    if (t == n - 1) Eend_s = Et;
+    __syncthreads();
+    const float dEnd = diff_f2(Eend_s, Et);  // E_end - E_t >= 0
+    float f[KK], s[KK], u[KK], dv[KK];
+#pragma unroll
+    for (int m = 0; m < KK; ++m) {
+        dv[m] = ex2_approx(-Et.x * l2t[m]);
+        u[m] = ex2_approx(-dEnd * l2t[m]);
+        f[m] = wr[m] * dv[m];
+        s[m] = -expm1f(-e * itau[m]) * ww[m] * u[m];
+    }
+    // row t: KK / 4 pieces of each kind, written row-coalesced across KK-lane groups
+    uint4 pc[KK];
+#pragma unroll
+    for (int q = 0; q < KK / 4; ++q) {
+        pc[q] = f4_bits(f[4 * q], f[4 * q + 1], f[4 * q + 2], f[4 * q + 3]);
+        pc[KK / 4 + q] = f4_bits(s[4 * q], s[4 * q + 1], s[4 * q + 2], s[4 * q + 3]);
+        pc[KK / 2 + q] = f4_bits(u[4 * q], u[4 * q + 1], u[4 * q + 2], u[4 * q + 3]);
+        pc[3 * KK / 4 + q] = f4_bits(dv[4 * q], dv[4 * q + 1], dv[4 * q + 2], dv[4 * q + 3]);
+    }
+    const int tg = t & ~(KK - 1);
+    put_rows<KK, false>(pc, reinterpret_cast<unsigned char *>(a.coef + blh(d, b, c0 + tg, h) * 4 * KK),
+                        size_t(d.H) * 4 * KK * 4, n - tg);
+}
+
+// Shared-memory plan of tc_state_pass (offsets from a 1024-aligned base): about 70 KB at N = 128,
+// so that three CTAs share an SM.
 struct StateSmem {
     int a_bytes, v_bytes, total;
-    __host__ __device__ StateSmem(int K, int N) {
-        a_bytes = (K / 4) * 2 * 16384;  // K/4 M-tiles x 2 M-atoms x (128 k rows x 128 B), MN-major
-        v_bytes = (N / 64) * 16384;     // N/64 boxes of [128 t][64 n]
-        total = a_bytes + v_bytes + TQ * KMAX * 4 /*cv*/ + 96 * 4 /*itau, dec, l2t*/ + 64 /*wsum*/ +
-                16 /*E_end*/ + 64 /*bars*/;
+    __host__ __device__ explicit StateSmem(int N) {
+        a_bytes = 2 * 16384;         // 2 M-atoms x (128 k rows x 128 B), MN-major
+        v_bytes = (N / 64) * 16384;  // N/64 boxes of [128 t][64 n]
+        total = a_bytes + v_bytes + 32 * 4 /*dec*/ + 64 /*bars*/;
     }
 };
 
-template <bool REV>
-__global__ void __launch_bounds__(kThreads, 2)
+// P-slice of one state-pass CTA: the 128 TMEM lanes hold (mode, p) for all KK modes.
+template <int KK>
+__host__ __device__ constexpr int state_tps() {
+    return TQ / KK;
+}
+
+template <bool REV, int KK>
+__global__ void __launch_bounds__(kThreads, 3)
     tc_state_pass(const __grid_constant__ CUtensorMap mapV, StateArgs a) {
+    constexpr int TPSK = state_tps<KK>();  // 16 (KK = 8) or 32 (KK = 4)
+    constexpr int NX = TPSK / 8;           // 16-byte pieces of one position's x slice
     extern __shared__ unsigned char smem_raw[];
     unsigned char *base =
         reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const ScanDims &d = a.d;
-    const int K = d.K, N = d.N, P = d.P;
-    const StateSmem plan(K, N);
+    const int N = d.N, P = d.P;
+    const StateSmem plan(N);
     unsigned char *sA = base;
     unsigned char *sV = sA + plan.a_bytes;
-    float *cv_s = reinterpret_cast<float *>(sV + plan.v_bytes);  // [128][KMAX] this chunk's s or f
-    float *itau = cv_s + TQ * KMAX;                               // [32] 1 / tau
-    float *dec = itau + 32;                                       // [32]
-    float *l2t = dec + 32;                                        // [32] log2(e) / tau
-    float2 *wsum = reinterpret_cast<float2 *>(l2t + 32);          // [8]
-    float2 *Eend_s = wsum + 8;                                    // [1] E at the chunk end (hi, lo)
-    uint64_t *bars = reinterpret_cast<uint64_t *>(Eend_s + 2);    // tma, mma
+    float *dec = reinterpret_cast<float *>(sV + plan.v_bytes);     // [32] this chunk's decay per mode
+    uint64_t *bars = reinterpret_cast<uint64_t *>(dec + 32);        // tma, mma
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 2);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
 
     const int tid = threadIdx.x, w = tid >> 5, j = tid & 31;
-    const int h = blockIdx.y, b = blockIdx.z, p0 = blockIdx.x * TPS;
+    const int h = blockIdx.y, b = blockIdx.z, p0 = blockIdx.x * TPSK;
     const int g = h / (d.H / d.G);
-    const int mtiles = K / 4;
-    const uint32_t ncols = uint32_t(mtiles * N);  // power of two >= 32 (checked by the host)
+    const uint32_t ncols = uint32_t(N);  // 64 or 128
     const size_t PN = size_t(P) * N;
     const size_t bh = size_t(b) * d.H + h;
+    // this thread's TMEM lane: mode lm, row p0 + lp of the slice
+    const int lm = tid / TPSK, lp = tid % TPSK;
 
     if (tid == 0) {
         mbar_init(&bars[0], 1);
@@ -92,114 +162,67 @@ __global__ void __launch_bounds__(kThreads, 2)
         *abort_s = 0;
         fence_barrier_init();
     }
-    if (tid < K) {
-        const float tv = a.tau[h * K + tid];
-        itau[tid] = 1.f / tv;
-        l2t[tid] = kLog2e / tv;
-    }
     if (w == 0) tmem_alloc_once(tslot, ncols);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tslot;
     const uint32_t lane_base = tmem + (uint32_t(w * 32) << 16);
-    float tmax = 0.f;
-    for (int m = 0; m < K; ++m) tmax = fmaxf(tmax, a.tau[h * K + m]);
-    const float log_cap = logf(64.f * tmax);
 
-    // initial state into tensor memory: lane (m % 4, p), columns (m / 4, n)
-    for (int mt = 0; mt < mtiles; ++mt) {
-        const int m = mt * 4 + w;
-        const float *src = a.init ? a.init + (bh * K + m) * PN + size_t(p0 + j) * N : nullptr;
+    // initial state into tensor memory: lane (mode, p), columns n
+    {
+        const float *src = a.init ? a.init + (bh * KK + lm) * PN + size_t(p0 + lp) * N : nullptr;
         for (int c8 = 0; c8 < N; c8 += 8) {
             float v[8];
 #pragma unroll
             for (int i = 0; i < 8; ++i) v[i] = src ? src[c8 + i] : 0.f;
-            tmem_st8(lane_base + mt * N + c8, v);
+            tmem_st8(lane_base + c8, v);
         }
     }
     tmem_st_wait();
 
-    // Thread t owns chunk position t: its row of x (or dy) and its mode coefficients stay in
+    // Thread t owns chunk position t: its slice of x (or dy) and its coefficient per mode
+    // (s = kappa exp(-(E_end - E_t)/tau) forward, f = w_read exp(-E_t/tau) reverse) stay in
     // registers, and the inputs of chunk ci + 1 are fetched while chunk ci is processed.
-    uint4 nx[4];
-    float ndt = 1.f, nal = 1.f, nlm = 1.f;
-    float nw[KMAX];
+    constexpr int NC = KK / 4;  // 16-byte pieces of one coefficient kind
+    uint4 nx[NX], ncv[NC];
+    float ndec = 0.f;
     auto fetch = [&](int ci_) {
         const int c_ = REV ? d.nc - 1 - ci_ : ci_;
         const int c0_ = c_ * TQ, n_ = min(TQ, d.L - c0_);
         const int t = tid;
-        {  // this position's 32 x values (64 bytes), read row-coalesced across each 4-lane group
-            const int t4 = t & ~3;
-            get_rows<4>(nx, reinterpret_cast<const unsigned char *>(a.U + blh(d, b, c0_ + t4, h) * P + p0),
-                        size_t(d.H) * P * 2, n_ - t4);
+        {  // the slice's TPSK x values and the coefficient row, read row-coalesced
+            const int tg = t & ~(NX - 1);
+            get_rows<NX>(nx, reinterpret_cast<const unsigned char *>(a.U + blh(d, b, c0_ + tg, h) * P + p0),
+                         size_t(d.H) * P * 2, n_ - tg);
+            const int tc = t & ~(NC - 1);
+            get_rows<NC>(ncv,
+                         reinterpret_cast<const unsigned char *>(a.coef + blh(d, b, c0_ + tc, h) * 4 * KK +
+                                                                 (REV ? 0 : KK)),
+                         size_t(d.H) * 4 * KK * 4, n_ - tc);
         }
-        if (t < n_) {
-            const size_t i = blh(d, b, c0_ + t, h);
-            ndt = a.dt[i];
-            nal = a.alpha[i];
-            nlm = a.lam[i];
-            if (K == 8) {
-                const uint4 wv = *reinterpret_cast<const uint4 *>(a.W + i * K);
-                const __nv_bfloat162 *w2 = reinterpret_cast<const __nv_bfloat162 *>(&wv);
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const float2 f = __bfloat1622float2(w2[q]);
-                    nw[2 * q] = f.x;
-                    nw[2 * q + 1] = f.y;
-                }
-            } else {
-#pragma unroll
-                for (int m = 0; m < KMAX; ++m) nw[m] = m < K ? to_f(a.W[i * K + m]) : 0.f;
-            }
-        } else {
-#pragma unroll
-            for (int m = 0; m < KMAX; ++m) nw[m] = 0.f;
-        }
+        if (t < KK) ndec = a.coef[blh(d, b, c0_ + n_ - 1, h) * 4 * KK + 3 * KK + t];
     };
     if (d.nc > 0) fetch(0);
 
     int phase = 0;
     for (int ci = 0; ci < d.nc; ++ci, phase ^= 1) {
         const int c = REV ? d.nc - 1 - ci : ci;
-        const int c0 = c * TQ, n = min(TQ, d.L - c0);
+        const int c0 = c * TQ;
         const int t = tid;
-        uint4 xr[4];
-        float wcur[KMAX];
+        uint4 xr[NX];
+        float cv[KK];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) xr[q] = nx[q];
+        for (int q = 0; q < NX; ++q) xr[q] = nx[q];
 #pragma unroll
-        for (int m = 0; m < KMAX; ++m) wcur[m] = nw[m];
-        float e = 0.f;
-        if (t < n) {
-            bool cl;
-            e = token_rate(ndt, nal, nlm, log_cap, &cl);
+        for (int q = 0; q < NC; ++q) {
+            cv[4 * q] = __uint_as_float(ncv[q].x);
+            cv[4 * q + 1] = __uint_as_float(ncv[q].y);
+            cv[4 * q + 2] = __uint_as_float(ncv[q].z);
+            cv[4 * q + 3] = __uint_as_float(ncv[q].w);
         }
-        const float2 Et = group_scan128_f2(e, wsum);
-        if (t == n - 1) *Eend_s = Et;
+        if (t < KK) dec[t] = ndec;  // the previous chunk's emit has passed the barrier before its MMAs
         if (ci + 1 < d.nc) fetch(ci + 1);
-        __syncthreads();
-        // this position's coefficient per mode: s = kappa exp(-(E_end - E_t)/tau) (forward) or
-        // f = w_read exp(-E_t/tau) (reverse)
-        const float2 Eend = *Eend_s;
-        const float dEnd = diff_f2(Eend, Et);  // E_end - E_t >= 0
-        float cv[KMAX];
-#pragma unroll
-        for (int m = 0; m < KMAX; ++m) {
-            cv[m] = 0.f;
-            if (m < K && t < n) {
-                if (!REV)
-                    cv[m] = -expm1f(-e * itau[m]) * wcur[m] * ex2_approx(-dEnd * l2t[m]);
-                else
-                    cv[m] = wcur[m] * ex2_approx(-Et.x * l2t[m]);
-            }
-        }
-        if (t < K) dec[t] = ex2_approx(-Eend.x * l2t[t]);
-        {
-            float4 *o = reinterpret_cast<float4 *>(cv_s + t * KMAX);  // this thread's own row
-            o[0] = make_float4(cv[0], cv[1], cv[2], cv[3]);
-            o[1] = make_float4(cv[4], cv[5], cv[6], cv[7]);
-        }
         if (ci > 0) {  // previous chunk's MMAs done: tensor memory, sA and sV are free
             if (!mbar_wait(&bars[1], phase ^ 1)) *abort_s = 1;
         }
@@ -211,67 +234,60 @@ __global__ void __launch_bounds__(kThreads, 2)
             for (int jb = 0; jb < N / 64; ++jb)
                 tma_load_3d(sV + jb * 16384, &mapV, &bars[0], g * N + 64 * jb, c0, b);
         }
-        // A[(m%4, p), k] = s_{k,m} x_{k,p} as bf16, MN-major: row k = this thread's position,
-        // 64-element M-atoms (modes 2a, 2a+1 of the tile x 32 p), 128-byte swizzle
-#pragma unroll 1
-        for (int ma = 0; ma < 2 * mtiles; ++ma) {  // (mode tile, M-atom): modes 2 ma, 2 ma + 1
+        // A[(m, p), k] = s_{k,m} x_{k,p} as bf16, MN-major: row k = this thread's position,
+        // 64-element M-atoms (64 / TPSK modes x TPSK p each), 128-byte swizzle
+#pragma unroll
+        for (int ma = 0; ma < 2; ++ma) {
             unsigned char *row = sA + ma * 16384 + t * 128;
-            const float2 s01 = *reinterpret_cast<const float2 *>(cv_s + t * KMAX + 2 * ma);
-            const float s0 = s01.x, s1 = s01.y;
-            {
 #pragma unroll
-                for (int c8 = 0; c8 < 8; ++c8) {
-                    const float s = c8 < 4 ? s0 : s1;  // mode of this 8-element run
-                    const uint4 xv = xr[c8 & 3];
-                    const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
-                    uint32_t r[4];
+            for (int c8 = 0; c8 < 8; ++c8) {  // elements M = 64 ma + 8 c8 ..: mode M / TPSK
+                const float s = cv[(64 * ma + 8 * c8) / TPSK];
+                const uint4 xv = xr[c8 % NX];
+                const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
+                uint32_t r[4];
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        const float2 f = bf16x2_to_float2(xw[i]);
-                        r[i] = pack_bf16x2(s * f.x, s * f.y);
-                    }
-                    *reinterpret_cast<uint4 *>(row + ((c8 ^ (t & 7)) * 16)) = make_uint4(r[0], r[1], r[2], r[3]);
+                for (int i = 0; i < 4; ++i) {
+                    const float2 f = bf16x2_to_float2(xw[i]);
+                    r[i] = pack_bf16x2(s * f.x, s * f.y);
                 }
+                *reinterpret_cast<uint4 *>(row + ((c8 ^ (t & 7)) * 16)) = make_uint4(r[0], r[1], r[2], r[3]);
             }
         }
-        // emit the entering state (bf16) and apply the chunk's decay in place
-        // (the TMEM load of the next 32 columns is in flight while the current ones are processed)
+        // emit the entering state (bf16) and apply the chunk's decay in place (the TMEM load of
+        // the next 32 columns is in flight while the current ones are processed).  Blocks come in
+        // pairs covering 64 columns, so lane j then holds 128 contiguous bytes of its row; an
+        // 8 x 8 transpose of 16-byte pieces within each 8-lane group (rows p of one mode) lets
+        // every store instruction write 4 full rows of 128 bytes.
         {
-            const int nblk = mtiles * (N / 32);
-            // Blocks come in pairs (blk even, blk + 1) that cover 64 columns of one mode, so lane j
-            // then holds 128 contiguous bytes of row p0 + j; an 8 x 8 transpose of 16-byte pieces
-            // within each 8-lane group lets every store instruction write 4 full rows of 128 bytes.
-            uint4 e[8];
+            const int nblk = N / 32;  // even
+            const float dm = dec[lm];
+            bf16 *erow = a.emit + ((bh * d.nc + c) * KK + lm) * PN + size_t(p0 + (lp & ~7)) * N + 8 * (j & 7);
+            uint4 e8[8];
             auto process = [&](float *v, int blk, int hb) {
-                const int mt = blk / (N / 32), c32 = (blk % (N / 32)) * 32;
-                const int m = mt * 4 + w;
-                const float dm = dec[m];
 #pragma unroll
                 for (int q = 0; q < 4; ++q)
-                    e[4 * hb + q] =
+                    e8[4 * hb + q] =
                         make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
                                    pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
 #pragma unroll
                 for (int i = 0; i < 32; ++i) v[i] *= dm;
 #pragma unroll
-                for (int q = 0; q < 4; ++q) tmem_st8(lane_base + mt * N + c32 + 8 * q, v + 8 * q);
+                for (int q = 0; q < 4; ++q) tmem_st8(lane_base + 32 * blk + 8 * q, v + 8 * q);
                 if (hb) {
-                    lane_transpose<8>(e, j);
-                    bf16 *o = a.emit + ((bh * d.nc + c) * K + m) * PN + size_t(p0 + (j & ~7)) * N + (c32 - 32) +
-                              8 * (j & 7);
+                    lane_transpose<8>(e8, j);
+                    bf16 *o = erow + 32 * (blk - 1);
 #pragma unroll
-                    for (int q = 0; q < 8; ++q) *reinterpret_cast<uint4 *>(o + size_t(q) * N) = e[q];
+                    for (int q = 0; q < 8; ++q) *reinterpret_cast<uint4 *>(o + size_t(q) * N) = e8[q];
                 }
             };
-            auto col = [&](int blk) { return lane_base + (blk / (N / 32)) * N + (blk % (N / 32)) * 32; };
             float v0[32], v1[32];
-            tmem_ld32(col(0), v0);
-            for (int blk = 0; blk < nblk; blk += 2) {  // nblk = (K / 4) (N / 32) is even
+            tmem_ld32(lane_base, v0);
+            for (int blk = 0; blk < nblk; blk += 2) {
                 tmem_ld_wait();
-                tmem_ld32(col(blk + 1), v1);
+                tmem_ld32(lane_base + 32 * (blk + 1), v1);
                 process(v0, blk, 0);
                 tmem_ld_wait();
-                if (blk + 2 < nblk) tmem_ld32(col(blk + 2), v0);
+                if (blk + 2 < nblk) tmem_ld32(lane_base + 32 * (blk + 2), v0);
                 process(v1, blk + 1, 1);
             }
         }
@@ -288,11 +304,9 @@ __global__ void __launch_bounds__(kThreads, 2)
                 // descriptors advance by (byte offset >> 4) in their start-address field
                 const uint64_t ad0 = desc_sw128(smem_u32(sA), 16384, 1024);
                 const uint64_t bd0 = desc_sw128(smem_u32(sV), 16384, 1024);
-                for (int mt = 0; mt < mtiles; ++mt)
 #pragma unroll
-                    for (int ks = 0; ks < TQ / 16; ++ks)
-                        mma_bf16(tmem + mt * N, ad0 + uint64_t((mt * 32768 + ks * 2048) >> 4),
-                                 bd0 + uint64_t((ks * 2048) >> 4), idesc, 1);
+                for (int ks = 0; ks < TQ / 16; ++ks)
+                    mma_bf16(tmem, ad0 + uint64_t((ks * 2048) >> 4), bd0 + uint64_t((ks * 2048) >> 4), idesc, 1);
                 mma_commit(&bars[1]);
             }
         }
@@ -305,17 +319,14 @@ __global__ void __launch_bounds__(kThreads, 2)
     __syncthreads();
     tc_fence_after();
     if (!*abort_s && a.fin) {
-        for (int mt = 0; mt < mtiles; ++mt) {
-            const int m = mt * 4 + w;
-            float *dst = a.fin + (bh * K + m) * PN + size_t(p0 + j) * N;
-            for (int c32 = 0; c32 < N; c32 += 32) {
-                float v[32];
-                tmem_ld32(lane_base + mt * N + c32, v);
-                tmem_ld_wait();
-                float4 *o = reinterpret_cast<float4 *>(dst + c32);
+        float *dst = a.fin + (bh * KK + lm) * PN + size_t(p0 + lp) * N;
+        for (int c32 = 0; c32 < N; c32 += 32) {
+            float v[32];
+            tmem_ld32(lane_base + c32, v);
+            tmem_ld_wait();
+            float4 *o = reinterpret_cast<float4 *>(dst + c32);
 #pragma unroll
-                for (int q = 0; q < 8; ++q) o[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-            }
+            for (int q = 0; q < 8; ++q) o[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
         }
     }
     if (*abort_s && tid == 0) atomicExch(a.err, kTimeoutCode);
@@ -705,10 +716,28 @@ size_t tc_state_elems(const ScanDims &d) {
     return size_t(d.B) * d.H * d.nc * d.K * d.P * d.N;
 }
 
+size_t tc_coef_elems(const ScanDims &d) { return size_t(d.B) * d.L * d.H * 4 * d.K; }
+
+cudaError_t tc_coef_launch(const ScanDims &d, const ScanPtrs &p, float *coef, cudaStream_t st) {
+    if (d.nc == 0) return cudaSuccess;
+    CoefArgs a;
+    a.d = d;
+    a.wr = (const bf16 *)p.wr;
+    a.ww = (const bf16 *)p.ww;
+    a.dt = p.dt; a.alpha = p.alpha; a.lam = p.lam; a.tau = p.tau;
+    a.coef = coef;
+    trace_begin("coef_tc", st);
+    if (d.K == 8)
+        tc_coef<8><<<dim3(d.H, d.nc, d.B), TQ, 0, st>>>(a);
+    else
+        tc_coef<4><<<dim3(d.H, d.nc, d.B), TQ, 0, st>>>(a);
+    trace_end(st);
+    return cudaGetLastError();
+}
+
 cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, const void *V,
-                                 const void *W, const float *dt, const float *alpha,
-                                 const float *lam, const float *tau, const float *init,
-                                 void *emit, float *fin, int *err, cudaStream_t st) {
+                                 const float *coef, const float *init, void *emit, float *fin,
+                                 int *err, cudaStream_t st) {
     CUtensorMap mapV;
     if (!tc_make_map3(&mapV, V, uint64_t(d.G) * d.N, d.L, d.B, uint64_t(d.G) * d.N * 2,
                    uint64_t(d.L) * d.G * d.N * 2, 64, TQ, 1))
@@ -716,34 +745,36 @@ cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, con
     StateArgs a;
     a.d = d;
     a.U = (const bf16 *)U;
-    a.W = (const bf16 *)W;
-    a.dt = dt; a.alpha = alpha; a.lam = lam; a.tau = tau;
+    a.coef = coef;
     a.init = init;
     a.emit = (bf16 *)emit;
     a.fin = fin;
     a.err = err;
-    const size_t smem = StateSmem(d.K, d.N).total + 1024;
-    dim3 grid(d.P / TPS, d.H, d.B);
-    if (rev) {
-        auto k = tc_state_pass<true>;
-        cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-        trace_begin("state_pass_rev_tc", st);
-        k<<<grid, kThreads, smem, st>>>(mapV, a);
+    const size_t smem = StateSmem(d.N).total + 1024;
+    auto launch = [&](auto kern, int tps, const char *name) {
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+        trace_begin(name, st);
+        kern<<<dim3(d.P / tps, d.H, d.B), kThreads, smem, st>>>(mapV, a);
         trace_end(st);
+    };
+    if (d.K == 8) {
+        if (rev)
+            launch(tc_state_pass<true, 8>, state_tps<8>(), "state_pass_rev_tc");
+        else
+            launch(tc_state_pass<false, 8>, state_tps<8>(), "state_pass_fwd_tc");
     } else {
-        auto k = tc_state_pass<false>;
-        cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-        trace_begin("state_pass_fwd_tc", st);
-        k<<<grid, kThreads, smem, st>>>(mapV, a);
-        trace_end(st);
+        if (rev)
+            launch(tc_state_pass<true, 4>, state_tps<4>(), "state_pass_rev_tc");
+        else
+            launch(tc_state_pass<false, 4>, state_tps<4>(), "state_pass_fwd_tc");
     }
     return cudaGetLastError();
 }
 
-cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, int *err,
+cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, float *coef, int *err,
                         cudaStream_t st) {
-    cudaError_t e = tc_state_pass_launch(d, false, p.x, p.Bm, p.ww, p.dt, p.alpha, p.lam, p.tau,
-                                         p.h0, S_in, p.h_final, err, st);
+    cudaError_t e = tc_coef_launch(d, p, coef, st);
+    if (e == cudaSuccess) e = tc_state_pass_launch(d, false, p.x, p.Bm, coef, p.h0, S_in, p.h_final, err, st);
     if (e != cudaSuccess || d.nc == 0) return e;
     CUtensorMap mapC, mapB, mapX, mapS;
     const uint64_t GN = uint64_t(d.G) * d.N, HP = uint64_t(d.H) * d.P;

@@ -175,40 +175,6 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         }
     }
     __syncthreads();
-    if (grp == 1) {
-        // the per-position mode coefficients of the state terms, for tc_bwd_state:
-        // f = w_read exp(-E/tau), s = kappa u, u = exp(-(E_end - E)/tau), exp(-E/tau)
-        const float dEnd = diff_f2(E_s[n - 1], Et2);
-        float fv[KMAX], sv[KMAX], uv[KMAX], dv[KMAX];
-#pragma unroll
-        for (int m = 0; m < KMAX; ++m) {
-            dv[m] = ex2_approx(-Et2.x * l2r[m]);  // l2r = 0 beyond K
-            uv[m] = ex2_approx(-dEnd * l2r[m]);
-            fv[m] = wr_t[m] * dv[m];
-            sv[m] = kap_t[m] * uv[m];
-        }
-        // row t: f, s, u, exp(-E/tau), K floats each (rows t >= n are not written)
-        const size_t rs = size_t(d.H) * 4 * K * 4;
-        if (K == 8) {
-            const int t8 = t & ~7;
-            uint4 e8[8];
-#pragma unroll
-            for (int q = 0; q < 2; ++q) {
-                e8[q] = f4_bits(fv[4 * q], fv[4 * q + 1], fv[4 * q + 2], fv[4 * q + 3]);
-                e8[2 + q] = f4_bits(sv[4 * q], sv[4 * q + 1], sv[4 * q + 2], sv[4 * q + 3]);
-                e8[4 + q] = f4_bits(uv[4 * q], uv[4 * q + 1], uv[4 * q + 2], uv[4 * q + 3]);
-                e8[6 + q] = f4_bits(dv[4 * q], dv[4 * q + 1], dv[4 * q + 2], dv[4 * q + 3]);
-            }
-            put_rows<8, false>(e8, reinterpret_cast<unsigned char *>(a.coef + blh(d, b, c0 + t8, h) * 4 * K), rs,
-                               n - t8);
-        } else {  // K == 4
-            const int t4 = t & ~3;
-            uint4 e4[4] = {f4_bits(fv[0], fv[1], fv[2], fv[3]), f4_bits(sv[0], sv[1], sv[2], sv[3]),
-                           f4_bits(uv[0], uv[1], uv[2], uv[3]), f4_bits(dv[0], dv[1], dv[2], dv[3])};
-            put_rows<4, false>(e4, reinterpret_cast<unsigned char *>(a.coef + blh(d, b, c0 + t4, h) * 4 * K), rs,
-                               n - t4);
-        }
-    }
     // ---- Gamma below the diagonal 32 x 32 blocks, factored through the log-decay E_a at the end
     // of the column block J (as in the forward output kernel): Gamma[t, k in J] =
     // sum_m U_J[t, m] V[k, m] and Gamma'[t, k] = sum_m U_J[t, m] V[k, m] / tau_m, tf32 products.
@@ -843,7 +809,7 @@ __global__ void __launch_bounds__(kStLaunch, 1)
             }
 #pragma unroll
             for (int k = 0; k < KMAX; ++k) acc_h[k] = 0.f;
-            // coefficients of this row from tc_bwd_intra (group 0: f, exp(-E/tau); group 1: s, u;
+            // coefficients of this row from tc_coef (group 0: f, exp(-E/tau); group 1: s, u;
             // both: s) and its row of dY / X, read row-coalesced across each 8-lane group
             const int t8 = t & ~7;
             const size_t r8 = blh(d, b, c0 + t8, h);
@@ -1097,6 +1063,7 @@ size_t tc_bwd_workspace_bytes(const ScanDims &d, TcBwdWorkspace *l, char *base) 
     };
     const size_t st = tc_state_elems(d) * 2;
     l->S_in = take(st);
+    l->coef = (float *)take(tc_coef_elems(d) * 4);  // S_in and coef as in the forward's workspace
     l->dS_out = take(st);
     l->dx_acc = (float *)take(blh_ * d.P * 4);
     l->dwr_acc = (float *)take(blh_ * d.K * 4);
@@ -1105,7 +1072,6 @@ size_t tc_bwd_workspace_bytes(const ScanDims &d, TcBwdWorkspace *l, char *base) 
     l->rect = (float *)take(blh_ * 4);
     l->cdot = (float *)take(size_t(d.B) * d.H * d.nc * d.K * 4);
     l->mh_total = (float *)take(size_t(d.B) * d.nc * d.G * TQ * TQ * 4);
-    l->coef = (float *)take(blh_ * 4 * d.K * 4);
     l->dB_acc = (float *)take(size_t(d.B) * d.L * d.G * d.N * 4);
     l->dC_acc = (float *)take(size_t(d.B) * d.L * d.G * d.N * 4);
     return off;
@@ -1121,11 +1087,10 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
     if ((e = cudaMemsetAsync(ws.cdot, 0, sizeof(float) * d.B * d.H * d.nc * d.K, st))) return e;
     if ((e = cudaMemsetAsync(ws.mh_total, 0, sizeof(float) * d.B * d.nc * d.G * TQ * TQ, st))) return e;
     if (!reuse_states &&
-        (e = tc_state_pass_launch(d, false, p.x, p.Bm, p.ww, p.dt, p.alpha, p.lam, p.tau, p.h0,
-                                  ws.S_in, nullptr, err, st)))
+        ((e = tc_coef_launch(d, p, ws.coef, st)) ||
+         (e = tc_state_pass_launch(d, false, p.x, p.Bm, ws.coef, p.h0, ws.S_in, nullptr, err, st))))
         return e;
-    if ((e = tc_state_pass_launch(d, true, p.dy, p.Cm, p.wr, p.dt, p.alpha, p.lam, p.tau,
-                                  p.dh_final, ws.dS_out, p.dh0, err, st)))
+    if ((e = tc_state_pass_launch(d, true, p.dy, p.Cm, ws.coef, p.dh_final, ws.dS_out, p.dh0, err, st)))
         return e;
     if (d.nc == 0) return cudaSuccess;
     const uint64_t GN = uint64_t(d.G) * d.N, HP = uint64_t(d.H) * d.P;
