@@ -345,6 +345,7 @@ struct OutArgs {
 };
 
 constexpr int kOutThreads = 256;  // two groups of four warps share the 128 TMEM lanes
+constexpr int kOutLaunch = kOutThreads + 32;  // a ninth warp issues the entering-state MMAs
 constexpr int kSBuf = 3;          // S_in tiles in flight
 
 // Shared-memory plan of tc_chunk_fwd (offsets from a 1024-aligned base): about 110 KB at
@@ -353,22 +354,78 @@ struct OutSmem {
     int c, m, x, s, total;
     __host__ __device__ explicit OutSmem(int N) {
         c = (N / 64) * 16384;  // C chunk [t][n], K-major, 64-wide n atoms
-        m = 2 * 16384;         // B chunk, then Gamma o G [t][k], then two (f o C) tiles
+        m = 2 * 16384;         // B chunk, then Gamma o G [t][k]
         x = 16384;             // x chunk [t][p]: the MN-major operand of the intra MMA
         s = kSBuf * 8192;      // S_in tiles, one (mode, 64-wide n half) each: [p][n]
         total = c + m + x + s + TQ * KMAX * 4 /*kappa*/ + TQ * 8 /*E*/ + 64 * 4 /*tau, l2t*/ +
-                64 /*wsum*/ + 8 * 8 /*bars*/ + 16;
+                64 /*wsum*/ + 24 * 8 /*bars*/ + 16;
     }
 };
 
-// One CTA per (b, h, chunk), headdim 64, all in one TMEM accumulator Y[t, p]:
-//   Y  = (Gamma o C B^T) X                      (intra-chunk pairs, K = t)
-//   Y += sum_m (f_m o C) S_in,m^T               (entering state, K = (m, n), 64-wide n steps)
-//   y  = Y + D x
-// G = C B^T comes from the tensor cores; Gamma is formed per position pair; the scaled copies
-// f_m o C are written by the threads into two alternating tiles while the tensor cores consume
-// the previous one, and the S_in tiles stream in by TMA three steps ahead.
-__global__ void __launch_bounds__(kOutThreads, 2)
+
+// The entering-state MMAs of tc_chunk_fwd (one thread of the ninth warp): S_in tiles j (mode
+// j / nhalf, 64-wide n half j % nhalf) stream through three buffers; Z_m = C S_in,m^T goes to
+// TMEM buffer m % 4 once the compute threads have read its previous contents.
+__device__ __forceinline__ void chunk_fwd_issuer(const ScanDims &d, unsigned char *sC, unsigned char *sS,
+                                                 uint64_t *bars, volatile int *abort_s, uint32_t tmem,
+                                                 const CUtensorMap &mapS, int srow) {
+    const int nhalf = d.N / 64, ntile = d.K * nhalf;
+    auto load = [&](int j) {
+        mbar_arrive_expect_tx(&bars[3 + j % kSBuf], 8192u);
+        tma_load_3d(sS + (j % kSBuf) * 8192, &mapS, &bars[3 + j % kSBuf], (j % nhalf) * 64, 0, srow + j / nhalf);
+    };
+    // the S ring holds the Gamma operands until their MMAs are done
+    if (!mbar_wait(&bars[1], 0)) {
+        *abort_s = 1;
+        return;
+    }
+    for (int j = 0; j < min(kSBuf, ntile); ++j) load(j);
+    // the intra Y MMA (issued after the Gamma o G pass) frees the G and Gamma columns
+    if (!mbar_wait(&bars[2], 0)) {
+        *abort_s = 1;
+        return;
+    }
+    tc_fence_after();
+    const uint32_t idZ = idesc_bf16(128, 64, false, false);
+    for (int j = 0; j < ntile && !*abort_s; ++j) {
+        const int m = j / nhalf, hn = j % nhalf, zb = m & 3;
+        if (hn == 0) {  // buffer zb read by all compute threads (buffer 3: first the intra Y)
+            const int k = m >> 2;
+            if ((zb == 3 || k > 0) && !mbar_wait(&bars[13 + zb], (zb == 3 ? k : k - 1) & 1)) {
+                *abort_s = 1;
+                break;
+            }
+        }
+        if (!mbar_wait(&bars[3 + j % kSBuf], (j / kSBuf) & 1)) {
+            *abort_s = 1;
+            break;
+        }
+        tc_fence_after();
+        const uint32_t sa = smem_u32(sC) + hn * 16384, sb = smem_u32(sS) + (j % kSBuf) * 8192;
+        for (int ks = 0; ks < 4; ++ks)
+            mma_bf16(tmem + 64 * zb, desc_sw128(sa + ks * 32, 16, 1024), desc_sw128(sb + ks * 32, 16, 1024), idZ,
+                     (hn > 0 || ks > 0) ? 1u : 0u);
+        mma_commit(&bars[6 + j % kSBuf]);
+        if (hn == nhalf - 1) mma_commit(&bars[9 + zb]);
+        // tile j - 1's MMAs done: its buffer takes tile j + 2
+        if (j >= 1 && j + 2 < ntile) {
+            if (!mbar_wait(&bars[6 + (j - 1) % kSBuf], ((j - 1) / kSBuf) & 1)) {
+                *abort_s = 1;
+                break;
+            }
+            load(j + 2);
+        }
+    }
+}
+
+// One CTA per (b, h, chunk), headdim 64:
+//   Y  = (Gamma o C B^T) X                      (intra-chunk pairs, K = t; tensor memory)
+//   y  = Y + sum_m f_m o (C S_in,m^T) + D x     (entering state)
+// G = C B^T comes from the tensor cores; Gamma is formed per position pair.  A ninth warp
+// streams Z_m = C S_in,m^T through four 64-column TMEM buffers (S_in tiles by TMA, three ahead)
+// while the 256 compute threads fold each Z_m into their rows of y with the weight f_m[t]:
+// no per-mode scaled operand and no CTA-wide barrier per mode.
+__global__ void __launch_bounds__(kOutLaunch, 2)
     tc_chunk_fwd(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapB,
                  const __grid_constant__ CUtensorMap mapX, const __grid_constant__ CUtensorMap mapS,
                  OutArgs a) {
@@ -387,20 +444,22 @@ __global__ void __launch_bounds__(kOutThreads, 2)
     float *tau_s = reinterpret_cast<float *>(E_s + TQ);           // [32]
     float *l2t = tau_s + 32;                                      // [32] log2(e) / tau
     float2 *wsum = reinterpret_cast<float2 *>(l2t + 32);          // [8]
-    // bars: 0 C, B, x loaded | 1 G done | 2 intra Y done | 3..5 S tile loaded | 6, 7 (f o C) tile consumed
+    // bars: 0 C, B, x loaded | 1 G done | 2 intra Y done | 3..5 S tile loaded | 6..8 S tile read
+    //       by its MMAs | 9..12 Z buffer written | 13..16 Z buffer read (all compute threads)
     uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);
-    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 8);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 17);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
 
     const int tid = threadIdx.x, grp = tid >> 7, t = tid & 127, w4 = (tid >> 5) & 3;
     const int h = blockIdx.x, c = blockIdx.y, b = blockIdx.z;
     const int g = h / (d.H / d.G);
     const int c0 = c * TQ, n = min(TQ, d.L - c0);
-    const int nhalf = N / 64, niter = K * nhalf;
+    const int nhalf = N / 64;
     const int srow = int(((size_t(b) * d.H + h) * d.nc + c) * K);
 
     if (tid == 0) {
-        for (int i = 0; i < 8; ++i) mbar_init(&bars[i], 1);
+        for (int i = 0; i < 13; ++i) mbar_init(&bars[i], 1);
+        for (int i = 13; i < 17; ++i) mbar_init(&bars[i], kOutThreads);
         *abort_s = 0;
         fence_barrier_init();
     }
@@ -429,8 +488,12 @@ __global__ void __launch_bounds__(kOutThreads, 2)
     tc_fence_after();
     const uint32_t tmem = *tslot;
     const uint32_t lane_base = tmem + (uint32_t(w4 * 32) << 16);
-    // TMEM: G = C B^T at [0, 128), the factored Gamma blocks at [128, 256); Y replaces G
-    constexpr uint32_t colG = 0, colGam = 128, colY = 0;
+    // TMEM: G = C B^T at [0, 128), the factored Gamma blocks at [128, 256); then the intra Y at
+    // [192, 256) and the Z_m buffers at 64 (m % 4) (buffer 3 once Y has been read)
+    constexpr uint32_t colG = 0, colGam = 128, colY = 192;
+    if (tid >= kOutThreads) {
+        if (tid == kOutThreads) chunk_fwd_issuer(a.d, sC, sS, bars, abort_s, tmem, mapS, srow);
+    } else {
 
     if (tid == 0) {
         mbar_arrive_expect_tx(&bars[0], uint32_t(2 * plan.c + plan.x));
@@ -448,7 +511,7 @@ __global__ void __launch_bounds__(kOutThreads, 2)
         bool cl;
         e = token_rate(dtv, alv, lmv, log_cap, &cl);
     }
-    const float2 Et2 = group_scan128_f2(e, wsum);  // in-chunk cumulative log-decay (hi, lo)
+    const float2 Et2 = group_scan128_f2<true>(e, wsum);  // in-chunk cumulative log-decay (hi, lo)
     if (grp == 0) E_s[t] = Et2;
     float f_t[KMAX], kap_t[KMAX];
 #pragma unroll
@@ -462,7 +525,7 @@ __global__ void __launch_bounds__(kOutThreads, 2)
             if (grp == 0) kap_s[t * KMAX + m] = kap_t[m];
         }
     }
-    __syncthreads();
+    sync_first256();
     // Gamma below the diagonal 32 x 32 blocks, factored through the log-decay E_a at the end of
     // the column block J: exp(-(E_t - E_k)/tau) = exp(-(E_t - E_a)/tau) exp(-(E_a - E_k)/tau),
     // both factors <= 1, so Gamma[t, k in J] = sum_m U_J[t, m] V[k, m] (a K = 8 tf32 product):
@@ -494,7 +557,7 @@ __global__ void __launch_bounds__(kOutThreads, 2)
         *reinterpret_cast<uint4 *>(row + (((2 * J + 1) ^ (r & 7)) * 16)) = make_uint4(v[4], v[5], v[6], v[7]);
     }
     fence_async_smem();
-    __syncthreads();
+    sync_first256();
     // G = C B^T (bf16) and the four Gamma column blocks (tf32)
     if (tid == 0) {
         if (!mbar_wait(&bars[0], 0)) {
@@ -514,17 +577,10 @@ __global__ void __launch_bounds__(kOutThreads, 2)
             mma_commit(&bars[1]);
         }
     }
-    __syncthreads();
+    sync_first256();
     if (!*abort_s && !mbar_wait(&bars[1], 0)) *abort_s = 1;
-    __syncthreads();
+    sync_first256();
     tc_fence_after();
-    // the S ring is free again: first S_in tiles
-    if (tid == 0 && !*abort_s) {
-        for (int j = 0; j < min(kSBuf, niter); ++j) {
-            mbar_arrive_expect_tx(&bars[3 + j], 8192u);
-            tma_load_3d(sS + j * 8192, &mapS, &bars[3 + j], (j % nhalf) * 64, 0, srow + j / nhalf);
-        }
-    }
     if (!*abort_s) {
         // row t of Gamma o G -> bf16, K-major [t][k] over the B tile.  Warp rows are one 32-block
         // I; column block kc < I takes the factored Gamma, kc == I the direct sum (pairs k <= t),
@@ -571,7 +627,7 @@ __global__ void __launch_bounds__(kOutThreads, 2)
     }
     fence_async_smem();
     tc_fence_before();
-    __syncthreads();
+    sync_first256();
     tc_fence_after();
     if (tid == 0 && !*abort_s) {  // Y = (Gamma o G) X: M = t, N = p, K = k (over G's columns)
         const uint32_t idY = idesc_bf16(128, 64, false, true);
@@ -580,71 +636,32 @@ __global__ void __launch_bounds__(kOutThreads, 2)
                      desc_sw128(smem_u32(sX) + ks * 2048, 16384, 1024), idY, ks > 0);
         mma_commit(&bars[2]);
     }
-    // the (f o C) tiles take the place of Gamma o G once the intra MMA has read it
+    // y row t (group g: p in [32 g, 32 g + 32)): the intra Y from tensor memory, then every
+    // mode's Z_m = C S_in,m^T weighted by f_m[t]; each buffer read is handed back to the issuer
+    float yv[32];
     if (!*abort_s && !mbar_wait(&bars[2], 0)) *abort_s = 1;
-    __syncthreads();
-    const uint32_t idS = idesc_bf16(128, 64, false, false);
-    for (int it = 0; it < niter; ++it) {
-        const int m = it / nhalf, hn = it % nhalf, buf = it & 1;
-        if (it >= 2 && !*abort_s) {  // the MMA of step it - 2 has released tile buffer `buf`
-            if (!mbar_wait(&bars[6 + buf], ((it - 2) >> 1) & 1)) *abort_s = 1;
-        }
-        // (f_m o C)[t, n] for this 64-wide n half; group g writes n in [32 g, 32 g + 32)
-        float fm = 0.f;
+    tc_fence_after();
+    tmem_ld32(lane_base + colY + grp * 32, yv);
+    tmem_ld_wait();
+    tc_fence_before();
+    mbar_arrive(&bars[13 + 3]);
 #pragma unroll
-        for (int q = 0; q < KMAX; ++q)
-            if (q == m) fm = f_t[q];
-        const unsigned char *crow = sC + hn * 16384 + t * 128;
-        unsigned char *drow = sM + buf * 16384 + t * 128;
+    for (int m = 0; m < KMAX; ++m) {
+        if (m < K) {
+            const int zb = m & 3;
+            if (!*abort_s && !mbar_wait(&bars[9 + zb], (m >> 2) & 1)) *abort_s = 1;
+            tc_fence_after();
+            float zv[32];
+            tmem_ld32(lane_base + 64 * zb + grp * 32, zv);
+            tmem_ld_wait();
+            tc_fence_before();
+            mbar_arrive(&bars[13 + zb]);
+            const float fm = f_t[m];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const int off = (((grp * 4 + q) ^ (t & 7)) * 16);
-            uint4 u = *reinterpret_cast<const uint4 *>(crow + off);
-            const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&u);
-            uint32_t r[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const float2 f = __bfloat1622float2(h2[i]);
-                r[i] = pack_bf16x2(f.x * fm, f.y * fm);
-            }
-            *reinterpret_cast<uint4 *>(drow + off) = make_uint4(r[0], r[1], r[2], r[3]);
-        }
-        // S tile it + 2 into the buffer the MMA of step it - 1 read (two steps of lead); issued
-        // by a thread of another warp than the MMA issuer, after its own tile row is written
-        if (tid == 32 && it >= 1 && it + 2 < niter && !*abort_s) {
-            if (!mbar_wait(&bars[6 + ((it - 1) & 1)], ((it - 1) >> 1) & 1)) {
-                *abort_s = 1;
-            } else {
-                const int j = it + 2;
-                mbar_arrive_expect_tx(&bars[3 + j % kSBuf], 8192u);
-                tma_load_3d(sS + (j % kSBuf) * 8192, &mapS, &bars[3 + j % kSBuf], (j % nhalf) * 64, 0,
-                            srow + j / nhalf);
-            }
-        }
-        fence_async_smem();
-        tc_fence_before();
-        __syncthreads();
-        if (tid == 0 && !*abort_s) {
-            const int sb = it % kSBuf;
-            if (!mbar_wait(&bars[3 + sb], (it / kSBuf) & 1)) {
-                *abort_s = 1;
-            } else {
-                tc_fence_after();
-                for (int ks = 0; ks < 4; ++ks)
-                    mma_bf16(tmem + colY, desc_sw128(smem_u32(sM + buf * 16384) + ks * 32, 16, 1024),
-                             desc_sw128(smem_u32(sS + sb * 8192) + ks * 32, 16, 1024), idS, 1);
-                mma_commit(&bars[6 + buf]);
-            }
+            for (int i = 0; i < 32; ++i) yv[i] = fmaf(fm, zv[i], yv[i]);
         }
     }
-    if (!*abort_s && niter > 0 && !mbar_wait(&bars[6 + ((niter - 1) & 1)], ((niter - 1) >> 1) & 1))
-        *abort_s = 1;
-    __syncthreads();
-    tc_fence_after();
-    {  // y = Y + D x; group g takes p in [32 g, 32 g + 32) (rows t >= n and aborted CTAs write nothing)
-        float v[32];
-        tmem_ld32(lane_base + colY + grp * 32, v);
-        tmem_ld_wait();
+    {  // y = Y + sum_m f_m Z_m + D x (rows t >= n and aborted CTAs write nothing)
         const float Dh = a.D[h];
         const unsigned char *xrow = sX + t * 128;
         uint4 e[4];
@@ -656,7 +673,7 @@ __global__ void __launch_bounds__(kOutThreads, 2)
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const float2 f = bf16x2_to_float2(xw[i]);
-                r[i] = pack_bf16x2(fmaf(Dh, f.x, v[8 * q + 2 * i]), fmaf(Dh, f.y, v[8 * q + 2 * i + 1]));
+                r[i] = pack_bf16x2(fmaf(Dh, f.x, yv[8 * q + 2 * i]), fmaf(Dh, f.y, yv[8 * q + 2 * i + 1]));
             }
             e[q] = make_uint4(r[0], r[1], r[2], r[3]);
         }
@@ -664,6 +681,7 @@ __global__ void __launch_bounds__(kOutThreads, 2)
         put_rows<4, false>(e, reinterpret_cast<unsigned char *>(a.y + blh(d, b, c0 + t4, h) * P + grp * 32),
                            size_t(d.H) * P * 2, *abort_s ? 0 : n - t4);
     }
+    }  // compute threads
     if (*abort_s && tid == 0) atomicExch(a.err, kTimeoutCode);
     tc_fence_before();
     __syncthreads();
@@ -795,7 +813,7 @@ cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, float 
     cudaFuncSetAttribute(tc_chunk_fwd, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
     dim3 grid(d.H, d.nc, d.B);
     trace_begin("chunk_fwd_tc", st);
-    tc_chunk_fwd<<<grid, kOutThreads, smem, st>>>(mapC, mapB, mapX, mapS, a);
+    tc_chunk_fwd<<<grid, kOutLaunch, smem, st>>>(mapC, mapB, mapX, mapS, a);
     trace_end(st);
     return cudaGetLastError();
 }

@@ -163,8 +163,22 @@ __device__ __forceinline__ float2 f2_add(float2 a, float2 b) {
     return make_float2(hi, lo - (hi - s));
 }
 
+// Barrier over the first 256 threads of the block only (named barrier 1), for kernels whose
+// extra warps take no part in the per-position work.
+__device__ __forceinline__ void sync_first256() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+
+template <bool FIRST256>
+__device__ __forceinline__ void block_or_first256_sync() {
+    if (FIRST256)
+        sync_first256();
+    else
+        __syncthreads();
+}
+
 // Inclusive prefix sum of one value per thread within groups of four warps (threads
 // 128 g .. 128 g + 127 scan independently), as a float pair; wsum holds one pair per warp.
+// FIRST256: only the first 256 threads call it (they synchronise on named barrier 1).
+template <bool FIRST256 = false>
 __device__ __forceinline__ float2 group_scan128_f2(float v, float2 *wsum) {
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
     float2 p = make_float2(v, 0.f);
@@ -174,11 +188,11 @@ __device__ __forceinline__ float2 group_scan128_f2(float v, float2 *wsum) {
         if (lane >= o) p = f2_add(p, u);
     }
     if (lane == 31) wsum[w] = p;
-    __syncthreads();
+    block_or_first256_sync<FIRST256>();
     float2 off = make_float2(0.f, 0.f);
     const int g0 = w & ~3;
     for (int i = g0; i < w; ++i) off = f2_add(off, wsum[i]);
-    __syncthreads();
+    block_or_first256_sync<FIRST256>();
     return f2_add(p, off);
 }
 
