@@ -1015,18 +1015,44 @@ __global__ void __launch_bounds__(kThreads) tc_bwd_final(BwdArgs a) {
         a.dlam[i] = ge / (alv * lmv);
         a.dalpha[i] = -ge * logf(lmv) / (alv * alv);
     }
-    // dx = dx_acc + D dy (bf16) and sum dy x, one warp per row, two p per lane
+    // dx = dx_acc + D dy (bf16) and sum dy x: each thread takes 8 p of 8 rows (rows r = 16 j + t / 8,
+    // p in [8 (t % 8), 8 (t % 8) + 8)), all loads issued before any is used; every instruction
+    // covers 16 whole 256-byte (or 128-byte) row segments
     const float Dh = a.D[h];
     float dd = 0.f;
-#pragma unroll 4
-    for (int r = w; r < n; r += 4) {
-        const size_t i0 = blh(d, b, c0 + r, h) * P;
-        for (int p = 2 * lane; p < P; p += 64) {
-            const float2 acc = *reinterpret_cast<const float2 *>(a.dx_acc + i0 + p);
-            const float2 dyv = bf16x2_to_float2(*reinterpret_cast<const uint32_t *>(a.dy + i0 + p));
-            const float2 xv = bf16x2_to_float2(*reinterpret_cast<const uint32_t *>(a.x + i0 + p));
-            *reinterpret_cast<uint32_t *>(a.dx + i0 + p) = pack_bf16x2(fmaf(Dh, dyv.x, acc.x), fmaf(Dh, dyv.y, acc.y));
-            dd = fmaf(dyv.x, xv.x, fmaf(dyv.y, xv.y, dd));
+    {
+        const int p8 = 8 * (t & 7), r0 = t >> 3;
+        float4 acc[8][2];
+        uint4 dyv[8], xv[8];
+#pragma unroll
+        for (int jr = 0; jr < 8; ++jr) {
+            const int r = 16 * jr + r0;
+            if (r < n) {
+                const size_t i0 = blh(d, b, c0 + r, h) * P + p8;
+                acc[jr][0] = *reinterpret_cast<const float4 *>(a.dx_acc + i0);
+                acc[jr][1] = *reinterpret_cast<const float4 *>(a.dx_acc + i0 + 4);
+                dyv[jr] = *reinterpret_cast<const uint4 *>(a.dy + i0);
+                xv[jr] = *reinterpret_cast<const uint4 *>(a.x + i0);
+            }
+        }
+#pragma unroll
+        for (int jr = 0; jr < 8; ++jr) {
+            const int r = 16 * jr + r0;
+            if (r < n) {
+                const size_t i0 = blh(d, b, c0 + r, h) * P + p8;
+                const float av8[8] = {acc[jr][0].x, acc[jr][0].y, acc[jr][0].z, acc[jr][0].w,
+                                      acc[jr][1].x, acc[jr][1].y, acc[jr][1].z, acc[jr][1].w};
+                const uint32_t dw[4] = {dyv[jr].x, dyv[jr].y, dyv[jr].z, dyv[jr].w};
+                const uint32_t xw[4] = {xv[jr].x, xv[jr].y, xv[jr].z, xv[jr].w};
+                uint32_t o[4];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float2 fy = bf16x2_to_float2(dw[q]), fx = bf16x2_to_float2(xw[q]);
+                    o[q] = pack_bf16x2(fmaf(Dh, fy.x, av8[2 * q]), fmaf(Dh, fy.y, av8[2 * q + 1]));
+                    dd = fmaf(fy.x, fx.x, fmaf(fy.y, fx.y, dd));
+                }
+                *reinterpret_cast<uint4 *>(a.dx + i0) = make_uint4(o[0], o[1], o[2], o[3]);
+            }
         }
     }
     dd = warp_sum(dd);
