@@ -49,7 +49,8 @@ struct BwdArgs {
     bf16 *dx, *dwr, *dww;
     float *ddt, *dalpha, *dlam, *dD;
     int *err;
-    int hg;  // heads per dC/dB group
+    int hg;      // heads per dC/dB group
+    int pf_sms;  // SMs of the device: CTAs of the persistent intra kernel
 };
 
 __device__ __forceinline__ void store_bf16x8(unsigned char *p, const float *v) {
@@ -72,7 +73,8 @@ struct IntraSmem {
         dy = 16384;                // dy chunk
         mg = 2 * 16384;            // Gamma o G, [t][k] K-major
         xx = TQ * XS * 4;          // fp32 Gamma' G H, then its row prefix sums
-        total = rcb + x + dy + mg + xx + 4 * TQ * KMAX * 4 + TQ * 8 + 64 * 4 + 64 + 64 + 64;
+        total = rcb + x + dy + mg + xx + 4 * TQ * KMAX * 4 + TQ * 8 + 64 * 4 + 64 + 64 + 64 +
+                3 * TQ * 4 + 2 * TQ * 16;  // + the next item's per-position inputs
     }
 };
 
@@ -100,40 +102,60 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     float *l2t = reinterpret_cast<float *>(E_s + TQ);
     float *tau_s = l2t + 32;
     float2 *wsum = reinterpret_cast<float2 *>(tau_s + 32);
+    // bars: 0 C, B, x of the item loaded | 1 G, H, Gamma MMAs done | 2 dx MMA done | 3 dy loaded
     uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);
-    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 3);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 4);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
+    // the next item's per-position inputs, staged by cp.async: dt, alpha, lam [3][128] floats and
+    // w_read, w_write [2][128] x 16 bytes
+    float *pf_f = reinterpret_cast<float *>(tslot + 4);
+    unsigned char *pf_w = reinterpret_cast<unsigned char *>(pf_f + 3 * TQ);
 
     const int tid = threadIdx.x, grp = tid >> 7, t = tid & 127, w4 = (tid >> 5) & 3;
-    const int h = blockIdx.x, c = blockIdx.y, b = blockIdx.z;
-    const int g = h / (d.H / d.G);
-    const int c0 = c * TQ, n = min(TQ, d.L - c0);
+    // persistent: items (h, c, b) in launch order, gridDim.x CTAs apart
+    const int nitems = d.H * d.nc * d.B;
+    auto item_hcb = [&](int item) { return make_int3(item % d.H, (item / d.H) % d.nc, item / (d.H * d.nc)); };
+    // tid 0: the item's C, B and x tiles (bars[0]) / its dy tile (bars[3]) by TMA
+    auto load_cbx = [&](int item) {
+        const int3 hcb = item_hcb(item);
+        const int h_ = hcb.x, c_ = hcb.y, b_ = hcb.z;
+        const int g_ = h_ / (d.H / d.G);
+        mbar_arrive_expect_tx(&bars[0], uint32_t(2 * (N / 64) * 16384 + 16384));
+        for (int jb = 0; jb < N / 64; ++jb) {
+            tma_load_3d(sC + jb * 16384, &mapC, &bars[0], g_ * N + 64 * jb, c_ * TQ, b_);
+            tma_load_3d(sB + jb * 16384, &mapB, &bars[0], g_ * N + 64 * jb, c_ * TQ, b_);
+        }
+        tma_load_3d(sX, &mapX, &bars[0], h_ * P, c_ * TQ, b_);
+    };
+    auto load_dy = [&](int item) {
+        const int3 hcb = item_hcb(item);
+        const int h_ = hcb.x, c_ = hcb.y, b_ = hcb.z;
+        mbar_arrive_expect_tx(&bars[3], 16384u);
+        tma_load_3d(sDY, &mapDY, &bars[3], h_ * P, c_ * TQ, b_);
+    };
+    // every thread: its position's dt, alpha, lam, w_read, w_write of the item into the staging area
+    auto stage_inputs = [&](int item) {
+        const int3 hcb = item_hcb(item);
+        const int h_ = hcb.x, c_ = hcb.y, b_ = hcb.z;
+        if (c_ * TQ + t < d.L && grp == 0) {
+            const size_t i = blh(d, b_, c_ * TQ + t, h_);
+            cp_async4(pf_f + t, a.dt + i);
+            cp_async4(pf_f + TQ + t, a.alpha + i);
+            cp_async4(pf_f + 2 * TQ + t, a.lam + i);
+        } else if (c_ * TQ + t < d.L) {
+            const size_t i = blh(d, b_, c_ * TQ + t, h_);
+            cp_async_bytes(pf_w + t * 16, a.wr + i * K, 2 * K);
+            cp_async_bytes(pf_w + TQ * 16 + t * 16, a.ww + i * K, 2 * K);
+        }
+        cp_async_commit();
+    };
 
     if (tid == 0) {
-        for (int i = 0; i < 3; ++i) mbar_init(&bars[i], 1);
+        for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
         *abort_s = 0;
         fence_barrier_init();
     }
-    if (tid < K) {
-        const float tv = a.tau[h * K + tid];
-        tau_s[tid] = tv;
-        l2t[tid] = kLog2e / tv;
-    }
     if (tid < 32) tmem_alloc_once(tslot, 512);
-    // per-position inputs of row t, all loads issued before anything waits on them
-    float dtv = 1.f, alv = 1.f, lmv = 1.f;
-    float wr_t[KMAX], ww_t[KMAX];
-    if (t < n) {
-        const size_t i = blh(d, b, c0 + t, h);
-        dtv = a.dt[i];
-        alv = a.alpha[i];
-        lmv = a.lam[i];
-        load_weights(a.wr + i * K, K, wr_t);
-        load_weights(a.ww + i * K, K, ww_t);
-    } else {
-#pragma unroll
-        for (int m = 0; m < KMAX; ++m) wr_t[m] = ww_t[m] = 0.f;
-    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -141,350 +163,389 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     const uint32_t lane_base = tmem + (uint32_t(w4 * 32) << 16);
     // TMEM: G, H, the factored Gamma and Gamma' blocks; dx_intra replaces G after the row pass
     const uint32_t colG = 0, colH = 128, colGam = 256, colGamP = 384, colX = 0;
+    if (int(blockIdx.x) < nitems) {
+        if (tid == 0) {
+            load_cbx(blockIdx.x);
+            load_dy(blockIdx.x);
+        }
+        stage_inputs(blockIdx.x);
+    }
 
-    if (tid == 0) {
-        mbar_arrive_expect_tx(&bars[0], uint32_t(2 * (N / 64) * 16384 + 2 * 16384));
-        for (int jb = 0; jb < N / 64; ++jb) {
-            tma_load_3d(sC + jb * 16384, &mapC, &bars[0], g * N + 64 * jb, c0, b);
-            tma_load_3d(sB + jb * 16384, &mapB, &bars[0], g * N + 64 * jb, c0, b);
-        }
-        tma_load_3d(sX, &mapX, &bars[0], h * P, c0, b);
-        tma_load_3d(sDY, &mapDY, &bars[0], h * P, c0, b);
-    }
-    float tmax = 0.f;
-    for (int m = 0; m < K; ++m) tmax = fmaxf(tmax, tau_s[m]);
-    const float log_cap = logf(64.f * tmax);
-    float e = 0.f;
-    if (t < n) {
-        bool cl;
-        e = token_rate(dtv, alv, lmv, log_cap, &cl);
-    }
-    const float2 Et2 = group_scan128_f2(e, wsum);  // in-chunk cumulative log-decay (hi, lo)
-    if (grp == 0) E_s[t] = Et2;
-    float l2r[KMAX];  // log2(e) / tau per mode, in registers
-    float kap_t[KMAX];
+    int kk_item = 0;
+    for (int item = blockIdx.x; item < nitems; item += gridDim.x, ++kk_item) {
+        const int ph = kk_item & 1;  // parity of this item's phase on every barrier
+        const int3 hcb = item_hcb(item);
+        const int h = hcb.x, c = hcb.y, b = hcb.z;
+        const int g = h / (d.H / d.G);
+        const int c0 = c * TQ, n = min(TQ, d.L - c0);
+        // per-position inputs of row t from the staging area, and the mode time constants
+        cp_async_wait_all();
+        __syncthreads();
+        float dtv = 1.f, alv = 1.f, lmv = 1.f;
+        float wr_t[KMAX], ww_t[KMAX], tau_r[KMAX];
 #pragma unroll
-    for (int m = 0; m < KMAX; ++m) {
-        l2r[m] = m < K ? l2t[m] : 0.f;
-        float kp = 0.f;
-        if (m < K && t < n) kp = -expm1f(-e / tau_s[m]) * ww_t[m];
-        kap_t[m] = kp;
-        if (grp == 0) {
-            wr_s[t * KMAX + m] = wr_t[m];
-            kap_s[t * KMAX + m] = kp;
-        }
-    }
-    __syncthreads();
-    // ---- Gamma below the diagonal 32 x 32 blocks, factored through the log-decay E_a at the end
-    // of the column block J (as in the forward output kernel): Gamma[t, k in J] =
-    // sum_m U_J[t, m] V[k, m] and Gamma'[t, k] = sum_m U_J[t, m] V[k, m] / tau_m, tf32 products.
-    // Operand tiles (128-byte swizzled) in the XX region: U [128 t][4 J x 8 m],
-    // V and V / tau [32 k mod 32][4 J x 8 m]; V also as fp32 in Vs for the intra dw_read.
-    unsigned char *sU = reinterpret_cast<unsigned char *>(XX), *sV = sU + 16384, *sVp = sV + 4096;
-    if (grp == 0) {
-        const int I = t >> 5;
-        unsigned char *row = sU + t * 128;
+        for (int m = 0; m < KMAX; ++m) tau_r[m] = m < K ? a.tau[h * K + m] : 1.f;
+        if (t < n) {
+            dtv = pf_f[t];
+            alv = pf_f[TQ + t];
+            lmv = pf_f[2 * TQ + t];
+            load_weights(reinterpret_cast<const bf16 *>(pf_w + t * 16), K, wr_t);
+            load_weights(reinterpret_cast<const bf16 *>(pf_w + TQ * 16 + t * 16), K, ww_t);
+        } else {
 #pragma unroll
-        for (int J = 0; J < 4; ++J) {
-            uint32_t u[8];
-            const float dE = diff_f2(Et2, E_s[32 * J + 31]);
-#pragma unroll
-            for (int m = 0; m < KMAX; ++m)
-                u[m] = (J < I && m < K && t < n) ? to_tf32(wr_t[m] * ex2_approx(-dE * l2r[m])) : 0u;
-            *reinterpret_cast<uint4 *>(row + (((2 * J) ^ (t & 7)) * 16)) = make_uint4(u[0], u[1], u[2], u[3]);
-            *reinterpret_cast<uint4 *>(row + (((2 * J + 1) ^ (t & 7)) * 16)) = make_uint4(u[4], u[5], u[6], u[7]);
+            for (int m = 0; m < KMAX; ++m) wr_t[m] = ww_t[m] = 0.f;
         }
-    } else {
-        const int J = t >> 5, r = t & 31;
-        const float dE = diff_f2(E_s[32 * J + 31], Et2);
-        uint32_t v[8], vp[8];
+        if (tid < K) {
+            const float tv = a.tau[h * K + tid];
+            tau_s[tid] = tv;
+            l2t[tid] = kLog2e / tv;
+        }
+        __syncthreads();  // the staging area is free again: the next item's inputs
+        if (item + int(gridDim.x) < nitems) stage_inputs(item + gridDim.x);
+        float tmax = 0.f;
+#pragma unroll
+        for (int m = 0; m < KMAX; ++m) tmax = fmaxf(tmax, m < K ? tau_r[m] : 0.f);
+        const float log_cap = logf(64.f * tmax);
+        float e = 0.f;
+        if (t < n) {
+            bool cl;
+            e = token_rate(dtv, alv, lmv, log_cap, &cl);
+        }
+        const float2 Et2 = group_scan128_f2(e, wsum);  // in-chunk cumulative log-decay (hi, lo)
+        if (grp == 0) E_s[t] = Et2;
+        float l2r[KMAX];  // log2(e) / tau per mode, in registers
+        float kap_t[KMAX];
 #pragma unroll
         for (int m = 0; m < KMAX; ++m) {
-            const float vv = m < K ? kap_t[m] * ex2_approx(-dE * l2r[m]) : 0.f;
-            Vs[t * KMAX + m] = vv;
-            v[m] = to_tf32(vv);
-            vp[m] = m < K ? to_tf32(vv / tau_s[m]) : 0u;
+            l2r[m] = m < K ? kLog2e / tau_r[m] : 0.f;
+            float kp = 0.f;
+            if (m < K && t < n) kp = -expm1f(-e / tau_r[m]) * ww_t[m];
+            kap_t[m] = kp;
+            if (grp == 0) {
+                wr_s[t * KMAX + m] = wr_t[m];
+                kap_s[t * KMAX + m] = kp;
+            }
         }
-        unsigned char *row = sV + r * 128, *rowp = sVp + r * 128;
-        *reinterpret_cast<uint4 *>(row + (((2 * J) ^ (r & 7)) * 16)) = make_uint4(v[0], v[1], v[2], v[3]);
-        *reinterpret_cast<uint4 *>(row + (((2 * J + 1) ^ (r & 7)) * 16)) = make_uint4(v[4], v[5], v[6], v[7]);
-        *reinterpret_cast<uint4 *>(rowp + (((2 * J) ^ (r & 7)) * 16)) = make_uint4(vp[0], vp[1], vp[2], vp[3]);
-        *reinterpret_cast<uint4 *>(rowp + (((2 * J + 1) ^ (r & 7)) * 16)) = make_uint4(vp[4], vp[5], vp[6], vp[7]);
-    }
-    fence_async_smem();
-    __syncthreads();
-    if (tid == 0) {
-        if (!mbar_wait(&bars[0], 0)) {
-            *abort_s = 1;
-        } else {
-            tc_fence_after();
-            const uint32_t idG = idesc_bf16(128, 128, false, false);
-            for (int ks = 0; ks < N / 16; ++ks) {
-                const uint32_t koff = (ks / 4) * 16384 + (ks % 4) * 32;
-                mma_bf16(tmem + colG, desc_sw128(smem_u32(sC) + koff, 16, 1024),
-                         desc_sw128(smem_u32(sB) + koff, 16, 1024), idG, ks > 0);
-            }
-            for (int ks = 0; ks < BP / 16; ++ks) {  // H = dY X^T, K = p
-                mma_bf16(tmem + colH, desc_sw128(smem_u32(sDY) + ks * 32, 16, 1024),
-                         desc_sw128(smem_u32(sX) + ks * 32, 16, 1024), idG, ks > 0);
-            }
-            const uint32_t idT = idesc_tf32(128, 32);
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+        // ---- Gamma below the diagonal 32 x 32 blocks, factored through the log-decay E_a at the end
+        // of the column block J (as in the forward output kernel): Gamma[t, k in J] =
+        // sum_m U_J[t, m] V[k, m] and Gamma'[t, k] = sum_m U_J[t, m] V[k, m] / tau_m, tf32 products.
+        // Operand tiles (128-byte swizzled) in the XX region: U [128 t][4 J x 8 m],
+        // V and V / tau [32 k mod 32][4 J x 8 m]; V also as fp32 in Vs for the intra dw_read.
+        unsigned char *sU = reinterpret_cast<unsigned char *>(XX), *sV = sU + 16384, *sVp = sV + 4096;
+        if (grp == 0) {
+            const int I = t >> 5;
+            unsigned char *row = sU + t * 128;
+#pragma unroll
             for (int J = 0; J < 4; ++J) {
-                mma_tf32(tmem + colGam + 32 * J, desc_sw128(smem_u32(sU) + 32 * J, 16, 1024),
-                         desc_sw128(smem_u32(sV) + 32 * J, 16, 1024), idT, 0);
-                mma_tf32(tmem + colGamP + 32 * J, desc_sw128(smem_u32(sU) + 32 * J, 16, 1024),
-                         desc_sw128(smem_u32(sVp) + 32 * J, 16, 1024), idT, 0);
+                uint32_t u[8];
+                const float dE = diff_f2(Et2, E_s[32 * J + 31]);
+#pragma unroll
+                for (int m = 0; m < KMAX; ++m)
+                    u[m] = (J < I && m < K && t < n) ? to_tf32(wr_t[m] * ex2_approx(-dE * l2r[m])) : 0u;
+                *reinterpret_cast<uint4 *>(row + (((2 * J) ^ (t & 7)) * 16)) = make_uint4(u[0], u[1], u[2], u[3]);
+                *reinterpret_cast<uint4 *>(row + (((2 * J + 1) ^ (t & 7)) * 16)) = make_uint4(u[4], u[5], u[6], u[7]);
             }
-            mma_commit(&bars[1]);
+        } else {
+            const int J = t >> 5, r = t & 31;
+            const float dE = diff_f2(E_s[32 * J + 31], Et2);
+            uint32_t v[8], vp[8];
+#pragma unroll
+            for (int m = 0; m < KMAX; ++m) {
+                const float vv = m < K ? kap_t[m] * ex2_approx(-dE * l2r[m]) : 0.f;
+                Vs[t * KMAX + m] = vv;
+                v[m] = to_tf32(vv);
+                vp[m] = m < K ? to_tf32(vv / tau_s[m]) : 0u;
+            }
+            unsigned char *row = sV + r * 128, *rowp = sVp + r * 128;
+            *reinterpret_cast<uint4 *>(row + (((2 * J) ^ (r & 7)) * 16)) = make_uint4(v[0], v[1], v[2], v[3]);
+            *reinterpret_cast<uint4 *>(row + (((2 * J + 1) ^ (r & 7)) * 16)) = make_uint4(v[4], v[5], v[6], v[7]);
+            *reinterpret_cast<uint4 *>(rowp + (((2 * J) ^ (r & 7)) * 16)) = make_uint4(vp[0], vp[1], vp[2], vp[3]);
+            *reinterpret_cast<uint4 *>(rowp + (((2 * J + 1) ^ (r & 7)) * 16)) = make_uint4(vp[4], vp[5], vp[6], vp[7]);
         }
-    }
-    __syncthreads();
-    if (!*abort_s && !mbar_wait(&bars[1], 0)) *abort_s = 1;
-    __syncthreads();
-    tc_fence_after();
-    // U rows as fp32 [128 t][4 J][8 m] in the x tile (free now) for the column pass, before the
-    // row pass overwrites the operand tiles with XX
-    float *Ufp = reinterpret_cast<float *>(sX);
-    if (grp == 0) {
-        const unsigned char *row = sU + t * 128;
-#pragma unroll
-        for (int c8 = 0; c8 < 8; ++c8)
-            *reinterpret_cast<uint4 *>(Ufp + t * 32 + 4 * c8) =
-                *reinterpret_cast<const uint4 *>(row + ((c8 ^ (t & 7)) * 16));
-    }
-    __syncthreads();
-    // ---- row pass (row t = this warp's row block I; group 0 takes column blocks 0, 1, group 1
-    // blocks 2, 3): Gamma o G tile, Gamma o H summed over heads in L2, Gamma' G H and G H tiles,
-    // intra dw_read.  Blocks below the diagonal take the factored Gamma from TMEM, the diagonal
-    // block sums its pairs k <= t directly, blocks above it are zero.
-    float dwr_i[KMAX];
-#pragma unroll
-    for (int m = 0; m < KMAX; ++m) dwr_i[m] = 0.f;
-    if (!*abort_s) {
-        const int I = t >> 5;
-        float *mh_row = a.mh_total + (((size_t(b) * d.nc + c) * d.G + g) * TQ + t) * TQ;
-        // 8-column work items (column block kc, eighth q8) alternate between the two groups, so
-        // that both take half of every block, the diagonal one included; loops stay rolled (the
-        // fully unrolled pass overflowed the instruction cache)
-        float acc[KMAX];
-#pragma unroll
-        for (int m = 0; m < KMAX; ++m) acc[m] = 0.f;
-#pragma unroll 1
-        for (int it = grp; it < 16; it += 2) {
-            const int kc = it >> 2, q8 = it & 3;
-            const int k0 = 32 * kc + 8 * q8;
-            unsigned char *mg = sMG + (kc >> 1) * 16384 + t * 128 + ((((kc & 1) * 4 + q8) ^ (t & 7)) * 16);
-            if (kc > I) {
-                *reinterpret_cast<uint4 *>(mg) = make_uint4(0, 0, 0, 0);
-#pragma unroll
-                for (int kk = 0; kk < 8; ++kk) XX[t * XS + k0 + kk] = 0.f;  // rows are 129 floats apart
-                continue;
-            }
-            float gv[8], hv[8];
-            tmem_ld8(lane_base + colG + k0, gv);
-            tmem_ld8(lane_base + colH + k0, hv);
-            if (kc < I) {
-                float gm[8], gp[8];
-                tmem_ld8(lane_base + colGam + k0, gm);
-                tmem_ld8(lane_base + colGamP + k0, gp);
-                tmem_ld_wait();
-#pragma unroll
-                for (int kk = 0; kk < 8; ++kk) {
-                    const int k = k0 + kk;
-                    const float gh = gv[kk] * hv[kk];
-                    XX[t * XS + k] = gp[kk] * gh;
-                    GHs[t * XS + k] = gh;
-                    const float4 v0 = *reinterpret_cast<const float4 *>(Vs + k * KMAX);
-                    const float4 v1 = *reinterpret_cast<const float4 *>(Vs + k * KMAX + 4);
-                    const float vk[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
-#pragma unroll
-                    for (int m = 0; m < KMAX; ++m) acc[m] = fmaf(vk[m], gh, acc[m]);
-                    gv[kk] *= gm[kk];  // Gamma o G
-                    hv[kk] *= gm[kk];  // Gamma o H
-                }
+        fence_async_smem();
+        __syncthreads();
+        if (tid == 0) {
+            if (!mbar_wait(&bars[0], ph) || !mbar_wait(&bars[3], ph)) {
+                *abort_s = 1;
             } else {
-                tmem_ld_wait();
+                tc_fence_after();
+                const uint32_t idG = idesc_bf16(128, 128, false, false);
+                for (int ks = 0; ks < N / 16; ++ks) {
+                    const uint32_t koff = (ks / 4) * 16384 + (ks % 4) * 32;
+                    mma_bf16(tmem + colG, desc_sw128(smem_u32(sC) + koff, 16, 1024),
+                             desc_sw128(smem_u32(sB) + koff, 16, 1024), idG, ks > 0);
+                }
+                for (int ks = 0; ks < BP / 16; ++ks) {  // H = dY X^T, K = p
+                    mma_bf16(tmem + colH, desc_sw128(smem_u32(sDY) + ks * 32, 16, 1024),
+                             desc_sw128(smem_u32(sX) + ks * 32, 16, 1024), idG, ks > 0);
+                }
+                const uint32_t idT = idesc_tf32(128, 32);
+                for (int J = 0; J < 4; ++J) {
+                    mma_tf32(tmem + colGam + 32 * J, desc_sw128(smem_u32(sU) + 32 * J, 16, 1024),
+                             desc_sw128(smem_u32(sV) + 32 * J, 16, 1024), idT, 0);
+                    mma_tf32(tmem + colGamP + 32 * J, desc_sw128(smem_u32(sU) + 32 * J, 16, 1024),
+                             desc_sw128(smem_u32(sVp) + 32 * J, 16, 1024), idT, 0);
+                }
+                mma_commit(&bars[1]);
+            }
+        }
+        __syncthreads();
+        if (!*abort_s && !mbar_wait(&bars[1], ph)) *abort_s = 1;
+        __syncthreads();
+        tc_fence_after();
+        // U rows as fp32 [128 t][4 J][8 m] in the x tile (free now) for the column pass, before the
+        // row pass overwrites the operand tiles with XX
+        float *Ufp = reinterpret_cast<float *>(sX);
+        if (grp == 0) {
+            const unsigned char *row = sU + t * 128;
 #pragma unroll
-                for (int kk = 0; kk < 8; ++kk) {
-                    const int k = k0 + kk;
-                    float gam = 0.f, gamt = 0.f, gh = 0.f;
-                    if (k <= t && t < n) {
-                        const float dE = diff_f2(Et2, E_s[k]);
-                        gh = gv[kk] * hv[kk];
+            for (int c8 = 0; c8 < 8; ++c8)
+                *reinterpret_cast<uint4 *>(Ufp + t * 32 + 4 * c8) =
+                    *reinterpret_cast<const uint4 *>(row + ((c8 ^ (t & 7)) * 16));
+        }
+        __syncthreads();
+        // ---- row pass (row t = this warp's row block I; group 0 takes column blocks 0, 1, group 1
+        // blocks 2, 3): Gamma o G tile, Gamma o H summed over heads in L2, Gamma' G H and G H tiles,
+        // intra dw_read.  Blocks below the diagonal take the factored Gamma from TMEM, the diagonal
+        // block sums its pairs k <= t directly, blocks above it are zero.
+        float dwr_i[KMAX];
+#pragma unroll
+        for (int m = 0; m < KMAX; ++m) dwr_i[m] = 0.f;
+        if (!*abort_s) {
+            const int I = t >> 5;
+            float *mh_row = a.mh_total + (((size_t(b) * d.nc + c) * d.G + g) * TQ + t) * TQ;
+            // 8-column work items (column block kc, eighth q8) alternate between the two groups, so
+            // that both take half of every block, the diagonal one included; loops stay rolled (the
+            // fully unrolled pass overflowed the instruction cache)
+            float acc[KMAX];
+#pragma unroll
+            for (int m = 0; m < KMAX; ++m) acc[m] = 0.f;
+#pragma unroll 1
+            for (int it = grp; it < 16; it += 2) {
+                const int kc = it >> 2, q8 = it & 3;
+                const int k0 = 32 * kc + 8 * q8;
+                unsigned char *mg = sMG + (kc >> 1) * 16384 + t * 128 + ((((kc & 1) * 4 + q8) ^ (t & 7)) * 16);
+                if (kc > I) {
+                    *reinterpret_cast<uint4 *>(mg) = make_uint4(0, 0, 0, 0);
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) XX[t * XS + k0 + kk] = 0.f;  // rows are 129 floats apart
+                    continue;
+                }
+                float gv[8], hv[8];
+                tmem_ld8(lane_base + colG + k0, gv);
+                tmem_ld8(lane_base + colH + k0, hv);
+                if (kc < I) {
+                    float gm[8], gp[8];
+                    tmem_ld8(lane_base + colGam + k0, gm);
+                    tmem_ld8(lane_base + colGamP + k0, gp);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) {
+                        const int k = k0 + kk;
+                        const float gh = gv[kk] * hv[kk];
+                        XX[t * XS + k] = gp[kk] * gh;
+                        GHs[t * XS + k] = gh;
+                        const float4 v0 = *reinterpret_cast<const float4 *>(Vs + k * KMAX);
+                        const float4 v1 = *reinterpret_cast<const float4 *>(Vs + k * KMAX + 4);
+                        const float vk[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+#pragma unroll
+                        for (int m = 0; m < KMAX; ++m) acc[m] = fmaf(vk[m], gh, acc[m]);
+                        gv[kk] *= gm[kk];  // Gamma o G
+                        hv[kk] *= gm[kk];  // Gamma o H
+                    }
+                } else {
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) {
+                        const int k = k0 + kk;
+                        float gam = 0.f, gamt = 0.f, gh = 0.f;
+                        if (k <= t && t < n) {
+                            const float dE = diff_f2(Et2, E_s[k]);
+                            gh = gv[kk] * hv[kk];
+#pragma unroll
+                            for (int m = 0; m < KMAX; ++m) {
+                                if (m < K) {
+                                    const float W = ex2_approx(-dE * l2r[m]);
+                                    const float kp = kap_s[k * KMAX + m];
+                                    const float aa = wr_t[m] * kp * W;
+                                    gam += aa;
+                                    gamt = fmaf(aa, l2r[m], gamt);  // times log2(e) / tau
+                                    dwr_i[m] = fmaf(kp * W, gh, dwr_i[m]);
+                                }
+                            }
+                        }
+                        gv[kk] = gam * gv[kk];
+                        hv[kk] = gam * hv[kk];
+                        XX[t * XS + k] = gamt * (1.f / kLog2e) * gh;
+                        GHs[t * XS + k] = gh;
+                    }
+                }
+                *reinterpret_cast<uint4 *>(mg) = make_uint4(pack_bf16x2(gv[0], gv[1]), pack_bf16x2(gv[2], gv[3]),
+                                                            pack_bf16x2(gv[4], gv[5]), pack_bf16x2(gv[6], gv[7]));
+                if (t < n && k0 <= t) {
+                    atomicAdd(reinterpret_cast<float4 *>(mh_row + k0), make_float4(hv[0], hv[1], hv[2], hv[3]));
+                    if (k0 + 4 <= t)
+                        atomicAdd(reinterpret_cast<float4 *>(mh_row + k0 + 4), make_float4(hv[4], hv[5], hv[6], hv[7]));
+                }
+                if (kc < I && q8 >= 2) {  // this thread's last item of the factored block kc
+                    const float dE = diff_f2(Et2, E_s[32 * kc + 31]);
+#pragma unroll
+                    for (int m = 0; m < KMAX; ++m) {
+                        if (m < K) dwr_i[m] = fmaf(ex2_approx(-dE * l2r[m]), acc[m], dwr_i[m]);
+                        acc[m] = 0.f;
+                    }
+                }
+            }
+            if (grp == 1) {
+#pragma unroll
+                for (int m = 0; m < KMAX; ++m) part[t * KMAX + m] = dwr_i[m];
+            }
+        }
+        fence_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+        if (!*abort_s && grp == 0 && t < n) {
+            float *o = a.dwr_acc + blh(d, b, c0 + t, h) * K;
+#pragma unroll
+            for (int m = 0; m < KMAX; ++m)
+                if (m < K) o[m] = dwr_i[m] + part[t * KMAX + m];
+        }
+        if (tid == 0 && !*abort_s) {  // dx_intra = (Gamma o G)^T dY: M = k, N = p, K = t
+            const uint32_t idX = idesc_bf16(128, BP, true, true);
+            for (int ks = 0; ks < TQ / 16; ++ks)
+                mma_bf16(tmem + colX, desc_sw128(smem_u32(sMG) + ks * 2048, 16384, 1024),
+                         desc_sw128(smem_u32(sDY) + ks * 2048, 16384, 1024), idX, ks > 0);
+            mma_commit(&bars[2]);
+        }
+        __syncthreads();  // part[] is reused below
+        // ---- column pass (group g takes the rows of parity g of column k): intra dkappa.  Rows of
+        // later blocks use the factored form exp(-(E_a - E_k)/tau) sum_t U_J[t, m] G H[t, k]; rows of
+        // the diagonal block (t >= k) sum directly.  Column block J has 128 - 32 J rows, so group 1's
+        // warp w takes block 3 - w: every SM sub-partition gets blocks J and 3 - J.
+        const int kcol = grp == 0 ? t : (((3 - (t >> 5)) << 5) | (t & 31));
+        float dk[KMAX];
+#pragma unroll
+        for (int m = 0; m < KMAX; ++m) dk[m] = 0.f;
+        if (!*abort_s) {
+            const int k = kcol, J = k >> 5;
+            const float2 Ek = E_s[k];
+            float dk2[KMAX];
+#pragma unroll
+            for (int m = 0; m < KMAX; ++m) dk2[m] = 0.f;
+            const int dend = min(n, 32 * J + 32);
+            for (int tt0 = 32 * J + grp; tt0 < dend; tt0 += 8) {
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int tt = tt0 + 2 * u;
+                    if (tt < dend && tt >= k) {
+                        const float dE = diff_f2(E_s[tt], Ek);
+                        const float gh = GHs[tt * XS + k];
 #pragma unroll
                         for (int m = 0; m < KMAX; ++m) {
                             if (m < K) {
-                                const float W = ex2_approx(-dE * l2r[m]);
-                                const float kp = kap_s[k * KMAX + m];
-                                const float aa = wr_t[m] * kp * W;
-                                gam += aa;
-                                gamt = fmaf(aa, l2r[m], gamt);  // times log2(e) / tau
-                                dwr_i[m] = fmaf(kp * W, gh, dwr_i[m]);
+                                const float v = wr_s[tt * KMAX + m] * ex2_approx(-dE * l2r[m]);
+                                if (u & 1)
+                                    dk2[m] = fmaf(v, gh, dk2[m]);
+                                else
+                                    dk[m] = fmaf(v, gh, dk[m]);
                             }
                         }
                     }
-                    gv[kk] = gam * gv[kk];
-                    hv[kk] = gam * hv[kk];
-                    XX[t * XS + k] = gamt * (1.f / kLog2e) * gh;
-                    GHs[t * XS + k] = gh;
                 }
             }
-            *reinterpret_cast<uint4 *>(mg) = make_uint4(pack_bf16x2(gv[0], gv[1]), pack_bf16x2(gv[2], gv[3]),
-                                                        pack_bf16x2(gv[4], gv[5]), pack_bf16x2(gv[6], gv[7]));
-            if (t < n && k0 <= t) {
-                atomicAdd(reinterpret_cast<float4 *>(mh_row + k0), make_float4(hv[0], hv[1], hv[2], hv[3]));
-                if (k0 + 4 <= t)
-                    atomicAdd(reinterpret_cast<float4 *>(mh_row + k0 + 4), make_float4(hv[4], hv[5], hv[6], hv[7]));
-            }
-            if (kc < I && q8 >= 2) {  // this thread's last item of the factored block kc
-                const float dE = diff_f2(Et2, E_s[32 * kc + 31]);
+            float s0[KMAX], s1[KMAX];
 #pragma unroll
-                for (int m = 0; m < KMAX; ++m) {
-                    if (m < K) dwr_i[m] = fmaf(ex2_approx(-dE * l2r[m]), acc[m], dwr_i[m]);
-                    acc[m] = 0.f;
-                }
-            }
-        }
-        if (grp == 1) {
+            for (int m = 0; m < KMAX; ++m) s0[m] = s1[m] = 0.f;
+            for (int tt0 = 32 * J + 32 + grp; tt0 < n; tt0 += 8) {
 #pragma unroll
-            for (int m = 0; m < KMAX; ++m) part[t * KMAX + m] = dwr_i[m];
-        }
-    }
-    fence_async_smem();
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    if (!*abort_s && grp == 0 && t < n) {
-        float *o = a.dwr_acc + blh(d, b, c0 + t, h) * K;
+                for (int u = 0; u < 4; ++u) {
+                    const int tt = tt0 + 2 * u;
+                    if (tt < n) {
+                        const float gh = GHs[tt * XS + k];
+                        const float4 u0 = *reinterpret_cast<const float4 *>(Ufp + tt * 32 + 8 * J);
+                        const float4 u1 = *reinterpret_cast<const float4 *>(Ufp + tt * 32 + 8 * J + 4);
+                        const float uu[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
 #pragma unroll
-        for (int m = 0; m < KMAX; ++m)
-            if (m < K) o[m] = dwr_i[m] + part[t * KMAX + m];
-    }
-    if (tid == 0 && !*abort_s) {  // dx_intra = (Gamma o G)^T dY: M = k, N = p, K = t
-        const uint32_t idX = idesc_bf16(128, BP, true, true);
-        for (int ks = 0; ks < TQ / 16; ++ks)
-            mma_bf16(tmem + colX, desc_sw128(smem_u32(sMG) + ks * 2048, 16384, 1024),
-                     desc_sw128(smem_u32(sDY) + ks * 2048, 16384, 1024), idX, ks > 0);
-        mma_commit(&bars[2]);
-    }
-    __syncthreads();  // part[] is reused below
-    // ---- column pass (group g takes the rows of parity g of column k): intra dkappa.  Rows of
-    // later blocks use the factored form exp(-(E_a - E_k)/tau) sum_t U_J[t, m] G H[t, k]; rows of
-    // the diagonal block (t >= k) sum directly.  Column block J has 128 - 32 J rows, so group 1's
-    // warp w takes block 3 - w: every SM sub-partition gets blocks J and 3 - J.
-    const int kcol = grp == 0 ? t : (((3 - (t >> 5)) << 5) | (t & 31));
-    float dk[KMAX];
-#pragma unroll
-    for (int m = 0; m < KMAX; ++m) dk[m] = 0.f;
-    if (!*abort_s) {
-        const int k = kcol, J = k >> 5;
-        const float2 Ek = E_s[k];
-        float dk2[KMAX];
-#pragma unroll
-        for (int m = 0; m < KMAX; ++m) dk2[m] = 0.f;
-        const int dend = min(n, 32 * J + 32);
-        for (int tt0 = 32 * J + grp; tt0 < dend; tt0 += 8) {
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int tt = tt0 + 2 * u;
-                if (tt < dend && tt >= k) {
-                    const float dE = diff_f2(E_s[tt], Ek);
-                    const float gh = GHs[tt * XS + k];
-#pragma unroll
-                    for (int m = 0; m < KMAX; ++m) {
-                        if (m < K) {
-                            const float v = wr_s[tt * KMAX + m] * ex2_approx(-dE * l2r[m]);
+                        for (int m = 0; m < KMAX; ++m) {
                             if (u & 1)
-                                dk2[m] = fmaf(v, gh, dk2[m]);
+                                s1[m] = fmaf(uu[m], gh, s1[m]);
                             else
-                                dk[m] = fmaf(v, gh, dk[m]);
+                                s0[m] = fmaf(uu[m], gh, s0[m]);
                         }
                     }
                 }
             }
-        }
-        float s0[KMAX], s1[KMAX];
+            const float dEa = diff_f2(E_s[32 * J + 31], Ek);
 #pragma unroll
-        for (int m = 0; m < KMAX; ++m) s0[m] = s1[m] = 0.f;
-        for (int tt0 = 32 * J + 32 + grp; tt0 < n; tt0 += 8) {
+            for (int m = 0; m < KMAX; ++m) {
+                dk[m] += dk2[m];
+                if (m < K) dk[m] = fmaf(ex2_approx(-dEa * l2r[m]), s0[m] + s1[m], dk[m]);
+            }
+            if (grp == 1) {
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int tt = tt0 + 2 * u;
-                if (tt < n) {
-                    const float gh = GHs[tt * XS + k];
-                    const float4 u0 = *reinterpret_cast<const float4 *>(Ufp + tt * 32 + 8 * J);
-                    const float4 u1 = *reinterpret_cast<const float4 *>(Ufp + tt * 32 + 8 * J + 4);
-                    const float uu[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
-#pragma unroll
-                    for (int m = 0; m < KMAX; ++m) {
-                        if (u & 1)
-                            s1[m] = fmaf(uu[m], gh, s1[m]);
-                        else
-                            s0[m] = fmaf(uu[m], gh, s0[m]);
-                    }
-                }
+                for (int m = 0; m < KMAX; ++m) part[k * KMAX + m] = dk[m];
             }
         }
-        const float dEa = diff_f2(E_s[32 * J + 31], Ek);
-#pragma unroll
-        for (int m = 0; m < KMAX; ++m) {
-            dk[m] += dk2[m];
-            if (m < K) dk[m] = fmaf(ex2_approx(-dEa * l2r[m]), s0[m] + s1[m], dk[m]);
+        // exclusive row prefix of XX (row t): group 0 over j in [0, 64) (its total in xtot), group 1
+        // over [64, 128) starting from 0; the column sums below add the suffix sum of xtot for the
+        // columns j >= 64
+        float *xtot = Vs;  // [128], free after the row pass
+        if (!*abort_s) {
+            float run = 0.f;
+            for (int j = 64 * grp; j < 64 * grp + 64; ++j) {
+                const float v = XX[t * XS + j];
+                XX[t * XS + j] = run;
+                run += v;
+            }
+            if (grp == 0) xtot[t] = run;
         }
-        if (grp == 1) {
-#pragma unroll
-            for (int m = 0; m < KMAX; ++m) part[k * KMAX + m] = dk[m];
+        __syncthreads();
+        // rect[j] = sum_{t' >= j} sum_{k < j} X[t', k]: column j's suffix sum of the row prefixes,
+        // rows of parity g in group g (column kcol, the column pass's balanced assignment)
+        float *rpart = Vs + TQ;  // [128] group 1's partial rect
+        float sr = 0.f;
+        if (!*abort_s) {
+            const int j = kcol;
+            for (int tp = j + ((j + grp) & 1); tp < n; tp += 2) {
+                sr += XX[tp * XS + j];
+                if (j >= 64) sr += xtot[tp];
+            }
         }
-    }
-    // exclusive row prefix of XX (row t): group 0 over j in [0, 64) (its total in xtot), group 1
-    // over [64, 128) starting from 0; the column sums below add the suffix sum of xtot for the
-    // columns j >= 64
-    float *xtot = Vs;  // [128], free after the row pass
-    if (!*abort_s) {
-        float run = 0.f;
-        for (int j = 64 * grp; j < 64 * grp + 64; ++j) {
-            const float v = XX[t * XS + j];
-            XX[t * XS + j] = run;
-            run += v;
-        }
-        if (grp == 0) xtot[t] = run;
-    }
-    __syncthreads();
-    // rect[j] = sum_{t' >= j} sum_{k < j} X[t', k]: column j's suffix sum of the row prefixes,
-    // rows of parity g in group g (column kcol, the column pass's balanced assignment)
-    float *rpart = Vs + TQ;  // [128] group 1's partial rect
-    float sr = 0.f;
-    if (!*abort_s) {
-        const int j = kcol;
-        for (int tp = j + ((j + grp) & 1); tp < n; tp += 2) {
-            sr += XX[tp * XS + j];
-            if (j >= 64) sr += xtot[tp];
-        }
-    }
-    if (grp == 1) rpart[kcol] = sr;
-    __syncthreads();
-    if (!*abort_s && grp == 0 && t < n) {
-        float *o = a.dkap_acc + blh(d, b, c0 + t, h) * K;
+        if (grp == 1) rpart[kcol] = sr;
+        __syncthreads();  // G H (in the C / B region) and the U copy (in the x tile) are read
+        if (tid == 0 && !*abort_s && item + int(gridDim.x) < nitems) load_cbx(item + gridDim.x);
+        if (!*abort_s && grp == 0 && t < n) {
+            float *o = a.dkap_acc + blh(d, b, c0 + t, h) * K;
 #pragma unroll
-        for (int m = 0; m < KMAX; ++m)
-            if (m < K) o[m] = dk[m] + part[t * KMAX + m];
-        a.rect[blh(d, b, c0 + t, h)] = sr + rpart[t];
-    }
-    __syncthreads();
-    if (!*abort_s && !mbar_wait(&bars[2], 0)) *abort_s = 1;
-    __syncthreads();
-    tc_fence_after();
-    {  // dx_intra row: group g takes columns [32 g, 32 g + 32) (nothing written after an abort)
-        float v[32];
-        tmem_ld32(lane_base + colX + grp * 32, v);
-        tmem_ld_wait();
-        uint4 e[8];
+            for (int m = 0; m < KMAX; ++m)
+                if (m < K) o[m] = dk[m] + part[t * KMAX + m];
+            a.rect[blh(d, b, c0 + t, h)] = sr + rpart[t];
+        }
+        __syncthreads();
+        if (!*abort_s && !mbar_wait(&bars[2], ph)) *abort_s = 1;
+        __syncthreads();
+        tc_fence_after();
+        if (tid == 0 && !*abort_s && item + int(gridDim.x) < nitems) load_dy(item + gridDim.x);
+        {  // dx_intra row: group g takes columns [32 g, 32 g + 32) (nothing written after an abort)
+            float v[32];
+            tmem_ld32(lane_base + colX + grp * 32, v);
+            tmem_ld_wait();
+            uint4 e[8];
 #pragma unroll
-        for (int q = 0; q < 8; ++q) e[q] = f4_bits(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-        const int t8 = t & ~7;
-        put_rows<8, false>(e, reinterpret_cast<unsigned char *>(a.dx_acc + blh(d, b, c0 + t8, h) * P + grp * 32),
-                           size_t(d.H) * P * 4, *abort_s ? 0 : n - t8);
-    }
+            for (int q = 0; q < 8; ++q) e[q] = f4_bits(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            const int t8 = t & ~7;
+            put_rows<8, false>(e, reinterpret_cast<unsigned char *>(a.dx_acc + blh(d, b, c0 + t8, h) * P + grp * 32),
+                               size_t(d.H) * P * 4, *abort_s ? 0 : n - t8);
+        }
+        tc_fence_before();
+        __syncthreads();  // this item's TMEM reads are done before the next item's MMAs
+        if (*abort_s) break;
+    }  // items
+    cp_async_wait_all();
     if (*abort_s && tid == 0) atomicExch(a.err, kTimeoutCode);
     tc_fence_before();
     __syncthreads();
@@ -1144,12 +1205,20 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
     a.ddt = p.ddt; a.dalpha = p.dalpha; a.dlam = p.dlam; a.dD = p.dD;
     a.err = err;
     a.hg = pick_hg(d);
+    {
+        int dev = 0, nsm = 0;
+        if ((e = cudaGetDevice(&dev)) || (e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)))
+            return e;
+        a.pf_sms = std::max(nsm, 1);
+    }
 
     {
         const size_t smem = IntraSmem().total + 1024;
         cudaFuncSetAttribute(tc_bwd_intra, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
         trace_begin("bwd_intra_tc", st);
-        tc_bwd_intra<<<dim3(d.H, d.nc, d.B), kIntraThreads, smem, st>>>(mapC, mapB, mapX, mapDY, a);
+        // persistent: one CTA per SM (shared memory), items (h, c, b) strided by the grid
+        const int items = d.H * d.nc * d.B;
+        tc_bwd_intra<<<std::min(items, a.pf_sms), kIntraThreads, smem, st>>>(mapC, mapB, mapX, mapDY, a);
         trace_end(st);
         if ((e = cudaGetLastError())) return e;
     }

@@ -121,6 +121,25 @@ __device__ __forceinline__ void get_rows(uint4 (&e)[NL], const unsigned char *ro
     lane_transpose<NL>(e, lane);
 }
 
+// Asynchronous global -> shared copies (cp.async, no register round trip): 4, 8 or 16 bytes,
+// both addresses aligned to the size; completed by cp_async_wait_all.
+__device__ __forceinline__ void cp_async4(void *dst, const void *src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
+                 "l"(src)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_bytes(void *dst, const void *src, int bytes) {
+    const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst));
+    if (bytes == 16)
+        asm volatile("cp.async.ca.shared.global [%0], [%1], 16;" ::"r"(d), "l"(src) : "memory");
+    else if (bytes == 8)
+        asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(d), "l"(src) : "memory");
+    else
+        asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(d), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
 // Inclusive prefix sum (double) of one value per thread over a 128-thread block.
 __device__ __forceinline__ double block_scan128(double v, double *wsum) {
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
