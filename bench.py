@@ -145,11 +145,12 @@ def kpn(s):
 # only while the kernel's sources hash to the digest they had when they were profiled.
 PROFILED_TRAFFIC_BATCH = 2
 PROFILED_TRAFFIC = {
-    "state_pass_fwd_tc": ("scan_tc.cu", "3d8105d2c52b5180", 85.136e6 + 481.196e6),
-    "chunk_fwd_tc": ("scan_tc.cu", "3d8105d2c52b5180", 631.424e6 + 59.975e6),
-    "state_pass_rev_tc": ("scan_tc.cu", "3d8105d2c52b5180", 87.261e6 + 481.387e6),
-    "bwd_intra_tc": ("scan_tc_bwd.cu", "cde6c695d8150f7c", 164.243e6 + 185.976e6),
-    "bwd_state_tc": ("scan_tc_bwd.cu", "cde6c695d8150f7c", 1462.450e6 + 173.401e6),
+    "coef_tc": ("scan_tc.cu", "3001ce054be74299", 23.103e6 + 9.001e6),
+    "state_pass_fwd_tc": ("scan_tc.cu", "3001ce054be74299", 137.495e6 + 477.948e6),
+    "chunk_fwd_tc": ("scan_tc.cu", "3001ce054be74299", 631.333e6 + 59.839e6),
+    "state_pass_rev_tc": ("scan_tc.cu", "3001ce054be74299", 137.340e6 + 478.024e6),
+    "bwd_intra_tc": ("scan_tc_bwd.cu", "d5477e9b592f55e7", 164.034e6 + 123.074e6),
+    "bwd_state_tc": ("scan_tc_bwd.cu", "d5477e9b592f55e7", 1461.271e6 + 172.064e6),
 }
 
 
@@ -189,6 +190,10 @@ def algorithmic_work(kernel: str, s, per_launch_units: float):
         return "flops", (8 * kpn(s) + 4 * q * s.dstate * s.ngroups / s.nheads) * per_launch_units
     if kernel == "bwd_intra_tc":
         return "flops", (2 * q * s.headdim + q * s.dstate * s.ngroups / s.nheads) * per_launch_units
+    if kernel == "coef_tc":  # dt, alpha, lam, w_read, w_write in; f, s, u, exp(-E/tau) out
+        return "bytes", (12 + 4 * s.nmodes + 16 * s.nmodes) * per_launch_units
+    if kernel == "bwd_final_tc":  # per-position terms, dx_acc, dy, x in; dx and the scalar grads out
+        return "bytes", (36 + 14 * s.nmodes + 10 * s.headdim) * per_launch_units
     if kernel == "decode_step":
         return "bytes", 2.0 * 4 * kpn(s) * per_launch_units
     return None, None
