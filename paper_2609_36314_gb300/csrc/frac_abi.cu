@@ -107,7 +107,7 @@ frac_status plan(const frac_dims *d, frac::ScanDims *sd, int *path, bool backwar
 constexpr size_t kStatusBytes = kAlign;
 
 struct FwdLayout {
-    size_t s_in, coef, total;
+    size_t s_in, coef, ek, total;
 };
 struct BwdLayout {
     size_t s_in, ds_out, db, dc, total;
@@ -119,7 +119,8 @@ FwdLayout fwd_layout(const frac_dims *d, const frac::ScanDims &sd, int path) {
     const size_t elems = path == PATH_TC ? frac::tc_state_elems(sd) : frac::simt_state_elems(sd);
     const size_t esz = path == PATH_TC ? 2 : elem(d);
     l.coef = kStatusBytes + round_up(elems * esz);  // tensor-core path: per-position coefficients
-    l.total = l.coef + (path == PATH_TC ? round_up(frac::tc_coef_elems(sd) * 4) : 0);
+    l.ek = l.coef + (path == PATH_TC ? round_up(frac::tc_coef_elems(sd) * 4) : 0);
+    l.total = l.ek + (path == PATH_TC ? round_up(frac::tc_ek_elems(sd) * 4) : 0);
     return l;
 }
 
@@ -255,7 +256,7 @@ frac_status frac_scan_fwd(const frac_dims *d, const void *x, const float *dt, co
     if (e == cudaSuccess) {
         if (path == PATH_TC)
             e = frac::tc_scan_fwd(sd, p, ws + l.s_in, reinterpret_cast<float *>(ws + l.coef),
-                                  reinterpret_cast<int *>(ws), st);
+                                  reinterpret_cast<float *>(ws + l.ek), reinterpret_cast<int *>(ws), st);
         else
             e = frac::simt_scan_fwd(sd, d->dtype, p, ws + l.s_in, st);
     }

@@ -54,11 +54,15 @@ cudaError_t simt_scan_bwd(const ScanDims &d, int dtype, const ScanPtrs &p, void 
 bool tc_supported(const ScanDims &d, int dtype);
 size_t tc_state_elems(const ScanDims &d);  // bf16 elements of the per-chunk state workspace
 size_t tc_coef_elems(const ScanDims &d);   // float elements of the per-position coefficients
+// floats per position of the {E hi, E lo, 0, 0, kappa[K]} array (padded to 16 bytes x 2^i)
+__host__ __device__ inline int tc_ek_width(int K) { return K == 8 ? 16 : 8; }
+size_t tc_ek_elems(const ScanDims &d);
 // coef: [B, L, H, 4, K] float (f, s, u, exp(-E/tau) per position), written by the forward
-cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, float *coef, int *err,
-                        cudaStream_t st);
+cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, float *coef, float *ek,
+                        int *err, cudaStream_t st);
 // Per-position mode coefficients of every chunk (the first kernel of both passes).
-cudaError_t tc_coef_launch(const ScanDims &d, const ScanPtrs &p, float *coef, cudaStream_t st);
+// ek: [B, L, H, tc_ek_width(K)] float: the in-chunk cumulative log-decay E (hi, lo) and kappa
+cudaError_t tc_coef_launch(const ScanDims &d, const ScanPtrs &p, float *coef, float *ek, cudaStream_t st);
 // Chunk-serial state pass on the tensor cores (forward: U = x, V = B, coefficients s; reverse:
 // U = dy, V = C, coefficients f).
 cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, const void *V,
@@ -74,6 +78,7 @@ struct TcBwdWorkspace {  // S_in and coef first, at the offsets the forward uses
     float *dx_acc, *dwr_acc, *dkap_acc;      // [B,L,H,P], [B,L,H,K] x 2
     float *ab_acc, *rect, *cdot, *mh_total;  // [B,L,H,2], [B,L,H], [B,H,nc,K], [B,nc,G,Q,Q]
     float *coef;                             // [B,L,H,4,K]: f, s, u, exp(-E/tau)
+    float *ek;                               // [B,L,H,tc_ek_width(K)]: E (hi, lo), kappa
     float *dB_acc, *dC_acc;                  // [B,L,G,N] x 2
 };
 size_t tc_bwd_workspace_bytes(const ScanDims &d, TcBwdWorkspace *layout, char *base);

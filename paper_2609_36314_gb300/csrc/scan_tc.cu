@@ -54,11 +54,14 @@ struct StateArgs {
 // kappa = (1 - exp(-e_t/tau)) w_write,
 //   f = w_read exp(-E_t/tau)   s = kappa u   u = exp(-(E_end - E_t)/tau)   d = exp(-E_t/tau)
 // stored as coef[b, t, h, {f, s, u, d}, K].  d at the chunk's last position is the chunk decay.
+// E_t (as the float pair hi + lo) and kappa go to a second array ek[b, t, h, :] for the kernels
+// that evaluate pairwise decays (the forward output and the intra-chunk backward).
 struct CoefArgs {
     ScanDims d;
     const bf16 *wr, *ww;
     const float *dt, *alpha, *lam, *tau;
     float *coef;
+    float *ek;  // per position {E hi, E lo, 0, 0, kappa[K], 0 ...}: tc_ek_width(K) floats
 };
 
 template <int KK>
@@ -90,13 +93,14 @@ __global__ void __launch_bounds__(TQ) tc_coef(CoefArgs a) {
     if (t == n - 1) Eend_s = Et;
     __syncthreads();
     const float dEnd = diff_f2(Eend_s, Et);  // E_end - E_t >= 0
-    float f[KK], s[KK], u[KK], dv[KK];
+    float f[KK], s[KK], u[KK], dv[KK], kp[KK];
 #pragma unroll
     for (int m = 0; m < KK; ++m) {
         dv[m] = ex2_approx(-Et.x * l2t[m]);
         u[m] = ex2_approx(-dEnd * l2t[m]);
         f[m] = wr[m] * dv[m];
-        s[m] = -expm1f(-e * itau[m]) * ww[m] * u[m];
+        kp[m] = -expm1f(-e * itau[m]) * ww[m];
+        s[m] = kp[m] * u[m];
     }
     // row t: KK / 4 pieces of each kind, written row-coalesced across KK-lane groups
     uint4 pc[KK];
@@ -110,6 +114,17 @@ __global__ void __launch_bounds__(TQ) tc_coef(CoefArgs a) {
     const int tg = t & ~(KK - 1);
     put_rows<KK, false>(pc, reinterpret_cast<unsigned char *>(a.coef + blh(d, b, c0 + tg, h) * 4 * KK),
                         size_t(d.H) * 4 * KK * 4, n - tg);
+    // ek row: {E hi, E lo, 0, 0}, kappa in KK / 4 pieces, zero padding (EK / 4 pieces in all)
+    constexpr int EK = KK == 8 ? 16 : 8;
+    uint4 pe[EK / 4];
+    pe[0] = f4_bits(Et.x, Et.y, 0.f, 0.f);
+#pragma unroll
+    for (int q = 0; q < KK / 4; ++q) pe[1 + q] = f4_bits(kp[4 * q], kp[4 * q + 1], kp[4 * q + 2], kp[4 * q + 3]);
+#pragma unroll
+    for (int q = 1 + KK / 4; q < EK / 4; ++q) pe[q] = make_uint4(0, 0, 0, 0);
+    const int te = t & ~(EK / 4 - 1);
+    put_rows<EK / 4, false>(pe, reinterpret_cast<unsigned char *>(a.ek + blh(d, b, c0 + te, h) * EK),
+                            size_t(d.H) * EK * 4, n - te);
 }
 
 // Shared-memory plan of tc_state_pass (offsets from a 1024-aligned base): about 70 KB at N = 128,
@@ -338,6 +353,7 @@ __global__ void __launch_bounds__(kThreads, 3)
 // ---------------------------------------------------------------------------------------------
 struct OutArgs {
     ScanDims d;
+    const float *coef, *ek;  // tc_coef's per-position coefficients and {E, kappa}
     const bf16 *wr, *ww;
     const float *dt, *alpha, *lam, *tau, *D;
     bf16 *y;
@@ -469,19 +485,49 @@ __global__ void __launch_bounds__(kOutLaunch, 2)
         l2t[tid] = kLog2e / tv;
     }
     if (tid < 32) tmem_alloc_once(tslot, 256);
-    // per-position inputs of row t, all loads issued before anything waits on them
-    float dtv = 1.f, alv = 1.f, lmv = 1.f;
-    float wr_t[KMAX], ww_t[KMAX];
-    if (t < n) {
-        const size_t i = blh(d, b, c0 + t, h);
-        dtv = a.dt[i];
-        alv = a.alpha[i];
-        lmv = a.lam[i];
-        load_weights(a.wr + i * K, K, wr_t);
-        load_weights(a.ww + i * K, K, ww_t);
-    } else {
+    // per-position inputs of row t, all loads issued before anything waits on them: w_read, and
+    // from tc_coef the cumulative log-decay E (hi, lo), kappa and f = w_read exp(-E/tau) (rows
+    // read row-coalesced; rows t >= n read as zero)
+    float wr_t[KMAX], kap_t[KMAX], f_t[KMAX];
+    float2 Et2;
+    {
+        if (t < n)
+            load_weights(a.wr + blh(d, b, c0 + t, h) * K, K, wr_t);
+        else
 #pragma unroll
-        for (int m = 0; m < KMAX; ++m) wr_t[m] = ww_t[m] = 0.f;
+            for (int m = 0; m < KMAX; ++m) wr_t[m] = 0.f;
+        auto fl = [](uint4 v, float *o) {
+            o[0] = __uint_as_float(v.x);
+            o[1] = __uint_as_float(v.y);
+            o[2] = __uint_as_float(v.z);
+            o[3] = __uint_as_float(v.w);
+        };
+        if (K == 8) {
+            uint4 pe[4], pf[2];
+            get_rows<4>(pe, reinterpret_cast<const unsigned char *>(a.ek + blh(d, b, c0 + (t & ~3), h) * 16),
+                        size_t(d.H) * 64, n - (t & ~3));
+            get_rows<2>(pf, reinterpret_cast<const unsigned char *>(a.coef + blh(d, b, c0 + (t & ~1), h) * 32),
+                        size_t(d.H) * 128, n - (t & ~1));
+            Et2 = make_float2(__uint_as_float(pe[0].x), __uint_as_float(pe[0].y));
+            fl(pe[1], kap_t);
+            fl(pe[2], kap_t + 4);
+            // past the end of a ragged chunk E stays at its last value (zero token rates)
+            if (t >= n) Et2 = *reinterpret_cast<const float2 *>(a.ek + blh(d, b, c0 + n - 1, h) * 16);
+            fl(pf[0], f_t);
+            fl(pf[1], f_t + 4);
+        } else {  // K == 4
+            uint4 pe[2], pf[1];
+            get_rows<2>(pe, reinterpret_cast<const unsigned char *>(a.ek + blh(d, b, c0 + (t & ~1), h) * 8),
+                        size_t(d.H) * 32, n - (t & ~1));
+            get_rows<1>(pf, reinterpret_cast<const unsigned char *>(a.coef + blh(d, b, c0 + t, h) * 16),
+                        size_t(d.H) * 64, n - t);
+            Et2 = make_float2(__uint_as_float(pe[0].x), __uint_as_float(pe[0].y));
+            fl(pe[1], kap_t);
+            fl(pf[0], f_t);
+            if (t >= n) Et2 = *reinterpret_cast<const float2 *>(a.ek + blh(d, b, c0 + n - 1, h) * 8);
+#pragma unroll
+            for (int m = 4; m < KMAX; ++m) kap_t[m] = f_t[m] = 0.f;
+        }
     }
     tc_fence_before();
     __syncthreads();
@@ -503,27 +549,10 @@ __global__ void __launch_bounds__(kOutLaunch, 2)
         }
         tma_load_3d(sX, &mapX, &bars[0], h * P, c0, b);
     }
-    float tmax = 0.f;
-    for (int m = 0; m < K; ++m) tmax = fmaxf(tmax, tau_s[m]);
-    const float log_cap = logf(64.f * tmax);
-    float e = 0.f;
-    if (t < n) {
-        bool cl;
-        e = token_rate(dtv, alv, lmv, log_cap, &cl);
-    }
-    const float2 Et2 = group_scan128_f2<true>(e, wsum);  // in-chunk cumulative log-decay (hi, lo)
-    if (grp == 0) E_s[t] = Et2;
-    float f_t[KMAX], kap_t[KMAX];
+    if (grp == 0) {
+        E_s[t] = Et2;
 #pragma unroll
-    for (int m = 0; m < KMAX; ++m) {
-        f_t[m] = kap_t[m] = 0.f;
-        if (m < K) {
-            if (t < n) {
-                kap_t[m] = -expm1f(-e / tau_s[m]) * ww_t[m];
-                f_t[m] = wr_t[m] * ex2_approx(-Et2.x * l2t[m]);
-            }
-            if (grp == 0) kap_s[t * KMAX + m] = kap_t[m];
-        }
+        for (int m = 0; m < KMAX; ++m) kap_s[t * KMAX + m] = kap_t[m];
     }
     sync_first256();
     // Gamma below the diagonal 32 x 32 blocks, factored through the log-decay E_a at the end of
@@ -736,7 +765,9 @@ size_t tc_state_elems(const ScanDims &d) {
 
 size_t tc_coef_elems(const ScanDims &d) { return size_t(d.B) * d.L * d.H * 4 * d.K; }
 
-cudaError_t tc_coef_launch(const ScanDims &d, const ScanPtrs &p, float *coef, cudaStream_t st) {
+size_t tc_ek_elems(const ScanDims &d) { return size_t(d.B) * d.L * d.H * tc_ek_width(d.K); }
+
+cudaError_t tc_coef_launch(const ScanDims &d, const ScanPtrs &p, float *coef, float *ek, cudaStream_t st) {
     if (d.nc == 0) return cudaSuccess;
     CoefArgs a;
     a.d = d;
@@ -744,6 +775,7 @@ cudaError_t tc_coef_launch(const ScanDims &d, const ScanPtrs &p, float *coef, cu
     a.ww = (const bf16 *)p.ww;
     a.dt = p.dt; a.alpha = p.alpha; a.lam = p.lam; a.tau = p.tau;
     a.coef = coef;
+    a.ek = ek;
     trace_begin("coef_tc", st);
     if (d.K == 8)
         tc_coef<8><<<dim3(d.H, d.nc, d.B), TQ, 0, st>>>(a);
@@ -789,9 +821,9 @@ cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, con
     return cudaGetLastError();
 }
 
-cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, float *coef, int *err,
-                        cudaStream_t st) {
-    cudaError_t e = tc_coef_launch(d, p, coef, st);
+cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, float *coef, float *ek,
+                        int *err, cudaStream_t st) {
+    cudaError_t e = tc_coef_launch(d, p, coef, ek, st);
     if (e == cudaSuccess) e = tc_state_pass_launch(d, false, p.x, p.Bm, coef, p.h0, S_in, p.h_final, err, st);
     if (e != cudaSuccess || d.nc == 0) return e;
     CUtensorMap mapC, mapB, mapX, mapS;
@@ -804,6 +836,8 @@ cudaError_t tc_scan_fwd(const ScanDims &d, const ScanPtrs &p, void *S_in, float 
         return cudaErrorInvalidValue;
     OutArgs a;
     a.d = d;
+    a.coef = coef;
+    a.ek = ek;
     a.wr = (const bf16 *)p.wr;
     a.ww = (const bf16 *)p.ww;
     a.dt = p.dt; a.alpha = p.alpha; a.lam = p.lam; a.tau = p.tau; a.D = p.D;

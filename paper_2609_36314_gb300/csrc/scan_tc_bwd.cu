@@ -46,6 +46,7 @@ struct BwdArgs {
     const bf16 *S_in, *dS_out;
     float *dx_acc, *dwr_acc, *dkap_acc, *ab_acc, *rect, *cdot, *mh_total, *dB_acc, *dC_acc;
     float *coef;  // per position: f, s, u, exp(-E/tau) for every mode [B, L, H, 4, K]
+    const float *ek;  // per position: {E hi, E lo, 0, 0, kappa[K]} [B, L, H, tc_ek_width(K)]
     bf16 *dx, *dwr, *dww;
     float *ddt, *dalpha, *dlam, *dD;
     int *err;
@@ -74,7 +75,7 @@ struct IntraSmem {
         mg = 2 * 16384;            // Gamma o G, [t][k] K-major
         xx = TQ * XS * 4;          // fp32 Gamma' G H, then its row prefix sums
         total = rcb + x + dy + mg + xx + 4 * TQ * KMAX * 4 + TQ * 8 + 64 * 4 + 64 + 64 + 64 +
-                3 * TQ * 4 + 2 * TQ * 16;  // + the next item's per-position inputs
+                12 * TQ * 4 + TQ * 16;  // + the next item's per-position inputs
     }
 };
 
@@ -106,10 +107,10 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 4);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
-    // the next item's per-position inputs, staged by cp.async: dt, alpha, lam [3][128] floats and
-    // w_read, w_write [2][128] x 16 bytes
-    float *pf_f = reinterpret_cast<float *>(tslot + 4);
-    unsigned char *pf_w = reinterpret_cast<unsigned char *>(pf_f + 3 * TQ);
+    // the next item's per-position inputs, staged by cp.async: {E hi, E lo, 0, 0, kappa[K]} from
+    // tc_coef [128][12] floats and w_read [128] x 16 bytes
+    float *pf_e = reinterpret_cast<float *>(tslot + 4);
+    unsigned char *pf_w = reinterpret_cast<unsigned char *>(pf_e + 12 * TQ);
 
     const int tid = threadIdx.x, grp = tid >> 7, t = tid & 127, w4 = (tid >> 5) & 3;
     // persistent: items (h, c, b) in launch order, gridDim.x CTAs apart
@@ -133,19 +134,19 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         mbar_arrive_expect_tx(&bars[3], 16384u);
         tma_load_3d(sDY, &mapDY, &bars[3], h_ * P, c_ * TQ, b_);
     };
-    // every thread: its position's dt, alpha, lam, w_read, w_write of the item into the staging area
+    // its position's {E, kappa} and w_read of the item into the staging area (group 0: {E, kappa},
+    // group 1: w_read)
+    const int ekw = tc_ek_width(K);
     auto stage_inputs = [&](int item) {
         const int3 hcb = item_hcb(item);
         const int h_ = hcb.x, c_ = hcb.y, b_ = hcb.z;
-        if (c_ * TQ + t < d.L && grp == 0) {
-            const size_t i = blh(d, b_, c_ * TQ + t, h_);
-            cp_async4(pf_f + t, a.dt + i);
-            cp_async4(pf_f + TQ + t, a.alpha + i);
-            cp_async4(pf_f + 2 * TQ + t, a.lam + i);
+        // rows past the end of a ragged chunk take the last row's E (zero token rates there)
+        const int tt = min(c_ * TQ + t, d.L - 1);
+        const size_t i = blh(d, b_, tt, h_);
+        if (grp == 0) {
+            for (int q = 0; q < 1 + K / 4; ++q) cp_async_bytes(pf_e + t * 12 + 4 * q, a.ek + i * ekw + 4 * q, 16);
         } else if (c_ * TQ + t < d.L) {
-            const size_t i = blh(d, b_, c_ * TQ + t, h_);
             cp_async_bytes(pf_w + t * 16, a.wr + i * K, 2 * K);
-            cp_async_bytes(pf_w + TQ * 16 + t * 16, a.ww + i * K, 2 * K);
         }
         cp_async_commit();
     };
@@ -181,19 +182,22 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         // per-position inputs of row t from the staging area, and the mode time constants
         cp_async_wait_all();
         __syncthreads();
-        float dtv = 1.f, alv = 1.f, lmv = 1.f;
-        float wr_t[KMAX], ww_t[KMAX], tau_r[KMAX];
+        float wr_t[KMAX], kap_t[KMAX], tau_r[KMAX];
+        float2 Et2 = make_float2(0.f, 0.f);  // in-chunk cumulative log-decay (hi, lo)
 #pragma unroll
-        for (int m = 0; m < KMAX; ++m) tau_r[m] = m < K ? a.tau[h * K + m] : 1.f;
+        for (int m = 0; m < KMAX; ++m) {
+            tau_r[m] = m < K ? a.tau[h * K + m] : 1.f;
+            wr_t[m] = kap_t[m] = 0.f;
+        }
+        {
+            const float4 e4 = *reinterpret_cast<const float4 *>(pf_e + t * 12);
+            Et2 = make_float2(e4.x, e4.y);
+        }
         if (t < n) {
-            dtv = pf_f[t];
-            alv = pf_f[TQ + t];
-            lmv = pf_f[2 * TQ + t];
-            load_weights(reinterpret_cast<const bf16 *>(pf_w + t * 16), K, wr_t);
-            load_weights(reinterpret_cast<const bf16 *>(pf_w + TQ * 16 + t * 16), K, ww_t);
-        } else {
 #pragma unroll
-            for (int m = 0; m < KMAX; ++m) wr_t[m] = ww_t[m] = 0.f;
+            for (int m = 0; m < KMAX; ++m)
+                if (m < K) kap_t[m] = pf_e[t * 12 + 4 + m];
+            load_weights(reinterpret_cast<const bf16 *>(pf_w + t * 16), K, wr_t);
         }
         if (tid < K) {
             const float tv = a.tau[h * K + tid];
@@ -202,28 +206,14 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         }
         __syncthreads();  // the staging area is free again: the next item's inputs
         if (item + int(gridDim.x) < nitems) stage_inputs(item + gridDim.x);
-        float tmax = 0.f;
-#pragma unroll
-        for (int m = 0; m < KMAX; ++m) tmax = fmaxf(tmax, m < K ? tau_r[m] : 0.f);
-        const float log_cap = logf(64.f * tmax);
-        float e = 0.f;
-        if (t < n) {
-            bool cl;
-            e = token_rate(dtv, alv, lmv, log_cap, &cl);
-        }
-        const float2 Et2 = group_scan128_f2(e, wsum);  // in-chunk cumulative log-decay (hi, lo)
         if (grp == 0) E_s[t] = Et2;
         float l2r[KMAX];  // log2(e) / tau per mode, in registers
-        float kap_t[KMAX];
 #pragma unroll
         for (int m = 0; m < KMAX; ++m) {
             l2r[m] = m < K ? kLog2e / tau_r[m] : 0.f;
-            float kp = 0.f;
-            if (m < K && t < n) kp = -expm1f(-e / tau_r[m]) * ww_t[m];
-            kap_t[m] = kp;
             if (grp == 0) {
                 wr_s[t * KMAX + m] = wr_t[m];
-                kap_s[t * KMAX + m] = kp;
+                kap_s[t * KMAX + m] = kap_t[m];
             }
         }
         tc_fence_before();
@@ -1150,7 +1140,8 @@ size_t tc_bwd_workspace_bytes(const ScanDims &d, TcBwdWorkspace *l, char *base) 
     };
     const size_t st = tc_state_elems(d) * 2;
     l->S_in = take(st);
-    l->coef = (float *)take(tc_coef_elems(d) * 4);  // S_in and coef as in the forward's workspace
+    l->coef = (float *)take(tc_coef_elems(d) * 4);  // S_in, coef and ek as in the forward's workspace
+    l->ek = (float *)take(tc_ek_elems(d) * 4);
     l->dS_out = take(st);
     l->dx_acc = (float *)take(blh_ * d.P * 4);
     l->dwr_acc = (float *)take(blh_ * d.K * 4);
@@ -1174,7 +1165,7 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
     if ((e = cudaMemsetAsync(ws.cdot, 0, sizeof(float) * d.B * d.H * d.nc * d.K, st))) return e;
     if ((e = cudaMemsetAsync(ws.mh_total, 0, sizeof(float) * d.B * d.nc * d.G * TQ * TQ, st))) return e;
     if (!reuse_states &&
-        ((e = tc_coef_launch(d, p, ws.coef, st)) ||
+        ((e = tc_coef_launch(d, p, ws.coef, ws.ek, st)) ||
          (e = tc_state_pass_launch(d, false, p.x, p.Bm, ws.coef, p.h0, ws.S_in, nullptr, err, st))))
         return e;
     if ((e = tc_state_pass_launch(d, true, p.dy, p.Cm, ws.coef, p.dh_final, ws.dS_out, p.dh0, err, st)))
@@ -1199,7 +1190,7 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
     a.dt = p.dt; a.alpha = p.alpha; a.lam = p.lam; a.tau = p.tau; a.D = p.D;
     a.S_in = (const bf16 *)ws.S_in; a.dS_out = (const bf16 *)ws.dS_out;
     a.dx_acc = ws.dx_acc; a.dwr_acc = ws.dwr_acc; a.dkap_acc = ws.dkap_acc; a.ab_acc = ws.ab_acc;
-    a.rect = ws.rect; a.cdot = ws.cdot; a.mh_total = ws.mh_total; a.coef = ws.coef;
+    a.rect = ws.rect; a.cdot = ws.cdot; a.mh_total = ws.mh_total; a.coef = ws.coef; a.ek = ws.ek;
     a.dB_acc = ws.dB_acc; a.dC_acc = ws.dC_acc;
     a.dx = (bf16 *)p.dx; a.dwr = (bf16 *)p.dwr; a.dww = (bf16 *)p.dww;
     a.ddt = p.ddt; a.dalpha = p.dalpha; a.dlam = p.dlam; a.dD = p.dD;
