@@ -75,7 +75,8 @@ struct IntraSmem {
         mg = 2 * 16384;            // Gamma o G, [t][k] K-major
         xx = TQ * XS * 4;          // fp32 Gamma' G H, then its row prefix sums
         total = rcb + x + dy + mg + xx + 4 * TQ * KMAX * 4 + TQ * 8 + 64 * 4 + 64 + 64 + 64 +
-                12 * TQ * 4 + TQ * 16;  // + the next item's per-position inputs
+                12 * TQ * 4 + TQ * 16 +  // + the next item's per-position inputs
+                3 * 64 * KMAX * 4;       // + the 16-anchor factors V16, V16 / tau, U16
     }
 };
 
@@ -111,6 +112,12 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     // tc_coef [128][12] floats and w_read [128] x 16 bytes
     float *pf_e = reinterpret_cast<float *>(tslot + 4);
     unsigned char *pf_w = reinterpret_cast<unsigned char *>(pf_e + 12 * TQ);
+    // the lower-left 16 x 16 quarter of each diagonal 32 x 32 block, factored through E at the
+    // block's 16th position: V16 [64 (block, k mod 16)][KMAX] = kappa exp(-(E_a16 - E_k)/tau),
+    // V16 / tau, and U16 [64 (block, t mod 16 of the lower half)][KMAX] = w_read exp(-(E_t - E_a16)/tau)
+    float *V16s = reinterpret_cast<float *>(pf_w + TQ * 16);
+    float *V16ps = V16s + 64 * KMAX;
+    float *U16s = V16ps + 64 * KMAX;
 
     const int tid = threadIdx.x, grp = tid >> 7, t = tid & 127, w4 = (tid >> 5) & 3;
     // persistent: items (h, c, b) in launch order, gridDim.x CTAs apart
@@ -238,6 +245,12 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
                 *reinterpret_cast<uint4 *>(row + (((2 * J) ^ (t & 7)) * 16)) = make_uint4(u[0], u[1], u[2], u[3]);
                 *reinterpret_cast<uint4 *>(row + (((2 * J + 1) ^ (t & 7)) * 16)) = make_uint4(u[4], u[5], u[6], u[7]);
             }
+            if ((t & 31) >= 16) {  // lower half of its block: U16 against the anchor 32 I + 15
+                const float dE = diff_f2(Et2, E_s[32 * I + 15]);
+#pragma unroll
+                for (int m = 0; m < KMAX; ++m)
+                    U16s[(16 * I + (t & 15)) * KMAX + m] = (m < K && t < n) ? wr_t[m] * ex2_approx(-dE * l2r[m]) : 0.f;
+            }
         } else {
             const int J = t >> 5, r = t & 31;
             const float dE = diff_f2(E_s[32 * J + 31], Et2);
@@ -254,6 +267,15 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
             *reinterpret_cast<uint4 *>(row + (((2 * J + 1) ^ (r & 7)) * 16)) = make_uint4(v[4], v[5], v[6], v[7]);
             *reinterpret_cast<uint4 *>(rowp + (((2 * J) ^ (r & 7)) * 16)) = make_uint4(vp[0], vp[1], vp[2], vp[3]);
             *reinterpret_cast<uint4 *>(rowp + (((2 * J + 1) ^ (r & 7)) * 16)) = make_uint4(vp[4], vp[5], vp[6], vp[7]);
+            if (r < 16) {  // left half of its block: V16 against the anchor 32 J + 15
+                const float dE16 = diff_f2(E_s[32 * J + 15], Et2);
+#pragma unroll
+                for (int m = 0; m < KMAX; ++m) {
+                    const float v16 = m < K ? kap_t[m] * ex2_approx(-dE16 * l2r[m]) : 0.f;
+                    V16s[(16 * J + r) * KMAX + m] = v16;
+                    V16ps[(16 * J + r) * KMAX + m] = m < K ? v16 / tau_s[m] : 0.f;
+                }
+            }
         }
         fence_async_smem();
         __syncthreads();
@@ -313,41 +335,42 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
             float acc[KMAX];
 #pragma unroll
             for (int m = 0; m < KMAX; ++m) acc[m] = 0.f;
-#pragma unroll 1
-            for (int it = grp; it < 16; it += 2) {
-                const int kc = it >> 2, q8 = it & 3;
-                const int k0 = 32 * kc + 8 * q8;
-                unsigned char *mg = sMG + (kc >> 1) * 16384 + t * 128 + ((((kc & 1) * 4 + q8) ^ (t & 7)) * 16);
-                if (kc > I) {
-                    *reinterpret_cast<uint4 *>(mg) = make_uint4(0, 0, 0, 0);
-#pragma unroll
-                    for (int kk = 0; kk < 8; ++kk) XX[t * XS + k0 + kk] = 0.f;  // rows are 129 floats apart
-                    continue;
+            // the Gamma o G tile (bf16) and the head-summed Gamma o H for 8 columns from k0
+            auto store_item = [&](const float *gv, const float *hv, unsigned char *mg, int k0) {
+                *reinterpret_cast<uint4 *>(mg) = make_uint4(pack_bf16x2(gv[0], gv[1]), pack_bf16x2(gv[2], gv[3]),
+                                                            pack_bf16x2(gv[4], gv[5]), pack_bf16x2(gv[6], gv[7]));
+                if (t < n && k0 <= t) {
+                    atomicAdd(reinterpret_cast<float4 *>(mh_row + k0), make_float4(hv[0], hv[1], hv[2], hv[3]));
+                    if (k0 + 4 <= t)
+                        atomicAdd(reinterpret_cast<float4 *>(mh_row + k0 + 4), make_float4(hv[4], hv[5], hv[6], hv[7]));
                 }
+            };
+            // the diagonal block I in 16 x 16 quarters: the two on the diagonal sum their pairs
+            // k <= t directly, the lower-left one is factored through E at 32 I + 15 (U16 V16,
+            // both factors <= 1), the upper-right one is zero.  Each step gives every lane 8
+            // columns: the direct step the lane's own diagonal quarter (upper rows: left half,
+            // lower rows: right half), the other step the rest (lower rows: factored, upper: zero).
+            auto diag_item = [&](int kc, bool dstep) {
+                const bool upper = (t & 31) < 16;
+                const int q8l = (dstep == upper) ? grp : grp + 2;  // this lane's 8 columns
+                const int k0 = 32 * kc + 8 * q8l;
+                unsigned char *mg = sMG + (kc >> 1) * 16384 + t * 128 + ((((kc & 1) * 4 + q8l) ^ (t & 7)) * 16);
                 float gv[8], hv[8];
-                tmem_ld8(lane_base + colG + k0, gv);
-                tmem_ld8(lane_base + colH + k0, hv);
-                if (kc < I) {
-                    float gm[8], gp[8];
-                    tmem_ld8(lane_base + colGam + k0, gm);
-                    tmem_ld8(lane_base + colGamP + k0, gp);
+                {
+                    float ga[8], gb[8], ha[8], hb[8];
+                    tmem_ld8(lane_base + colG + 32 * kc + 8 * grp, ga);
+                    tmem_ld8(lane_base + colG + 32 * kc + 8 * grp + 16, gb);
+                    tmem_ld8(lane_base + colH + 32 * kc + 8 * grp, ha);
+                    tmem_ld8(lane_base + colH + 32 * kc + 8 * grp + 16, hb);
                     tmem_ld_wait();
+                    const bool lo = q8l == grp;
 #pragma unroll
                     for (int kk = 0; kk < 8; ++kk) {
-                        const int k = k0 + kk;
-                        const float gh = gv[kk] * hv[kk];
-                        XX[t * XS + k] = gp[kk] * gh;
-                        GHs[t * XS + k] = gh;
-                        const float4 v0 = *reinterpret_cast<const float4 *>(Vs + k * KMAX);
-                        const float4 v1 = *reinterpret_cast<const float4 *>(Vs + k * KMAX + 4);
-                        const float vk[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
-#pragma unroll
-                        for (int m = 0; m < KMAX; ++m) acc[m] = fmaf(vk[m], gh, acc[m]);
-                        gv[kk] *= gm[kk];  // Gamma o G
-                        hv[kk] *= gm[kk];  // Gamma o H
+                        gv[kk] = lo ? ga[kk] : gb[kk];
+                        hv[kk] = lo ? ha[kk] : hb[kk];
                     }
-                } else {
-                    tmem_ld_wait();
+                }
+                if (dstep) {
 #pragma unroll
                     for (int kk = 0; kk < 8; ++kk) {
                         const int k = k0 + kk;
@@ -372,14 +395,88 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
                         XX[t * XS + k] = gamt * (1.f / kLog2e) * gh;
                         GHs[t * XS + k] = gh;
                     }
+                } else if (!upper) {
+                    const float *u16 = U16s + (16 * kc + (t & 15)) * KMAX;
+                    const float4 ua = *reinterpret_cast<const float4 *>(u16), ub = *reinterpret_cast<const float4 *>(u16 + 4);
+                    const float uu[8] = {ua.x, ua.y, ua.z, ua.w, ub.x, ub.y, ub.z, ub.w};
+                    float a16[KMAX];
+#pragma unroll
+                    for (int m = 0; m < KMAX; ++m) a16[m] = 0.f;
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) {
+                        const int k = k0 + kk, j16 = 16 * kc + (k & 15);
+                        const float gh = t < n ? gv[kk] * hv[kk] : 0.f;
+                        const float4 v0 = *reinterpret_cast<const float4 *>(V16s + j16 * KMAX);
+                        const float4 v1 = *reinterpret_cast<const float4 *>(V16s + j16 * KMAX + 4);
+                        const float4 p0 = *reinterpret_cast<const float4 *>(V16ps + j16 * KMAX);
+                        const float4 p1 = *reinterpret_cast<const float4 *>(V16ps + j16 * KMAX + 4);
+                        const float vk[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+                        const float pk[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
+                        float gam = 0.f, gamp = 0.f;
+#pragma unroll
+                        for (int m = 0; m < KMAX; ++m) {
+                            gam = fmaf(uu[m], vk[m], gam);
+                            gamp = fmaf(uu[m], pk[m], gamp);
+                            a16[m] = fmaf(vk[m], gh, a16[m]);
+                        }
+                        XX[t * XS + k] = gamp * gh;
+                        GHs[t * XS + k] = gh;
+                        gv[kk] *= gam;
+                        hv[kk] *= gam;
+                    }
+                    // intra dw_read of these pairs: exp(-(E_t - E_a16)/tau) sum_k V16[k] G H
+                    const float dE = diff_f2(Et2, E_s[32 * kc + 15]);
+#pragma unroll
+                    for (int m = 0; m < KMAX; ++m)
+                        if (m < K) dwr_i[m] = fmaf(ex2_approx(-dE * l2r[m]), a16[m], dwr_i[m]);
+                } else {
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) {
+                        gv[kk] = hv[kk] = 0.f;
+                        XX[t * XS + k0 + kk] = 0.f;
+                    }
                 }
-                *reinterpret_cast<uint4 *>(mg) = make_uint4(pack_bf16x2(gv[0], gv[1]), pack_bf16x2(gv[2], gv[3]),
-                                                            pack_bf16x2(gv[4], gv[5]), pack_bf16x2(gv[6], gv[7]));
-                if (t < n && k0 <= t) {
-                    atomicAdd(reinterpret_cast<float4 *>(mh_row + k0), make_float4(hv[0], hv[1], hv[2], hv[3]));
-                    if (k0 + 4 <= t)
-                        atomicAdd(reinterpret_cast<float4 *>(mh_row + k0 + 4), make_float4(hv[4], hv[5], hv[6], hv[7]));
+                store_item(gv, hv, mg, k0);
+            };
+#pragma unroll 1
+            for (int it = grp; it < 16; it += 2) {
+                const int kc = it >> 2, q8 = it & 3;
+                if (kc == I) {
+                    diag_item(kc, q8 == grp);
+                    continue;
                 }
+                const int k0 = 32 * kc + 8 * q8;
+                unsigned char *mg = sMG + (kc >> 1) * 16384 + t * 128 + ((((kc & 1) * 4 + q8) ^ (t & 7)) * 16);
+                if (kc > I) {
+                    *reinterpret_cast<uint4 *>(mg) = make_uint4(0, 0, 0, 0);
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) XX[t * XS + k0 + kk] = 0.f;  // rows are 129 floats apart
+                    continue;
+                }
+                float gv[8], hv[8];
+                tmem_ld8(lane_base + colG + k0, gv);
+                tmem_ld8(lane_base + colH + k0, hv);
+                {
+                    float gm[8], gp[8];
+                    tmem_ld8(lane_base + colGam + k0, gm);
+                    tmem_ld8(lane_base + colGamP + k0, gp);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) {
+                        const int k = k0 + kk;
+                        const float gh = gv[kk] * hv[kk];
+                        XX[t * XS + k] = gp[kk] * gh;
+                        GHs[t * XS + k] = gh;
+                        const float4 v0 = *reinterpret_cast<const float4 *>(Vs + k * KMAX);
+                        const float4 v1 = *reinterpret_cast<const float4 *>(Vs + k * KMAX + 4);
+                        const float vk[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+#pragma unroll
+                        for (int m = 0; m < KMAX; ++m) acc[m] = fmaf(vk[m], gh, acc[m]);
+                        gv[kk] *= gm[kk];  // Gamma o G
+                        hv[kk] *= gm[kk];  // Gamma o H
+                    }
+                }
+                store_item(gv, hv, mg, k0);
                 if (kc < I && q8 >= 2) {  // this thread's last item of the factored block kc
                     const float dE = diff_f2(Et2, E_s[32 * kc + 31]);
 #pragma unroll
