@@ -374,7 +374,7 @@ struct OutSmem {
         x = 16384;             // x chunk [t][p]: the MN-major operand of the intra MMA
         s = kSBuf * 8192;      // S_in tiles, one (mode, 64-wide n half) each: [p][n]
         total = c + m + x + s + TQ * KMAX * 4 /*kappa*/ + TQ * 8 /*E*/ + 64 * 4 /*tau, l2t*/ +
-                64 /*wsum*/ + 24 * 8 /*bars*/ + 16;
+                64 /*wsum*/ + 24 * 8 /*bars*/ + 16 + 64 * KMAX * 4 /*V16*/;
     }
 };
 
@@ -465,6 +465,9 @@ __global__ void __launch_bounds__(kOutLaunch, 2)
     uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 17);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
+    // the lower-left 16 x 16 quarter of each diagonal 32 x 32 block, factored through E at the
+    // block's 16th position: V16 [64 (block, k mod 16)][KMAX] = kappa exp(-(E_a16 - E_k)/tau)
+    float *V16s = reinterpret_cast<float *>(bars + 24);
 
     const int tid = threadIdx.x, grp = tid >> 7, t = tid & 127, w4 = (tid >> 5) & 3;
     const int h = blockIdx.x, c = blockIdx.y, b = blockIdx.z;
@@ -584,6 +587,12 @@ __global__ void __launch_bounds__(kOutLaunch, 2)
         unsigned char *row = sVt + r * 128;
         *reinterpret_cast<uint4 *>(row + (((2 * J) ^ (r & 7)) * 16)) = make_uint4(v[0], v[1], v[2], v[3]);
         *reinterpret_cast<uint4 *>(row + (((2 * J + 1) ^ (r & 7)) * 16)) = make_uint4(v[4], v[5], v[6], v[7]);
+        if (r < 16) {  // left half of its block: V16 against the anchor 32 J + 15
+            const float dE16 = diff_f2(E_s[32 * J + 15], Et2);
+#pragma unroll
+            for (int m = 0; m < KMAX; ++m)
+                V16s[(16 * J + r) * KMAX + m] = m < K ? kap_t[m] * ex2_approx(-dE16 * l2t[m]) : 0.f;
+        }
     }
     fence_async_smem();
     sync_first256();
@@ -618,33 +627,67 @@ __global__ void __launch_bounds__(kOutLaunch, 2)
         const int I = t >> 5;
 #pragma unroll 1
         for (int it = grp; it < 16; it += 2) {
-            const int kc = it >> 2, q8 = it & 3;
-            const int k0 = 32 * kc + 8 * q8;
+            const int kc = it >> 2;
+            int q8 = it & 3;
             float gv[8];
-            if (kc < I) {
+            if (kc == I) {
+                // the diagonal block in 16 x 16 quarters: the two on the diagonal sum their pairs
+                // k <= t directly, the lower-left one is factored through E at 32 I + 15 (both
+                // factors <= 1), the upper-right one is zero.  The direct step gives every lane
+                // its own diagonal quarter (upper rows: left half, lower rows: right half), the
+                // other step the rest (lower rows: factored, upper rows: zero).
+                const bool upper = (t & 31) < 16, dstep = q8 == grp;
+                q8 = (dstep == upper) ? grp : grp + 2;  // this lane's 8 columns
+                const int k0 = 32 * kc + 8 * q8;
+                {
+                    float ga[8], gb[8];
+                    tmem_ld8(lane_base + colG + 32 * kc + 8 * grp, ga);
+                    tmem_ld8(lane_base + colG + 32 * kc + 8 * grp + 16, gb);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) gv[kk] = q8 == grp ? ga[kk] : gb[kk];
+                }
+                if (dstep) {
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) {
+                        const int k = k0 + kk;
+                        float v = 0.f;
+                        if (k <= t && t < n) {
+                            const float dE = diff_f2(Et2, E_s[k]);
+                            float gam = 0.f;
+#pragma unroll
+                            for (int m = 0; m < KMAX; ++m)
+                                if (m < K) gam = fmaf(wr_t[m] * kap_s[k * KMAX + m], ex2_approx(-dE * l2t[m]), gam);
+                            v = gam * gv[kk];
+                        }
+                        gv[kk] = v;
+                    }
+                } else if (!upper) {
+                    const float dE = diff_f2(Et2, E_s[32 * kc + 15]);
+                    float u16[KMAX];
+#pragma unroll
+                    for (int m = 0; m < KMAX; ++m) u16[m] = m < K ? wr_t[m] * ex2_approx(-dE * l2t[m]) : 0.f;
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) {
+                        const float *v16 = V16s + (16 * kc + ((k0 + kk) & 15)) * KMAX;
+                        const float4 v0 = *reinterpret_cast<const float4 *>(v16);
+                        const float4 v1 = *reinterpret_cast<const float4 *>(v16 + 4);
+                        const float gam = u16[0] * v0.x + u16[1] * v0.y + u16[2] * v0.z + u16[3] * v0.w +
+                                          u16[4] * v1.x + u16[5] * v1.y + u16[6] * v1.z + u16[7] * v1.w;
+                        gv[kk] = t < n ? gam * gv[kk] : 0.f;
+                    }
+                } else {
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) gv[kk] = 0.f;
+                }
+            } else if (kc < I) {
+                const int k0 = 32 * kc + 8 * q8;
                 float gm[8];
                 tmem_ld8(lane_base + colG + k0, gv);
                 tmem_ld8(lane_base + colGam + k0, gm);
                 tmem_ld_wait();
 #pragma unroll
                 for (int kk = 0; kk < 8; ++kk) gv[kk] *= gm[kk];
-            } else if (kc == I) {
-                tmem_ld8(lane_base + colG + k0, gv);
-                tmem_ld_wait();
-#pragma unroll
-                for (int kk = 0; kk < 8; ++kk) {
-                    const int k = k0 + kk;
-                    float v = 0.f;
-                    if (k <= t && t < n) {
-                        const float dE = diff_f2(Et2, E_s[k]);
-                        float gam = 0.f;
-#pragma unroll
-                        for (int m = 0; m < KMAX; ++m)
-                            if (m < K) gam = fmaf(wr_t[m] * kap_s[k * KMAX + m], ex2_approx(-dE * l2t[m]), gam);
-                        v = gam * gv[kk];
-                    }
-                    gv[kk] = v;
-                }
             } else {
 #pragma unroll
                 for (int kk = 0; kk < 8; ++kk) gv[kk] = 0.f;
