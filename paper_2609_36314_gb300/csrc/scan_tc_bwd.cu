@@ -523,12 +523,15 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
             float dk2[KMAX];
 #pragma unroll
             for (int m = 0; m < KMAX; ++m) dk2[m] = 0.f;
-            const int dend = min(n, 32 * J + 32);
-            for (int tt0 = 32 * J + grp; tt0 < dend; tt0 += 8) {
+            // direct rows: k's own 16-row quarter of the diagonal block (t >= k), rows of this
+            // group's parity
+            const bool left = (k & 31) < 16;
+            const int dend = min(n, 32 * J + (left ? 16 : 32));
+            for (int tt0 = k + ((k + grp) & 1); tt0 < dend; tt0 += 8) {
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     const int tt = tt0 + 2 * u;
-                    if (tt < dend && tt >= k) {
+                    if (tt < dend) {
                         const float dE = diff_f2(E_s[tt], Ek);
                         const float gh = GHs[tt * XS + k];
 #pragma unroll
@@ -543,6 +546,25 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
                         }
                     }
                 }
+            }
+            if (left) {  // lower half of the diagonal block: factored through E at 32 J + 15
+                float a16[KMAX];
+#pragma unroll
+                for (int m = 0; m < KMAX; ++m) a16[m] = 0.f;
+                const int lend = min(n, 32 * J + 32);
+                for (int tt = 32 * J + 16 + grp; tt < lend; tt += 2) {
+                    const float gh = GHs[tt * XS + k];
+                    const float *u16 = U16s + (16 * J + (tt & 15)) * KMAX;
+                    const float4 u0 = *reinterpret_cast<const float4 *>(u16);
+                    const float4 u1 = *reinterpret_cast<const float4 *>(u16 + 4);
+                    const float uu[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+#pragma unroll
+                    for (int m = 0; m < KMAX; ++m) a16[m] = fmaf(uu[m], gh, a16[m]);
+                }
+                const float dE16 = diff_f2(E_s[32 * J + 15], Ek);
+#pragma unroll
+                for (int m = 0; m < KMAX; ++m)
+                    if (m < K) dk2[m] = fmaf(ex2_approx(-dE16 * l2r[m]), a16[m], dk2[m]);
             }
             float s0[KMAX], s1[KMAX];
 #pragma unroll
