@@ -962,6 +962,16 @@ __global__ void __launch_bounds__(kStLaunch, 1)
             }
             if (k < L.tile / 16) acc0 = dot_bf16x8(ps[k], pd[k], acc0);
             mbar_arrive(&bars[9 + q]);
+            if (i % K == 1 && i / K + 1 < a.hg) {  // the next head's dY, X and coefficient rows into L2
+                const int hn = h_first + i / K + 1;
+                for (int r = ct; r < 3 * TQ; r += kCdThreads) {
+                    const int tr = min(r % TQ, n - 1), kind = r / TQ;
+                    const size_t ir = blh(d, b, c0 + tr, hn);
+                    prefetch_l2(kind == 0 ? static_cast<const void *>(a.dy + ir * P)
+                                          : kind == 1 ? static_cast<const void *>(a.x + ir * P)
+                                                      : static_cast<const void *>(a.coef + ir * 4 * K));
+                }
+            }
             const float v = warp_sum(acc0 + acc1);
             if ((tid & 31) == 0)
                 atomicAdd(a.cdot + ((size_t(b) * d.H + h_first + i / K) * d.nc + c) * K + i % K, v);

@@ -140,6 +140,11 @@ __device__ __forceinline__ void cp_async_bytes(void *dst, const void *src, int b
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 
+// Hint: bring the 128-byte line holding p into L2 (no register result, nothing waits on it).
+__device__ __forceinline__ void prefetch_l2(const void *p) {
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(reinterpret_cast<uint64_t>(p)));
+}
+
 // Inclusive prefix sum (double) of one value per thread over a 128-thread block.
 __device__ __forceinline__ double block_scan128(double v, double *wsum) {
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
