@@ -315,11 +315,14 @@ def main():
                  dD=torch.empty_like(inp["D"]), dh0=None)
     a = inp
 
-    def train_step():
+    def train_step_on(a, y, grads):
         scan_fwd(a["x"], a["dt"], a["alpha"], a["lam"], a["tau"], a["B"], a["C"], a["w_read"],
                  a["w_write"], a["D"], want_final_state=False, y=y, workspace=ws_f)
         scan_bwd(a["x"], a["dt"], a["alpha"], a["lam"], a["tau"], a["B"], a["C"], a["w_read"],
                  a["w_write"], a["D"], a["dy"], workspace=ws_b, out=grads, reuse_fwd_states=True)
+
+    def train_step():
+        train_step_on(a, y, grads)
 
     for _ in range(max(args.warmup, 3)):
         train_step()
@@ -396,21 +399,62 @@ def main():
         h2d = sum(v.numel() * v.element_size() for v in hin.values())
         d2h = sum(v.numel() * v.element_size() for v in hout.values())
 
-        def e2e_step():
-            for k, v in hin.items():
-                inp[k].copy_(v, non_blocking=True)
-            train_step()
-            for k, v in hout.items():
-                v.copy_(grads[k] if k != "y" else y, non_blocking=True)
+        # Steps pipelined over two device copies of the inputs and of the results: step s copies
+        # its inputs (pinned host -> set s % 2) on one stream while step s - 1 computes, and
+        # reads its results back (set s % 2 -> pinned host) on another while step s + 1
+        # computes.  Every step's copies lie inside the timed region.
+        sets_in = [inp, {k: torch.empty_like(v) for k, v in inp.items()}]
+        sets_out = [(y, grads), (torch.empty_like(y),
+                                 {k: (torch.empty_like(v) if v is not None else None) for k, v in grads.items()})]
+        comp = torch.cuda.current_stream()
+        s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
+        ev_in = [torch.cuda.Event(), torch.cuda.Event()]    # inputs of set i on the device
+        ev_done = [torch.cuda.Event(), torch.cuda.Event()]  # the step that used set i has finished
+        ev_out = [torch.cuda.Event(), torch.cuda.Event()]   # results of set i read back
 
-        e2e_step()
+        def copy_in(st):
+            i = st % 2
+            with torch.cuda.stream(s_in):
+                if st >= 2:
+                    s_in.wait_event(ev_done[i])
+                for k, v in hin.items():
+                    sets_in[i][k].copy_(v, non_blocking=True)
+                ev_in[i].record(s_in)
+
+        def compute(st):
+            i = st % 2
+            comp.wait_event(ev_in[i])
+            if st >= 2:
+                comp.wait_event(ev_out[i])
+            train_step_on(sets_in[i], sets_out[i][0], sets_out[i][1])
+            ev_done[i].record(comp)
+
+        def copy_out(st):
+            i = st % 2
+            y_i, g_i = sets_out[i]
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(ev_done[i])
+                for k, v in hout.items():
+                    v.copy_(g_i[k] if k != "y" else y_i, non_blocking=True)
+                ev_out[i].record(s_out)
+
+        def e2e_run(nsteps):
+            copy_in(0)
+            for st in range(nsteps):
+                if st + 1 < nsteps:
+                    copy_in(st + 1)
+                compute(st)
+                copy_out(st)
+            comp.wait_event(ev_out[(nsteps - 1) % 2])
+
+        e2e_run(2)
         torch.cuda.synchronize()
         barrier()
-        ev0.record(stream)
-        n_e2e = max(2, args.steps // 2)
-        for _ in range(n_e2e):
-            e2e_step()
-        ev1.record(stream)
+        n_e2e = max(2, args.steps)
+        ev0.record(comp)
+        s_in.wait_event(ev0)
+        e2e_run(n_e2e)
+        ev1.record(comp)
         torch.cuda.synchronize()
         barrier()
         ms_e2e = max_over_ranks(ev0.elapsed_time(ev1) / n_e2e)
