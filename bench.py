@@ -191,7 +191,7 @@ def algorithmic_work(kernel: str, s, per_launch_units: float):
     if kernel == "bwd_intra_tc":
         return "flops", (2 * q * s.headdim + q * s.dstate * s.ngroups / s.nheads) * per_launch_units
     if kernel == "coef_tc":  # dt, alpha, lam, w_read, w_write in; f, s, u, exp(-E/tau), E, kappa out
-        return "bytes", (12 + 4 * s.nmodes + 16 * s.nmodes + 64) * per_launch_units
+        return "bytes", (12 + 4 * s.nmodes + 16 * s.nmodes + 4 * (16 if s.nmodes == 8 else 8)) * per_launch_units
     if kernel == "bwd_final_tc":  # per-position terms, dx_acc, dy, x in; dx and the scalar grads out
         return "bytes", (36 + 14 * s.nmodes + 10 * s.headdim) * per_launch_units
     if kernel == "decode_step":
