@@ -206,15 +206,16 @@ __global__ void __launch_bounds__(kThreads, 3)
         const int c_ = REV ? d.nc - 1 - ci_ : ci_;
         const int c0_ = c_ * TQ, n_ = min(TQ, d.L - c0_);
         const int t = tid;
-        {  // the slice's TPSK x values and the coefficient row, read row-coalesced
+        {  // the slice's TPSK x values and the coefficient row, read row-coalesced (the lane
+           // transposes that complete them wait until the chunk that uses them)
             const int tg = t & ~(NX - 1);
-            get_rows<NX>(nx, reinterpret_cast<const unsigned char *>(a.U + blh(d, b, c0_ + tg, h) * P + p0),
-                         size_t(d.H) * P * 2, n_ - tg);
+            load_rows<NX>(nx, reinterpret_cast<const unsigned char *>(a.U + blh(d, b, c0_ + tg, h) * P + p0),
+                          size_t(d.H) * P * 2, n_ - tg);
             const int tc = t & ~(NC - 1);
-            get_rows<NC>(ncv,
-                         reinterpret_cast<const unsigned char *>(a.coef + blh(d, b, c0_ + tc, h) * 4 * KK +
-                                                                 (REV ? 0 : KK)),
-                         size_t(d.H) * 4 * KK * 4, n_ - tc);
+            load_rows<NC>(ncv,
+                          reinterpret_cast<const unsigned char *>(a.coef + blh(d, b, c0_ + tc, h) * 4 * KK +
+                                                                  (REV ? 0 : KK)),
+                          size_t(d.H) * 4 * KK * 4, n_ - tc);
         }
         if (t < KK) ndec = a.coef[blh(d, b, c0_ + n_ - 1, h) * 4 * KK + 3 * KK + t];
     };
@@ -229,6 +230,8 @@ __global__ void __launch_bounds__(kThreads, 3)
         float cv[KK];
 #pragma unroll
         for (int q = 0; q < NX; ++q) xr[q] = nx[q];
+        lane_transpose<NX>(xr, j);
+        lane_transpose<NC>(ncv, j);
 #pragma unroll
         for (int q = 0; q < NC; ++q) {
             cv[4 * q] = __uint_as_float(ncv[q].x);

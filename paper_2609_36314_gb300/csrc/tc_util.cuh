@@ -110,15 +110,20 @@ __device__ __forceinline__ void put_rows(uint4 (&e)[NL], unsigned char *row0, si
 // The converse of put_rows: lane l of each NL-lane group receives in e[0 .. NL) the NL 16-byte
 // pieces of row l of the group (rows `stride` bytes apart from row0), loaded so that each
 // instruction reads 32 / NL whole row segments; rows >= nvalid read as zero.  Every lane of the
-// warp must call it.
+// warp must call it.  load_rows issues the loads alone (lane_transpose<NL> completes them
+// later), so that their latency can overlap other work.
 template <int NL>
-__device__ __forceinline__ void get_rows(uint4 (&e)[NL], const unsigned char *row0, size_t stride, int nvalid) {
-    const int lane = threadIdx.x & 31, i = lane & (NL - 1);
+__device__ __forceinline__ void load_rows(uint4 (&e)[NL], const unsigned char *row0, size_t stride, int nvalid) {
+    const int i = threadIdx.x & (NL - 1);
 #pragma unroll
     for (int q = 0; q < NL; ++q)
         e[q] = q < nvalid ? *reinterpret_cast<const uint4 *>(row0 + size_t(q) * stride + 16 * i)
                           : make_uint4(0, 0, 0, 0);
-    lane_transpose<NL>(e, lane);
+}
+template <int NL>
+__device__ __forceinline__ void get_rows(uint4 (&e)[NL], const unsigned char *row0, size_t stride, int nvalid) {
+    load_rows<NL>(e, row0, stride, nvalid);
+    lane_transpose<NL>(e, threadIdx.x & 31);
 }
 
 // Asynchronous global -> shared copies (cp.async, no register round trip): 4, 8 or 16 bytes,
