@@ -70,7 +70,7 @@ cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, con
                                  int *err, cudaStream_t st);
 bool tc_make_map3(CUtensorMap *m, const void *ptr, uint64_t d0, uint64_t d1, uint64_t d2,
                   uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1,
-                  uint32_t b2);
+                  uint32_t b2, int swizzle_bytes = 128);
 // Tensor-core backward (headdim 64 in addition to the forward's conditions).
 bool tc_bwd_supported(const ScanDims &d, int dtype);
 struct TcBwdWorkspace {  // S_in and coef first, at the offsets the forward uses

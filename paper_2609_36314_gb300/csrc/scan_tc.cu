@@ -134,7 +134,8 @@ struct StateSmem {
     __host__ __device__ explicit StateSmem(int N) {
         a_bytes = 2 * 16384;         // 2 M-atoms x (128 k rows x 128 B), MN-major
         v_bytes = (N / 64) * 16384;  // N/64 boxes of [128 t][64 n]
-        total = a_bytes + v_bytes + 32 * 4 /*dec*/ + 64 /*bars*/;
+        total = a_bytes + v_bytes + 4 * 2048 /*emit staging, one 2 KB tile per warp*/ + 32 * 4 /*dec*/ +
+                64 /*bars*/;
     }
 };
 
@@ -146,7 +147,7 @@ __host__ __device__ constexpr int state_tps() {
 
 template <bool REV, int KK>
 __global__ void __launch_bounds__(kThreads, 3)
-    tc_state_pass(const __grid_constant__ CUtensorMap mapV, StateArgs a) {
+    tc_state_pass(const __grid_constant__ CUtensorMap mapV, const __grid_constant__ CUtensorMap mapE, StateArgs a) {
     constexpr int TPSK = state_tps<KK>();  // 16 (KK = 8) or 32 (KK = 4)
     constexpr int NX = TPSK / 8;           // 16-byte pieces of one position's x slice
     extern __shared__ unsigned char smem_raw[];
@@ -157,7 +158,8 @@ __global__ void __launch_bounds__(kThreads, 3)
     const StateSmem plan(N);
     unsigned char *sA = base;
     unsigned char *sV = sA + plan.a_bytes;
-    float *dec = reinterpret_cast<float *>(sV + plan.v_bytes);     // [32] this chunk's decay per mode
+    unsigned char *sE = sV + plan.v_bytes;                          // [4 warps][32 rows x 64 B] emit staging
+    float *dec = reinterpret_cast<float *>(sE + 4 * 2048);          // [32] this chunk's decay per mode
     uint64_t *bars = reinterpret_cast<uint64_t *>(dec + 32);        // tma, mma
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 2);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
@@ -272,41 +274,42 @@ __global__ void __launch_bounds__(kThreads, 3)
             }
         }
         // emit the entering state (bf16) and apply the chunk's decay in place (the TMEM load of
-        // the next 32 columns is in flight while the current ones are processed).  Blocks come in
-        // pairs covering 64 columns, so lane j then holds 128 contiguous bytes of its row; an
-        // 8 x 8 transpose of 16-byte pieces within each 8-lane group (rows p of one mode) lets
-        // every store instruction write 4 full rows of 128 bytes.
+        // the next 32 columns is in flight while the current ones are processed).  Each warp's 32
+        // rows x 32 columns go through a 2 KB staging tile (64-byte swizzle) and one TMA store:
+        // rows (mode, p) of the warp are (32 w / TPSK + lane / TPSK, p0 + lane % TPSK).
         {
-            const int nblk = N / 32;  // even
+            const int nblk = N / 32;
             const float dm = dec[lm];
-            bf16 *erow = a.emit + ((bh * d.nc + c) * KK + lm) * PN + size_t(p0 + (lp & ~7)) * N + 8 * (j & 7);
-            uint4 e8[8];
-            auto process = [&](float *v, int blk, int hb) {
+            unsigned char *stg = sE + w * 2048;
+            const int rowE = int((bh * d.nc + c) * KK + (32 * w) / TPSK);
+            auto process = [&](float *v, int blk) {
+                if (j == 0) bulk_wait_read();  // the previous store has read the staging tile
+                __syncwarp();
 #pragma unroll
                 for (int q = 0; q < 4; ++q)
-                    e8[4 * hb + q] =
+                    *reinterpret_cast<uint4 *>(stg + j * 64 + ((q ^ ((j >> 1) & 3)) * 16)) =
                         make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
                                    pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+                fence_async_smem();
+                __syncwarp();
+                if (j == 0) {
+                    tma_store_3d(&mapE, stg, 32 * blk, p0, rowE);
+                    bulk_commit();
+                }
 #pragma unroll
                 for (int i = 0; i < 32; ++i) v[i] *= dm;
 #pragma unroll
                 for (int q = 0; q < 4; ++q) tmem_st8(lane_base + 32 * blk + 8 * q, v + 8 * q);
-                if (hb) {
-                    lane_transpose<8>(e8, j);
-                    bf16 *o = erow + 32 * (blk - 1);
-#pragma unroll
-                    for (int q = 0; q < 8; ++q) *reinterpret_cast<uint4 *>(o + size_t(q) * N) = e8[q];
-                }
             };
             float v0[32], v1[32];
             tmem_ld32(lane_base, v0);
-            for (int blk = 0; blk < nblk; blk += 2) {
+            for (int blk = 0; blk < nblk; blk += 2) {  // nblk = N / 32 is even
                 tmem_ld_wait();
                 tmem_ld32(lane_base + 32 * (blk + 1), v1);
-                process(v0, blk, 0);
+                process(v0, blk);
                 tmem_ld_wait();
                 if (blk + 2 < nblk) tmem_ld32(lane_base + 32 * (blk + 2), v0);
-                process(v1, blk + 1, 1);
+                process(v1, blk + 1);
             }
         }
         tmem_st_wait();
@@ -347,6 +350,7 @@ __global__ void __launch_bounds__(kThreads, 3)
             for (int q = 0; q < 8; ++q) o[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
         }
     }
+    if (j == 0) bulk_wait_all();  // this warp's emit stores are complete
     if (*abort_s && tid == 0) atomicExch(a.err, kTimeoutCode);
     tc_fence_before();
     __syncthreads();
@@ -787,7 +791,7 @@ EncodeTiledFn encode_fn() {
 // 3-D bf16 tensor map, innermost dimension first; 128-byte swizzle.
 bool tc_make_map3(CUtensorMap *m, const void *ptr, uint64_t d0, uint64_t d1, uint64_t d2,
                uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1,
-               uint32_t b2) {
+               uint32_t b2, int swizzle_bytes) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     const cuuint64_t dims[3] = {d0, d1, d2};
@@ -795,7 +799,8 @@ bool tc_make_map3(CUtensorMap *m, const void *ptr, uint64_t d0, uint64_t d1, uin
     const cuuint32_t box[3] = {b0, b1, b2};
     const cuuint32_t es[3] = {1, 1, 1};
     return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), dims, strides, box,
-              es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+              swizzle_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B,
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -838,6 +843,13 @@ cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, con
     if (!tc_make_map3(&mapV, V, uint64_t(d.G) * d.N, d.L, d.B, uint64_t(d.G) * d.N * 2,
                    uint64_t(d.L) * d.G * d.N * 2, 64, TQ, 1))
         return cudaErrorInvalidValue;
+    // per-chunk states [B, H, nc, K, P, N] as (n, p, (b, h, c, m)) rows; a box is one warp's
+    // 32 columns x 32 TMEM lanes = 128 / K ... modes x P-slice rows
+    CUtensorMap mapE;
+    const int tps = 128 / d.K;
+    if (!tc_make_map3(&mapE, emit, d.N, d.P, uint64_t(d.B) * d.H * d.nc * d.K, uint64_t(d.N) * 2,
+                      uint64_t(d.P) * d.N * 2, 32, uint32_t(tps), uint32_t(32 / tps), 64))
+        return cudaErrorInvalidValue;
     StateArgs a;
     a.d = d;
     a.U = (const bf16 *)U;
@@ -850,7 +862,7 @@ cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, con
     auto launch = [&](auto kern, int tps, const char *name) {
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
         trace_begin(name, st);
-        kern<<<dim3(d.P / tps, d.H, d.B), kThreads, smem, st>>>(mapV, a);
+        kern<<<dim3(d.P / tps, d.H, d.B), kThreads, smem, st>>>(mapV, mapE, a);
         trace_end(st);
     };
     if (d.K == 8) {
