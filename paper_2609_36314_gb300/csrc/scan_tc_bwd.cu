@@ -76,7 +76,8 @@ struct IntraSmem {
         xx = TQ * XS * 4;          // fp32 Gamma' G H, then its row prefix sums
         total = rcb + x + dy + mg + xx + 4 * TQ * KMAX * 4 + TQ * 8 + 64 * 4 + 64 + 64 + 64 +
                 12 * TQ * 4 + TQ * 16 +  // + the next item's per-position inputs
-                3 * 64 * KMAX * 4;       // + the 16-anchor factors V16, V16 / tau, U16
+                3 * 64 * KMAX * 4 +      // + the 16-anchor factors V16, V16 / tau, U16
+                KMAX * 4;                // + the next item's time constants
     }
 };
 
@@ -118,6 +119,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     float *V16s = reinterpret_cast<float *>(pf_w + TQ * 16);
     float *V16ps = V16s + 64 * KMAX;
     float *U16s = V16ps + 64 * KMAX;
+    float *pf_tau = U16s + 64 * KMAX;  // the next item's mode time constants [KMAX] (staged)
 
     const int tid = threadIdx.x, grp = tid >> 7, t = tid & 127, w4 = (tid >> 5) & 3;
     // persistent: items (h, c, b) in launch order, gridDim.x CTAs apart
@@ -152,6 +154,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         const size_t i = blh(d, b_, tt, h_);
         if (grp == 0) {
             for (int q = 0; q < 1 + K / 4; ++q) cp_async_bytes(pf_e + t * 12 + 4 * q, a.ek + i * ekw + 4 * q, 16);
+            if (t < K / 4) cp_async_bytes(pf_tau + 4 * t, a.tau + h_ * K + 4 * t, 16);
         } else if (c_ * TQ + t < d.L) {
             cp_async_bytes(pf_w + t * 16, a.wr + i * K, 2 * K);
         }
@@ -193,7 +196,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         float2 Et2 = make_float2(0.f, 0.f);  // in-chunk cumulative log-decay (hi, lo)
 #pragma unroll
         for (int m = 0; m < KMAX; ++m) {
-            tau_r[m] = m < K ? a.tau[h * K + m] : 1.f;
+            tau_r[m] = m < K ? pf_tau[m] : 1.f;
             wr_t[m] = kap_t[m] = 0.f;
         }
         {
@@ -207,7 +210,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
             load_weights(reinterpret_cast<const bf16 *>(pf_w + t * 16), K, wr_t);
         }
         if (tid < K) {
-            const float tv = a.tau[h * K + tid];
+            const float tv = pf_tau[tid];
             tau_s[tid] = tv;
             l2t[tid] = kLog2e / tv;
         }
