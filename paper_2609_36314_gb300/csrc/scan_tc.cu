@@ -804,6 +804,20 @@ bool tc_make_map3(CUtensorMap *m, const void *ptr, uint64_t d0, uint64_t d1, uin
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 4-D float32 tensor map, innermost dimension first; 128-byte swizzle (inner box of 32 floats).
+bool tc_make_map4_f32(CUtensorMap *m, const void *ptr, const uint64_t dims[4], const uint64_t strides_bytes[3],
+                      const uint32_t box[4]) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dd[4] = {dims[0], dims[1], dims[2], dims[3]};
+    const cuuint64_t ss[3] = {strides_bytes[0], strides_bytes[1], strides_bytes[2]};
+    const cuuint32_t bb[4] = {box[0], box[1], box[2], box[3]};
+    const cuuint32_t es[4] = {1, 1, 1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<void *>(ptr), dd, ss, bb, es,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 bool tc_supported(const ScanDims &d, int dtype) {
     if (dtype != 1) return false;
     if (d.P != 64 || (d.N != 64 && d.N != 128) || (d.K != 4 && d.K != 8)) return false;

@@ -716,6 +716,7 @@ __device__ __forceinline__ uint4 scale_bf16x8(uint4 a, float s) {
 __global__ void __launch_bounds__(kStLaunch, 1)
     tc_bwd_state(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapB,
                  const __grid_constant__ CUtensorMap mapS, const __grid_constant__ CUtensorMap mapD,
+                 const __grid_constant__ CUtensorMap mapdC, const __grid_constant__ CUtensorMap mapdB,
                  BwdArgs a) {
     extern __shared__ unsigned char smem_raw[];
     unsigned char *base = align1024(smem_raw);
@@ -1058,24 +1059,36 @@ __global__ void __launch_bounds__(kStLaunch, 1)
     if (nsteps > 0 && tid < kStThreads) readout(nsteps - 1);
     // the group's dC / dB into the float32 accumulators (group g takes n in [64 g, 64 g + 64))
     tc_fence_after();
+    // the group's dC / dB into the float32 accumulators by TMA reduce-add: every warp has left
+    // the tiles and the generated operands, which now stage dC (generator buffers) and dB (tile
+    // buffers) as [N / 32 boxes][128 t][32 n] float32 with the 128-byte swizzle
+    __syncthreads();
     if (tid < kStThreads && grp < N / 64) {
-        const int t8 = t & ~7;
-        const int nv = *abort_s ? 0 : n - t8;
-        const size_t gi = ((size_t(b) * d.L + c0 + t8) * d.G + g) * N + grp * 64;
-        const size_t rs = size_t(d.G) * N * 4;
         for (int n32 = 0; n32 < 64; n32 += 32) {
             float vc[32], vb[32];
             tmem_ld32(lane_base + colC + grp * 64 + n32, vc);
             tmem_ld32(lane_base + colB + grp * 64 + n32, vb);
             tmem_ld_wait();
-            uint4 e[8];
+            const int q = (grp * 64 + n32) / 32;
+            unsigned char *rc = sG + q * 16384 + t * 128, *rb = sT + q * 16384 + t * 128;
 #pragma unroll
-            for (int k = 0; k < 8; ++k) e[k] = f4_bits(vc[4 * k], vc[4 * k + 1], vc[4 * k + 2], vc[4 * k + 3]);
-            put_rows<8, true>(e, reinterpret_cast<unsigned char *>(a.dC_acc + gi + n32), rs, nv);
-#pragma unroll
-            for (int k = 0; k < 8; ++k) e[k] = f4_bits(vb[4 * k], vb[4 * k + 1], vb[4 * k + 2], vb[4 * k + 3]);
-            put_rows<8, true>(e, reinterpret_cast<unsigned char *>(a.dB_acc + gi + n32), rs, nv);
+            for (int k = 0; k < 8; ++k) {
+                *reinterpret_cast<float4 *>(rc + ((k ^ (t & 7)) * 16)) =
+                    make_float4(vc[4 * k], vc[4 * k + 1], vc[4 * k + 2], vc[4 * k + 3]);
+                *reinterpret_cast<float4 *>(rb + ((k ^ (t & 7)) * 16)) =
+                    make_float4(vb[4 * k], vb[4 * k + 1], vb[4 * k + 2], vb[4 * k + 3]);
+            }
         }
+        fence_async_smem();
+    }
+    __syncthreads();
+    if (tid == 0 && !*abort_s) {  // rows past the end of the sequence fall outside the map
+        for (int q = 0; q < N / 32; ++q) {
+            tma_reduce_add_4d(&mapdC, sG + q * 16384, 32 * q, g, c0, b);
+            tma_reduce_add_4d(&mapdB, sT + q * 16384, 32 * q, g, c0, b);
+        }
+        bulk_commit();
+        bulk_wait_all();
     }
     if (*abort_s && tid == 0) atomicExch(a.err, kTimeoutCode);
     tc_fence_before();
@@ -1304,7 +1317,7 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
         return e;
     if (d.nc == 0) return cudaSuccess;
     const uint64_t GN = uint64_t(d.G) * d.N, HP = uint64_t(d.H) * d.P;
-    CUtensorMap mapC, mapB, mapX, mapDY, mapS, mapD;
+    CUtensorMap mapC, mapB, mapX, mapDY, mapS, mapD, mapdC, mapdB;
     const uint64_t srows = uint64_t(d.B) * d.H * d.nc * d.K;
     if (!tc_make_map3(&mapC, p.Cm, GN, d.L, d.B, GN * 2, uint64_t(d.L) * GN * 2, 64, TQ, 1) ||
         !tc_make_map3(&mapB, p.Bm, GN, d.L, d.B, GN * 2, uint64_t(d.L) * GN * 2, 64, TQ, 1) ||
@@ -1315,6 +1328,14 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
         !tc_make_map3(&mapD, ws.dS_out, d.N, d.P, srows, uint64_t(d.N) * 2, uint64_t(d.P) * d.N * 2, 64,
                       64, 1))
         return cudaErrorInvalidValue;
+    {  // dC / dB float32 accumulators [B, L, G, N] as (n, g, l, b); a box is 32 n x 128 positions
+        const uint64_t dims[4] = {uint64_t(d.N), uint64_t(d.G), uint64_t(d.L), uint64_t(d.B)};
+        const uint64_t strides[3] = {uint64_t(d.N) * 4, uint64_t(d.G) * d.N * 4, uint64_t(d.L) * d.G * d.N * 4};
+        const uint32_t box[4] = {32, 1, TQ, 1};
+        if (!tc_make_map4_f32(&mapdC, ws.dC_acc, dims, strides, box) ||
+            !tc_make_map4_f32(&mapdB, ws.dB_acc, dims, strides, box))
+            return cudaErrorInvalidValue;
+    }
     BwdArgs a;
     a.d = d;
     a.x = (const bf16 *)p.x; a.dy = (const bf16 *)p.dy;
@@ -1349,7 +1370,8 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
         const size_t smem = StSmem(d.N).total + 1024;
         cudaFuncSetAttribute(tc_bwd_state, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
         trace_begin("bwd_state_tc", st);
-        tc_bwd_state<<<dim3(d.H / a.hg, d.nc, d.B), kStLaunch, smem, st>>>(mapC, mapB, mapS, mapD, a);
+        tc_bwd_state<<<dim3(d.H / a.hg, d.nc, d.B), kStLaunch, smem, st>>>(mapC, mapB, mapS, mapD, mapdC, mapdB,
+                                                                              a);
         trace_end(st);
         if ((e = cudaGetLastError())) return e;
     }
