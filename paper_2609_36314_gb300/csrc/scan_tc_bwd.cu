@@ -734,7 +734,8 @@ __global__ void __launch_bounds__(kStLaunch, 1)
     //       7, 8 generated operands of step parity written (all 256 threads arrive) |
     //       9, 10 tile buffer read by the <dS_out, S_in> warps (all 96 threads arrive)
     uint64_t *bars = reinterpret_cast<uint64_t *>(Eend_s + 2);
-    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 11);
+    //       11, 12 Z and U of step parity written (their readout need not wait for dC / dB)
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 13);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
 
     const int tid = threadIdx.x, grp = tid >> 7, t = tid & 127, w = tid >> 5, w4 = w & 3;
@@ -752,6 +753,8 @@ __global__ void __launch_bounds__(kStLaunch, 1)
         mbar_init(&bars[8], kStThreads);
         mbar_init(&bars[9], kCdThreads);
         mbar_init(&bars[10], kCdThreads);
+        mbar_init(&bars[11], 1);
+        mbar_init(&bars[12], 1);
         *abort_s = 0;
         fence_barrier_init();
     }
@@ -839,7 +842,7 @@ __global__ void __launch_bounds__(kStLaunch, 1)
     // read out step j (its MMAs complete): Z (group 0) or U (group 1) against this row, and
     // dx[t, p] += s_m U_m[t, p] with group g taking p in [32 g, 32 g + 32)
     auto readout = [&](int j) {
-        if (!*abort_s && !mbar_wait(&bars[3 + (j & 1)], (j >> 1) & 1)) *abort_s = 1;
+        if (!*abort_s && !mbar_wait(&bars[11 + (j & 1)], (j >> 1) & 1)) *abort_s = 1;
         tc_fence_after();
         const int mj = j % K, hj = h_first + j / K;
         if (!*abort_s) {
@@ -936,6 +939,7 @@ __global__ void __launch_bounds__(kStLaunch, 1)
                 mma_bf16(tmem + zc + 64, desc_sw128(smem_u32(sB) + ko, 16, 1024),
                          desc_sw128(sD + to, 16, 1024), id64, ks > 0);
             }
+            mma_commit(&bars[11 + gb]);  // Z, U of step i: the readout may start
             const bool acc0 = intra || i > 0;
             for (int ks = 0; ks < 4; ++ks) {  // K = p
                 mma_bf16(tmem + colC, desc_sw128(g1 + ks * 32, 16, 1024), desc_sw128(sS + ks * 2048, 8192, 1024),
@@ -1041,7 +1045,8 @@ __global__ void __launch_bounds__(kStLaunch, 1)
 #pragma unroll
             for (int p = 0; p < 32; ++p) dxr[p] = 0.f;
         }
-        // generated operands of step i into buffer gb (step i - 2 has finished reading it)
+        // generated operands of step i into buffer gb, once step i - 2's MMAs have read it
+        if (i >= 2 && !*abort_s && !mbar_wait(&bars[3 + gb], ((i - 2) >> 1) & 1)) *abort_s = 1;
         {
             const float sc = my_coef[m];
             unsigned char *dst = sG + gb * L.gen + grp * 16384 + t * 128;
@@ -1058,6 +1063,11 @@ __global__ void __launch_bounds__(kStLaunch, 1)
     }
     if (nsteps > 0 && tid < kStThreads) readout(nsteps - 1);
     // the group's dC / dB into the float32 accumulators (group g takes n in [64 g, 64 g + 64))
+    tc_fence_after();
+    // every MMA (dC, dB of the last step included) has completed before the accumulators are read
+    if (tid < kStThreads && nsteps > 0 && !*abort_s &&
+        !mbar_wait(&bars[3 + ((nsteps - 1) & 1)], ((nsteps - 1) >> 1) & 1))
+        *abort_s = 1;
     tc_fence_after();
     // the group's dC / dB into the float32 accumulators by TMA reduce-add: every warp has left
     // the tiles and the generated operands, which now stage dC (generator buffers) and dB (tile
