@@ -145,12 +145,12 @@ def kpn(s):
 # only while the kernel's sources hash to the digest they had when they were profiled.
 PROFILED_TRAFFIC_BATCH = 2
 PROFILED_TRAFFIC = {
-    "coef_tc": ("scan_tc.cu", "3001ce054be74299", 23.103e6 + 9.001e6),
-    "state_pass_fwd_tc": ("scan_tc.cu", "3001ce054be74299", 137.495e6 + 477.948e6),
-    "chunk_fwd_tc": ("scan_tc.cu", "3001ce054be74299", 631.333e6 + 59.839e6),
-    "state_pass_rev_tc": ("scan_tc.cu", "3001ce054be74299", 137.340e6 + 478.024e6),
-    "bwd_intra_tc": ("scan_tc_bwd.cu", "d5477e9b592f55e7", 164.034e6 + 123.074e6),
-    "bwd_state_tc": ("scan_tc_bwd.cu", "d5477e9b592f55e7", 1461.271e6 + 172.064e6),
+    "coef_tc": ("scan_tc.cu", "09720b9f1cca6e42", 23.104e6 + 41.807e6),
+    "state_pass_fwd_tc": ("scan_tc.cu", "09720b9f1cca6e42", 137.385e6 + 481.808e6),
+    "chunk_fwd_tc": ("scan_tc.cu", "09720b9f1cca6e42", 717.406e6 + 61.123e6),
+    "state_pass_rev_tc": ("scan_tc.cu", "09720b9f1cca6e42", 137.387e6 + 481.919e6),
+    "bwd_intra_tc": ("scan_tc_bwd.cu", "cfa2234782159636", 182.944e6 + 125.978e6),
+    "bwd_state_tc": ("scan_tc_bwd.cu", "cfa2234782159636", 1472.593e6 + 170.162e6),
 }
 
 
