@@ -369,7 +369,7 @@ struct OutArgs {
 
 constexpr int kOutThreads = 256;  // two groups of four warps share the 128 TMEM lanes
 constexpr int kOutLaunch = kOutThreads + 32;  // a ninth warp issues the entering-state MMAs
-constexpr int kSBuf = 3;          // S_in tiles in flight
+constexpr int kSBuf = 3;          // 8 KB units of the S ring (the Gamma operands, then one S_in pair slot)
 
 // Shared-memory plan of tc_chunk_fwd (offsets from a 1024-aligned base): about 110 KB at
 // N = 128, so that two CTAs share an SM.
@@ -379,64 +379,76 @@ struct OutSmem {
         c = (N / 64) * 16384;  // C chunk [t][n], K-major, 64-wide n atoms
         m = 2 * 16384;         // B chunk, then Gamma o G [t][k]
         x = 16384;             // x chunk [t][p]: the MN-major operand of the intra MMA
-        s = kSBuf * 8192;      // S_in tiles, one (mode, 64-wide n half) each: [p][n]
+        s = kSBuf * 8192;      // U / V tf32 tiles of Gamma, then one S_in pair slot: [2 x 64 p][64 n]
         total = c + m + x + s + TQ * KMAX * 4 /*kappa*/ + TQ * 8 /*E*/ + 64 * 4 /*tau, l2t*/ +
                 64 /*wsum*/ + 24 * 8 /*bars*/ + 16 + 64 * KMAX * 4 /*V16*/;
     }
 };
 
 
-// The entering-state MMAs of tc_chunk_fwd (one thread of the ninth warp): S_in tiles j (mode
-// j / nhalf, 64-wide n half j % nhalf) stream through three buffers; Z_m = C S_in,m^T goes to
-// TMEM buffer m % 4 once the compute threads have read its previous contents.
+// The entering-state MMAs of tc_chunk_fwd (one thread of the ninth warp).  Two modes go
+// together: pair tile j = (mode pair j / nhalf, 64-wide n half j % nhalf) stacks the [64 p][64 n]
+// S_in tiles of modes 2 mp and 2 mp + 1 into one 16 KB slot, the B operand of one N = 128
+// product, so Z_{2mp}, Z_{2mp+1} = C S_in^T land side by side in TMEM buffer mp % 2 (128
+// columns) once the compute threads have read its previous contents.  Slots: the first 16 KB
+// of the S ring, then the two halves of the Gamma o G tile once the intra MMA has read it.
+// bars: 3 + s slot s loaded | 6 + s slot s read by its MMAs | 9 + zb Z buffer written |
+//       13 + zb Z buffer read by all compute threads (buffer 1: first the intra Y)
+constexpr int kZSlots = 3;
 __device__ __forceinline__ void chunk_fwd_issuer(const ScanDims &d, unsigned char *sC, unsigned char *sS,
-                                                 uint64_t *bars, volatile int *abort_s, uint32_t tmem,
-                                                 const CUtensorMap &mapS, int srow) {
-    const int nhalf = d.N / 64, ntile = d.K * nhalf;
+                                                 unsigned char *sM, uint64_t *bars, volatile int *abort_s,
+                                                 uint32_t tmem, const CUtensorMap &mapS, int srow) {
+    const int nhalf = d.N / 64, npair = d.K / 2, ntile = npair * nhalf;
+    auto slot = [&](int s) { return s == 0 ? sS : sM + (s - 1) * 16384; };
     auto load = [&](int j) {
-        mbar_arrive_expect_tx(&bars[3 + j % kSBuf], 8192u);
-        tma_load_3d(sS + (j % kSBuf) * 8192, &mapS, &bars[3 + j % kSBuf], (j % nhalf) * 64, 0, srow + j / nhalf);
+        const int s = j % kZSlots, mp = j / nhalf, hn = j % nhalf;
+        mbar_arrive_expect_tx(&bars[3 + s], 16384u);
+        tma_load_3d(slot(s), &mapS, &bars[3 + s], hn * 64, 0, srow + 2 * mp);
+        tma_load_3d(slot(s) + 8192, &mapS, &bars[3 + s], hn * 64, 0, srow + 2 * mp + 1);
     };
     // the S ring holds the Gamma operands until their MMAs are done
     if (!mbar_wait(&bars[1], 0)) {
         *abort_s = 1;
         return;
     }
-    for (int j = 0; j < min(kSBuf, ntile); ++j) load(j);
-    // the intra Y MMA (issued after the Gamma o G pass) frees the G and Gamma columns
+    if (ntile > 0) load(0);
+    // the intra Y MMA (issued after the Gamma o G pass) frees the G and Gamma columns and the
+    // Gamma o G tile
     if (!mbar_wait(&bars[2], 0)) {
         *abort_s = 1;
         return;
     }
+    for (int j = 1; j < min(kZSlots, ntile); ++j) load(j);
     tc_fence_after();
-    const uint32_t idZ = idesc_bf16(128, 64, false, false);
+    const uint32_t idZ = idesc_bf16(128, 128, false, false);
     for (int j = 0; j < ntile && !*abort_s; ++j) {
-        const int m = j / nhalf, hn = j % nhalf, zb = m & 3;
-        if (hn == 0) {  // buffer zb read by all compute threads (buffer 3: first the intra Y)
-            const int k = m >> 2;
-            if ((zb == 3 || k > 0) && !mbar_wait(&bars[13 + zb], (zb == 3 ? k : k - 1) & 1)) {
+        const int mp = j / nhalf, hn = j % nhalf, zb = mp & 1, s = j % kZSlots;
+        if (hn == 0) {  // buffer zb read by all compute threads (buffer 1: first the intra Y)
+            const int k = mp >> 1;
+            if ((zb == 1 || k > 0) && !mbar_wait(&bars[13 + zb], (zb == 1 ? k : k - 1) & 1)) {
                 *abort_s = 1;
                 break;
             }
         }
-        if (!mbar_wait(&bars[3 + j % kSBuf], (j / kSBuf) & 1)) {
+        if (!mbar_wait(&bars[3 + s], (j / kZSlots) & 1)) {
             *abort_s = 1;
             break;
         }
         tc_fence_after();
-        const uint32_t sa = smem_u32(sC) + hn * 16384, sb = smem_u32(sS) + (j % kSBuf) * 8192;
+        const uint32_t sa = smem_u32(sC) + hn * 16384, sb = smem_u32(slot(s));
         for (int ks = 0; ks < 4; ++ks)
-            mma_bf16(tmem + 64 * zb, desc_sw128(sa + ks * 32, 16, 1024), desc_sw128(sb + ks * 32, 16, 1024), idZ,
+            mma_bf16(tmem + 128 * zb, desc_sw128(sa + ks * 32, 16, 1024), desc_sw128(sb + ks * 32, 16, 1024), idZ,
                      (hn > 0 || ks > 0) ? 1u : 0u);
-        mma_commit(&bars[6 + j % kSBuf]);
+        mma_commit(&bars[6 + s]);
         if (hn == nhalf - 1) mma_commit(&bars[9 + zb]);
-        // tile j - 1's MMAs done: its buffer takes tile j + 2
-        if (j >= 1 && j + 2 < ntile) {
-            if (!mbar_wait(&bars[6 + (j - 1) % kSBuf], ((j - 1) / kSBuf) & 1)) {
+        // tile j - 1's MMAs done: its slot takes tile j + 2
+        if (j >= 1 && j - 1 + kZSlots < ntile) {
+            const int sp = (j - 1) % kZSlots;
+            if (!mbar_wait(&bars[6 + sp], ((j - 1) / kZSlots) & 1)) {
                 *abort_s = 1;
                 break;
             }
-            load(j + 2);
+            load(j - 1 + kZSlots);
         }
     }
 }
@@ -445,9 +457,9 @@ __device__ __forceinline__ void chunk_fwd_issuer(const ScanDims &d, unsigned cha
 //   Y  = (Gamma o C B^T) X                      (intra-chunk pairs, K = t; tensor memory)
 //   y  = Y + sum_m f_m o (C S_in,m^T) + D x     (entering state)
 // G = C B^T comes from the tensor cores; Gamma is formed per position pair.  A ninth warp
-// streams Z_m = C S_in,m^T through four 64-column TMEM buffers (S_in tiles by TMA, three ahead)
-// while the 256 compute threads fold each Z_m into their rows of y with the weight f_m[t]:
-// no per-mode scaled operand and no CTA-wide barrier per mode.
+// streams Z_m = C S_in,m^T, two modes per N = 128 product, through two 128-column TMEM buffers
+// (S_in tiles by TMA, two pair tiles ahead) while the 256 compute threads fold each Z_m into
+// their rows of y with the weight f_m[t]: no per-mode scaled operand and no CTA-wide barrier.
 __global__ void __launch_bounds__(kOutLaunch, 2)
     tc_chunk_fwd(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapB,
                  const __grid_constant__ CUtensorMap mapX, const __grid_constant__ CUtensorMap mapS,
@@ -485,7 +497,7 @@ __global__ void __launch_bounds__(kOutLaunch, 2)
 
     if (tid == 0) {
         for (int i = 0; i < 13; ++i) mbar_init(&bars[i], 1);
-        for (int i = 13; i < 17; ++i) mbar_init(&bars[i], kOutThreads);
+        for (int i = 13; i < 15; ++i) mbar_init(&bars[i], kOutThreads);
         *abort_s = 0;
         fence_barrier_init();
     }
@@ -545,10 +557,10 @@ __global__ void __launch_bounds__(kOutLaunch, 2)
     const uint32_t tmem = *tslot;
     const uint32_t lane_base = tmem + (uint32_t(w4 * 32) << 16);
     // TMEM: G = C B^T at [0, 128), the factored Gamma blocks at [128, 256); then the intra Y at
-    // [192, 256) and the Z_m buffers at 64 (m % 4) (buffer 3 once Y has been read)
+    // [192, 256) and the Z buffers of mode pairs at 128 (pair % 2) (buffer 1 once Y has been read)
     constexpr uint32_t colG = 0, colGam = 128, colY = 192;
     if (tid >= kOutThreads) {
-        if (tid == kOutThreads) chunk_fwd_issuer(a.d, sC, sS, bars, abort_s, tmem, mapS, srow);
+        if (tid == kOutThreads) chunk_fwd_issuer(a.d, sC, sS, sM, bars, abort_s, tmem, mapS, srow);
     } else {
 
     if (tid == 0) {
@@ -723,21 +735,22 @@ __global__ void __launch_bounds__(kOutLaunch, 2)
     tmem_ld32(lane_base + colY + grp * 32, yv);
     tmem_ld_wait();
     tc_fence_before();
-    mbar_arrive(&bars[13 + 3]);
+    mbar_arrive(&bars[13 + 1]);
 #pragma unroll
-    for (int m = 0; m < KMAX; ++m) {
-        if (m < K) {
-            const int zb = m & 3;
-            if (!*abort_s && !mbar_wait(&bars[9 + zb], (m >> 2) & 1)) *abort_s = 1;
+    for (int mp = 0; mp < KMAX / 2; ++mp) {
+        if (2 * mp < K) {
+            const int zb = mp & 1;
+            if (!*abort_s && !mbar_wait(&bars[9 + zb], (mp >> 1) & 1)) *abort_s = 1;
             tc_fence_after();
-            float zv[32];
-            tmem_ld32(lane_base + 64 * zb + grp * 32, zv);
+            float z0[32], z1[32];
+            tmem_ld32(lane_base + 128 * zb + grp * 32, z0);
+            tmem_ld32(lane_base + 128 * zb + 64 + grp * 32, z1);
             tmem_ld_wait();
             tc_fence_before();
             mbar_arrive(&bars[13 + zb]);
-            const float fm = f_t[m];
+            const float f0 = f_t[2 * mp], f1 = f_t[2 * mp + 1];
 #pragma unroll
-            for (int i = 0; i < 32; ++i) yv[i] = fmaf(fm, zv[i], yv[i]);
+            for (int i = 0; i < 32; ++i) yv[i] = fmaf(f1, z1[i], fmaf(f0, z0[i], yv[i]));
         }
     }
     {  // y = Y + sum_m f_m Z_m + D x (rows t >= n and aborted CTAs write nothing)
