@@ -6,7 +6,7 @@
 //   tc_coef        (one CTA per (b, h, chunk)): the per-position mode coefficients of the
 //        chunk (f, s = kappa u, u, exp(-E/tau) from the float-pair cumulative log-decay E), read
 //        by the state passes and the backward instead of being recomputed per P-slice.
-//   tc_state_pass  (chunk-serial; one CTA per (b, h, 128/K-wide slice of P), three per SM):
+//   tc_state_pass  (chunk-serial; one CTA of 256 threads per (b, h, 128/K-wide slice of P)):
 //        the P-slice of every mode's state lives in tensor memory as fp32, lanes = (mode, p),
 //        columns = n.  Per chunk: emit the entering state (bf16) for the output kernel, scale
 //        it by d_m = exp(-E_end/tau_m) in place, then accumulate
@@ -36,7 +36,6 @@ namespace {
 using namespace tc;
 using bf16 = __nv_bfloat16;
 
-constexpr int kThreads = 128;
 
 struct StateArgs {
     ScanDims d;
@@ -127,14 +126,14 @@ __global__ void __launch_bounds__(TQ) tc_coef(CoefArgs a) {
                             size_t(d.H) * EK * 4, n - te);
 }
 
-// Shared-memory plan of tc_state_pass (offsets from a 1024-aligned base): about 70 KB at N = 128,
-// so that three CTAs share an SM.
+// Shared-memory plan of tc_state_pass (offsets from a 1024-aligned base): about 83 KB at N = 128
+// (two CTAs share an SM).
 struct StateSmem {
     int a_bytes, v_bytes, total;
     __host__ __device__ explicit StateSmem(int N) {
         a_bytes = 2 * 16384;         // 2 M-atoms x (128 k rows x 128 B), MN-major
         v_bytes = (N / 64) * 16384;  // N/64 boxes of [128 t][64 n]
-        total = a_bytes + v_bytes + 4 * 2048 /*emit staging, one 2 KB tile per warp*/ + 32 * 4 /*dec*/ +
+        total = a_bytes + v_bytes + 8 * 2048 /*emit staging, one 2 KB tile per warp*/ + 32 * 4 /*dec*/ +
                 64 /*bars*/;
     }
 };
@@ -145,8 +144,12 @@ __host__ __device__ constexpr int state_tps() {
     return TQ / KK;
 }
 
+// Two groups of four warps share the 128 TMEM lanes: group g writes M-atom g of the A tile and
+// emits / decays the state columns [g N / 2, (g + 1) N / 2).
+constexpr int kSPThreads = 256;
+
 template <bool REV, int KK>
-__global__ void __launch_bounds__(kThreads, 3)
+__global__ void __launch_bounds__(kSPThreads, 2)
     tc_state_pass(const __grid_constant__ CUtensorMap mapV, const __grid_constant__ CUtensorMap mapE, StateArgs a) {
     constexpr int TPSK = state_tps<KK>();  // 16 (KK = 8) or 32 (KK = 4)
     constexpr int NX = TPSK / 8;           // 16-byte pieces of one position's x slice
@@ -158,20 +161,21 @@ __global__ void __launch_bounds__(kThreads, 3)
     const StateSmem plan(N);
     unsigned char *sA = base;
     unsigned char *sV = sA + plan.a_bytes;
-    unsigned char *sE = sV + plan.v_bytes;                          // [4 warps][32 rows x 64 B] emit staging
-    float *dec = reinterpret_cast<float *>(sE + 4 * 2048);          // [32] this chunk's decay per mode
+    unsigned char *sE = sV + plan.v_bytes;                          // [8 warps][32 rows x 64 B] emit staging
+    float *dec = reinterpret_cast<float *>(sE + 8 * 2048);          // [32] this chunk's decay per mode
     uint64_t *bars = reinterpret_cast<uint64_t *>(dec + 32);        // tma, mma
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 2);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
 
-    const int tid = threadIdx.x, w = tid >> 5, j = tid & 31;
+    const int tid = threadIdx.x, w = tid >> 5, j = tid & 31, grp = tid >> 7, t = tid & 127, w4 = w & 3;
     const int h = blockIdx.y, b = blockIdx.z, p0 = blockIdx.x * TPSK;
     const int g = h / (d.H / d.G);
     const uint32_t ncols = uint32_t(N);  // 64 or 128
     const size_t PN = size_t(P) * N;
     const size_t bh = size_t(b) * d.H + h;
-    // this thread's TMEM lane: mode lm, row p0 + lp of the slice
-    const int lm = tid / TPSK, lp = tid % TPSK;
+    // this thread's TMEM lane: mode lm, row p0 + lp of the slice; its column half
+    const int lm = t / TPSK, lp = t % TPSK;
+    const int nblk = N / 32, hb0 = grp * (nblk / 2);  // 32-column blocks [hb0, hb0 + nblk / 2)
 
     if (tid == 0) {
         mbar_init(&bars[0], 1);
@@ -184,12 +188,12 @@ __global__ void __launch_bounds__(kThreads, 3)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tslot;
-    const uint32_t lane_base = tmem + (uint32_t(w * 32) << 16);
+    const uint32_t lane_base = tmem + (uint32_t(w4 * 32) << 16);
 
-    // initial state into tensor memory: lane (mode, p), columns n
+    // initial state into tensor memory: lane (mode, p), columns n (this group's half)
     {
         const float *src = a.init ? a.init + (bh * KK + lm) * PN + size_t(p0 + lp) * N : nullptr;
-        for (int c8 = 0; c8 < N; c8 += 8) {
+        for (int c8 = 32 * hb0; c8 < 32 * hb0 + N / 2; c8 += 8) {
             float v[8];
 #pragma unroll
             for (int i = 0; i < 8; ++i) v[i] = src ? src[c8 + i] : 0.f;
@@ -198,16 +202,15 @@ __global__ void __launch_bounds__(kThreads, 3)
     }
     tmem_st_wait();
 
-    // Thread t owns chunk position t: its slice of x (or dy) and its coefficient per mode
-    // (s = kappa exp(-(E_end - E_t)/tau) forward, f = w_read exp(-E_t/tau) reverse) stay in
-    // registers, and the inputs of chunk ci + 1 are fetched while chunk ci is processed.
+    // Thread t of each group owns chunk position t: its slice of x (or dy) and its coefficient
+    // per mode (s = kappa exp(-(E_end - E_t)/tau) forward, f = w_read exp(-E_t/tau) reverse) stay
+    // in registers, and the inputs of chunk ci + 1 are fetched while chunk ci is processed.
     constexpr int NC = KK / 4;  // 16-byte pieces of one coefficient kind
     uint4 nx[NX], ncv[NC];
     float ndec = 0.f;
     auto fetch = [&](int ci_) {
         const int c_ = REV ? d.nc - 1 - ci_ : ci_;
         const int c0_ = c_ * TQ, n_ = min(TQ, d.L - c0_);
-        const int t = tid;
         {  // the slice's TPSK x values and the coefficient row, read row-coalesced (the lane
            // transposes that complete them wait until the chunk that uses them)
             const int tg = t & ~(NX - 1);
@@ -219,7 +222,7 @@ __global__ void __launch_bounds__(kThreads, 3)
                                                                   (REV ? 0 : KK)),
                           size_t(d.H) * 4 * KK * 4, n_ - tc);
         }
-        if (t < KK) ndec = a.coef[blh(d, b, c0_ + n_ - 1, h) * 4 * KK + 3 * KK + t];
+        if (tid < KK) ndec = a.coef[blh(d, b, c0_ + n_ - 1, h) * 4 * KK + 3 * KK + tid];
     };
     if (d.nc > 0) fetch(0);
 
@@ -227,7 +230,6 @@ __global__ void __launch_bounds__(kThreads, 3)
     for (int ci = 0; ci < d.nc; ++ci, phase ^= 1) {
         const int c = REV ? d.nc - 1 - ci : ci;
         const int c0 = c * TQ;
-        const int t = tid;
         uint4 xr[NX];
         float cv[KK];
 #pragma unroll
@@ -241,7 +243,7 @@ __global__ void __launch_bounds__(kThreads, 3)
             cv[4 * q + 2] = __uint_as_float(ncv[q].z);
             cv[4 * q + 3] = __uint_as_float(ncv[q].w);
         }
-        if (t < KK) dec[t] = ndec;  // the previous chunk's emit has passed the barrier before its MMAs
+        if (tid < KK) dec[tid] = ndec;  // the previous chunk's emit has passed the barrier before its MMAs
         if (ci + 1 < d.nc) fetch(ci + 1);
         if (ci > 0) {  // previous chunk's MMAs done: tensor memory, sA and sV are free
             if (!mbar_wait(&bars[1], phase ^ 1)) *abort_s = 1;
@@ -255,13 +257,12 @@ __global__ void __launch_bounds__(kThreads, 3)
                 tma_load_3d(sV + jb * 16384, &mapV, &bars[0], g * N + 64 * jb, c0, b);
         }
         // A[(m, p), k] = s_{k,m} x_{k,p} as bf16, MN-major: row k = this thread's position,
-        // 64-element M-atoms (64 / TPSK modes x TPSK p each), 128-byte swizzle
+        // 64-element M-atoms (64 / TPSK modes x TPSK p each), 128-byte swizzle; group g writes atom g
+        {
+            unsigned char *row = sA + grp * 16384 + t * 128;
 #pragma unroll
-        for (int ma = 0; ma < 2; ++ma) {
-            unsigned char *row = sA + ma * 16384 + t * 128;
-#pragma unroll
-            for (int c8 = 0; c8 < 8; ++c8) {  // elements M = 64 ma + 8 c8 ..: mode M / TPSK
-                const float s = cv[(64 * ma + 8 * c8) / TPSK];
+            for (int c8 = 0; c8 < 8; ++c8) {  // elements M = 64 grp + 8 c8 ..: mode M / TPSK
+                const float s = grp == 0 ? cv[(8 * c8) / TPSK] : cv[(64 + 8 * c8) / TPSK];
                 const uint4 xv = xr[c8 % NX];
                 const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
                 uint32_t r[4];
@@ -276,12 +277,11 @@ __global__ void __launch_bounds__(kThreads, 3)
         // emit the entering state (bf16) and apply the chunk's decay in place (the TMEM load of
         // the next 32 columns is in flight while the current ones are processed).  Each warp's 32
         // rows x 32 columns go through a 2 KB staging tile (64-byte swizzle) and one TMA store:
-        // rows (mode, p) of the warp are (32 w / TPSK + lane / TPSK, p0 + lane % TPSK).
+        // rows (mode, p) of the warp are (32 w4 / TPSK + lane / TPSK, p0 + lane % TPSK).
         {
-            const int nblk = N / 32;
             const float dm = dec[lm];
             unsigned char *stg = sE + w * 2048;
-            const int rowE = int((bh * d.nc + c) * KK + (32 * w) / TPSK);
+            const int rowE = int((bh * d.nc + c) * KK + (32 * w4) / TPSK);
             auto process = [&](float *v, int blk) {
                 if (j == 0) bulk_wait_read();  // the previous store has read the staging tile
                 __syncwarp();
@@ -302,14 +302,16 @@ __global__ void __launch_bounds__(kThreads, 3)
                 for (int q = 0; q < 4; ++q) tmem_st8(lane_base + 32 * blk + 8 * q, v + 8 * q);
             };
             float v0[32], v1[32];
-            tmem_ld32(lane_base, v0);
-            for (int blk = 0; blk < nblk; blk += 2) {  // nblk = N / 32 is even
+            tmem_ld32(lane_base + 32 * hb0, v0);
+            if (nblk == 4) {
                 tmem_ld_wait();
-                tmem_ld32(lane_base + 32 * (blk + 1), v1);
-                process(v0, blk);
+                tmem_ld32(lane_base + 32 * (hb0 + 1), v1);
+                process(v0, hb0);
                 tmem_ld_wait();
-                if (blk + 2 < nblk) tmem_ld32(lane_base + 32 * (blk + 2), v0);
-                process(v1, blk + 1);
+                process(v1, hb0 + 1);
+            } else {  // N = 64: one block per group
+                tmem_ld_wait();
+                process(v0, hb0);
             }
         }
         tmem_st_wait();
@@ -341,7 +343,7 @@ __global__ void __launch_bounds__(kThreads, 3)
     tc_fence_after();
     if (!*abort_s && a.fin) {
         float *dst = a.fin + (bh * KK + lm) * PN + size_t(p0 + lp) * N;
-        for (int c32 = 0; c32 < N; c32 += 32) {
+        for (int c32 = 32 * hb0; c32 < 32 * hb0 + N / 2; c32 += 32) {
             float v[32];
             tmem_ld32(lane_base + c32, v);
             tmem_ld_wait();
@@ -889,7 +891,7 @@ cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, con
     auto launch = [&](auto kern, int tps, const char *name) {
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
         trace_begin(name, st);
-        kern<<<dim3(d.P / tps, d.H, d.B), kThreads, smem, st>>>(mapV, mapE, a);
+        kern<<<dim3(d.P / tps, d.H, d.B), kSPThreads, smem, st>>>(mapV, mapE, a);
         trace_end(st);
     };
     if (d.K == 8) {
