@@ -126,13 +126,8 @@ __device__ __forceinline__ void get_rows(uint4 (&e)[NL], const unsigned char *ro
     lane_transpose<NL>(e, threadIdx.x & 31);
 }
 
-// Asynchronous global -> shared copies (cp.async, no register round trip): 4, 8 or 16 bytes,
+// Asynchronous global -> shared copy (cp.async, no register round trip) of 4, 8 or 16 bytes,
 // both addresses aligned to the size; completed by cp_async_wait_all.
-__device__ __forceinline__ void cp_async4(void *dst, const void *src) {
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
-                 "l"(src)
-                 : "memory");
-}
 __device__ __forceinline__ void cp_async_bytes(void *dst, const void *src, int bytes) {
     const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst));
     if (bytes == 16)
@@ -150,18 +145,6 @@ __device__ __forceinline__ void prefetch_l2(const void *p) {
     asm volatile("prefetch.global.L2 [%0];" ::"l"(reinterpret_cast<uint64_t>(p)));
 }
 
-// Inclusive prefix sum (double) of one value per thread over a 128-thread block.
-__device__ __forceinline__ double block_scan128(double v, double *wsum) {
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    v = warp_inclusive_scan_d(v);
-    if (lane == 31) wsum[w] = v;
-    __syncthreads();
-    double off = 0.0;
-    for (int i = 0; i < w; ++i) off += wsum[i];
-    __syncthreads();
-    return v + off;
-}
-
 // 2^x with the hardware approximation (relative error ~2^-22); exp(-d / tau) is evaluated as
 // 2^(-d * l2t) with l2t = log2(e) / tau precomputed.
 __device__ __forceinline__ float ex2_approx(float x) {
@@ -171,13 +154,8 @@ __device__ __forceinline__ float ex2_approx(float x) {
 }
 constexpr float kLog2e = 1.4426950408889634f;
 
-// A cumulative log-decay kept as an unevaluated float pair hi + lo (hi = E rounded to float):
-// the difference of two such values is accurate to float precision of the difference itself,
-// without a double-precision subtraction per pair.
-__device__ __forceinline__ float2 split_f2(double E) {
-    const float hi = float(E);
-    return make_float2(hi, float(E - double(hi)));
-}
+// A cumulative log-decay kept as an unevaluated float pair hi + lo: the difference of two such
+// values is accurate to float precision of the difference itself.
 __device__ __forceinline__ float diff_f2(float2 a, float2 b) { return (a.x - b.x) + (a.y - b.y); }
 
 // Float-pair (hi + lo) arithmetic for the cumulative log-decay: Knuth's TwoSum keeps the
@@ -196,18 +174,8 @@ __device__ __forceinline__ float2 f2_add(float2 a, float2 b) {
 // extra warps take no part in the per-position work.
 __device__ __forceinline__ void sync_first256() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
 
-template <bool FIRST256>
-__device__ __forceinline__ void block_or_first256_sync() {
-    if (FIRST256)
-        sync_first256();
-    else
-        __syncthreads();
-}
-
 // Inclusive prefix sum of one value per thread within groups of four warps (threads
 // 128 g .. 128 g + 127 scan independently), as a float pair; wsum holds one pair per warp.
-// FIRST256: only the first 256 threads call it (they synchronise on named barrier 1).
-template <bool FIRST256 = false>
 __device__ __forceinline__ float2 group_scan128_f2(float v, float2 *wsum) {
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
     float2 p = make_float2(v, 0.f);
@@ -217,26 +185,12 @@ __device__ __forceinline__ float2 group_scan128_f2(float v, float2 *wsum) {
         if (lane >= o) p = f2_add(p, u);
     }
     if (lane == 31) wsum[w] = p;
-    block_or_first256_sync<FIRST256>();
+    __syncthreads();
     float2 off = make_float2(0.f, 0.f);
     const int g0 = w & ~3;
     for (int i = g0; i < w; ++i) off = f2_add(off, wsum[i]);
-    block_or_first256_sync<FIRST256>();
+    __syncthreads();
     return f2_add(p, off);
-}
-
-// Inclusive prefix sum (double) of one value per thread within groups of four warps (threads
-// 128 g .. 128 g + 127 scan independently); wsum holds one slot per warp.
-__device__ __forceinline__ double group_scan128(double v, double *wsum) {
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    v = warp_inclusive_scan_d(v);
-    if (lane == 31) wsum[w] = v;
-    __syncthreads();
-    double off = 0.0;
-    const int g0 = w & ~3;
-    for (int i = g0; i < w; ++i) off += wsum[i];
-    __syncthreads();
-    return v + off;
 }
 
 }  // namespace frac
