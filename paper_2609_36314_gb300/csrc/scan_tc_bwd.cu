@@ -668,9 +668,12 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
 // One CTA per (b, c, group of hg heads of one B/C group), 256 compute threads plus an issuing warp
 // and three dot-product warps, software-pipelined over the (head, mode) steps.  Step i, with the
 // mode's S_in and dS_out tiles [p][n] streamed in by TMA (two buffers):
-//   Z_m = C S_in,m^T,  U_m = B dS_out,m^T                  (TMEM, two buffers of 2 x 64 columns)
+//   Z_m = C S_in,m^T,  U_m = B dS_out,m^T                  (TMEM, one buffer of 2 x 64 columns)
 //   dC += (f_m o dY) S_in,m,  dB += (s_m o X) dS_out,m       (TMEM, summed over modes and heads)
-// While the tensor cores run step i, the threads read out step i - 1: group 0 contracts Z_m with
+// The generated operands f_m o dY and s_m o X are written by the threads straight into TMEM (each
+// thread owns the lane of its row; two buffers) and feed the dC / dB MMAs as the A operand, so
+// they cost no shared-memory traffic.  Step i's Z / U MMAs start once step i - 1 has been read
+// out; the threads read out step i - 1 after writing step i's operands: group 0 contracts Z_m with
 // its dY row (dw_read, the a term), group 1 contracts U_m with its X row (dkappa, the b term) and
 // accumulates dx = sum_m s_m U_m in registers.  Three more warps form <dS_out,m, S_in,m> from the
 // two tiles in shared memory.  The head-summed intra tile Gamma o H adds M_H B to dC and M_H^T C to dB once
@@ -687,7 +690,7 @@ struct StSmem {
     __host__ __device__ explicit StSmem(int N) {
         cb = (N / 64) * 16384;   // one of C / B: [t][n]
         tile = (N / 64) * 8192;  // one S_in or dS_out mode tile: [p = 64][n], 64-wide n atoms
-        gen = 2 * 16384;         // f o dY and s o X: [t][p] each; two buffers (the first holds M_H)
+        gen = 2 * 16384;         // two units: M_H [t][k] at the start, dC staging at the end
         total = 2 * cb + kStBuf * 2 * tile + 2 * gen + kStThreads * kCoefStride * 4 + 384;
     }
 };
@@ -732,9 +735,11 @@ __global__ void __launch_bounds__(kStLaunch, 1)
     double *Eend_s = wsum + 8;                                  // [1]
     // bars: 0..2 tile buffers | 3, 4 MMA of step parity | 5 C, B | 6 intra MMA |
     //       7, 8 generated operands of step parity written (all 256 threads arrive) |
-    //       9, 10 tile buffer read by the <dS_out, S_in> warps (all 96 threads arrive)
+    //       9, 10 tile buffer released: read by the <dS_out, S_in> warps (all 96 threads arrive)
+    //             and by every MMA of its step (one arrival from the issuer's commit)
     uint64_t *bars = reinterpret_cast<uint64_t *>(Eend_s + 2);
-    //       11, 12 Z and U of step parity written (their readout need not wait for dC / dB)
+    //       11 Z and U of the step written (their readout need not wait for dC / dB) |
+    //       12 Z and U of the step read out (all 256 threads arrive)
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 13);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
 
@@ -745,16 +750,18 @@ __global__ void __launch_bounds__(kStLaunch, 1)
     const int c0 = c * TQ, n = min(TQ, d.L - c0);
     const int nsteps = a.hg * K;
     const bool intra = (h_first % (d.H / d.G)) == 0;
-    constexpr uint32_t colC = 0, colB = 128, colZU = 256;  // Z / U of buffer q at 256 + 128 q (+ 64)
+    // TMEM columns: dC, dB accumulators; Z (+0) and U (+64); generated operands of buffer gb at
+    // colG + 64 gb, f o dY (+0, group 0) and s o X (+32, group 1) as packed bf16 pairs
+    constexpr uint32_t colC = 0, colB = 128, colZU = 256, colG = 384;
 
     if (tid == 0) {
         for (int i = 0; i < 7; ++i) mbar_init(&bars[i], 1);
         mbar_init(&bars[7], kStThreads);
         mbar_init(&bars[8], kStThreads);
-        mbar_init(&bars[9], kCdThreads);
-        mbar_init(&bars[10], kCdThreads);
+        mbar_init(&bars[9], kCdThreads + 1);
+        mbar_init(&bars[10], kCdThreads + 1);
         mbar_init(&bars[11], 1);
-        mbar_init(&bars[12], 1);
+        mbar_init(&bars[12], kStThreads);
         *abort_s = 0;
         fence_barrier_init();
     }
@@ -767,7 +774,7 @@ __global__ void __launch_bounds__(kStLaunch, 1)
     const uint32_t lane_base = tmem + (uint32_t(w4 * 32) << 16);
 
     const bool issuer = tid == kStThreads;  // lane 0 of the ninth warp
-    auto issue_tiles = [&](int i) {  // issuer: S_in / dS_out tiles of step i into buffer i % 3
+    auto issue_tiles = [&](int i) {  // S_in / dS_out tiles of step i into buffer i % kStBuf
         const int q = i % kStBuf;
         const int srow = int(((size_t(b) * d.H + h_first + i / K) * d.nc + c) * K + i % K);
         mbar_arrive_expect_tx(&bars[q], uint32_t(2 * L.tile));
@@ -842,11 +849,11 @@ __global__ void __launch_bounds__(kStLaunch, 1)
     // read out step j (its MMAs complete): Z (group 0) or U (group 1) against this row, and
     // dx[t, p] += s_m U_m[t, p] with group g taking p in [32 g, 32 g + 32)
     auto readout = [&](int j) {
-        if (!*abort_s && !mbar_wait(&bars[11 + (j & 1)], (j >> 1) & 1)) *abort_s = 1;
+        if (!*abort_s && !mbar_wait(&bars[11], j & 1)) *abort_s = 1;
         tc_fence_after();
         const int mj = j % K, hj = h_first + j / K;
         if (!*abort_s) {
-            const uint32_t zu = lane_base + colZU + 128 * (j & 1);  // Z at +0, U at +64
+            const uint32_t zu = lane_base + colZU;  // Z at +0, U at +64
             const float sj = my_coef[2 * KMAX + mj], aj = my_coef[mj], bj = my_coef[KMAX + mj];
             float dp[4] = {0.f, 0.f, 0.f, 0.f};  // independent partial sums
 #pragma unroll
@@ -879,6 +886,8 @@ __global__ void __launch_bounds__(kStLaunch, 1)
                     for (int i = 0; i < 16; ++i) dxr[16 * pc + i] = fmaf(sj, zv[i], dxr[16 * pc + i]);
                 }
             }
+            tc_fence_before();
+            mbar_arrive(&bars[12]);  // the Z / U columns may take step j + 1
             const float dotv = (dp[0] + dp[1]) + (dp[2] + dp[3]);
 #pragma unroll
             for (int m = 0; m < KMAX; ++m) {
@@ -907,48 +916,51 @@ __global__ void __launch_bounds__(kStLaunch, 1)
     };
 
     if (issuer) {
-        // the MMAs of step i once all compute threads have written its generated operands; then,
-        // once step i - 1 has finished, its tile buffer takes the tiles of step i + 2
+        // step i: Z / U once its tiles are in and step i - 1 has been read out, then dC / dB once
+        // the threads have written step i's generated operands into TMEM; the descriptors of the
+        // K slices are fixed offsets from those of the operands
+        const uint32_t id64 = idesc_bf16(128, 64, false, false);
+        const uint32_t idN = idesc_bf16(128, N, false, true);
+        const uint64_t dC0 = desc_sw128(smem_u32(sC), 16, 1024), dB0 = desc_sw128(smem_u32(sB), 16, 1024);
+        const int nks = N / 16;
         for (int i = 0; i < nsteps && !*abort_s; ++i) {
             const int gb = i & 1, q = i % kStBuf;
-            // step i - 1's MMAs are done (they were issued at the tensor cores' pace): its tile
-            // buffer takes the tiles of step i - 1 + kStBuf before step i's operands are awaited
-            if (i >= 1) {
-                const int qp = (i - 1) % kStBuf;
-                if (!mbar_wait(&bars[3 + ((i - 1) & 1)], ((i - 1) >> 1) & 1) ||
-                    !mbar_wait(&bars[9 + qp], ((i - 1) / kStBuf) & 1)) {
-                    *abort_s = 1;
-                    break;
-                }
-                if (i - 1 + kStBuf < nsteps) issue_tiles(i - 1 + kStBuf);
-            }
-            if (!mbar_wait(&bars[7 + gb], (i >> 1) & 1) || !mbar_wait(&bars[q], (i / kStBuf) & 1)) {
+            if (!mbar_wait(&bars[q], (i / kStBuf) & 1) || (i >= 1 && !mbar_wait(&bars[12], (i - 1) & 1))) {
                 *abort_s = 1;
                 break;
             }
             tc_fence_after();
             const uint32_t sS = smem_u32(sT + (2 * q) * L.tile), sD = smem_u32(sT + (2 * q + 1) * L.tile);
-            const uint32_t g1 = smem_u32(sG + gb * L.gen), g2 = g1 + 16384;
-            const uint32_t id64 = idesc_bf16(128, 64, false, false);
-            const uint32_t idN = idesc_bf16(128, N, false, true);
-            const uint32_t zc = colZU + 128 * gb;
-            for (int ks = 0; ks < N / 16; ++ks) {
-                const uint32_t ko = (ks / 4) * 16384 + (ks % 4) * 32, to = (ks / 4) * 8192 + (ks % 4) * 32;
-                mma_bf16(tmem + zc, desc_sw128(smem_u32(sC) + ko, 16, 1024), desc_sw128(sS + to, 16, 1024),
-                         id64, ks > 0);
-                mma_bf16(tmem + zc + 64, desc_sw128(smem_u32(sB) + ko, 16, 1024),
-                         desc_sw128(sD + to, 16, 1024), id64, ks > 0);
+            const uint64_t dS = desc_sw128(sS, 16, 1024), dD = desc_sw128(sD, 16, 1024);
+#pragma unroll
+            for (int ks = 0; ks < 8; ++ks) {
+                if (ks < nks) {
+                    const uint32_t ko = (ks / 4) * 16384 + (ks % 4) * 32, to = (ks / 4) * 8192 + (ks % 4) * 32;
+                    mma_bf16(tmem + colZU, desc_add(dC0, ko), desc_add(dS, to), id64, ks > 0);
+                    mma_bf16(tmem + colZU + 64, desc_add(dB0, ko), desc_add(dD, to), id64, ks > 0);
+                }
             }
-            mma_commit(&bars[11 + gb]);  // Z, U of step i: the readout may start
-            const bool acc0 = intra || i > 0;
-            for (int ks = 0; ks < 4; ++ks) {  // K = p
-                mma_bf16(tmem + colC, desc_sw128(g1 + ks * 32, 16, 1024), desc_sw128(sS + ks * 2048, 8192, 1024),
-                         idN, (acc0 || ks > 0) ? 1u : 0u);
-                mma_bf16(tmem + colB, desc_sw128(g2 + ks * 32, 16, 1024), desc_sw128(sD + ks * 2048, 8192, 1024),
-                         idN, (acc0 || ks > 0) ? 1u : 0u);
+            mma_commit(&bars[11]);  // Z, U of step i: the readout may start
+            if (!mbar_wait(&bars[7 + gb], (i >> 1) & 1)) {
+                *abort_s = 1;
+                break;
             }
-            mma_commit(&bars[3 + gb]);
+            tc_fence_after();
+            const uint32_t g1 = tmem + colG + 64 * gb, g2 = g1 + 32;
+            const uint64_t dSn = desc_sw128(sS, 8192, 1024), dDn = desc_sw128(sD, 8192, 1024);
+            const uint32_t acc0 = (intra || i > 0) ? 1u : 0u;
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks) {  // K = p, 16 per MMA: 8 columns of packed pairs
+                mma_bf16_ts(tmem + colC, g1 + 8 * ks, desc_add(dSn, ks * 2048), idN, ks > 0 ? 1u : acc0);
+                mma_bf16_ts(tmem + colB, g2 + 8 * ks, desc_add(dDn, ks * 2048), idN, ks > 0 ? 1u : acc0);
+            }
+            mma_commit(&bars[9 + q]);   // the tile buffer, once every MMA of step i has read it
+            mma_commit(&bars[3 + gb]);  // the generated operands of buffer gb, and dC / dB
         }
+        // the releases of the last tile buffers complete before the CTA ends (nothing else waits
+        // for them)
+        for (int i = max(0, nsteps - kStBuf); i < nsteps && !*abort_s; ++i)
+            if (!mbar_wait(&bars[9 + i % kStBuf], (i / kStBuf) & 1)) *abort_s = 1;
     }
     if (tid >= kStThreads + 32) {
         // <dS_out,m, S_in,m> of every step from its two tiles (the same swizzle in both), then the
@@ -956,7 +968,8 @@ __global__ void __launch_bounds__(kStLaunch, 1)
         const int ct = tid - (kStThreads + 32);
         for (int i = 0; i < nsteps; ++i) {
             const int q = i % kStBuf;
-            if (*abort_s || !mbar_wait(&bars[q], (i / kStBuf) & 1)) {
+            // the warp leaves together (its lanes meet in the shuffles below)
+            if (!__all_sync(0xffffffffu, !*abort_s && mbar_wait(&bars[q], (i / kStBuf) & 1))) {
                 *abort_s = 1;
                 break;
             }
@@ -983,6 +996,13 @@ __global__ void __launch_bounds__(kStLaunch, 1)
             const float v = warp_sum(acc0 + acc1);
             if ((tid & 31) == 0)
                 atomicAdd(a.cdot + ((size_t(b) * d.H + h_first + i / K) * d.nc + c) * K + i % K, v);
+            // the tile buffer of step i takes the tiles of step i + kStBuf once it is released
+            if (ct == 0 && i + kStBuf < nsteps) {
+                if (*abort_s || !mbar_wait(&bars[9 + q], (i / kStBuf) & 1))
+                    *abort_s = 1;
+                else
+                    issue_tiles(i + kStBuf);
+            }
         }
     }
     for (int i = 0; i < nsteps && tid < kStThreads; ++i) {
@@ -1045,17 +1065,26 @@ __global__ void __launch_bounds__(kStLaunch, 1)
 #pragma unroll
             for (int p = 0; p < 32; ++p) dxr[p] = 0.f;
         }
-        // generated operands of step i into buffer gb, once step i - 2's MMAs have read it
+        // generated operands of step i into TMEM buffer gb (this thread's lane), once step i - 2's
+        // MMAs have read it
         if (i >= 2 && !*abort_s && !mbar_wait(&bars[3 + gb], ((i - 2) >> 1) & 1)) *abort_s = 1;
+        tc_fence_after();
         {
             const float sc = my_coef[m];
-            unsigned char *dst = sG + gb * L.gen + grp * 16384 + t * 128;
+            const uint32_t dst = lane_base + colG + 64 * gb + 32 * grp;
 #pragma unroll
-            for (int k = 0; k < 8; ++k)
-                *reinterpret_cast<uint4 *>(dst + ((k ^ (t & 7)) * 16)) = scale_bf16x8(row[k], sc);
+            for (int hf = 0; hf < 2; ++hf) {
+                uint32_t v[16];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const uint4 g = scale_bf16x8(row[4 * hf + k], sc);
+                    v[4 * k] = g.x; v[4 * k + 1] = g.y; v[4 * k + 2] = g.z; v[4 * k + 3] = g.w;
+                }
+                tmem_st16(dst + 16 * hf, v);
+            }
+            tmem_st_wait();
         }
         // hand the generated operands to the MMA issuer (no CTA-wide barrier in the loop)
-        fence_async_smem();
         tc_fence_before();
         mbar_arrive(&bars[7 + gb]);
         // step i - 1 is read out while the tensor cores run step i

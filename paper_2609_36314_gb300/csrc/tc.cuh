@@ -129,6 +129,17 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64
         "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
+// D[tmem] (+)= A[tmem] * B[smem desc], bf16 inputs, fp32 accumulation; one thread issues. A is
+// M = 128 rows on lanes 0..127 of the columns at a_tmem, K-major: column a_tmem + j of lane r
+// holds A[r][2j] (low half) and A[r][2j + 1] (high half).
+__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
+                                            uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
 // Arrive on `bar` once every previously issued MMA of this thread has completed.
 __device__ __forceinline__ void mma_commit(uint64_t *bar) {
     asm volatile(
@@ -206,6 +217,15 @@ __device__ __forceinline__ void tmem_st8(uint32_t taddr, const float *v) {
                  "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7]))
                  : "memory");
 }
+// 16 consecutive 32-bit columns of this thread's lane.
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t *v) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+        "%14,%15,%16};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+        "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+        : "memory");
+}
 __device__ __forceinline__ void tmem_st_wait() {
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
@@ -222,6 +242,13 @@ __device__ __forceinline__ uint64_t desc_sw128(uint32_t smem_addr, uint32_t lbo_
     d |= uint64_t(1) << 46;
     d |= uint64_t(2) << 61;
     return d;
+}
+
+// A descriptor whose start address is `bytes` further on (a multiple of 16; the address field
+// does not overflow for shared-memory addresses below 256 KB, so only the low word changes).
+__device__ __forceinline__ uint64_t desc_add(uint64_t d, uint32_t bytes) {
+    const uint32_t lo = uint32_t(d) + (bytes >> 4), hi = uint32_t(d >> 32);
+    return (uint64_t(hi) << 32) | lo;
 }
 
 // Instruction descriptor of tcgen05.mma kind::f16: bf16 A and B, fp32 D, M x N tile;
