@@ -71,6 +71,10 @@ cudaError_t tc_state_pass_launch(const ScanDims &d, bool rev, const void *U, con
 bool tc_make_map3(CUtensorMap *m, const void *ptr, uint64_t d0, uint64_t d1, uint64_t d2,
                   uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1,
                   uint32_t b2, int swizzle_bytes = 128);
+// 3-D float32 tensor map with 128- or 64-byte swizzle (b0 = 32 or 16 floats)
+bool tc_make_map3_f32(CUtensorMap *m, const void *ptr, uint64_t d0, uint64_t d1, uint64_t d2,
+                      uint64_t stride1_bytes, uint64_t stride2_bytes, uint32_t b0, uint32_t b1,
+                      uint32_t b2, int swizzle_bytes);
 // 4-D float32 tensor map with 128-byte swizzle (box[0] = 32 floats)
 bool tc_make_map4_f32(CUtensorMap *m, const void *ptr, const uint64_t dims[4], const uint64_t strides_bytes[3],
                       const uint32_t box[4]);

@@ -684,6 +684,11 @@ constexpr int kCdThreads = 96;   // three more warps form <dS_out,m, S_in,m> fro
 constexpr int kStLaunch = kStThreads + 32 + kCdThreads;
 constexpr int kStBuf = 2;   // S_in / dS_out tile buffers
 constexpr int kCoefStride = 3 * KMAX + 1;  // per-thread coefficient row (odd: no bank conflicts)
+// the next head's inputs staged by TMA in the generator region: dY [128 t][64 p] and X (bf16,
+// 128-byte rows), then the coefficient rows [128 t][4 K] (fp32, 128- or 64-byte rows), each
+// with the TMA swizzle so that eight threads reading the same chunk of their rows hit distinct
+// banks
+constexpr int kStageX = 16384, kStageCoef = 32768;
 
 struct StSmem {
     int cb, tile, gen, total;
@@ -720,7 +725,8 @@ __global__ void __launch_bounds__(kStLaunch, 1)
     tc_bwd_state(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapB,
                  const __grid_constant__ CUtensorMap mapS, const __grid_constant__ CUtensorMap mapD,
                  const __grid_constant__ CUtensorMap mapdC, const __grid_constant__ CUtensorMap mapdB,
-                 BwdArgs a) {
+                 const __grid_constant__ CUtensorMap mapDY, const __grid_constant__ CUtensorMap mapX,
+                 const __grid_constant__ CUtensorMap mapCf, BwdArgs a) {
     extern __shared__ unsigned char smem_raw[];
     unsigned char *base = align1024(smem_raw);
     const ScanDims &d = a.d;
@@ -739,8 +745,8 @@ __global__ void __launch_bounds__(kStLaunch, 1)
     //             and by every MMA of its step (one arrival from the issuer's commit)
     uint64_t *bars = reinterpret_cast<uint64_t *>(Eend_s + 2);
     //       11 Z and U of the step written (their readout need not wait for dC / dB) |
-    //       12 Z and U of the step read out (all 256 threads arrive)
-    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 13);
+    //       12 Z and U of the step read out (all 256 threads arrive) | 13 next head staged
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 14);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
 
     const int tid = threadIdx.x, grp = tid >> 7, t = tid & 127, w = tid >> 5, w4 = w & 3;
@@ -762,6 +768,7 @@ __global__ void __launch_bounds__(kStLaunch, 1)
         mbar_init(&bars[10], kCdThreads + 1);
         mbar_init(&bars[11], 1);
         mbar_init(&bars[12], kStThreads);
+        mbar_init(&bars[13], 1);
         *abort_s = 0;
         fence_barrier_init();
     }
@@ -983,16 +990,6 @@ __global__ void __launch_bounds__(kStLaunch, 1)
             }
             if (k < L.tile / 16) acc0 = dot_bf16x8(ps[k], pd[k], acc0);
             mbar_arrive(&bars[9 + q]);
-            if (i % K == 1 && i / K + 1 < a.hg) {  // the next head's dY, X and coefficient rows into L2
-                const int hn = h_first + i / K + 1;
-                for (int r = ct; r < 3 * TQ; r += kCdThreads) {
-                    const int tr = min(r % TQ, n - 1), kind = r / TQ;
-                    const size_t ir = blh(d, b, c0 + tr, hn);
-                    prefetch_l2(kind == 0 ? static_cast<const void *>(a.dy + ir * P)
-                                          : kind == 1 ? static_cast<const void *>(a.x + ir * P)
-                                                      : static_cast<const void *>(a.coef + ir * 4 * K));
-                }
-            }
             const float v = warp_sum(acc0 + acc1);
             if ((tid & 31) == 0)
                 atomicAdd(a.cdot + ((size_t(b) * d.H + h_first + i / K) * d.nc + c) * K + i % K, v);
@@ -1017,6 +1014,27 @@ __global__ void __launch_bounds__(kStLaunch, 1)
             }
 #pragma unroll
             for (int k = 0; k < KMAX; ++k) acc_h[k] = 0.f;
+            if (hh > 0) {
+                // from the staged tiles: this thread's row of dY / X and its coefficient pieces
+                // (group 0: f, exp(-E/tau), s; group 1: s, u, s), unswizzled
+                if (!*abort_s && !mbar_wait(&bars[13], (hh - 1) & 1)) *abort_s = 1;
+                const unsigned char *ry = sG + (grp == 0 ? 0 : kStageX) + t * 128;
+#pragma unroll
+                for (int k = 0; k < 8; ++k) row[k] = *reinterpret_cast<const uint4 *>(ry + ((k ^ (t & 7)) * 16));
+                const unsigned char *rc = sG + kStageCoef + t * (16 * K);
+                const int kinds[3] = {grp == 0 ? 0 : 1, grp == 0 ? 3 : 2, 1};  // f s u exp(-E/tau) = 0 1 2 3
+#pragma unroll
+                for (int k = 0; k < 3; ++k)
+                    for (int j = 0; j < K / 4; ++j) {
+                        const int ch = kinds[k] * (K / 4) + j;
+                        const int cs = K == 8 ? (ch ^ (t & 7)) : (ch ^ ((t >> 1) & 3));
+                        const float4 v = *reinterpret_cast<const float4 *>(rc + cs * 16);
+                        float *dst = my_coef + k * KMAX + 4 * j;
+                        dst[0] = v.x; dst[1] = v.y; dst[2] = v.z; dst[3] = v.w;
+                    }
+                fence_async_smem();
+                sync_first256();  // every row is out of the staged tiles
+            } else {
             // coefficients of this row from tc_coef (group 0: f, exp(-E/tau); group 1: s, u;
             // both: s) and its row of dY / X, read row-coalesced across each 8-lane group
             const int t8 = t & ~7;
@@ -1060,6 +1078,13 @@ __global__ void __launch_bounds__(kStLaunch, 1)
             for (int k = 0; k < 6; ++k) {  // this thread's row: scalar stores (the row stride is odd)
                 float *dst = my_coef + (k >> 1) * KMAX + (k & 1) * 4;
                 dst[0] = c4[k].x; dst[1] = c4[k].y; dst[2] = c4[k].z; dst[3] = c4[k].w;
+            }
+            }
+            if (tid == 0 && hh + 1 < a.hg) {  // the next head's dY, X and coefficient tiles
+                mbar_arrive_expect_tx(&bars[13], uint32_t(2 * 16384 + TQ * 16 * K));
+                tma_load_3d(sG, &mapDY, &bars[13], (h + 1) * P, c0, b);
+                tma_load_3d(sG + kStageX, &mapX, &bars[13], (h + 1) * P, c0, b);
+                tma_load_3d(sG + kStageCoef, &mapCf, &bars[13], (h + 1) * 4 * K, c0, b);
             }
             ab_h = 0.f;
 #pragma unroll
@@ -1356,7 +1381,7 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
         return e;
     if (d.nc == 0) return cudaSuccess;
     const uint64_t GN = uint64_t(d.G) * d.N, HP = uint64_t(d.H) * d.P;
-    CUtensorMap mapC, mapB, mapX, mapDY, mapS, mapD, mapdC, mapdB;
+    CUtensorMap mapC, mapB, mapX, mapDY, mapS, mapD, mapdC, mapdB, mapCf;
     const uint64_t srows = uint64_t(d.B) * d.H * d.nc * d.K;
     if (!tc_make_map3(&mapC, p.Cm, GN, d.L, d.B, GN * 2, uint64_t(d.L) * GN * 2, 64, TQ, 1) ||
         !tc_make_map3(&mapB, p.Bm, GN, d.L, d.B, GN * 2, uint64_t(d.L) * GN * 2, 64, TQ, 1) ||
@@ -1365,7 +1390,10 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
         !tc_make_map3(&mapS, ws.S_in, d.N, d.P, srows, uint64_t(d.N) * 2, uint64_t(d.P) * d.N * 2, 64,
                       64, 1) ||
         !tc_make_map3(&mapD, ws.dS_out, d.N, d.P, srows, uint64_t(d.N) * 2, uint64_t(d.P) * d.N * 2, 64,
-                      64, 1))
+                      64, 1) ||
+        // per-position coefficients [B, L, H, 4 K] as (h 4K, l, b); a box is one head's 128 rows
+        !tc_make_map3_f32(&mapCf, ws.coef, uint64_t(d.H) * 4 * d.K, d.L, d.B, uint64_t(d.H) * 4 * d.K * 4,
+                          uint64_t(d.L) * d.H * 4 * d.K * 4, 4 * d.K, TQ, 1, d.K == 8 ? 128 : 64))
         return cudaErrorInvalidValue;
     {  // dC / dB float32 accumulators [B, L, G, N] as (n, g, l, b); a box is 32 n x 128 positions
         const uint64_t dims[4] = {uint64_t(d.N), uint64_t(d.G), uint64_t(d.L), uint64_t(d.B)};
@@ -1410,7 +1438,7 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
         cudaFuncSetAttribute(tc_bwd_state, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
         trace_begin("bwd_state_tc", st);
         tc_bwd_state<<<dim3(d.H / a.hg, d.nc, d.B), kStLaunch, smem, st>>>(mapC, mapB, mapS, mapD, mapdC, mapdB,
-                                                                              a);
+                                                                              mapDY, mapX, mapCf, a);
         trace_end(st);
         if ((e = cudaGetLastError())) return e;
     }
