@@ -103,8 +103,8 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     float *Vs = part + TQ * KMAX;                            // [128][KMAX] kappa exp(-(E_a - E_k)/tau)
     float2 *E_s = reinterpret_cast<float2 *>(Vs + TQ * KMAX);  // hi / lo pairs
     float *l2t = reinterpret_cast<float *>(E_s + TQ);
-    float *tau_s = l2t + 32;
-    float2 *wsum = reinterpret_cast<float2 *>(tau_s + 32);
+    float *inv_tau_s = l2t + 32;  // 1 / tau per mode
+    float2 *wsum = reinterpret_cast<float2 *>(inv_tau_s + 32);
     // bars: 0 C, B, x of the item loaded | 1 G, H, Gamma MMAs done | 2 dx MMA done | 3 dy loaded
     uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 4);
@@ -211,7 +211,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         }
         if (tid < K) {
             const float tv = pf_tau[tid];
-            tau_s[tid] = tv;
+            inv_tau_s[tid] = 1.f / tv;
             l2t[tid] = kLog2e / tv;
         }
         __syncthreads();  // the staging area is free again: the next item's inputs
@@ -240,11 +240,13 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
             unsigned char *row = sU + t * 128;
 #pragma unroll
             for (int J = 0; J < 4; ++J) {
-                uint32_t u[8];
-                const float dE = diff_f2(Et2, E_s[32 * J + 31]);
+                uint32_t u[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+                if (J < I) {  // blocks at or above the row's own are zero (I is uniform in a warp)
+                    const float dE = diff_f2(Et2, E_s[32 * J + 31]);
 #pragma unroll
-                for (int m = 0; m < KMAX; ++m)
-                    u[m] = (J < I && m < K && t < n) ? to_tf32(wr_t[m] * ex2_approx(-dE * l2r[m])) : 0u;
+                    for (int m = 0; m < KMAX; ++m)
+                        u[m] = (m < K && t < n) ? to_tf32(wr_t[m] * ex2_approx(-dE * l2r[m])) : 0u;
+                }
                 *reinterpret_cast<uint4 *>(row + (((2 * J) ^ (t & 7)) * 16)) = make_uint4(u[0], u[1], u[2], u[3]);
                 *reinterpret_cast<uint4 *>(row + (((2 * J + 1) ^ (t & 7)) * 16)) = make_uint4(u[4], u[5], u[6], u[7]);
             }
@@ -263,7 +265,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
                 const float vv = m < K ? kap_t[m] * ex2_approx(-dE * l2r[m]) : 0.f;
                 Vs[t * KMAX + m] = vv;
                 v[m] = to_tf32(vv);
-                vp[m] = m < K ? to_tf32(vv / tau_s[m]) : 0u;
+                vp[m] = m < K ? to_tf32(vv * inv_tau_s[m]) : 0u;
             }
             unsigned char *row = sV + r * 128, *rowp = sVp + r * 128;
             *reinterpret_cast<uint4 *>(row + (((2 * J) ^ (r & 7)) * 16)) = make_uint4(v[0], v[1], v[2], v[3]);
@@ -276,7 +278,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
                 for (int m = 0; m < KMAX; ++m) {
                     const float v16 = m < K ? kap_t[m] * ex2_approx(-dE16 * l2r[m]) : 0.f;
                     V16s[(16 * J + r) * KMAX + m] = v16;
-                    V16ps[(16 * J + r) * KMAX + m] = m < K ? v16 / tau_s[m] : 0.f;
+                    V16ps[(16 * J + r) * KMAX + m] = m < K ? v16 * inv_tau_s[m] : 0.f;
                 }
             }
         }
@@ -314,12 +316,14 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         // U rows as fp32 [128 t][4 J][8 m] in the x tile (free now) for the column pass, before the
         // row pass overwrites the operand tiles with XX
         float *Ufp = reinterpret_cast<float *>(sX);
-        if (grp == 0) {
+        {  // group g copies the chunks [4 g, 4 g + 4) of row t
             const unsigned char *row = sU + t * 128;
 #pragma unroll
-            for (int c8 = 0; c8 < 8; ++c8)
+            for (int c4 = 0; c4 < 4; ++c4) {
+                const int c8 = 4 * grp + c4;
                 *reinterpret_cast<uint4 *>(Ufp + t * 32 + 4 * c8) =
                     *reinterpret_cast<const uint4 *>(row + ((c8 ^ (t & 7)) * 16));
+            }
         }
         __syncthreads();
         // ---- row pass (row t = this warp's row block I; group 0 takes column blocks 0, 1, group 1
