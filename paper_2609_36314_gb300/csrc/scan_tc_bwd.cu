@@ -867,34 +867,39 @@ __global__ void __launch_bounds__(kStLaunch, 1)
             const uint32_t zu = lane_base + colZU;  // Z at +0, U at +64
             const float sj = my_coef[2 * KMAX + mj], aj = my_coef[mj], bj = my_coef[KMAX + mj];
             float dp[4] = {0.f, 0.f, 0.f, 0.f};  // independent partial sums
+            // 16-column chunks, the next one loading while the current one is used: group 0 reads
+            // Z (4 chunks, against dY) and U's first half (2, dx); group 1 reads U (4, against X,
+            // the second half also for dx)
+            const int nch = grp == 0 ? 6 : 4;
+            auto col = [&](int ch) -> uint32_t {
+                return grp == 0 ? (ch < 4 ? 16u * ch : 64u + 16u * (ch - 4)) : 64u + 16u * ch;
+            };
+            float za[16], zb[16];
+            tmem_ld16(zu + col(0), za);
+            tmem_ld_wait16(za);
 #pragma unroll
-            for (int pc = 0; pc < 4; ++pc) {
-                float zv[16];
-                tmem_ld16(zu + 64 * grp + 16 * pc, zv);
-                tmem_ld_wait();
+            for (int ch = 0; ch < 6; ++ch) {
+                if (ch < nch) {
+                    float *cur = (ch & 1) ? zb : za, *nxt = (ch & 1) ? za : zb;
+                    if (ch + 1 < nch) tmem_ld16(zu + col(ch + 1), nxt);
+                    if (ch < 4) {
 #pragma unroll
-                for (int q = 0; q < 2; ++q) {
-                    const uint4 rv = row[2 * pc + q];
-                    const uint32_t rr[4] = {rv.x, rv.y, rv.z, rv.w};
+                        for (int q = 0; q < 2; ++q) {
+                            const uint4 rv = row[2 * ch + q];
+                            const uint32_t rr[4] = {rv.x, rv.y, rv.z, rv.w};
 #pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        const float2 f = bf16x2_to_float2(rr[k]);
-                        dp[k] = fmaf(f.x, zv[8 * q + 2 * k], fmaf(f.y, zv[8 * q + 2 * k + 1], dp[k]));
+                            for (int k = 0; k < 4; ++k) {
+                                const float2 f = bf16x2_to_float2(rr[k]);
+                                dp[k] = fmaf(f.x, cur[8 * q + 2 * k], fmaf(f.y, cur[8 * q + 2 * k + 1], dp[k]));
+                            }
+                        }
                     }
-                }
-                if (grp == 1 && pc >= 2) {
+                    if (ch >= 2 && (grp == 1 || ch >= 4)) {  // dx: U columns [0, 32) (group 0) / [32, 64)
+                        const int o = 16 * ((ch - 2) & 1);
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) dxr[16 * (pc - 2) + i] = fmaf(sj, zv[i], dxr[16 * (pc - 2) + i]);
-                }
-            }
-            if (grp == 0) {
-#pragma unroll
-                for (int pc = 0; pc < 2; ++pc) {
-                    float zv[16];
-                    tmem_ld16(zu + 64 + 16 * pc, zv);
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) dxr[16 * pc + i] = fmaf(sj, zv[i], dxr[16 * pc + i]);
+                        for (int i = 0; i < 16; ++i) dxr[o + i] = fmaf(sj, cur[i], dxr[o + i]);
+                    }
+                    if (ch + 1 < nch) tmem_ld_wait16(nxt);
                 }
             }
             tc_fence_before();
