@@ -145,12 +145,12 @@ def kpn(s):
 # only while the kernel's sources hash to the digest they had when they were profiled.
 PROFILED_TRAFFIC_BATCH = 2
 PROFILED_TRAFFIC = {
-    "coef_tc": ("scan_tc.cu", "82d4db0a5d22ef9f", 23.103e6 + 41.900e6),
-    "state_pass_fwd_tc": ("scan_tc.cu", "82d4db0a5d22ef9f", 138.695e6 + 482.264e6),
-    "chunk_fwd_tc": ("scan_tc.cu", "82d4db0a5d22ef9f", 717.349e6 + 60.971e6),
-    "state_pass_rev_tc": ("scan_tc.cu", "82d4db0a5d22ef9f", 138.546e6 + 482.132e6),
-    "bwd_intra_tc": ("scan_tc_bwd.cu", "cfa2234782159636", 182.946e6 + 125.968e6),
-    "bwd_state_tc": ("scan_tc_bwd.cu", "cfa2234782159636", 1472.299e6 + 170.651e6),
+    "coef_tc": ("scan_tc.cu", "8fd98f818d670956", 23.101e6 + 41.741e6),
+    "state_pass_fwd_tc": ("scan_tc.cu", "8fd98f818d670956", 139.070e6 + 482.044e6),
+    "chunk_fwd_tc": ("scan_tc.cu", "8fd98f818d670956", 717.340e6 + 61.417e6),
+    "state_pass_rev_tc": ("scan_tc.cu", "8fd98f818d670956", 138.652e6 + 482.024e6),
+    "bwd_intra_tc": ("scan_tc_bwd.cu", "acff14ca05619fd2", 182.955e6 + 126.264e6),
+    "bwd_state_tc": ("scan_tc_bwd.cu", "acff14ca05619fd2", 1464.025e6 + 168.238e6),
 }
 
 
