@@ -370,7 +370,8 @@ struct OutArgs {
 };
 
 constexpr int kOutThreads = 256;  // two groups of four warps share the 128 TMEM lanes
-constexpr int kOutLaunch = kOutThreads + 32;  // a ninth warp issues the entering-state MMAs
+constexpr int kOutLaunch = kOutThreads + 64;  // a ninth warp issues the entering-state MMAs, a
+                                              // tenth loads their S_in tiles
 constexpr int kSBuf = 3;          // 8 KB units of the S ring (the Gamma operands, then one S_in pair slot)
 
 // Shared-memory plan of tc_chunk_fwd (offsets from a 1024-aligned base): about 110 KB at
@@ -399,28 +400,14 @@ struct OutSmem {
 constexpr int kZSlots = 3;
 __device__ __forceinline__ void chunk_fwd_issuer(const ScanDims &d, unsigned char *sC, unsigned char *sS,
                                                  unsigned char *sM, uint64_t *bars, volatile int *abort_s,
-                                                 uint32_t tmem, const CUtensorMap &mapS, int srow) {
+                                                 uint32_t tmem) {
     const int nhalf = d.N / 64, npair = d.K / 2, ntile = npair * nhalf;
     auto slot = [&](int s) { return s == 0 ? sS : sM + (s - 1) * 16384; };
-    auto load = [&](int j) {
-        const int s = j % kZSlots, mp = j / nhalf, hn = j % nhalf;
-        mbar_arrive_expect_tx(&bars[3 + s], 16384u);
-        tma_load_3d(slot(s), &mapS, &bars[3 + s], hn * 64, 0, srow + 2 * mp);
-        tma_load_3d(slot(s) + 8192, &mapS, &bars[3 + s], hn * 64, 0, srow + 2 * mp + 1);
-    };
-    // the S ring holds the Gamma operands until their MMAs are done
-    if (!mbar_wait(&bars[1], 0)) {
-        *abort_s = 1;
-        return;
-    }
-    if (ntile > 0) load(0);
-    // the intra Y MMA (issued after the Gamma o G pass) frees the G and Gamma columns and the
-    // Gamma o G tile
+    // the intra Y MMA (issued after the Gamma o G pass) frees the G and Gamma columns
     if (!mbar_wait(&bars[2], 0)) {
         *abort_s = 1;
         return;
     }
-    for (int j = 1; j < min(kZSlots, ntile); ++j) load(j);
     tc_fence_after();
     const uint32_t idZ = idesc_bf16(128, 128, false, false);
     for (int j = 0; j < ntile && !*abort_s; ++j) {
@@ -437,21 +424,45 @@ __device__ __forceinline__ void chunk_fwd_issuer(const ScanDims &d, unsigned cha
             break;
         }
         tc_fence_after();
-        const uint32_t sa = smem_u32(sC) + hn * 16384, sb = smem_u32(slot(s));
+        const uint64_t da = desc_sw128(smem_u32(sC) + hn * 16384, 16, 1024), db = desc_sw128(smem_u32(slot(s)), 16, 1024);
+#pragma unroll
         for (int ks = 0; ks < 4; ++ks)
-            mma_bf16(tmem + 128 * zb, desc_sw128(sa + ks * 32, 16, 1024), desc_sw128(sb + ks * 32, 16, 1024), idZ,
-                     (hn > 0 || ks > 0) ? 1u : 0u);
-        mma_commit(&bars[6 + s]);
+            mma_bf16(tmem + 128 * zb, desc_add(da, ks * 32), desc_add(db, ks * 32), idZ, (hn > 0 || ks > 0) ? 1u : 0u);
+        mma_commit(&bars[6 + s]);  // the slot, once its MMAs have read it
         if (hn == nhalf - 1) mma_commit(&bars[9 + zb]);
-        // tile j - 1's MMAs done: its slot takes tile j + 2
-        if (j >= 1 && j - 1 + kZSlots < ntile) {
-            const int sp = (j - 1) % kZSlots;
-            if (!mbar_wait(&bars[6 + sp], ((j - 1) / kZSlots) & 1)) {
-                *abort_s = 1;
-                break;
-            }
-            load(j - 1 + kZSlots);
+    }
+}
+
+// The S_in pair tiles of tc_chunk_fwd (one thread of the tenth warp): slot s of the ring takes
+// tile j + kZSlots once the MMAs of tile j have read it.  The first slot waits for the Gamma
+// MMAs (it held their operands), the other two for the intra Y MMA (the Gamma o G tile).
+__device__ __forceinline__ void chunk_fwd_loader(const ScanDims &d, unsigned char *sS, unsigned char *sM,
+                                                 uint64_t *bars, volatile int *abort_s, const CUtensorMap &mapS,
+                                                 int srow) {
+    const int nhalf = d.N / 64, npair = d.K / 2, ntile = npair * nhalf;
+    auto slot = [&](int s) { return s == 0 ? sS : sM + (s - 1) * 16384; };
+    auto load = [&](int j) {
+        const int s = j % kZSlots, mp = j / nhalf, hn = j % nhalf;
+        mbar_arrive_expect_tx(&bars[3 + s], 16384u);
+        tma_load_3d(slot(s), &mapS, &bars[3 + s], hn * 64, 0, srow + 2 * mp);
+        tma_load_3d(slot(s) + 8192, &mapS, &bars[3 + s], hn * 64, 0, srow + 2 * mp + 1);
+    };
+    if (!mbar_wait(&bars[1], 0)) {
+        *abort_s = 1;
+        return;
+    }
+    if (ntile > 0) load(0);
+    if (!mbar_wait(&bars[2], 0)) {
+        *abort_s = 1;
+        return;
+    }
+    for (int j = 1; j < min(kZSlots, ntile); ++j) load(j);
+    for (int j = 0; j + kZSlots < ntile && !*abort_s; ++j) {
+        if (!mbar_wait(&bars[6 + j % kZSlots], (j / kZSlots) & 1)) {
+            *abort_s = 1;
+            break;
         }
+        load(j + kZSlots);
     }
 }
 
@@ -562,7 +573,8 @@ __global__ void __launch_bounds__(kOutLaunch, 2)
     // [192, 256) and the Z buffers of mode pairs at 128 (pair % 2) (buffer 1 once Y has been read)
     constexpr uint32_t colG = 0, colGam = 128, colY = 192;
     if (tid >= kOutThreads) {
-        if (tid == kOutThreads) chunk_fwd_issuer(a.d, sC, sS, sM, bars, abort_s, tmem, mapS, srow);
+        if (tid == kOutThreads) chunk_fwd_issuer(a.d, sC, sS, sM, bars, abort_s, tmem);
+        if (tid == kOutThreads + 32) chunk_fwd_loader(a.d, sS, sM, bars, abort_s, mapS, srow);
     } else {
 
     if (tid == 0) {
