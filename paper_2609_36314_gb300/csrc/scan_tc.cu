@@ -508,11 +508,17 @@ __global__ void __launch_bounds__(kOutLaunch, 2)
     const int nhalf = N / 64;
     const int srow = int(((size_t(b) * d.H + h) * d.nc + c) * K);
 
-    if (tid == 0) {
+    if (tid == kOutThreads + 32) {  // the loading warp: barriers, then C, B and x at once
         for (int i = 0; i < 13; ++i) mbar_init(&bars[i], 1);
         for (int i = 13; i < 15; ++i) mbar_init(&bars[i], kOutThreads);
         *abort_s = 0;
         fence_barrier_init();
+        mbar_arrive_expect_tx(&bars[0], uint32_t(2 * plan.c + plan.x));
+        for (int jb = 0; jb < nhalf; ++jb) {
+            tma_load_3d(sC + jb * 16384, &mapC, &bars[0], g * N + 64 * jb, c0, b);
+            tma_load_3d(sM + jb * 16384, &mapB, &bars[0], g * N + 64 * jb, c0, b);
+        }
+        tma_load_3d(sX, &mapX, &bars[0], h * P, c0, b);
     }
     if (tid < K) {
         const float tv = a.tau[h * K + tid];
@@ -577,14 +583,6 @@ __global__ void __launch_bounds__(kOutLaunch, 2)
         if (tid == kOutThreads + 32) chunk_fwd_loader(a.d, sS, sM, bars, abort_s, mapS, srow);
     } else {
 
-    if (tid == 0) {
-        mbar_arrive_expect_tx(&bars[0], uint32_t(2 * plan.c + plan.x));
-        for (int jb = 0; jb < nhalf; ++jb) {
-            tma_load_3d(sC + jb * 16384, &mapC, &bars[0], g * N + 64 * jb, c0, b);
-            tma_load_3d(sM + jb * 16384, &mapB, &bars[0], g * N + 64 * jb, c0, b);
-        }
-        tma_load_3d(sX, &mapX, &bars[0], h * P, c0, b);
-    }
     if (grp == 0) {
         E_s[t] = Et2;
 #pragma unroll
