@@ -65,6 +65,7 @@ __device__ __forceinline__ unsigned char *align1024(unsigned char *p) {
 
 // ============================================================================= intra
 constexpr int kIntraThreads = 256;  // two groups of four warps share the 128 TMEM lanes
+constexpr int kIntraLaunch = kIntraThreads + 32;  // a ninth warp issues the MMAs and TMA loads
 
 struct IntraSmem {
     int rcb, x, dy, mg, xx, total;
@@ -81,7 +82,7 @@ struct IntraSmem {
     }
 };
 
-__global__ void __launch_bounds__(kIntraThreads, 1)
+__global__ void __launch_bounds__(kIntraLaunch, 1)
     tc_bwd_intra(const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapB,
                  const __grid_constant__ CUtensorMap mapX, const __grid_constant__ CUtensorMap mapDY,
                  BwdArgs a) {
@@ -105,9 +106,11 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     float *l2t = reinterpret_cast<float *>(E_s + TQ);
     float *inv_tau_s = l2t + 32;  // 1 / tau per mode
     float2 *wsum = reinterpret_cast<float2 *>(inv_tau_s + 32);
-    // bars: 0 C, B, x of the item loaded | 1 G, H, Gamma MMAs done | 2 dx MMA done | 3 dy loaded
+    // bars: 0 C, B, x of the item loaded | 1 G, H, Gamma MMAs done | 2 dx MMA done | 3 dy loaded |
+    //       the compute threads (256 arrive): 4 U, V operands written | 5 Gamma o G tile written
+    //       and G read | 6 C / B region and x tile read | 7 dx read from TMEM
     uint64_t *bars = reinterpret_cast<uint64_t *>(wsum + 8);
-    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 4);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 8);
     volatile int *abort_s = reinterpret_cast<volatile int *>(tslot + 1);
     // the next item's per-position inputs, staged by cp.async: {E hi, E lo, 0, 0, kappa[K]} from
     // tc_coef [128][12] floats and w_read [128] x 16 bytes
@@ -163,6 +166,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
 
     if (tid == 0) {
         for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
+        for (int i = 4; i < 8; ++i) mbar_init(&bars[i], kIntraThreads);
         *abort_s = 0;
         fence_barrier_init();
     }
@@ -175,15 +179,81 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
     // TMEM: G, H, the factored Gamma and Gamma' blocks; dx_intra replaces G after the row pass
     const uint32_t colG = 0, colH = 128, colGam = 256, colGamP = 384, colX = 0;
     if (int(blockIdx.x) < nitems) {
-        if (tid == 0) {
+        if (tid == kIntraThreads) {
             load_cbx(blockIdx.x);
             load_dy(blockIdx.x);
         }
-        stage_inputs(blockIdx.x);
+        if (tid < kIntraThreads) stage_inputs(blockIdx.x);
+    }
+
+    if (tid == kIntraThreads) {
+        // the issuing thread: an item's G = C B^T once its C and B tiles are in (and the previous
+        // item's dx has left TMEM), H = dY X^T once dY is in, the Gamma blocks once the threads
+        // have written U and V, dx_intra once they have written the Gamma o G tile; then the
+        // next item's dy (its tile free once dx_intra is done) and C, B, x (once read)
+        int kk = 0;
+        for (int item = blockIdx.x; item < nitems && !*abort_s; item += gridDim.x, ++kk) {
+            const int ph = kk & 1;
+            unsigned char *sU = reinterpret_cast<unsigned char *>(XX), *sV = sU + 16384, *sVp = sV + 4096;
+            const uint32_t idG = idesc_bf16(128, 128, false, false);
+            if ((kk > 0 && !mbar_wait(&bars[7], (kk - 1) & 1)) || !mbar_wait(&bars[0], ph)) {
+                *abort_s = 1;
+                break;
+            }
+            tc_fence_after();
+            for (int ks = 0; ks < N / 16; ++ks) {
+                const uint32_t koff = (ks / 4) * 16384 + (ks % 4) * 32;
+                mma_bf16(tmem + colG, desc_sw128(smem_u32(sC) + koff, 16, 1024),
+                         desc_sw128(smem_u32(sB) + koff, 16, 1024), idG, ks > 0);
+            }
+            if (!mbar_wait(&bars[3], ph)) {
+                *abort_s = 1;
+                break;
+            }
+            tc_fence_after();
+            for (int ks = 0; ks < BP / 16; ++ks)  // H = dY X^T, K = p
+                mma_bf16(tmem + colH, desc_sw128(smem_u32(sDY) + ks * 32, 16, 1024),
+                         desc_sw128(smem_u32(sX) + ks * 32, 16, 1024), idG, ks > 0);
+            if (!mbar_wait(&bars[4], ph)) {
+                *abort_s = 1;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t idT = idesc_tf32(128, 32);
+            for (int J = 0; J < 4; ++J) {
+                mma_tf32(tmem + colGam + 32 * J, desc_sw128(smem_u32(sU) + 32 * J, 16, 1024),
+                         desc_sw128(smem_u32(sV) + 32 * J, 16, 1024), idT, 0);
+                mma_tf32(tmem + colGamP + 32 * J, desc_sw128(smem_u32(sU) + 32 * J, 16, 1024),
+                         desc_sw128(smem_u32(sVp) + 32 * J, 16, 1024), idT, 0);
+            }
+            mma_commit(&bars[1]);
+            if (!mbar_wait(&bars[5], ph)) {
+                *abort_s = 1;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t idX = idesc_bf16(128, BP, true, true);  // dx_intra = (Gamma o G)^T dY
+            for (int ks = 0; ks < TQ / 16; ++ks)
+                mma_bf16(tmem + colX, desc_sw128(smem_u32(sMG) + ks * 2048, 16384, 1024),
+                         desc_sw128(smem_u32(sDY) + ks * 2048, 16384, 1024), idX, ks > 0);
+            mma_commit(&bars[2]);
+            if (item + int(gridDim.x) < nitems) {
+                if (!mbar_wait(&bars[2], ph)) {
+                    *abort_s = 1;
+                    break;
+                }
+                load_dy(item + gridDim.x);
+                if (!mbar_wait(&bars[6], ph)) {
+                    *abort_s = 1;
+                    break;
+                }
+                load_cbx(item + gridDim.x);
+            }
+        }
     }
 
     int kk_item = 0;
-    for (int item = blockIdx.x; item < nitems; item += gridDim.x, ++kk_item) {
+    for (int item = blockIdx.x; item < nitems && tid < kIntraThreads; item += gridDim.x, ++kk_item) {
         const int ph = kk_item & 1;  // parity of this item's phase on every barrier
         const int3 hcb = item_hcb(item);
         const int h = hcb.x, c = hcb.y, b = hcb.z;
@@ -191,7 +261,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         const int c0 = c * TQ, n = min(TQ, d.L - c0);
         // per-position inputs of row t from the staging area, and the mode time constants
         cp_async_wait_all();
-        __syncthreads();
+        sync_first256();
         float wr_t[KMAX], kap_t[KMAX], tau_r[KMAX];
         float2 Et2 = make_float2(0.f, 0.f);  // in-chunk cumulative log-decay (hi, lo)
 #pragma unroll
@@ -214,7 +284,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
             inv_tau_s[tid] = 1.f / tv;
             l2t[tid] = kLog2e / tv;
         }
-        __syncthreads();  // the staging area is free again: the next item's inputs
+        sync_first256();  // the staging area is free again: the next item's inputs
         if (item + int(gridDim.x) < nitems) stage_inputs(item + gridDim.x);
         if (grp == 0) E_s[t] = Et2;
         float l2r[KMAX];  // log2(e) / tau per mode, in registers
@@ -227,7 +297,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
             }
         }
         tc_fence_before();
-        __syncthreads();
+        sync_first256();
         tc_fence_after();
         // ---- Gamma below the diagonal 32 x 32 blocks, factored through the log-decay E_a at the end
         // of the column block J (as in the forward output kernel): Gamma[t, k in J] =
@@ -283,35 +353,9 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
             }
         }
         fence_async_smem();
-        __syncthreads();
-        if (tid == 0) {
-            if (!mbar_wait(&bars[0], ph) || !mbar_wait(&bars[3], ph)) {
-                *abort_s = 1;
-            } else {
-                tc_fence_after();
-                const uint32_t idG = idesc_bf16(128, 128, false, false);
-                for (int ks = 0; ks < N / 16; ++ks) {
-                    const uint32_t koff = (ks / 4) * 16384 + (ks % 4) * 32;
-                    mma_bf16(tmem + colG, desc_sw128(smem_u32(sC) + koff, 16, 1024),
-                             desc_sw128(smem_u32(sB) + koff, 16, 1024), idG, ks > 0);
-                }
-                for (int ks = 0; ks < BP / 16; ++ks) {  // H = dY X^T, K = p
-                    mma_bf16(tmem + colH, desc_sw128(smem_u32(sDY) + ks * 32, 16, 1024),
-                             desc_sw128(smem_u32(sX) + ks * 32, 16, 1024), idG, ks > 0);
-                }
-                const uint32_t idT = idesc_tf32(128, 32);
-                for (int J = 0; J < 4; ++J) {
-                    mma_tf32(tmem + colGam + 32 * J, desc_sw128(smem_u32(sU) + 32 * J, 16, 1024),
-                             desc_sw128(smem_u32(sV) + 32 * J, 16, 1024), idT, 0);
-                    mma_tf32(tmem + colGamP + 32 * J, desc_sw128(smem_u32(sU) + 32 * J, 16, 1024),
-                             desc_sw128(smem_u32(sVp) + 32 * J, 16, 1024), idT, 0);
-                }
-                mma_commit(&bars[1]);
-            }
-        }
-        __syncthreads();
+        mbar_arrive(&bars[4]);  // U, V written: the Gamma MMAs may go
         if (!*abort_s && !mbar_wait(&bars[1], ph)) *abort_s = 1;
-        __syncthreads();
+        sync_first256();
         tc_fence_after();
         // U rows as fp32 [128 t][4 J][8 m] in the x tile (free now) for the column pass, before the
         // row pass overwrites the operand tiles with XX
@@ -325,7 +369,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
                     *reinterpret_cast<const uint4 *>(row + ((c8 ^ (t & 7)) * 16));
             }
         }
-        __syncthreads();
+        sync_first256();
         // ---- row pass (row t = this warp's row block I; group 0 takes column blocks 0, 1, group 1
         // blocks 2, 3): Gamma o G tile, Gamma o H summed over heads in L2, Gamma' G H and G H tiles,
         // intra dw_read.  Blocks below the diagonal take the factored Gamma from TMEM, the diagonal
@@ -500,7 +544,8 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
         }
         fence_async_smem();
         tc_fence_before();
-        __syncthreads();
+        mbar_arrive(&bars[5]);  // the Gamma o G tile written, G read: dx_intra may go
+        sync_first256();
         tc_fence_after();
         if (!*abort_s && grp == 0 && t < n) {
             float *o = a.dwr_acc + blh(d, b, c0 + t, h) * K;
@@ -508,14 +553,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
             for (int m = 0; m < KMAX; ++m)
                 if (m < K) o[m] = dwr_i[m] + part[t * KMAX + m];
         }
-        if (tid == 0 && !*abort_s) {  // dx_intra = (Gamma o G)^T dY: M = k, N = p, K = t
-            const uint32_t idX = idesc_bf16(128, BP, true, true);
-            for (int ks = 0; ks < TQ / 16; ++ks)
-                mma_bf16(tmem + colX, desc_sw128(smem_u32(sMG) + ks * 2048, 16384, 1024),
-                         desc_sw128(smem_u32(sDY) + ks * 2048, 16384, 1024), idX, ks > 0);
-            mma_commit(&bars[2]);
-        }
-        __syncthreads();  // part[] is reused below
+        sync_first256();  // part[] is reused below
         // ---- column pass (group g takes the rows of parity g of column k): intra dkappa.  Rows of
         // later blocks use the factored form exp(-(E_a - E_k)/tau) sum_t U_J[t, m] G H[t, k]; rows of
         // the diagonal block (t >= k) sum directly.  Column block J has 128 - 32 J rows, so group 1's
@@ -619,7 +657,7 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
             }
             if (grp == 0) xtot[t] = run;
         }
-        __syncthreads();
+        sync_first256();
         // rect[j] = sum_{t' >= j} sum_{k < j} X[t', k]: column j's suffix sum of the row prefixes,
         // rows of parity g in group g (column kcol, the column pass's balanced assignment)
         float *rpart = Vs + TQ;  // [128] group 1's partial rect
@@ -632,8 +670,8 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
             }
         }
         if (grp == 1) rpart[kcol] = sr;
-        __syncthreads();  // G H (in the C / B region) and the U copy (in the x tile) are read
-        if (tid == 0 && !*abort_s && item + int(gridDim.x) < nitems) load_cbx(item + gridDim.x);
+        sync_first256();  // G H (in the C / B region) and the U copy (in the x tile) are read
+        mbar_arrive(&bars[6]);  // the next item's C, B, x may load
         if (!*abort_s && grp == 0 && t < n) {
             float *o = a.dkap_acc + blh(d, b, c0 + t, h) * K;
 #pragma unroll
@@ -641,11 +679,10 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
                 if (m < K) o[m] = dk[m] + part[t * KMAX + m];
             a.rect[blh(d, b, c0 + t, h)] = sr + rpart[t];
         }
-        __syncthreads();
+        sync_first256();
         if (!*abort_s && !mbar_wait(&bars[2], ph)) *abort_s = 1;
-        __syncthreads();
+        sync_first256();
         tc_fence_after();
-        if (tid == 0 && !*abort_s && item + int(gridDim.x) < nitems) load_dy(item + gridDim.x);
         {  // dx_intra row: group g takes columns [32 g, 32 g + 32) (nothing written after an abort)
             float v[32];
             tmem_ld32(lane_base + colX + grp * 32, v);
@@ -658,7 +695,8 @@ __global__ void __launch_bounds__(kIntraThreads, 1)
                                size_t(d.H) * P * 4, *abort_s ? 0 : n - t8);
         }
         tc_fence_before();
-        __syncthreads();  // this item's TMEM reads are done before the next item's MMAs
+        mbar_arrive(&bars[7]);  // this item's TMEM reads are done: the next item's MMAs may go
+        sync_first256();
         if (*abort_s) break;
     }  // items
     cp_async_wait_all();
@@ -1438,7 +1476,7 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
         trace_begin("bwd_intra_tc", st);
         // persistent: one CTA per SM (shared memory), items (h, c, b) strided by the grid
         const int items = d.H * d.nc * d.B;
-        tc_bwd_intra<<<std::min(items, a.pf_sms), kIntraThreads, smem, st>>>(mapC, mapB, mapX, mapDY, a);
+        tc_bwd_intra<<<std::min(items, a.pf_sms), kIntraLaunch, smem, st>>>(mapC, mapB, mapX, mapDY, a);
         trace_end(st);
         if ((e = cudaGetLastError())) return e;
     }
