@@ -738,7 +738,7 @@ struct StSmem {
         cb = (N / 64) * 16384;   // one of C / B: [t][n]
         tile = (N / 64) * 8192;  // one S_in or dS_out mode tile: [p = 64][n], 64-wide n atoms
         gen = 2 * 16384;         // two units: M_H [t][k] at the start, dC staging at the end
-        total = 2 * cb + kStBuf * 2 * tile + 2 * gen + kStThreads * kCoefStride * 4 + 512;
+        total = 2 * cb + kStBuf * 2 * tile + 2 * gen + kStThreads * kCoefStride * 4 + 1024;
     }
 };
 
@@ -778,8 +778,8 @@ __global__ void __launch_bounds__(kStLaunch, 1)
     unsigned char *sG = sT + kStBuf * 2 * L.tile;             // [buf][f o dY | s o X]
     // this thread's mode coefficients for the current head: cA (f or s), cB (exp(-E/tau) or u), s
     float *coef_s = reinterpret_cast<float *>(sG + 2 * L.gen);  // [256][kCoefStride]
-    float *itau_s = coef_s + kStThreads * kCoefStride;         // [hg][K] 1 / tau (hg <= 8)
-    double *wsum = reinterpret_cast<double *>(itau_s + 8 * KMAX);  // [8]
+    float *itau_s = coef_s + kStThreads * kCoefStride;         // [hg][K] 1 / tau (hg <= 16)
+    double *wsum = reinterpret_cast<double *>(itau_s + 16 * KMAX);  // [8]
     double *Eend_s = wsum + 8;                                  // [1]
     // bars: 0..2 tile buffers | 3, 4 MMA of step parity | 5 C, B | 6 intra MMA |
     //       7, 8 generated operands of step parity written (all 256 threads arrive) |
@@ -815,7 +815,7 @@ __global__ void __launch_bounds__(kStLaunch, 1)
         fence_barrier_init();
     }
     if (w == 0) tmem_alloc_once(tslot, 512);
-    if (tid < a.hg * K) itau_s[tid] = 1.f / a.tau[h_first * K + tid];
+    for (int i = tid; i < a.hg * K; i += kStLaunch) itau_s[i] = 1.f / a.tau[h_first * K + i];
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -1373,10 +1373,10 @@ __global__ void f32_to_bf16_tc(const float *__restrict__ in, bf16 *__restrict__ 
         out[i] = __float2bfloat16_rn(in[i]);
 }
 
-// Heads per CTA of tc_bwd_state: a divisor of the heads of one B/C group, at most 8.
+// Heads per CTA of tc_bwd_state: a divisor of the heads of one B/C group, at most 16.
 int pick_hg(const ScanDims &d) {
     const int hpg = d.H / d.G;
-    for (int hg = 8; hg >= 1; --hg)
+    for (int hg = 16; hg >= 1; --hg)
         if (hpg % hg == 0) return hg;
     return 1;
 }

@@ -141,10 +141,10 @@ def test_tensor_path_modes_and_groups(N, K, G):
     assert {"state_pass_fwd_tc", "chunk_fwd_tc", "state_pass_rev_tc", "bwd_intra_tc"} <= names
 
 
-def test_tensor_path_eight_heads_per_group():
-    """bf16, eight heads sharing B/C: the state-term backward takes all eight heads of the group
-    in one CTA (seven head switches with staged inputs), on a ragged sequence."""
-    s = synth.Shape(1, 200, 8, 64, 1, 128, 8, 0, "bf16")
+def test_tensor_path_sixteen_heads_per_group():
+    """bf16, sixteen heads sharing B/C: the state-term backward takes all sixteen heads of the
+    group in one CTA (fifteen head switches with staged inputs), on a ragged sequence."""
+    s = synth.Shape(1, 200, 16, 64, 1, 128, 8, 0, "bf16")
     _check_fwd(s, seed=41, h0=True)
     _check_bwd(s, seed=42, h0=True, dhf=True)
 
