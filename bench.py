@@ -145,12 +145,12 @@ def kpn(s):
 # only while the kernel's sources hash to the digest they had when they were profiled.
 PROFILED_TRAFFIC_BATCH = 2
 PROFILED_TRAFFIC = {
-    "coef_tc": ("scan_tc.cu", "fde0bbbd1a3a9ef6", 23.115e6 + 41.926e6),
-    "state_pass_fwd_tc": ("scan_tc.cu", "fde0bbbd1a3a9ef6", 138.952e6 + 482.410e6),
-    "chunk_fwd_tc": ("scan_tc.cu", "fde0bbbd1a3a9ef6", 717.341e6 + 60.948e6),
-    "state_pass_rev_tc": ("scan_tc.cu", "fde0bbbd1a3a9ef6", 138.908e6 + 481.935e6),
-    "bwd_intra_tc": ("scan_tc_bwd.cu", "c2dc34424a6cb5d4", 182.902e6 + 126.582e6),
-    "bwd_state_tc": ("scan_tc_bwd.cu", "c2dc34424a6cb5d4", 1463.968e6 + 168.001e6),
+    "coef_tc": ("scan_tc.cu", "fde0bbbd1a3a9ef6", 23.101e6 + 41.631e6),
+    "state_pass_fwd_tc": ("scan_tc.cu", "fde0bbbd1a3a9ef6", 138.760e6 + 481.840e6),
+    "chunk_fwd_tc": ("scan_tc.cu", "fde0bbbd1a3a9ef6", 717.318e6 + 60.756e6),
+    "state_pass_rev_tc": ("scan_tc.cu", "fde0bbbd1a3a9ef6", 139.129e6 + 482.585e6),
+    "bwd_intra_tc": ("scan_tc_bwd.cu", "2995a748538032e4", 182.952e6 + 126.667e6),
+    "bwd_state_tc": ("scan_tc_bwd.cu", "2995a748538032e4", 1464.175e6 + 165.234e6),
 }
 
 
