@@ -149,8 +149,8 @@ PROFILED_TRAFFIC = {
     "state_pass_fwd_tc": ("scan_tc.cu", "fde0bbbd1a3a9ef6", 138.760e6 + 481.840e6),
     "chunk_fwd_tc": ("scan_tc.cu", "fde0bbbd1a3a9ef6", 717.318e6 + 60.756e6),
     "state_pass_rev_tc": ("scan_tc.cu", "fde0bbbd1a3a9ef6", 139.129e6 + 482.585e6),
-    "bwd_intra_tc": ("scan_tc_bwd.cu", "2995a748538032e4", 182.952e6 + 126.667e6),
-    "bwd_state_tc": ("scan_tc_bwd.cu", "2995a748538032e4", 1464.175e6 + 165.234e6),
+    "bwd_intra_tc": ("scan_tc_bwd.cu", "b5059f52658823c0", 182.952e6 + 126.667e6),
+    "bwd_state_tc": ("scan_tc_bwd.cu", "b5059f52658823c0", 1464.175e6 + 165.234e6),
 }
 
 

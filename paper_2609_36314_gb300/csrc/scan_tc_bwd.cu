@@ -128,7 +128,7 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
     // persistent: items (h, c, b) in launch order, gridDim.x CTAs apart
     const int nitems = d.H * d.nc * d.B;
     auto item_hcb = [&](int item) { return make_int3(item % d.H, (item / d.H) % d.nc, item / (d.H * d.nc)); };
-    // tid 0: the item's C, B and x tiles (bars[0]) / its dy tile (bars[3]) by TMA
+    // the issuing thread: the item's C, B and x tiles (bars[0]) / its dy tile (bars[3]) by TMA
     auto load_cbx = [&](int item) {
         const int3 hcb = item_hcb(item);
         const int h_ = hcb.x, c_ = hcb.y, b_ = hcb.z;
@@ -718,10 +718,12 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
 // out; the threads read out step i - 1 after writing step i's operands: group 0 contracts Z_m with
 // its dY row (dw_read, the a term), group 1 contracts U_m with its X row (dkappa, the b term) and
 // accumulates dx = sum_m s_m U_m in registers.  Three more warps form <dS_out,m, S_in,m> from the
-// two tiles in shared memory.  The head-summed intra tile Gamma o H adds M_H B to dC and M_H^T C to dB once
-// per (b, c, B/C group).
+// two tiles in shared memory, and one of their lanes refills a tile buffer once its step's MMAs
+// and the three warps are done with it.  The next head's dY, X and coefficient rows are staged by
+// TMA a whole head ahead.  The head-summed intra tile Gamma o H adds M_H B to dC and M_H^T C to dB
+// once per (b, c, B/C group).
 constexpr int kStThreads = 256;  // compute threads (two warpgroups); a ninth warp issues the MMAs
-                                 // and TMA loads (one thread)
+                                 // (one thread)
 constexpr int kCdThreads = 96;   // three more warps form <dS_out,m, S_in,m> from each step's tiles
 constexpr int kStLaunch = kStThreads + 32 + kCdThreads;
 constexpr int kStBuf = 2;   // S_in / dS_out tile buffers
