@@ -154,6 +154,12 @@ PROFILED_TRAFFIC = {
 }
 
 
+# DRAM bytes (read + write) of one decode_step launch of the decode workload (B128 H64 P64 N128
+# K8, float32 state), from one ncu capture (profiles/decode_step_b128.md); used only while
+# decode.cu hashes to the digest it had when profiled.
+PROFILED_DECODE_TRAFFIC = ("decode.cu", "5a6ee76a91d8f3d2", 2151.500e6 + 2097.820e6)
+
+
 def source_digest(fname: str) -> str:
     import hashlib
     src = os.path.join(os.path.dirname(os.path.abspath(__file__)), "paper_2609_36314_gb300", "csrc")
@@ -591,7 +597,10 @@ def bench_decode(args, dev, peaks, world, max_over_ranks, barrier):
             "us_per_step": 1e3 * ms_step,
             "roofline": {"kernel": "decode_step", "bound": "hbm", "achieved": gbs,
                          "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                         "frac": gbs / peaks["hbm_gbs"], "traffic": None,
+                         "frac": gbs / peaks["hbm_gbs"],
+                         "traffic": (PROFILED_DECODE_TRAFFIC[2]
+                                     if source_digest(PROFILED_DECODE_TRAFFIC[0]) == PROFILED_DECODE_TRAFFIC[1]
+                                     else None),
                          "peak_source": peaks["source"]}}
 
 
