@@ -151,6 +151,7 @@ PROFILED_TRAFFIC = {
     "state_pass_rev_tc": ("scan_tc.cu", "fde0bbbd1a3a9ef6", 139.129e6 + 482.585e6),
     "bwd_intra_tc": ("scan_tc_bwd.cu", "b5059f52658823c0", 182.952e6 + 126.667e6),
     "bwd_state_tc": ("scan_tc_bwd.cu", "b5059f52658823c0", 1464.175e6 + 165.234e6),
+    "bwd_final_tc": ("scan_tc_bwd.cu", "b5059f52658823c0", 323.524e6 + 70.281e6),
 }
 
 
