@@ -44,6 +44,7 @@ def parse():
     ap.add_argument("--decode-steps", type=int, default=1024)
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-prefill", action="store_true")
+    ap.add_argument("--no-paper-shape", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--batch", type=int, default=0,
@@ -475,6 +476,9 @@ def main():
     prefill = None
     if not args.no_prefill:
         prefill = bench_prefill(args, dev, world, max_over_ranks, barrier)
+    paper_shape = None
+    if not args.no_paper_shape:
+        paper_shape = bench_paper_shape(dev, max_over_ranks, barrier)
 
     if rank == 0:
         line = {
@@ -492,7 +496,8 @@ def main():
                        "parallelism": f"replicas{world}" if world > 1 else "single",
                        "l2": "inputs larger than L2 (0.78 GB per step), no flush"},
             "roofline": roofline, "kernels": kern, "gpu_launches": launches,
-            "e2e": e2e, "decode": decode, "prefill": prefill, "clocks": clk,
+            "e2e": e2e, "decode": decode, "prefill": prefill, "paper_shape_prefill": paper_shape,
+            "clocks": clk,
             "peaks_source": peaks["source"],
         }
         if args.batch:
@@ -548,6 +553,43 @@ def bench_prefill(args, dev, world, max_over_ranks, barrier):
                         "kept; chunk 128 (results are chunk-independent)",
             "value": world * s.batch * s.seqlen / (ms / 1e3), "unit": "tokens/s", "ms_per_forward": ms,
             "kernels": kern}
+
+
+def bench_paper_shape(dev, max_over_ranks, barrier):
+    """The paper's own layer shape (H16, head dim 256, N = 1, K = 16 modes on the 1 .. 2^17
+    bank), batch-1 prefill at 1K, 4K and 16K tokens: forward tokens/s per length (inputs
+    resident; CUDA-core path, these shapes are outside the tensor-core kernels)."""
+    import torch
+
+    from paper_2609_36314_gb300 import scan_fwd, synth
+    pts = []
+    for L in (1024, 4096, 16384):
+        s = synth.Shape(1, L, 16, 256, 1, 1, 16, 0, "bf16")
+        a = synth.make_scan_inputs_torch(s, seed=13, device=dev)
+        y = torch.empty_like(a["x"])
+
+        def fwd():
+            scan_fwd(a["x"], a["dt"], a["alpha"], a["lam"], a["tau"], a["B"], a["C"], a["w_read"],
+                     a["w_write"], a["D"], y=y)
+
+        for _ in range(3):
+            fwd()
+        torch.cuda.synchronize()
+        barrier()
+        stream = torch.cuda.current_stream()
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        n = 10
+        ev0.record(stream)
+        for _ in range(n):
+            fwd()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        ms = max_over_ranks(ev0.elapsed_time(ev1) / n)
+        pts.append({"seqlen": L, "ms_per_forward": ms, "tokens_per_s": L / (ms / 1e3)})
+        del a, y
+    return {"workload": "paper layer shape: B1 H16 P256 N1 K16, tau geometric in [1, 2^17], bf16 "
+                        "inputs, forward only", "unit": "tokens/s", "points": pts}
 
 
 def bench_decode(args, dev, peaks, world, max_over_ranks, barrier):

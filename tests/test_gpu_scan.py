@@ -149,6 +149,15 @@ def test_tensor_path_sixteen_heads_per_group():
     _check_bwd(s, seed=42, h0=True, dhf=True)
 
 
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_paper_layer_shape(dtype):
+    """The paper's own layer shape, cut to two heads and 300 tokens: head dim 256, N = 1, K = 16
+    modes on the geometric 1 .. 2^17 bank (the CUDA-core path)."""
+    s = synth.Shape(1, 300, 2, 256, 1, 1, 16, 0, dtype)
+    _check_fwd(s, seed=50, h0=True)
+    _check_bwd(s, seed=51, h0=True, dhf=True)
+
+
 def test_force_simt_matches_default_path():
     s = synth.Shape(2, 260, 4, 64, 1, 128, 8, 0, "bf16")
     host = synth.make_scan_inputs(s, seed=12, with_dy=True)
