@@ -848,8 +848,190 @@ cudaError_t run_state_pass(const ScanDims &d, bool rev, const void *U, const voi
     return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------------------------------------
+// N = 1 (the paper's own layer: scalar B, C per position): each (mode, p) is a scalar
+// recurrence S <- rho S + kappa B x, y = sum_m w_read C S + D x, so the forward runs it directly
+// (K fused multiply-adds per mode row and token) instead of the pairwise intra-chunk form.
+// Per chunk, the coefficients of its positions and modes go to shared memory first:
+// rho = exp(-e/tau), kappa B = -expm1(-e/tau) w_write B and (output kernel) w_read C.
+constexpr int kN1Modes = 32;  // nmodes <= 32 (checked at the boundary)
+
+template <typename T>
+__device__ void n1_chunk_coefs(const ScanDims &d, int b, int h, int c0, int n, float log_cap,
+                               const float *__restrict__ itau, const T *__restrict__ Bm,
+                               const T *__restrict__ Cm, const T *__restrict__ ww,
+                               const T *__restrict__ wr, const float *__restrict__ dt,
+                               const float *__restrict__ alpha, const float *__restrict__ lam,
+                               float *e_s, float *rho_s, float *kb_s, float *wc_s) {
+    const int K = d.K, g = h / (d.H / d.G);
+    for (int t = threadIdx.x; t < n; t += blockDim.x) {
+        const size_t i = blh(d, b, c0 + t, h);
+        bool cl = false;
+        e_s[t] = token_rate(dt[i], alpha[i], lam[i], log_cap, &cl);
+    }
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < n * K; idx += blockDim.x) {
+        const int t = idx / K, m = idx - t * K;
+        const size_t i = blh(d, b, c0 + t, h);
+        const size_t ig = (size_t(b) * d.L + c0 + t) * d.G + g;  // N = 1: one B, C per group
+        const float z = e_s[t] * itau[m];
+        rho_s[idx] = expf(-z);
+        kb_s[idx] = -expm1f(-z) * to_f(ww[i * K + m]) * to_f(Bm[ig]);
+        if (wc_s) wc_s[idx] = to_f(wr[i * K + m]) * to_f(Cm[ig]);
+    }
+    __syncthreads();
+}
+
+// Chunk-serial state pass: one thread per p of a 64-wide slice; emits every chunk's entering
+// state S_in [B, H, nc, K, P] (the general layout with N = 1) and the final state.
+template <typename T, typename TS>
+__global__ void __launch_bounds__(64) n1_state_pass(ScanDims d, const T *__restrict__ x,
+                                                    const T *__restrict__ Bm, const T *__restrict__ ww,
+                                                    const float *__restrict__ dt, const float *__restrict__ alpha,
+                                                    const float *__restrict__ lam, const float *__restrict__ tau,
+                                                    const float *__restrict__ init, TS *__restrict__ emit,
+                                                    float *__restrict__ fin) {
+    __shared__ float e_s[kQMax], itau[kN1Modes];
+    __shared__ __align__(16) float rho_s[kQMax * kN1Modes];
+    __shared__ __align__(16) float kb_s[kQMax * kN1Modes];
+    __shared__ float x_s[kQMax * 64];  // the chunk's x rows of this slice
+    const int K = d.K, P = d.P;
+    const int b = blockIdx.z, h = blockIdx.y, p = blockIdx.x * 64 + threadIdx.x;
+    const bool active = p < P;
+    const size_t bh = size_t(b) * d.H + h;
+    if (threadIdx.x < K) itau[threadIdx.x] = 1.f / tau[h * K + threadIdx.x];
+    const float log_cap = head_log_cap(tau, h, K);
+    float S[kN1Modes];
+#pragma unroll
+    for (int m = 0; m < kN1Modes; ++m) S[m] = (active && m < K && init) ? init[(bh * K + m) * P + p] : 0.f;
+    __syncthreads();
+    for (int c = 0; c < d.nc; ++c) {
+        const int c0 = c * d.Q, n = min(d.Q, d.L - c0);
+        // the chunk's x rows of the slice, every load in flight at once (the barriers in
+        // n1_chunk_coefs publish them); the serial recurrence then reads shared memory
+#pragma unroll 8
+        for (int t = 0; t < n; ++t) x_s[t * 64 + threadIdx.x] = active ? to_f(x[blh(d, b, c0 + t, h) * P + p]) : 0.f;
+        n1_chunk_coefs<T>(d, b, h, c0, n, log_cap, itau, Bm, nullptr, ww, nullptr, dt, alpha, lam, e_s,
+                          rho_s, kb_s, nullptr);
+        if (active) {
+#pragma unroll
+            for (int m = 0; m < kN1Modes; ++m)
+                if (m < K) emit[((bh * d.nc + c) * K + m) * P + p] = from_f<TS>(S[m]);
+            for (int t = 0; t < n; ++t) {
+                const float xv = x_s[t * 64 + threadIdx.x];
+                if ((K & 3) == 0) {  // rows of 16-byte pieces
+                    const float4 *r4 = reinterpret_cast<const float4 *>(rho_s + t * K);
+                    const float4 *k4 = reinterpret_cast<const float4 *>(kb_s + t * K);
+#pragma unroll
+                    for (int q = 0; q < kN1Modes / 4; ++q) {
+                        if (4 * q < K) {
+                            const float4 r = r4[q], kv = k4[q];
+                            S[4 * q] = fmaf(r.x, S[4 * q], kv.x * xv);
+                            S[4 * q + 1] = fmaf(r.y, S[4 * q + 1], kv.y * xv);
+                            S[4 * q + 2] = fmaf(r.z, S[4 * q + 2], kv.z * xv);
+                            S[4 * q + 3] = fmaf(r.w, S[4 * q + 3], kv.w * xv);
+                        }
+                    }
+                } else {
+#pragma unroll
+                    for (int m = 0; m < kN1Modes; ++m)
+                        if (m < K) S[m] = fmaf(rho_s[t * K + m], S[m], kb_s[t * K + m] * xv);
+                }
+            }
+        }
+        __syncthreads();  // the coefficients are rewritten for the next chunk
+    }
+    if (active && fin) {
+#pragma unroll
+        for (int m = 0; m < kN1Modes; ++m)
+            if (m < K) fin[(bh * K + m) * P + p] = S[m];
+    }
+}
+
+// Chunk-parallel output: from the chunk's entering state, the recurrence again with
+// y_t = sum_m w_read C S_m + D x_t after each update; one thread per p of a 128-wide slice.
+template <typename T, typename TS>
+__global__ void __launch_bounds__(128) n1_chunk_fwd(ScanDims d, const T *__restrict__ x,
+                                                    const T *__restrict__ Bm, const T *__restrict__ Cm,
+                                                    const T *__restrict__ wr, const T *__restrict__ ww,
+                                                    const float *__restrict__ dt, const float *__restrict__ alpha,
+                                                    const float *__restrict__ lam, const float *__restrict__ tau,
+                                                    const float *__restrict__ Dp, const TS *__restrict__ S_in,
+                                                    T *__restrict__ y) {
+    __shared__ float e_s[kQMax], itau[kN1Modes];
+    __shared__ __align__(16) float rho_s[kQMax * kN1Modes];
+    __shared__ __align__(16) float kb_s[kQMax * kN1Modes];
+    __shared__ __align__(16) float wc_s[kQMax * kN1Modes];
+    const int K = d.K, P = d.P;
+    const int npb = (P + 127) / 128;
+    const int c = blockIdx.x, h = blockIdx.y / npb, b = blockIdx.z;
+    const int p = (blockIdx.y % npb) * 128 + threadIdx.x;
+    const bool active = p < P;
+    const size_t bh = size_t(b) * d.H + h;
+    const int c0 = c * d.Q, n = min(d.Q, d.L - c0);
+    if (threadIdx.x < K) itau[threadIdx.x] = 1.f / tau[h * K + threadIdx.x];
+    const float log_cap = head_log_cap(tau, h, K);
+    __syncthreads();
+    n1_chunk_coefs<T>(d, b, h, c0, n, log_cap, itau, Bm, Cm, ww, wr, dt, alpha, lam, e_s, rho_s, kb_s,
+                      wc_s);
+    if (!active) return;
+    float S[kN1Modes];
+#pragma unroll
+    for (int m = 0; m < kN1Modes; ++m) S[m] = m < K ? to_f(S_in[((bh * d.nc + c) * K + m) * P + p]) : 0.f;
+    const float Dh = Dp[h];
+#pragma unroll 4
+    for (int t = 0; t < n; ++t) {
+        const size_t i = blh(d, b, c0 + t, h) * P + p;
+        const float xv = to_f(x[i]);
+        float yv = Dh * xv;
+        if ((K & 3) == 0) {  // rows of 16-byte pieces
+            const float4 *r4 = reinterpret_cast<const float4 *>(rho_s + t * K);
+            const float4 *k4 = reinterpret_cast<const float4 *>(kb_s + t * K);
+            const float4 *w4 = reinterpret_cast<const float4 *>(wc_s + t * K);
+#pragma unroll
+            for (int q = 0; q < kN1Modes / 4; ++q) {
+                if (4 * q < K) {
+                    const float4 r = r4[q], kv = k4[q], wv = w4[q];
+                    S[4 * q] = fmaf(r.x, S[4 * q], kv.x * xv);
+                    S[4 * q + 1] = fmaf(r.y, S[4 * q + 1], kv.y * xv);
+                    S[4 * q + 2] = fmaf(r.z, S[4 * q + 2], kv.z * xv);
+                    S[4 * q + 3] = fmaf(r.w, S[4 * q + 3], kv.w * xv);
+                    yv = fmaf(wv.x, S[4 * q], fmaf(wv.y, S[4 * q + 1], fmaf(wv.z, S[4 * q + 2], fmaf(wv.w, S[4 * q + 3], yv))));
+                }
+            }
+        } else {
+#pragma unroll
+            for (int m = 0; m < kN1Modes; ++m) {
+                if (m < K) {
+                    S[m] = fmaf(rho_s[t * K + m], S[m], kb_s[t * K + m] * xv);
+                    yv = fmaf(wc_s[t * K + m], S[m], yv);
+                }
+            }
+        }
+        y[i] = from_f<T>(yv);
+    }
+}
+
+template <typename T, typename TS>
+cudaError_t fwd_n1(const ScanDims &d, const ScanPtrs &p, void *S_in, cudaStream_t st) {
+    trace_begin("state_pass_fwd_n1", st);
+    n1_state_pass<T, TS><<<dim3((d.P + 63) / 64, d.H, d.B), 64, 0, st>>>(
+        d, (const T *)p.x, (const T *)p.Bm, (const T *)p.ww, p.dt, p.alpha, p.lam, p.tau, p.h0,
+        (TS *)S_in, p.h_final);
+    trace_end(st);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess || d.nc == 0) return e;  // L = 0: h_final = h0 was written
+    trace_begin("chunk_fwd_n1", st);
+    n1_chunk_fwd<T, TS><<<dim3(d.nc, d.H * ((d.P + 127) / 128), d.B), 128, 0, st>>>(
+        d, (const T *)p.x, (const T *)p.Bm, (const T *)p.Cm, (const T *)p.wr, (const T *)p.ww, p.dt,
+        p.alpha, p.lam, p.tau, p.D, (const TS *)S_in, (T *)p.y);
+    trace_end(st);
+    return cudaGetLastError();
+}
+
 template <typename T, typename TS>
 cudaError_t fwd_t(const ScanDims &d, const ScanPtrs &p, void *S_in, cudaStream_t st) {
+    if (d.N == 1 && d.Q <= kQMax && d.K <= kN1Modes) return fwd_n1<T, TS>(d, p, S_in, st);
     cudaError_t e = run_state_pass<T, TS>(d, false, p.x, p.Bm, p.ww, p, p.h0, S_in, p.h_final, st);
     if (e != cudaSuccess || d.nc == 0) return e;  // L = 0: h_final = h0 was written
     const size_t smem = chunk_fwd_smem(d);

@@ -158,6 +158,17 @@ def test_paper_layer_shape(dtype):
     _check_bwd(s, seed=51, h0=True, dhf=True)
 
 
+@pytest.mark.parametrize("shape", [
+    synth.Shape(2, 77, 3, 200, 1, 1, 5, 16, "f32"),   # K = 5 (per-mode loop), two p blocks, ragged
+    synth.Shape(1, 130, 2, 64, 2, 1, 8, 32, "bf16"),  # one head per B/C group, chunk 32
+    synth.Shape(1, 0, 2, 32, 1, 1, 4, 0, "f32"),      # empty sequence: h_final = h0
+])
+def test_n1_forward_shapes(shape):
+    """N = 1 forward (the direct per-mode recurrence): mode counts off a multiple of 4, p blocks
+    past the head dimension, groups, chunk sizes, ragged and empty sequences."""
+    _check_fwd(shape, seed=60 + shape.nmodes, h0=True)
+
+
 def test_force_simt_matches_default_path():
     s = synth.Shape(2, 260, 4, 64, 1, 128, 8, 0, "bf16")
     host = synth.make_scan_inputs(s, seed=12, with_dy=True)
