@@ -14,10 +14,10 @@
 //        (A = s o x generated in shared memory, B = the chunk of B loaded by TMA).
 //        Run over the chunks in reverse with (dy, C, f) it carries dS for the backward.
 //   tc_chunk_fwd   (chunk-parallel; one CTA per (b, c, h), headdim 64):
-//        G = C B^T on the tensor cores, Gamma_{t,k} G_{t,k} per position pair -> bf16 tile,
-//        then one TMEM accumulator Y[t, p] collects (Gamma o G) X and sum_m (f_m o C) S_in,m^T
-//        (K = (mode, n) in 64-wide steps, S_in tiles by TMA, f o C tiles written by the
-//        threads), and y = Y + D x.
+//        G = C B^T and the factored Gamma blocks on the tensor cores, Gamma o G -> bf16 tile,
+//        Y = (Gamma o G) X in TMEM; then Z_m = C S_in,m^T, two modes per product (S_in tiles
+//        streamed by TMA by a loading warp, MMAs issued by an issuing warp), which the threads
+//        fold into their rows with f_m[t]: y = Y + sum_m f_m o Z_m + D x.
 //
 // All mbarrier waits are bounded (a few seconds); on a timeout the kernel records
 // FRAC_ERR_TIMEOUT in the error word, stops issuing work, frees its tensor memory and exits.
