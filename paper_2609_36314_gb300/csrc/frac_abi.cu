@@ -183,7 +183,7 @@ frac_status frac_scan_fwd_workspace_size(const frac_dims *d, size_t *bytes) {
     if (s) return s;
     if (!bytes) return fail(FRAC_ERR_INVALID_ARGUMENT, "bytes must not be NULL");
     frac::ScanDims sd;
-    int path;
+    int path = 0;
     if ((s = plan(d, &sd, &path, false))) return s;
     *bytes = fwd_layout(d, sd, path).total;
     return FRAC_OK;
@@ -195,7 +195,7 @@ frac_status frac_scan_bwd_workspace_size(const frac_dims *d, size_t *bytes) {
     if (s) return s;
     if (!bytes) return fail(FRAC_ERR_INVALID_ARGUMENT, "bytes must not be NULL");
     frac::ScanDims sd;
-    int path;
+    int path = 0;
     if ((s = plan(d, &sd, &path, true))) return s;
     *bytes = bwd_layout(d, sd, path).total;
     return FRAC_OK;
@@ -225,7 +225,7 @@ frac_status frac_scan_fwd(const frac_dims *d, const void *x, const float *dt, co
         REQUIRE_T(y);
     }
     frac::ScanDims sd;
-    int path;
+    int path = 0;
     if ((s = plan(d, &sd, &path, false))) return s;
     const FwdLayout l = fwd_layout(d, sd, path);
     if (path == PATH_TC && d->seqlen > 0) {
@@ -287,7 +287,7 @@ frac_status frac_scan_bwd(const frac_dims *d, const void *x, const float *dt, co
         REQUIRE_T(dw_write);
     }
     frac::ScanDims sd;
-    int path;
+    int path = 0;
     if ((s = plan(d, &sd, &path, true))) return s;
     const BwdLayout l = bwd_layout(d, sd, path);
     const bool reuse = (d->flags & FRAC_FLAG_BWD_REUSE_FWD_STATES) != 0;
