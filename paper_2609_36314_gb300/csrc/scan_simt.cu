@@ -1031,7 +1031,8 @@ cudaError_t fwd_n1(const ScanDims &d, const ScanPtrs &p, void *S_in, cudaStream_
 
 template <typename T, typename TS>
 cudaError_t fwd_t(const ScanDims &d, const ScanPtrs &p, void *S_in, cudaStream_t st) {
-    if (d.N == 1 && d.Q <= kQMax && d.K <= kN1Modes) return fwd_n1<T, TS>(d, p, S_in, st);
+    if (d.N == 1 && d.Q <= kQMax && d.K <= kN1Modes && size_t(d.H) * ((d.P + 127) / 128) <= 65535)
+        return fwd_n1<T, TS>(d, p, S_in, st);  // (grid y of the output kernel: heads x p blocks)
     cudaError_t e = run_state_pass<T, TS>(d, false, p.x, p.Bm, p.ww, p, p.h0, S_in, p.h_final, st);
     if (e != cudaSuccess || d.nc == 0) return e;  // L = 0: h_final = h0 was written
     const size_t smem = chunk_fwd_smem(d);
