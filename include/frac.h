@@ -70,7 +70,8 @@ enum {
     /* Use the CUDA-core chunked kernels even where tensor-core ones exist.  Without it, bf16
        calls with headdim 64, dstate in {64, 128} and nmodes in {4, 8} run the forward and the
        backward on the tensor cores (TMA-fed tcgen05 MMAs, chunk 128); they need the dtype
-       tensors and the states 16-byte aligned. */
+       tensors and the states 16-byte aligned.  On the CUDA-core path, dstate 1 (the paper's
+       scalar B, C per position) runs the forward as the direct per-mode recurrence. */
     FRAC_FLAG_FORCE_SIMT = 1,
     /* frac_scan_bwd only: the workspace already holds the per-chunk states that a frac_scan_fwd
        call with the same inputs, h0 and dims left in this same workspace (give both calls one
