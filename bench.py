@@ -150,9 +150,9 @@ PROFILED_TRAFFIC = {
     "state_pass_fwd_tc": ("scan_tc.cu", "900e85af153e741a", 138.760e6 + 481.840e6),
     "chunk_fwd_tc": ("scan_tc.cu", "900e85af153e741a", 717.318e6 + 60.756e6),
     "state_pass_rev_tc": ("scan_tc.cu", "900e85af153e741a", 139.129e6 + 482.585e6),
-    "bwd_intra_tc": ("scan_tc_bwd.cu", "b5059f52658823c0", 182.952e6 + 126.667e6),
-    "bwd_state_tc": ("scan_tc_bwd.cu", "b5059f52658823c0", 1464.175e6 + 165.234e6),
-    "bwd_final_tc": ("scan_tc_bwd.cu", "b5059f52658823c0", 323.524e6 + 70.281e6),
+    "bwd_intra_tc": ("scan_tc_bwd.cu", "a135ecad70d3c440", 182.952e6 + 126.667e6),
+    "bwd_state_tc": ("scan_tc_bwd.cu", "a135ecad70d3c440", 1464.175e6 + 165.234e6),
+    "bwd_final_tc": ("scan_tc_bwd.cu", "a135ecad70d3c440", 323.524e6 + 70.281e6),
 }
 
 

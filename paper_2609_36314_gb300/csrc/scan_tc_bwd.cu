@@ -1375,12 +1375,19 @@ __global__ void f32_to_bf16_tc(const float *__restrict__ in, bf16 *__restrict__ 
         out[i] = __float2bfloat16_rn(in[i]);
 }
 
-// Heads per CTA of tc_bwd_state: a divisor of the heads of one B/C group, at most 16.
-int pick_hg(const ScanDims &d) {
+// Heads per CTA of tc_bwd_state: a divisor of the heads of one B/C group, at most 16 (more
+// heads amortise the CTA's set-up and dC / dB epilogue), but no more than leaves two waves of
+// CTAs on the SMs; when even one head per CTA leaves fewer, the largest divisor.
+int pick_hg(const ScanDims &d, int sms) {
     const int hpg = d.H / d.G;
-    for (int hg = 16; hg >= 1; --hg)
-        if (hpg % hg == 0) return hg;
-    return 1;
+    const size_t per_head = size_t(d.nc) * d.B, want = 2 * size_t(sms);
+    int largest = 1, fits = 0;
+    for (int hg = 1; hg <= 16; ++hg) {
+        if (hpg % hg) continue;
+        largest = hg;
+        if (size_t(d.H / hg) * per_head >= want) fits = hg;
+    }
+    return fits ? fits : largest;
 }
 
 }  // namespace
@@ -1464,13 +1471,13 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
     a.dx = (bf16 *)p.dx; a.dwr = (bf16 *)p.dwr; a.dww = (bf16 *)p.dww;
     a.ddt = p.ddt; a.dalpha = p.dalpha; a.dlam = p.dlam; a.dD = p.dD;
     a.err = err;
-    a.hg = pick_hg(d);
     {
         int dev = 0, nsm = 0;
         if ((e = cudaGetDevice(&dev)) || (e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)))
             return e;
         a.pf_sms = std::max(nsm, 1);
     }
+    a.hg = pick_hg(d, a.pf_sms);
 
     {
         const size_t smem = IntraSmem().total + 1024;
