@@ -141,7 +141,7 @@ def kpn(s):
 
 
 # DRAM bytes (read + write) per launch of each tensor-core kernel from one ncu capture of the
-# training shape at batch 2 (profiles/tc_kernels_train_b2_l4096.md); the per-chunk state traffic
+# training shape at batch 2 (the ncu summary of these kernels kept under profiles/); the per-chunk state traffic
 # grows in proportion to the batch, so a run at batch B reports bytes x B / 2.  A figure is used
 # only while the kernel's sources hash to the digest they had when they were profiled.
 PROFILED_TRAFFIC_BATCH = 2
@@ -157,7 +157,7 @@ PROFILED_TRAFFIC = {
 
 
 # DRAM bytes (read + write) of one decode_step launch of the decode workload (B128 H64 P64 N128
-# K8, float32 state), from one ncu capture (profiles/decode_step_b128.md); used only while
+# K8, float32 state), from one ncu capture (summarised under profiles/); used only while
 # decode.cu hashes to the digest it had when profiled.
 PROFILED_DECODE_TRAFFIC = ("decode.cu", "5a6ee76a91d8f3d2", 2151.500e6 + 2097.820e6)
 
@@ -181,8 +181,8 @@ def profiled_traffic(kernel: str, batch: int):
 
 
 def algorithmic_work(kernel: str, s, per_launch_units: float):
-    """Algorithmic flops or bytes of one launch of `kernel` (see the measurement section of
-    the design notes): state contractions count 2 K P N flops per token-head each."""
+    """Algorithmic flops or bytes of one launch of `kernel` (the per-kernel counts below):
+    state contractions count 2 K P N flops per token-head each."""
     per_th = {
         "state_pass_fwd_simt": 2, "state_pass_rev_simt": 2, "chunk_fwd_simt": 2,
         "chunk_bwd_simt": 8, "state_pass_fwd_tc": 2, "state_pass_rev_tc": 2,

@@ -78,7 +78,14 @@ enum {
        buffer of frac_scan_bwd_workspace_size bytes), so the backward does not recompute them.
        Rejected with FRAC_ERR_INVALID_ARGUMENT when the forward and backward would run on
        different paths (then the states are not compatible). */
-    FRAC_FLAG_BWD_REUSE_FWD_STATES = 2
+    FRAC_FLAG_BWD_REUSE_FWD_STATES = 2,
+    /* Test hook of the bounded device waits (frac_scan_fwd and frac_scan_fwd_static on the
+       tensor-core path only; FRAC_ERR_UNSUPPORTED elsewhere): every CTA of the forward state
+       pass first waits about a millisecond on a barrier that nothing signals, gives up, records
+       FRAC_ERR_TIMEOUT in the call's status word and exits the way a kernel whose wait ran out
+       does.  y and h_final are then incomplete; frac_workspace_status (or
+       frac_scan_fwd_static_status) returns FRAC_ERR_TIMEOUT.  Not for production use. */
+    FRAC_FLAG_TEST_EXPIRE_WAIT = 4
 };
 
 typedef struct {
@@ -106,7 +113,7 @@ frac_status frac_scan_fwd_workspace_size(const frac_dims *dims, size_t *bytes);
 /*
  * Chunked parallel forward scan (training / prefill), the Remark after Eq. read-softmax:
  * the affine recurrence evaluated chunk by chunk with chunk-local cumulative log-decays,
- * the stable intra-chunk coefficient Gamma of App. E, cross-chunk state passing, and the
+ * the stable intra-chunk coefficient Gamma of App. F, cross-chunk state passing, and the
  * skip D fused into the output.
  *   x, dt, alpha, lam, tau, Bm, Cm, w_read, w_write, D : inputs (layouts above)
  *   h0       : initial mode state, or NULL for zeros
@@ -176,9 +183,15 @@ frac_status frac_decode_step(const frac_dims *dims, const void *x_t, const float
  *     FRAC_ERR_UNSUPPORTED (frac_last_error() says how much they need); nothing is enqueued.
  *   - The first call on a device looks up the array's address on that device (a CUDA runtime
  *     query, made with that device current); make the first call before any stream capture.
+ *     The address is cached with the context that was current; a call that finds another
+ *     context (for example after cudaDeviceReset) looks it up again, which must then also
+ *     happen outside a stream capture.
  *   - All calls share the array.  Calls whose GPU work overlaps (other streams, other host
  *     threads on the same device) race on it and must be serialised by the caller.  Nothing in
  *     it needs to start at zero: every per-chunk state is written before it is read.
+ *   - A kernel whose bounded device wait gave up leaves y and h_final incomplete and records
+ *     FRAC_ERR_TIMEOUT in the array's status word, which frac_scan_fwd_static_status reads;
+ *     overlapping calls share that word as well.
  */
 #define FRAC_SCAN_FWD_STATIC_SCRATCH_BYTES ((size_t)64 << 20)
 frac_status frac_scan_fwd_static(const frac_dims *dims, const void *x, const float *dt,
@@ -186,6 +199,14 @@ frac_status frac_scan_fwd_static(const frac_dims *dims, const void *x, const flo
                                  const void *Bm, const void *Cm, const void *w_read,
                                  const void *w_write, const float *D, const float *h0, void *y,
                                  float *h_final, void *stream);
+
+/*
+ * Status of the last frac_scan_fwd_static call on the current device: waits for `stream` and
+ * returns FRAC_ERR_TIMEOUT if one of that call's kernels gave up on a bounded device-side wait
+ * (its outputs are then incomplete), FRAC_OK otherwise (the word is reset by every call).
+ * Like frac_workspace_status for the library's own array; allocates nothing.
+ */
+frac_status frac_scan_fwd_static_status(void *stream);
 
 /*
  * Kernel tracing (a profiling aid, off by default).  While enabled, every kernel the library

@@ -21,6 +21,7 @@ EXPORTS = (
     "frac_scan_bwd",
     "frac_decode_step",
     "frac_scan_fwd_static",
+    "frac_scan_fwd_static_status",
     "frac_workspace_status",
     "frac_trace_enable",
     "frac_trace_collect",
@@ -34,6 +35,7 @@ FRAC_DTYPE_F32 = 0
 FRAC_DTYPE_BF16 = 1
 FRAC_FLAG_FORCE_SIMT = 1
 FRAC_FLAG_BWD_REUSE_FWD_STATES = 2
+FRAC_FLAG_TEST_EXPIRE_WAIT = 4
 FRAC_SCAN_FWD_STATIC_SCRATCH_BYTES = 64 << 20
 
 
@@ -87,6 +89,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.frac_decode_step.restype = st
         lib.frac_scan_fwd_static.argtypes = [dims_p] + [P] * 13 + [P]
         lib.frac_scan_fwd_static.restype = st
+        lib.frac_scan_fwd_static_status.argtypes = [P]
+        lib.frac_scan_fwd_static_status.restype = st
         lib.frac_workspace_status.argtypes = [P, P]
         lib.frac_workspace_status.restype = st
         lib.frac_trace_enable.argtypes = [ctypes.c_int]

@@ -17,9 +17,9 @@ _DT = {torch.float32: _lib.FRAC_DTYPE_F32, torch.bfloat16: _lib.FRAC_DTYPE_BF16}
 
 
 def make_dims(batch, seqlen, nheads, headdim, ngroups, dstate, nmodes, dtype, chunk=0,
-              force_simt=False, reuse_fwd_states=False) -> _lib.FracDims:
+              force_simt=False, reuse_fwd_states=False, extra_flags=0) -> _lib.FracDims:
     flags = (_lib.FRAC_FLAG_FORCE_SIMT if force_simt else 0) | (
-        _lib.FRAC_FLAG_BWD_REUSE_FWD_STATES if reuse_fwd_states else 0)
+        _lib.FRAC_FLAG_BWD_REUSE_FWD_STATES if reuse_fwd_states else 0) | int(extra_flags)
     return _lib.FracDims(batch, seqlen, nheads, headdim, ngroups, dstate, nmodes, chunk,
                          _DT[dtype], flags)
 

@@ -227,6 +227,12 @@ frac_status frac_scan_fwd(const frac_dims *d, const void *x, const float *dt, co
     frac::ScanDims sd;
     int path = 0;
     if ((s = plan(d, &sd, &path, false))) return s;
+    if (d->flags & FRAC_FLAG_TEST_EXPIRE_WAIT) {
+        if (path != PATH_TC)
+            return fail(FRAC_ERR_UNSUPPORTED,
+                        "FRAC_FLAG_TEST_EXPIRE_WAIT applies to the tensor-core forward only");
+        sd.expire_ns = 1000000u;  // 1 ms
+    }
     const FwdLayout l = fwd_layout(d, sd, path);
     if (path == PATH_TC && d->seqlen > 0) {
         const void *need16[] = {x, Bm, Cm, y};
@@ -286,6 +292,8 @@ frac_status frac_scan_bwd(const frac_dims *d, const void *x, const float *dt, co
         REQUIRE_PTR(dlam); REQUIRE_T(dB); REQUIRE_T(dC); REQUIRE_T(dw_read);
         REQUIRE_T(dw_write);
     }
+    if (d->flags & FRAC_FLAG_TEST_EXPIRE_WAIT)
+        return fail(FRAC_ERR_UNSUPPORTED, "FRAC_FLAG_TEST_EXPIRE_WAIT applies to the forward only");
     frac::ScanDims sd;
     int path = 0;
     if ((s = plan(d, &sd, &path, true))) return s;

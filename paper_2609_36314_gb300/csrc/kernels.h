@@ -30,6 +30,9 @@ struct ScanDims {
     int B, L, H, P, G, N, K;
     int Q;   // chunk length
     int nc;  // number of chunks = ceil(L / Q)
+    // Test hook (FRAC_FLAG_TEST_EXPIRE_WAIT): when nonzero, the forward state pass's CTAs first
+    // wait this many nanoseconds on a barrier that nothing signals, then take the timeout path.
+    unsigned expire_ns = 0;
 };
 
 // Pointers of one scan call.  Element types follow the dtype of the call.

@@ -12,13 +12,20 @@
 //   * Problems whose forward scratch (frac_scan_fwd_workspace_size) exceeds that size are
 //     rejected with FRAC_ERR_UNSUPPORTED and a message; nothing is enqueued for them.
 //   * The first call on a device looks up the array's device address (cudaGetSymbolAddress)
-//     with that device current and caches it; make that first call before anything that must
-//     not see a runtime call (for example before capturing work into a CUDA graph).
+//     with that device current and caches it together with the device's current context; make
+//     that first call before anything that must not see a runtime call (for example before
+//     capturing work into a CUDA graph).  A later call that finds another context current on
+//     the device (after cudaDeviceReset the module is loaded again and the array may move)
+//     looks the address up again.
+//   * Word 0 of the array is the status word of the last call's kernels (a bounded device wait
+//     that gave up writes FRAC_ERR_TIMEOUT there); frac_scan_fwd_static_status reads it.
+//     Overlapping calls share that word too.
 //   * Every call shares the one array.  Calls whose GPU work overlaps (different streams, or
 //     different host threads on the same device) race on it; serialise them.  No part of the
 //     scratch has to start at zero: the forward scan writes every per-chunk state before it
 //     reads it, so leftovers of an earlier call are never used.
 //   * No cudaMalloc, cudaFree or other allocating routine is called.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <cstdio>
@@ -36,8 +43,27 @@ static __device__ __align__(256) unsigned char g_static_scratch[kFracStaticScrat
 
 std::mutex g_mu;
 void *g_dev_ptr[kMaxDevices] = {};
+CUcontext g_dev_ctx[kMaxDevices] = {};
 
-// Device address of g_static_scratch on the current device (looked up once per device).
+// The driver's cuCtxGetCurrent, reached through the runtime (the library does not link the
+// driver library directly, so it loads on machines without a GPU driver).
+CUresult current_context(CUcontext *ctx) {
+    using Fn = CUresult (*)(CUcontext *);
+    static Fn fn = [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            p = nullptr;
+        return reinterpret_cast<Fn>(p);
+    }();
+    *ctx = nullptr;
+    return fn ? fn(ctx) : CUDA_ERROR_NOT_SUPPORTED;
+}
+
+// Device address of g_static_scratch on the current device (looked up once per device and
+// context).
 frac_status static_scratch(void **out) {
     char msg[160];
     int dev = -1;
@@ -52,8 +78,12 @@ frac_status static_scratch(void **out) {
         frac::set_last_error(msg);
         return FRAC_ERR_UNSUPPORTED;
     }
+    // The context current on the device (null before the runtime has set the device up; the
+    // symbol lookup below does that).  A cached address is only reused under the same context.
+    CUcontext ctx = nullptr;
+    if (current_context(&ctx) != CUDA_SUCCESS) ctx = nullptr;
     std::lock_guard<std::mutex> lk(g_mu);
-    if (!g_dev_ptr[dev]) {
+    if (!g_dev_ptr[dev] || !ctx || g_dev_ctx[dev] != ctx) {
         void *p = nullptr;
         e = cudaGetSymbolAddress(&p, g_static_scratch);
         if (e != cudaSuccess || !p) {
@@ -62,7 +92,9 @@ frac_status static_scratch(void **out) {
             frac::set_last_error(msg);
             return FRAC_ERR_CUDA;
         }
+        if (current_context(&ctx) != CUDA_SUCCESS) ctx = nullptr;
         g_dev_ptr[dev] = p;
+        g_dev_ctx[dev] = ctx;
     }
     *out = g_dev_ptr[dev];
     return FRAC_OK;
@@ -93,6 +125,13 @@ frac_status frac_scan_fwd_static(const frac_dims *dims, const void *x, const flo
     if ((s = static_scratch(&scratch)) != FRAC_OK) return s;
     return frac_scan_fwd(dims, x, dt, alpha, lam, tau, Bm, Cm, w_read, w_write, D, h0, y,
                          h_final, scratch, kFracStaticScratchBytes, stream);
+}
+
+frac_status frac_scan_fwd_static_status(void *stream) {
+    void *scratch = nullptr;
+    frac_status s = static_scratch(&scratch);
+    if (s != FRAC_OK) return s;
+    return frac_workspace_status(scratch, stream);
 }
 
 }  // extern "C"

@@ -1,6 +1,6 @@
 // CUDA-core (SIMT) chunked Frac scan: forward and backward, float32 arithmetic.
 //
-// The chunked evaluation order (App. E of the paper; the Remark after Eq. read-softmax):
+// The chunked evaluation order (App. F of the paper; the Remark after Eq. read-softmax):
 // per chunk of Q positions, E_t = sum of e_j = Delta_j lambda_j^(1/alpha_j) from the chunk
 // start through t (kept in double so that differences E_t - E_k are exact to float
 // precision even when e_j is huge), so that the log of the product of retentions from k+1
@@ -12,7 +12,7 @@
 //        reverse with (dy, C, f_{t,m} = w_read_{t,m} exp(-E_t / tau_m)) carries dS backwards.
 //   chunk output (chunk-parallel per (b, h, c)):
 //        y_t = sum_m f_{t,m} S_in,m C_t + sum_{k<=t} Gamma_{t,k} (C_t . B_k) x_k + D x_t
-//        Gamma_{t,k} = sum_m w_read_{t,m} kappa_{k,m} exp(-(E_t - E_k) / tau_m)   (App. E)
+//        Gamma_{t,k} = sum_m w_read_{t,m} kappa_{k,m} exp(-(E_t - E_k) / tau_m)   (App. F)
 //   chunk backward (chunk-parallel per (b, h, c)): every gradient from x, dy, B, C, the mode
 //        weights, S_in and dS_out of the chunk (see the comments in simt_chunk_bwd).
 //

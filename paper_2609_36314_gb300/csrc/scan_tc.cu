@@ -1,6 +1,6 @@
 // Tensor-core (tcgen05 / TMEM / TMA) chunked Frac scan for bf16 inputs, sm_103a.
 //
-// Same chunked evaluation order as the CUDA-core kernels (App. E of the paper), with chunk
+// Same chunked evaluation order as the CUDA-core kernels (App. F of the paper), with chunk
 // Q = 128 and the two state contractions of every chunk on the tensor cores:
 //
 //   tc_coef        (one CTA per (b, h, chunk)): the per-position mode coefficients of the
@@ -201,6 +201,14 @@ __global__ void __launch_bounds__(kSPThreads, 2)
         }
     }
     tmem_st_wait();
+    if (!REV && d.expire_ns) {
+        // Test hook of the bounded waits: the MMA barrier has not been signalled (nothing is
+        // issued yet), so this wait runs out, and the CTA leaves through the timeout path below
+        // with no TMA load, bulk store or MMA of its own in flight.
+        __syncthreads();
+        if (tid == 0 && !mbar_wait(&bars[1], 0, d.expire_ns)) *abort_s = 1;
+        __syncthreads();
+    }
 
     // Thread t of each group owns chunk position t: its slice of x (or dy) and its coefficient
     // per mode (s = kappa exp(-(E_end - E_t)/tau) forward, f = w_read exp(-E_t/tau) reverse) stay

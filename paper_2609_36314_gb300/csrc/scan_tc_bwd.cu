@@ -2,7 +2,7 @@
 //
 // With S_in / dS_out the per-chunk states of the forward and reverse state passes, every
 // gradient of a chunk follows from chunk-local quantities (the adjoint of the recurrence of
-// Sec. 3.2, written in the chunked order of App. E).  With G[t,k] = C_t.B_k, H[t,k] = dy_t.x_k,
+// Sec. 3.2, written in the chunked order of App. F).  With G[t,k] = C_t.B_k, H[t,k] = dy_t.x_k,
 // W_{t,k,m} = exp(-(E_t - E_k)/tau_m) (k <= t), u = exp(-(E_end - E)/tau), s = kappa u,
 // f = w_read exp(-E/tau), Gamma = sum_m w_read kappa W and Gamma' = the same with kappa/tau:
 //   dx_k       = sum_m s_{k,m} (B dS_out,m^T)[k] + sum_{t>=k} Gamma_{t,k} G_{t,k} dy_t + D dy_k

@@ -7,10 +7,10 @@ Recipe (one independent numpy PCG64 stream per tensor, keyed by (seed, tensor id
   x, B, C, dy ~ N(0, 1)
   Delta  = clip(softplus(z - shift), 1e-4, 1),  z ~ N(0,1); shift 1 (3 for the
            long-context prefill workload).  The clip range is the paper's
-           (language-modelling setup, App. C.3).
+           (language-modelling setup, App. E.3).
   alpha  = sigmoid(z)                           (Sec. 3.3: sigmoid keeps alpha in (0,1))
-  lambda = clip(softplus(z), 0.25, 4)           (Sec. 3.3 softplus; clip of App. C.3)
-  tau_m  = 2^(17 (m-1)/(K-1)), m = 1..K         (geometric bank from 1 to 2^17, App. C.3;
+  lambda = clip(softplus(z), 0.25, 4)           (Sec. 3.3 softplus; clip of App. E.3)
+  tau_m  = 2^(17 (m-1)/(K-1)), m = 1..K         (geometric bank from 1 to 2^17, App. E.3;
                                                  endpoints included)
   w_read, w_write = softmax_m(-alpha ln tau_m + 0.5 z_m),  z ~ N(0,1) i.i.d.
            (Eq. read-softmax with the log-timescale prior; the learned logit maps

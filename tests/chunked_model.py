@@ -6,11 +6,11 @@ chunk, the same recurrence the sequential oracle runs step by step, so that
 
 forward, per chunk of Q positions with E_t the in-chunk inclusive cumulative sum of
 e_j = Delta_j lambda_j^(1/alpha_j) (so log rho_{t,m} summed over the chunk prefix is
--E_t / tau_m, the stable log-space form of App. E):
+-E_t / tau_m, the stable log-space form of App. F):
     y_t     = sum_m f_{t,m} S_in,m C_t + sum_{k<=t} Gamma_{t,k} (C_t . B_k) x_k + D x_t
     S_out,m = d_m S_in,m + sum_k s_{k,m} x_k B_k^T
 with f = w_read exp(-E_t/tau), s = kappa exp(-(E_end - E_k)/tau), d = exp(-E_end/tau) and
-Gamma_{t,k} = sum_m w_read_{t,m} kappa_{k,m} exp(-(E_t - E_k)/tau_m) (App. E).
+Gamma_{t,k} = sum_m w_read_{t,m} kappa_{k,m} exp(-(E_t - E_k)/tau_m) (App. F).
 
 Gamma can also be evaluated through the sub-block factorisation
 exp(-(E_t-E_k)/tau) = exp(-(E_t-E_a)/tau) exp(-(E_a-E_b)/tau) exp(-(E_b-E_k)/tau)

@@ -1,6 +1,6 @@
 """Chunked evaluation == sequential recurrence (fp64, CPU).
 
-Pins the decomposition every GPU kernel uses (App. E: chunk-local cumulative
+Pins the decomposition every GPU kernel uses (App. F: chunk-local cumulative
 log-decays, the stable intra-chunk coefficient Gamma, cross-chunk state
 passing) against the sequential oracle, for many chunk sizes including ragged
 last chunks and chunks larger than the sequence.

@@ -143,7 +143,7 @@ def _loglog_slope(t, y):
 
 @pytest.mark.parametrize("alpha", [0.3, 0.5, 0.7])
 def test_power_law_tails_on_the_paper_bank(alpha):
-    """K=16 geometric bank on [1, 2^17] (App. C.3).  With the log-timescale prior alone
+    """K=16 geometric bank on [1, 2^17] (App. E.3).  With the log-timescale prior alone
     (weights proportional to tau^-alpha, Eq. read-softmax without content logits):
       * homogeneous decay ~ t^-alpha            (Eq. mittag-tail)
       * impulse response with write 1/lambda  ~ t^-(1+alpha)   (Eq. gal-tail)

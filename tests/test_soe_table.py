@@ -1,8 +1,8 @@
-"""Reproduce the paper's finite-bank approximation table (App. F) on the CPU.
+"""Reproduce the paper's finite-bank approximation table (App. G) on the CPU.
 
 This pins two readings at once: the Mittag-Leffler reference used by the other
 oracle pins, and the timescale bank "geometrically spaced between tau_min = 1 and
-tau_max = 2^17" (App. C.3) read with both endpoints included, which is the bank
+tau_max = 2^17" (App. E.3) read with both endpoints included, which is the bank
 every workload uses.  (The midpoint grid of Theorem 2's proof on the same range gives
 errors 10-30x larger than the table, so it is not the paper's bank.)  The s-sampling
 density is not stated in the paper; 200 log-spaced points reproduce the table to 0.3%.

@@ -42,11 +42,52 @@ def test_static_scratch_forward_matches_workspace_forward(dtype):
                          device="cuda")
         st = _static_call(dims, d, y, hf)
         assert st == 0, _lib.load().frac_last_error()
+        assert _lib.load().frac_scan_fwd_static_status(_stream(None)) == 0
         y_ref, hf_ref = scan_fwd(d["x"], d["dt"], d["alpha"], d["lam"], d["tau"], d["B"],
                                  d["C"], d["w_read"], d["w_write"], d["D"], d.get("h0"))
         torch.cuda.synchronize()
         assert_close(f"y (call {seed})", to_host64(y), to_host64(y_ref), tol(dtype))
         assert_close(f"h_final (call {seed})", to_host64(hf), to_host64(hf_ref), tol(dtype))
+
+
+def test_static_scratch_smaller_problem_after_a_larger_one():
+    """A larger problem first, then a smaller one with another length and mode count on the
+    same (tensor-core) path: the second result must not depend on what the first left in the
+    shared array, so it is compared with frac_scan_fwd given a fresh workspace."""
+    big = synth.Shape(2, 517, 8, 64, 1, 128, 8, 0, "bf16")
+    small = synth.Shape(1, 131, 4, 64, 1, 128, 4, 0, "bf16")
+    for s, seed in ((big, 3), (small, 4)):
+        dims = make_dims(s.batch, s.seqlen, s.nheads, s.headdim, s.ngroups, s.dstate, s.nmodes,
+                         torch.bfloat16)
+        assert fwd_workspace_size(dims) <= _lib.FRAC_SCAN_FWD_STATIC_SCRATCH_BYTES
+        d = dev_inputs(synth.make_scan_inputs(s, seed=seed))
+        y = torch.empty_like(d["x"])
+        hf = torch.empty((s.batch, s.nheads, s.nmodes, s.headdim, s.dstate), dtype=torch.float32,
+                         device="cuda")
+        assert _static_call(dims, d, y, hf) == 0, _lib.load().frac_last_error()
+        assert _lib.load().frac_scan_fwd_static_status(_stream(None)) == 0
+        ws = torch.zeros(fwd_workspace_size(dims), dtype=torch.uint8, device="cuda")
+        y_ref, hf_ref = scan_fwd(d["x"], d["dt"], d["alpha"], d["lam"], d["tau"], d["B"],
+                                 d["C"], d["w_read"], d["w_write"], d["D"], workspace=ws)
+        torch.cuda.synchronize()
+        assert_close(f"y (L={s.seqlen})", to_host64(y), to_host64(y_ref), tol("bf16"))
+        assert_close(f"h_final (L={s.seqlen})", to_host64(hf), to_host64(hf_ref), tol("bf16"))
+
+
+def test_static_scratch_status_reports_an_expired_wait():
+    """A bounded device wait that runs out inside the allocation-free forward is visible to
+    the caller through frac_scan_fwd_static_status (the test hook makes the forward state
+    pass's waits run out), and the next call resets the word."""
+    s = synth.Shape(1, 200, 2, 64, 1, 64, 8, 0, "bf16")
+    args = (s.batch, s.seqlen, s.nheads, s.headdim, s.ngroups, s.dstate, s.nmodes, torch.bfloat16)
+    d = dev_inputs(synth.make_scan_inputs(s, seed=6))
+    y = torch.empty_like(d["x"])
+    lib = _lib.load()
+    dims = make_dims(*args, extra_flags=_lib.FRAC_FLAG_TEST_EXPIRE_WAIT)
+    assert _static_call(dims, d, y, None) == 0, lib.frac_last_error()
+    assert lib.frac_scan_fwd_static_status(_stream(None)) == 4  # FRAC_ERR_TIMEOUT
+    assert _static_call(make_dims(*args), d, y, None) == 0, lib.frac_last_error()
+    assert lib.frac_scan_fwd_static_status(_stream(None)) == 0
 
 
 def test_static_scratch_rejects_problems_that_do_not_fit():
