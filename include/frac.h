@@ -209,6 +209,75 @@ frac_status frac_scan_fwd_static(const frac_dims *dims, const void *x, const flo
 frac_status frac_scan_fwd_static_status(void *stream);
 
 /*
+ * Scan-parameter construction (the fused "scan parameter" kernel of App. F, and its backward).
+ * From the outputs of the layer's projections it forms the scan's controls and mode weights,
+ * per position (b, t) and head h (Sec. 3.3; Eq. read-softmax; Algorithm 1 of App. D):
+ *   Delta   = clip(softplus(dt_raw + dt_bias_h), dt_min, dt_max)    (linear map with learned bias,
+ *                                                                     then softplus; clip of App. E.3)
+ *   alpha   = sigmoid(alpha_raw)                                     (0 < alpha < 1)
+ *   lambda  = clip(softplus(lam_raw), lam_min, lam_max)              (clip of App. E.3)
+ *   w_read  = softmax_m(-alpha ln tau_m + g_read_m)                  (Eq. read-softmax)
+ *   w_write = softmax_m(-alpha ln tau_m + g_write_m)                 (same form, own logits)
+ * g_read / g_write are the mode-wise residual logits (the learned maps applied to the content
+ * signal).  The outputs feed frac_scan_fwd / frac_scan_bwd / frac_decode_step directly.
+ * Variants (frac_prep_config.flags):
+ *   FRAC_PREP_ZOH_INJECTION : w_write is divided by lambda, so that the scan's
+ *       kappa = (1 - rho) w_write is the exact zero-order-hold injection (1 - rho~)/lambda of
+ *       Eq. rho-beta-def-frac instead of Algorithm 1's 1 - rho~.
+ *   FRAC_PREP_NO_SOFTMAX    : weights = the logits themselves (App. G ablation "w/o softmax R/W";
+ *       the normalisation is removed and nothing replaces it).
+ *   FRAC_PREP_NO_READ_PRIOR / FRAC_PREP_NO_WRITE_PRIOR : drop -alpha ln tau from the read / write
+ *       logits (App. G ablations "w/o write prior"; both: the "pure multiscale bank").
+ *   FRAC_PREP_ALPHA_ONE     : alpha = 1 for every token (App. G ablation; alpha_raw may be NULL
+ *       and gets a zero gradient).
+ * dims: batch and seqlen (rows = batch x seqlen positions; seqlen 1 for a decode step), nheads,
+ * nmodes (1..32) and dtype (of the logits, the weights and their gradients) are used; the other
+ * fields are ignored.  Layouts:
+ *   dt_raw, alpha_raw, lam_raw, dt, alpha, lam (+ grads)  [batch, seqlen, nheads]  float32
+ *   g_read, g_write, w_read, w_write (+ grads)             [batch, seqlen, nheads, nmodes]  dtype
+ *   dt_bias, ddt_bias [nheads] float32 (NULL = no bias / not wanted); tau, dtau [nheads, nmodes]
+ * Arithmetic is float32.  Errors as for the scan calls (everything checked before anything is
+ * enqueued); no workspace is needed.
+ */
+typedef struct {
+    float dt_min, dt_max;   /* clip of Delta: the language-modelling setting uses [1e-4, 1] */
+    float lam_min, lam_max; /* clip of lambda: [0.25, 4] there */
+    int32_t flags;          /* FRAC_PREP_* */
+    int32_t reserved;       /* must be 0 */
+} frac_prep_config;
+
+enum {
+    FRAC_PREP_ZOH_INJECTION = 1,
+    FRAC_PREP_NO_SOFTMAX = 2,
+    FRAC_PREP_NO_READ_PRIOR = 4,
+    FRAC_PREP_NO_WRITE_PRIOR = 8,
+    FRAC_PREP_ALPHA_ONE = 16
+};
+
+frac_status frac_param_prep_fwd(const frac_dims *dims, const frac_prep_config *cfg,
+                                const float *dt_raw, const float *dt_bias, const float *alpha_raw,
+                                const float *lam_raw, const void *g_read, const void *g_write,
+                                const float *tau, float *dt, float *alpha, float *lam,
+                                void *w_read, void *w_write, void *stream);
+
+/*
+ * Backward of frac_param_prep_fwd: from the gradients of its outputs (ddt, dalpha, dlam,
+ * dw_read, dw_write: typically those frac_scan_bwd returned) to the gradients of its inputs.
+ * Clipping passes the gradient where the clipped value lies inside [min, max] (bounds
+ * included).  ddt_bias [nheads] sums the Delta gradient over positions; dtau [nheads, nmodes]
+ * is the part of the timescale gradient that flows through the -alpha ln tau prior (add
+ * frac_scan_bwd's dtau for learned timescales).  Both are overwritten; NULL = not wanted.
+ * The sums over positions use float atomics: their rounding order is not fixed.
+ */
+frac_status frac_param_prep_bwd(const frac_dims *dims, const frac_prep_config *cfg,
+                                const float *dt_raw, const float *dt_bias, const float *alpha_raw,
+                                const float *lam_raw, const void *g_read, const void *g_write,
+                                const float *tau, const float *ddt, const float *dalpha,
+                                const float *dlam, const void *dw_read, const void *dw_write,
+                                float *ddt_raw, float *dalpha_raw, float *dlam_raw, void *dg_read,
+                                void *dg_write, float *ddt_bias, float *dtau, void *stream);
+
+/*
  * Kernel tracing (a profiling aid, off by default).  While enabled, every kernel the library
  * launches is bracketed by two CUDA events recorded on its launch stream (do not enable it
  * while a stream is being captured into a CUDA graph).  frac_trace_collect waits for the

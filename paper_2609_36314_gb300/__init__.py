@@ -3,9 +3,9 @@
 The scan runs in hand-written CUDA kernels behind the C ABI of include/frac.h
 (libfrac.so, built in-tree); this package only marshals torch tensors to it.
 """
-from .api import (bwd_workspace_size, decode_step, fwd_workspace_size, make_dims, scan_bwd,
-                  scan_fwd)
+from .api import (bwd_workspace_size, decode_step, fwd_workspace_size, make_dims,
+                  param_prep_bwd, param_prep_fwd, prep_config, scan_bwd, scan_fwd)
 from ._lib import FracError
 
 __all__ = ["scan_fwd", "scan_bwd", "decode_step", "fwd_workspace_size", "bwd_workspace_size",
-           "make_dims", "FracError"]
+           "make_dims", "param_prep_fwd", "param_prep_bwd", "prep_config", "FracError"]

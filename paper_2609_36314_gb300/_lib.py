@@ -23,6 +23,8 @@ EXPORTS = (
     "frac_scan_fwd_static",
     "frac_scan_fwd_static_status",
     "frac_workspace_status",
+    "frac_param_prep_fwd",
+    "frac_param_prep_bwd",
     "frac_trace_enable",
     "frac_trace_collect",
     "frac_trace_reset",
@@ -45,6 +47,19 @@ class FracDims(ctypes.Structure):
                 ("ngroups", ctypes.c_int64), ("dstate", ctypes.c_int64),
                 ("nmodes", ctypes.c_int64), ("chunk", ctypes.c_int64),
                 ("dtype", ctypes.c_int32), ("flags", ctypes.c_int32)]
+
+
+class FracPrepConfig(ctypes.Structure):
+    _fields_ = [("dt_min", ctypes.c_float), ("dt_max", ctypes.c_float),
+                ("lam_min", ctypes.c_float), ("lam_max", ctypes.c_float),
+                ("flags", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+FRAC_PREP_ZOH_INJECTION = 1
+FRAC_PREP_NO_SOFTMAX = 2
+FRAC_PREP_NO_READ_PRIOR = 4
+FRAC_PREP_NO_WRITE_PRIOR = 8
+FRAC_PREP_ALPHA_ONE = 16
 
 
 class FracTraceEntry(ctypes.Structure):
@@ -91,6 +106,11 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.frac_scan_fwd_static.restype = st
         lib.frac_scan_fwd_static_status.argtypes = [P]
         lib.frac_scan_fwd_static_status.restype = st
+        cfg_p = ctypes.POINTER(FracPrepConfig)
+        lib.frac_param_prep_fwd.argtypes = [dims_p, cfg_p] + [P] * 12 + [P]
+        lib.frac_param_prep_fwd.restype = st
+        lib.frac_param_prep_bwd.argtypes = [dims_p, cfg_p] + [P] * 19 + [P]
+        lib.frac_param_prep_bwd.restype = st
         lib.frac_workspace_status.argtypes = [P, P]
         lib.frac_workspace_status.restype = st
         lib.frac_trace_enable.argtypes = [ctypes.c_int]

@@ -192,3 +192,80 @@ def decode_step(x_t, dt, alpha, lam, tau, B_t, C_t, w_read, w_write, D, state, y
         _ptr(C_t), _ptr(w_read), _ptr(w_write), _ptr(D), _ptr(state), _ptr(y_t),
         _stream(stream)), "frac_decode_step")
     return y_t
+
+
+def prep_config(dt_min=1e-4, dt_max=1.0, lam_min=0.25, lam_max=4.0, zoh_injection=False,
+                no_softmax=False, no_read_prior=False, no_write_prior=False,
+                alpha_one=False) -> _lib.FracPrepConfig:
+    """Clip ranges (defaults: the language-modelling setting) and variant flags of the
+    scan-parameter construction."""
+    flags = ((_lib.FRAC_PREP_ZOH_INJECTION if zoh_injection else 0) |
+             (_lib.FRAC_PREP_NO_SOFTMAX if no_softmax else 0) |
+             (_lib.FRAC_PREP_NO_READ_PRIOR if no_read_prior else 0) |
+             (_lib.FRAC_PREP_NO_WRITE_PRIOR if no_write_prior else 0) |
+             (_lib.FRAC_PREP_ALPHA_ONE if alpha_one else 0))
+    return _lib.FracPrepConfig(dt_min, dt_max, lam_min, lam_max, flags, 0)
+
+
+def _prep_dims(dt_raw, g_read, tau):
+    if dt_raw.dim() < 1 or g_read.dim() != dt_raw.dim() + 1 or tau.dim() != 2:
+        raise ValueError("dt_raw [..., H], g_read [..., H, K], tau [H, K] expected")
+    H, K = tau.shape
+    if dt_raw.shape[-1] != H or g_read.shape[-1] != K:
+        raise ValueError("head / mode counts of dt_raw, g_read and tau differ")
+    rows = dt_raw.numel() // H
+    return make_dims(1, rows, H, 1, 1, 1, K, g_read.dtype)
+
+
+def param_prep_fwd(dt_raw, alpha_raw, lam_raw, g_read, g_write, tau, dt_bias=None, cfg=None,
+                   out=None, stream=None):
+    """Scan controls and mode weights from the projections' outputs.  Returns a dict with
+    dt, alpha, lam (float32, shape of dt_raw) and w_read, w_write (dtype of g_read)."""
+    cfg = cfg or prep_config()
+    dims = _prep_dims(dt_raw, g_read, tau)
+    f32 = torch.float32
+    for name, t in (("dt_raw", dt_raw), ("lam_raw", lam_raw), ("tau", tau)):
+        _need(t, name, f32)
+    if alpha_raw is not None:
+        _need(alpha_raw, "alpha_raw", f32, dt_raw.shape)
+    _need(lam_raw, "lam_raw", f32, dt_raw.shape)
+    _need(g_write, "g_write", g_read.dtype, g_read.shape)
+    _need(g_read, "g_read", g_read.dtype)
+    if dt_bias is not None:
+        _need(dt_bias, "dt_bias", f32, (tau.shape[0],))
+    o = out if out is not None else dict(
+        dt=torch.empty_like(dt_raw), alpha=torch.empty_like(dt_raw), lam=torch.empty_like(dt_raw),
+        w_read=torch.empty_like(g_read), w_write=torch.empty_like(g_read))
+    _lib.check(_lib.load().frac_param_prep_fwd(
+        ctypes.byref(dims), ctypes.byref(cfg), _ptr(dt_raw), _ptr(dt_bias), _ptr(alpha_raw),
+        _ptr(lam_raw), _ptr(g_read), _ptr(g_write), _ptr(tau), _ptr(o["dt"]), _ptr(o["alpha"]),
+        _ptr(o["lam"]), _ptr(o["w_read"]), _ptr(o["w_write"]), _stream(stream)),
+        "frac_param_prep_fwd")
+    return o
+
+
+def param_prep_bwd(dt_raw, alpha_raw, lam_raw, g_read, g_write, tau, ddt, dalpha, dlam, dw_read,
+                   dw_write, dt_bias=None, cfg=None, want_dt_bias=True, want_dtau=True,
+                   stream=None):
+    """Backward of param_prep_fwd.  Returns a dict with ddt_raw, dalpha_raw, dlam_raw,
+    dg_read, dg_write, and ddt_bias [H] / dtau [H, K] (None when not wanted)."""
+    cfg = cfg or prep_config()
+    dims = _prep_dims(dt_raw, g_read, tau)
+    f32 = torch.float32
+    for name, t in (("ddt", ddt), ("dalpha", dalpha), ("dlam", dlam)):
+        _need(t, name, f32, dt_raw.shape)
+    for name, t in (("dw_read", dw_read), ("dw_write", dw_write)):
+        _need(t, name, g_read.dtype, g_read.shape)
+    H, K = tau.shape
+    g = dict(ddt_raw=torch.empty_like(dt_raw), dalpha_raw=torch.empty_like(dt_raw),
+             dlam_raw=torch.empty_like(dt_raw), dg_read=torch.empty_like(g_read),
+             dg_write=torch.empty_like(g_read),
+             ddt_bias=torch.empty(H, dtype=f32, device=tau.device) if want_dt_bias else None,
+             dtau=torch.empty((H, K), dtype=f32, device=tau.device) if want_dtau else None)
+    _lib.check(_lib.load().frac_param_prep_bwd(
+        ctypes.byref(dims), ctypes.byref(cfg), _ptr(dt_raw), _ptr(dt_bias), _ptr(alpha_raw),
+        _ptr(lam_raw), _ptr(g_read), _ptr(g_write), _ptr(tau), _ptr(ddt), _ptr(dalpha),
+        _ptr(dlam), _ptr(dw_read), _ptr(dw_write), _ptr(g["ddt_raw"]), _ptr(g["dalpha_raw"]),
+        _ptr(g["dlam_raw"]), _ptr(g["dg_read"]), _ptr(g["dg_write"]), _ptr(g["ddt_bias"]),
+        _ptr(g["dtau"]), _stream(stream)), "frac_param_prep_bwd")
+    return g

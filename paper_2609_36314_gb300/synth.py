@@ -28,7 +28,8 @@ import numpy as np
 
 # tensor ids for the per-tensor streams
 _IDS = dict(x=0, dt=1, alpha=2, lam=3, B=4, C=5, w_read=6, w_write=7, D=8, dy=9, h0=10,
-            dh_final=11)
+            dh_final=11, up_dt=12, up_alpha=13, up_lam=14, up_w_read=15, up_w_write=16,
+            u=17, conv_w=18, conv_b=19, z=20, norm_w=21, dout=22, conv_state=23)
 
 
 @dataclasses.dataclass(frozen=True)
@@ -171,6 +172,29 @@ def make_decode_inputs(s: Shape, steps: int, seed: int = 0) -> dict:
         w_write=cast(mode_weights(alpha, tau, normal(seed, "w_write", (steps, Bz, H, K), sub)), s.dtype),
         D=normal(seed, "D", (H,)),
     )
+
+
+def make_prep_inputs(s: Shape, seed: int = 0, with_grads: bool = False) -> dict:
+    """Inputs of the scan-parameter construction with the same distributions as the scan recipe
+    above: the raw controls are the z draws (Delta's shift is the per-head bias), the logits
+    0.5 z (sigma(0) z).  With with_grads, upstream gradients of its five outputs ~ N(0, 1)."""
+    Bz, L, H, K = s.batch, s.seqlen, s.nheads, s.nmodes
+    out = dict(
+        dt_raw=normal(seed, "dt", (Bz, L, H)),
+        alpha_raw=normal(seed, "alpha", (Bz, L, H)),
+        lam_raw=normal(seed, "lam", (Bz, L, H)),
+        g_read=cast(0.5 * normal(seed, "w_read", (Bz, L, H, K)), s.dtype),
+        g_write=cast(0.5 * normal(seed, "w_write", (Bz, L, H, K)), s.dtype),
+        tau=timescales(K, H),
+        dt_bias=np.full((H,), -s.dt_shift, dtype=np.float32),
+    )
+    if with_grads:
+        out.update(
+            ddt=normal(seed, "up_dt", (Bz, L, H)), dalpha=normal(seed, "up_alpha", (Bz, L, H)),
+            dlam=normal(seed, "up_lam", (Bz, L, H)),
+            dw_read=cast(normal(seed, "up_w_read", (Bz, L, H, K)), s.dtype),
+            dw_write=cast(normal(seed, "up_w_write", (Bz, L, H, K)), s.dtype))
+    return out
 
 
 def rel_l2(a, b) -> float:

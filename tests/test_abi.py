@@ -108,3 +108,22 @@ def test_decode_rejects_null_state():
     st = lib.frac_decode_step(ctypes.byref(dims), p, p, p, p, p, p, p, p, p, p, None, p, None)
     assert st == 1
     assert b"state" in lib.frac_last_error()
+
+
+@pytest.mark.parametrize("bad", ["flags", "order", "modes", "null_cfg"])
+def test_param_prep_rejects_bad_arguments(bad):
+    """The scan-parameter calls check dims and the config before touching the device."""
+    import torch
+    from paper_2609_36314_gb300.api import prep_config
+    lib = _lib.load()
+    dims = make_dims(batch=1, seqlen=8, nheads=2, headdim=1, ngroups=1, dstate=1,
+                     nmodes=33 if bad == "modes" else 4, dtype=torch.float32)
+    cfg = prep_config(dt_min=2.0 if bad == "order" else 1e-4)
+    if bad == "flags":
+        cfg.flags = 1 << 10
+    p = ctypes.c_void_p(0x1000)
+    cfg_ref = None if bad == "null_cfg" else ctypes.byref(cfg)
+    st = lib.frac_param_prep_fwd(ctypes.byref(dims), cfg_ref, *([p] * 12), None)
+    assert st == 1
+    st = lib.frac_param_prep_bwd(ctypes.byref(dims), cfg_ref, *([p] * 19), None)
+    assert st == 1
