@@ -166,7 +166,9 @@ int frac_oracle_decode(int64_t Bsz, int64_t H, int64_t P, int64_t G, int64_t N, 
  *   dDelta     = sum_m dz_m z_m / Delta
  *   dlambda    = sum_m dz_m z_m / (alpha lambda)
  *   dalpha     = sum_m dz_m z_m (-ln lambda / alpha^2)
- * (rho_m z_m is taken as its limit 0 when z_m = +inf.)  dh0 = final dS.
+ *   dtau_m     = sum over b, t of dz_m z_m (-1 / tau_m)   (z = Delta lambda^(1/alpha) / tau: the
+ *                timescale gradient of the App. G "learned timescales" variant)
+ * (rho_m z_m is taken as its limit 0 when z_m = +inf.)  dh0 = final dS.  dtau may be NULL.
  */
 int frac_oracle_bwd(int64_t Bsz, int64_t L, int64_t H, int64_t P, int64_t G, int64_t N, int64_t K,
                     const double *x, const double *dt, const double *alpha, const double *lam,
@@ -174,7 +176,7 @@ int frac_oracle_bwd(int64_t Bsz, int64_t L, int64_t H, int64_t P, int64_t G, int
                     const double *ww, const double *D, const double *h0, const double *dy,
                     const double *dh_final, double *dx, double *ddt, double *dalpha, double *dlam,
                     double *dB, double *dC, double *dwr, double *dww, double *dD, double *dh0,
-                    int64_t seg, int nthreads) {
+                    double *dtau, int64_t seg, int nthreads) {
     dims_t d = {Bsz, L, H, P, G, N, K};
     if (!valid(&d)) return 2;
     if (seg <= 0) seg = 32;
@@ -184,7 +186,8 @@ int frac_oracle_bwd(int64_t Bsz, int64_t L, int64_t H, int64_t P, int64_t G, int
     double *pB = (double *)calloc((size_t)(Bsz * H * L * N > 0 ? Bsz * H * L * N : 1), sizeof(double));
     double *pC = (double *)calloc((size_t)(Bsz * H * L * N > 0 ? Bsz * H * L * N : 1), sizeof(double));
     double *pD = (double *)calloc((size_t)(Bsz * H > 0 ? Bsz * H : 1), sizeof(double));
-    if (!pB || !pC || !pD) { free(pB); free(pC); free(pD); return 1; }
+    double *pT = (double *)calloc((size_t)(Bsz * H * K > 0 ? Bsz * H * K : 1), sizeof(double));
+    if (!pB || !pC || !pD || !pT) { free(pB); free(pC); free(pD); free(pT); return 1; }
     int err = 0;
 #pragma omp parallel for schedule(dynamic, 1) num_threads(nthreads > 0 ? nthreads : 1)
     for (int64_t bh = 0; bh < Bsz * H; ++bh) {
@@ -278,6 +281,7 @@ int frac_oracle_bwd(int64_t Bsz, int64_t L, int64_t H, int64_t P, int64_t G, int
                     gdt += dz_z / dt[i];
                     glm += dz_z / (al * lam[i]);
                     gal += dz_z * (-lnl / (al * al));
+                    pT[bh * K + m] += dz_z * (-1.0 / tau[h * K + m]);
                 }
                 ddt[i] = gdt;
                 dlam[i] = glm;
@@ -304,8 +308,15 @@ int frac_oracle_bwd(int64_t Bsz, int64_t L, int64_t H, int64_t P, int64_t G, int
             for (int64_t b = 0; b < Bsz; ++b) s += pD[b * H + h];
             dD[h] = s;
         }
+        if (dtau)
+            for (int64_t h = 0; h < H; ++h)
+                for (int64_t m = 0; m < K; ++m) {
+                    double s = 0.0;
+                    for (int64_t b = 0; b < Bsz; ++b) s += pT[(b * H + h) * K + m];
+                    dtau[h * K + m] = s;
+                }
     }
-    free(pB); free(pC); free(pD);
+    free(pB); free(pC); free(pD); free(pT);
     return err;
 }
 

@@ -54,7 +54,7 @@ def _load():
             i64, dp, ci = ctypes.c_int64, ctypes.c_void_p, ctypes.c_int
             lib.frac_oracle_fwd.argtypes = [i64] * 7 + [dp] * 13 + [ci]
             lib.frac_oracle_fwd.restype = ci
-            lib.frac_oracle_bwd.argtypes = [i64] * 7 + [dp] * 23 + [i64, ci]
+            lib.frac_oracle_bwd.argtypes = [i64] * 7 + [dp] * 24 + [i64, ci]
             lib.frac_oracle_bwd.restype = ci
             lib.frac_oracle_decode.argtypes = [i64] * 6 + [dp] * 12
             lib.frac_oracle_decode.restype = ci
@@ -105,7 +105,8 @@ def bwd(x, dt, alpha, lam, tau, Bm, Cm, w_read, w_write, D, dy, h0=None, dh_fina
         seg=32, nthreads=None):
     """fp64 adjoint of the sequential recurrence.
 
-    Returns a dict with dx, ddt, dalpha, dlam, dB, dC, dw_read, dw_write, dD, dh0.
+    Returns a dict with dx, ddt, dalpha, dlam, dB, dC, dw_read, dw_write, dD, dh0 and dtau
+    (the gradient of the timescales tau [H, K]).
     """
     x, dt, alpha, lam, tau, Bm, Cm, w_read, w_write, D, dy, h0, dh_final = map(
         _f64, (x, dt, alpha, lam, tau, Bm, Cm, w_read, w_write, D, dy, h0, dh_final))
@@ -113,14 +114,14 @@ def bwd(x, dt, alpha, lam, tau, Bm, Cm, w_read, w_write, D, dy, h0=None, dh_fina
     out = dict(dx=np.empty_like(x), ddt=np.empty_like(dt), dalpha=np.empty_like(alpha),
                dlam=np.empty_like(lam), dB=np.empty_like(Bm), dC=np.empty_like(Cm),
                dw_read=np.empty_like(w_read), dw_write=np.empty_like(w_write),
-               dD=np.empty_like(D), dh0=np.empty((Bsz, H, K, P, N)))
+               dD=np.empty_like(D), dh0=np.empty((Bsz, H, K, P, N)), dtau=np.empty_like(tau))
     nt = nthreads or max_threads()
     rc = _load().frac_oracle_bwd(
         Bsz, L, H, P, G, N, K, _ptr(x), _ptr(dt), _ptr(alpha), _ptr(lam), _ptr(tau), _ptr(Bm),
         _ptr(Cm), _ptr(w_read), _ptr(w_write), _ptr(D), _ptr(h0), _ptr(dy), _ptr(dh_final),
         _ptr(out["dx"]), _ptr(out["ddt"]), _ptr(out["dalpha"]), _ptr(out["dlam"]),
         _ptr(out["dB"]), _ptr(out["dC"]), _ptr(out["dw_read"]), _ptr(out["dw_write"]),
-        _ptr(out["dD"]), _ptr(out["dh0"]), int(seg), nt)
+        _ptr(out["dD"]), _ptr(out["dh0"]), _ptr(out["dtau"]), int(seg), nt)
     if rc:
         raise RuntimeError(f"frac_oracle_bwd failed with code {rc}")
     return out

@@ -23,6 +23,15 @@ terms that each carry their own decay factor (pairs k < t <= t' inside the chunk
 the S_in / dS_out terms), not as a difference of suffix sums: the latter cancels
 catastrophically once e_t is large, because the true value is then ~0 while the summands
 are O(1) and get multiplied by e_t in dDelta.
+
+The timescale gradient needs the same quantity per mode, weighted by e_t:
+dtau_m = tau_m^-2 sum_t e_t (rho_t <dS_t, S_{t-1}>_m - dkappa_{t,m} rho_{t,m} w_write_{t,m}).
+Each term of the chunked decomposition covers a span of positions whose e_t sum in closed form
+(sum over t in (k, t'] of e_t = E_t' - E_k), so per chunk and mode
+  sum_t e_t rho_t <dS_t, S_{t-1}>_m = E_end d_m <dS_out, S_in>_m
+      + sum_k (E_end - E_k) kappa_k dkappa^inter_k + sum_t E_t w_read_t dw_read_t
+      - sum_k E_k kappa_k dkappa^intra_k
+with dkappa^inter / dkappa^intra the parts of dkappa from dS_out and from the chunk's own pairs.
 """
 from __future__ import annotations
 
@@ -158,6 +167,7 @@ def bwd(x, dt, alpha, lam, tau, Bm, Cm, wr, ww, D, dy, h0=None, dh_final=None, Q
     dD = np.zeros(H)
     dh0 = np.zeros((Bz, H, K, P, N))
     Rp = np.zeros_like(dt)          # sum_m rho_t <dS_t, S_{t-1}>_m / tau_m
+    Te = np.zeros((H, K))           # sum over b, t of e_t rho_t <dS_t, S_{t-1}>_m
     for b in range(Bz):
         for h in range(H):
             g = h // hpg
@@ -187,8 +197,14 @@ def bwd(x, dt, alpha, lam, tau, Bm, Cm, wr, ww, D, dy, h0=None, dh_final=None, Q
                 GH = Gm * Hm
                 xU = np.einsum("kp,kmp->km", xc, U)
                 dyZ = np.einsum("tp,tmp->tm", dyc, Z)
-                dkap[b, c0:c1, h] = u * xU + np.einsum("tm,tkm,tk->km", w_r, W, GH)
+                dk_inter = u * xU
+                dk_intra = np.einsum("tm,tkm,tk->km", w_r, W, GH)
+                dkap[b, c0:c1, h] = dk_inter + dk_intra
                 dwr[b, c0:c1, h] = fdec * dyZ + np.einsum("km,tkm,tk->tm", k_, W, GH)
+                cdot = np.einsum("mpn,mpn->m", dS, S_in)
+                Te[h] += (E[-1] * dm * cdot + np.sum((E[-1] - E)[:, None] * k_ * dk_inter, axis=0)
+                          + np.sum(E[:, None] * w_r * dwr[b, c0:c1, h], axis=0)
+                          - np.sum(E[:, None] * k_ * dk_intra, axis=0))
                 dC[b, c0:c1, g] += (np.einsum("tm,tp,mpn->tn", f, dyc, S_in)
                                     + (Gam * Hm) @ Bc)
                 dB[b, c0:c1, g] += (np.einsum("km,kp,mpn->kn", s, xc, dS)
@@ -210,5 +226,6 @@ def bwd(x, dt, alpha, lam, tau, Bm, Cm, wr, ww, D, dy, h0=None, dh_final=None, Q
     dlam = de * e / (alpha * lam)
     dalpha = -de * e * np.log(lam) / alpha ** 2
     dww = dkap * (-np.expm1(-e[..., None] / tau[None, None]))
+    dtau = (Te - np.einsum("blh,blhm->hm", e, dkap * rho * ww)) / tau ** 2
     return dict(dx=dx, ddt=ddt, dalpha=dalpha, dlam=dlam, dB=dB, dC=dC, dw_read=dwr,
-                dw_write=dww, dD=dD, dh0=dh0)
+                dw_write=dww, dD=dD, dh0=dh0, dtau=dtau)

@@ -13,9 +13,9 @@ import torch
 from oracle import oracle
 from paper_2609_36314_gb300 import synth
 
-NAMES = ["x", "dt", "alpha", "lam", "B", "C", "w_read", "w_write", "D", "h0"]
+NAMES = ["x", "dt", "alpha", "lam", "B", "C", "w_read", "w_write", "D", "h0", "tau"]
 GRAD = dict(x="dx", dt="ddt", alpha="dalpha", lam="dlam", B="dB", C="dC", w_read="dw_read",
-            w_write="dw_write", D="dD", h0="dh0")
+            w_write="dw_write", D="dD", h0="dh0", tau="dtau")
 
 
 def _inputs(seed=2, L=9, shift=0.0):
@@ -24,6 +24,9 @@ def _inputs(seed=2, L=9, shift=0.0):
     d = {k: synth.to_f64(v) for k, v in d.items()}
     # keep lambda^(1/alpha) moderate so finite differences are well conditioned
     d["alpha"] = 0.3 + 0.6 * d["alpha"]
+    # per-head timescales that differ between heads (learned-timescale variant), spanning the
+    # range where the modes neither die within a step nor stay constant over the sequence
+    d["tau"] = (2.0 ** np.linspace(-1.0, 5.0, d["tau"].size)).reshape(d["tau"].shape)
     return d
 
 
@@ -86,7 +89,7 @@ def test_backward_matches_torch_autograd_of_naive_layer():
         synth.Shape(2, 11, 4, 3, 2, 2, 3, 0, "f32"), seed=5)["alpha"])
     g = _grads(d)
     T = {k: torch.tensor(d[k], dtype=torch.float64, requires_grad=(k in NAMES))
-         for k in NAMES + ["tau"]}
+         for k in NAMES}
     y, hf = _torch_layer(T["x"], T["dt"], T["alpha"], T["lam"], T["tau"], T["B"], T["C"],
                          T["w_read"], T["w_write"], T["D"], T["h0"])
     yo, hfo = oracle.fwd(d["x"], d["dt"], d["alpha"], d["lam"], d["tau"], d["B"], d["C"],
