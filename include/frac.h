@@ -145,6 +145,10 @@ frac_status frac_scan_bwd_workspace_size(const frac_dims *dims, size_t *bytes);
  *   ddt, dalpha, dlam : gradients (float32)
  *   dD       : gradient of D (float32 [H]), summed over batch and sequence
  *   dh0      : gradient of h0 (float32), or NULL if not wanted
+ *   dtau     : gradient of the timescales tau (float32 [H, K], summed over batch and sequence),
+ *              or NULL if not wanted: the learned-timescale variant (App. G).  It is the e_t-
+ *              weighted per-mode decay gradient, gathered chunk by chunk from terms whose spans
+ *              of e_t sum in closed form; its sums use float atomics (rounding order not fixed).
  * dB / dC sum over the heads of each group.  All outputs are overwritten (not accumulated).
  */
 frac_status frac_scan_bwd(const frac_dims *dims, const void *x, const float *dt,
@@ -153,7 +157,7 @@ frac_status frac_scan_bwd(const frac_dims *dims, const void *x, const float *dt,
                           const void *w_write, const float *D, const float *h0,
                           const void *dy, const float *dh_final, void *dx, float *ddt,
                           float *dalpha, float *dlam, void *dB, void *dC, void *dw_read,
-                          void *dw_write, float *dD, float *dh0, void *workspace,
+                          void *dw_write, float *dD, float *dh0, float *dtau, void *workspace,
                           size_t workspace_bytes, void *stream);
 
 /*

@@ -98,7 +98,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.frac_scan_bwd_workspace_size.restype = st
         lib.frac_scan_fwd.argtypes = [dims_p] + [P] * 13 + [P, ctypes.c_size_t, P]
         lib.frac_scan_fwd.restype = st
-        lib.frac_scan_bwd.argtypes = [dims_p] + [P] * 23 + [P, ctypes.c_size_t, P]
+        lib.frac_scan_bwd.argtypes = [dims_p] + [P] * 24 + [P, ctypes.c_size_t, P]
         lib.frac_scan_bwd.restype = st
         lib.frac_decode_step.argtypes = [dims_p] + [P] * 12 + [P]
         lib.frac_decode_step.restype = st

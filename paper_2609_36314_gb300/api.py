@@ -129,11 +129,12 @@ def scan_fwd_static(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, h0=None, *
 
 
 def scan_bwd(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, dy, h0=None, dh_final=None, *,
-             chunk=0, force_simt=False, want_dh0=True, workspace=None, out=None, stream=None,
-             reuse_fwd_states=False):
+             chunk=0, force_simt=False, want_dh0=True, want_dtau=False, workspace=None, out=None,
+             stream=None, reuse_fwd_states=False):
     """Backward of scan_fwd.  Returns a dict of gradients (dx, ddt, dalpha, dlam, dB, dC,
-    dw_read, dw_write, dD, dh0).  With reuse_fwd_states, `workspace` must be the buffer a
-    scan_fwd call on the same inputs just used (sized with bwd_workspace_size)."""
+    dw_read, dw_write, dD, dh0, dtau; dh0 / dtau None when not wanted).  With reuse_fwd_states,
+    `workspace` must be the buffer a scan_fwd call on the same inputs just used (sized with
+    bwd_workspace_size)."""
     if reuse_fwd_states and workspace is None:
         raise ValueError("reuse_fwd_states needs the workspace of the forward call")
     dims, (Bz, L, H, P, G, N, K) = _scan_dims(x, B, tau, chunk, force_simt, reuse_fwd_states)
@@ -153,14 +154,16 @@ def scan_bwd(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, dy, h0=None, dh_f
         dlam=torch.empty_like(lam), dB=torch.empty_like(B), dC=torch.empty_like(C),
         dw_read=torch.empty_like(w_read), dw_write=torch.empty_like(w_write),
         dD=torch.empty_like(D),
-        dh0=torch.empty((Bz, H, K, P, N), dtype=f32, device=x.device) if want_dh0 else None)
+        dh0=torch.empty((Bz, H, K, P, N), dtype=f32, device=x.device) if want_dh0 else None,
+        dtau=torch.empty((H, K), dtype=f32, device=x.device) if want_dtau else None)
     ws = _workspace(bwd_workspace_size(dims), x.device, workspace)
     _lib.check(_lib.load().frac_scan_bwd(
         ctypes.byref(dims), _ptr(x), _ptr(dt), _ptr(alpha), _ptr(lam), _ptr(tau), _ptr(B),
         _ptr(C), _ptr(w_read), _ptr(w_write), _ptr(D), _ptr(h0), _ptr(dy), _ptr(dh_final),
         _ptr(g["dx"]), _ptr(g["ddt"]), _ptr(g["dalpha"]), _ptr(g["dlam"]), _ptr(g["dB"]),
         _ptr(g["dC"]), _ptr(g["dw_read"]), _ptr(g["dw_write"]), _ptr(g["dD"]),
-        _ptr(g.get("dh0")), _ptr(ws), ws.numel(), _stream(stream)), "frac_scan_bwd")
+        _ptr(g.get("dh0")), _ptr(g.get("dtau")), _ptr(ws), ws.numel(), _stream(stream)),
+        "frac_scan_bwd")
     return g
 
 

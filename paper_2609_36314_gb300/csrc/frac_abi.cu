@@ -274,8 +274,8 @@ frac_status frac_scan_bwd(const frac_dims *d, const void *x, const float *dt, co
                           const void *w_read, const void *w_write, const float *D,
                           const float *h0, const void *dy, const float *dh_final, void *dx,
                           float *ddt, float *dalpha, float *dlam, void *dB, void *dC,
-                          void *dw_read, void *dw_write, float *dD, float *dh0, void *workspace,
-                          size_t workspace_bytes, void *stream) {
+                          void *dw_read, void *dw_write, float *dD, float *dh0, float *dtau,
+                          void *workspace, size_t workspace_bytes, void *stream) {
     g_err[0] = 0;
     frac_status s = check_dims(d, true);
     if (s) return s;
@@ -285,6 +285,7 @@ frac_status frac_scan_bwd(const frac_dims *d, const void *x, const float *dt, co
     OPTIONAL_PTR(h0);
     OPTIONAL_PTR(dh_final);
     OPTIONAL_PTR(dh0);
+    OPTIONAL_PTR(dtau);
     if (d->seqlen > 0) {
         REQUIRE_T(x); REQUIRE_PTR(dt); REQUIRE_PTR(alpha); REQUIRE_PTR(lam);
         REQUIRE_T(Bm); REQUIRE_T(Cm); REQUIRE_T(w_read); REQUIRE_T(w_write);
@@ -333,7 +334,7 @@ frac_status frac_scan_bwd(const frac_dims *d, const void *x, const float *dt, co
     p.dt = dt; p.alpha = alpha; p.lam = lam; p.tau = tau; p.D = D; p.h0 = h0;
     p.dh_final = dh_final;
     p.dx = dx; p.dB = dB; p.dC = dC; p.dwr = dw_read; p.dww = dw_write;
-    p.ddt = ddt; p.dalpha = dalpha; p.dlam = dlam; p.dD = dD; p.dh0 = dh0;
+    p.ddt = ddt; p.dalpha = dalpha; p.dlam = dlam; p.dD = dD; p.dh0 = dh0; p.dtau = dtau;
     char *ws = static_cast<char *>(workspace);
     float *dB_acc = d->dtype == FRAC_DTYPE_BF16 ? reinterpret_cast<float *>(ws + l.db)
                                                 : static_cast<float *>(dB);

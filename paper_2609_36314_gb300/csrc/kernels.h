@@ -41,6 +41,7 @@ struct ScanPtrs {
     const float *dt, *alpha, *lam, *tau, *D, *h0, *dh_final;
     void *y, *dx, *dB, *dC, *dwr, *dww;
     float *h_final, *ddt, *dalpha, *dlam, *dD, *dh0;
+    float *dtau;  // [H, K] timescale gradient, or null when not wanted
 };
 
 // CUDA-core (SIMT) chunked path; works for float32 and bf16 I/O.
@@ -90,6 +91,7 @@ struct TcBwdWorkspace {  // S_in and coef first, at the offsets the forward uses
     float *coef;                             // [B,L,H,4,K]: f, s, u, exp(-E/tau)
     float *ek;                               // [B,L,H,tc_ek_width(K)]: E (hi, lo), kappa
     float *dB_acc, *dC_acc;                  // [B,L,G,N] x 2
+    float *dkap_intra;                       // [B,L,H,K]: the intra-chunk part of dkappa (dtau)
 };
 size_t tc_bwd_workspace_bytes(const ScanDims &d, TcBwdWorkspace *layout, char *base);
 cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspace &ws, int *err,

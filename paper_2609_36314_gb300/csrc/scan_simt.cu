@@ -232,7 +232,8 @@ __global__ void __launch_bounds__(kThreads) simt_chunk_fwd(
     const int tid = threadIdx.x;
 
     double *E_s = reinterpret_cast<double *>(smem_raw);
-    float *e_s = reinterpret_cast<float *>(E_s + kQMax);
+    double *dtq_s = E_s + kQMax;    // [32] per mode: sum over the chunk of the dtau terms
+    float *e_s = reinterpret_cast<float *>(dtq_s + 32);
     float *itau = e_s + kQMax;
     float *wr_s = itau + 32;            // [Q][K]
     float *kap_s = wr_s + Q * K;        // [Q][K]
@@ -419,7 +420,7 @@ __global__ void __launch_bounds__(kThreads) simt_chunk_bwd(
     const TS *__restrict__ dS_out, T *__restrict__ dx, T *__restrict__ dwr_o,
     T *__restrict__ dww_o, float *__restrict__ ddt, float *__restrict__ dalpha,
     float *__restrict__ dlam, float *__restrict__ dD, float *__restrict__ dB_acc,
-    float *__restrict__ dC_acc) {
+    float *__restrict__ dC_acc, float *__restrict__ dtau) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
     const int g = h / (d.H / d.G);
@@ -430,12 +431,14 @@ __global__ void __launch_bounds__(kThreads) simt_chunk_bwd(
     const int QK = Q * K;
 
     double *E_s = reinterpret_cast<double *>(smem_raw);
-    float *e_s = reinterpret_cast<float *>(E_s + kQMax);
+    double *dtq_s = E_s + kQMax;    // [32] per mode: sum over the chunk of the dtau terms
+    float *e_s = reinterpret_cast<float *>(dtq_s + 32);
     float *cl_s = e_s + kQMax;
     float *itau = cl_s + kQMax;     // [32]
     float *dec = itau + 32;         // [32]
     float *red = dec + 32;          // [32]
-    float *a_s = red + 32;          // [kQMax]
+    float *cdm_s = red + 32;        // [32] per mode: <S_in, dS_out>
+    float *a_s = cdm_s + 32;        // [kQMax]
     float *b_s = a_s + kQMax;       // [kQMax]
     float *rp_s = b_s + kQMax;      // [kQMax]
     float *wr_s = rp_s + kQMax;     // [Q][K] x 11
@@ -462,6 +465,10 @@ __global__ void __launch_bounds__(kThreads) simt_chunk_bwd(
 
     // ---- loads
     if (tid < K) itau[tid] = 1.f / tau[h * K + tid];
+    if (tid < 32) {
+        dtq_s[tid] = 0.0;
+        cdm_s[tid] = 0.f;
+    }
     const float log_cap = head_log_cap(tau, h, K);
     chunk_rates(d, b, h, c0, n, log_cap, dt, alpha, lam, e_s, E_s, cl_s);
     for (int idx = tid; idx < Q * P; idx += blockDim.x) {
@@ -643,6 +650,7 @@ __global__ void __launch_bounds__(kThreads) simt_chunk_bwd(
             dot = fmaf(sv, dv, dot);
         }
         cpart = fmaf(dec[mm] * itau[mm], dot, cpart);
+        if (dtau) atomicAdd(&cdm_s[mm], dot);
         __syncthreads();
         if (has_x) {
             float Uq[4][4] = {}, Zq[4][4] = {};
@@ -784,6 +792,16 @@ __global__ void __launch_bounds__(kThreads) simt_chunk_bwd(
             de = fmaf(dk * rho_s[q] * ww_s[q], itau[mm], de);
             dwr_o[wi0 + mm] = from_f<T>(dw);
             dww_o[wi0 + mm] = from_f<T>(dk * omr_s[q]);
+            if (dtau) {
+                // e_t-weighted decay gradient of this position and mode: every term of the chunked
+                // decomposition spans positions whose e sum in closed form (E_t, E_end - E_t, E_end)
+                const double Et = E_s[t], Eend = E_s[n - 1];
+                const double tq = Et * double(wr_s[q]) * double(dw) +
+                                  (Eend - Et) * double(kap_s[q]) * double(dk) -
+                                  Eend * double(kap_s[q]) * double(dkpi[q]) -
+                                  double(e_s[t]) * double(dk) * double(rho_s[q]) * double(ww_s[q]);
+                atomicAdd(&dtq_s[mm], tq);
+            }
         }
         const size_t i = blh(d, b, c0 + t, h);
         const float e = e_s[t];
@@ -794,13 +812,20 @@ __global__ void __launch_bounds__(kThreads) simt_chunk_bwd(
         dlam[i] = ge / (al * lm);
         dalpha[i] = -ge * logf(lm) / (al * al);
     }
+    if (dtau) {  // dtau_m += (sum_t ... + E_end d_m <dS_out, S_in>_m) / tau_m^2
+        __syncthreads();
+        if (tid < K)
+            atomicAdd(&dtau[h * K + tid],
+                      float((dtq_s[tid] + E_s[n - 1] * double(dec[tid]) * double(cdm_s[tid])) *
+                            double(itau[tid]) * double(itau[tid])));
+    }
 }
 
 size_t chunk_bwd_smem(const ScanDims &d) {
     const size_t Q = d.Q, P1 = d.P + 1, N1 = d.N + 1;
     const size_t uni = std::max(3 * Q * (Q + 1), 2 * size_t(d.P) * N1);
-    return sizeof(double) * kQMax +
-           sizeof(float) * (2 * kQMax + 3 * 32 + 3 * kQMax + 11 * Q * d.K + 2 * Q * P1 +
+    return sizeof(double) * (kQMax + 32) +
+           sizeof(float) * (2 * kQMax + 4 * 32 + 3 * kQMax + 11 * Q * d.K + 2 * Q * P1 +
                             2 * Q * N1 + uni);
 }
 
@@ -1058,6 +1083,7 @@ cudaError_t bwd_t(const ScanDims &d, const ScanPtrs &p, void *S_in, void *dS_out
     if ((e = cudaMemsetAsync(p.dD, 0, sizeof(float) * d.H, st)) != cudaSuccess) return e;
     if ((e = cudaMemsetAsync(dB_acc, 0, sizeof(float) * ngn, st)) != cudaSuccess) return e;
     if ((e = cudaMemsetAsync(dC_acc, 0, sizeof(float) * ngn, st)) != cudaSuccess) return e;
+    if (p.dtau && (e = cudaMemsetAsync(p.dtau, 0, sizeof(float) * d.H * d.K, st)) != cudaSuccess) return e;
     if (d.nc == 0) return cudaSuccess;  // L = 0: dh0 = dh_final was written, dD = 0
     const size_t smem = chunk_bwd_smem(d);
     auto k = simt_chunk_bwd<T, TS>;
@@ -1067,7 +1093,7 @@ cudaError_t bwd_t(const ScanDims &d, const ScanPtrs &p, void *S_in, void *dS_out
         d, (const T *)p.x, (const T *)p.Bm, (const T *)p.Cm, (const T *)p.wr, (const T *)p.ww,
         (const T *)p.dy, p.dt, p.alpha, p.lam, p.tau, p.D, (const TS *)S_in,
         (const TS *)dS_out, (T *)p.dx, (T *)p.dwr, (T *)p.dww, p.ddt, p.dalpha, p.dlam, p.dD,
-        dB_acc, dC_acc);
+        dB_acc, dC_acc, p.dtau);
     trace_end(st);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if (sizeof(T) == 2 && ngn > 0) {

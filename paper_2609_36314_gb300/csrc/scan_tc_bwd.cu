@@ -49,6 +49,7 @@ struct BwdArgs {
     const float *ek;  // per position: {E hi, E lo, 0, 0, kappa[K]} [B, L, H, tc_ek_width(K)]
     bf16 *dx, *dwr, *dww;
     float *ddt, *dalpha, *dlam, *dD;
+    float *dkap_intra, *dtau;  // both null unless the timescale gradient is wanted
     int *err;
     int hg;      // heads per dC/dB group
     int pf_sms;  // SMs of the device: CTAs of the persistent intra kernel
@@ -677,6 +678,12 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
 #pragma unroll
             for (int m = 0; m < KMAX; ++m)
                 if (m < K) o[m] = dk[m] + part[t * KMAX + m];
+            if (a.dkap_intra) {  // kept apart from the inter-chunk part for the timescale gradient
+                float *oi = a.dkap_intra + blh(d, b, c0 + t, h) * K;
+#pragma unroll
+                for (int m = 0; m < KMAX; ++m)
+                    if (m < K) oi[m] = dk[m] + part[t * KMAX + m];
+            }
             a.rect[blh(d, b, c0 + t, h)] = sr + rpart[t];
         }
         sync_first256();
@@ -1249,6 +1256,7 @@ __global__ void __launch_bounds__(kThreads) tc_bwd_final(BwdArgs a) {
     __shared__ float itau[32], tau_sh[32];
     __shared__ float sh[4];
     __shared__ float red[4];
+    __shared__ float tq_sh[4][KMAX];  // per warp and mode: sums of the timescale-gradient terms
     if (t < K) {
         const float tv = a.tau[h * K + t];
         tau_sh[t] = tv;
@@ -1323,6 +1331,45 @@ __global__ void __launch_bounds__(kThreads) tc_bwd_final(BwdArgs a) {
         a.ddt[i] = ge / dtv;
         a.dlam[i] = ge / (alv * lmv);
         a.dalpha[i] = -ge * logf(lmv) / (alv * alv);
+    }
+    if (a.dtau) {
+        // Timescale gradient: per mode, the e_t-weighted decay gradient of this position.  Every
+        // term of the chunked decomposition spans positions whose e sum in closed form (E_t from
+        // the chunk start, E_end - E_t to its end), so with the intra-chunk part of dkappa apart:
+        //   E_t w_read dw_read + (E_end - E_t) kappa dkappa - E_end kappa dkappa_intra
+        //   - e_t dkappa rho w_write,  plus E_end d_m <dS_out, S_in>_m once per chunk.
+        float wrv[KMAX], dki[KMAX];
+#pragma unroll
+        for (int m = 0; m < KMAX; ++m) wrv[m] = dki[m] = 0.f;
+        if (t < n) {
+            load_weights(a.wr + i * K, K, wrv);
+#pragma unroll
+            for (int q = 0; q < KMAX / 4; ++q)
+                if (4 * q < K) {
+                    const float4 u = *reinterpret_cast<const float4 *>(a.dkap_intra + i * K + 4 * q);
+                    dki[4 * q] = u.x; dki[4 * q + 1] = u.y; dki[4 * q + 2] = u.z; dki[4 * q + 3] = u.w;
+                }
+        }
+#pragma unroll
+        for (int m = 0; m < KMAX; ++m) {
+            float v = 0.f;
+            if (t < n && m < K) {
+                const float z = e * itau[m];
+                const float rho = expf(-z), kap = -expm1f(-z) * ww[m];
+                // E_end - E_t as the exclusive suffix of e (scanned directly, no difference of sums)
+                v = pe * wrv[m] * dwv[m] + (se - e) * kap * dkv[m] - Eend * kap * dki[m] -
+                    e * dkv[m] * rho * ww[m];
+            }
+            v = warp_sum(v);
+            if (lane == 0) tq_sh[w][m] = v;
+        }
+        __syncthreads();
+        if (t < K) {
+            const float cd = a.cdot[((size_t(b) * d.H + h) * d.nc + c) * K + t];
+            const float sum = (tq_sh[0][t] + tq_sh[1][t]) + (tq_sh[2][t] + tq_sh[3][t]) +
+                              Eend * expf(-Eend * itau[t]) * cd;
+            atomicAdd(a.dtau + h * K + t, sum * itau[t] * itau[t]);
+        }
     }
     // dx = dx_acc + D dy (bf16) and sum dy x: each thread takes 8 p of 8 rows (rows r = 16 j + t / 8,
     // p in [8 (t % 8), 8 (t % 8) + 8)), all loads issued before any is used; every instruction
@@ -1417,6 +1464,7 @@ size_t tc_bwd_workspace_bytes(const ScanDims &d, TcBwdWorkspace *l, char *base) 
     l->mh_total = (float *)take(size_t(d.B) * d.nc * d.G * TQ * TQ * 4);
     l->dB_acc = (float *)take(size_t(d.B) * d.L * d.G * d.N * 4);
     l->dC_acc = (float *)take(size_t(d.B) * d.L * d.G * d.N * 4);
+    l->dkap_intra = (float *)take(blh_ * d.K * 4);
     return off;
 }
 
@@ -1429,6 +1477,7 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
     if ((e = cudaMemsetAsync(ws.dC_acc, 0, sizeof(float) * ngn, st))) return e;
     if ((e = cudaMemsetAsync(ws.cdot, 0, sizeof(float) * d.B * d.H * d.nc * d.K, st))) return e;
     if ((e = cudaMemsetAsync(ws.mh_total, 0, sizeof(float) * d.B * d.nc * d.G * TQ * TQ, st))) return e;
+    if (p.dtau && (e = cudaMemsetAsync(p.dtau, 0, sizeof(float) * d.H * d.K, st))) return e;
     if (!reuse_states &&
         ((e = tc_coef_launch(d, p, ws.coef, ws.ek, st)) ||
          (e = tc_state_pass_launch(d, false, p.x, p.Bm, ws.coef, p.h0, ws.S_in, nullptr, err, st))))
@@ -1470,6 +1519,8 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
     a.dB_acc = ws.dB_acc; a.dC_acc = ws.dC_acc;
     a.dx = (bf16 *)p.dx; a.dwr = (bf16 *)p.dwr; a.dww = (bf16 *)p.dww;
     a.ddt = p.ddt; a.dalpha = p.dalpha; a.dlam = p.dlam; a.dD = p.dD;
+    a.dtau = p.dtau;
+    a.dkap_intra = p.dtau ? ws.dkap_intra : nullptr;
     a.err = err;
     {
         int dev = 0, nsm = 0;

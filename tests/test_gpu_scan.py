@@ -302,3 +302,51 @@ def test_bwd_reusing_forward_states(dtype):
     torch.cuda.synchronize()
     for k in GRADS:
         assert torch.equal(g[k], g_ref[k]) or synth.rel_l2(to_host64(g[k]), to_host64(g_ref[k])) < 1e-6, k
+
+
+# ------------------------------------------------------------------ learned timescales (dtau)
+def _learned_tau(d64, dv, seed):
+    """Per-head timescales off the geometric grid (the learned-timescale variant, App. G)."""
+    rng = np.random.default_rng(seed)
+    tau = (d64["tau"] * np.exp(0.3 * rng.standard_normal(d64["tau"].shape))).astype(np.float32)
+    d64["tau"] = tau.astype(np.float64)
+    dv["tau"] = torch.from_numpy(tau).cuda()
+
+
+@pytest.mark.parametrize("dtype,shape", [
+    ("f32", synth.Shape(2, 150, 3, 16, 1, 8, 4, 32, "f32")),          # CUDA-core path
+    ("bf16", synth.Shape(2, 260, 4, 64, 1, 64, 8, 0, "bf16")),        # tensor-core path
+    ("bf16", synth.Shape(1, 300, 4, 64, 2, 128, 4, 0, "bf16")),       # tensor-core, K = 4, G = 2
+    ("f32", synth.Shape(1, 200, 2, 256, 1, 1, 16, 0, "f32")),         # the paper's N = 1 shape
+])
+def test_bwd_timescale_gradient(dtype, shape):
+    host = synth.make_scan_inputs(shape, seed=31, with_dy=True, with_h0=True, with_dh_final=True)
+    d64 = f64_inputs(host)
+    dv = dev_inputs(host)
+    _learned_tau(d64, dv, 32)
+    g = _gpu_bwd(dv, chunk=shape.chunk, want_dtau=True)
+    torch.cuda.synchronize()
+    ref = _ora_bwd(d64)
+    assert_close("dtau", to_host64(g["dtau"]), ref["dtau"], tol(dtype))
+    assert_close("ddt", to_host64(g["ddt"]), ref["ddt"], tol(dtype))
+
+
+def test_bwd_timescale_gradient_reusing_forward_states():
+    """The benchmarked mode (one workspace, the backward reusing the forward's states) with
+    the timescale gradient, on the tensor-core path."""
+    s = synth.Shape(2, 384, 4, 64, 1, 128, 8, 0, "bf16")
+    host = synth.make_scan_inputs(s, seed=33, with_dy=True)
+    d64 = f64_inputs(host)
+    dv = dev_inputs(host)
+    _learned_tau(d64, dv, 34)
+    from paper_2609_36314_gb300.api import bwd_workspace_size, fwd_workspace_size, make_dims
+    dims = make_dims(s.batch, s.seqlen, s.nheads, s.headdim, s.ngroups, s.dstate, s.nmodes,
+                     torch.bfloat16)
+    ws = torch.empty(max(bwd_workspace_size(dims), fwd_workspace_size(dims)), dtype=torch.uint8,
+                     device="cuda")
+    _gpu_fwd(dv, workspace=ws, want_final_state=False)
+    g = _gpu_bwd(dv, workspace=ws, reuse_fwd_states=True, want_dtau=True)
+    torch.cuda.synchronize()
+    ref = _ora_bwd(d64)
+    for k in GRADS + ["dtau"]:
+        assert_close(k, to_host64(g[k]), ref[k], 1e-2)
