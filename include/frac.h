@@ -282,6 +282,73 @@ frac_status frac_param_prep_bwd(const frac_dims *dims, const frac_prep_config *c
                                 void *dg_write, float *ddt_bias, float *dtau, void *stream);
 
 /*
+ * Depthwise causal 1-D convolution of the FracMixer content branch (Sec. 3.3: u_t comes from a
+ * local depthwise causal convolution along the sequence; width d_conv = 4 in App. E.2 / E.4):
+ *   pre[b, t, c] = bias_c + sum_{j=0}^{W-1} w[c, j] x[b, t - (W-1) + j, c]
+ *   u = pre, or u = silu(pre) = pre * sigmoid(pre) with FRAC_CONV_SILU (the activation of the
+ *   Mamba-family mixers the layer follows; the paper names only the convolution)
+ * Positions before the sequence start read a carried state of the W - 1 previous inputs
+ * (state_in [B, C, W-1], oldest first; NULL = zeros), which makes prefill -> decode and split
+ * sequences exact.  Layouts: x, u, du, dx [B, L, C] and states in dims->dtype; w [C, W], bias
+ * [C] (NULL = none) and their gradients float32.  W <= 8, L <= 16,776,960.  Arithmetic is
+ * float32.
+ */
+typedef struct {
+    int64_t batch;    /* B >= 1 */
+    int64_t seqlen;   /* L >= 0 (ignored by frac_conv1d_step) */
+    int64_t channels; /* C >= 1 */
+    int64_t width;    /* W, 1 <= W <= 8 */
+    int32_t dtype;    /* frac_dtype of x, u, the states and their gradients */
+    int32_t flags;    /* FRAC_CONV_* */
+} frac_conv_dims;
+
+enum { FRAC_CONV_SILU = 1 };
+
+/* Forward over a sequence.  state_out [B, C, W-1] (or NULL) receives the last W - 1 inputs
+   (the carried state for a continuation); it must not alias state_in. */
+frac_status frac_conv1d_fwd(const frac_conv_dims *dims, const void *x, const float *w,
+                            const float *bias, const void *state_in, void *u, void *state_out,
+                            void *stream);
+
+/* Backward of frac_conv1d_fwd's u: dx; dw [C, W] and dbias [C] summed over batch and sequence
+   (overwritten; float atomics, rounding order not fixed); dstate_in [B, C, W-1] (or NULL) the
+   gradient of the carried inputs. */
+frac_status frac_conv1d_bwd(const frac_conv_dims *dims, const void *x, const float *w,
+                            const float *bias, const void *state_in, const void *du, void *dx,
+                            float *dw, float *dbias, void *dstate_in, void *stream);
+
+/* One decode step: x_t, u_t [B, C]; state [B, C, W-1] is read and shifted in place (the newest
+   input x_t enters at the end). */
+frac_status frac_conv1d_step(const frac_conv_dims *dims, const void *x_t, const float *w,
+                             const float *bias, void *state, void *u_t, void *stream);
+
+/*
+ * Gated RMS normalisation of the scan output before the output projection (Sec. 3.3 "gated
+ * normalization", read as the Mamba2 form the layer design follows):
+ *   v = y * silu(z)  (v = y when z is NULL),   out = v / sqrt(mean_group(v^2) + eps) * weight
+ * with the mean over consecutive groups of group_size features of each row.  y, z, out and
+ * their gradients [rows, dim] in dtype (16-byte aligned); weight, dweight [dim] float32.
+ * group_size must be a multiple of 8 that divides dim; dim <= 32768.
+ */
+typedef struct {
+    int64_t rows;       /* >= 0 (e.g. batch x seqlen) */
+    int64_t dim;        /* features per row */
+    int64_t group_size; /* features per normalisation group (dim for one group) */
+    float eps;          /* >= 0, e.g. 1e-5 */
+    int32_t dtype;      /* frac_dtype */
+    int32_t flags;      /* 0 */
+} frac_norm_dims;
+
+frac_status frac_gated_rmsnorm_fwd(const frac_norm_dims *dims, const void *y, const void *z,
+                                   const float *weight, void *out, void *stream);
+
+/* Backward: dy, dz (NULL when z is NULL) and dweight (overwritten, summed over rows by float
+   atomics: rounding order not fixed). */
+frac_status frac_gated_rmsnorm_bwd(const frac_norm_dims *dims, const void *y, const void *z,
+                                   const float *weight, const void *dout, void *dy, void *dz,
+                                   float *dweight, void *stream);
+
+/*
  * Kernel tracing (a profiling aid, off by default).  While enabled, every kernel the library
  * launches is bracketed by two CUDA events recorded on its launch stream (do not enable it
  * while a stream is being captured into a CUDA graph).  frac_trace_collect waits for the

@@ -25,6 +25,11 @@ EXPORTS = (
     "frac_workspace_status",
     "frac_param_prep_fwd",
     "frac_param_prep_bwd",
+    "frac_conv1d_fwd",
+    "frac_conv1d_bwd",
+    "frac_conv1d_step",
+    "frac_gated_rmsnorm_fwd",
+    "frac_gated_rmsnorm_bwd",
     "frac_trace_enable",
     "frac_trace_collect",
     "frac_trace_reset",
@@ -60,6 +65,21 @@ FRAC_PREP_NO_SOFTMAX = 2
 FRAC_PREP_NO_READ_PRIOR = 4
 FRAC_PREP_NO_WRITE_PRIOR = 8
 FRAC_PREP_ALPHA_ONE = 16
+
+
+class FracConvDims(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int64), ("seqlen", ctypes.c_int64),
+                ("channels", ctypes.c_int64), ("width", ctypes.c_int64),
+                ("dtype", ctypes.c_int32), ("flags", ctypes.c_int32)]
+
+
+FRAC_CONV_SILU = 1
+
+
+class FracNormDims(ctypes.Structure):
+    _fields_ = [("rows", ctypes.c_int64), ("dim", ctypes.c_int64),
+                ("group_size", ctypes.c_int64), ("eps", ctypes.c_float),
+                ("dtype", ctypes.c_int32), ("flags", ctypes.c_int32)]
 
 
 class FracTraceEntry(ctypes.Structure):
@@ -111,6 +131,18 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.frac_param_prep_fwd.restype = st
         lib.frac_param_prep_bwd.argtypes = [dims_p, cfg_p] + [P] * 19 + [P]
         lib.frac_param_prep_bwd.restype = st
+        conv_p = ctypes.POINTER(FracConvDims)
+        norm_p = ctypes.POINTER(FracNormDims)
+        lib.frac_conv1d_fwd.argtypes = [conv_p] + [P] * 6 + [P]
+        lib.frac_conv1d_fwd.restype = st
+        lib.frac_conv1d_bwd.argtypes = [conv_p] + [P] * 9 + [P]
+        lib.frac_conv1d_bwd.restype = st
+        lib.frac_conv1d_step.argtypes = [conv_p] + [P] * 5 + [P]
+        lib.frac_conv1d_step.restype = st
+        lib.frac_gated_rmsnorm_fwd.argtypes = [norm_p] + [P] * 4 + [P]
+        lib.frac_gated_rmsnorm_fwd.restype = st
+        lib.frac_gated_rmsnorm_bwd.argtypes = [norm_p] + [P] * 7 + [P]
+        lib.frac_gated_rmsnorm_bwd.restype = st
         lib.frac_workspace_status.argtypes = [P, P]
         lib.frac_workspace_status.restype = st
         lib.frac_trace_enable.argtypes = [ctypes.c_int]

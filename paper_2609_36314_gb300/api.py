@@ -272,3 +272,94 @@ def param_prep_bwd(dt_raw, alpha_raw, lam_raw, g_read, g_write, tau, ddt, dalpha
         _ptr(g["dlam_raw"]), _ptr(g["dg_read"]), _ptr(g["dg_write"]), _ptr(g["ddt_bias"]),
         _ptr(g["dtau"]), _stream(stream)), "frac_param_prep_bwd")
     return g
+
+
+# ----------------------------------------------------------------------------- mixer glue
+def _conv_dims(x, w, silu):
+    if x.dim() != 3 or w.dim() != 2 or w.shape[0] != x.shape[2]:
+        raise ValueError("x [B, L, C], w [C, W] expected")
+    return _lib.FracConvDims(x.shape[0], x.shape[1], x.shape[2], w.shape[1], _DT[x.dtype],
+                             _lib.FRAC_CONV_SILU if silu else 0)
+
+
+def conv1d_fwd(x, w, bias=None, state=None, *, silu=False, want_state=False, stream=None):
+    """Depthwise causal conv1d over [B, L, C] (optionally SiLU).  Returns (u, final state
+    [B, C, W-1] or None)."""
+    dims = _conv_dims(x, w, silu)
+    _need(x, "x", x.dtype)
+    _need(w, "w", torch.float32)
+    B, L, C = x.shape
+    W = w.shape[1]
+    if bias is not None:
+        _need(bias, "bias", torch.float32, (C,))
+    if state is not None:
+        _need(state, "state", x.dtype, (B, C, W - 1))
+    u = torch.empty_like(x)
+    fin = torch.empty((B, C, W - 1), dtype=x.dtype, device=x.device) if want_state else None
+    _lib.check(_lib.load().frac_conv1d_fwd(ctypes.byref(dims), _ptr(x), _ptr(w), _ptr(bias),
+                                           _ptr(state), _ptr(u), _ptr(fin), _stream(stream)),
+               "frac_conv1d_fwd")
+    return u, fin
+
+
+def conv1d_bwd(x, w, du, bias=None, state=None, *, silu=False, want_dstate=False, stream=None):
+    """Backward of conv1d_fwd.  Returns dict(dx, dw, dbias, dstate)."""
+    dims = _conv_dims(x, w, silu)
+    B, L, C = x.shape
+    W = w.shape[1]
+    _need(du, "du", x.dtype, x.shape)
+    g = dict(dx=torch.empty_like(x), dw=torch.empty_like(w),
+             dbias=torch.empty(C, dtype=torch.float32, device=x.device) if bias is not None else None,
+             dstate=torch.empty((B, C, W - 1), dtype=x.dtype, device=x.device) if want_dstate else None)
+    _lib.check(_lib.load().frac_conv1d_bwd(
+        ctypes.byref(dims), _ptr(x), _ptr(w), _ptr(bias), _ptr(state), _ptr(du), _ptr(g["dx"]),
+        _ptr(g["dw"]), _ptr(g["dbias"]), _ptr(g["dstate"]), _stream(stream)), "frac_conv1d_bwd")
+    return g
+
+
+def conv1d_step(x_t, w, state, bias=None, *, silu=False, u_t=None, stream=None):
+    """One decode step of the conv: x_t [B, C]; state [B, C, W-1] shifts in place."""
+    B, C = x_t.shape
+    W = w.shape[1]
+    _need(x_t, "x_t", x_t.dtype)
+    _need(state, "state", x_t.dtype, (B, C, W - 1))
+    dims = _lib.FracConvDims(B, 1, C, W, _DT[x_t.dtype], _lib.FRAC_CONV_SILU if silu else 0)
+    if u_t is None:
+        u_t = torch.empty_like(x_t)
+    _lib.check(_lib.load().frac_conv1d_step(ctypes.byref(dims), _ptr(x_t), _ptr(w), _ptr(bias),
+                                            _ptr(state), _ptr(u_t), _stream(stream)),
+               "frac_conv1d_step")
+    return u_t
+
+
+def _norm_dims(y, group_size, eps):
+    if y.dim() != 2:
+        raise ValueError("y [rows, dim] expected")
+    R, D = y.shape
+    return _lib.FracNormDims(R, D, group_size or D, float(eps), _DT[y.dtype], 0)
+
+
+def gated_rmsnorm_fwd(y, z, weight, group_size=0, eps=1e-5, stream=None):
+    """RMSNorm(y * silu(z)) * weight over groups of group_size features (0: the whole row)."""
+    dims = _norm_dims(y, group_size, eps)
+    _need(y, "y", y.dtype)
+    if z is not None:
+        _need(z, "z", y.dtype, y.shape)
+    _need(weight, "weight", torch.float32, (y.shape[1],))
+    out = torch.empty_like(y)
+    _lib.check(_lib.load().frac_gated_rmsnorm_fwd(ctypes.byref(dims), _ptr(y), _ptr(z),
+                                                  _ptr(weight), _ptr(out), _stream(stream)),
+               "frac_gated_rmsnorm_fwd")
+    return out
+
+
+def gated_rmsnorm_bwd(y, z, weight, dout, group_size=0, eps=1e-5, stream=None):
+    """Backward of gated_rmsnorm_fwd.  Returns dict(dy, dz, dweight)."""
+    dims = _norm_dims(y, group_size, eps)
+    _need(dout, "dout", y.dtype, y.shape)
+    g = dict(dy=torch.empty_like(y), dz=torch.empty_like(y) if z is not None else None,
+             dweight=torch.empty_like(weight))
+    _lib.check(_lib.load().frac_gated_rmsnorm_bwd(
+        ctypes.byref(dims), _ptr(y), _ptr(z), _ptr(weight), _ptr(dout), _ptr(g["dy"]),
+        _ptr(g["dz"]), _ptr(g["dweight"]), _stream(stream)), "frac_gated_rmsnorm_bwd")
+    return g

@@ -1,0 +1,716 @@
+// The FracMixer operations around the scan (Sec. 3.3), HBM-bound:
+//
+//   depthwise causal conv1d   u[b,t,c] = act(bias_c + sum_j w[c,j] x[b, t-(W-1)+j, c])
+//        (the content branch; width d_conv, 4 in App. E.2 / E.4; act = identity or SiLU; the
+//        W-1 inputs before the sequence come from a carried state, zeros by default), its
+//        backward, and one decode step that shifts the carried state;
+//   gated RMS normalisation   out = v / sqrt(mean_group(v^2) + eps) * weight,  v = y * silu(z)
+//        (before the output projection), and its backward.
+//
+// conv1d: a thread owns two adjacent channels and a run of kRun consecutive positions; a warp
+// covers 64 contiguous channels of one position per access.  The filter window of the last W-1
+// inputs stays in registers.  The backward streams g = du * act'(pre) through a register ring of
+// the last W values (dx_t needs g at t .. t+W-1), and reduces dw / dbias over the block's rows
+// of runs in shared memory before one atomic per channel and block.
+// RMSNorm: one CTA per row, 8-element vectors, per-group sums by shared-memory atomics.  The
+// backward is persistent over rows: each thread owns fixed feature positions, so its dweight
+// partials sit in shared memory without atomics until one global atomic per feature and CTA.
+#include <algorithm>
+#include <cstdio>
+
+#include "../../include/frac.h"
+#include "common.cuh"
+#include "kernels.h"
+
+namespace frac {
+namespace {
+
+constexpr int kRun = 32;      // positions per thread (conv1d)
+constexpr int kRows = 8;      // runs per block (threadIdx.y)
+constexpr int kMaxW = 8;      // largest conv width
+
+__device__ __forceinline__ float sigm(float a) {
+    const float e = expf(-fabsf(a));
+    return a >= 0.f ? 1.f / (1.f + e) : e / (1.f + e);
+}
+__device__ __forceinline__ float silu_f(float a) { return a * sigm(a); }
+__device__ __forceinline__ float silu_grad_f(float a) {
+    const float s = sigm(a);
+    return s * (1.f + a * (1.f - s));
+}
+
+// two adjacent channels (c, c + 1) of one position; VEC2: one 2-element access (C even, aligned)
+template <typename T, bool VEC2>
+__device__ __forceinline__ float2 ld2(const T *p, bool has1) {
+    if constexpr (VEC2) {
+        if constexpr (sizeof(T) == 2) {
+            const __nv_bfloat162 v = *reinterpret_cast<const __nv_bfloat162 *>(p);
+            return __bfloat1622float2(v);
+        } else {
+            return *reinterpret_cast<const float2 *>(p);
+        }
+    } else {
+        return make_float2(to_f(p[0]), has1 ? to_f(p[1]) : 0.f);
+    }
+}
+template <typename T, bool VEC2>
+__device__ __forceinline__ void st2(T *p, float2 v, bool has1) {
+    if constexpr (VEC2) {
+        if constexpr (sizeof(T) == 2)
+            *reinterpret_cast<__nv_bfloat162 *>(p) = __floats2bfloat162_rn(v.x, v.y);
+        else
+            *reinterpret_cast<float2 *>(p) = v;
+    } else {
+        p[0] = from_f<T>(v.x);
+        if (has1) p[1] = from_f<T>(v.y);
+    }
+}
+
+struct ConvArgs {
+    int B, L, C, W;
+    bool silu;
+    const void *x, *state_in, *du;
+    const float *w, *bias;
+    void *u, *state_out, *dx, *dstate;
+    float *dw, *dbias;
+};
+
+// input at position t (t < 0 reads the carried state: index W-1+t, oldest first) for channel c
+template <typename T>
+__device__ __forceinline__ float x_at(const ConvArgs &a, int b, int t, int c) {
+    if (t >= 0) return to_f(static_cast<const T *>(a.x)[(size_t(b) * a.L + t) * a.C + c]);
+    if (!a.state_in) return 0.f;
+    return to_f(static_cast<const T *>(a.state_in)[(size_t(b) * a.C + c) * (a.W - 1) + (a.W - 1 + t)]);
+}
+
+template <typename T, int W, bool VEC2>
+__global__ void __launch_bounds__(32 * kRows) conv1d_fwd_kernel(ConvArgs a) {
+    const int c = 2 * (blockIdx.x * 32 + threadIdx.x);
+    const int t0 = (blockIdx.y * kRows + threadIdx.y) * kRun;
+    const int b = blockIdx.z;
+    if (c >= a.C || t0 >= a.L) return;
+    const bool has1 = c + 1 < a.C;
+    float w0[W], w1[W];
+#pragma unroll
+    for (int j = 0; j < W; ++j) {
+        w0[j] = a.w[c * W + j];
+        w1[j] = has1 ? a.w[(c + 1) * W + j] : 0.f;
+    }
+    const float b0 = a.bias ? a.bias[c] : 0.f, b1 = (a.bias && has1) ? a.bias[c + 1] : 0.f;
+    float win0[W], win1[W];  // win[j] = input at t - (W-1) + j
+#pragma unroll
+    for (int j = 0; j < W - 1; ++j) {
+        const int t = t0 - (W - 1) + j;
+        if (t >= 0) {
+            const float2 v = ld2<T, VEC2>(static_cast<const T *>(a.x) + (size_t(b) * a.L + t) * a.C + c, has1);
+            win0[j] = v.x;
+            win1[j] = v.y;
+        } else {
+            win0[j] = x_at<T>(a, b, t, c);
+            win1[j] = has1 ? x_at<T>(a, b, t, c + 1) : 0.f;
+        }
+    }
+    const int t1 = min(t0 + kRun, a.L);
+    for (int t = t0; t < t1; ++t) {
+        const size_t off = (size_t(b) * a.L + t) * a.C + c;
+        const float2 xv = ld2<T, VEC2>(static_cast<const T *>(a.x) + off, has1);
+        win0[W - 1] = xv.x;
+        win1[W - 1] = xv.y;
+        float p0 = b0, p1 = b1;
+#pragma unroll
+        for (int j = 0; j < W; ++j) {
+            p0 = fmaf(w0[j], win0[j], p0);
+            p1 = fmaf(w1[j], win1[j], p1);
+        }
+        if (a.silu) {
+            p0 = silu_f(p0);
+            p1 = silu_f(p1);
+        }
+        st2<T, VEC2>(static_cast<T *>(a.u) + off, make_float2(p0, p1), has1);
+        if (a.state_out && t >= a.L - (W - 1)) {  // the last W-1 inputs become the carried state
+            T *so = static_cast<T *>(a.state_out);
+            const int k = t - (a.L - (W - 1));
+            so[(size_t(b) * a.C + c) * (W - 1) + k] = from_f<T>(xv.x);
+            if (has1) so[(size_t(b) * a.C + c + 1) * (W - 1) + k] = from_f<T>(xv.y);
+        }
+#pragma unroll
+        for (int j = 0; j < W - 1; ++j) {
+            win0[j] = win0[j + 1];
+            win1[j] = win1[j + 1];
+        }
+    }
+    if (a.state_out && t0 == 0 && a.L < W - 1) {  // short sequence: part of the old state stays
+        T *so = static_cast<T *>(a.state_out);
+        for (int k = 0; k < W - 1 - a.L; ++k) {
+            so[(size_t(b) * a.C + c) * (W - 1) + k] = from_f<T>(x_at<T>(a, b, k + a.L - (W - 1), c));
+            if (has1)
+                so[(size_t(b) * a.C + c + 1) * (W - 1) + k] = from_f<T>(x_at<T>(a, b, k + a.L - (W - 1), c + 1));
+        }
+    }
+}
+
+template <typename T, int W, bool VEC2>
+__global__ void __launch_bounds__(32 * kRows) conv1d_bwd_kernel(ConvArgs a) {
+    __shared__ float red[kRows][W + 1][64];  // per run row: dw taps and dbias of the 64 channels
+    const int lane = threadIdx.x, ry = threadIdx.y;
+    const int c = 2 * (blockIdx.x * 32 + lane);
+    const int t0 = (blockIdx.y * kRows + ry) * kRun;
+    const int b = blockIdx.z;
+    const bool active = c < a.C && t0 < a.L;
+    const bool has1 = c + 1 < a.C;
+    float acc0[W + 1], acc1[W + 1];  // dw taps, then dbias
+#pragma unroll
+    for (int j = 0; j <= W; ++j) acc0[j] = acc1[j] = 0.f;
+    if (active) {
+        float w0[W], w1[W];
+#pragma unroll
+        for (int j = 0; j < W; ++j) {
+            w0[j] = a.w[c * W + j];
+            w1[j] = has1 ? a.w[(c + 1) * W + j] : 0.f;
+        }
+        const float b0 = a.bias ? a.bias[c] : 0.f, b1 = (a.bias && has1) ? a.bias[c + 1] : 0.f;
+        float win0[W], win1[W], g0[W], g1[W];  // inputs t-(W-1) .. t; g at t-(W-1) .. t
+#pragma unroll
+        for (int j = 0; j < W; ++j) g0[j] = g1[j] = 0.f;
+#pragma unroll
+        for (int j = 0; j < W - 1; ++j) {
+            const int t = t0 - (W - 1) + j;
+            win0[j] = x_at<T>(a, b, t, c);
+            win1[j] = has1 ? x_at<T>(a, b, t, c + 1) : 0.f;
+        }
+        const int tr = min(t0 + kRun, a.L);          // this run's positions: [t0, tr)
+        const int tg = min(tr + W - 1, a.L);         // g is needed up to tg - 1 for dx of the run
+        for (int t = t0; t < tg; ++t) {
+            const size_t off = (size_t(b) * a.L + t) * a.C + c;
+            const float2 xv = ld2<T, VEC2>(static_cast<const T *>(a.x) + off, has1);
+            const float2 dv = ld2<T, VEC2>(static_cast<const T *>(a.du) + off, has1);
+            win0[W - 1] = xv.x;
+            win1[W - 1] = xv.y;
+            float p0 = b0, p1 = b1;
+#pragma unroll
+            for (int j = 0; j < W; ++j) {
+                p0 = fmaf(w0[j], win0[j], p0);
+                p1 = fmaf(w1[j], win1[j], p1);
+            }
+            const float gg0 = a.silu ? dv.x * silu_grad_f(p0) : dv.x;
+            const float gg1 = a.silu ? dv.y * silu_grad_f(p1) : dv.y;
+#pragma unroll
+            for (int j = 0; j < W - 1; ++j) {
+                g0[j] = g0[j + 1];
+                g1[j] = g1[j + 1];
+            }
+            g0[W - 1] = gg0;
+            g1[W - 1] = gg1;
+            if (t < tr) {  // this run's own positions: dw and dbias terms
+#pragma unroll
+                for (int j = 0; j < W; ++j) {
+                    acc0[j] = fmaf(gg0, win0[j], acc0[j]);
+                    acc1[j] = fmaf(gg1, win1[j], acc1[j]);
+                }
+                acc0[W] += gg0;
+                acc1[W] += gg1;
+            }
+            // dx at s = t - (W-1) (all of its g are in the ring once t = s + W - 1 or t = L - 1)
+            const int s = t - (W - 1);
+            if (s >= t0) {
+                float d0 = 0.f, d1 = 0.f;
+#pragma unroll
+                for (int j = 0; j < W; ++j) {  // g at s + (W-1) - j = ring slot W-1-j
+                    d0 = fmaf(w0[j], g0[W - 1 - j], d0);
+                    d1 = fmaf(w1[j], g1[W - 1 - j], d1);
+                }
+                st2<T, VEC2>(static_cast<T *>(a.dx) + (size_t(b) * a.L + s) * a.C + c, make_float2(d0, d1), has1);
+            }
+            if (a.dstate && t0 == 0 && t == min(W - 2, a.L - 1)) {
+                // gradient of the carried inputs i = 0 .. W-2 (position i - (W-1)):
+                // sum over taps j <= i of w_j g[i - j], g[t] at ring slot W-1-(tcur-t)
+                for (int i = 0; i < W - 1; ++i) {
+                    float d0 = 0.f, d1 = 0.f;
+                    for (int j = 0; j <= i && j < W; ++j) {
+                        const int tt = i - j;
+                        if (tt <= t) {
+                            d0 = fmaf(w0[j], g0[W - 1 - (t - tt)], d0);
+                            d1 = fmaf(w1[j], g1[W - 1 - (t - tt)], d1);
+                        }
+                    }
+                    T *ds = static_cast<T *>(a.dstate);
+                    ds[(size_t(b) * a.C + c) * (W - 1) + i] = from_f<T>(d0);
+                    if (has1) ds[(size_t(b) * a.C + c + 1) * (W - 1) + i] = from_f<T>(d1);
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < W - 1; ++j) {
+                win0[j] = win0[j + 1];
+                win1[j] = win1[j + 1];
+            }
+        }
+        // the run's tail positions s in [max(t0, tg - (W-1)), tr): the g beyond the end are 0
+        for (int s = max(t0, tg - (W - 1)); s < tr; ++s) {
+            const int sh = (tg - 1) - s;  // g at s + k sits at ring slot W-1-(tg-1-(s+k))
+            float d0 = 0.f, d1 = 0.f;
+            for (int j = 0; j < W; ++j) {
+                const int k = (W - 1) - j;  // tap j reads g at s + k
+                if (k <= sh) {
+                    d0 = fmaf(w0[j], g0[W - 1 - (sh - k)], d0);
+                    d1 = fmaf(w1[j], g1[W - 1 - (sh - k)], d1);
+                }
+            }
+            st2<T, VEC2>(static_cast<T *>(a.dx) + (size_t(b) * a.L + s) * a.C + c, make_float2(d0, d1), has1);
+        }
+    }
+#pragma unroll
+    for (int j = 0; j <= W; ++j) {
+        red[ry][j][2 * lane] = acc0[j];
+        red[ry][j][2 * lane + 1] = acc1[j];
+    }
+    __syncthreads();
+    // one atomic per channel and tap: threads (lane, ry) split the (W + 1) x 64 sums
+    for (int q = ry * 32 + lane; q < (W + 1) * 64; q += 32 * kRows) {
+        const int j = q / 64, cc = q % 64;
+        const int ch = blockIdx.x * 64 + cc;
+        if (ch >= a.C) continue;
+        float s = 0.f;
+#pragma unroll
+        for (int r = 0; r < kRows; ++r) s += red[r][j][cc];
+        if (j < W)
+            atomicAdd(a.dw + ch * W + j, s);
+        else if (a.dbias)
+            atomicAdd(a.dbias + ch, s);
+    }
+}
+
+// one decode step: window = carried state (W-1 inputs) then x_t; the state shifts by one
+template <typename T>
+__global__ void __launch_bounds__(256) conv1d_step_kernel(ConvArgs a, const T *__restrict__ xt, T *__restrict__ ut) {
+    const int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (i >= int64_t(a.B) * a.C) return;
+    const int c = int(i % a.C);
+    const int W = a.W;
+    T *st = W > 1 ? static_cast<T *>(a.state_out) + i * (W - 1) : nullptr;
+    float p = a.bias ? a.bias[c] : 0.f;
+    float prev[kMaxW];
+    for (int j = 0; j < W - 1; ++j) prev[j] = to_f(st[j]);
+    const float x = to_f(xt[i]);
+    for (int j = 0; j < W - 1; ++j) p = fmaf(a.w[c * W + j], prev[j], p);
+    p = fmaf(a.w[c * W + W - 1], x, p);
+    ut[i] = from_f<T>(a.silu ? silu_f(p) : p);
+    for (int j = 0; j + 1 < W - 1; ++j) st[j] = from_f<T>(prev[j + 1]);
+    if (W > 1) st[W - 2] = from_f<T>(x);
+}
+
+// ------------------------------------------------------------------ gated RMSNorm
+struct NormArgs {
+    int64_t R;
+    int D, gs;
+    float eps;
+    const void *y, *z, *dout;
+    const float *weight;
+    void *out, *dy, *dz;
+    float *dweight;
+};
+
+// 8 consecutive features of one row
+template <typename T>
+__device__ __forceinline__ void ld8(const T *p, float *v) {
+    if constexpr (sizeof(T) == 2) {
+        const uint4 u = *reinterpret_cast<const uint4 *>(p);
+        const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&u);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 f = __bfloat1622float2(h[i]);
+            v[2 * i] = f.x;
+            v[2 * i + 1] = f.y;
+        }
+    } else {
+        const float4 a = reinterpret_cast<const float4 *>(p)[0], b = reinterpret_cast<const float4 *>(p)[1];
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    }
+}
+template <typename T>
+__device__ __forceinline__ void st8(T *p, const float *v) {
+    if constexpr (sizeof(T) == 2) {
+        uint4 u;
+        __nv_bfloat162 *h = reinterpret_cast<__nv_bfloat162 *>(&u);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) h[i] = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+        *reinterpret_cast<uint4 *>(p) = u;
+    } else {
+        reinterpret_cast<float4 *>(p)[0] = make_float4(v[0], v[1], v[2], v[3]);
+        reinterpret_cast<float4 *>(p)[1] = make_float4(v[4], v[5], v[6], v[7]);
+    }
+}
+
+// v = y * silu(z) for 8 features at f of row r
+template <typename T>
+__device__ __forceinline__ void gated8(const NormArgs &a, int64_t r, int f, float *v, float *zv) {
+    ld8<T>(static_cast<const T *>(a.y) + r * a.D + f, v);
+    if (a.z) {
+        ld8<T>(static_cast<const T *>(a.z) + r * a.D + f, zv);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[i] *= silu_f(zv[i]);
+    }
+}
+
+// Requires gs % 8 == 0 and D % 8 == 0 (host-checked): every 8-vector lies in one group.
+template <typename T>
+__global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(NormArgs a) {
+    extern __shared__ float gsum[];  // [D / gs]
+    const int ng = a.D / a.gs;
+    for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x) {
+        for (int g = threadIdx.x; g < ng; g += blockDim.x) gsum[g] = 0.f;
+        __syncthreads();
+        for (int f = 8 * threadIdx.x; f < a.D; f += 8 * blockDim.x) {
+            float v[8], zv[8];
+            gated8<T>(a, r, f, v, zv);
+            float s = 0.f;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) s = fmaf(v[i], v[i], s);
+            atomicAdd(&gsum[f / a.gs], s);
+        }
+        __syncthreads();
+        for (int g = threadIdx.x; g < ng; g += blockDim.x) gsum[g] = rsqrtf(gsum[g] / a.gs + a.eps);
+        __syncthreads();
+        for (int f = 8 * threadIdx.x; f < a.D; f += 8 * blockDim.x) {
+            float v[8], zv[8];
+            gated8<T>(a, r, f, v, zv);
+            const float inv = gsum[f / a.gs];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) v[i] = v[i] * inv * a.weight[f + i];
+            st8<T>(static_cast<T *>(a.out) + r * a.D + f, v);
+        }
+        __syncthreads();
+    }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) rmsnorm_bwd_kernel(NormArgs a) {
+    extern __shared__ float sm[];
+    const int ng = a.D / a.gs;
+    float *dwp = sm;            // [D] this CTA's dweight partials (feature f owned by one thread)
+    float *inv = sm + a.D;      // [ng] 1 / rms per group
+    float *dot = inv + ng;      // [ng] sum over the group of dn * n
+    for (int f = threadIdx.x; f < a.D; f += blockDim.x) dwp[f] = 0.f;
+    for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x) {
+        for (int g = threadIdx.x; g < ng; g += blockDim.x) inv[g] = dot[g] = 0.f;
+        __syncthreads();
+        for (int f = 8 * threadIdx.x; f < a.D; f += 8 * blockDim.x) {
+            float v[8], zv[8];
+            gated8<T>(a, r, f, v, zv);
+            float s = 0.f;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) s = fmaf(v[i], v[i], s);
+            atomicAdd(&inv[f / a.gs], s);
+        }
+        __syncthreads();
+        for (int g = threadIdx.x; g < ng; g += blockDim.x) inv[g] = rsqrtf(inv[g] / a.gs + a.eps);
+        __syncthreads();
+        for (int f = 8 * threadIdx.x; f < a.D; f += 8 * blockDim.x) {
+            float v[8], zv[8], go[8];
+            gated8<T>(a, r, f, v, zv);
+            ld8<T>(static_cast<const T *>(a.dout) + r * a.D + f, go);
+            const float iv = inv[f / a.gs];
+            float s = 0.f;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const float n = v[i] * iv;
+                dwp[f + i] = fmaf(go[i], n, dwp[f + i]);
+                s = fmaf(go[i] * a.weight[f + i], n, s);
+            }
+            atomicAdd(&dot[f / a.gs], s);
+        }
+        __syncthreads();
+        for (int f = 8 * threadIdx.x; f < a.D; f += 8 * blockDim.x) {
+            float v[8], zv[8], go[8], dyv[8], dzv[8];
+            gated8<T>(a, r, f, v, zv);
+            ld8<T>(static_cast<const T *>(a.dout) + r * a.D + f, go);
+            const float iv = inv[f / a.gs], m = dot[f / a.gs] / a.gs;
+            const float *yrow = nullptr;
+            float yv[8];
+            if (a.z) {
+                ld8<T>(static_cast<const T *>(a.y) + r * a.D + f, yv);
+                yrow = yv;
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const float n = v[i] * iv;
+                const float dv = (go[i] * a.weight[f + i] - n * m) * iv;  // (dn - n mean(dn n)) / rms
+                if (yrow) {
+                    dyv[i] = dv * silu_f(zv[i]);
+                    dzv[i] = dv * yrow[i] * silu_grad_f(zv[i]);
+                } else {
+                    dyv[i] = dv;
+                }
+            }
+            st8<T>(static_cast<T *>(a.dy) + r * a.D + f, dyv);
+            if (a.z) st8<T>(static_cast<T *>(a.dz) + r * a.D + f, dzv);
+        }
+        __syncthreads();
+    }
+    for (int f = threadIdx.x; f < a.D; f += blockDim.x) atomicAdd(a.dweight + f, dwp[f]);
+}
+
+int num_sms() {
+    int dev = 0, sms = 152;
+    if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    return std::max(sms, 1);
+}
+
+template <typename T, int W>
+cudaError_t conv_launch_w(const ConvArgs &a, bool bwd, bool vec, cudaStream_t st) {
+    dim3 block(32, kRows);
+    dim3 grid((a.C + 63) / 64, (a.L + kRows * kRun - 1) / (kRows * kRun), a.B);
+    if (grid.y == 0) return cudaSuccess;
+    if (!bwd) {
+        trace_begin("conv1d_fwd", st);
+        if (vec) conv1d_fwd_kernel<T, W, true><<<grid, block, 0, st>>>(a);
+        else conv1d_fwd_kernel<T, W, false><<<grid, block, 0, st>>>(a);
+    } else {
+        trace_begin("conv1d_bwd", st);
+        if (vec) conv1d_bwd_kernel<T, W, true><<<grid, block, 0, st>>>(a);
+        else conv1d_bwd_kernel<T, W, false><<<grid, block, 0, st>>>(a);
+    }
+    trace_end(st);
+    return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t conv_launch(const ConvArgs &a, bool bwd, bool vec, cudaStream_t st) {
+    switch (a.W) {
+        case 1: return conv_launch_w<T, 1>(a, bwd, vec, st);
+        case 2: return conv_launch_w<T, 2>(a, bwd, vec, st);
+        case 3: return conv_launch_w<T, 3>(a, bwd, vec, st);
+        case 4: return conv_launch_w<T, 4>(a, bwd, vec, st);
+        case 5: return conv_launch_w<T, 5>(a, bwd, vec, st);
+        case 6: return conv_launch_w<T, 6>(a, bwd, vec, st);
+        case 7: return conv_launch_w<T, 7>(a, bwd, vec, st);
+        default: return conv_launch_w<T, 8>(a, bwd, vec, st);
+    }
+}
+
+frac_status glue_fail(frac_status s, const char *msg) {
+    set_last_error(msg);
+    return s;
+}
+
+frac_status glue_cuda(cudaError_t e, const char *where) {
+    if (e == cudaSuccess) return FRAC_OK;
+    char m[160];
+    std::snprintf(m, sizeof(m), "%s: %s", where, cudaGetErrorString(e));
+    return glue_fail(FRAC_ERR_CUDA, m);
+}
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+frac_status conv_check(const frac_conv_dims *d, bool need_seq) {
+    if (!d) return glue_fail(FRAC_ERR_INVALID_ARGUMENT, "dims must not be NULL");
+    if (d->batch < 1 || (need_seq && d->seqlen < 0) || d->channels < 1 || d->width < 1)
+        return glue_fail(FRAC_ERR_INVALID_ARGUMENT, "need batch >= 1, seqlen >= 0, channels >= 1, width >= 1");
+    if (d->width > kMaxW) return glue_fail(FRAC_ERR_UNSUPPORTED, "width above 8 is not supported");
+    if (d->dtype != FRAC_DTYPE_F32 && d->dtype != FRAC_DTYPE_BF16)
+        return glue_fail(FRAC_ERR_INVALID_ARGUMENT, "unknown dtype");
+    if (d->flags & ~int32_t(FRAC_CONV_SILU)) return glue_fail(FRAC_ERR_INVALID_ARGUMENT, "unknown flag");
+    // grid: (channels / 64, seqlen / (kRows kRun), batch) within the launch limits
+    if (d->batch > 65535 || d->seqlen > int64_t(65535) * kRows * kRun || d->channels > (int64_t(1) << 24))
+        return glue_fail(FRAC_ERR_UNSUPPORTED, "dimension too large");
+    return FRAC_OK;
+}
+
+frac_status norm_check(const frac_norm_dims *d) {
+    if (!d) return glue_fail(FRAC_ERR_INVALID_ARGUMENT, "dims must not be NULL");
+    if (d->rows < 0 || d->dim < 8 || d->group_size < 8 || d->dim % d->group_size || d->group_size % 8 ||
+        !(d->eps >= 0.f))
+        return glue_fail(FRAC_ERR_INVALID_ARGUMENT,
+                         "need rows >= 0, group_size a multiple of 8 dividing dim, eps >= 0");
+    if (d->dtype != FRAC_DTYPE_F32 && d->dtype != FRAC_DTYPE_BF16)
+        return glue_fail(FRAC_ERR_INVALID_ARGUMENT, "unknown dtype");
+    // the backward keeps dim + 2 dim / group_size floats in shared memory (<= 160 KB)
+    if (d->dim > 32768) return glue_fail(FRAC_ERR_UNSUPPORTED, "dim above 32768 is not supported");
+    if (d->flags) return glue_fail(FRAC_ERR_INVALID_ARGUMENT, "flags must be 0");
+    return FRAC_OK;
+}
+
+}  // namespace
+}  // namespace frac
+
+#define GLUE_REQ(p, a)                                                                             \
+    do {                                                                                           \
+        if (!(p) || !frac::aligned(p, a)) {                                                        \
+            char m_[96];                                                                           \
+            std::snprintf(m_, sizeof(m_), "%s must be non-NULL and %d-byte aligned", #p, int(a));  \
+            return frac::glue_fail(FRAC_ERR_INVALID_ARGUMENT, m_);                                 \
+        }                                                                                          \
+    } while (0)
+#define GLUE_OPT(p, a)                                                                             \
+    do {                                                                                           \
+        if ((p) && !frac::aligned(p, a))                                                           \
+            return frac::glue_fail(FRAC_ERR_INVALID_ARGUMENT, #p " is misaligned");                \
+    } while (0)
+
+extern "C" {
+
+frac_status frac_conv1d_fwd(const frac_conv_dims *dims, const void *x, const float *w,
+                            const float *bias, const void *state_in, void *u, void *state_out,
+                            void *stream) {
+    frac::set_last_error("");
+    frac_status s = frac::conv_check(dims, true);
+    if (s) return s;
+    const size_t es = dims->dtype == FRAC_DTYPE_BF16 ? 2 : 4;
+    GLUE_REQ(w, 4);
+    GLUE_OPT(bias, 4);
+    GLUE_OPT(state_in, es);
+    GLUE_OPT(state_out, es);
+    if (dims->seqlen > 0) {
+        GLUE_REQ(x, es);
+        GLUE_REQ(u, es);
+    }
+    if (state_out && state_out == state_in)
+        return frac::glue_fail(FRAC_ERR_INVALID_ARGUMENT, "state_out must not alias state_in");
+    frac::ConvArgs a = {};
+    a.B = int(dims->batch); a.L = int(dims->seqlen); a.C = int(dims->channels); a.W = int(dims->width);
+    a.silu = dims->flags & FRAC_CONV_SILU;
+    a.x = x; a.w = w; a.bias = bias; a.state_in = state_in; a.u = u; a.state_out = state_out;
+    cudaStream_t st = (cudaStream_t)stream;
+    if (a.L == 0) {  // nothing to convolve: the carried state passes through unchanged
+        if (!state_out) return FRAC_OK;
+        const size_t n = size_t(a.B) * a.C * (a.W - 1) * es;
+        return frac::glue_cuda(state_in ? cudaMemcpyAsync(state_out, state_in, n, cudaMemcpyDeviceToDevice, st)
+                                        : cudaMemsetAsync(state_out, 0, n, st),
+                               "frac_conv1d_fwd");
+    }
+    const bool vec = a.C % 2 == 0 && frac::aligned(x, 2 * es) && frac::aligned(u, 2 * es);
+    return frac::glue_cuda(dims->dtype == FRAC_DTYPE_BF16 ? frac::conv_launch<__nv_bfloat16>(a, false, vec, st)
+                                                          : frac::conv_launch<float>(a, false, vec, st),
+                           "frac_conv1d_fwd");
+}
+
+frac_status frac_conv1d_bwd(const frac_conv_dims *dims, const void *x, const float *w,
+                            const float *bias, const void *state_in, const void *du, void *dx,
+                            float *dw, float *dbias, void *dstate_in, void *stream) {
+    frac::set_last_error("");
+    frac_status s = frac::conv_check(dims, true);
+    if (s) return s;
+    const size_t es = dims->dtype == FRAC_DTYPE_BF16 ? 2 : 4;
+    GLUE_REQ(w, 4);
+    GLUE_REQ(dw, 4);
+    GLUE_OPT(bias, 4);
+    GLUE_OPT(dbias, 4);
+    GLUE_OPT(state_in, es);
+    GLUE_OPT(dstate_in, es);
+    if (dims->seqlen > 0) {
+        GLUE_REQ(x, es);
+        GLUE_REQ(du, es);
+        GLUE_REQ(dx, es);
+    }
+    frac::ConvArgs a = {};
+    a.B = int(dims->batch); a.L = int(dims->seqlen); a.C = int(dims->channels); a.W = int(dims->width);
+    a.silu = dims->flags & FRAC_CONV_SILU;
+    a.x = x; a.w = w; a.bias = bias; a.state_in = state_in; a.du = du; a.dx = dx; a.dw = dw;
+    a.dbias = dbias; a.dstate = dstate_in;
+    cudaStream_t st = (cudaStream_t)stream;
+    cudaError_t e = cudaMemsetAsync(dw, 0, sizeof(float) * a.C * a.W, st);
+    if (e == cudaSuccess && dbias) e = cudaMemsetAsync(dbias, 0, sizeof(float) * a.C, st);
+    // the carried inputs that no output reads (only when L < W - 1 leaves some untouched) get 0
+    if (e == cudaSuccess && dstate_in && a.W > 1)
+        e = cudaMemsetAsync(dstate_in, 0, size_t(a.B) * a.C * (a.W - 1) * es, st);
+    if (e == cudaSuccess && a.L > 0) {
+        const bool vec = a.C % 2 == 0 && frac::aligned(x, 2 * es) && frac::aligned(du, 2 * es) &&
+                         frac::aligned(dx, 2 * es);
+        e = dims->dtype == FRAC_DTYPE_BF16 ? frac::conv_launch<__nv_bfloat16>(a, true, vec, st)
+                                           : frac::conv_launch<float>(a, true, vec, st);
+    }
+    return frac::glue_cuda(e, "frac_conv1d_bwd");
+}
+
+frac_status frac_conv1d_step(const frac_conv_dims *dims, const void *x_t, const float *w,
+                             const float *bias, void *state, void *u_t, void *stream) {
+    frac::set_last_error("");
+    frac_status s = frac::conv_check(dims, false);
+    if (s) return s;
+    const size_t es = dims->dtype == FRAC_DTYPE_BF16 ? 2 : 4;
+    GLUE_REQ(x_t, es);
+    GLUE_REQ(w, 4);
+    GLUE_OPT(bias, 4);
+    GLUE_REQ(u_t, es);
+    if (dims->width > 1) GLUE_REQ(state, es);
+    frac::ConvArgs a = {};
+    a.B = int(dims->batch); a.L = 1; a.C = int(dims->channels); a.W = int(dims->width);
+    a.silu = dims->flags & FRAC_CONV_SILU;
+    a.w = w; a.bias = bias; a.state_out = state;
+    cudaStream_t st = (cudaStream_t)stream;
+    const int64_t n = int64_t(a.B) * a.C;
+    const unsigned blocks = unsigned((n + 255) / 256);
+    frac::trace_begin("conv1d_step", st);
+    if (dims->dtype == FRAC_DTYPE_BF16)
+        frac::conv1d_step_kernel<__nv_bfloat16><<<blocks, 256, 0, st>>>(
+            a, static_cast<const __nv_bfloat16 *>(x_t), static_cast<__nv_bfloat16 *>(u_t));
+    else
+        frac::conv1d_step_kernel<float><<<blocks, 256, 0, st>>>(a, static_cast<const float *>(x_t),
+                                                                static_cast<float *>(u_t));
+    frac::trace_end(st);
+    return frac::glue_cuda(cudaGetLastError(), "frac_conv1d_step");
+}
+
+frac_status frac_gated_rmsnorm_fwd(const frac_norm_dims *dims, const void *y, const void *z,
+                                   const float *weight, void *out, void *stream) {
+    frac::set_last_error("");
+    frac_status s = frac::norm_check(dims);
+    if (s) return s;
+    GLUE_REQ(weight, 4);
+    if (dims->rows == 0) return FRAC_OK;
+    GLUE_REQ(y, 16);
+    GLUE_OPT(z, 16);
+    GLUE_REQ(out, 16);
+    frac::NormArgs a = {};
+    a.R = dims->rows; a.D = int(dims->dim); a.gs = int(dims->group_size); a.eps = dims->eps;
+    a.y = y; a.z = z; a.weight = weight; a.out = out;
+    cudaStream_t st = (cudaStream_t)stream;
+    const int blocks = int(std::min<int64_t>(a.R, int64_t(frac::num_sms()) * 16));
+    const size_t smem = sizeof(float) * (a.D / a.gs);
+    frac::trace_begin("gated_rmsnorm_fwd", st);
+    if (dims->dtype == FRAC_DTYPE_BF16)
+        frac::rmsnorm_fwd_kernel<__nv_bfloat16><<<blocks, 256, smem, st>>>(a);
+    else
+        frac::rmsnorm_fwd_kernel<float><<<blocks, 256, smem, st>>>(a);
+    frac::trace_end(st);
+    return frac::glue_cuda(cudaGetLastError(), "frac_gated_rmsnorm_fwd");
+}
+
+frac_status frac_gated_rmsnorm_bwd(const frac_norm_dims *dims, const void *y, const void *z,
+                                   const float *weight, const void *dout, void *dy, void *dz,
+                                   float *dweight, void *stream) {
+    frac::set_last_error("");
+    frac_status s = frac::norm_check(dims);
+    if (s) return s;
+    GLUE_REQ(weight, 4);
+    GLUE_REQ(dweight, 4);
+    if (dims->rows > 0) {
+        GLUE_REQ(y, 16);
+        GLUE_REQ(dout, 16);
+        GLUE_REQ(dy, 16);
+        if (z) GLUE_REQ(dz, 16);
+        GLUE_OPT(z, 16);
+    }
+    frac::NormArgs a = {};
+    a.R = dims->rows; a.D = int(dims->dim); a.gs = int(dims->group_size); a.eps = dims->eps;
+    a.y = y; a.z = z; a.dout = dout; a.weight = weight; a.dy = dy; a.dz = dz; a.dweight = dweight;
+    cudaStream_t st = (cudaStream_t)stream;
+    cudaError_t e = cudaMemsetAsync(dweight, 0, sizeof(float) * a.D, st);
+    if (e == cudaSuccess && a.R > 0) {
+        const int blocks = int(std::min<int64_t>(a.R, int64_t(frac::num_sms()) * 4));
+        const size_t smem = sizeof(float) * (a.D + 2 * (a.D / a.gs));
+        auto k16 = frac::rmsnorm_bwd_kernel<__nv_bfloat16>;
+        auto k32 = frac::rmsnorm_bwd_kernel<float>;
+        cudaFuncSetAttribute(k16, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+        cudaFuncSetAttribute(k32, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+        frac::trace_begin("gated_rmsnorm_bwd", st);
+        if (dims->dtype == FRAC_DTYPE_BF16)
+            k16<<<blocks, 256, smem, st>>>(a);
+        else
+            k32<<<blocks, 256, smem, st>>>(a);
+        frac::trace_end(st);
+        e = cudaGetLastError();
+    }
+    return frac::glue_cuda(e, "frac_gated_rmsnorm_bwd");
+}
+
+}  // extern "C"

@@ -232,8 +232,7 @@ __global__ void __launch_bounds__(kThreads) simt_chunk_fwd(
     const int tid = threadIdx.x;
 
     double *E_s = reinterpret_cast<double *>(smem_raw);
-    double *dtq_s = E_s + kQMax;    // [32] per mode: sum over the chunk of the dtau terms
-    float *e_s = reinterpret_cast<float *>(dtq_s + 32);
+    float *e_s = reinterpret_cast<float *>(E_s + kQMax);
     float *itau = e_s + kQMax;
     float *wr_s = itau + 32;            // [Q][K]
     float *kap_s = wr_s + Q * K;        // [Q][K]

@@ -197,6 +197,27 @@ def make_prep_inputs(s: Shape, seed: int = 0, with_grads: bool = False) -> dict:
     return out
 
 
+def make_conv_inputs(batch, seqlen, channels, width, dtype, seed=0, with_state=True):
+    """Inputs of the causal conv1d: x, du ~ N(0,1) [B, L, C] and a carried state ~ N(0,1)
+    [B, C, W-1] in dtype; w ~ N(0, 1/W) [C, W] and bias ~ N(0, 0.01) [C] in float32."""
+    out = dict(
+        x=cast(normal(seed, "u", (batch, seqlen, channels)), dtype),
+        w=(normal(seed, "conv_w", (channels, width)) / np.sqrt(width)).astype(np.float32),
+        bias=(0.1 * normal(seed, "conv_b", (channels,))).astype(np.float32),
+        du=cast(normal(seed, "dout", (batch, seqlen, channels)), dtype))
+    if with_state:
+        out["state"] = cast(normal(seed, "conv_state", (batch, channels, width - 1)), dtype)
+    return out
+
+
+def make_norm_inputs(rows, dim, dtype, seed=0):
+    """Inputs of the gated RMSNorm: y, z, dout ~ N(0,1) [rows, dim] in dtype; weight
+    1 + N(0, 0.01) [dim] in float32."""
+    return dict(y=cast(normal(seed, "x", (rows, dim)), dtype), z=cast(normal(seed, "z", (rows, dim)), dtype),
+                weight=(1.0 + 0.1 * normal(seed, "norm_w", (dim,))).astype(np.float32),
+                dout=cast(normal(seed, "dout", (rows, dim)), dtype))
+
+
 def rel_l2(a, b) -> float:
     """||a - b||_2 / max(||b||_2, 1e-30), in fp64."""
     a = np.asarray(a, dtype=np.float64)
