@@ -91,9 +91,12 @@ struct TcBwdWorkspace {  // S_in and coef first, at the offsets the forward uses
     float *coef;                             // [B,L,H,4,K]: f, s, u, exp(-E/tau)
     float *ek;                               // [B,L,H,tc_ek_width(K)]: E (hi, lo), kappa
     float *dB_acc, *dC_acc;                  // [B,L,G,N] x 2
-    float *dkap_intra;                       // [B,L,H,K]: the intra-chunk part of dkappa (dtau)
+    float *inter_acc;                        // [B,L,H,2,K]: inter-chunk dw_read, dkappa (dtau)
 };
 size_t tc_bwd_workspace_bytes(const ScanDims &d, TcBwdWorkspace *layout, char *base);
+// The intra-chunk pairs of the timescale gradient (both paths; a no-op unless p.dtau): adds
+// tau^-2 sum_{k<t} (E_t - E_k) w_read_t kappa_k exp(-(E_t - E_k)/tau) G_tk H_tk per mode.
+cudaError_t dtau_pairs_launch(const ScanDims &d, int dtype, const ScanPtrs &p, cudaStream_t st);
 cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspace &ws, int *err,
                         bool reuse_states, cudaStream_t st);
 

@@ -792,12 +792,11 @@ __global__ void __launch_bounds__(kThreads) simt_chunk_bwd(
             dwr_o[wi0 + mm] = from_f<T>(dw);
             dww_o[wi0 + mm] = from_f<T>(dk * omr_s[q]);
             if (dtau) {
-                // e_t-weighted decay gradient of this position and mode: every term of the chunked
-                // decomposition spans positions whose e sum in closed form (E_t, E_end - E_t, E_end)
+                // timescale gradient, the terms with S_in or dS_out, each weighted by the e_t it
+                // spans (E_t, E_end - E_t); the pairs inside the chunk come from dtau_pairs
                 const double Et = E_s[t], Eend = E_s[n - 1];
-                const double tq = Et * double(wr_s[q]) * double(dw) +
-                                  (Eend - Et) * double(kap_s[q]) * double(dk) -
-                                  Eend * double(kap_s[q]) * double(dkpi[q]) -
+                const double tq = Et * double(wr_s[q]) * double(fd_s[q] * dyZ[q]) +
+                                  (Eend - Et) * double(kap_s[q]) * double(u_s[q] * xU[q]) -
                                   double(e_s[t]) * double(dk) * double(rho_s[q]) * double(ww_s[q]);
                 atomicAdd(&dtq_s[mm], tq);
             }
@@ -1095,6 +1094,7 @@ cudaError_t bwd_t(const ScanDims &d, const ScanPtrs &p, void *S_in, void *dS_out
         dB_acc, dC_acc, p.dtau);
     trace_end(st);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = dtau_pairs_launch(d, sizeof(T) == 2 ? 1 : 0, p, st)) != cudaSuccess) return e;
     if (sizeof(T) == 2 && ngn > 0) {
         const unsigned blocks = unsigned(std::min<size_t>((ngn + 255) / 256, 4096));
         trace_begin("f32_to_bf16", st);

@@ -49,7 +49,7 @@ struct BwdArgs {
     const float *ek;  // per position: {E hi, E lo, 0, 0, kappa[K]} [B, L, H, tc_ek_width(K)]
     bf16 *dx, *dwr, *dww;
     float *ddt, *dalpha, *dlam, *dD;
-    float *dkap_intra, *dtau;  // both null unless the timescale gradient is wanted
+    float *inter_acc, *dtau;  // both null unless the timescale gradient is wanted
     int *err;
     int hg;      // heads per dC/dB group
     int pf_sms;  // SMs of the device: CTAs of the persistent intra kernel
@@ -678,12 +678,6 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
 #pragma unroll
             for (int m = 0; m < KMAX; ++m)
                 if (m < K) o[m] = dk[m] + part[t * KMAX + m];
-            if (a.dkap_intra) {  // kept apart from the inter-chunk part for the timescale gradient
-                float *oi = a.dkap_intra + blh(d, b, c0 + t, h) * K;
-#pragma unroll
-                for (int m = 0; m < KMAX; ++m)
-                    if (m < K) oi[m] = dk[m] + part[t * KMAX + m];
-            }
             a.rect[blh(d, b, c0 + t, h)] = sr + rpart[t];
         }
         sync_first256();
@@ -968,6 +962,13 @@ __global__ void __launch_bounds__(kStLaunch, 1)
                         atomicAdd(acc_dst + q,
                                   make_float4(acc_h[4 * q], acc_h[4 * q + 1], acc_h[4 * q + 2], acc_h[4 * q + 3]));
                 a.ab_acc[i0 * 2 + grp] = ab_h;
+                if (a.inter_acc) {  // the inter-chunk parts kept apart (timescale gradient)
+                    float4 *o = reinterpret_cast<float4 *>(a.inter_acc + (i0 * 2 + grp) * K);
+#pragma unroll
+                    for (int q = 0; q < KMAX / 4; ++q)
+                        if (4 * q < K)
+                            o[q] = make_float4(acc_h[4 * q], acc_h[4 * q + 1], acc_h[4 * q + 2], acc_h[4 * q + 3]);
+                }
             }
             uint4 e[8];
 #pragma unroll
@@ -1333,21 +1334,23 @@ __global__ void __launch_bounds__(kThreads) tc_bwd_final(BwdArgs a) {
         a.dalpha[i] = -ge * logf(lmv) / (alv * alv);
     }
     if (a.dtau) {
-        // Timescale gradient: per mode, the e_t-weighted decay gradient of this position.  Every
-        // term of the chunked decomposition spans positions whose e sum in closed form (E_t from
-        // the chunk start, E_end - E_t to its end), so with the intra-chunk part of dkappa apart:
-        //   E_t w_read dw_read + (E_end - E_t) kappa dkappa - E_end kappa dkappa_intra
-        //   - e_t dkappa rho w_write,  plus E_end d_m <dS_out, S_in>_m once per chunk.
-        float wrv[KMAX], dki[KMAX];
+        // Timescale gradient, the terms with S_in or dS_out: per mode, each weighted by the e_t
+        // it spans (E_t from the chunk start, E_end - E_t to its end, E_end for the whole chunk):
+        //   E_t w_read dw_read^inter + (E_end - E_t) kappa dkappa^inter - e_t dkappa rho w_write
+        // plus E_end d_m <dS_out, S_in>_m once per chunk; the pairs inside the chunk come from
+        // the dtau_pairs kernel.
+        float wrv[KMAX], dwi[KMAX], dki[KMAX];
 #pragma unroll
-        for (int m = 0; m < KMAX; ++m) wrv[m] = dki[m] = 0.f;
+        for (int m = 0; m < KMAX; ++m) wrv[m] = dwi[m] = dki[m] = 0.f;
         if (t < n) {
             load_weights(a.wr + i * K, K, wrv);
 #pragma unroll
             for (int q = 0; q < KMAX / 4; ++q)
                 if (4 * q < K) {
-                    const float4 u = *reinterpret_cast<const float4 *>(a.dkap_intra + i * K + 4 * q);
-                    dki[4 * q] = u.x; dki[4 * q + 1] = u.y; dki[4 * q + 2] = u.z; dki[4 * q + 3] = u.w;
+                    const float4 u = *reinterpret_cast<const float4 *>(a.inter_acc + (i * 2) * K + 4 * q);
+                    const float4 v = *reinterpret_cast<const float4 *>(a.inter_acc + (i * 2 + 1) * K + 4 * q);
+                    dwi[4 * q] = u.x; dwi[4 * q + 1] = u.y; dwi[4 * q + 2] = u.z; dwi[4 * q + 3] = u.w;
+                    dki[4 * q] = v.x; dki[4 * q + 1] = v.y; dki[4 * q + 2] = v.z; dki[4 * q + 3] = v.w;
                 }
         }
 #pragma unroll
@@ -1357,8 +1360,7 @@ __global__ void __launch_bounds__(kThreads) tc_bwd_final(BwdArgs a) {
                 const float z = e * itau[m];
                 const float rho = expf(-z), kap = -expm1f(-z) * ww[m];
                 // E_end - E_t as the exclusive suffix of e (scanned directly, no difference of sums)
-                v = pe * wrv[m] * dwv[m] + (se - e) * kap * dkv[m] - Eend * kap * dki[m] -
-                    e * dkv[m] * rho * ww[m];
+                v = pe * wrv[m] * dwi[m] + (se - e) * kap * dki[m] - e * dkv[m] * rho * ww[m];
             }
             v = warp_sum(v);
             if (lane == 0) tq_sh[w][m] = v;
@@ -1464,7 +1466,7 @@ size_t tc_bwd_workspace_bytes(const ScanDims &d, TcBwdWorkspace *l, char *base) 
     l->mh_total = (float *)take(size_t(d.B) * d.nc * d.G * TQ * TQ * 4);
     l->dB_acc = (float *)take(size_t(d.B) * d.L * d.G * d.N * 4);
     l->dC_acc = (float *)take(size_t(d.B) * d.L * d.G * d.N * 4);
-    l->dkap_intra = (float *)take(blh_ * d.K * 4);
+    l->inter_acc = (float *)take(blh_ * 2 * d.K * 4);
     return off;
 }
 
@@ -1520,7 +1522,7 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
     a.dx = (bf16 *)p.dx; a.dwr = (bf16 *)p.dwr; a.dww = (bf16 *)p.dww;
     a.ddt = p.ddt; a.dalpha = p.dalpha; a.dlam = p.dlam; a.dD = p.dD;
     a.dtau = p.dtau;
-    a.dkap_intra = p.dtau ? ws.dkap_intra : nullptr;
+    a.inter_acc = p.dtau ? ws.inter_acc : nullptr;
     a.err = err;
     {
         int dev = 0, nsm = 0;
@@ -1553,6 +1555,7 @@ cudaError_t tc_scan_bwd(const ScanDims &d, const ScanPtrs &p, const TcBwdWorkspa
     tc_bwd_final<<<dim3(d.nc, d.H, d.B), kThreads, 0, st>>>(a);
     trace_end(st);
     if ((e = cudaGetLastError())) return e;
+    if ((e = dtau_pairs_launch(d, 1, p, st))) return e;
     if (ngn > 0) {
         const unsigned blocks = unsigned(std::min<size_t>((ngn + 255) / 256, 4096));
         trace_begin("f32_to_bf16", st);
