@@ -1,5 +1,6 @@
 // C ABI of the Frac scan library: argument validation, workspace layout, path selection.
 // Every check happens before anything is enqueued; kernels live in the other files.
+#include <algorithm>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -119,7 +120,9 @@ FwdLayout fwd_layout(const frac_dims *d, const frac::ScanDims &sd, int path) {
     const size_t elems = path == PATH_TC ? frac::tc_state_elems(sd) : frac::simt_state_elems(sd);
     const size_t esz = path == PATH_TC ? 2 : elem(d);
     l.coef = kStatusBytes + round_up(elems * esz);  // tensor-core path: per-position coefficients
-    l.ek = l.coef + (path == PATH_TC ? round_up(frac::tc_coef_elems(sd) * 4) : 0);
+    // CUDA-core path at N = 1: the forward's float scratch takes the coefficient slot
+    l.ek = l.coef + (path == PATH_TC ? round_up(frac::tc_coef_elems(sd) * 4)
+                                     : round_up(frac::simt_n1_scratch_elems(sd) * 4));
     l.total = l.ek + (path == PATH_TC ? round_up(frac::tc_ek_elems(sd) * 4) : 0);
     return l;
 }
@@ -140,6 +143,9 @@ BwdLayout bwd_layout(const frac_dims *d, const frac::ScanDims &sd, int path) {
     const size_t acc = (d->dtype == FRAC_DTYPE_BF16) ? round_up(ngn * sizeof(float)) : 0;
     l.dc = l.db + acc;
     l.total = l.dc + acc;
+    // one buffer serves a forward and the backward that reuses its states
+    // (FRAC_FLAG_BWD_REUSE_FWD_STATES): cover the forward's scratch as well
+    l.total = std::max(l.total, fwd_layout(d, sd, path).total);
     return l;
 }
 
@@ -264,7 +270,7 @@ frac_status frac_scan_fwd(const frac_dims *d, const void *x, const float *dt, co
             e = frac::tc_scan_fwd(sd, p, ws + l.s_in, reinterpret_cast<float *>(ws + l.coef),
                                   reinterpret_cast<float *>(ws + l.ek), reinterpret_cast<int *>(ws), st);
         else
-            e = frac::simt_scan_fwd(sd, d->dtype, p, ws + l.s_in, st);
+            e = frac::simt_scan_fwd(sd, d->dtype, p, ws + l.s_in, reinterpret_cast<float *>(ws + l.coef), st);
     }
     return cuda_status(e, "frac_scan_fwd");
 }

@@ -47,7 +47,9 @@ struct ScanPtrs {
 // CUDA-core (SIMT) chunked path; works for float32 and bf16 I/O.
 int simt_pick_chunk(const ScanDims &d, int requested);     // 0 if the shape is unsupported
 size_t simt_state_elems(const ScanDims &d);                 // per-chunk state workspace elements
-cudaError_t simt_scan_fwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in,
+// float scratch of the N = 1 forward (local end states and chunk decays); 0 for other shapes
+size_t simt_n1_scratch_elems(const ScanDims &d);
+cudaError_t simt_scan_fwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in, float *n1_scratch,
                           cudaStream_t st);
 // reuse_states: S_in already holds the forward's per-chunk states (no recompute)
 cudaError_t simt_scan_bwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in,

@@ -905,70 +905,86 @@ __device__ void n1_chunk_coefs(const ScanDims &d, int b, int h, int c0, int n, f
     __syncthreads();
 }
 
-// Chunk-serial state pass: one thread per p of a 64-wide slice; emits every chunk's entering
-// state S_in [B, H, nc, K, P] (the general layout with N = 1) and the final state.
-template <typename T, typename TS>
-__global__ void __launch_bounds__(64) n1_state_pass(ScanDims d, const T *__restrict__ x,
-                                                    const T *__restrict__ Bm, const T *__restrict__ ww,
-                                                    const float *__restrict__ dt, const float *__restrict__ alpha,
-                                                    const float *__restrict__ lam, const float *__restrict__ tau,
-                                                    const float *__restrict__ init, TS *__restrict__ emit,
-                                                    float *__restrict__ fin) {
+// Chunk-local pass: per chunk, the state the chunk alone leaves at its end (from zero) for each
+// (mode, p), and (threads of the first p block) the chunk's decay prod_t rho_t per mode, the
+// same products the recurrence applies.  One thread per p of a 128-wide slice.
+template <typename T>
+__global__ void __launch_bounds__(128) n1_local(ScanDims d, const T *__restrict__ x, const T *__restrict__ Bm,
+                                               const T *__restrict__ ww, const float *__restrict__ dt,
+                                               const float *__restrict__ alpha, const float *__restrict__ lam,
+                                               const float *__restrict__ tau, float *__restrict__ loc,
+                                               float *__restrict__ dec) {
     __shared__ float e_s[kQMax], itau[kN1Modes];
     __shared__ __align__(16) float rho_s[kQMax * kN1Modes];
     __shared__ __align__(16) float kb_s[kQMax * kN1Modes];
-    __shared__ float x_s[kQMax * 64];  // the chunk's x rows of this slice
     const int K = d.K, P = d.P;
-    const int b = blockIdx.z, h = blockIdx.y, p = blockIdx.x * 64 + threadIdx.x;
-    const bool active = p < P;
+    const int npb = (P + 127) / 128;
+    const int c = blockIdx.x, h = blockIdx.y / npb, b = blockIdx.z, pb = blockIdx.y % npb;
+    const int p = pb * 128 + threadIdx.x;
     const size_t bh = size_t(b) * d.H + h;
+    const int c0 = c * d.Q, n = min(d.Q, d.L - c0);
     if (threadIdx.x < K) itau[threadIdx.x] = 1.f / tau[h * K + threadIdx.x];
     const float log_cap = head_log_cap(tau, h, K);
+    __syncthreads();
+    n1_chunk_coefs<T>(d, b, h, c0, n, log_cap, itau, Bm, nullptr, ww, nullptr, dt, alpha, lam, e_s, rho_s,
+                      kb_s, nullptr);
+    if (pb == 0 && threadIdx.x < K) {
+        float a = 1.f;
+        for (int t = 0; t < n; ++t) a *= rho_s[t * K + threadIdx.x];
+        dec[(bh * d.nc + c) * K + threadIdx.x] = a;
+    }
+    if (p >= P) return;
     float S[kN1Modes];
 #pragma unroll
-    for (int m = 0; m < kN1Modes; ++m) S[m] = (active && m < K && init) ? init[(bh * K + m) * P + p] : 0.f;
-    __syncthreads();
-    for (int c = 0; c < d.nc; ++c) {
-        const int c0 = c * d.Q, n = min(d.Q, d.L - c0);
-        // the chunk's x rows of the slice, every load in flight at once (the barriers in
-        // n1_chunk_coefs publish them); the serial recurrence then reads shared memory
-#pragma unroll 8
-        for (int t = 0; t < n; ++t) x_s[t * 64 + threadIdx.x] = active ? to_f(x[blh(d, b, c0 + t, h) * P + p]) : 0.f;
-        n1_chunk_coefs<T>(d, b, h, c0, n, log_cap, itau, Bm, nullptr, ww, nullptr, dt, alpha, lam, e_s,
-                          rho_s, kb_s, nullptr);
-        if (active) {
+    for (int m = 0; m < kN1Modes; ++m) S[m] = 0.f;
+#pragma unroll 4
+    for (int t = 0; t < n; ++t) {
+        const float xv = to_f(x[blh(d, b, c0 + t, h) * P + p]);
+        if ((K & 3) == 0) {
+            const float4 *r4 = reinterpret_cast<const float4 *>(rho_s + t * K);
+            const float4 *k4 = reinterpret_cast<const float4 *>(kb_s + t * K);
 #pragma unroll
-            for (int m = 0; m < kN1Modes; ++m)
-                if (m < K) emit[((bh * d.nc + c) * K + m) * P + p] = from_f<TS>(S[m]);
-            for (int t = 0; t < n; ++t) {
-                const float xv = x_s[t * 64 + threadIdx.x];
-                if ((K & 3) == 0) {  // rows of 16-byte pieces
-                    const float4 *r4 = reinterpret_cast<const float4 *>(rho_s + t * K);
-                    const float4 *k4 = reinterpret_cast<const float4 *>(kb_s + t * K);
-#pragma unroll
-                    for (int q = 0; q < kN1Modes / 4; ++q) {
-                        if (4 * q < K) {
-                            const float4 r = r4[q], kv = k4[q];
-                            S[4 * q] = fmaf(r.x, S[4 * q], kv.x * xv);
-                            S[4 * q + 1] = fmaf(r.y, S[4 * q + 1], kv.y * xv);
-                            S[4 * q + 2] = fmaf(r.z, S[4 * q + 2], kv.z * xv);
-                            S[4 * q + 3] = fmaf(r.w, S[4 * q + 3], kv.w * xv);
-                        }
-                    }
-                } else {
-#pragma unroll
-                    for (int m = 0; m < kN1Modes; ++m)
-                        if (m < K) S[m] = fmaf(rho_s[t * K + m], S[m], kb_s[t * K + m] * xv);
+            for (int q = 0; q < kN1Modes / 4; ++q) {
+                if (4 * q < K) {
+                    const float4 r = r4[q], kv = k4[q];
+                    S[4 * q] = fmaf(r.x, S[4 * q], kv.x * xv);
+                    S[4 * q + 1] = fmaf(r.y, S[4 * q + 1], kv.y * xv);
+                    S[4 * q + 2] = fmaf(r.z, S[4 * q + 2], kv.z * xv);
+                    S[4 * q + 3] = fmaf(r.w, S[4 * q + 3], kv.w * xv);
                 }
             }
-        }
-        __syncthreads();  // the coefficients are rewritten for the next chunk
-    }
-    if (active && fin) {
+        } else {
 #pragma unroll
-        for (int m = 0; m < kN1Modes; ++m)
-            if (m < K) fin[(bh * K + m) * P + p] = S[m];
+            for (int m = 0; m < kN1Modes; ++m)
+                if (m < K) S[m] = fmaf(rho_s[t * K + m], S[m], kb_s[t * K + m] * xv);
+        }
     }
+#pragma unroll
+    for (int m = 0; m < kN1Modes; ++m)
+        if (m < K) loc[((bh * d.nc + c) * K + m) * P + p] = S[m];
+}
+
+// Serial combine over chunks, one thread per (b, h, mode, p): S_in[c] = S, then
+// S = decay_c S + local_c; the last S is the final state.
+template <typename TS>
+__global__ void __launch_bounds__(256) n1_combine(ScanDims d, const float *__restrict__ loc,
+                                                 const float *__restrict__ dec, const float *__restrict__ init,
+                                                 TS *__restrict__ emit, float *__restrict__ fin) {
+    const size_t total = size_t(d.B) * d.H * d.K * d.P;
+    const size_t idx = size_t(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (idx >= total) return;
+    const int p = int(idx % d.P);
+    const size_t bhm = idx / d.P;  // (b h) K + m
+    const int m = int(bhm % d.K);
+    const size_t bh = bhm / d.K;
+    float S = init ? init[idx] : 0.f;  // [B, H, K, P] (N = 1)
+#pragma unroll 4
+    for (int c = 0; c < d.nc; ++c) {
+        const size_t ic = ((bh * d.nc + c) * d.K + m) * d.P + p;
+        emit[ic] = from_f<TS>(S);
+        S = fmaf(dec[(bh * d.nc + c) * d.K + m], S, loc[ic]);
+    }
+    if (fin) fin[idx] = S;
 }
 
 // Chunk-parallel output: from the chunk's entering state, the recurrence again with
@@ -1036,26 +1052,38 @@ __global__ void __launch_bounds__(128) n1_chunk_fwd(ScanDims d, const T *__restr
 }
 
 template <typename T, typename TS>
-cudaError_t fwd_n1(const ScanDims &d, const ScanPtrs &p, void *S_in, cudaStream_t st) {
-    trace_begin("state_pass_fwd_n1", st);
-    n1_state_pass<T, TS><<<dim3((d.P + 63) / 64, d.H, d.B), 64, 0, st>>>(
-        d, (const T *)p.x, (const T *)p.Bm, (const T *)p.ww, p.dt, p.alpha, p.lam, p.tau, p.h0,
-        (TS *)S_in, p.h_final);
+cudaError_t fwd_n1(const ScanDims &d, const ScanPtrs &p, void *S_in, float *scratch, cudaStream_t st) {
+    const int npb = (d.P + 127) / 128;
+    float *loc = scratch, *dec = scratch + size_t(d.B) * d.H * d.nc * d.K * d.P;
+    cudaError_t e = cudaSuccess;
+    if (d.nc > 0) {
+        trace_begin("local_fwd_n1", st);
+        n1_local<T><<<dim3(d.nc, d.H * npb, d.B), 128, 0, st>>>(d, (const T *)p.x, (const T *)p.Bm,
+                                                                (const T *)p.ww, p.dt, p.alpha, p.lam,
+                                                                p.tau, loc, dec);
+        trace_end(st);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    const size_t total = size_t(d.B) * d.H * d.K * d.P;
+    trace_begin("combine_fwd_n1", st);
+    n1_combine<TS><<<unsigned((total + 255) / 256), 256, 0, st>>>(d, loc, dec, p.h0, (TS *)S_in, p.h_final);
     trace_end(st);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess || d.nc == 0) return e;  // L = 0: h_final = h0 was written
+    if ((e = cudaGetLastError()) != cudaSuccess || d.nc == 0) return e;  // L = 0: h_final = h0
     trace_begin("chunk_fwd_n1", st);
-    n1_chunk_fwd<T, TS><<<dim3(d.nc, d.H * ((d.P + 127) / 128), d.B), 128, 0, st>>>(
+    n1_chunk_fwd<T, TS><<<dim3(d.nc, d.H * npb, d.B), 128, 0, st>>>(
         d, (const T *)p.x, (const T *)p.Bm, (const T *)p.Cm, (const T *)p.wr, (const T *)p.ww, p.dt,
         p.alpha, p.lam, p.tau, p.D, (const TS *)S_in, (T *)p.y);
     trace_end(st);
     return cudaGetLastError();
 }
 
+bool uses_n1(const ScanDims &d) {  // grid y of the chunk kernels: heads x p blocks
+    return d.N == 1 && d.Q <= kQMax && d.K <= kN1Modes && size_t(d.H) * ((d.P + 127) / 128) <= 65535;
+}
+
 template <typename T, typename TS>
-cudaError_t fwd_t(const ScanDims &d, const ScanPtrs &p, void *S_in, cudaStream_t st) {
-    if (d.N == 1 && d.Q <= kQMax && d.K <= kN1Modes && size_t(d.H) * ((d.P + 127) / 128) <= 65535)
-        return fwd_n1<T, TS>(d, p, S_in, st);  // (grid y of the output kernel: heads x p blocks)
+cudaError_t fwd_t(const ScanDims &d, const ScanPtrs &p, void *S_in, float *scratch, cudaStream_t st) {
+    if (uses_n1(d)) return fwd_n1<T, TS>(d, p, S_in, scratch, st);
     cudaError_t e = run_state_pass<T, TS>(d, false, p.x, p.Bm, p.ww, p, p.h0, S_in, p.h_final, st);
     if (e != cudaSuccess || d.nc == 0) return e;  // L = 0: h_final = h0 was written
     const size_t smem = chunk_fwd_smem(d);
@@ -1133,10 +1161,14 @@ size_t simt_state_elems(const ScanDims &d) {
     return size_t(d.B) * d.H * d.nc * d.K * d.P * d.N;
 }
 
-cudaError_t simt_scan_fwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in,
+size_t simt_n1_scratch_elems(const ScanDims &d) {
+    return uses_n1(d) ? size_t(d.B) * d.H * d.nc * d.K * (size_t(d.P) + 1) : 0;
+}
+
+cudaError_t simt_scan_fwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in, float *n1_scratch,
                           cudaStream_t st) {
-    if (dtype == 0) return fwd_t<float, float>(d, p, S_in, st);
-    return fwd_t<__nv_bfloat16, __nv_bfloat16>(d, p, S_in, st);
+    if (dtype == 0) return fwd_t<float, float>(d, p, S_in, n1_scratch, st);
+    return fwd_t<__nv_bfloat16, __nv_bfloat16>(d, p, S_in, n1_scratch, st);
 }
 
 cudaError_t simt_scan_bwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in,

@@ -115,3 +115,23 @@ def test_decode_workload_sampled():
     got = torch.stack(ys)
     assert_close("y", to_host64(got), yr, 1e-2)
     assert_close("state", to_host64(state[bt][:, ht]), st_r, 1e-2)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_decode_paper_layer_shape(dtype):
+    """The paper's layer (H16, head dim 256, N = 1, K = 16 on the 1 .. 2^17 bank): a 300-token
+    prefill through the chunk-parallel N = 1 forward, then 16 decode steps (Algorithm 1's
+    one-step form), against the oracle's prefill and steps on the same bytes."""
+    s = synth.Shape(2, 300, 16, 256, 1, 1, 16, 0, dtype)
+    host = synth.make_scan_inputs(s, seed=12)
+    dv = dev_inputs(host)
+    _, hf = scan_fwd(dv["x"], dv["dt"], dv["alpha"], dv["lam"], dv["tau"], dv["B"], dv["C"],
+                     dv["w_read"], dv["w_write"], dv["D"])
+    dec, y, st = _run_decode(s, 16, 13, to_host64(hf))
+    o = f64_inputs(host)
+    _, h_or = oracle.fwd(o["x"], o["dt"], o["alpha"], o["lam"], o["tau"], o["B"], o["C"],
+                         o["w_read"], o["w_write"], o["D"])
+    assert_close("prefill state", to_host64(hf), h_or, tol(dtype))
+    yr, str_ = _oracle_decode(dec, h_or, 16)
+    assert_close("y", to_host64(y), yr, tol(dtype))
+    assert_close("state", to_host64(st), str_, tol(dtype))

@@ -350,3 +350,31 @@ def test_bwd_timescale_gradient_reusing_forward_states():
     ref = _ora_bwd(d64)
     for k in GRADS + ["dtau"]:
         assert_close(k, to_host64(g[k]), ref[k], 1e-2)
+
+
+def test_paper_layer_shape_all_heads_long():
+    """All 16 heads of the paper's layer at 4096 tokens (64 chunks through the chunk-parallel
+    N = 1 forward's local pass, serial combine and output pass), every output compared."""
+    s = synth.Shape(1, 4096, 16, 256, 1, 1, 16, 0, "bf16")
+    _check_fwd(s, seed=52, h0=True)
+
+
+def test_paper_layer_shape_backward_reusing_forward_states():
+    """One buffer of frac_scan_bwd_workspace_size serves the N = 1 forward (whose scratch holds
+    the chunk-local states) and the backward that reuses its per-chunk states."""
+    from paper_2609_36314_gb300.api import bwd_workspace_size, make_dims
+    s = synth.Shape(1, 700, 4, 256, 1, 1, 16, 0, "bf16")
+    host = synth.make_scan_inputs(s, seed=53, with_dy=True)
+    dv = dev_inputs(host)
+    dims = make_dims(s.batch, s.seqlen, s.nheads, s.headdim, s.ngroups, s.dstate, s.nmodes,
+                     torch.bfloat16)
+    ws = torch.empty(bwd_workspace_size(dims), dtype=torch.uint8, device="cuda")
+    y, _ = _gpu_fwd(dv, workspace=ws, want_final_state=False)
+    g = _gpu_bwd(dv, workspace=ws, reuse_fwd_states=True)
+    torch.cuda.synchronize()
+    d64 = f64_inputs(host)
+    yr, _ = _ora_fwd(d64)
+    assert_close("y", to_host64(y), yr, 1e-2)
+    ref = _ora_bwd(d64)
+    for k in GRADS:
+        assert_close(k, to_host64(g[k]), ref[k], 1e-2)
