@@ -351,7 +351,21 @@ __device__ __forceinline__ void gated8(const NormArgs &a, int64_t r, int f, floa
     }
 }
 
-// Requires gs % 8 == 0 and D % 8 == 0 (host-checked): every 8-vector lies in one group.
+// Adds a thread's partial s (of the 8 features at f) to its group's sum.  When groups are whole
+// multiples of 256 features, the 32 lanes of a warp (256 consecutive features) share a group:
+// one warp sum and one shared atomic per warp instead of 32 atomics on one address.
+__device__ __forceinline__ void group_add(float *sums, int f, int gs, bool valid, float s) {
+    if (gs % 256 == 0) {
+        s = warp_sum(valid ? s : 0.f);
+        if ((threadIdx.x & 31) == 0 && valid) atomicAdd(&sums[f / gs], s);
+    } else if (valid) {
+        atomicAdd(&sums[f / gs], s);
+    }
+}
+
+// Requires gs % 8 == 0 and D % 8 == 0 (host-checked): every 8-vector lies in one group.  The
+// feature loops step by 8 blockDim features with every lane in every step (warp sums need
+// the whole warp), `valid` marking the lanes past the end of the row.
 template <typename T>
 __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(NormArgs a) {
     extern __shared__ float gsum[];  // [D / gs]
@@ -359,13 +373,17 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(NormArgs a) {
     for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x) {
         for (int g = threadIdx.x; g < ng; g += blockDim.x) gsum[g] = 0.f;
         __syncthreads();
-        for (int f = 8 * threadIdx.x; f < a.D; f += 8 * blockDim.x) {
-            float v[8], zv[8];
-            gated8<T>(a, r, f, v, zv);
+        for (int f0 = 0; f0 < a.D; f0 += 8 * blockDim.x) {
+            const int f = f0 + 8 * threadIdx.x;
+            const bool valid = f < a.D;
             float s = 0.f;
+            if (valid) {
+                float v[8], zv[8];
+                gated8<T>(a, r, f, v, zv);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) s = fmaf(v[i], v[i], s);
-            atomicAdd(&gsum[f / a.gs], s);
+                for (int i = 0; i < 8; ++i) s = fmaf(v[i], v[i], s);
+            }
+            group_add(gsum, f, a.gs, valid, s);
         }
         __syncthreads();
         for (int g = threadIdx.x; g < ng; g += blockDim.x) gsum[g] = rsqrtf(gsum[g] / a.gs + a.eps);
@@ -386,37 +404,47 @@ template <typename T>
 __global__ void __launch_bounds__(256) rmsnorm_bwd_kernel(NormArgs a) {
     extern __shared__ float sm[];
     const int ng = a.D / a.gs;
-    float *dwp = sm;            // [D] this CTA's dweight partials (feature f owned by one thread)
+    float *dwp = sm;            // this CTA's dweight partials: feature f + i at i (D / 8) + f / 8,
+                                // owned by one thread, consecutive threads in consecutive words
     float *inv = sm + a.D;      // [ng] 1 / rms per group
     float *dot = inv + ng;      // [ng] sum over the group of dn * n
     for (int f = threadIdx.x; f < a.D; f += blockDim.x) dwp[f] = 0.f;
     for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x) {
         for (int g = threadIdx.x; g < ng; g += blockDim.x) inv[g] = dot[g] = 0.f;
         __syncthreads();
-        for (int f = 8 * threadIdx.x; f < a.D; f += 8 * blockDim.x) {
-            float v[8], zv[8];
-            gated8<T>(a, r, f, v, zv);
+        for (int f0 = 0; f0 < a.D; f0 += 8 * blockDim.x) {
+            const int f = f0 + 8 * threadIdx.x;
+            const bool valid = f < a.D;
             float s = 0.f;
+            if (valid) {
+                float v[8], zv[8];
+                gated8<T>(a, r, f, v, zv);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) s = fmaf(v[i], v[i], s);
-            atomicAdd(&inv[f / a.gs], s);
+                for (int i = 0; i < 8; ++i) s = fmaf(v[i], v[i], s);
+            }
+            group_add(inv, f, a.gs, valid, s);
         }
         __syncthreads();
         for (int g = threadIdx.x; g < ng; g += blockDim.x) inv[g] = rsqrtf(inv[g] / a.gs + a.eps);
         __syncthreads();
-        for (int f = 8 * threadIdx.x; f < a.D; f += 8 * blockDim.x) {
-            float v[8], zv[8], go[8];
-            gated8<T>(a, r, f, v, zv);
-            ld8<T>(static_cast<const T *>(a.dout) + r * a.D + f, go);
-            const float iv = inv[f / a.gs];
+        const int D8 = a.D / 8;
+        for (int f0 = 0; f0 < a.D; f0 += 8 * blockDim.x) {
+            const int f = f0 + 8 * threadIdx.x;
+            const bool valid = f < a.D;
             float s = 0.f;
+            if (valid) {
+                float v[8], zv[8], go[8];
+                gated8<T>(a, r, f, v, zv);
+                ld8<T>(static_cast<const T *>(a.dout) + r * a.D + f, go);
+                const float iv = inv[f / a.gs];
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                const float n = v[i] * iv;
-                dwp[f + i] = fmaf(go[i], n, dwp[f + i]);
-                s = fmaf(go[i] * a.weight[f + i], n, s);
+                for (int i = 0; i < 8; ++i) {
+                    const float n = v[i] * iv;
+                    dwp[i * D8 + f / 8] = fmaf(go[i], n, dwp[i * D8 + f / 8]);
+                    s = fmaf(go[i] * a.weight[f + i], n, s);
+                }
             }
-            atomicAdd(&dot[f / a.gs], s);
+            group_add(dot, f, a.gs, valid, s);
         }
         __syncthreads();
         for (int f = 8 * threadIdx.x; f < a.D; f += 8 * blockDim.x) {
@@ -446,7 +474,8 @@ __global__ void __launch_bounds__(256) rmsnorm_bwd_kernel(NormArgs a) {
         }
         __syncthreads();
     }
-    for (int f = threadIdx.x; f < a.D; f += blockDim.x) atomicAdd(a.dweight + f, dwp[f]);
+    for (int q = threadIdx.x; q < a.D; q += blockDim.x)  // q = i (D / 8) + f / 8
+        atomicAdd(a.dweight + 8 * (q % (a.D / 8)) + q / (a.D / 8), dwp[q]);
 }
 
 int num_sms() {

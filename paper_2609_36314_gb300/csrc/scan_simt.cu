@@ -878,6 +878,7 @@ cudaError_t run_state_pass(const ScanDims &d, bool rev, const void *U, const voi
 // Per chunk, the coefficients of its positions and modes go to shared memory first:
 // rho = exp(-e/tau), kappa B = -expm1(-e/tau) w_write B and (output kernel) w_read C.
 constexpr int kN1Modes = 32;  // nmodes <= 32 (checked at the boundary)
+constexpr int kN1P = 256;     // p per CTA of the N = 1 chunk kernels (one thread each)
 
 template <typename T>
 __device__ void n1_chunk_coefs(const ScanDims &d, int b, int h, int c0, int n, float log_cap,
@@ -905,41 +906,88 @@ __device__ void n1_chunk_coefs(const ScanDims &d, int b, int h, int c0, int n, f
     __syncthreads();
 }
 
+// The chunk's x rows of one 256-wide p block into shared memory (row stride 256 elements):
+// 16-byte asynchronous copies when every row segment is a whole number of aligned 16-byte
+// pieces (VEC), element loads otherwise.  Issued before the coefficients are computed, so the
+// recurrence never waits on HBM; completed by n1_x_wait.
+template <typename T, bool VEC>
+__device__ __forceinline__ void n1_x_issue(const ScanDims &d, const T *__restrict__ x, int b, int h, int c0,
+                                           int n, int p0, int np, T *x_s) {
+    if constexpr (VEC) {
+        constexpr int PER = 16 / sizeof(T);
+        const int pieces = np / PER;
+        for (int idx = threadIdx.x; idx < n * pieces; idx += blockDim.x) {
+            const int t = idx / pieces, q = idx - t * pieces;
+            const uint32_t dst = static_cast<uint32_t>(__cvta_generic_to_shared(x_s + t * kN1P + q * PER));
+            const T *src = x + blh(d, b, c0 + t, h) * d.P + p0 + q * PER;
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    } else {
+        for (int idx = threadIdx.x; idx < n * kN1P; idx += blockDim.x) {
+            const int t = idx / kN1P, q = idx - t * kN1P;
+            if (q < np) x_s[t * kN1P + q] = x[blh(d, b, c0 + t, h) * d.P + p0 + q];
+        }
+    }
+}
+template <bool VEC>
+__device__ __forceinline__ void n1_x_wait() {
+    if constexpr (VEC) asm volatile("cp.async.wait_all;" ::: "memory");
+    __syncthreads();
+}
+
+struct N1Smem {  // dynamic shared memory of the N = 1 chunk kernels
+    size_t e, itau, rho, kb, wc, x, total;
+    __host__ __device__ N1Smem(size_t esz) {
+        e = 0;
+        itau = e + sizeof(float) * kQMax;
+        rho = itau + sizeof(float) * kN1Modes;
+        kb = rho + sizeof(float) * kQMax * kN1Modes;
+        wc = kb + sizeof(float) * kQMax * kN1Modes;
+        x = wc + sizeof(float) * kQMax * kN1Modes;
+        total = x + esz * kQMax * kN1P;
+    }
+};
+
 // Chunk-local pass: per chunk, the state the chunk alone leaves at its end (from zero) for each
 // (mode, p), and (threads of the first p block) the chunk's decay prod_t rho_t per mode, the
-// same products the recurrence applies.  One thread per p of a 128-wide slice.
-template <typename T>
-__global__ void __launch_bounds__(128) n1_local(ScanDims d, const T *__restrict__ x, const T *__restrict__ Bm,
-                                               const T *__restrict__ ww, const float *__restrict__ dt,
-                                               const float *__restrict__ alpha, const float *__restrict__ lam,
-                                               const float *__restrict__ tau, float *__restrict__ loc,
-                                               float *__restrict__ dec) {
-    __shared__ float e_s[kQMax], itau[kN1Modes];
-    __shared__ __align__(16) float rho_s[kQMax * kN1Modes];
-    __shared__ __align__(16) float kb_s[kQMax * kN1Modes];
+// same products the recurrence applies.  One thread per p of a 256-wide block.
+template <typename T, bool VEC>
+__global__ void __launch_bounds__(kN1P) n1_local(ScanDims d, const T *__restrict__ x, const T *__restrict__ Bm,
+                                                const T *__restrict__ ww, const float *__restrict__ dt,
+                                                const float *__restrict__ alpha, const float *__restrict__ lam,
+                                                const float *__restrict__ tau, float *__restrict__ loc,
+                                                float *__restrict__ dec) {
+    extern __shared__ __align__(16) unsigned char n1_smem[];
+    const N1Smem L_(sizeof(T));
+    float *e_s = reinterpret_cast<float *>(n1_smem + L_.e), *itau = reinterpret_cast<float *>(n1_smem + L_.itau);
+    float *rho_s = reinterpret_cast<float *>(n1_smem + L_.rho), *kb_s = reinterpret_cast<float *>(n1_smem + L_.kb);
+    T *x_s = reinterpret_cast<T *>(n1_smem + L_.x);
     const int K = d.K, P = d.P;
-    const int npb = (P + 127) / 128;
+    const int npb = (P + kN1P - 1) / kN1P;
     const int c = blockIdx.x, h = blockIdx.y / npb, b = blockIdx.z, pb = blockIdx.y % npb;
-    const int p = pb * 128 + threadIdx.x;
+    const int p0 = pb * kN1P, np = min(kN1P, P - p0), p = p0 + threadIdx.x;
     const size_t bh = size_t(b) * d.H + h;
     const int c0 = c * d.Q, n = min(d.Q, d.L - c0);
+    n1_x_issue<T, VEC>(d, x, b, h, c0, n, p0, np, x_s);
     if (threadIdx.x < K) itau[threadIdx.x] = 1.f / tau[h * K + threadIdx.x];
     const float log_cap = head_log_cap(tau, h, K);
     __syncthreads();
     n1_chunk_coefs<T>(d, b, h, c0, n, log_cap, itau, Bm, nullptr, ww, nullptr, dt, alpha, lam, e_s, rho_s,
                       kb_s, nullptr);
+    n1_x_wait<VEC>();
     if (pb == 0 && threadIdx.x < K) {
         float a = 1.f;
         for (int t = 0; t < n; ++t) a *= rho_s[t * K + threadIdx.x];
         dec[(bh * d.nc + c) * K + threadIdx.x] = a;
     }
-    if (p >= P) return;
+    if (threadIdx.x >= np) return;
     float S[kN1Modes];
 #pragma unroll
     for (int m = 0; m < kN1Modes; ++m) S[m] = 0.f;
 #pragma unroll 4
     for (int t = 0; t < n; ++t) {
-        const float xv = to_f(x[blh(d, b, c0 + t, h) * P + p]);
+        const float xv = to_f(x_s[t * kN1P + threadIdx.x]);
         if ((K & 3) == 0) {
             const float4 *r4 = reinterpret_cast<const float4 *>(rho_s + t * K);
             const float4 *k4 = reinterpret_cast<const float4 *>(kb_s + t * K);
@@ -965,11 +1013,13 @@ __global__ void __launch_bounds__(128) n1_local(ScanDims d, const T *__restrict_
 }
 
 // Serial combine over chunks, one thread per (b, h, mode, p): S_in[c] = S, then
-// S = decay_c S + local_c; the last S is the final state.
+// S = decay_c S + local_c; the last S is the final state.  The local states and decays of 16
+// chunks are loaded at once (all in flight) before their dependent updates.
 template <typename TS>
 __global__ void __launch_bounds__(256) n1_combine(ScanDims d, const float *__restrict__ loc,
                                                  const float *__restrict__ dec, const float *__restrict__ init,
                                                  TS *__restrict__ emit, float *__restrict__ fin) {
+    constexpr int kBatch = 16;
     const size_t total = size_t(d.B) * d.H * d.K * d.P;
     const size_t idx = size_t(blockIdx.x) * blockDim.x + threadIdx.x;
     if (idx >= total) return;
@@ -978,50 +1028,65 @@ __global__ void __launch_bounds__(256) n1_combine(ScanDims d, const float *__res
     const int m = int(bhm % d.K);
     const size_t bh = bhm / d.K;
     float S = init ? init[idx] : 0.f;  // [B, H, K, P] (N = 1)
-#pragma unroll 4
-    for (int c = 0; c < d.nc; ++c) {
-        const size_t ic = ((bh * d.nc + c) * d.K + m) * d.P + p;
-        emit[ic] = from_f<TS>(S);
-        S = fmaf(dec[(bh * d.nc + c) * d.K + m], S, loc[ic]);
+    for (int c0 = 0; c0 < d.nc; c0 += kBatch) {
+        float lv[kBatch], dv[kBatch];
+#pragma unroll
+        for (int j = 0; j < kBatch; ++j) {
+            const int c = c0 + j;
+            lv[j] = c < d.nc ? loc[((bh * d.nc + c) * d.K + m) * d.P + p] : 0.f;
+            dv[j] = c < d.nc ? dec[(bh * d.nc + c) * d.K + m] : 0.f;
+        }
+#pragma unroll
+        for (int j = 0; j < kBatch; ++j) {
+            const int c = c0 + j;
+            if (c < d.nc) {
+                emit[((bh * d.nc + c) * d.K + m) * d.P + p] = from_f<TS>(S);
+                S = fmaf(dv[j], S, lv[j]);
+            }
+        }
     }
     if (fin) fin[idx] = S;
 }
 
 // Chunk-parallel output: from the chunk's entering state, the recurrence again with
-// y_t = sum_m w_read C S_m + D x_t after each update; one thread per p of a 128-wide slice.
-template <typename T, typename TS>
-__global__ void __launch_bounds__(128) n1_chunk_fwd(ScanDims d, const T *__restrict__ x,
-                                                    const T *__restrict__ Bm, const T *__restrict__ Cm,
-                                                    const T *__restrict__ wr, const T *__restrict__ ww,
-                                                    const float *__restrict__ dt, const float *__restrict__ alpha,
-                                                    const float *__restrict__ lam, const float *__restrict__ tau,
-                                                    const float *__restrict__ Dp, const TS *__restrict__ S_in,
-                                                    T *__restrict__ y) {
-    __shared__ float e_s[kQMax], itau[kN1Modes];
-    __shared__ __align__(16) float rho_s[kQMax * kN1Modes];
-    __shared__ __align__(16) float kb_s[kQMax * kN1Modes];
-    __shared__ __align__(16) float wc_s[kQMax * kN1Modes];
+// y_t = sum_m w_read C S_m + D x_t after each update; one thread per p of a 256-wide block.
+template <typename T, typename TS, bool VEC>
+__global__ void __launch_bounds__(kN1P) n1_chunk_fwd(ScanDims d, const T *__restrict__ x,
+                                                     const T *__restrict__ Bm, const T *__restrict__ Cm,
+                                                     const T *__restrict__ wr, const T *__restrict__ ww,
+                                                     const float *__restrict__ dt, const float *__restrict__ alpha,
+                                                     const float *__restrict__ lam, const float *__restrict__ tau,
+                                                     const float *__restrict__ Dp, const TS *__restrict__ S_in,
+                                                     T *__restrict__ y) {
+    extern __shared__ __align__(16) unsigned char n1_smem[];
+    const N1Smem L_(sizeof(T));
+    float *e_s = reinterpret_cast<float *>(n1_smem + L_.e), *itau = reinterpret_cast<float *>(n1_smem + L_.itau);
+    float *rho_s = reinterpret_cast<float *>(n1_smem + L_.rho), *kb_s = reinterpret_cast<float *>(n1_smem + L_.kb);
+    float *wc_s = reinterpret_cast<float *>(n1_smem + L_.wc);
+    T *x_s = reinterpret_cast<T *>(n1_smem + L_.x);
     const int K = d.K, P = d.P;
-    const int npb = (P + 127) / 128;
+    const int npb = (P + kN1P - 1) / kN1P;
     const int c = blockIdx.x, h = blockIdx.y / npb, b = blockIdx.z;
-    const int p = (blockIdx.y % npb) * 128 + threadIdx.x;
-    const bool active = p < P;
+    const int p0 = (blockIdx.y % npb) * kN1P, np = min(kN1P, P - p0), p = p0 + threadIdx.x;
+    const bool active = threadIdx.x < np;
     const size_t bh = size_t(b) * d.H + h;
     const int c0 = c * d.Q, n = min(d.Q, d.L - c0);
+    n1_x_issue<T, VEC>(d, x, b, h, c0, n, p0, np, x_s);
     if (threadIdx.x < K) itau[threadIdx.x] = 1.f / tau[h * K + threadIdx.x];
     const float log_cap = head_log_cap(tau, h, K);
+    float S[kN1Modes];
+#pragma unroll
+    for (int m = 0; m < kN1Modes; ++m)
+        S[m] = (active && m < K) ? to_f(S_in[((bh * d.nc + c) * K + m) * P + p]) : 0.f;
     __syncthreads();
     n1_chunk_coefs<T>(d, b, h, c0, n, log_cap, itau, Bm, Cm, ww, wr, dt, alpha, lam, e_s, rho_s, kb_s,
                       wc_s);
+    n1_x_wait<VEC>();
     if (!active) return;
-    float S[kN1Modes];
-#pragma unroll
-    for (int m = 0; m < kN1Modes; ++m) S[m] = m < K ? to_f(S_in[((bh * d.nc + c) * K + m) * P + p]) : 0.f;
     const float Dh = Dp[h];
 #pragma unroll 4
     for (int t = 0; t < n; ++t) {
-        const size_t i = blh(d, b, c0 + t, h) * P + p;
-        const float xv = to_f(x[i]);
+        const float xv = to_f(x_s[t * kN1P + threadIdx.x]);
         float yv = Dh * xv;
         if ((K & 3) == 0) {  // rows of 16-byte pieces
             const float4 *r4 = reinterpret_cast<const float4 *>(rho_s + t * K);
@@ -1047,20 +1112,24 @@ __global__ void __launch_bounds__(128) n1_chunk_fwd(ScanDims d, const T *__restr
                 }
             }
         }
-        y[i] = from_f<T>(yv);
+        y[blh(d, b, c0 + t, h) * P + p] = from_f<T>(yv);
     }
 }
 
 template <typename T, typename TS>
 cudaError_t fwd_n1(const ScanDims &d, const ScanPtrs &p, void *S_in, float *scratch, cudaStream_t st) {
-    const int npb = (d.P + 127) / 128;
+    const int npb = (d.P + kN1P - 1) / kN1P;
     float *loc = scratch, *dec = scratch + size_t(d.B) * d.H * d.nc * d.K * d.P;
+    // 16-byte copies of the x rows when x is 16-byte aligned and a head's row is whole pieces
+    const bool vec = (reinterpret_cast<uintptr_t>(p.x) % 16 == 0) && ((size_t(d.P) * sizeof(T)) % 16 == 0);
+    const size_t smem = N1Smem(sizeof(T)).total;
     cudaError_t e = cudaSuccess;
     if (d.nc > 0) {
+        auto kl = vec ? n1_local<T, true> : n1_local<T, false>;
+        cudaFuncSetAttribute(kl, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
         trace_begin("local_fwd_n1", st);
-        n1_local<T><<<dim3(d.nc, d.H * npb, d.B), 128, 0, st>>>(d, (const T *)p.x, (const T *)p.Bm,
-                                                                (const T *)p.ww, p.dt, p.alpha, p.lam,
-                                                                p.tau, loc, dec);
+        kl<<<dim3(d.nc, d.H * npb, d.B), kN1P, smem, st>>>(d, (const T *)p.x, (const T *)p.Bm, (const T *)p.ww,
+                                                           p.dt, p.alpha, p.lam, p.tau, loc, dec);
         trace_end(st);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
@@ -1069,8 +1138,10 @@ cudaError_t fwd_n1(const ScanDims &d, const ScanPtrs &p, void *S_in, float *scra
     n1_combine<TS><<<unsigned((total + 255) / 256), 256, 0, st>>>(d, loc, dec, p.h0, (TS *)S_in, p.h_final);
     trace_end(st);
     if ((e = cudaGetLastError()) != cudaSuccess || d.nc == 0) return e;  // L = 0: h_final = h0
+    auto ko = vec ? n1_chunk_fwd<T, TS, true> : n1_chunk_fwd<T, TS, false>;
+    cudaFuncSetAttribute(ko, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
     trace_begin("chunk_fwd_n1", st);
-    n1_chunk_fwd<T, TS><<<dim3(d.nc, d.H * npb, d.B), 128, 0, st>>>(
+    ko<<<dim3(d.nc, d.H * npb, d.B), kN1P, smem, st>>>(
         d, (const T *)p.x, (const T *)p.Bm, (const T *)p.Cm, (const T *)p.wr, (const T *)p.ww, p.dt,
         p.alpha, p.lam, p.tau, p.D, (const TS *)S_in, (T *)p.y);
     trace_end(st);
@@ -1078,7 +1149,7 @@ cudaError_t fwd_n1(const ScanDims &d, const ScanPtrs &p, void *S_in, float *scra
 }
 
 bool uses_n1(const ScanDims &d) {  // grid y of the chunk kernels: heads x p blocks
-    return d.N == 1 && d.Q <= kQMax && d.K <= kN1Modes && size_t(d.H) * ((d.P + 127) / 128) <= 65535;
+    return d.N == 1 && d.Q <= kQMax && d.K <= kN1Modes && size_t(d.H) * ((d.P + kN1P - 1) / kN1P) <= 65535;
 }
 
 template <typename T, typename TS>
