@@ -19,6 +19,7 @@
 // Threads own register tiles of the small per-chunk contractions; shared-memory rows are
 // padded by one float so that both row and column walks are free of bank conflicts.
 #include <algorithm>
+#include <type_traits>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -952,7 +953,7 @@ struct N1Smem {  // dynamic shared memory of the N = 1 chunk kernels
 // Chunk-local pass: per chunk, the state the chunk alone leaves at its end (from zero) for each
 // (mode, p), and (threads of the first p block) the chunk's decay prod_t rho_t per mode, the
 // same products the recurrence applies.  One thread per p of a 256-wide block.
-template <typename T, bool VEC>
+template <typename T, bool VEC, int KP>
 __global__ void __launch_bounds__(kN1P) n1_local(ScanDims d, const T *__restrict__ x, const T *__restrict__ Bm,
                                                 const T *__restrict__ ww, const float *__restrict__ dt,
                                                 const float *__restrict__ alpha, const float *__restrict__ lam,
@@ -982,9 +983,9 @@ __global__ void __launch_bounds__(kN1P) n1_local(ScanDims d, const T *__restrict
         dec[(bh * d.nc + c) * K + threadIdx.x] = a;
     }
     if (threadIdx.x >= np) return;
-    float S[kN1Modes];
+    float S[KP];
 #pragma unroll
-    for (int m = 0; m < kN1Modes; ++m) S[m] = 0.f;
+    for (int m = 0; m < KP; ++m) S[m] = 0.f;
 #pragma unroll 4
     for (int t = 0; t < n; ++t) {
         const float xv = to_f(x_s[t * kN1P + threadIdx.x]);
@@ -992,7 +993,7 @@ __global__ void __launch_bounds__(kN1P) n1_local(ScanDims d, const T *__restrict
             const float4 *r4 = reinterpret_cast<const float4 *>(rho_s + t * K);
             const float4 *k4 = reinterpret_cast<const float4 *>(kb_s + t * K);
 #pragma unroll
-            for (int q = 0; q < kN1Modes / 4; ++q) {
+            for (int q = 0; q < KP / 4; ++q) {
                 if (4 * q < K) {
                     const float4 r = r4[q], kv = k4[q];
                     S[4 * q] = fmaf(r.x, S[4 * q], kv.x * xv);
@@ -1003,12 +1004,12 @@ __global__ void __launch_bounds__(kN1P) n1_local(ScanDims d, const T *__restrict
             }
         } else {
 #pragma unroll
-            for (int m = 0; m < kN1Modes; ++m)
+            for (int m = 0; m < KP; ++m)
                 if (m < K) S[m] = fmaf(rho_s[t * K + m], S[m], kb_s[t * K + m] * xv);
         }
     }
 #pragma unroll
-    for (int m = 0; m < kN1Modes; ++m)
+    for (int m = 0; m < KP; ++m)
         if (m < K) loc[((bh * d.nc + c) * K + m) * P + p] = S[m];
 }
 
@@ -1050,7 +1051,7 @@ __global__ void __launch_bounds__(256) n1_combine(ScanDims d, const float *__res
 
 // Chunk-parallel output: from the chunk's entering state, the recurrence again with
 // y_t = sum_m w_read C S_m + D x_t after each update; one thread per p of a 256-wide block.
-template <typename T, typename TS, bool VEC>
+template <typename T, typename TS, bool VEC, int KP>
 __global__ void __launch_bounds__(kN1P) n1_chunk_fwd(ScanDims d, const T *__restrict__ x,
                                                      const T *__restrict__ Bm, const T *__restrict__ Cm,
                                                      const T *__restrict__ wr, const T *__restrict__ ww,
@@ -1074,9 +1075,9 @@ __global__ void __launch_bounds__(kN1P) n1_chunk_fwd(ScanDims d, const T *__rest
     n1_x_issue<T, VEC>(d, x, b, h, c0, n, p0, np, x_s);
     if (threadIdx.x < K) itau[threadIdx.x] = 1.f / tau[h * K + threadIdx.x];
     const float log_cap = head_log_cap(tau, h, K);
-    float S[kN1Modes];
+    float S[KP];
 #pragma unroll
-    for (int m = 0; m < kN1Modes; ++m)
+    for (int m = 0; m < KP; ++m)
         S[m] = (active && m < K) ? to_f(S_in[((bh * d.nc + c) * K + m) * P + p]) : 0.f;
     __syncthreads();
     n1_chunk_coefs<T>(d, b, h, c0, n, log_cap, itau, Bm, Cm, ww, wr, dt, alpha, lam, e_s, rho_s, kb_s,
@@ -1087,32 +1088,35 @@ __global__ void __launch_bounds__(kN1P) n1_chunk_fwd(ScanDims d, const T *__rest
 #pragma unroll 4
     for (int t = 0; t < n; ++t) {
         const float xv = to_f(x_s[t * kN1P + threadIdx.x]);
-        float yv = Dh * xv;
+        float ya[4] = {Dh * xv, 0.f, 0.f, 0.f};  // four independent partial readout sums
         if ((K & 3) == 0) {  // rows of 16-byte pieces
             const float4 *r4 = reinterpret_cast<const float4 *>(rho_s + t * K);
             const float4 *k4 = reinterpret_cast<const float4 *>(kb_s + t * K);
             const float4 *w4 = reinterpret_cast<const float4 *>(wc_s + t * K);
 #pragma unroll
-            for (int q = 0; q < kN1Modes / 4; ++q) {
+            for (int q = 0; q < KP / 4; ++q) {
                 if (4 * q < K) {
                     const float4 r = r4[q], kv = k4[q], wv = w4[q];
                     S[4 * q] = fmaf(r.x, S[4 * q], kv.x * xv);
                     S[4 * q + 1] = fmaf(r.y, S[4 * q + 1], kv.y * xv);
                     S[4 * q + 2] = fmaf(r.z, S[4 * q + 2], kv.z * xv);
                     S[4 * q + 3] = fmaf(r.w, S[4 * q + 3], kv.w * xv);
-                    yv = fmaf(wv.x, S[4 * q], fmaf(wv.y, S[4 * q + 1], fmaf(wv.z, S[4 * q + 2], fmaf(wv.w, S[4 * q + 3], yv))));
+                    ya[0] = fmaf(wv.x, S[4 * q], ya[0]);
+                    ya[1] = fmaf(wv.y, S[4 * q + 1], ya[1]);
+                    ya[2] = fmaf(wv.z, S[4 * q + 2], ya[2]);
+                    ya[3] = fmaf(wv.w, S[4 * q + 3], ya[3]);
                 }
             }
         } else {
 #pragma unroll
-            for (int m = 0; m < kN1Modes; ++m) {
+            for (int m = 0; m < KP; ++m) {
                 if (m < K) {
                     S[m] = fmaf(rho_s[t * K + m], S[m], kb_s[t * K + m] * xv);
-                    yv = fmaf(wc_s[t * K + m], S[m], yv);
+                    ya[m & 3] = fmaf(wc_s[t * K + m], S[m], ya[m & 3]);
                 }
             }
         }
-        y[blh(d, b, c0 + t, h) * P + p] = from_f<T>(yv);
+        y[blh(d, b, c0 + t, h) * P + p] = from_f<T>((ya[0] + ya[1]) + (ya[2] + ya[3]));
     }
 }
 
@@ -1124,8 +1128,22 @@ cudaError_t fwd_n1(const ScanDims &d, const ScanPtrs &p, void *S_in, float *scra
     const bool vec = (reinterpret_cast<uintptr_t>(p.x) % 16 == 0) && ((size_t(d.P) * sizeof(T)) % 16 == 0);
     const size_t smem = N1Smem(sizeof(T)).total;
     cudaError_t e = cudaSuccess;
+    const int KP = d.K <= 4 ? 4 : d.K <= 8 ? 8 : d.K <= 16 ? 16 : 32;
+    auto pick_local = [&](auto kp) {
+        constexpr int V = decltype(kp)::value;
+        return vec ? n1_local<T, true, V> : n1_local<T, false, V>;
+    };
+    auto pick_out = [&](auto kp) {
+        constexpr int V = decltype(kp)::value;
+        return vec ? n1_chunk_fwd<T, TS, true, V> : n1_chunk_fwd<T, TS, false, V>;
+    };
+    using I4 = std::integral_constant<int, 4>;
+    using I8 = std::integral_constant<int, 8>;
+    using I16 = std::integral_constant<int, 16>;
+    using I32 = std::integral_constant<int, 32>;
+    auto kl = KP == 4 ? pick_local(I4{}) : KP == 8 ? pick_local(I8{}) : KP == 16 ? pick_local(I16{}) : pick_local(I32{});
+    auto ko = KP == 4 ? pick_out(I4{}) : KP == 8 ? pick_out(I8{}) : KP == 16 ? pick_out(I16{}) : pick_out(I32{});
     if (d.nc > 0) {
-        auto kl = vec ? n1_local<T, true> : n1_local<T, false>;
         cudaFuncSetAttribute(kl, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
         trace_begin("local_fwd_n1", st);
         kl<<<dim3(d.nc, d.H * npb, d.B), kN1P, smem, st>>>(d, (const T *)p.x, (const T *)p.Bm, (const T *)p.ww,
@@ -1138,7 +1156,6 @@ cudaError_t fwd_n1(const ScanDims &d, const ScanPtrs &p, void *S_in, float *scra
     n1_combine<TS><<<unsigned((total + 255) / 256), 256, 0, st>>>(d, loc, dec, p.h0, (TS *)S_in, p.h_final);
     trace_end(st);
     if ((e = cudaGetLastError()) != cudaSuccess || d.nc == 0) return e;  // L = 0: h_final = h0
-    auto ko = vec ? n1_chunk_fwd<T, TS, true> : n1_chunk_fwd<T, TS, false>;
     cudaFuncSetAttribute(ko, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
     trace_begin("chunk_fwd_n1", st);
     ko<<<dim3(d.nc, d.H * npb, d.B), kN1P, smem, st>>>(
