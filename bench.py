@@ -690,6 +690,29 @@ def bench_paper_shape(ctx):
                     "kernels": kernel_table(trace, 10),
                     "roofline": roofline_of("whole forward", "bytes", work, ms, ctx.peaks)})
         del a, y
+    # training-shaped step at the paper's layer: forward + backward over 4 packed 4K sequences
+    from paper_2609_36314_gb300 import scan_bwd
+    from paper_2609_36314_gb300.api import bwd_workspace_size, make_dims
+    s = synth.Shape(4, 4096, 16, 256, 1, 1, 16, 0, "bf16")
+    a = synth.make_scan_inputs_torch(s, seed=15, device=ctx.dev, with_dy=True)
+    dims = make_dims(s.batch, s.seqlen, s.nheads, s.headdim, s.ngroups, s.dstate, s.nmodes,
+                     torch.bfloat16)
+    ws = torch.empty(bwd_workspace_size(dims), dtype=torch.uint8, device=ctx.dev)
+    y = torch.empty_like(a["x"])
+
+    def train():
+        scan_fwd(a["x"], a["dt"], a["alpha"], a["lam"], a["tau"], a["B"], a["C"], a["w_read"],
+                 a["w_write"], a["D"], y=y, want_final_state=False, workspace=ws)
+        scan_bwd(a["x"], a["dt"], a["alpha"], a["lam"], a["tau"], a["B"], a["C"], a["w_read"],
+                 a["w_write"], a["D"], a["dy"], workspace=ws, reuse_fwd_states=True)
+
+    ms, trace = ctx.time(train, 5)
+    tr = {"workload": "B4 L4096 H16 P256 N1 K16 bf16, forward + backward (the backward reuses "
+                      "the forward's per-chunk states)",
+          "ms_per_step": ms, "tokens_per_s": s.batch * s.seqlen / (ms / 1e3),
+          "kernels": kernel_table(trace, 5)}
+    del a, ws, y
+    torch.cuda.empty_cache()
     s = synth.Shape(1, 64, 16, 256, 1, 1, 16, 0, "bf16")
     stp = synth.make_scan_inputs_torch(s, seed=14, device=ctx.dev)
     stp = {k: (v.transpose(0, 1).contiguous() if k not in ("tau", "D") else v) for k, v in stp.items()}
@@ -714,7 +737,7 @@ def bench_paper_shape(ctx):
                    "bound, not bandwidth bound"}
     return {"workload": "paper layer shape: B1 H16 P256 N1 K16, tau geometric in [1, 2^17], bf16 "
                         "inputs; prefill = forward with L2 flushed before each call",
-            "unit": "tokens/s", "prefill": pts, "decode": dec}
+            "unit": "tokens/s", "prefill": pts, "decode": dec, "train": tr}
 
 
 def bench_mixer(ctx):
