@@ -111,7 +111,7 @@ struct FwdLayout {
     size_t s_in, coef, ek, total;
 };
 struct BwdLayout {
-    size_t s_in, ds_out, db, dc, total;
+    size_t s_in, ds_out, db, dc, n1, total;
 };
 
 FwdLayout fwd_layout(const frac_dims *d, const frac::ScanDims &sd, int path) {
@@ -131,7 +131,7 @@ BwdLayout bwd_layout(const frac_dims *d, const frac::ScanDims &sd, int path) {
     BwdLayout l;
     if (path == PATH_TC) {
         frac::TcBwdWorkspace t;
-        l.s_in = l.ds_out = l.db = l.dc = 0;
+        l.s_in = l.ds_out = l.db = l.dc = l.n1 = 0;
         l.total = kStatusBytes + frac::tc_bwd_workspace_bytes(sd, &t, nullptr);
         return l;
     }
@@ -142,7 +142,8 @@ BwdLayout bwd_layout(const frac_dims *d, const frac::ScanDims &sd, int path) {
     l.db = l.ds_out + st;
     const size_t acc = (d->dtype == FRAC_DTYPE_BF16) ? round_up(ngn * sizeof(float)) : 0;
     l.dc = l.db + acc;
-    l.total = l.dc + acc;
+    l.n1 = l.dc + acc;  // the N = 1 backward's chunk carries (0 bytes for other shapes)
+    l.total = l.n1 + round_up(frac::simt_n1_scratch_elems(sd) * 4);
     // one buffer serves a forward and the backward that reuses its states
     // (FRAC_FLAG_BWD_REUSE_FWD_STATES): cover the forward's scratch as well
     l.total = std::max(l.total, fwd_layout(d, sd, path).total);
@@ -355,7 +356,7 @@ frac_status frac_scan_bwd(const frac_dims *d, const void *x, const float *dt, co
             e = frac::tc_scan_bwd(sd, p, t, reinterpret_cast<int *>(ws), reuse, st);
         } else {
             e = frac::simt_scan_bwd(sd, d->dtype, p, ws + l.s_in, ws + l.ds_out, dB_acc, dC_acc,
-                                    reuse, st);
+                                    reinterpret_cast<float *>(ws + l.n1), reuse, st);
         }
     }
     return cuda_status(e, "frac_scan_bwd");

@@ -1185,9 +1185,548 @@ cudaError_t fwd_t(const ScanDims &d, const ScanPtrs &p, void *S_in, float *scrat
     return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------------------------------------
+// N = 1 backward (the paper's layer shape).  The adjoint of the scalar recurrence per (mode, p),
+// g_t = w_read_t C_t dy_t + rho_{t+1} g_{t+1}, is carried across chunks the way the forward
+// carries the state: a reverse chunk-local pass gives each chunk's carry
+// loc_c = rho_{c0} g^loc_{c0} (its own positions only) and its decay prod rho, a reverse serial
+// combine turns them into the adjoint entering each chunk from the right (gamma_c, emitted in
+// the dS_out layout) and dh0, and a chunk-parallel gradient kernel forms every gradient of the
+// chunk from S_in and gamma in the pairwise chunked form (H = dY X^T over p, the per-mode pair
+// sums with their own decays, and the S_in / gamma dot products over p).
+
+// Reverse chunk-local pass: one thread per p of a 256-wide block (dy rows staged like x in the
+// forward), the modes in registers; g walks the chunk from its last position to its first.
+template <typename T, bool VEC, int KP>
+__global__ void __launch_bounds__(kN1P) n1_rev_local(ScanDims d, const T *__restrict__ dy, const T *__restrict__ Cm,
+                                                    const T *__restrict__ wr, const float *__restrict__ dt,
+                                                    const float *__restrict__ alpha, const float *__restrict__ lam,
+                                                    const float *__restrict__ tau, float *__restrict__ loc,
+                                                    float *__restrict__ dec) {
+    extern __shared__ __align__(16) unsigned char n1_smem[];
+    const N1Smem L_(sizeof(T));
+    float *e_s = reinterpret_cast<float *>(n1_smem + L_.e), *itau = reinterpret_cast<float *>(n1_smem + L_.itau);
+    float *rho_s = reinterpret_cast<float *>(n1_smem + L_.rho), *wc_s = reinterpret_cast<float *>(n1_smem + L_.wc);
+    float *kb_s = reinterpret_cast<float *>(n1_smem + L_.kb);
+    T *y_s = reinterpret_cast<T *>(n1_smem + L_.x);
+    const int K = d.K, P = d.P;
+    const int npb = (P + kN1P - 1) / kN1P;
+    const int c = blockIdx.x, h = blockIdx.y / npb, b = blockIdx.z, pb = blockIdx.y % npb;
+    const int p0 = pb * kN1P, np = min(kN1P, P - p0), p = p0 + threadIdx.x;
+    const size_t bh = size_t(b) * d.H + h;
+    const int c0 = c * d.Q, n = min(d.Q, d.L - c0);
+    n1_x_issue<T, VEC>(d, dy, b, h, c0, n, p0, np, y_s);
+    if (threadIdx.x < K) itau[threadIdx.x] = 1.f / tau[h * K + threadIdx.x];
+    const float log_cap = head_log_cap(tau, h, K);
+    __syncthreads();
+    // rho and (in the kb slot, unused here) kappa B; w_read C in the wc slot
+    n1_chunk_coefs<T>(d, b, h, c0, n, log_cap, itau, Cm, Cm, wr, wr, dt, alpha, lam, e_s, rho_s, kb_s, wc_s);
+    n1_x_wait<VEC>();
+    if (pb == 0 && threadIdx.x < K) {
+        float a = 1.f;
+        for (int t = 0; t < n; ++t) a *= rho_s[t * K + threadIdx.x];
+        dec[(bh * d.nc + c) * K + threadIdx.x] = a;
+    }
+    if (threadIdx.x >= np) return;
+    float g[KP];
+#pragma unroll
+    for (int m = 0; m < KP; ++m) g[m] = 0.f;
+    for (int t = n - 1; t >= 0; --t) {
+        const float dv = to_f(y_s[t * kN1P + threadIdx.x]);
+#pragma unroll
+        for (int m = 0; m < KP; ++m) {
+            if (m < K) {
+                const float rn = t + 1 < n ? rho_s[(t + 1) * K + m] : 0.f;
+                g[m] = fmaf(rn, g[m], wc_s[t * K + m] * dv);
+            }
+        }
+    }
+#pragma unroll
+    for (int m = 0; m < KP; ++m)
+        if (m < K) loc[((bh * d.nc + c) * K + m) * P + p] = n > 0 ? rho_s[m] * g[m] : 0.f;
+}
+
+// Reverse serial combine: gamma of the last chunk is dh_final; going left, emit gamma_c (the
+// adjoint entering chunk c from the right, in the dS_out layout), then
+// gamma_{c-1} = decay_c gamma_c + loc_c; what leaves chunk 0 is dh0.
+template <typename TS>
+__global__ void __launch_bounds__(256) n1_combine_rev(ScanDims d, const float *__restrict__ loc,
+                                                     const float *__restrict__ dec, const float *__restrict__ init,
+                                                     TS *__restrict__ emit, float *__restrict__ fin) {
+    constexpr int kBatch = 16;
+    const size_t total = size_t(d.B) * d.H * d.K * d.P;
+    const size_t idx = size_t(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (idx >= total) return;
+    const int p = int(idx % d.P);
+    const size_t bhm = idx / d.P;
+    const int m = int(bhm % d.K);
+    const size_t bh = bhm / d.K;
+    float S = init ? init[idx] : 0.f;
+    for (int c1 = d.nc - 1; c1 >= 0; c1 -= kBatch) {
+        float lv[kBatch], dv[kBatch];
+#pragma unroll
+        for (int j = 0; j < kBatch; ++j) {
+            const int c = c1 - j;
+            lv[j] = c >= 0 ? loc[((bh * d.nc + c) * d.K + m) * d.P + p] : 0.f;
+            dv[j] = c >= 0 ? dec[(bh * d.nc + c) * d.K + m] : 0.f;
+        }
+#pragma unroll
+        for (int j = 0; j < kBatch; ++j) {
+            const int c = c1 - j;
+            if (c >= 0) {
+                emit[((bh * d.nc + c) * d.K + m) * d.P + p] = from_f<TS>(S);
+                S = fmaf(dv[j], S, lv[j]);
+            }
+        }
+    }
+    if (fin) fin[idx] = S;
+}
+
+constexpr int kN1BQ = 32;  // chunk of the N = 1 backward (shared-memory tiles [Q][P])
+
+struct N1BwdSmem {
+    size_t E, e, cl, itau, red, cdot, dtq, qk, x, y, sin, gam, H, Gm, XR, total;
+    int P;
+    __host__ __device__ N1BwdSmem(int P_, int K, size_t esz) : P(P_) {
+        E = 0;                                                   // double [Q]
+        e = E + sizeof(double) * kN1BQ;                          // float [Q]
+        cl = e + sizeof(float) * kN1BQ;                          // float [Q]
+        itau = cl + sizeof(float) * kN1BQ;                       // float [32]
+        red = itau + sizeof(float) * 32;                         // float [64]
+        cdot = red + sizeof(float) * 64;                         // float [32]
+        dtq = cdot + sizeof(float) * 32;                         // float [32]: dtau sums per mode
+        qk = dtq + sizeof(float) * 32;                           // float [14][Q][K]
+        x = qk + sizeof(float) * 14 * kN1BQ * K;                 // T [Q][P]
+        x = (x + 15) / 16 * 16;
+        y = x + esz * kN1BQ * P;                                 // T [Q][P]
+        y = (y + 15) / 16 * 16;
+        sin = y + esz * kN1BQ * P;                               // float [K][P]
+        gam = sin + sizeof(float) * K * P;                       // float [K][P]
+        H = gam + sizeof(float) * K * P;                         // float [Q][Q + 1]
+        Gm = H + sizeof(float) * kN1BQ * (kN1BQ + 1);            // float [Q][Q + 1]
+        XR = Gm + sizeof(float) * kN1BQ * (kN1BQ + 1);           // float [Q][Q + 1]
+        total = XR + sizeof(float) * kN1BQ * (kN1BQ + 1);
+    }
+};
+
+// Gradients of one chunk of one head (one CTA, 256 threads; Q <= 32, all of P).
+template <typename T, typename TS, bool VEC, int KP>
+__global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
+    ScanDims d, const T *__restrict__ x, const T *__restrict__ Bm, const T *__restrict__ Cm,
+    const T *__restrict__ wr, const T *__restrict__ ww, const T *__restrict__ dy,
+    const float *__restrict__ dt, const float *__restrict__ alpha, const float *__restrict__ lam,
+    const float *__restrict__ tau, const float *__restrict__ Dv, const TS *__restrict__ S_in,
+    const TS *__restrict__ dS_out, T *__restrict__ dx, T *__restrict__ dwr_o, T *__restrict__ dww_o,
+    float *__restrict__ ddt, float *__restrict__ dalpha, float *__restrict__ dlam, float *__restrict__ dD,
+    float *__restrict__ dB_acc, float *__restrict__ dC_acc, float *__restrict__ dtau) {
+    extern __shared__ __align__(16) unsigned char sm_raw[];
+    const int K = d.K, P = d.P, Q = d.Q;
+    const N1BwdSmem L_(P, K, sizeof(T));
+    double *E_s = reinterpret_cast<double *>(sm_raw + L_.E);
+    float *e_s = reinterpret_cast<float *>(sm_raw + L_.e), *cl_s = reinterpret_cast<float *>(sm_raw + L_.cl);
+    float *itau = reinterpret_cast<float *>(sm_raw + L_.itau), *red = reinterpret_cast<float *>(sm_raw + L_.red);
+    float *cdot = reinterpret_cast<float *>(sm_raw + L_.cdot);
+    float *dtq = reinterpret_cast<float *>(sm_raw + L_.dtq);
+    float *qk = reinterpret_cast<float *>(sm_raw + L_.qk);
+    const int QK = kN1BQ * K;
+    // [Q][K] arrays: coefficients, then the dot products and pair sums
+    float *rho_s = qk, *kap_s = qk + QK, *kb_s = qk + 2 * QK, *wc_s = qk + 3 * QK, *A_s = qk + 4 * QK,
+          *u_s = qk + 5 * QK, *ww_s = qk + 6 * QK, *wr_s = qk + 7 * QK, *XG = qk + 8 * QK, *YS = qk + 9 * QK,
+          *dwci = qk + 10 * QK, *dkbi = qk + 11 * QK, *Bq = qk + 12 * QK, *Cq = qk + 13 * QK;
+    T *xs = reinterpret_cast<T *>(sm_raw + L_.x), *dys = reinterpret_cast<T *>(sm_raw + L_.y);
+    float *Sin = reinterpret_cast<float *>(sm_raw + L_.sin), *Gam = reinterpret_cast<float *>(sm_raw + L_.gam);
+    float *H = reinterpret_cast<float *>(sm_raw + L_.H), *Gm = reinterpret_cast<float *>(sm_raw + L_.Gm);
+    float *XR = reinterpret_cast<float *>(sm_raw + L_.XR);
+    constexpr int Q1 = kN1BQ + 1;
+    const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
+    const int g = h / (d.H / d.G);
+    const int c0 = c * Q, n = min(Q, d.L - c0);
+    const size_t bh = size_t(b) * d.H + h;
+
+    // ---- P0: tiles, states, rates and per-(position, mode) coefficients
+    if constexpr (VEC) {
+        constexpr int PER = 16 / sizeof(T);
+        const int pieces = P / PER;
+        for (int idx = tid; idx < n * pieces; idx += blockDim.x) {
+            const int t = idx / pieces, q = idx - t * pieces;
+            const size_t src = blh(d, b, c0 + t, h) * P + q * PER;
+            const uint32_t dx_ = static_cast<uint32_t>(__cvta_generic_to_shared(xs + t * P + q * PER));
+            const uint32_t dy_ = static_cast<uint32_t>(__cvta_generic_to_shared(dys + t * P + q * PER));
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dx_), "l"(x + src) : "memory");
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dy_), "l"(dy + src) : "memory");
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    } else {
+        for (int idx = tid; idx < n * P; idx += blockDim.x) {
+            const int t = idx / P, q = idx - t * P;
+            xs[t * P + q] = x[blh(d, b, c0 + t, h) * P + q];
+            dys[t * P + q] = dy[blh(d, b, c0 + t, h) * P + q];
+        }
+    }
+    for (int idx = tid; idx < (Q - n) * P; idx += blockDim.x) {  // rows past a ragged end
+        const int t = n + idx / P, q = idx % P;
+        xs[t * P + q] = from_f<T>(0.f);
+        dys[t * P + q] = from_f<T>(0.f);
+    }
+    const size_t sbase = (bh * d.nc + c) * size_t(K) * P;
+    for (int idx = tid; idx < K * P; idx += blockDim.x) {
+        Sin[idx] = to_f(S_in[sbase + idx]);
+        Gam[idx] = to_f(dS_out[sbase + idx]);
+    }
+    if (tid < K) itau[tid] = 1.f / tau[h * K + tid];
+    if (tid < 64) red[tid] = 0.f;
+    if (tid < 32) cdot[tid] = dtq[tid] = 0.f;
+    const float log_cap = head_log_cap(tau, h, K);
+    chunk_rates(d, b, h, c0, n, log_cap, dt, alpha, lam, e_s, E_s, cl_s);
+    __syncthreads();
+    const double Eend = E_s[n - 1];
+    for (int idx = tid; idx < QK; idx += blockDim.x) {
+        const int t = idx / K, m = idx - t * K;
+        float rho = 0.f, kap = 0.f, A = 0.f, u = 0.f, w_w = 0.f, w_r = 0.f, Bt = 0.f, Ct = 0.f;
+        if (t < n) {
+            const size_t wi = blh(d, b, c0 + t, h) * K + m;
+            const size_t gi = (size_t(b) * d.L + c0 + t) * d.G + g;
+            w_w = to_f(ww[wi]);
+            w_r = to_f(wr[wi]);
+            Bt = to_f(Bm[gi]);
+            Ct = to_f(Cm[gi]);
+            const float z = e_s[t] * itau[m];
+            rho = expf(-z);
+            kap = -expm1f(-z) * w_w;
+            A = expf(-float(E_s[t]) * itau[m]);
+            u = expf(-float(Eend - E_s[t]) * itau[m]);
+        }
+        rho_s[idx] = rho; kap_s[idx] = kap; kb_s[idx] = kap * Bt; wc_s[idx] = w_r * Ct;
+        A_s[idx] = A; u_s[idx] = u; ww_s[idx] = w_w; wr_s[idx] = w_r; Bq[idx] = Bt; Cq[idx] = Ct;
+        XG[idx] = 0.f; YS[idx] = 0.f;
+    }
+    for (int idx = tid; idx < kN1BQ * Q1; idx += blockDim.x) H[idx] = 0.f;
+    if constexpr (VEC) asm volatile("cp.async.wait_all;" ::: "memory");
+    __syncthreads();
+
+    // ---- P1: H = dY X^T (4 x 4 tiles over 8 p-segments), the dot products over p of x with
+    // gamma, dy with S_in and gamma with S_in (4 x 4 tiles over 8 p-segments), by partial sums
+    // added into shared memory
+    {
+        const int qt = Q / 4, seg = (P + 7) / 8;
+        for (int item = tid; item < qt * qt * 8; item += blockDim.x) {
+            const int tile = item >> 3, s8 = item & 7;
+            const int t0 = 4 * (tile / qt), k0 = 4 * (tile % qt);
+            if (k0 > t0 + 3) continue;
+            float acc[4][4] = {};
+            for (int q = s8 * seg; q < min(P, (s8 + 1) * seg); ++q) {
+                float dv[4], xv[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    dv[i] = to_f(dys[(t0 + i) * P + q]);
+                    xv[i] = to_f(xs[(k0 + i) * P + q]);
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(dv[i], xv[j], acc[i][j]);
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) atomicAdd(&H[(t0 + i) * Q1 + k0 + j], acc[i][j]);
+        }
+        const int mt = (K + 3) / 4;
+        for (int item = tid; item < qt * mt * 8; item += blockDim.x) {
+            const int tile = item >> 3, s8 = item & 7;
+            const int t0 = 4 * (tile / mt), m0 = 4 * (tile % mt);
+            float ag[4][4] = {}, as[4][4] = {}, ac[4] = {};
+            for (int q = s8 * seg; q < min(P, (s8 + 1) * seg); ++q) {
+                float xv[4], dv[4], gv[4], sv[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    xv[i] = to_f(xs[(t0 + i) * P + q]);
+                    dv[i] = to_f(dys[(t0 + i) * P + q]);
+                    gv[i] = m0 + i < K ? Gam[(m0 + i) * P + q] : 0.f;
+                    sv[i] = m0 + i < K ? Sin[(m0 + i) * P + q] : 0.f;
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        ag[i][j] = fmaf(xv[i], gv[j], ag[i][j]);
+                        as[i][j] = fmaf(dv[i], sv[j], as[i][j]);
+                    }
+                if (t0 == 0)
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) ac[j] = fmaf(gv[j], sv[j], ac[j]);
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    if (m0 + j < K) {
+                        atomicAdd(&XG[(t0 + i) * K + m0 + j], ag[i][j]);
+                        atomicAdd(&YS[(t0 + i) * K + m0 + j], as[i][j]);
+                    }
+            if (t0 == 0)
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    if (m0 + j < K) atomicAdd(&cdot[m0 + j], ac[j]);
+        }
+    }
+    __syncthreads();
+
+    // ---- P2: pair passes, one warp per group of four modes (KP / 4 warps).  Row pass (lane =
+    // row t): Gamma row, Gamma' o H row (rect), intra dw_read-like sums; column pass (lane = k):
+    // intra dkappa B-like sums.  Gamma and Gamma' o H add up over the mode groups.
+    for (int idx = tid; idx < kN1BQ * Q1; idx += blockDim.x) Gm[idx] = XR[idx] = 0.f;
+    __syncthreads();
+    {
+        const int w = tid >> 5, lane = tid & 31;
+        if (w < KP / 4 && lane < Q) {
+            const int m0 = 4 * w;
+            {  // row pass
+                const int t = lane;
+                float dw[4] = {0.f, 0.f, 0.f, 0.f};
+                if (t < n) {
+                    for (int k = 0; k <= t; ++k) {
+                        const float dE = float(E_s[t] - E_s[k]);
+                        const float hv = H[t * Q1 + k];
+                        float gam = 0.f, gamt = 0.f;
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            const int m = m0 + j;
+                            if (m < K) {
+                                const float W = expf(-dE * itau[m]);
+                                const float kw = kb_s[k * K + m] * W;
+                                const float a = wc_s[t * K + m] * kw;
+                                gam += a;
+                                gamt = fmaf(a, itau[m], gamt);
+                                dw[j] = fmaf(kw, hv, dw[j]);
+                            }
+                        }
+                        atomicAdd(&Gm[t * Q1 + k], gam);
+                        atomicAdd(&XR[t * Q1 + k], gamt * hv);
+                    }
+                }
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    if (m0 + j < K) dwci[t * K + m0 + j] = dw[j];
+            }
+            {  // column pass
+                const int k = lane;
+                float dk[4] = {0.f, 0.f, 0.f, 0.f};
+                if (k < n) {
+                    for (int t = k; t < n; ++t) {
+                        const float dE = float(E_s[t] - E_s[k]);
+                        const float hv = H[t * Q1 + k];
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            const int m = m0 + j;
+                            if (m < K) dk[j] = fmaf(wc_s[t * K + m] * expf(-dE * itau[m]), hv, dk[j]);
+                        }
+                    }
+                }
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    if (m0 + j < K) dkbi[k * K + m0 + j] = dk[j];
+            }
+        }
+    }
+    __syncthreads();
+
+    // ---- P3: rectangle sums of Gamma' o H over pairs k < t <= t' (row prefix, column suffix)
+    float *rp_s = red + 32;  // [Q <= 32] (block_sum below uses red[0 .. 8))
+    if (tid < Q) {
+        float run = 0.f;
+        for (int j = 0; j < Q; ++j) {
+            const float v = XR[tid * Q1 + j];
+            XR[tid * Q1 + j] = run;
+            run += v;
+        }
+    }
+    __syncthreads();
+    if (tid < Q) {
+        float s = 0.f;
+        for (int tp = tid; tp < n; ++tp) s += XR[tp * Q1 + tid];
+        rp_s[tid] = s;
+    }
+
+    // ---- P4: dx[k][p] = sum_m s_{k,m} gamma_m[p] + sum_{t>=k} Gamma[t][k] dy_t[p] + D dy_k[p]
+    // (one thread per p; the dy column and gamma of the thread's p in registers)
+    const float Dh = Dv[h];
+    float ddv = 0.f;  // sum dy x for dD
+    for (int q = tid; q < P; q += blockDim.x) {
+        float dyc[kN1BQ], gv[KP];
+#pragma unroll
+        for (int t = 0; t < kN1BQ; ++t) dyc[t] = t < Q ? to_f(dys[t * P + q]) : 0.f;
+#pragma unroll
+        for (int m = 0; m < KP; ++m) gv[m] = m < K ? Gam[m * P + q] : 0.f;
+        for (int k = 0; k < n; ++k) {
+            float acc = Dh * dyc[k];
+#pragma unroll
+            for (int m = 0; m < KP; ++m)
+                if (m < K) acc = fmaf(kb_s[k * K + m] * u_s[k * K + m], gv[m], acc);
+#pragma unroll
+            for (int t = 0; t < kN1BQ; ++t)
+                if (t >= k && t < n) acc = fmaf(Gm[t * Q1 + k], dyc[t], acc);
+            dx[blh(d, b, c0 + k, h) * P + q] = from_f<T>(acc);
+            ddv = fmaf(dyc[k], to_f(xs[k * P + q]), ddv);
+        }
+    }
+    ddv = block_sum(ddv, red);  // contains __syncthreads (also publishes rp_s)
+    if (tid == 0) atomicAdd(&dD[h], ddv);
+
+    // ---- P5: per-position scalars.  a_t / b_k are the S_in / gamma terms of
+    // sum_m rho <g_t, S_{t-1}>_m / tau_m (suffix and exclusive prefix sums), c the
+    // <gamma, S_in> term, rp_s the pairs; then dDelta, dalpha, dlambda, the weights, dB, dC.
+    float *a_s = XR, *b_s = XR + 64;  // XR is free now
+    if (tid < n) {
+        const int t = tid;
+        float a = 0.f, bb = 0.f;
+        for (int m = 0; m < K; ++m) {
+            const int q = t * K + m;
+            a = fmaf(wc_s[q] * A_s[q] * YS[q], itau[m], a);
+            bb = fmaf(kb_s[q] * u_s[q] * XG[q], itau[m], bb);
+        }
+        a_s[t] = a;
+        b_s[t] = bb;
+    }
+    __syncthreads();
+    float cprime = 0.f;
+    for (int m = 0; m < K; ++m) cprime = fmaf(expf(-float(Eend) * itau[m]) * itau[m], cdot[m], cprime);
+    if (tid < n) {
+        const int t = tid;
+        float suf = 0.f, pre = 0.f;
+        for (int j = t; j < n; ++j) suf += a_s[j];
+        for (int j = 0; j < t; ++j) pre += b_s[j];
+        const float R = suf + pre + cprime + rp_s[t];
+        float de = -R, sB = 0.f, sC = 0.f;
+        const size_t i = blh(d, b, c0 + t, h);
+        for (int m = 0; m < K; ++m) {
+            const int q = t * K + m;
+            const float dkb = u_s[q] * XG[q] + dkbi[q];   // d(kappa B)
+            const float dwc = A_s[q] * YS[q] + dwci[q];   // d(w_read C)
+            const float dk = dkb * Bq[q];                 // d kappa
+            de = fmaf(dk * rho_s[q] * ww_s[q], itau[m], de);
+            dwr_o[i * K + m] = from_f<T>(dwc * Cq[q]);
+            dww_o[i * K + m] = from_f<T>(dk * (-expm1f(-e_s[t] * itau[m])));
+            sB = fmaf(dkb, kap_s[q], sB);
+            sC = fmaf(dwc, wr_s[q], sC);
+            if (dtau) {
+                const double Et = E_s[t];
+                const double tq = Et * double(wc_s[q] * A_s[q] * YS[q]) +
+                                  (Eend - Et) * double(kb_s[q] * u_s[q] * XG[q]) -
+                                  double(e_s[t]) * double(dk) * double(rho_s[q]) * double(ww_s[q]);
+                atomicAdd(&dtq[m], float(tq));
+            }
+        }
+        const size_t gi = (size_t(b) * d.L + c0 + t) * d.G + g;
+        atomicAdd(&dB_acc[gi], sB);
+        atomicAdd(&dC_acc[gi], sC);
+        const float e = e_s[t];
+        const bool cl = cl_s[t] != 0.f;
+        const float al = alpha[i], lm = lam[i], dtv = dt[i];
+        const float ge = cl ? 0.f : de * e;
+        ddt[i] = ge / dtv;
+        dlam[i] = ge / (al * lm);
+        dalpha[i] = -ge * logf(lm) / (al * al);
+    }
+    if (dtau) {
+        __syncthreads();
+        if (tid < K) {
+            const float it = itau[tid];
+            const float chunk_term = float(Eend) * expf(-float(Eend) * it) * cdot[tid];
+            atomicAdd(&dtau[h * K + tid], (dtq[tid] + chunk_term) * it * it);
+        }
+    }
+}
+
+bool n1_bwd_fits(const ScanDims &d, size_t esz) {
+    return d.N == 1 && d.Q <= kN1BQ && d.K <= 32 && N1BwdSmem(d.P, d.K, esz).total <= 227 * 1024 &&
+           size_t(d.H) * ((d.P + kN1P - 1) / kN1P) <= 65535;
+}
+
+template <typename T, typename TS>
+cudaError_t bwd_n1(const ScanDims &d, const ScanPtrs &p, void *S_in, void *dS_out, float *dB_acc,
+                   float *dC_acc, float *scratch, bool reuse, cudaStream_t st) {
+    const int npb = (d.P + kN1P - 1) / kN1P;
+    float *loc = scratch, *dec = scratch + size_t(d.B) * d.H * d.nc * d.K * d.P;
+    const bool vec = (reinterpret_cast<uintptr_t>(p.x) % 16 == 0) && (reinterpret_cast<uintptr_t>(p.dy) % 16 == 0) &&
+                     ((size_t(d.P) * sizeof(T)) % 16 == 0);
+    const int KP = d.K <= 4 ? 4 : d.K <= 8 ? 8 : d.K <= 16 ? 16 : 32;
+    using I4 = std::integral_constant<int, 4>;
+    using I8 = std::integral_constant<int, 8>;
+    using I16 = std::integral_constant<int, 16>;
+    using I32 = std::integral_constant<int, 32>;
+    auto pick = [&](auto f) { return KP == 4 ? f(I4{}) : KP == 8 ? f(I8{}) : KP == 16 ? f(I16{}) : f(I32{}); };
+    const size_t n1smem = N1Smem(sizeof(T)).total;
+    const size_t total = size_t(d.B) * d.H * d.K * d.P;
+    cudaError_t e = cudaSuccess;
+    if (!reuse && d.nc > 0) {  // the forward's per-chunk entering states
+        auto kl = pick([&](auto kp) {
+            constexpr int V = decltype(kp)::value;
+            return vec ? n1_local<T, true, V> : n1_local<T, false, V>;
+        });
+        cudaFuncSetAttribute(kl, cudaFuncAttributeMaxDynamicSharedMemorySize, int(n1smem));
+        trace_begin("local_fwd_n1", st);
+        kl<<<dim3(d.nc, d.H * npb, d.B), kN1P, n1smem, st>>>(d, (const T *)p.x, (const T *)p.Bm, (const T *)p.ww,
+                                                             p.dt, p.alpha, p.lam, p.tau, loc, dec);
+        trace_end(st);
+        trace_begin("combine_fwd_n1", st);
+        n1_combine<TS><<<unsigned((total + 255) / 256), 256, 0, st>>>(d, loc, dec, p.h0, (TS *)S_in, nullptr);
+        trace_end(st);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    const size_t ngn = size_t(d.B) * d.L * d.G * d.N;
+    if ((e = cudaMemsetAsync(p.dD, 0, sizeof(float) * d.H, st)) != cudaSuccess) return e;
+    if ((e = cudaMemsetAsync(dB_acc, 0, sizeof(float) * ngn, st)) != cudaSuccess) return e;
+    if ((e = cudaMemsetAsync(dC_acc, 0, sizeof(float) * ngn, st)) != cudaSuccess) return e;
+    if (p.dtau && (e = cudaMemsetAsync(p.dtau, 0, sizeof(float) * d.H * d.K, st)) != cudaSuccess) return e;
+    if (d.nc > 0) {  // the adjoint's chunk carries
+        auto kr = pick([&](auto kp) {
+            constexpr int V = decltype(kp)::value;
+            return vec ? n1_rev_local<T, true, V> : n1_rev_local<T, false, V>;
+        });
+        cudaFuncSetAttribute(kr, cudaFuncAttributeMaxDynamicSharedMemorySize, int(n1smem));
+        trace_begin("local_rev_n1", st);
+        kr<<<dim3(d.nc, d.H * npb, d.B), kN1P, n1smem, st>>>(d, (const T *)p.dy, (const T *)p.Cm, (const T *)p.wr,
+                                                             p.dt, p.alpha, p.lam, p.tau, loc, dec);
+        trace_end(st);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    trace_begin("combine_rev_n1", st);
+    n1_combine_rev<TS><<<unsigned((total + 255) / 256), 256, 0, st>>>(d, loc, dec, p.dh_final, (TS *)dS_out, p.dh0);
+    trace_end(st);
+    if ((e = cudaGetLastError()) != cudaSuccess || d.nc == 0) return e;  // L = 0: dh0 = dh_final
+    const size_t smem = N1BwdSmem(d.P, d.K, sizeof(T)).total;
+    auto kb = pick([&](auto kp) {
+        constexpr int V = decltype(kp)::value;
+        return vec ? n1_chunk_bwd<T, TS, true, V> : n1_chunk_bwd<T, TS, false, V>;
+    });
+    cudaFuncSetAttribute(kb, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    trace_begin("chunk_bwd_n1", st);
+    kb<<<dim3(d.nc, d.H, d.B), kThreads, smem, st>>>(
+        d, (const T *)p.x, (const T *)p.Bm, (const T *)p.Cm, (const T *)p.wr, (const T *)p.ww, (const T *)p.dy,
+        p.dt, p.alpha, p.lam, p.tau, p.D, (const TS *)S_in, (const TS *)dS_out, (T *)p.dx, (T *)p.dwr,
+        (T *)p.dww, p.ddt, p.dalpha, p.dlam, p.dD, dB_acc, dC_acc, p.dtau);
+    trace_end(st);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = dtau_pairs_launch(d, sizeof(T) == 2 ? 1 : 0, p, st)) != cudaSuccess) return e;
+    if (sizeof(T) == 2 && ngn > 0) {
+        const unsigned blocks = unsigned(std::min<size_t>((ngn + 255) / 256, 4096));
+        trace_begin("f32_to_bf16", st);
+        f32_to_bf16_kernel<<<blocks, 256, 0, st>>>(dB_acc, (__nv_bfloat16 *)p.dB, ngn);
+        trace_end(st);
+        trace_begin("f32_to_bf16", st);
+        f32_to_bf16_kernel<<<blocks, 256, 0, st>>>(dC_acc, (__nv_bfloat16 *)p.dC, ngn);
+        trace_end(st);
+        e = cudaGetLastError();
+    }
+    return e;
+}
+
 template <typename T, typename TS>
 cudaError_t bwd_t(const ScanDims &d, const ScanPtrs &p, void *S_in, void *dS_out, float *dB_acc,
-                  float *dC_acc, bool reuse, cudaStream_t st) {
+                  float *dC_acc, float *n1_scratch, bool reuse, cudaStream_t st) {
+    if (uses_n1(d) && n1_bwd_fits(d, sizeof(T)))
+        return bwd_n1<T, TS>(d, p, S_in, dS_out, dB_acc, dC_acc, n1_scratch, reuse, st);
     cudaError_t e = cudaSuccess;
     if (!reuse) e = run_state_pass<T, TS>(d, false, p.x, p.Bm, p.ww, p, p.h0, S_in, nullptr, st);
     if (e != cudaSuccess) return e;
@@ -1227,6 +1766,14 @@ cudaError_t bwd_t(const ScanDims &d, const ScanPtrs &p, void *S_in, void *dS_out
 }  // namespace
 
 int simt_pick_chunk(const ScanDims &d0, int requested) {
+    if (d0.N == 1) {  // the N = 1 kernels: chunk 32 unless 16 is asked for (the backward's tiles)
+        for (int Q : {32, 16}) {
+            if (requested && requested != Q) continue;
+            ScanDims d = d0;
+            d.Q = Q;
+            if (uses_n1(d) && n1_bwd_fits(d, 4)) return Q;
+        }
+    }
     const int cands[3] = {64, 32, 16};
     for (int qi = 0; qi < 3; ++qi) {
         const int Q = cands[qi];
@@ -1260,9 +1807,10 @@ cudaError_t simt_scan_fwd(const ScanDims &d, int dtype, const ScanPtrs &p, void 
 }
 
 cudaError_t simt_scan_bwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in,
-                          void *dS_out, float *dB_acc, float *dC_acc, bool reuse, cudaStream_t st) {
-    if (dtype == 0) return bwd_t<float, float>(d, p, S_in, dS_out, dB_acc, dC_acc, reuse, st);
-    return bwd_t<__nv_bfloat16, __nv_bfloat16>(d, p, S_in, dS_out, dB_acc, dC_acc, reuse, st);
+                          void *dS_out, float *dB_acc, float *dC_acc, float *n1_scratch, bool reuse,
+                          cudaStream_t st) {
+    if (dtype == 0) return bwd_t<float, float>(d, p, S_in, dS_out, dB_acc, dC_acc, n1_scratch, reuse, st);
+    return bwd_t<__nv_bfloat16, __nv_bfloat16>(d, p, S_in, dS_out, dB_acc, dC_acc, n1_scratch, reuse, st);
 }
 
 }  // namespace frac

@@ -378,3 +378,16 @@ def test_paper_layer_shape_backward_reusing_forward_states():
     ref = _ora_bwd(d64)
     for k in GRADS:
         assert_close(k, to_host64(g[k]), ref[k], 1e-2)
+
+
+@pytest.mark.parametrize("shape", [
+    synth.Shape(2, 77, 3, 200, 1, 1, 5, 16, "f32"),   # K = 5, P off a multiple of 256, chunk 16, ragged
+    synth.Shape(1, 130, 2, 64, 2, 1, 8, 32, "bf16"),  # one head per B/C group
+    synth.Shape(1, 96, 4, 256, 2, 1, 16, 0, "f32"),   # two heads per group, whole chunks
+    synth.Shape(1, 0, 2, 32, 1, 1, 4, 0, "f32"),      # empty sequence: dh0 = dh_final
+])
+def test_n1_backward_shapes(shape):
+    """N = 1 backward (reverse chunk carries and the per-chunk gradient kernel): mode counts off a
+    multiple of 4, p blocks past the head dimension, groups (dB, dC summed over their heads),
+    chunk sizes, ragged and empty sequences."""
+    _check_bwd(shape, seed=70 + shape.nmodes, h0=True, dhf=True, chunk=shape.chunk)
