@@ -111,9 +111,17 @@ __global__ void __launch_bounds__(32 * kRows) conv1d_fwd_kernel(ConvArgs a) {
         }
     }
     const int t1 = min(t0 + kRun, a.L);
+    constexpr int kB = 8;  // positions whose inputs are loaded together (all in flight at once)
+    float2 xb[kB];
     for (int t = t0; t < t1; ++t) {
+        if ((t - t0) % kB == 0) {
+#pragma unroll
+            for (int j = 0; j < kB; ++j)
+                xb[j] = t + j < t1 ? ld2<T, VEC2>(static_cast<const T *>(a.x) + (size_t(b) * a.L + t + j) * a.C + c, has1)
+                                   : make_float2(0.f, 0.f);
+        }
         const size_t off = (size_t(b) * a.L + t) * a.C + c;
-        const float2 xv = ld2<T, VEC2>(static_cast<const T *>(a.x) + off, has1);
+        const float2 xv = xb[(t - t0) % kB];
         win0[W - 1] = xv.x;
         win1[W - 1] = xv.y;
         float p0 = b0, p1 = b1;
@@ -180,10 +188,20 @@ __global__ void __launch_bounds__(32 * kRows) conv1d_bwd_kernel(ConvArgs a) {
         }
         const int tr = min(t0 + kRun, a.L);          // this run's positions: [t0, tr)
         const int tg = min(tr + W - 1, a.L);         // g is needed up to tg - 1 for dx of the run
+        constexpr int kB = 8;  // positions whose inputs are loaded together
+        float2 xb[kB], db[kB];
         for (int t = t0; t < tg; ++t) {
-            const size_t off = (size_t(b) * a.L + t) * a.C + c;
-            const float2 xv = ld2<T, VEC2>(static_cast<const T *>(a.x) + off, has1);
-            const float2 dv = ld2<T, VEC2>(static_cast<const T *>(a.du) + off, has1);
+            if ((t - t0) % kB == 0) {
+#pragma unroll
+                for (int j = 0; j < kB; ++j) {
+                    const bool in = t + j < tg;
+                    const size_t o = (size_t(b) * a.L + t + j) * a.C + c;
+                    xb[j] = in ? ld2<T, VEC2>(static_cast<const T *>(a.x) + o, has1) : make_float2(0.f, 0.f);
+                    db[j] = in ? ld2<T, VEC2>(static_cast<const T *>(a.du) + o, has1) : make_float2(0.f, 0.f);
+                }
+            }
+            const float2 xv = xb[(t - t0) % kB];
+            const float2 dv = db[(t - t0) % kB];
             win0[W - 1] = xv.x;
             win1[W - 1] = xv.y;
             float p0 = b0, p1 = b1;

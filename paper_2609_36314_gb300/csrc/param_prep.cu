@@ -257,7 +257,9 @@ cudaError_t launch_kp(const PrepArgs &a, bool backward, bool vec, cudaStream_t s
     int dev = 0, sms = 152;
     if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int64_t want = (a.n + threads - 1) / threads;
-    const int blocks = int(std::max<int64_t>(1, std::min<int64_t>(want, int64_t(sms) * 8)));
+    // the forward has no sums: one row per thread; the backward caps its grid (its per-block
+    // reductions end in global atomics)
+    const int blocks = int(std::max<int64_t>(1, std::min<int64_t>(want, backward ? int64_t(sms) * 8 : int64_t(1) << 30)));
     if (!backward) {
         trace_begin("param_prep_fwd", st);
         if (vec)

@@ -1404,70 +1404,98 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
     if constexpr (VEC) asm volatile("cp.async.wait_all;" ::: "memory");
     __syncthreads();
 
-    // ---- P1: H = dY X^T (4 x 4 tiles over 8 p-segments), the dot products over p of x with
-    // gamma, dy with S_in and gamma with S_in (4 x 4 tiles over 8 p-segments), by partial sums
-    // added into shared memory
+    // ---- P1: H = dY X^T and the dot products over p of x with gamma, dy with S_in and gamma with
+    // S_in: one warp per 4 x 4 output tile, the lanes on consecutive p (no bank conflicts), the
+    // 16 partial sums reduced across the warp by halving exchanges (lane l ends with one value)
     {
-        const int qt = Q / 4, seg = (P + 7) / 8;
-        for (int item = tid; item < qt * qt * 8; item += blockDim.x) {
-            const int tile = item >> 3, s8 = item & 7;
-            const int t0 = 4 * (tile / qt), k0 = 4 * (tile % qt);
-            if (k0 > t0 + 3) continue;
-            float acc[4][4] = {};
-            for (int q = s8 * seg; q < min(P, (s8 + 1) * seg); ++q) {
-                float dv[4], xv[4];
+        const int w = tid >> 5, lane = tid & 31, nw = blockDim.x >> 5;
+        const int qt = Q / 4, mt = (K + 3) / 4;
+        const int nH = qt * (qt + 1) / 2;  // tiles on or below the diagonal
+        for (int item = w; item < nH + qt * mt; item += nw) {
+            float v[16], v2[16];
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    dv[i] = to_f(dys[(t0 + i) * P + q]);
-                    xv[i] = to_f(xs[(k0 + i) * P + q]);
+            for (int i = 0; i < 16; ++i) v[i] = v2[i] = 0.f;
+            float vc[4] = {0.f, 0.f, 0.f, 0.f};
+            int r0, c0t;
+            const bool isH = item < nH;
+            if (isH) {  // item -> (row tile, column tile <= row tile)
+                int rt = 0, rem = item;
+                while (rem > rt) rem -= ++rt;
+                r0 = 4 * rt;
+                c0t = 4 * rem;
+                for (int q = lane; q < P; q += 32) {
+                    float dv[4], xv[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        dv[i] = to_f(dys[(r0 + i) * P + q]);
+                        xv[i] = to_f(xs[(c0t + i) * P + q]);
+                    }
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) v[4 * i + j] = fmaf(dv[i], xv[j], v[4 * i + j]);
                 }
+            } else {
+                const int it = item - nH;
+                r0 = 4 * (it / mt);
+                c0t = 4 * (it % mt);  // first mode
+                for (int q = lane; q < P; q += 32) {
+                    float xv[4], dv[4], gv[4], sv[4];
 #pragma unroll
-                for (int i = 0; i < 4; ++i)
+                    for (int i = 0; i < 4; ++i) {
+                        xv[i] = to_f(xs[(r0 + i) * P + q]);
+                        dv[i] = to_f(dys[(r0 + i) * P + q]);
+                        gv[i] = c0t + i < K ? Gam[(c0t + i) * P + q] : 0.f;
+                        sv[i] = c0t + i < K ? Sin[(c0t + i) * P + q] : 0.f;
+                    }
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(dv[i], xv[j], acc[i][j]);
+                    for (int i = 0; i < 4; ++i)
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            v[4 * i + j] = fmaf(xv[i], gv[j], v[4 * i + j]);
+                            v2[4 * i + j] = fmaf(dv[i], sv[j], v2[4 * i + j]);
+                        }
+                    if (r0 == 0)
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) vc[j] = fmaf(gv[j], sv[j], vc[j]);
+                }
             }
+            // halving exchanges: after offsets 16, 8, 4, 2 lane l holds value
+            // 8 b4 + 4 b3 + 2 b2 + b1 (bk = bit k of l) summed over 16 lanes; offset 1 completes it
+            auto reduce16 = [&](float *a) {
 #pragma unroll
-            for (int i = 0; i < 4; ++i)
+                for (int o = 16, cnt = 8; o >= 2; o >>= 1, cnt >>= 1) {
+                    const bool up = (lane & o) != 0;
 #pragma unroll
-                for (int j = 0; j < 4; ++j) atomicAdd(&H[(t0 + i) * Q1 + k0 + j], acc[i][j]);
-        }
-        const int mt = (K + 3) / 4;
-        for (int item = tid; item < qt * mt * 8; item += blockDim.x) {
-            const int tile = item >> 3, s8 = item & 7;
-            const int t0 = 4 * (tile / mt), m0 = 4 * (tile % mt);
-            float ag[4][4] = {}, as[4][4] = {}, ac[4] = {};
-            for (int q = s8 * seg; q < min(P, (s8 + 1) * seg); ++q) {
-                float xv[4], dv[4], gv[4], sv[4];
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    xv[i] = to_f(xs[(t0 + i) * P + q]);
-                    dv[i] = to_f(dys[(t0 + i) * P + q]);
-                    gv[i] = m0 + i < K ? Gam[(m0 + i) * P + q] : 0.f;
-                    sv[i] = m0 + i < K ? Sin[(m0 + i) * P + q] : 0.f;
+                    for (int i = 0; i < 8; ++i) {
+                        if (i < cnt) {
+                            const float send = up ? a[i] : a[i + cnt];
+                            const float keep = up ? a[i + cnt] : a[i];
+                            a[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+                        }
+                    }
                 }
-#pragma unroll
-                for (int i = 0; i < 4; ++i)
+                a[0] += __shfl_xor_sync(0xffffffffu, a[0], 1);
+            };
+            const int vi = 8 * ((lane >> 4) & 1) + 4 * ((lane >> 3) & 1) + 2 * ((lane >> 2) & 1) + ((lane >> 1) & 1);
+            const int ri = vi >> 2, ci = vi & 3;
+            reduce16(v);
+            if (isH) {
+                if ((lane & 1) == 0) H[(r0 + ri) * Q1 + c0t + ci] = v[0];
+            } else {
+                reduce16(v2);
+                if ((lane & 1) == 0 && c0t + ci < K) {
+                    XG[(r0 + ri) * K + c0t + ci] = v[0];
+                    YS[(r0 + ri) * K + c0t + ci] = v2[0];
+                }
+                if (r0 == 0) {
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
-                        ag[i][j] = fmaf(xv[i], gv[j], ag[i][j]);
-                        as[i][j] = fmaf(dv[i], sv[j], as[i][j]);
+                        const float sc = warp_sum(vc[j]);
+                        if (lane == 0 && c0t + j < K) cdot[c0t + j] = sc;
                     }
-                if (t0 == 0)
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) ac[j] = fmaf(gv[j], sv[j], ac[j]);
+                }
             }
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-#pragma unroll
-                for (int j = 0; j < 4; ++j)
-                    if (m0 + j < K) {
-                        atomicAdd(&XG[(t0 + i) * K + m0 + j], ag[i][j]);
-                        atomicAdd(&YS[(t0 + i) * K + m0 + j], as[i][j]);
-                    }
-            if (t0 == 0)
-#pragma unroll
-                for (int j = 0; j < 4; ++j)
-                    if (m0 + j < K) atomicAdd(&cdot[m0 + j], ac[j]);
         }
     }
     __syncthreads();
