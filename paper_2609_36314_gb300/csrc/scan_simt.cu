@@ -1283,28 +1283,30 @@ __global__ void __launch_bounds__(256) n1_combine_rev(ScanDims d, const float *_
 }
 
 constexpr int kN1BQ = 32;  // chunk of the N = 1 backward (shared-memory tiles [Q][P])
+constexpr int kGS = 36;    // row stride of its Gamma tile (rows read as 16-byte pieces)
 
 struct N1BwdSmem {
-    size_t E, e, cl, itau, red, cdot, dtq, qk, x, y, sin, gam, H, Gm, XR, total;
+    size_t E, Ef, e, cl, itau, red, cdot, dtq, qk, x, y, sin, gam, H, Gm, XR, total;
     int P;
     __host__ __device__ N1BwdSmem(int P_, int K, size_t esz) : P(P_) {
         E = 0;                                                   // double [Q]
-        e = E + sizeof(double) * kN1BQ;                          // float [Q]
+        Ef = E + sizeof(double) * kN1BQ;                         // float2 [Q]: E as hi + lo
+        e = Ef + sizeof(float) * 2 * kN1BQ;                      // float [Q]
         cl = e + sizeof(float) * kN1BQ;                          // float [Q]
         itau = cl + sizeof(float) * kN1BQ;                       // float [32]
         red = itau + sizeof(float) * 32;                         // float [64]
         cdot = red + sizeof(float) * 64;                         // float [32]
         dtq = cdot + sizeof(float) * 32;                         // float [32]: dtau sums per mode
-        qk = dtq + sizeof(float) * 32;                           // float [14][Q][K]
-        x = qk + sizeof(float) * 14 * kN1BQ * K;                 // T [Q][P]
+        qk = dtq + sizeof(float) * 32;                           // float [15][Q][K]
+        x = qk + sizeof(float) * 15 * kN1BQ * K;                 // T [Q][P]
         x = (x + 15) / 16 * 16;
         y = x + esz * kN1BQ * P;                                 // T [Q][P]
         y = (y + 15) / 16 * 16;
         sin = y + esz * kN1BQ * P;                               // float [K][P]
         gam = sin + sizeof(float) * K * P;                       // float [K][P]
-        H = gam + sizeof(float) * K * P;                         // float [Q][Q + 1]
-        Gm = H + sizeof(float) * kN1BQ * (kN1BQ + 1);            // float [Q][Q + 1]
-        XR = Gm + sizeof(float) * kN1BQ * (kN1BQ + 1);           // float [Q][Q + 1]
+        H = (gam + sizeof(float) * K * P + 15) / 16 * 16;         // float [Q][Q + 1]
+        Gm = H + sizeof(float) * kN1BQ * (kN1BQ + 1);            // float [Q][kGS]
+        XR = Gm + sizeof(float) * kN1BQ * kGS;                   // float [Q][Q + 1]
         total = XR + sizeof(float) * kN1BQ * (kN1BQ + 1);
     }
 };
@@ -1323,6 +1325,7 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
     const int K = d.K, P = d.P, Q = d.Q;
     const N1BwdSmem L_(P, K, sizeof(T));
     double *E_s = reinterpret_cast<double *>(sm_raw + L_.E);
+    float2 *Ef_s = reinterpret_cast<float2 *>(sm_raw + L_.Ef);
     float *e_s = reinterpret_cast<float *>(sm_raw + L_.e), *cl_s = reinterpret_cast<float *>(sm_raw + L_.cl);
     float *itau = reinterpret_cast<float *>(sm_raw + L_.itau), *red = reinterpret_cast<float *>(sm_raw + L_.red);
     float *cdot = reinterpret_cast<float *>(sm_raw + L_.cdot);
@@ -1332,7 +1335,8 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
     // [Q][K] arrays: coefficients, then the dot products and pair sums
     float *rho_s = qk, *kap_s = qk + QK, *kb_s = qk + 2 * QK, *wc_s = qk + 3 * QK, *A_s = qk + 4 * QK,
           *u_s = qk + 5 * QK, *ww_s = qk + 6 * QK, *wr_s = qk + 7 * QK, *XG = qk + 8 * QK, *YS = qk + 9 * QK,
-          *dwci = qk + 10 * QK, *dkbi = qk + 11 * QK, *Bq = qk + 12 * QK, *Cq = qk + 13 * QK;
+          *dwci = qk + 10 * QK, *dkbi = qk + 11 * QK, *Bq = qk + 12 * QK, *Cq = qk + 13 * QK,
+          *s_s = qk + 14 * QK;  // kappa B u, mode-major [K][Q]
     T *xs = reinterpret_cast<T *>(sm_raw + L_.x), *dys = reinterpret_cast<T *>(sm_raw + L_.y);
     float *Sin = reinterpret_cast<float *>(sm_raw + L_.sin), *Gam = reinterpret_cast<float *>(sm_raw + L_.gam);
     float *H = reinterpret_cast<float *>(sm_raw + L_.H), *Gm = reinterpret_cast<float *>(sm_raw + L_.Gm);
@@ -1363,7 +1367,7 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
             dys[t * P + q] = dy[blh(d, b, c0 + t, h) * P + q];
         }
     }
-    for (int idx = tid; idx < (Q - n) * P; idx += blockDim.x) {  // rows past a ragged end
+    for (int idx = tid; idx < (kN1BQ - n) * P; idx += blockDim.x) {  // rows past a ragged end
         const int t = n + idx / P, q = idx % P;
         xs[t * P + q] = from_f<T>(0.f);
         dys[t * P + q] = from_f<T>(0.f);
@@ -1398,9 +1402,15 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
         }
         rho_s[idx] = rho; kap_s[idx] = kap; kb_s[idx] = kap * Bt; wc_s[idx] = w_r * Ct;
         A_s[idx] = A; u_s[idx] = u; ww_s[idx] = w_w; wr_s[idx] = w_r; Bq[idx] = Bt; Cq[idx] = Ct;
+        s_s[m * kN1BQ + t] = kap * Bt * u;
         XG[idx] = 0.f; YS[idx] = 0.f;
     }
     for (int idx = tid; idx < kN1BQ * Q1; idx += blockDim.x) H[idx] = 0.f;
+    if (tid < kN1BQ) {  // E as an unevaluated float pair: pair differences without FP64
+        const double Ev = tid < n ? E_s[tid] : 0.0;
+        const float hi = float(Ev);
+        Ef_s[tid] = make_float2(hi, float(Ev - double(hi)));
+    }
     if constexpr (VEC) asm volatile("cp.async.wait_all;" ::: "memory");
     __syncthreads();
 
@@ -1503,7 +1513,8 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
     // ---- P2: pair passes, one warp per group of four modes (KP / 4 warps).  Row pass (lane =
     // row t): Gamma row, Gamma' o H row (rect), intra dw_read-like sums; column pass (lane = k):
     // intra dkappa B-like sums.  Gamma and Gamma' o H add up over the mode groups.
-    for (int idx = tid; idx < kN1BQ * Q1; idx += blockDim.x) Gm[idx] = XR[idx] = 0.f;
+    for (int idx = tid; idx < kN1BQ * kGS; idx += blockDim.x) Gm[idx] = 0.f;
+    for (int idx = tid; idx < kN1BQ * Q1; idx += blockDim.x) XR[idx] = 0.f;
     __syncthreads();
     {
         const int w = tid >> 5, lane = tid & 31;
@@ -1513,8 +1524,10 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
                 const int t = lane;
                 float dw[4] = {0.f, 0.f, 0.f, 0.f};
                 if (t < n) {
+                    const float2 Et = Ef_s[t];
                     for (int k = 0; k <= t; ++k) {
-                        const float dE = float(E_s[t] - E_s[k]);
+                        const float2 Ek = Ef_s[k];
+                        const float dE = (Et.x - Ek.x) + (Et.y - Ek.y);
                         const float hv = H[t * Q1 + k];
                         float gam = 0.f, gamt = 0.f;
 #pragma unroll
@@ -1529,7 +1542,7 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
                                 dw[j] = fmaf(kw, hv, dw[j]);
                             }
                         }
-                        atomicAdd(&Gm[t * Q1 + k], gam);
+                        atomicAdd(&Gm[t * kGS + k], gam);
                         atomicAdd(&XR[t * Q1 + k], gamt * hv);
                     }
                 }
@@ -1541,8 +1554,10 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
                 const int k = lane;
                 float dk[4] = {0.f, 0.f, 0.f, 0.f};
                 if (k < n) {
+                    const float2 Ek = Ef_s[k];
                     for (int t = k; t < n; ++t) {
-                        const float dE = float(E_s[t] - E_s[k]);
+                        const float2 Et = Ef_s[t];
+                        const float dE = (Et.x - Ek.x) + (Et.y - Ek.y);
                         const float hv = H[t * Q1 + k];
 #pragma unroll
                         for (int j = 0; j < 4; ++j) {
@@ -1577,26 +1592,44 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
     }
 
     // ---- P4: dx[k][p] = sum_m s_{k,m} gamma_m[p] + sum_{t>=k} Gamma[t][k] dy_t[p] + D dy_k[p]
-    // (one thread per p; the dy column and gamma of the thread's p in registers)
+    // (one thread per p).  Gamma is zero above the diagonal and on rows past the chunk's end, so
+    // every row adds to all 32 accumulators, read as 16-byte broadcast pieces.
     const float Dh = Dv[h];
     float ddv = 0.f;  // sum dy x for dD
     for (int q = tid; q < P; q += blockDim.x) {
-        float dyc[kN1BQ], gv[KP];
+        float acc[kN1BQ];
 #pragma unroll
-        for (int t = 0; t < kN1BQ; ++t) dyc[t] = t < Q ? to_f(dys[t * P + q]) : 0.f;
+        for (int k = 0; k < kN1BQ; ++k) acc[k] = 0.f;
+#pragma unroll 1
+        for (int t = 0; t < n; ++t) {
+            const float dv = to_f(dys[t * P + q]);
+            ddv = fmaf(dv, to_f(xs[t * P + q]), ddv);
+            const float4 *g4 = reinterpret_cast<const float4 *>(Gm + t * kGS);
 #pragma unroll
-        for (int m = 0; m < KP; ++m) gv[m] = m < K ? Gam[m * P + q] : 0.f;
-        for (int k = 0; k < n; ++k) {
-            float acc = Dh * dyc[k];
-#pragma unroll
-            for (int m = 0; m < KP; ++m)
-                if (m < K) acc = fmaf(kb_s[k * K + m] * u_s[k * K + m], gv[m], acc);
-#pragma unroll
-            for (int t = 0; t < kN1BQ; ++t)
-                if (t >= k && t < n) acc = fmaf(Gm[t * Q1 + k], dyc[t], acc);
-            dx[blh(d, b, c0 + k, h) * P + q] = from_f<T>(acc);
-            ddv = fmaf(dyc[k], to_f(xs[k * P + q]), ddv);
+            for (int k4 = 0; k4 < kN1BQ / 4; ++k4) {
+                const float4 gv = g4[k4];
+                acc[4 * k4] = fmaf(gv.x, dv, acc[4 * k4]);
+                acc[4 * k4 + 1] = fmaf(gv.y, dv, acc[4 * k4 + 1]);
+                acc[4 * k4 + 2] = fmaf(gv.z, dv, acc[4 * k4 + 2]);
+                acc[4 * k4 + 3] = fmaf(gv.w, dv, acc[4 * k4 + 3]);
+            }
         }
+#pragma unroll 1
+        for (int m = 0; m < K; ++m) {
+            const float gv = Gam[m * P + q];
+            const float4 *s4 = reinterpret_cast<const float4 *>(s_s + m * kN1BQ);
+#pragma unroll
+            for (int k4 = 0; k4 < kN1BQ / 4; ++k4) {
+                const float4 sv = s4[k4];
+                acc[4 * k4] = fmaf(sv.x, gv, acc[4 * k4]);
+                acc[4 * k4 + 1] = fmaf(sv.y, gv, acc[4 * k4 + 1]);
+                acc[4 * k4 + 2] = fmaf(sv.z, gv, acc[4 * k4 + 2]);
+                acc[4 * k4 + 3] = fmaf(sv.w, gv, acc[4 * k4 + 3]);
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < kN1BQ; ++k)
+            if (k < n) dx[blh(d, b, c0 + k, h) * P + q] = from_f<T>(fmaf(Dh, to_f(dys[k * P + q]), acc[k]));
     }
     ddv = block_sum(ddv, red);  // contains __syncthreads (also publishes rp_s)
     if (tid == 0) atomicAdd(&dD[h], ddv);
