@@ -1510,65 +1510,97 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
     }
     __syncthreads();
 
-    // ---- P2: pair passes, one warp per group of four modes (KP / 4 warps).  Row pass (lane =
-    // row t): Gamma row, Gamma' o H row (rect), intra dw_read-like sums; column pass (lane = k):
-    // intra dkappa B-like sums.  Gamma and Gamma' o H add up over the mode groups.
+    // ---- P2: pair passes, one thread per (row, mode): 32 / KP rows per warp, the lanes of a row
+    // on consecutive modes; row groups go to the warps in snake order (long rows with short ones).
+    // Row pass (thread = (t, m)): the intra dw_read-like sums, and Gamma and Gamma' o H, which the
+    // row's lanes sum over the modes four columns at a time by halving exchanges; column pass
+    // (thread = (k, m)): the intra dkappa B-like sums.  Every entry has one writer (no atomics).
     for (int idx = tid; idx < kN1BQ * kGS; idx += blockDim.x) Gm[idx] = 0.f;
     for (int idx = tid; idx < kN1BQ * Q1; idx += blockDim.x) XR[idx] = 0.f;
     __syncthreads();
     {
-        const int w = tid >> 5, lane = tid & 31;
-        if (w < KP / 4 && lane < Q) {
-            const int m0 = 4 * w;
-            {  // row pass
-                const int t = lane;
-                float dw[4] = {0.f, 0.f, 0.f, 0.f};
-                if (t < n) {
-                    const float2 Et = Ef_s[t];
-                    for (int k = 0; k <= t; ++k) {
+        constexpr int RPW = 32 / KP;
+        constexpr int kCnt = KP >= 8 ? 1 : 8 / KP;    // values a lane holds after the exchanges
+        constexpr int kDup = KP >= 8 ? KP / 8 - 1 : 0; // lane bits that hold copies of one value
+        const int w = tid >> 5, lane = tid & 31, nw = blockDim.x >> 5;
+        const int m = lane % KP, sub = lane / KP;
+        const bool mok = m < K;
+        const float itm = mok ? itau[m] : 0.f;
+        const int ngrp = (n + RPW - 1) / RPW;
+        for (int pass = 0; pass * nw < ngrp; ++pass) {  // row pass
+            const int gi = pass * nw + ((pass & 1) ? nw - 1 - w : w);
+            if (gi >= ngrp) continue;  // warp-uniform
+            const int t = gi * RPW + sub;
+            const int tlast = min(gi * RPW + RPW - 1, n - 1);  // warp-uniform
+            const bool live = t < n && mok;
+            const float wct = live ? wc_s[t * K + m] : 0.f;
+            const float2 Et = Ef_s[t];
+            float dw = 0.f;
+            for (int k0 = 0; k0 <= tlast; k0 += 4) {
+                float v[8];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const int k = k0 + j;
+                    float a = 0.f, hv = 0.f;
+                    if (live && k <= t) {
                         const float2 Ek = Ef_s[k];
                         const float dE = (Et.x - Ek.x) + (Et.y - Ek.y);
-                        const float hv = H[t * Q1 + k];
-                        float gam = 0.f, gamt = 0.f;
+                        const float kw = kb_s[k * K + m] * expf(-dE * itm);
+                        hv = H[t * Q1 + k];
+                        a = wct * kw;
+                        dw = fmaf(kw, hv, dw);
+                    }
+                    v[j] = a;
+                    v[4 + j] = a * itm * hv;
+                }
+                // halving exchanges over the row's KP lanes: at offset o a lane keeps the half of
+                // its values picked by bit o of its lane index and adds its partner's copy of it
+                int cnt = 8, base = 0;
 #pragma unroll
-                        for (int j = 0; j < 4; ++j) {
-                            const int m = m0 + j;
-                            if (m < K) {
-                                const float W = expf(-dE * itau[m]);
-                                const float kw = kb_s[k * K + m] * W;
-                                const float a = wc_s[t * K + m] * kw;
-                                gam += a;
-                                gamt = fmaf(a, itau[m], gamt);
-                                dw[j] = fmaf(kw, hv, dw[j]);
+                for (int o = KP / 2; o >= 1; o >>= 1) {
+                    if (cnt > 1) {
+                        const int half = cnt / 2;
+                        const bool up = (lane & o) != 0;
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            if (i < half) {
+                                const float send = up ? v[i] : v[i + half];
+                                const float keep = up ? v[i + half] : v[i];
+                                v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
                             }
                         }
-                        atomicAdd(&Gm[t * kGS + k], gam);
-                        atomicAdd(&XR[t * Q1 + k], gamt * hv);
+                        if (up) base += half;
+                        cnt = half;
+                    } else {
+                        v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
                     }
                 }
+                if (t < n && (lane & kDup) == 0) {
 #pragma unroll
-                for (int j = 0; j < 4; ++j)
-                    if (m0 + j < K) dwci[t * K + m0 + j] = dw[j];
-            }
-            {  // column pass
-                const int k = lane;
-                float dk[4] = {0.f, 0.f, 0.f, 0.f};
-                if (k < n) {
-                    const float2 Ek = Ef_s[k];
-                    for (int t = k; t < n; ++t) {
-                        const float2 Et = Ef_s[t];
-                        const float dE = (Et.x - Ek.x) + (Et.y - Ek.y);
-                        const float hv = H[t * Q1 + k];
-#pragma unroll
-                        for (int j = 0; j < 4; ++j) {
-                            const int m = m0 + j;
-                            if (m < K) dk[j] = fmaf(wc_s[t * K + m] * expf(-dE * itau[m]), hv, dk[j]);
+                    for (int i = 0; i < kCnt; ++i) {
+                        const int vi = base + i, k = k0 + (vi & 3);
+                        if (k <= t) {
+                            if (vi < 4) Gm[t * kGS + k] = v[i];
+                            else XR[t * Q1 + k] = v[i];
                         }
                     }
                 }
-#pragma unroll
-                for (int j = 0; j < 4; ++j)
-                    if (m0 + j < K) dkbi[k * K + m0 + j] = dk[j];
+            }
+            if (live) dwci[t * K + m] = dw;
+        }
+        for (int pass = 0; pass * nw < ngrp; ++pass) {  // column pass
+            const int gi = pass * nw + ((pass & 1) ? nw - 1 - w : w);
+            if (gi >= ngrp) continue;
+            const int k = gi * RPW + sub;
+            if (k < n && mok) {
+                const float2 Ek = Ef_s[k];
+                float dk = 0.f;
+                for (int t = k; t < n; ++t) {
+                    const float2 Et = Ef_s[t];
+                    const float dE = (Et.x - Ek.x) + (Et.y - Ek.y);
+                    dk = fmaf(wc_s[t * K + m] * expf(-dE * itm), H[t * Q1 + k], dk);
+                }
+                dkbi[k * K + m] = dk;
             }
         }
     }
