@@ -356,7 +356,7 @@ frac_status frac_scan_bwd(const frac_dims *d, const void *x, const float *dt, co
             e = frac::tc_scan_bwd(sd, p, t, reinterpret_cast<int *>(ws), reuse, st);
         } else {
             e = frac::simt_scan_bwd(sd, d->dtype, p, ws + l.s_in, ws + l.ds_out, dB_acc, dC_acc,
-                                    reinterpret_cast<float *>(ws + l.n1), reuse, st);
+                                    reinterpret_cast<float *>(ws + l.n1), reuse, reinterpret_cast<int *>(ws), st);
         }
     }
     return cuda_status(e, "frac_scan_bwd");

@@ -53,9 +53,10 @@ cudaError_t simt_scan_fwd(const ScanDims &d, int dtype, const ScanPtrs &p, void 
                           cudaStream_t st);
 // reuse_states: S_in already holds the forward's per-chunk states (no recompute)
 // n1_scratch: simt_n1_scratch_elems floats (the N = 1 backward's chunk carries)
+// err: the call's device status word (a kernel whose bounded wait gave up writes FRAC_ERR_TIMEOUT)
 cudaError_t simt_scan_bwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in,
                           void *dS_out, float *dB_acc, float *dC_acc, float *n1_scratch,
-                          bool reuse_states, cudaStream_t st);
+                          bool reuse_states, int *err, cudaStream_t st);
 
 // Tensor-core (tcgen05) path: bf16 inputs, chunk 128, P = 64, N in {64, 128}, K in {4, 8}.
 bool tc_supported(const ScanDims &d, int dtype);

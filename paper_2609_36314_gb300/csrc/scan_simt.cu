@@ -23,6 +23,7 @@
 
 #include "common.cuh"
 #include "kernels.h"
+#include "tc.cuh"
 
 namespace frac {
 namespace {
@@ -1283,6 +1284,7 @@ __global__ void __launch_bounds__(256) n1_combine_rev(ScanDims d, const float *_
 }
 
 constexpr int kN1BQ = 32;  // chunk of the N = 1 backward (shared-memory tiles [Q][P])
+constexpr int kN1Timeout = 4;  // FRAC_ERR_TIMEOUT in the call's status word
 constexpr int kGS = 36;    // row stride of its Gamma tile (rows read as 16-byte pieces)
 
 struct N1BwdSmem {
@@ -1311,6 +1313,243 @@ struct N1BwdSmem {
     }
 };
 
+// The [Q][K] float arrays of the N = 1 gradient kernels (shared memory): per-(position, mode)
+// coefficients, then the dot products over p and the pair sums.
+struct N1Arrays {
+    float *rho, *kap, *kb, *wc, *A, *u, *ww, *wr, *XG, *YS, *dwci, *dkbi, *Bq, *Cq;
+    float *s;  // kappa B u, mode-major [K][Q]
+    __device__ N1Arrays(float *qk, int K) {
+        const int QK = kN1BQ * K;
+        rho = qk; kap = qk + QK; kb = qk + 2 * QK; wc = qk + 3 * QK; A = qk + 4 * QK; u = qk + 5 * QK;
+        ww = qk + 6 * QK; wr = qk + 7 * QK; XG = qk + 8 * QK; YS = qk + 9 * QK; dwci = qk + 10 * QK;
+        dkbi = qk + 11 * QK; Bq = qk + 12 * QK; Cq = qk + 13 * QK; s = qk + 14 * QK;
+    }
+};
+
+// Per-(position, mode) coefficients of one chunk: rho = exp(-e/tau), kappa = -expm1(-e/tau) w_write,
+// kappa B, w_read C, A = exp(-E_t/tau) (entering state to position t), u = exp(-(E_end - E_t)/tau)
+// (position t to the chunk's end) and s = kappa B u; zeros past the chunk's end.
+template <typename T>
+__device__ __forceinline__ void n1_bwd_coefs(const ScanDims &d, int b, int h, int g, int c0, int n, double Eend,
+                                             const float *itau, const float *e_s, const double *E_s,
+                                             const T *__restrict__ ww, const T *__restrict__ wr,
+                                             const T *__restrict__ Bm, const T *__restrict__ Cm, const N1Arrays &a) {
+    const int K = d.K;
+    for (int idx = threadIdx.x; idx < kN1BQ * K; idx += blockDim.x) {
+        const int t = idx / K, m = idx - t * K;
+        float rho = 0.f, kap = 0.f, A = 0.f, u = 0.f, w_w = 0.f, w_r = 0.f, Bt = 0.f, Ct = 0.f;
+        if (t < n) {
+            const size_t wi = blh(d, b, c0 + t, h) * K + m;
+            const size_t gi = (size_t(b) * d.L + c0 + t) * d.G + g;
+            w_w = to_f(ww[wi]);
+            w_r = to_f(wr[wi]);
+            Bt = to_f(Bm[gi]);
+            Ct = to_f(Cm[gi]);
+            const float z = e_s[t] * itau[m];
+            rho = expf(-z);
+            kap = -expm1f(-z) * w_w;
+            A = expf(-float(E_s[t]) * itau[m]);
+            u = expf(-float(Eend - E_s[t]) * itau[m]);
+        }
+        a.rho[idx] = rho; a.kap[idx] = kap; a.kb[idx] = kap * Bt; a.wc[idx] = w_r * Ct;
+        a.A[idx] = A; a.u[idx] = u; a.ww[idx] = w_w; a.wr[idx] = w_r; a.Bq[idx] = Bt; a.Cq[idx] = Ct;
+        a.s[m * kN1BQ + t] = kap * Bt * u;
+        a.XG[idx] = 0.f; a.YS[idx] = 0.f;
+    }
+}
+
+// Pair passes over k <= t for every mode, one thread per (row, mode): 32 / KP rows per warp, the
+// lanes of a row on consecutive modes; row groups go to the warps in snake order (long rows with
+// short ones).  Row pass (thread = (t, m)): the intra dw_read-like sums, and Gamma and
+// Gamma' o H, which the row's lanes sum over the modes four columns at a time by halving
+// exchanges; put(t, k, Gamma_tk) stores Gamma, XR takes Gamma' o H.  Column pass (thread =
+// (k, m)): the intra dkappa B-like sums.  Every entry has one writer (no atomics).
+template <int KP, typename PutGamma>
+__device__ __forceinline__ void n1_pair_passes(int n, int K, const float *itau, const float2 *Ef_s,
+                                               const N1Arrays &a, const float *H, float *XR, PutGamma put) {
+    constexpr int Q1 = kN1BQ + 1;
+    constexpr int RPW = 32 / KP;
+    constexpr int kCnt = KP >= 8 ? 1 : 8 / KP;    // values a lane holds after the exchanges
+    constexpr int kDup = KP >= 8 ? KP / 8 - 1 : 0; // lane bits that hold copies of one value
+    const int tid = threadIdx.x, w = tid >> 5, lane = tid & 31, nw = blockDim.x >> 5;
+    const int m = lane % KP, sub = lane / KP;
+    const bool mok = m < K;
+    const float itm = mok ? itau[m] : 0.f;
+    const int ngrp = (n + RPW - 1) / RPW;
+    for (int pass = 0; pass * nw < ngrp; ++pass) {  // row pass
+        const int gi = pass * nw + ((pass & 1) ? nw - 1 - w : w);
+        if (gi >= ngrp) continue;  // warp-uniform
+        const int t = gi * RPW + sub;
+        const int tlast = min(gi * RPW + RPW - 1, n - 1);  // warp-uniform
+        const bool live = t < n && mok;
+        const float wct = live ? a.wc[t * K + m] : 0.f;
+        const float2 Et = Ef_s[t];
+        float dw = 0.f;
+        for (int k0 = 0; k0 <= tlast; k0 += 4) {
+            float v[8];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int k = k0 + j;
+                float av = 0.f, hv = 0.f;
+                if (live && k <= t) {
+                    const float2 Ek = Ef_s[k];
+                    const float dE = (Et.x - Ek.x) + (Et.y - Ek.y);
+                    const float kw = a.kb[k * K + m] * expf(-dE * itm);
+                    hv = H[t * Q1 + k];
+                    av = wct * kw;
+                    dw = fmaf(kw, hv, dw);
+                }
+                v[j] = av;
+                v[4 + j] = av * itm * hv;
+            }
+            // halving exchanges over the row's KP lanes: at offset o a lane keeps the half of
+            // its values picked by bit o of its lane index and adds its partner's copy of it
+            int cnt = 8, base = 0;
+#pragma unroll
+            for (int o = KP / 2; o >= 1; o >>= 1) {
+                if (cnt > 1) {
+                    const int half = cnt / 2;
+                    const bool up = (lane & o) != 0;
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        if (i < half) {
+                            const float send = up ? v[i] : v[i + half];
+                            const float keep = up ? v[i + half] : v[i];
+                            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+                        }
+                    }
+                    if (up) base += half;
+                    cnt = half;
+                } else {
+                    v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
+                }
+            }
+            if (t < n && (lane & kDup) == 0) {
+#pragma unroll
+                for (int i = 0; i < kCnt; ++i) {
+                    const int vi = base + i, k = k0 + (vi & 3);
+                    if (k <= t) {
+                        if (vi < 4) put(t, k, v[i]);
+                        else XR[t * Q1 + k] = v[i];
+                    }
+                }
+            }
+        }
+        if (live) a.dwci[t * K + m] = dw;
+    }
+    for (int pass = 0; pass * nw < ngrp; ++pass) {  // column pass
+        const int gi = pass * nw + ((pass & 1) ? nw - 1 - w : w);
+        if (gi >= ngrp) continue;
+        const int k = gi * RPW + sub;
+        if (k < n && mok) {
+            const float2 Ek = Ef_s[k];
+            float dk = 0.f;
+            for (int t = k; t < n; ++t) {
+                const float2 Et = Ef_s[t];
+                const float dE = (Et.x - Ek.x) + (Et.y - Ek.y);
+                dk = fmaf(a.wc[t * K + m] * expf(-dE * itm), H[t * Q1 + k], dk);
+            }
+            a.dkbi[k * K + m] = dk;
+        }
+    }
+}
+
+// Rectangle sums of Gamma' o H over pairs k < t <= t': XR rows become exclusive row prefixes,
+// then rp_s[t] = sum over t' >= t of row t' at column t.  Ends before the column sums are
+// published (the caller synchronises).
+__device__ __forceinline__ void n1_rect(int n, int Q, float *XR, float *rp_s) {
+    constexpr int Q1 = kN1BQ + 1;
+    const int tid = threadIdx.x;
+    if (tid < Q) {
+        float run = 0.f;
+        for (int j = 0; j < Q; ++j) {
+            const float v = XR[tid * Q1 + j];
+            XR[tid * Q1 + j] = run;
+            run += v;
+        }
+    }
+    __syncthreads();
+    if (tid < Q) {
+        float s = 0.f;
+        for (int tp = tid; tp < n; ++tp) s += XR[tp * Q1 + tid];
+        rp_s[tid] = s;
+    }
+}
+
+// Per-position gradients of one chunk.  a_t / b_k are the S_in / gamma terms of
+// sum_m rho <g_t, S_{t-1}>_m / tau_m (suffix and exclusive prefix sums), c the <gamma, S_in>
+// term, rp_s the pairs; then dDelta, dalpha, dlambda, the mode weights, dB, dC and (when asked)
+// the inter-chunk and per-position terms of dtau.  scratch: 128 floats no longer in use.
+template <typename T>
+__device__ __forceinline__ void n1_position_grads(
+    const ScanDims &d, int b, int h, int g, int c0, int n, double Eend, const N1Arrays &a, const float *itau,
+    const float *e_s, const double *E_s, const float *cl_s, const float *cdot, const float *rp_s, float *scratch,
+    float *dtq, const float *__restrict__ dt, const float *__restrict__ alpha, const float *__restrict__ lam,
+    T *__restrict__ dwr_o, T *__restrict__ dww_o, float *__restrict__ ddt, float *__restrict__ dalpha,
+    float *__restrict__ dlam, float *__restrict__ dB_acc, float *__restrict__ dC_acc, float *__restrict__ dtau) {
+    const int K = d.K, tid = threadIdx.x;
+    float *a_s = scratch, *b_s = scratch + 64;
+    if (tid < n) {
+        const int t = tid;
+        float av = 0.f, bv = 0.f;
+        for (int m = 0; m < K; ++m) {
+            const int q = t * K + m;
+            av = fmaf(a.wc[q] * a.A[q] * a.YS[q], itau[m], av);
+            bv = fmaf(a.kb[q] * a.u[q] * a.XG[q], itau[m], bv);
+        }
+        a_s[t] = av;
+        b_s[t] = bv;
+    }
+    __syncthreads();
+    float cprime = 0.f;
+    for (int m = 0; m < K; ++m) cprime = fmaf(expf(-float(Eend) * itau[m]) * itau[m], cdot[m], cprime);
+    if (tid < n) {
+        const int t = tid;
+        float suf = 0.f, pre = 0.f;
+        for (int j = t; j < n; ++j) suf += a_s[j];
+        for (int j = 0; j < t; ++j) pre += b_s[j];
+        const float R = suf + pre + cprime + rp_s[t];
+        float de = -R, sB = 0.f, sC = 0.f;
+        const size_t i = blh(d, b, c0 + t, h);
+        for (int m = 0; m < K; ++m) {
+            const int q = t * K + m;
+            const float dkb = a.u[q] * a.XG[q] + a.dkbi[q];  // d(kappa B)
+            const float dwc = a.A[q] * a.YS[q] + a.dwci[q];  // d(w_read C)
+            const float dk = dkb * a.Bq[q];                  // d kappa
+            de = fmaf(dk * a.rho[q] * a.ww[q], itau[m], de);
+            dwr_o[i * K + m] = from_f<T>(dwc * a.Cq[q]);
+            dww_o[i * K + m] = from_f<T>(dk * (-expm1f(-e_s[t] * itau[m])));
+            sB = fmaf(dkb, a.kap[q], sB);
+            sC = fmaf(dwc, a.wr[q], sC);
+            if (dtau) {
+                const double Et = E_s[t];
+                const double tq = Et * double(a.wc[q] * a.A[q] * a.YS[q]) +
+                                  (Eend - Et) * double(a.kb[q] * a.u[q] * a.XG[q]) -
+                                  double(e_s[t]) * double(dk) * double(a.rho[q]) * double(a.ww[q]);
+                atomicAdd(&dtq[m], float(tq));
+            }
+        }
+        const size_t gi = (size_t(b) * d.L + c0 + t) * d.G + g;
+        atomicAdd(&dB_acc[gi], sB);
+        atomicAdd(&dC_acc[gi], sC);
+        const float e = e_s[t];
+        const bool cl = cl_s[t] != 0.f;
+        const float al = alpha[i], lm = lam[i], dtv = dt[i];
+        const float ge = cl ? 0.f : de * e;
+        ddt[i] = ge / dtv;
+        dlam[i] = ge / (al * lm);
+        dalpha[i] = -ge * logf(lm) / (al * al);
+    }
+    if (dtau) {
+        __syncthreads();
+        if (tid < K) {
+            const float it = itau[tid];
+            const float chunk_term = float(Eend) * expf(-float(Eend) * it) * cdot[tid];
+            atomicAdd(&dtau[h * K + tid], (dtq[tid] + chunk_term) * it * it);
+        }
+    }
+}
+
 // Gradients of one chunk of one head (one CTA, 256 threads; Q <= 32, all of P).
 template <typename T, typename TS, bool VEC, int KP>
 __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
@@ -1331,12 +1570,8 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
     float *cdot = reinterpret_cast<float *>(sm_raw + L_.cdot);
     float *dtq = reinterpret_cast<float *>(sm_raw + L_.dtq);
     float *qk = reinterpret_cast<float *>(sm_raw + L_.qk);
-    const int QK = kN1BQ * K;
-    // [Q][K] arrays: coefficients, then the dot products and pair sums
-    float *rho_s = qk, *kap_s = qk + QK, *kb_s = qk + 2 * QK, *wc_s = qk + 3 * QK, *A_s = qk + 4 * QK,
-          *u_s = qk + 5 * QK, *ww_s = qk + 6 * QK, *wr_s = qk + 7 * QK, *XG = qk + 8 * QK, *YS = qk + 9 * QK,
-          *dwci = qk + 10 * QK, *dkbi = qk + 11 * QK, *Bq = qk + 12 * QK, *Cq = qk + 13 * QK,
-          *s_s = qk + 14 * QK;  // kappa B u, mode-major [K][Q]
+    const N1Arrays a(qk, K);
+    float *XG = a.XG, *YS = a.YS, *s_s = a.s;
     T *xs = reinterpret_cast<T *>(sm_raw + L_.x), *dys = reinterpret_cast<T *>(sm_raw + L_.y);
     float *Sin = reinterpret_cast<float *>(sm_raw + L_.sin), *Gam = reinterpret_cast<float *>(sm_raw + L_.gam);
     float *H = reinterpret_cast<float *>(sm_raw + L_.H), *Gm = reinterpret_cast<float *>(sm_raw + L_.Gm);
@@ -1384,27 +1619,7 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
     chunk_rates(d, b, h, c0, n, log_cap, dt, alpha, lam, e_s, E_s, cl_s);
     __syncthreads();
     const double Eend = E_s[n - 1];
-    for (int idx = tid; idx < QK; idx += blockDim.x) {
-        const int t = idx / K, m = idx - t * K;
-        float rho = 0.f, kap = 0.f, A = 0.f, u = 0.f, w_w = 0.f, w_r = 0.f, Bt = 0.f, Ct = 0.f;
-        if (t < n) {
-            const size_t wi = blh(d, b, c0 + t, h) * K + m;
-            const size_t gi = (size_t(b) * d.L + c0 + t) * d.G + g;
-            w_w = to_f(ww[wi]);
-            w_r = to_f(wr[wi]);
-            Bt = to_f(Bm[gi]);
-            Ct = to_f(Cm[gi]);
-            const float z = e_s[t] * itau[m];
-            rho = expf(-z);
-            kap = -expm1f(-z) * w_w;
-            A = expf(-float(E_s[t]) * itau[m]);
-            u = expf(-float(Eend - E_s[t]) * itau[m]);
-        }
-        rho_s[idx] = rho; kap_s[idx] = kap; kb_s[idx] = kap * Bt; wc_s[idx] = w_r * Ct;
-        A_s[idx] = A; u_s[idx] = u; ww_s[idx] = w_w; wr_s[idx] = w_r; Bq[idx] = Bt; Cq[idx] = Ct;
-        s_s[m * kN1BQ + t] = kap * Bt * u;
-        XG[idx] = 0.f; YS[idx] = 0.f;
-    }
+    n1_bwd_coefs<T>(d, b, h, g, c0, n, Eend, itau, e_s, E_s, ww, wr, Bm, Cm, a);
     for (int idx = tid; idx < kN1BQ * Q1; idx += blockDim.x) H[idx] = 0.f;
     if (tid < kN1BQ) {  // E as an unevaluated float pair: pair differences without FP64
         const double Ev = tid < n ? E_s[tid] : 0.0;
@@ -1510,118 +1725,16 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
     }
     __syncthreads();
 
-    // ---- P2: pair passes, one thread per (row, mode): 32 / KP rows per warp, the lanes of a row
-    // on consecutive modes; row groups go to the warps in snake order (long rows with short ones).
-    // Row pass (thread = (t, m)): the intra dw_read-like sums, and Gamma and Gamma' o H, which the
-    // row's lanes sum over the modes four columns at a time by halving exchanges; column pass
-    // (thread = (k, m)): the intra dkappa B-like sums.  Every entry has one writer (no atomics).
+    // ---- P2: pair passes (n1_pair_passes); Gamma into the row-major Gm tile
     for (int idx = tid; idx < kN1BQ * kGS; idx += blockDim.x) Gm[idx] = 0.f;
     for (int idx = tid; idx < kN1BQ * Q1; idx += blockDim.x) XR[idx] = 0.f;
     __syncthreads();
-    {
-        constexpr int RPW = 32 / KP;
-        constexpr int kCnt = KP >= 8 ? 1 : 8 / KP;    // values a lane holds after the exchanges
-        constexpr int kDup = KP >= 8 ? KP / 8 - 1 : 0; // lane bits that hold copies of one value
-        const int w = tid >> 5, lane = tid & 31, nw = blockDim.x >> 5;
-        const int m = lane % KP, sub = lane / KP;
-        const bool mok = m < K;
-        const float itm = mok ? itau[m] : 0.f;
-        const int ngrp = (n + RPW - 1) / RPW;
-        for (int pass = 0; pass * nw < ngrp; ++pass) {  // row pass
-            const int gi = pass * nw + ((pass & 1) ? nw - 1 - w : w);
-            if (gi >= ngrp) continue;  // warp-uniform
-            const int t = gi * RPW + sub;
-            const int tlast = min(gi * RPW + RPW - 1, n - 1);  // warp-uniform
-            const bool live = t < n && mok;
-            const float wct = live ? wc_s[t * K + m] : 0.f;
-            const float2 Et = Ef_s[t];
-            float dw = 0.f;
-            for (int k0 = 0; k0 <= tlast; k0 += 4) {
-                float v[8];
-#pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    const int k = k0 + j;
-                    float a = 0.f, hv = 0.f;
-                    if (live && k <= t) {
-                        const float2 Ek = Ef_s[k];
-                        const float dE = (Et.x - Ek.x) + (Et.y - Ek.y);
-                        const float kw = kb_s[k * K + m] * expf(-dE * itm);
-                        hv = H[t * Q1 + k];
-                        a = wct * kw;
-                        dw = fmaf(kw, hv, dw);
-                    }
-                    v[j] = a;
-                    v[4 + j] = a * itm * hv;
-                }
-                // halving exchanges over the row's KP lanes: at offset o a lane keeps the half of
-                // its values picked by bit o of its lane index and adds its partner's copy of it
-                int cnt = 8, base = 0;
-#pragma unroll
-                for (int o = KP / 2; o >= 1; o >>= 1) {
-                    if (cnt > 1) {
-                        const int half = cnt / 2;
-                        const bool up = (lane & o) != 0;
-#pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            if (i < half) {
-                                const float send = up ? v[i] : v[i + half];
-                                const float keep = up ? v[i + half] : v[i];
-                                v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
-                            }
-                        }
-                        if (up) base += half;
-                        cnt = half;
-                    } else {
-                        v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
-                    }
-                }
-                if (t < n && (lane & kDup) == 0) {
-#pragma unroll
-                    for (int i = 0; i < kCnt; ++i) {
-                        const int vi = base + i, k = k0 + (vi & 3);
-                        if (k <= t) {
-                            if (vi < 4) Gm[t * kGS + k] = v[i];
-                            else XR[t * Q1 + k] = v[i];
-                        }
-                    }
-                }
-            }
-            if (live) dwci[t * K + m] = dw;
-        }
-        for (int pass = 0; pass * nw < ngrp; ++pass) {  // column pass
-            const int gi = pass * nw + ((pass & 1) ? nw - 1 - w : w);
-            if (gi >= ngrp) continue;
-            const int k = gi * RPW + sub;
-            if (k < n && mok) {
-                const float2 Ek = Ef_s[k];
-                float dk = 0.f;
-                for (int t = k; t < n; ++t) {
-                    const float2 Et = Ef_s[t];
-                    const float dE = (Et.x - Ek.x) + (Et.y - Ek.y);
-                    dk = fmaf(wc_s[t * K + m] * expf(-dE * itm), H[t * Q1 + k], dk);
-                }
-                dkbi[k * K + m] = dk;
-            }
-        }
-    }
+    n1_pair_passes<KP>(n, K, itau, Ef_s, a, H, XR, [&](int t, int k, float v) { Gm[t * kGS + k] = v; });
     __syncthreads();
 
     // ---- P3: rectangle sums of Gamma' o H over pairs k < t <= t' (row prefix, column suffix)
     float *rp_s = red + 32;  // [Q <= 32] (block_sum below uses red[0 .. 8))
-    if (tid < Q) {
-        float run = 0.f;
-        for (int j = 0; j < Q; ++j) {
-            const float v = XR[tid * Q1 + j];
-            XR[tid * Q1 + j] = run;
-            run += v;
-        }
-    }
-    __syncthreads();
-    if (tid < Q) {
-        float s = 0.f;
-        for (int tp = tid; tp < n; ++tp) s += XR[tp * Q1 + tid];
-        rp_s[tid] = s;
-    }
+    n1_rect(n, Q, XR, rp_s);
 
     // ---- P4: dx[k][p] = sum_m s_{k,m} gamma_m[p] + sum_{t>=k} Gamma[t][k] dy_t[p] + D dy_k[p]
     // (one thread per p).  Gamma is zero above the diagonal and on rows past the chunk's end, so
@@ -1666,68 +1779,272 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
     ddv = block_sum(ddv, red);  // contains __syncthreads (also publishes rp_s)
     if (tid == 0) atomicAdd(&dD[h], ddv);
 
-    // ---- P5: per-position scalars.  a_t / b_k are the S_in / gamma terms of
-    // sum_m rho <g_t, S_{t-1}>_m / tau_m (suffix and exclusive prefix sums), c the
-    // <gamma, S_in> term, rp_s the pairs; then dDelta, dalpha, dlambda, the weights, dB, dC.
-    float *a_s = XR, *b_s = XR + 64;  // XR is free now
-    if (tid < n) {
-        const int t = tid;
-        float a = 0.f, bb = 0.f;
-        for (int m = 0; m < K; ++m) {
-            const int q = t * K + m;
-            a = fmaf(wc_s[q] * A_s[q] * YS[q], itau[m], a);
-            bb = fmaf(kb_s[q] * u_s[q] * XG[q], itau[m], bb);
+    // ---- P5: per-position scalars (XR is free now)
+    n1_position_grads<T>(d, b, h, g, c0, n, Eend, a, itau, e_s, E_s, cl_s, cdot, rp_s, XR, dtq, dt, alpha, lam,
+                         dwr_o, dww_o, ddt, dalpha, dlam, dB_acc, dC_acc, dtau);
+}
+
+// ----------------------------------------------------------------------------------------------
+// Tensor-core variant of the N = 1 gradient kernel (bf16 inputs and states, P a multiple of 128,
+// chunk 32).  The contractions over p and over positions run on tcgen05:
+//   P1: one M = 128 chain over K = p of the rows [dy (32) | x (32) | gamma (KS) | S_in (KS)] (A,
+//       from row 0) against the rows [x | gamma | S_in] (B, from row 32), K-major, gives in one
+//       accumulator H = dY X^T, YS = dY S_in^T, XG = X gamma^T and diag(gamma S_in^T); every
+//       product is of two bf16 values, so only the order of the fp32 sums differs.
+//   P4: dx^T = [dY ; gamma]^T [Gamma ; s^T] per 128 p: A is the same tiles read MN-major (M = p,
+//       K = position or mode), B the Gamma and s = kappa B u coefficients as bf16 hi + lo pairs
+//       (K doubled), so the fp32 coefficients keep ~16 mantissa bits.
+// The tiles arrive by TMA as 128-byte-swizzled 64-column panels of 64 + 2 KS rows (KS = 16 or 32
+// rows for the modes); the phases between stay on the CUDA cores (the shared functions above).
+struct N1BwdTcSmem {
+    size_t pan, bimg, E, Ef, e, cl, itau, red, cdot, dtq, qk, H, XR, bars, total;
+    uint32_t panel, bimg_rows;
+    int KS;
+    __host__ __device__ N1BwdTcSmem(int P, int K) {
+        KS = K <= 16 ? 16 : 32;
+        panel = uint32_t(64 + 2 * KS) * 128;                       // bytes of one 64-column panel
+        pan = 0;                                                   // [P / 64] panels (1024-aligned)
+        bimg = pan + size_t(P / 64) * panel;                       // B of P4: [2 (32 + KS)][128 B]
+        bimg_rows = uint32_t(2 * (32 + KS));
+        E = bimg + size_t(bimg_rows) * 128;                        // double [Q]
+        Ef = E + sizeof(double) * kN1BQ;                           // float2 [Q]
+        e = Ef + sizeof(float) * 2 * kN1BQ;                        // float [Q]
+        cl = e + sizeof(float) * kN1BQ;                            // float [Q]
+        itau = cl + sizeof(float) * kN1BQ;                         // float [32]
+        red = itau + sizeof(float) * 32;                           // float [64]
+        cdot = red + sizeof(float) * 64;                           // float [32]
+        dtq = cdot + sizeof(float) * 32;                           // float [32]
+        qk = dtq + sizeof(float) * 32;                             // float [15][Q][K]
+        H = qk + sizeof(float) * 15 * kN1BQ * K;                   // float [Q][Q + 1]
+        XR = H + sizeof(float) * kN1BQ * (kN1BQ + 1);              // float [Q][Q + 1]
+        bars = (XR + sizeof(float) * kN1BQ * (kN1BQ + 1) + 7) / 8 * 8;  // 3 mbarriers, TMEM slot
+        total = bars + 32 + 1024;                                  // + slack to align the base
+    }
+};
+// TMEM columns of the variant: P1's accumulator (32 + 2 KS) and P4's (64 per 128 p), reused.
+__host__ __device__ inline uint32_t n1_tc_tmem_cols(int P, int K) {
+    const uint32_t need = uint32_t(std::max(32 + 2 * (K <= 16 ? 16 : 32), P / 2));
+    uint32_t c = 32;
+    while (c < need) c <<= 1;
+    return c;
+}
+
+__device__ __forceinline__ void st_bf16_pair(unsigned char *img, uint32_t row_hi, uint32_t row_lo, uint32_t col,
+                                             float v) {
+    const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+    const __nv_bfloat16 lo = __float2bfloat16_rn(v - __bfloat162float(hi));
+    *reinterpret_cast<__nv_bfloat16 *>(img + tc::sw128_offset(row_hi, col)) = hi;
+    *reinterpret_cast<__nv_bfloat16 *>(img + tc::sw128_offset(row_lo, col)) = lo;
+}
+
+template <int KP>
+__global__ void __launch_bounds__(kThreads) n1_chunk_bwd_tc(
+    const __grid_constant__ CUtensorMap mapX, const __grid_constant__ CUtensorMap mapDY,
+    const __grid_constant__ CUtensorMap mapS, const __grid_constant__ CUtensorMap mapG, ScanDims d,
+    const __nv_bfloat16 *__restrict__ Bm, const __nv_bfloat16 *__restrict__ Cm,
+    const __nv_bfloat16 *__restrict__ wr, const __nv_bfloat16 *__restrict__ ww, const float *__restrict__ dt,
+    const float *__restrict__ alpha, const float *__restrict__ lam, const float *__restrict__ tau,
+    const float *__restrict__ Dv, __nv_bfloat16 *__restrict__ dx, __nv_bfloat16 *__restrict__ dwr_o,
+    __nv_bfloat16 *__restrict__ dww_o, float *__restrict__ ddt, float *__restrict__ dalpha,
+    float *__restrict__ dlam, float *__restrict__ dD, float *__restrict__ dB_acc, float *__restrict__ dC_acc,
+    float *__restrict__ dtau, int *__restrict__ err, uint32_t tmem_cols) {
+    using namespace tc;
+    using bf16 = __nv_bfloat16;
+    constexpr int KS = KP <= 16 ? 16 : 32;
+    constexpr int N1 = 32 + 2 * KS;
+    constexpr int Q1 = kN1BQ + 1;
+    extern __shared__ __align__(1024) unsigned char sm_raw0[];
+    unsigned char *sm = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(sm_raw0) + 1023) &
+                                                          ~uintptr_t(1023));
+    const int K = d.K, P = d.P, Q = d.Q;
+    const N1BwdTcSmem L_(P, K);
+    double *E_s = reinterpret_cast<double *>(sm + L_.E);
+    float2 *Ef_s = reinterpret_cast<float2 *>(sm + L_.Ef);
+    float *e_s = reinterpret_cast<float *>(sm + L_.e), *cl_s = reinterpret_cast<float *>(sm + L_.cl);
+    float *itau = reinterpret_cast<float *>(sm + L_.itau), *red = reinterpret_cast<float *>(sm + L_.red);
+    float *cdot = reinterpret_cast<float *>(sm + L_.cdot), *dtq = reinterpret_cast<float *>(sm + L_.dtq);
+    const N1Arrays a(reinterpret_cast<float *>(sm + L_.qk), K);
+    float *H = reinterpret_cast<float *>(sm + L_.H), *XR = reinterpret_cast<float *>(sm + L_.XR);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sm + L_.bars);  // copies in, P1 done, P4 done
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 3);
+    unsigned char *img = sm + L_.bimg;
+    const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z, tid = threadIdx.x, w = tid >> 5, lane = tid & 31;
+    const int g = h / (d.H / d.G);
+    const int c0 = c * Q, n = min(Q, d.L - c0);
+    const size_t bh = size_t(b) * d.H + h;
+    const int NP = P / 64;
+    const uint32_t pan_a = smem_u32(sm + L_.pan), img_a = smem_u32(img);
+
+    // ---- P0: barriers, TMEM, the tile copies, rates and coefficients
+    if (tid == 0) {
+        for (int i = 0; i < 3; ++i) mbar_init(&bars[i], 1);
+        fence_barrier_init();
+    }
+    if (w == 0) tmem_alloc_once(tslot, tmem_cols);
+    for (uint32_t i = tid; i < L_.bimg_rows * 8; i += blockDim.x)
+        reinterpret_cast<uint4 *>(img)[i] = make_uint4(0u, 0u, 0u, 0u);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tslot;
+    bool issued1 = false, issued2 = false;  // (thread 0) MMA groups committed
+    if (tid == 0) {
+        mbar_arrive_expect_tx(&bars[0], uint32_t(NP) * L_.panel);
+        const int sc = int(bh * d.nc + c);
+        for (int j = 0; j < NP; ++j) {
+            unsigned char *pj = sm + L_.pan + size_t(j) * L_.panel;
+            tma_load_3d(pj, &mapDY, &bars[0], h * P + 64 * j, c0, b);
+            tma_load_3d(pj + 32 * 128, &mapX, &bars[0], h * P + 64 * j, c0, b);
+            tma_load_3d(pj + 64 * 128, &mapG, &bars[0], 64 * j, 0, sc);
+            tma_load_3d(pj + (64 + KS) * 128, &mapS, &bars[0], 64 * j, 0, sc);
         }
-        a_s[t] = a;
-        b_s[t] = bb;
+    }
+    if (tid < K) itau[tid] = 1.f / tau[h * K + tid];
+    if (tid < 64) red[tid] = 0.f;
+    if (tid < 32) cdot[tid] = dtq[tid] = 0.f;
+    const float log_cap = head_log_cap(tau, h, K);
+    chunk_rates(d, b, h, c0, n, log_cap, dt, alpha, lam, e_s, E_s, cl_s);
+    __syncthreads();
+    const double Eend = E_s[n - 1];
+    n1_bwd_coefs<bf16>(d, b, h, g, c0, n, Eend, itau, e_s, E_s, ww, wr, Bm, Cm, a);
+    for (int idx = tid; idx < kN1BQ * Q1; idx += blockDim.x) XR[idx] = 0.f;
+    if (tid < kN1BQ) {
+        const double Ev = tid < n ? E_s[tid] : 0.0;
+        const float hi = float(Ev);
+        Ef_s[tid] = make_float2(hi, float(Ev - double(hi)));
+    }
+
+    // ---- P1 on the tensor cores
+    int bad = !mbar_wait(&bars[0], 0);
+    bad = __syncthreads_or(bad);
+    if (!bad && tid == 0) {
+        tc_fence_after();
+        constexpr uint32_t id1 = idesc_bf16(128, N1, false, false);
+        for (int j = 0; j < NP; ++j)
+            for (int kk = 0; kk < 4; ++kk) {
+                const uint32_t a0 = pan_a + uint32_t(j) * L_.panel + kk * 32;
+                mma_bf16(tmem, desc_sw128(a0, 16, 1024), desc_sw128(a0 + 32 * 128, 16, 1024), id1, (j | kk) != 0);
+            }
+        mma_commit(&bars[1]);
+        issued1 = true;
+    }
+    if (!bad) bad = !mbar_wait(&bars[1], 0);
+    bad = __syncthreads_or(bad);
+    if (!bad) {
+        tc_fence_after();
+        if (w == 0) {  // lanes = dy rows t: H row t (columns 0..31), YS row t (columns 32 + KS ..)
+            float hv[32], ys[KS];
+            tmem_ld32(tmem, hv);
+            if constexpr (KS == 16) tmem_ld16(tmem + 32 + KS, ys);
+            else tmem_ld32(tmem + 32 + KS, ys);
+            tmem_ld_wait();
+            float dd = 0.f;
+#pragma unroll
+            for (int k = 0; k < 32; ++k) {
+                H[lane * Q1 + k] = hv[k];
+                if (k == lane && lane < n) dd = hv[k];  // sum_p dy x of row t (for dD)
+            }
+#pragma unroll
+            for (int m = 0; m < KS; ++m)
+                if (m < K) a.YS[lane * K + m] = ys[m];
+            dd = warp_sum(dd);
+            if (lane == 0) atomicAdd(&dD[h], dd);
+        } else if (w == 1) {  // lanes = x rows t: XG row t (columns 32 ..)
+            float xg[KS];
+            if constexpr (KS == 16) tmem_ld16(tmem + (32u << 16) + 32, xg);
+            else tmem_ld32(tmem + (32u << 16) + 32, xg);
+            tmem_ld_wait();
+#pragma unroll
+            for (int m = 0; m < KS; ++m)
+                if (m < K) a.XG[lane * K + m] = xg[m];
+        } else if (w == 2) {  // lanes = gamma rows m: <gamma_m, S_in,m> on the diagonal
+            float cv[KS];
+            if constexpr (KS == 16) tmem_ld16(tmem + (64u << 16) + 32 + KS, cv);
+            else tmem_ld32(tmem + (64u << 16) + 32 + KS, cv);
+            tmem_ld_wait();
+            float v = 0.f;
+#pragma unroll
+            for (int m = 0; m < KS; ++m)
+                if (m == lane) v = cv[m];
+            if (lane < K) cdot[lane] = v;
+        }
     }
     __syncthreads();
-    float cprime = 0.f;
-    for (int m = 0; m < K; ++m) cprime = fmaf(expf(-float(Eend) * itau[m]) * itau[m], cdot[m], cprime);
-    if (tid < n) {
-        const int t = tid;
-        float suf = 0.f, pre = 0.f;
-        for (int j = t; j < n; ++j) suf += a_s[j];
-        for (int j = 0; j < t; ++j) pre += b_s[j];
-        const float R = suf + pre + cprime + rp_s[t];
-        float de = -R, sB = 0.f, sC = 0.f;
-        const size_t i = blh(d, b, c0 + t, h);
-        for (int m = 0; m < K; ++m) {
-            const int q = t * K + m;
-            const float dkb = u_s[q] * XG[q] + dkbi[q];   // d(kappa B)
-            const float dwc = A_s[q] * YS[q] + dwci[q];   // d(w_read C)
-            const float dk = dkb * Bq[q];                 // d kappa
-            de = fmaf(dk * rho_s[q] * ww_s[q], itau[m], de);
-            dwr_o[i * K + m] = from_f<T>(dwc * Cq[q]);
-            dww_o[i * K + m] = from_f<T>(dk * (-expm1f(-e_s[t] * itau[m])));
-            sB = fmaf(dkb, kap_s[q], sB);
-            sC = fmaf(dwc, wr_s[q], sC);
-            if (dtau) {
-                const double Et = E_s[t];
-                const double tq = Et * double(wc_s[q] * A_s[q] * YS[q]) +
-                                  (Eend - Et) * double(kb_s[q] * u_s[q] * XG[q]) -
-                                  double(e_s[t]) * double(dk) * double(rho_s[q]) * double(ww_s[q]);
-                atomicAdd(&dtq[m], float(tq));
+
+    // ---- P2: pair passes; Gamma (hi, lo) into rows t and 32 + KS + t of P4's B, column k, and
+    // s = kappa B u into rows 32 + m and 64 + KS + m
+    if (!bad) {
+        n1_pair_passes<KP>(n, K, itau, Ef_s, a, H, XR, [&](int t, int k, float v) {
+            st_bf16_pair(img, uint32_t(t), uint32_t(32 + KS + t), uint32_t(k), v);
+        });
+        for (int idx = tid; idx < K * kN1BQ; idx += blockDim.x) {
+            const int m = idx / kN1BQ, k = idx - m * kN1BQ;
+            st_bf16_pair(img, uint32_t(32 + m), uint32_t(64 + KS + m), uint32_t(k), a.s[idx]);
+        }
+        fence_async_smem();
+    }
+    tc_fence_before();
+    __syncthreads();
+
+    // ---- P4 on the tensor cores (issued now, read after P3 and P5)
+    if (!bad && tid == 0) {
+        tc_fence_after();
+        constexpr uint32_t id4 = idesc_bf16(128, 64, true, true);
+        constexpr int half = 2 + KS / 16;  // K steps of 16 rows per (hi or lo) half
+        for (int i = 0; i < NP / 2; ++i)
+            for (int st = 0; st < 2 * half; ++st) {
+                const int sh = st % half;
+                const int ra = sh < 2 ? 16 * sh : 64 + 16 * (sh - 2);  // dy rows, then gamma rows
+                const uint32_t ad = pan_a + uint32_t(2 * i) * L_.panel + uint32_t(ra) * 128;
+                const uint32_t bd = img_a + uint32_t(st) * 16 * 128;
+                mma_bf16(tmem + 64 * i, desc_sw128(ad, L_.panel, 1024), desc_sw128(bd, L_.bimg_rows * 128, 1024),
+                         id4, st > 0);
+            }
+        mma_commit(&bars[2]);
+        issued2 = true;
+    }
+
+    // ---- P3 and P5 on the CUDA cores meanwhile
+    float *rp_s = red + 32;
+    if (!bad) {
+        n1_rect(n, Q, XR, rp_s);
+        __syncthreads();
+        n1_position_grads<bf16>(d, b, h, g, c0, n, Eend, a, itau, e_s, E_s, cl_s, cdot, rp_s, XR, dtq, dt, alpha,
+                                lam, dwr_o, dww_o, ddt, dalpha, dlam, dB_acc, dC_acc, dtau);
+    }
+
+    // ---- P4 epilogue: dx[k][p] = (dx^T)[p][k] + D dy[k][p], one thread per p
+    if (!bad) bad = !mbar_wait(&bars[2], 0);
+    bad = __syncthreads_or(bad);
+    if (!bad) {
+        tc_fence_after();
+        const float Dh = Dv[h];
+        for (int i = w / 4; i < NP / 2; i += 2) {
+            const int p = 128 * i + 32 * (w & 3) + lane;
+            float acc[32];
+            tmem_ld32(tmem + (uint32_t(32 * (w & 3)) << 16) + 64 * i, acc);
+            tmem_ld_wait();
+            const unsigned char *pp = sm + L_.pan + size_t(p >> 6) * L_.panel;
+#pragma unroll
+            for (int k = 0; k < kN1BQ; ++k) {
+                if (k < n) {
+                    const float dyv = __bfloat162float(*reinterpret_cast<const bf16 *>(pp + sw128_offset(k, p & 63)));
+                    dx[blh(d, b, c0 + k, h) * P + p] = __float2bfloat16_rn(fmaf(Dh, dyv, acc[k]));
+                }
             }
         }
-        const size_t gi = (size_t(b) * d.L + c0 + t) * d.G + g;
-        atomicAdd(&dB_acc[gi], sB);
-        atomicAdd(&dC_acc[gi], sC);
-        const float e = e_s[t];
-        const bool cl = cl_s[t] != 0.f;
-        const float al = alpha[i], lm = lam[i], dtv = dt[i];
-        const float ge = cl ? 0.f : de * e;
-        ddt[i] = ge / dtv;
-        dlam[i] = ge / (al * lm);
-        dalpha[i] = -ge * logf(lm) / (al * al);
     }
-    if (dtau) {
-        __syncthreads();
-        if (tid < K) {
-            const float it = itau[tid];
-            const float chunk_term = float(Eend) * expf(-float(Eend) * it) * cdot[tid];
-            atomicAdd(&dtau[h * K + tid], (dtq[tid] + chunk_term) * it * it);
-        }
+    if (bad && tid == 0) {  // a wait gave up: record it, let copies and MMAs in flight finish
+        atomicExch(err, kN1Timeout);
+        mbar_wait(&bars[0], 0);
+        if (issued1) mbar_wait(&bars[1], 0);
+        if (issued2) mbar_wait(&bars[2], 0);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (w == 0) {
+        tc_fence_after();
+        tmem_dealloc(tmem, tmem_cols);
     }
 }
 
@@ -1736,9 +2053,49 @@ bool n1_bwd_fits(const ScanDims &d, size_t esz) {
            size_t(d.H) * ((d.P + kN1P - 1) / kN1P) <= 65535;
 }
 
+// Whether the tensor-core variant of the N = 1 gradient kernel takes a bf16 call: P a multiple of
+// 128 up to 512, chunk 32, x, dy and the per-chunk states 16-byte aligned, and its shared memory
+// within the per-CTA limit.
+bool n1_bwd_tc_ok(const ScanDims &d, const ScanPtrs &p, const void *S_in, const void *dS_out) {
+    auto al16 = [](const void *q) { return (reinterpret_cast<uintptr_t>(q) & 15u) == 0; };
+    return d.N == 1 && d.Q == kN1BQ && d.P % 128 == 0 && d.P <= 512 && d.K <= 32 && al16(p.x) && al16(p.dy) &&
+           al16(S_in) && al16(dS_out) && N1BwdTcSmem(d.P, d.K).total <= 227 * 1024;
+}
+
+// Launches n1_chunk_bwd_tc; *launched stays false (and nothing is enqueued) when a tensor map
+// cannot be encoded, so that the caller runs the CUDA-core kernel instead.
+cudaError_t launch_n1_bwd_tc(const ScanDims &d, const ScanPtrs &p, void *S_in, void *dS_out, float *dB_acc,
+                             float *dC_acc, int *err, cudaStream_t st, bool *launched) {
+    using bf = __nv_bfloat16;
+    *launched = false;
+    const int KS = d.K <= 16 ? 16 : 32;
+    const uint64_t HP = uint64_t(d.H) * d.P;
+    const uint64_t chunks = uint64_t(d.B) * d.H * d.nc;
+    CUtensorMap mapX, mapDY, mapS, mapG;
+    if (!tc_make_map3(&mapX, p.x, HP, d.L, d.B, HP * 2, uint64_t(d.L) * HP * 2, 64, kN1BQ, 1) ||
+        !tc_make_map3(&mapDY, p.dy, HP, d.L, d.B, HP * 2, uint64_t(d.L) * HP * 2, 64, kN1BQ, 1) ||
+        !tc_make_map3(&mapS, S_in, d.P, d.K, chunks, uint64_t(d.P) * 2, uint64_t(d.K) * d.P * 2, 64, KS, 1) ||
+        !tc_make_map3(&mapG, dS_out, d.P, d.K, chunks, uint64_t(d.P) * 2, uint64_t(d.K) * d.P * 2, 64, KS, 1))
+        return cudaSuccess;
+    const size_t smem = N1BwdTcSmem(d.P, d.K).total;
+    const uint32_t cols = n1_tc_tmem_cols(d.P, d.K);
+    const int KP = d.K <= 4 ? 4 : d.K <= 8 ? 8 : d.K <= 16 ? 16 : 32;
+    auto k = KP == 4 ? n1_chunk_bwd_tc<4> : KP == 8 ? n1_chunk_bwd_tc<8> : KP == 16 ? n1_chunk_bwd_tc<16>
+                                                                                  : n1_chunk_bwd_tc<32>;
+    cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    trace_begin("chunk_bwd_n1_tc", st);
+    k<<<dim3(d.nc, d.H, d.B), kThreads, smem, st>>>(
+        mapX, mapDY, mapS, mapG, d, (const bf *)p.Bm, (const bf *)p.Cm, (const bf *)p.wr, (const bf *)p.ww, p.dt,
+        p.alpha, p.lam, p.tau, p.D, (bf *)p.dx, (bf *)p.dwr, (bf *)p.dww, p.ddt, p.dalpha, p.dlam, p.dD, dB_acc,
+        dC_acc, p.dtau, err, cols);
+    trace_end(st);
+    *launched = true;
+    return cudaGetLastError();
+}
+
 template <typename T, typename TS>
 cudaError_t bwd_n1(const ScanDims &d, const ScanPtrs &p, void *S_in, void *dS_out, float *dB_acc,
-                   float *dC_acc, float *scratch, bool reuse, cudaStream_t st) {
+                   float *dC_acc, float *scratch, bool reuse, int *err, cudaStream_t st) {
     const int npb = (d.P + kN1P - 1) / kN1P;
     float *loc = scratch, *dec = scratch + size_t(d.B) * d.H * d.nc * d.K * d.P;
     const bool vec = (reinterpret_cast<uintptr_t>(p.x) % 16 == 0) && (reinterpret_cast<uintptr_t>(p.dy) % 16 == 0) &&
@@ -1788,19 +2145,27 @@ cudaError_t bwd_n1(const ScanDims &d, const ScanPtrs &p, void *S_in, void *dS_ou
     n1_combine_rev<TS><<<unsigned((total + 255) / 256), 256, 0, st>>>(d, loc, dec, p.dh_final, (TS *)dS_out, p.dh0);
     trace_end(st);
     if ((e = cudaGetLastError()) != cudaSuccess || d.nc == 0) return e;  // L = 0: dh0 = dh_final
-    const size_t smem = N1BwdSmem(d.P, d.K, sizeof(T)).total;
-    auto kb = pick([&](auto kp) {
-        constexpr int V = decltype(kp)::value;
-        return vec ? n1_chunk_bwd<T, TS, true, V> : n1_chunk_bwd<T, TS, false, V>;
-    });
-    cudaFuncSetAttribute(kb, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-    trace_begin("chunk_bwd_n1", st);
-    kb<<<dim3(d.nc, d.H, d.B), kThreads, smem, st>>>(
-        d, (const T *)p.x, (const T *)p.Bm, (const T *)p.Cm, (const T *)p.wr, (const T *)p.ww, (const T *)p.dy,
-        p.dt, p.alpha, p.lam, p.tau, p.D, (const TS *)S_in, (const TS *)dS_out, (T *)p.dx, (T *)p.dwr,
-        (T *)p.dww, p.ddt, p.dalpha, p.dlam, p.dD, dB_acc, dC_acc, p.dtau);
-    trace_end(st);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    bool done = false;
+    if constexpr (std::is_same<T, __nv_bfloat16>::value && std::is_same<TS, __nv_bfloat16>::value) {
+        if (n1_bwd_tc_ok(d, p, S_in, dS_out)) {
+            if ((e = launch_n1_bwd_tc(d, p, S_in, dS_out, dB_acc, dC_acc, err, st, &done)) != cudaSuccess) return e;
+        }
+    }
+    if (!done) {
+        const size_t smem = N1BwdSmem(d.P, d.K, sizeof(T)).total;
+        auto kb = pick([&](auto kp) {
+            constexpr int V = decltype(kp)::value;
+            return vec ? n1_chunk_bwd<T, TS, true, V> : n1_chunk_bwd<T, TS, false, V>;
+        });
+        cudaFuncSetAttribute(kb, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+        trace_begin("chunk_bwd_n1", st);
+        kb<<<dim3(d.nc, d.H, d.B), kThreads, smem, st>>>(
+            d, (const T *)p.x, (const T *)p.Bm, (const T *)p.Cm, (const T *)p.wr, (const T *)p.ww, (const T *)p.dy,
+            p.dt, p.alpha, p.lam, p.tau, p.D, (const TS *)S_in, (const TS *)dS_out, (T *)p.dx, (T *)p.dwr,
+            (T *)p.dww, p.ddt, p.dalpha, p.dlam, p.dD, dB_acc, dC_acc, p.dtau);
+        trace_end(st);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
     if ((e = dtau_pairs_launch(d, sizeof(T) == 2 ? 1 : 0, p, st)) != cudaSuccess) return e;
     if (sizeof(T) == 2 && ngn > 0) {
         const unsigned blocks = unsigned(std::min<size_t>((ngn + 255) / 256, 4096));
@@ -1817,9 +2182,9 @@ cudaError_t bwd_n1(const ScanDims &d, const ScanPtrs &p, void *S_in, void *dS_ou
 
 template <typename T, typename TS>
 cudaError_t bwd_t(const ScanDims &d, const ScanPtrs &p, void *S_in, void *dS_out, float *dB_acc,
-                  float *dC_acc, float *n1_scratch, bool reuse, cudaStream_t st) {
+                  float *dC_acc, float *n1_scratch, bool reuse, int *err, cudaStream_t st) {
     if (uses_n1(d) && n1_bwd_fits(d, sizeof(T)))
-        return bwd_n1<T, TS>(d, p, S_in, dS_out, dB_acc, dC_acc, n1_scratch, reuse, st);
+        return bwd_n1<T, TS>(d, p, S_in, dS_out, dB_acc, dC_acc, n1_scratch, reuse, err, st);
     cudaError_t e = cudaSuccess;
     if (!reuse) e = run_state_pass<T, TS>(d, false, p.x, p.Bm, p.ww, p, p.h0, S_in, nullptr, st);
     if (e != cudaSuccess) return e;
@@ -1901,9 +2266,9 @@ cudaError_t simt_scan_fwd(const ScanDims &d, int dtype, const ScanPtrs &p, void 
 
 cudaError_t simt_scan_bwd(const ScanDims &d, int dtype, const ScanPtrs &p, void *S_in,
                           void *dS_out, float *dB_acc, float *dC_acc, float *n1_scratch, bool reuse,
-                          cudaStream_t st) {
-    if (dtype == 0) return bwd_t<float, float>(d, p, S_in, dS_out, dB_acc, dC_acc, n1_scratch, reuse, st);
-    return bwd_t<__nv_bfloat16, __nv_bfloat16>(d, p, S_in, dS_out, dB_acc, dC_acc, n1_scratch, reuse, st);
+                          int *err, cudaStream_t st) {
+    if (dtype == 0) return bwd_t<float, float>(d, p, S_in, dS_out, dB_acc, dC_acc, n1_scratch, reuse, err, st);
+    return bwd_t<__nv_bfloat16, __nv_bfloat16>(d, p, S_in, dS_out, dB_acc, dC_acc, n1_scratch, reuse, err, st);
 }
 
 }  // namespace frac

@@ -318,6 +318,7 @@ def _learned_tau(d64, dv, seed):
     ("bf16", synth.Shape(2, 260, 4, 64, 1, 64, 8, 0, "bf16")),        # tensor-core path
     ("bf16", synth.Shape(1, 300, 4, 64, 2, 128, 4, 0, "bf16")),       # tensor-core, K = 4, G = 2
     ("f32", synth.Shape(1, 200, 2, 256, 1, 1, 16, 0, "f32")),         # the paper's N = 1 shape
+    ("bf16", synth.Shape(2, 200, 2, 256, 1, 1, 16, 0, "bf16")),       # N = 1, tensor-core gradients
 ])
 def test_bwd_timescale_gradient(dtype, shape):
     host = synth.make_scan_inputs(shape, seed=31, with_dy=True, with_h0=True, with_dh_final=True)
@@ -391,3 +392,25 @@ def test_n1_backward_shapes(shape):
     multiple of 4, p blocks past the head dimension, groups (dB, dC summed over their heads),
     chunk sizes, ragged and empty sequences."""
     _check_bwd(shape, seed=70 + shape.nmodes, h0=True, dhf=True, chunk=shape.chunk)
+
+
+@pytest.mark.parametrize("shape", [
+    synth.Shape(2, 75, 4, 128, 2, 1, 4, 0, "bf16"),    # K = 4, P = 128, two sequences with ragged ends, groups
+    synth.Shape(1, 150, 2, 256, 1, 1, 5, 0, "bf16"),   # K = 5 (eight lanes per row), ragged
+    synth.Shape(1, 96, 2, 384, 1, 1, 16, 0, "bf16"),   # P = 384: three 128-wide dx tiles, whole chunks
+    synth.Shape(1, 70, 2, 128, 1, 1, 20, 0, "bf16"),   # K = 20 (32-row mode slots, 32 lanes per row)
+    synth.Shape(1, 20, 3, 256, 1, 1, 16, 0, "bf16"),   # one chunk, shorter than 32
+])
+def test_n1_backward_tensor_core_variant(shape):
+    """bf16 N = 1 backward with the head dimension a multiple of 128: the per-chunk gradient kernel
+    whose contractions over p and over positions run on tcgen05 (the trace shows it ran), for each
+    mode-slot layout, tile count and ragged or short sequence."""
+    from paper_2609_36314_gb300 import _lib
+    _lib.trace_reset()
+    _lib.trace_enable(True)
+    try:
+        _check_bwd(shape, seed=90 + shape.nmodes, h0=True, dhf=True)
+        names = set(_lib.trace_collect())
+    finally:
+        _lib.trace_enable(False)
+    assert "chunk_bwd_n1_tc" in names and "chunk_bwd_n1" not in names
