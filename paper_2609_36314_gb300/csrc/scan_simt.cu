@@ -1229,17 +1229,37 @@ __global__ void __launch_bounds__(kN1P) n1_rev_local(ScanDims d, const T *__rest
         dec[(bh * d.nc + c) * K + threadIdx.x] = a;
     }
     if (threadIdx.x >= np) return;
+    // g = w_read C dy at the chunk's last position, then g = rho_{t+1} g + w_read C dy going left
+    // (16-byte pieces of the coefficient rows when K is a multiple of 4, as in the forward)
     float g[KP];
 #pragma unroll
     for (int m = 0; m < KP; ++m) g[m] = 0.f;
-    for (int t = n - 1; t >= 0; --t) {
-        const float dv = to_f(y_s[t * kN1P + threadIdx.x]);
+    if (n > 0) {
+        const float dv = to_f(y_s[(n - 1) * kN1P + threadIdx.x]);
 #pragma unroll
-        for (int m = 0; m < KP; ++m) {
-            if (m < K) {
-                const float rn = t + 1 < n ? rho_s[(t + 1) * K + m] : 0.f;
-                g[m] = fmaf(rn, g[m], wc_s[t * K + m] * dv);
+        for (int m = 0; m < KP; ++m)
+            if (m < K) g[m] = wc_s[(n - 1) * K + m] * dv;
+    }
+#pragma unroll 4
+    for (int t = n - 2; t >= 0; --t) {
+        const float dv = to_f(y_s[t * kN1P + threadIdx.x]);
+        if ((K & 3) == 0) {
+            const float4 *r4 = reinterpret_cast<const float4 *>(rho_s + (t + 1) * K);
+            const float4 *w4 = reinterpret_cast<const float4 *>(wc_s + t * K);
+#pragma unroll
+            for (int q = 0; q < KP / 4; ++q) {
+                if (4 * q < K) {
+                    const float4 r = r4[q], wv = w4[q];
+                    g[4 * q] = fmaf(r.x, g[4 * q], wv.x * dv);
+                    g[4 * q + 1] = fmaf(r.y, g[4 * q + 1], wv.y * dv);
+                    g[4 * q + 2] = fmaf(r.z, g[4 * q + 2], wv.z * dv);
+                    g[4 * q + 3] = fmaf(r.w, g[4 * q + 3], wv.w * dv);
+                }
             }
+        } else {
+#pragma unroll
+            for (int m = 0; m < KP; ++m)
+                if (m < K) g[m] = fmaf(rho_s[(t + 1) * K + m], g[m], wc_s[t * K + m] * dv);
         }
     }
 #pragma unroll
