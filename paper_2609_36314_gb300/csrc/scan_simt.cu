@@ -1305,6 +1305,8 @@ __global__ void __launch_bounds__(256) n1_combine_rev(ScanDims d, const float *_
 
 constexpr int kN1BQ = 32;  // chunk of the N = 1 backward (shared-memory tiles [Q][P])
 constexpr int kN1Timeout = 4;  // FRAC_ERR_TIMEOUT in the call's status word
+// floats of the N1Arrays block (15 [Q][K] arrays and two [Q] arrays)
+__host__ __device__ constexpr size_t n1_arrays_floats(int K) { return size_t(15) * kN1BQ * K + 2 * kN1BQ; }
 constexpr int kGS = 36;    // row stride of its Gamma tile (rows read as 16-byte pieces)
 
 struct N1BwdSmem {
@@ -1319,8 +1321,8 @@ struct N1BwdSmem {
         red = itau + sizeof(float) * 32;                         // float [64]
         cdot = red + sizeof(float) * 64;                         // float [32]
         dtq = cdot + sizeof(float) * 32;                         // float [32]: dtau sums per mode
-        qk = dtq + sizeof(float) * 32;                           // float [15][Q][K]
-        x = qk + sizeof(float) * 15 * kN1BQ * K;                 // T [Q][P]
+        qk = dtq + sizeof(float) * 32;                           // float N1Arrays
+        x = qk + sizeof(float) * n1_arrays_floats(K);            // T [Q][P]
         x = (x + 15) / 16 * 16;
         y = x + esz * kN1BQ * P;                                 // T [Q][P]
         y = (y + 15) / 16 * 16;
@@ -1336,13 +1338,15 @@ struct N1BwdSmem {
 // The [Q][K] float arrays of the N = 1 gradient kernels (shared memory): per-(position, mode)
 // coefficients, then the dot products over p and the pair sums.
 struct N1Arrays {
-    float *rho, *kap, *kb, *wc, *A, *u, *ww, *wr, *XG, *YS, *dwci, *dkbi, *Bq, *Cq;
-    float *s;  // kappa B u, mode-major [K][Q]
+    float *rho, *kap, *kb, *wc, *A, *u, *ww, *wr, *XG, *YS, *dwci, *dkbi;
+    float *kbT, *wcT, *s;  // kappa B, w_read C and kappa B u, mode-major [K][Q]
+    float *Bt, *Ct;        // [Q]
     __device__ N1Arrays(float *qk, int K) {
         const int QK = kN1BQ * K;
         rho = qk; kap = qk + QK; kb = qk + 2 * QK; wc = qk + 3 * QK; A = qk + 4 * QK; u = qk + 5 * QK;
         ww = qk + 6 * QK; wr = qk + 7 * QK; XG = qk + 8 * QK; YS = qk + 9 * QK; dwci = qk + 10 * QK;
-        dkbi = qk + 11 * QK; Bq = qk + 12 * QK; Cq = qk + 13 * QK; s = qk + 14 * QK;
+        dkbi = qk + 11 * QK; kbT = qk + 12 * QK; wcT = qk + 13 * QK; s = qk + 14 * QK;
+        Bt = qk + 15 * QK; Ct = Bt + kN1BQ;
     }
 };
 
@@ -1372,175 +1376,192 @@ __device__ __forceinline__ void n1_bwd_coefs(const ScanDims &d, int b, int h, in
             u = expf(-float(Eend - E_s[t]) * itau[m]);
         }
         a.rho[idx] = rho; a.kap[idx] = kap; a.kb[idx] = kap * Bt; a.wc[idx] = w_r * Ct;
-        a.A[idx] = A; a.u[idx] = u; a.ww[idx] = w_w; a.wr[idx] = w_r; a.Bq[idx] = Bt; a.Cq[idx] = Ct;
-        a.s[m * kN1BQ + t] = kap * Bt * u;
+        a.A[idx] = A; a.u[idx] = u; a.ww[idx] = w_w; a.wr[idx] = w_r;
+        a.kbT[m * kN1BQ + t] = kap * Bt; a.wcT[m * kN1BQ + t] = w_r * Ct; a.s[m * kN1BQ + t] = kap * Bt * u;
+        if (m == 0) {
+            a.Bt[t] = Bt;
+            a.Ct[t] = Ct;
+        }
         a.XG[idx] = 0.f; a.YS[idx] = 0.f;
     }
 }
 
-// Pair passes over k <= t for every mode, one thread per (row, mode): 32 / KP rows per warp, the
-// lanes of a row on consecutive modes; row groups go to the warps in snake order (long rows with
-// short ones).  Row pass (thread = (t, m)): the intra dw_read-like sums, and Gamma and
-// Gamma' o H, which the row's lanes sum over the modes four columns at a time by halving
-// exchanges; put(t, k, Gamma_tk) stores Gamma, XR takes Gamma' o H.  Column pass (thread =
-// (k, m)): the intra dkappa B-like sums.  Every entry has one writer (no atomics).
+// Sums NV (a power of two <= 32) values over the 32 lanes of a warp by halving exchanges: at
+// offset o a lane keeps the half of its values picked by bit o of its lane index and adds its
+// partner's copy of that half.  Returns the index of the total that v[0] then holds; lanes whose
+// low 5 - log2(NV) bits are not all zero hold copies.
+template <int NV>
+__device__ __forceinline__ int warp_halving_sum(float (&v)[NV], int lane) {
+    int cnt = NV, base = 0;
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+        if (cnt > 1) {
+            const int half = cnt / 2;
+            const bool up = (lane & o) != 0;
+#pragma unroll
+            for (int i = 0; i < NV / 2; ++i) {
+                if (i < half) {
+                    const float send = up ? v[i] : v[i + half];
+                    const float keep = up ? v[i + half] : v[i];
+                    v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+                }
+            }
+            if (up) base += half;
+            cnt = half;
+        } else {
+            v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
+        }
+    }
+    return base;
+}
+
+// Pair passes over k <= t.  Row pass, one warp per row t with the lanes on the columns k: the
+// pair decays of every mode in registers (independent exponentials), Gamma_tk = sum_m w_read C_t
+// kappa B_k exp(-(E_t - E_k)/tau_m) to put(t, k, .), Gamma' o H to XR, and the intra dw_read-like
+// sums over k (a halving-exchange sum across the warp).  Column pass, one warp per column k with
+// the lanes on the rows t: the intra dkappa B-like sums over t.  Every entry has one writer.
 template <int KP, typename PutGamma>
 __device__ __forceinline__ void n1_pair_passes(int n, int K, const float *itau, const float2 *Ef_s,
                                                const N1Arrays &a, const float *H, float *XR, PutGamma put) {
     constexpr int Q1 = kN1BQ + 1;
-    constexpr int RPW = 32 / KP;
-    constexpr int kCnt = KP >= 8 ? 1 : 8 / KP;    // values a lane holds after the exchanges
-    constexpr int kDup = KP >= 8 ? KP / 8 - 1 : 0; // lane bits that hold copies of one value
-    const int tid = threadIdx.x, w = tid >> 5, lane = tid & 31, nw = blockDim.x >> 5;
-    const int m = lane % KP, sub = lane / KP;
-    const bool mok = m < K;
-    const float itm = mok ? itau[m] : 0.f;
-    const int ngrp = (n + RPW - 1) / RPW;
-    for (int pass = 0; pass * nw < ngrp; ++pass) {  // row pass
-        const int gi = pass * nw + ((pass & 1) ? nw - 1 - w : w);
-        if (gi >= ngrp) continue;  // warp-uniform
-        const int t = gi * RPW + sub;
-        const int tlast = min(gi * RPW + RPW - 1, n - 1);  // warp-uniform
-        const bool live = t < n && mok;
-        const float wct = live ? a.wc[t * K + m] : 0.f;
+    constexpr int kDup = 32 / KP - 1;  // lane bits holding copies after warp_halving_sum<KP>
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+    float it[KP];
+#pragma unroll
+    for (int m = 0; m < KP; ++m) it[m] = m < K ? itau[m] : 0.f;
+    const float2 Elane = Ef_s[lane];
+    for (int t = w; t < n; t += nw) {  // row pass
         const float2 Et = Ef_s[t];
-        float dw = 0.f;
-        for (int k0 = 0; k0 <= tlast; k0 += 4) {
-            float v[8];
+        const bool ok = lane <= t;
+        const float dE = (Et.x - Elane.x) + (Et.y - Elane.y);
+        const float hv = ok ? H[t * Q1 + lane] : 0.f;
+        float gam = 0.f, gamt = 0.f, dw[KP];
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const int k = k0 + j;
-                float av = 0.f, hv = 0.f;
-                if (live && k <= t) {
-                    const float2 Ek = Ef_s[k];
-                    const float dE = (Et.x - Ek.x) + (Et.y - Ek.y);
-                    const float kw = a.kb[k * K + m] * expf(-dE * itm);
-                    hv = H[t * Q1 + k];
-                    av = wct * kw;
-                    dw = fmaf(kw, hv, dw);
-                }
-                v[j] = av;
-                v[4 + j] = av * itm * hv;
+        for (int m = 0; m < KP; ++m) {
+            float av = 0.f, kw = 0.f;
+            if (m < K && ok) {
+                kw = a.kbT[m * kN1BQ + lane] * expf(-dE * it[m]);
+                av = a.wc[t * K + m] * kw;
             }
-            // halving exchanges over the row's KP lanes: at offset o a lane keeps the half of
-            // its values picked by bit o of its lane index and adds its partner's copy of it
-            int cnt = 8, base = 0;
-#pragma unroll
-            for (int o = KP / 2; o >= 1; o >>= 1) {
-                if (cnt > 1) {
-                    const int half = cnt / 2;
-                    const bool up = (lane & o) != 0;
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        if (i < half) {
-                            const float send = up ? v[i] : v[i + half];
-                            const float keep = up ? v[i + half] : v[i];
-                            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
-                        }
-                    }
-                    if (up) base += half;
-                    cnt = half;
-                } else {
-                    v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
-                }
-            }
-            if (t < n && (lane & kDup) == 0) {
-#pragma unroll
-                for (int i = 0; i < kCnt; ++i) {
-                    const int vi = base + i, k = k0 + (vi & 3);
-                    if (k <= t) {
-                        if (vi < 4) put(t, k, v[i]);
-                        else XR[t * Q1 + k] = v[i];
-                    }
-                }
-            }
+            gam += av;
+            gamt = fmaf(av, it[m], gamt);
+            dw[m] = kw * hv;
         }
-        if (live) a.dwci[t * K + m] = dw;
+        if (ok) {
+            put(t, lane, gam);
+            XR[t * Q1 + lane] = gamt * hv;
+        }
+        const int m0 = warp_halving_sum<KP>(dw, lane);
+        if ((lane & kDup) == 0 && m0 < K) a.dwci[t * K + m0] = dw[0];
     }
-    for (int pass = 0; pass * nw < ngrp; ++pass) {  // column pass
-        const int gi = pass * nw + ((pass & 1) ? nw - 1 - w : w);
-        if (gi >= ngrp) continue;
-        const int k = gi * RPW + sub;
-        if (k < n && mok) {
-            const float2 Ek = Ef_s[k];
-            float dk = 0.f;
-            for (int t = k; t < n; ++t) {
-                const float2 Et = Ef_s[t];
-                const float dE = (Et.x - Ek.x) + (Et.y - Ek.y);
-                dk = fmaf(a.wc[t * K + m] * expf(-dE * itm), H[t * Q1 + k], dk);
-            }
-            a.dkbi[k * K + m] = dk;
-        }
+    for (int k = w; k < n; k += nw) {  // column pass
+        const float2 Ek = Ef_s[k];
+        const bool ok = lane >= k && lane < n;
+        const float dE = (Elane.x - Ek.x) + (Elane.y - Ek.y);
+        const float hv = ok ? H[lane * Q1 + k] : 0.f;
+        float dk[KP];
+#pragma unroll
+        for (int m = 0; m < KP; ++m)
+            dk[m] = (m < K && ok) ? a.wcT[m * kN1BQ + lane] * expf(-dE * it[m]) * hv : 0.f;
+        const int m0 = warp_halving_sum<KP>(dk, lane);
+        if ((lane & kDup) == 0 && m0 < K) a.dkbi[k * K + m0] = dk[0];
     }
 }
 
-// Rectangle sums of Gamma' o H over pairs k < t <= t': XR rows become exclusive row prefixes,
-// then rp_s[t] = sum over t' >= t of row t' at column t.  Ends before the column sums are
-// published (the caller synchronises).
-__device__ __forceinline__ void n1_rect(int n, int Q, float *XR, float *rp_s) {
+// Rectangle sums of Gamma' o H over pairs k < t <= t': each row of XR becomes its exclusive
+// prefix (a warp scan per row), then rp_s[t] = sum over t' >= t of row t' at column t (a warp sum
+// per column).  Ends with rp_s published.
+__device__ __forceinline__ void n1_rect(int n, float *XR, float *rp_s) {
     constexpr int Q1 = kN1BQ + 1;
-    const int tid = threadIdx.x;
-    if (tid < Q) {
-        float run = 0.f;
-        for (int j = 0; j < Q; ++j) {
-            const float v = XR[tid * Q1 + j];
-            XR[tid * Q1 + j] = run;
-            run += v;
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+    for (int t = w; t < n; t += nw) {
+        float incl = XR[t * Q1 + lane];
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const float u = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += u;
         }
+        const float excl = __shfl_up_sync(0xffffffffu, incl, 1);  // no cancellation of v
+        XR[t * Q1 + lane] = lane > 0 ? excl : 0.f;
     }
     __syncthreads();
-    if (tid < Q) {
-        float s = 0.f;
-        for (int tp = tid; tp < n; ++tp) s += XR[tp * Q1 + tid];
-        rp_s[tid] = s;
+    for (int t = w; t < n; t += nw) {
+        const float v = (lane >= t && lane < n) ? XR[lane * Q1 + t] : 0.f;
+        const float sum = warp_sum(v);
+        if (lane == 0) rp_s[t] = sum;
     }
+    __syncthreads();
 }
 
-// Per-position gradients of one chunk.  a_t / b_k are the S_in / gamma terms of
-// sum_m rho <g_t, S_{t-1}>_m / tau_m (suffix and exclusive prefix sums), c the <gamma, S_in>
-// term, rp_s the pairs; then dDelta, dalpha, dlambda, the mode weights, dB, dC and (when asked)
-// the inter-chunk and per-position terms of dtau.  scratch: 128 floats no longer in use.
-template <typename T>
+// Per-position gradients of one chunk, one thread per (position, mode) with 32 / KP positions per
+// warp (the lanes of a position on consecutive modes).  a_t / b_k are the S_in / gamma terms of
+// sum_m rho <g_t, S_{t-1}>_m / tau_m (suffix and exclusive prefix sums over the chunk, warp
+// scans), c the <gamma, S_in> term, rp_s the pairs; then the mode-weight gradients per (t, m) and,
+// summed over the position's lanes, dDelta, dalpha, dlambda, dB, dC and (when asked) the
+// inter-chunk and per-position terms of dtau.  scratch: 96 floats no longer in use.
+template <typename T, int KP>
 __device__ __forceinline__ void n1_position_grads(
     const ScanDims &d, int b, int h, int g, int c0, int n, double Eend, const N1Arrays &a, const float *itau,
     const float *e_s, const double *E_s, const float *cl_s, const float *cdot, const float *rp_s, float *scratch,
     float *dtq, const float *__restrict__ dt, const float *__restrict__ alpha, const float *__restrict__ lam,
     T *__restrict__ dwr_o, T *__restrict__ dww_o, float *__restrict__ ddt, float *__restrict__ dalpha,
     float *__restrict__ dlam, float *__restrict__ dB_acc, float *__restrict__ dC_acc, float *__restrict__ dtau) {
-    const int K = d.K, tid = threadIdx.x;
-    float *a_s = scratch, *b_s = scratch + 64;
-    if (tid < n) {
-        const int t = tid;
-        float av = 0.f, bv = 0.f;
-        for (int m = 0; m < K; ++m) {
+    constexpr int RPW = 32 / KP;
+    const int K = d.K, tid = threadIdx.x, w = tid >> 5, lane = tid & 31, nw = blockDim.x >> 5;
+    const int m = lane % KP, sub = lane / KP;
+    const bool mok = m < K;
+    const float itm = mok ? itau[m] : 0.f;
+    float *a_s = scratch, *b_s = scratch + 32, *R_s = scratch + 64;
+    const int ngrp = (n + RPW - 1) / RPW;
+    for (int gi = w; gi < ngrp; gi += nw) {
+        const int t = gi * RPW + sub;
+        float va = 0.f, vb = 0.f;
+        if (t < n && mok) {
             const int q = t * K + m;
-            av = fmaf(a.wc[q] * a.A[q] * a.YS[q], itau[m], av);
-            bv = fmaf(a.kb[q] * a.u[q] * a.XG[q], itau[m], bv);
+            va = a.wc[q] * a.A[q] * a.YS[q] * itm;
+            vb = a.kb[q] * a.u[q] * a.XG[q] * itm;
         }
-        a_s[t] = av;
-        b_s[t] = bv;
+#pragma unroll
+        for (int o = KP / 2; o >= 1; o >>= 1) {
+            va += __shfl_xor_sync(0xffffffffu, va, o);
+            vb += __shfl_xor_sync(0xffffffffu, vb, o);
+        }
+        if (m == 0 && t < n) {
+            a_s[t] = va;
+            b_s[t] = vb;
+        }
     }
     __syncthreads();
-    float cprime = 0.f;
-    for (int m = 0; m < K; ++m) cprime = fmaf(expf(-float(Eend) * itau[m]) * itau[m], cdot[m], cprime);
-    if (tid < n) {
-        const int t = tid;
-        float suf = 0.f, pre = 0.f;
-        for (int j = t; j < n; ++j) suf += a_s[j];
-        for (int j = 0; j < t; ++j) pre += b_s[j];
-        const float R = suf + pre + cprime + rp_s[t];
-        float de = -R, sB = 0.f, sC = 0.f;
-        const size_t i = blh(d, b, c0 + t, h);
-        for (int m = 0; m < K; ++m) {
+    if (w == 0) {
+        float cp = lane < K ? expf(-float(Eend) * itau[lane]) * itau[lane] * cdot[lane] : 0.f;
+        cp = warp_sum(cp);
+        const float av = lane < n ? a_s[lane] : 0.f, bv = lane < n ? b_s[lane] : 0.f;
+        float suf = av, pre = bv;  // inclusive suffix sums of a, inclusive prefix sums of b
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const float us = __shfl_down_sync(0xffffffffu, suf, o);
+            const float up = __shfl_up_sync(0xffffffffu, pre, o);
+            if (lane + o < 32) suf += us;
+            if (lane >= o) pre += up;
+        }
+        const float pre_x = __shfl_up_sync(0xffffffffu, pre, 1);  // exclusive prefix of b
+        if (lane < n) R_s[lane] = suf + (lane > 0 ? pre_x : 0.f) + cp + rp_s[lane];
+    }
+    __syncthreads();
+    for (int gi = w; gi < ngrp; gi += nw) {
+        const int t = gi * RPW + sub;
+        float de = 0.f, sB = 0.f, sC = 0.f;
+        const size_t i = t < n ? blh(d, b, c0 + t, h) : 0;
+        if (t < n && mok) {
             const int q = t * K + m;
             const float dkb = a.u[q] * a.XG[q] + a.dkbi[q];  // d(kappa B)
             const float dwc = a.A[q] * a.YS[q] + a.dwci[q];  // d(w_read C)
-            const float dk = dkb * a.Bq[q];                  // d kappa
-            de = fmaf(dk * a.rho[q] * a.ww[q], itau[m], de);
-            dwr_o[i * K + m] = from_f<T>(dwc * a.Cq[q]);
-            dww_o[i * K + m] = from_f<T>(dk * (-expm1f(-e_s[t] * itau[m])));
-            sB = fmaf(dkb, a.kap[q], sB);
-            sC = fmaf(dwc, a.wr[q], sC);
+            const float dk = dkb * a.Bt[t];                  // d kappa
+            de = dk * a.rho[q] * a.ww[q] * itm;
+            dwr_o[i * K + m] = from_f<T>(dwc * a.Ct[t]);
+            dww_o[i * K + m] = from_f<T>(dk * (-expm1f(-e_s[t] * itm)));
+            sB = dkb * a.kap[q];
+            sC = dwc * a.wr[q];
             if (dtau) {
                 const double Et = E_s[t];
                 const double tq = Et * double(a.wc[q] * a.A[q] * a.YS[q]) +
@@ -1549,16 +1570,25 @@ __device__ __forceinline__ void n1_position_grads(
                 atomicAdd(&dtq[m], float(tq));
             }
         }
-        const size_t gi = (size_t(b) * d.L + c0 + t) * d.G + g;
-        atomicAdd(&dB_acc[gi], sB);
-        atomicAdd(&dC_acc[gi], sC);
-        const float e = e_s[t];
-        const bool cl = cl_s[t] != 0.f;
-        const float al = alpha[i], lm = lam[i], dtv = dt[i];
-        const float ge = cl ? 0.f : de * e;
-        ddt[i] = ge / dtv;
-        dlam[i] = ge / (al * lm);
-        dalpha[i] = -ge * logf(lm) / (al * al);
+#pragma unroll
+        for (int o = KP / 2; o >= 1; o >>= 1) {
+            de += __shfl_xor_sync(0xffffffffu, de, o);
+            sB += __shfl_xor_sync(0xffffffffu, sB, o);
+            sC += __shfl_xor_sync(0xffffffffu, sC, o);
+        }
+        if (m == 0 && t < n) {
+            de -= R_s[t];
+            const size_t gq = (size_t(b) * d.L + c0 + t) * d.G + g;
+            atomicAdd(&dB_acc[gq], sB);
+            atomicAdd(&dC_acc[gq], sC);
+            const float e = e_s[t];
+            const bool cl = cl_s[t] != 0.f;
+            const float al = alpha[i], lm = lam[i], dtv = dt[i];
+            const float ge = cl ? 0.f : de * e;
+            ddt[i] = ge / dtv;
+            dlam[i] = ge / (al * lm);
+            dalpha[i] = -ge * logf(lm) / (al * al);
+        }
     }
     if (dtau) {
         __syncthreads();
@@ -1754,7 +1784,7 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
 
     // ---- P3: rectangle sums of Gamma' o H over pairs k < t <= t' (row prefix, column suffix)
     float *rp_s = red + 32;  // [Q <= 32] (block_sum below uses red[0 .. 8))
-    n1_rect(n, Q, XR, rp_s);
+    n1_rect(n, XR, rp_s);
 
     // ---- P4: dx[k][p] = sum_m s_{k,m} gamma_m[p] + sum_{t>=k} Gamma[t][k] dy_t[p] + D dy_k[p]
     // (one thread per p).  Gamma is zero above the diagonal and on rows past the chunk's end, so
@@ -1800,7 +1830,7 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
     if (tid == 0) atomicAdd(&dD[h], ddv);
 
     // ---- P5: per-position scalars (XR is free now)
-    n1_position_grads<T>(d, b, h, g, c0, n, Eend, a, itau, e_s, E_s, cl_s, cdot, rp_s, XR, dtq, dt, alpha, lam,
+    n1_position_grads<T, KP>(d, b, h, g, c0, n, Eend, a, itau, e_s, E_s, cl_s, cdot, rp_s, XR, dtq, dt, alpha, lam,
                          dwr_o, dww_o, ddt, dalpha, dlam, dB_acc, dC_acc, dtau);
 }
 
@@ -1834,8 +1864,8 @@ struct N1BwdTcSmem {
         red = itau + sizeof(float) * 32;                           // float [64]
         cdot = red + sizeof(float) * 64;                           // float [32]
         dtq = cdot + sizeof(float) * 32;                           // float [32]
-        qk = dtq + sizeof(float) * 32;                             // float [15][Q][K]
-        H = qk + sizeof(float) * 15 * kN1BQ * K;                   // float [Q][Q + 1]
+        qk = dtq + sizeof(float) * 32;                             // float N1Arrays
+        H = qk + sizeof(float) * n1_arrays_floats(K);              // float [Q][Q + 1]
         XR = H + sizeof(float) * kN1BQ * (kN1BQ + 1);              // float [Q][Q + 1]
         bars = (XR + sizeof(float) * kN1BQ * (kN1BQ + 1) + 7) / 8 * 8;  // 3 mbarriers, TMEM slot
         total = bars + 32 + 1024;                                  // + slack to align the base
@@ -2027,9 +2057,8 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd_tc(
     // ---- P3 and P5 on the CUDA cores meanwhile
     float *rp_s = red + 32;
     if (!bad) {
-        n1_rect(n, Q, XR, rp_s);
-        __syncthreads();
-        n1_position_grads<bf16>(d, b, h, g, c0, n, Eend, a, itau, e_s, E_s, cl_s, cdot, rp_s, XR, dtq, dt, alpha,
+        n1_rect(n, XR, rp_s);
+        n1_position_grads<bf16, KP>(d, b, h, g, c0, n, Eend, a, itau, e_s, E_s, cl_s, cdot, rp_s, XR, dtq, dt, alpha,
                                 lam, dwr_o, dww_o, ddt, dalpha, dlam, dB_acc, dC_acc, dtau);
     }
 
