@@ -263,13 +263,10 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
         // per-position inputs of row t from the staging area, and the mode time constants
         cp_async_wait_all();
         sync_first256();
-        float wr_t[KMAX], kap_t[KMAX], tau_r[KMAX];
+        float wr_t[KMAX], kap_t[KMAX];
         float2 Et2 = make_float2(0.f, 0.f);  // in-chunk cumulative log-decay (hi, lo)
 #pragma unroll
-        for (int m = 0; m < KMAX; ++m) {
-            tau_r[m] = m < K ? pf_tau[m] : 1.f;
-            wr_t[m] = kap_t[m] = 0.f;
-        }
+        for (int m = 0; m < KMAX; ++m) wr_t[m] = kap_t[m] = 0.f;
         {
             const float4 e4 = *reinterpret_cast<const float4 *>(pf_e + t * 12);
             Et2 = make_float2(e4.x, e4.y);
@@ -288,13 +285,16 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
         sync_first256();  // the staging area is free again: the next item's inputs
         if (item + int(gridDim.x) < nitems) stage_inputs(item + gridDim.x);
         if (grp == 0) E_s[t] = Et2;
-        float l2r[KMAX];  // log2(e) / tau per mode, in registers
+        float l2r[KMAX];  // log2(e) / tau per mode, in registers (the table tid < K wrote)
 #pragma unroll
-        for (int m = 0; m < KMAX; ++m) {
-            l2r[m] = m < K ? kLog2e / tau_r[m] : 0.f;
-            if (grp == 0) {
-                wr_s[t * KMAX + m] = wr_t[m];
-                kap_s[t * KMAX + m] = kap_t[m];
+        for (int m = 0; m < KMAX; ++m) l2r[m] = m < K ? l2t[m] : 0.f;
+        if (grp == 0) {
+#pragma unroll
+            for (int q = 0; q < KMAX / 4; ++q) {
+                *reinterpret_cast<float4 *>(wr_s + t * KMAX + 4 * q) =
+                    make_float4(wr_t[4 * q], wr_t[4 * q + 1], wr_t[4 * q + 2], wr_t[4 * q + 3]);
+                *reinterpret_cast<float4 *>(kap_s + t * KMAX + 4 * q) =
+                    make_float4(kap_t[4 * q], kap_t[4 * q + 1], kap_t[4 * q + 2], kap_t[4 * q + 3]);
             }
         }
         tc_fence_before();
@@ -359,13 +359,18 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
         sync_first256();
         tc_fence_after();
         // U rows as fp32 [128 t][4 J][8 m] in the x tile (free now) for the column pass, before the
-        // row pass overwrites the operand tiles with XX
+        // row pass overwrites the operand tiles with XX.  Group g copies four of the eight 16-byte
+        // pieces of row t: piece c = (a t) xor (4 g + c4), with a t the product by the generator of
+        // GF(8) (x^3 + x + 1).  For eight neighbouring threads both the destination pieces c and the
+        // swizzled source pieces c xor t = ((a + 1) t) xor (4 g + c4) are all different, so neither
+        // the reads nor the writes meet a bank conflict
         float *Ufp = reinterpret_cast<float *>(sX);
-        {  // group g copies the chunks [4 g, 4 g + 4) of row t
+        {
             const unsigned char *row = sU + t * 128;
+            const int t7 = t & 7, at = ((t7 << 1) & 7) ^ ((t7 >> 2) * 3);
 #pragma unroll
             for (int c4 = 0; c4 < 4; ++c4) {
-                const int c8 = 4 * grp + c4;
+                const int c8 = at ^ (4 * grp + c4);
                 *reinterpret_cast<uint4 *>(Ufp + t * 32 + 4 * c8) =
                     *reinterpret_cast<const uint4 *>(row + ((c8 ^ (t & 7)) * 16));
             }
@@ -423,25 +428,31 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
                     }
                 }
                 if (dstep) {
+                    // branch-free over the eight columns: a pair above the diagonal (k > t) runs
+                    // the same arithmetic with its decay exponent clamped to zero (every factor
+                    // finite) and a zero G H, and its Gamma is masked to zero
 #pragma unroll
                     for (int kk = 0; kk < 8; ++kk) {
                         const int k = k0 + kk;
-                        float gam = 0.f, gamt = 0.f, gh = 0.f;
-                        if (k <= t && t < n) {
-                            const float dE = diff_f2(Et2, E_s[k]);
-                            gh = gv[kk] * hv[kk];
+                        const bool valid = k <= t && t < n;
+                        const float dE = fmaxf(diff_f2(Et2, E_s[k]), 0.f);
+                        const float gh = valid ? gv[kk] * hv[kk] : 0.f;
+                        const float4 ka = *reinterpret_cast<const float4 *>(kap_s + k * KMAX);
+                        const float4 kb = *reinterpret_cast<const float4 *>(kap_s + k * KMAX + 4);
+                        const float kpv[8] = {ka.x, ka.y, ka.z, ka.w, kb.x, kb.y, kb.z, kb.w};
+                        float gam = 0.f, gamt = 0.f;
 #pragma unroll
-                            for (int m = 0; m < KMAX; ++m) {
-                                if (m < K) {
-                                    const float W = ex2_approx(-dE * l2r[m]);
-                                    const float kp = kap_s[k * KMAX + m];
-                                    const float aa = wr_t[m] * kp * W;
-                                    gam += aa;
-                                    gamt = fmaf(aa, l2r[m], gamt);  // times log2(e) / tau
-                                    dwr_i[m] = fmaf(kp * W, gh, dwr_i[m]);
-                                }
+                        for (int m = 0; m < KMAX; ++m) {
+                            if (m < K) {
+                                const float W = ex2_approx(-dE * l2r[m]);
+                                const float kp = kpv[m];
+                                const float aa = wr_t[m] * kp * W;
+                                gam += aa;
+                                gamt = fmaf(aa, l2r[m], gamt);  // times log2(e) / tau
+                                dwr_i[m] = fmaf(kp * W, gh, dwr_i[m]);
                             }
                         }
+                        gam = valid ? gam : 0.f;
                         gv[kk] = gam * gv[kk];
                         hv[kk] = gam * hv[kk];
                         XX[t * XS + k] = gamt * (1.f / kLog2e) * gh;
@@ -549,10 +560,15 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
         sync_first256();
         tc_fence_after();
         if (!*abort_s && grp == 0 && t < n) {
-            float *o = a.dwr_acc + blh(d, b, c0 + t, h) * K;
+            float4 *o = reinterpret_cast<float4 *>(a.dwr_acc + blh(d, b, c0 + t, h) * K);
 #pragma unroll
-            for (int m = 0; m < KMAX; ++m)
-                if (m < K) o[m] = dwr_i[m] + part[t * KMAX + m];
+            for (int q = 0; q < KMAX / 4; ++q) {
+                if (4 * q < K) {
+                    const float4 pq = *reinterpret_cast<const float4 *>(part + t * KMAX + 4 * q);
+                    o[q] = make_float4(dwr_i[4 * q] + pq.x, dwr_i[4 * q + 1] + pq.y, dwr_i[4 * q + 2] + pq.z,
+                                       dwr_i[4 * q + 3] + pq.w);
+                }
+            }
         }
         sync_first256();  // part[] is reused below
         // ---- column pass (group g takes the rows of parity g of column k): intra dkappa.  Rows of
@@ -570,26 +586,28 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
 #pragma unroll
             for (int m = 0; m < KMAX; ++m) dk2[m] = 0.f;
             // direct rows: k's own 16-row quarter of the diagonal block (t >= k), rows of this
-            // group's parity
+            // group's parity.  Every lane walks the eight rows of its quarter of that parity (the
+            // same rows in a half-warp: broadcast reads); rows above the column (t < k) or past
+            // the chunk run with a zero decay exponent and a zero G H
             const bool left = (k & 31) < 16;
-            const int dend = min(n, 32 * J + (left ? 16 : 32));
-            for (int tt0 = k + ((k + grp) & 1); tt0 < dend; tt0 += 8) {
+            const int qs = 32 * J + (left ? 0 : 16) + grp;
 #pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    const int tt = tt0 + 2 * u;
-                    if (tt < dend) {
-                        const float dE = diff_f2(E_s[tt], Ek);
-                        const float gh = GHs[tt * XS + k];
+            for (int i = 0; i < 8; ++i) {
+                const int tt = qs + 2 * i;
+                const bool valid = tt >= k && tt < n;
+                const float dE = fmaxf(diff_f2(E_s[tt], Ek), 0.f);
+                const float gh = valid ? GHs[tt * XS + k] : 0.f;
+                const float4 w0 = *reinterpret_cast<const float4 *>(wr_s + tt * KMAX);
+                const float4 w1 = *reinterpret_cast<const float4 *>(wr_s + tt * KMAX + 4);
+                const float wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
 #pragma unroll
-                        for (int m = 0; m < KMAX; ++m) {
-                            if (m < K) {
-                                const float v = wr_s[tt * KMAX + m] * ex2_approx(-dE * l2r[m]);
-                                if (u & 1)
-                                    dk2[m] = fmaf(v, gh, dk2[m]);
-                                else
-                                    dk[m] = fmaf(v, gh, dk[m]);
-                            }
-                        }
+                for (int m = 0; m < KMAX; ++m) {
+                    if (m < K) {
+                        const float v = wv[m] * ex2_approx(-dE * l2r[m]);
+                        if (i & 1)
+                            dk2[m] = fmaf(v, gh, dk2[m]);
+                        else
+                            dk[m] = fmaf(v, gh, dk[m]);
                     }
                 }
             }
@@ -651,10 +669,16 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
         float *xtot = Vs;  // [128], free after the row pass
         if (!*abort_s) {
             float run = 0.f;
-            for (int j = 64 * grp; j < 64 * grp + 64; ++j) {
-                const float v = XX[t * XS + j];
-                XX[t * XS + j] = run;
-                run += v;
+#pragma unroll 2
+            for (int j0 = 64 * grp; j0 < 64 * grp + 64; j0 += 8) {
+                float v[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) v[i] = XX[t * XS + j0 + i];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    XX[t * XS + j0 + i] = run;
+                    run += v[i];
+                }
             }
             if (grp == 0) xtot[t] = run;
         }
@@ -665,22 +689,38 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
         float sr = 0.f;
         if (!*abort_s) {
             const int j = kcol;
-            for (int tp = j + ((j + grp) & 1); tp < n; tp += 2) {
-                sr += XX[tp * XS + j];
-                if (j >= 64) sr += xtot[tp];
+            const bool upper = j >= 64;  // uniform in a warp
+            float s4[4] = {0.f, 0.f, 0.f, 0.f};
+            int tp = j + ((j + grp) & 1);
+            for (; tp + 6 < n; tp += 8) {
+                float v[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) v[u] = XX[(tp + 2 * u) * XS + j];
+                if (upper) {
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) v[u] += xtot[tp + 2 * u];
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u) s4[u] += v[u];
             }
+            for (; tp < n; tp += 2) s4[0] += XX[tp * XS + j] + (upper ? xtot[tp] : 0.f);
+            sr = (s4[0] + s4[1]) + (s4[2] + s4[3]);
         }
         if (grp == 1) rpart[kcol] = sr;
         sync_first256();  // G H (in the C / B region) and the U copy (in the x tile) are read
         mbar_arrive(&bars[6]);  // the next item's C, B, x may load
         if (!*abort_s && grp == 0 && t < n) {
-            float *o = a.dkap_acc + blh(d, b, c0 + t, h) * K;
+            float4 *o = reinterpret_cast<float4 *>(a.dkap_acc + blh(d, b, c0 + t, h) * K);
 #pragma unroll
-            for (int m = 0; m < KMAX; ++m)
-                if (m < K) o[m] = dk[m] + part[t * KMAX + m];
+            for (int q = 0; q < KMAX / 4; ++q) {
+                if (4 * q < K) {
+                    const float4 pq = *reinterpret_cast<const float4 *>(part + t * KMAX + 4 * q);
+                    o[q] = make_float4(dk[4 * q] + pq.x, dk[4 * q + 1] + pq.y, dk[4 * q + 2] + pq.z,
+                                       dk[4 * q + 3] + pq.w);
+                }
+            }
             a.rect[blh(d, b, c0 + t, h)] = sr + rpart[t];
         }
-        sync_first256();
         if (!*abort_s && !mbar_wait(&bars[2], ph)) *abort_s = 1;
         sync_first256();
         tc_fence_after();
