@@ -7,14 +7,18 @@
 //   gated RMS normalisation   out = v / sqrt(mean_group(v^2) + eps) * weight,  v = y * silu(z)
 //        (before the output projection), and its backward.
 //
-// conv1d: a thread owns two adjacent channels and a run of kRun consecutive positions; a warp
-// covers 64 contiguous channels of one position per access.  The filter window of the last W-1
-// inputs stays in registers.  The backward streams g = du * act'(pre) through a register ring of
-// the last W values (dx_t needs g at t .. t+W-1), and reduces dw / dbias over the block's rows
-// of runs in shared memory before one atomic per channel and block.
-// RMSNorm: one CTA per row, 8-element vectors, per-group sums by shared-memory atomics.  The
-// backward is persistent over rows: each thread owns fixed feature positions, so its dweight
-// partials sit in shared memory without atomics until one global atomic per feature and CTA.
+// conv1d: a thread owns four adjacent channels (channel counts a multiple of 4; else two, else
+// one) and a run of kRun consecutive positions; a warp covers 128 contiguous channels of one
+// position per access, and the next batch of positions is loaded while the current one is
+// convolved.  The filter window of the last W-1 inputs stays in registers.  The backward streams
+// g = du * act'(pre) through a register ring of the last W values (dx_t needs g at t .. t+W-1),
+// and reduces dw / dbias over the block's rows of runs in shared memory before one atomic per
+// channel and block.
+// RMSNorm (dim <= 8192 forward, <= 4096 backward): a CTA per row holds the row in registers,
+// 8-element vectors per thread, so each row is read from HBM once; per-group sums by
+// shared-memory atomics.  The backward is persistent over rows, loads the next row while it
+// processes the current one, and keeps each thread's dweight partials in registers until one
+// global atomic per feature and CTA.  Wider rows take streaming kernels that re-read the row.
 #include <algorithm>
 #include <cstdio>
 
@@ -29,9 +33,14 @@ constexpr int kRun = 32;      // positions per thread (conv1d)
 constexpr int kRows = 8;      // runs per block (threadIdx.y)
 constexpr int kMaxW = 8;      // largest conv width
 
+// logistic sigmoid 1 / (1 + 2^(-a log2 e)) from the approximate hardware exp2 and reciprocal
+// (relative error ~1e-6 for |a| <= 20, well inside the float32 tolerance of the glue); for
+// a < -88 the exponential is +inf and its reciprocal 0, for large a the exponential is 0
 __device__ __forceinline__ float sigm(float a) {
-    const float e = expf(-fabsf(a));
-    return a >= 0.f ? 1.f / (1.f + e) : e / (1.f + e);
+    float e, r;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(e) : "f"(-1.4426950408889634f * a));
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(1.f + e));
+    return r;
 }
 __device__ __forceinline__ float silu_f(float a) { return a * sigm(a); }
 __device__ __forceinline__ float silu_grad_f(float a) {
@@ -297,6 +306,292 @@ __global__ void __launch_bounds__(32 * kRows) conv1d_bwd_kernel(ConvArgs a) {
     }
 }
 
+// Four adjacent channels of one position as loaded (bf16: 8 bytes, float32: 16 bytes).
+template <typename T> struct Raw4;
+template <> struct Raw4<__nv_bfloat16> {
+    uint2 u;
+    __device__ __forceinline__ void load(const __nv_bfloat16 *p) { u = *reinterpret_cast<const uint2 *>(p); }
+    __device__ __forceinline__ void get(float *v) const {
+        const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&u);
+        const float2 a = __bfloat1622float2(h[0]), b = __bfloat1622float2(h[1]);
+        v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y;
+    }
+    __device__ __forceinline__ void zero() { u = make_uint2(0u, 0u); }
+};
+template <> struct Raw4<float> {
+    float4 u;
+    __device__ __forceinline__ void load(const float *p) { u = *reinterpret_cast<const float4 *>(p); }
+    __device__ __forceinline__ void get(float *v) const { v[0] = u.x; v[1] = u.y; v[2] = u.z; v[3] = u.w; }
+    __device__ __forceinline__ void zero() { u = make_float4(0.f, 0.f, 0.f, 0.f); }
+};
+template <typename T> __device__ __forceinline__ void st4(T *p, const float *v);
+template <> __device__ __forceinline__ void st4<__nv_bfloat16>(__nv_bfloat16 *p, const float *v) {
+    uint2 u;
+    __nv_bfloat162 *h = reinterpret_cast<__nv_bfloat162 *>(&u);
+    h[0] = __floats2bfloat162_rn(v[0], v[1]);
+    h[1] = __floats2bfloat162_rn(v[2], v[3]);
+    *reinterpret_cast<uint2 *>(p) = u;
+}
+template <> __device__ __forceinline__ void st4<float>(float *p, const float *v) {
+    *reinterpret_cast<float4 *>(p) = make_float4(v[0], v[1], v[2], v[3]);
+}
+
+// The same convolution with four channels per thread (channels a multiple of 4, 4-element aligned
+// rows): a warp covers 128 contiguous channels of one position per access, and the inputs of the
+// next kB4 positions are loaded while the current ones are convolved, so every thread keeps two
+// batches of loads in flight.
+constexpr int kB4 = 8;
+
+template <typename T, int W>
+__global__ void __launch_bounds__(32 * kRows) conv1d_fwd4_kernel(ConvArgs a) {
+    const int c = 4 * (blockIdx.x * 32 + threadIdx.x);
+    const int t0 = (blockIdx.y * kRows + threadIdx.y) * kRun;
+    const int b = blockIdx.z;
+    if (c >= a.C || t0 >= a.L) return;
+    const T *xb = static_cast<const T *>(a.x) + size_t(b) * a.L * a.C + c;
+    float w[4][W], bs[4], win[4][W];  // win[k][j] = input at t - (W-1) + j, channel c + k
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+#pragma unroll
+        for (int j = 0; j < W; ++j) w[k][j] = a.w[(c + k) * W + j];
+        bs[k] = a.bias ? a.bias[c + k] : 0.f;
+    }
+#pragma unroll
+    for (int j = 0; j < W - 1; ++j) {
+        const int t = t0 - (W - 1) + j;
+        if (t >= 0) {
+            Raw4<T> r;
+            r.load(xb + size_t(t) * a.C);
+            float v[4];
+            r.get(v);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) win[k][j] = v[k];
+        } else {
+#pragma unroll
+            for (int k = 0; k < 4; ++k) win[k][j] = x_at<T>(a, b, t, c + k);
+        }
+    }
+    const int t1 = min(t0 + kRun, a.L);
+    Raw4<T> cur[kB4], nxt[kB4];
+#pragma unroll
+    for (int i = 0; i < kB4; ++i) {
+        if (t0 + i < t1) cur[i].load(xb + size_t(t0 + i) * a.C);
+        else cur[i].zero();
+    }
+    for (int tb = t0; tb < t1; tb += kB4) {
+#pragma unroll
+        for (int i = 0; i < kB4; ++i) {  // the next batch, in flight while this one is convolved
+            const int t = tb + kB4 + i;
+            if (t < t1) nxt[i].load(xb + size_t(t) * a.C);
+            else nxt[i].zero();
+        }
+#pragma unroll
+        for (int i = 0; i < kB4; ++i) {
+            const int t = tb + i;
+            if (t < t1) {
+                float xv[4], p[4];
+                cur[i].get(xv);
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    win[k][W - 1] = xv[k];
+                    p[k] = bs[k];
+#pragma unroll
+                    for (int j = 0; j < W; ++j) p[k] = fmaf(w[k][j], win[k][j], p[k]);
+                    if (a.silu) p[k] = silu_f(p[k]);
+                }
+                st4<T>(static_cast<T *>(a.u) + (size_t(b) * a.L + t) * a.C + c, p);
+                if (a.state_out && t >= a.L - (W - 1)) {  // the last W-1 inputs become the carried state
+                    T *so = static_cast<T *>(a.state_out);
+                    const int ks = t - (a.L - (W - 1));
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) so[(size_t(b) * a.C + c + k) * (W - 1) + ks] = from_f<T>(xv[k]);
+                }
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+#pragma unroll
+                    for (int j = 0; j < W - 1; ++j) win[k][j] = win[k][j + 1];
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < kB4; ++i) cur[i] = nxt[i];
+    }
+    if (a.state_out && t0 == 0 && a.L < W - 1) {  // short sequence: part of the old state stays
+        T *so = static_cast<T *>(a.state_out);
+        for (int ks = 0; ks < W - 1 - a.L; ++ks)
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+                so[(size_t(b) * a.C + c + k) * (W - 1) + ks] = from_f<T>(x_at<T>(a, b, ks + a.L - (W - 1), c + k));
+    }
+}
+
+constexpr int kB4b = 4;  // positions per batch of the backward (two streams in flight)
+
+// r[idx] for a run-time idx by unrolled selects, so that the ring stays in registers
+template <int W>
+__device__ __forceinline__ float ring_at(const float (&r)[W], int idx) {
+    float v = 0.f;
+#pragma unroll
+    for (int i = 0; i < W; ++i) v = i == idx ? r[i] : v;
+    return v;
+}
+
+template <typename T, int W>
+__global__ void __launch_bounds__(32 * kRows, 2) conv1d_bwd4_kernel(ConvArgs a) {
+    __shared__ float red[kRows][W + 1][128];  // per run row: dw taps and dbias of the 128 channels
+    const int lane = threadIdx.x, ry = threadIdx.y;
+    const int c = 4 * (blockIdx.x * 32 + lane);
+    const int t0 = (blockIdx.y * kRows + ry) * kRun;
+    const int b = blockIdx.z;
+    const bool active = c < a.C && t0 < a.L;
+    float acc[4][W + 1];  // dw taps, then dbias
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+#pragma unroll
+        for (int j = 0; j <= W; ++j) acc[k][j] = 0.f;
+    if (active) {
+        const size_t rowb = size_t(b) * a.L * a.C + c;
+        const T *xb = static_cast<const T *>(a.x) + rowb;
+        const T *db = static_cast<const T *>(a.du) + rowb;
+        T *dxb = static_cast<T *>(a.dx) + rowb;
+        float w[4][W], bs[4], win[4][W], g[4][W];  // inputs t-(W-1) .. t; g at t-(W-1) .. t
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+#pragma unroll
+            for (int j = 0; j < W; ++j) {
+                w[k][j] = a.w[(c + k) * W + j];
+                g[k][j] = 0.f;
+            }
+            bs[k] = a.bias ? a.bias[c + k] : 0.f;
+        }
+#pragma unroll
+        for (int j = 0; j < W - 1; ++j)
+#pragma unroll
+            for (int k = 0; k < 4; ++k) win[k][j] = x_at<T>(a, b, t0 - (W - 1) + j, c + k);
+        const int tr = min(t0 + kRun, a.L);   // this run's positions: [t0, tr)
+        const int tg = min(tr + W - 1, a.L);  // g is needed up to tg - 1 for dx of the run
+        Raw4<T> cx[kB4b], cd[kB4b], nx[kB4b], nd[kB4b];
+#pragma unroll
+        for (int i = 0; i < kB4b; ++i) {
+            if (t0 + i < tg) {
+                cx[i].load(xb + size_t(t0 + i) * a.C);
+                cd[i].load(db + size_t(t0 + i) * a.C);
+            } else {
+                cx[i].zero();
+                cd[i].zero();
+            }
+        }
+        for (int tb = t0; tb < tg; tb += kB4b) {
+#pragma unroll
+            for (int i = 0; i < kB4b; ++i) {
+                const int t = tb + kB4b + i;
+                if (t < tg) {
+                    nx[i].load(xb + size_t(t) * a.C);
+                    nd[i].load(db + size_t(t) * a.C);
+                } else {
+                    nx[i].zero();
+                    nd[i].zero();
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < kB4b; ++i) {
+                const int t = tb + i;
+                if (t < tg) {
+                    float xv[4], dv[4];
+                    cx[i].get(xv);
+                    cd[i].get(dv);
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        win[k][W - 1] = xv[k];
+                        float p = bs[k];
+#pragma unroll
+                        for (int j = 0; j < W; ++j) p = fmaf(w[k][j], win[k][j], p);
+                        const float gg = a.silu ? dv[k] * silu_grad_f(p) : dv[k];
+#pragma unroll
+                        for (int j = 0; j < W - 1; ++j) g[k][j] = g[k][j + 1];
+                        g[k][W - 1] = gg;
+                        if (t < tr) {  // this run's own positions: dw and dbias terms
+#pragma unroll
+                            for (int j = 0; j < W; ++j) acc[k][j] = fmaf(gg, win[k][j], acc[k][j]);
+                            acc[k][W] += gg;
+                        }
+                    }
+                    // dx at s = t - (W-1) (all of its g are in the ring once t = s + W - 1)
+                    const int s = t - (W - 1);
+                    if (s >= t0) {
+                        float dx[4];
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            dx[k] = 0.f;
+#pragma unroll
+                            for (int j = 0; j < W; ++j) dx[k] = fmaf(w[k][j], g[k][W - 1 - j], dx[k]);
+                        }
+                        st4<T>(dxb + size_t(s) * a.C, dx);
+                    }
+                    if (a.dstate && t0 == 0 && t == min(W - 2, a.L - 1)) {
+                        // gradient of the carried inputs i = 0 .. W-2 (position i - (W-1)):
+                        // sum over taps j <= i of w_j g[i - j], g[tt] at ring slot W-1-(t-tt)
+                        T *ds = static_cast<T *>(a.dstate);
+                        for (int ii = 0; ii < W - 1; ++ii) {
+#pragma unroll
+                            for (int k = 0; k < 4; ++k) {
+                                float d = 0.f;
+#pragma unroll
+                                for (int j = 0; j < W; ++j) {
+                                    const int tt = ii - j;
+                                    if (j <= ii && tt <= t) d = fmaf(w[k][j], ring_at<W>(g[k], W - 1 - (t - tt)), d);
+                                }
+                                ds[(size_t(b) * a.C + c + k) * (W - 1) + ii] = from_f<T>(d);
+                            }
+                        }
+                    }
+#pragma unroll
+                    for (int k = 0; k < 4; ++k)
+#pragma unroll
+                        for (int j = 0; j < W - 1; ++j) win[k][j] = win[k][j + 1];
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < kB4b; ++i) {
+                cx[i] = nx[i];
+                cd[i] = nd[i];
+            }
+        }
+        // the run's tail positions s in [max(t0, tg - (W-1)), tr): the g beyond the end are 0
+        for (int s = max(t0, tg - (W - 1)); s < tr; ++s) {
+            const int sh = (tg - 1) - s;  // g at s + kk sits at ring slot W-1-(tg-1-(s+kk))
+            float dx[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                dx[k] = 0.f;
+#pragma unroll
+                for (int j = 0; j < W; ++j) {
+                    const int kk = (W - 1) - j;  // tap j reads g at s + kk
+                    if (kk <= sh) dx[k] = fmaf(w[k][j], ring_at<W>(g[k], W - 1 - (sh - kk)), dx[k]);
+                }
+            }
+            st4<T>(dxb + size_t(s) * a.C, dx);
+        }
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+#pragma unroll
+        for (int j = 0; j <= W; ++j) red[ry][j][4 * lane + k] = acc[k][j];
+    __syncthreads();
+    // one atomic per channel and tap: threads (lane, ry) split the (W + 1) x 128 sums
+    for (int q = ry * 32 + lane; q < (W + 1) * 128; q += 32 * kRows) {
+        const int j = q / 128, cc = q % 128;
+        const int ch = blockIdx.x * 128 + cc;
+        if (ch >= a.C) continue;
+        float sum = 0.f;
+#pragma unroll
+        for (int r = 0; r < kRows; ++r) sum += red[r][j][cc];
+        if (j < W)
+            atomicAdd(a.dw + ch * W + j, sum);
+        else if (a.dbias)
+            atomicAdd(a.dbias + ch, sum);
+    }
+}
+
 // one decode step: window = carried state (W-1 inputs) then x_t; the state shifts by one
 template <typename T>
 __global__ void __launch_bounds__(256) conv1d_step_kernel(ConvArgs a, const T *__restrict__ xt, T *__restrict__ ut) {
@@ -496,17 +791,272 @@ __global__ void __launch_bounds__(256) rmsnorm_bwd_kernel(NormArgs a) {
         atomicAdd(a.dweight + 8 * (q % (a.D / 8)) + q / (a.D / 8), dwp[q]);
 }
 
+// Register-resident rows (dim <= 8192): a CTA of NT threads per row, thread i owning the 8-feature
+// vectors at 8 (i + NT j), j < VPT, so a row is read from HBM once, with every load of the row in
+// flight at the same time, and never re-read.  Group sums as in the kernels above (smem, one shared atomic per warp when
+// groups span whole warps).  Two sum buffers alternate between consecutive rows of a CTA, so a
+// row needs no barrier after its last use of the sums.
+template <typename T, int VPT, int NT>
+__global__ void __launch_bounds__(NT) rmsnorm_fwd_reg_kernel(NormArgs a) {
+    extern __shared__ float gsum2[];  // [2][ng]
+    const int ng = a.D / a.gs;
+    int par = 0;
+    for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x, par ^= 1) {
+        float *gsum = gsum2 + par * ng;
+        float v[VPT][8];
+#pragma unroll
+        for (int j = 0; j < VPT; ++j) {
+            const int f = 8 * (threadIdx.x + NT * j);
+            if (f < a.D) {
+                float zv[8];
+                gated8<T>(a, r, f, v[j], zv);
+            }
+        }
+        for (int g = threadIdx.x; g < ng; g += blockDim.x) gsum[g] = 0.f;
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < VPT; ++j) {
+            const int f = 8 * (threadIdx.x + NT * j);
+            const bool valid = f < a.D;
+            float sq = 0.f;
+            if (valid)
+#pragma unroll
+                for (int i = 0; i < 8; ++i) sq = fmaf(v[j][i], v[j][i], sq);
+            if (8 * NT * j < a.D) group_add(gsum, f, a.gs, valid, sq);  // whole warps take part
+        }
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < VPT; ++j) {
+            const int f = 8 * (threadIdx.x + NT * j);
+            if (f < a.D) {
+                const float inv = rsqrtf(gsum[f / a.gs] / a.gs + a.eps);
+                const float4 w0 = reinterpret_cast<const float4 *>(a.weight + f)[0];
+                const float4 w1 = reinterpret_cast<const float4 *>(a.weight + f)[1];
+                const float wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+#pragma unroll
+                for (int i = 0; i < 8; ++i) v[j][i] = v[j][i] * inv * wv[i];
+                st8<T>(static_cast<T *>(a.out) + r * a.D + f, v[j]);
+            }
+        }
+    }
+}
+
+// Eight elements of a row kept as loaded (bf16: one 16-byte register quad), unpacked on use.
+template <typename T> struct Raw8;
+template <> struct Raw8<__nv_bfloat16> {
+    uint4 u;
+    __device__ __forceinline__ void load(const __nv_bfloat16 *p) { u = *reinterpret_cast<const uint4 *>(p); }
+    __device__ __forceinline__ void get(float *v) const {
+        const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&u);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 f = __bfloat1622float2(h[i]);
+            v[2 * i] = f.x;
+            v[2 * i + 1] = f.y;
+        }
+    }
+};
+template <> struct Raw8<float> {
+    float4 a, b;
+    __device__ __forceinline__ void load(const float *p) {
+        a = reinterpret_cast<const float4 *>(p)[0];
+        b = reinterpret_cast<const float4 *>(p)[1];
+    }
+    __device__ __forceinline__ void get(float *v) const {
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    }
+};
+
+// Backward with register-resident rows, persistent over rows: y, z and dout stay as loaded, the
+// gate's sigmoid is evaluated once per element (silu(z) = z s, silu'(z) = s (1 + z (1 - s))), and
+// each thread keeps the dweight partials of its own features in registers until one global atomic
+// per feature and CTA.
+template <typename T, int VPT, int NT>
+__global__ void __launch_bounds__(NT, NT <= 256 ? 2 : 1) rmsnorm_bwd_reg_kernel(NormArgs a) {
+    extern __shared__ float sums[];  // [2][2 ng]: sum(v^2), then sum(dn n), per row parity
+    const int ng = a.D / a.gs;
+    const bool gated = a.z != nullptr;
+    float dwp[VPT][8];
+#pragma unroll
+    for (int j = 0; j < VPT; ++j)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) dwp[j][i] = 0.f;
+    // the next row's inputs are loaded while the current row is processed
+    Raw8<T> ry[VPT], rz[VPT], rg[VPT], ny[VPT], nz[VPT], nd[VPT];
+    auto fetch = [&](int64_t row, Raw8<T> *yy, Raw8<T> *zz, Raw8<T> *dd) {
+#pragma unroll
+        for (int j = 0; j < VPT; ++j) {
+            const int f = 8 * (threadIdx.x + NT * j);
+            if (f < a.D) {
+                const size_t o = size_t(row) * a.D + f;
+                yy[j].load(static_cast<const T *>(a.y) + o);
+                if (gated) zz[j].load(static_cast<const T *>(a.z) + o);
+                dd[j].load(static_cast<const T *>(a.dout) + o);
+            }
+        }
+    };
+    if (blockIdx.x < a.R) fetch(blockIdx.x, ry, rz, rg);
+    int par = 0;
+    for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x, par ^= 1) {
+        float *ssq = sums + par * 2 * ng, *dot = ssq + ng;
+        if (r + gridDim.x < a.R) fetch(r + gridDim.x, ny, nz, nd);
+        for (int g = threadIdx.x; g < 2 * ng; g += blockDim.x) ssq[g] = 0.f;
+        __syncthreads();
+        float sg[VPT][8];  // sigmoid(z) of the gate; the gate factor is silu(z) = z sg (1 without the gate)
+#pragma unroll
+        for (int j = 0; j < VPT; ++j) {
+            const int f = 8 * (threadIdx.x + NT * j);
+            const bool valid = f < a.D;
+            float sq = 0.f;
+            if (valid) {
+                float y[8], z[8];
+                ry[j].get(y);
+                if (gated) rz[j].get(z);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    sg[j][i] = gated ? sigm(z[i]) : 1.f;
+                    const float v = y[i] * (gated ? z[i] * sg[j][i] : 1.f);
+                    sq = fmaf(v, v, sq);
+                }
+            }
+            if (8 * NT * j < a.D) group_add(ssq, f, a.gs, valid, sq);  // whole warps take part
+        }
+        __syncthreads();
+        float iv[VPT];
+#pragma unroll
+        for (int j = 0; j < VPT; ++j) {
+            const int f = 8 * (threadIdx.x + NT * j);
+            const bool valid = f < a.D;
+            float sd = 0.f;
+            iv[j] = 0.f;
+            if (valid) {
+                iv[j] = rsqrtf(ssq[f / a.gs] / a.gs + a.eps);
+                float y[8], go[8], z[8];
+                ry[j].get(y);
+                rg[j].get(go);
+                if (gated) rz[j].get(z);
+                const float4 w0 = reinterpret_cast<const float4 *>(a.weight + f)[0];
+                const float4 w1 = reinterpret_cast<const float4 *>(a.weight + f)[1];
+                const float wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const float n = y[i] * (gated ? z[i] * sg[j][i] : 1.f) * iv[j];
+                    dwp[j][i] = fmaf(go[i], n, dwp[j][i]);
+                    sd = fmaf(go[i] * wv[i], n, sd);
+                }
+            }
+            if (8 * NT * j < a.D) group_add(dot, f, a.gs, valid, sd);
+        }
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < VPT; ++j) {
+            const int f = 8 * (threadIdx.x + NT * j);
+            if (f < a.D) {
+                const float m = dot[f / a.gs] / a.gs;
+                float y[8], go[8], dyv[8], dzv[8];
+                ry[j].get(y);
+                rg[j].get(go);
+                const float4 w0 = reinterpret_cast<const float4 *>(a.weight + f)[0];
+                const float4 w1 = reinterpret_cast<const float4 *>(a.weight + f)[1];
+                const float wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+                float z[8];
+                if (gated) rz[j].get(z);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const float gz = (gated ? z[i] * sg[j][i] : 1.f);
+                    const float n = y[i] * gz * iv[j];
+                    const float dv = (go[i] * wv[i] - n * m) * iv[j];  // (dn - n mean(dn n)) / rms
+                    dyv[i] = dv * gz;
+                    dzv[i] = gated ? dv * y[i] * (sg[j][i] * (1.f + z[i] * (1.f - sg[j][i]))) : 0.f;
+                }
+                const size_t o = size_t(r) * a.D + f;
+                st8<T>(static_cast<T *>(a.dy) + o, dyv);
+                if (gated) st8<T>(static_cast<T *>(a.dz) + o, dzv);
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < VPT; ++j) {
+            ry[j] = ny[j];
+            rz[j] = nz[j];
+            rg[j] = nd[j];
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < VPT; ++j) {
+        const int f = 8 * (threadIdx.x + NT * j);
+        if (f < a.D)
+#pragma unroll
+            for (int i = 0; i < 8; ++i) atomicAdd(a.dweight + f + i, dwp[j][i]);
+    }
+}
+
 int num_sms() {
     int dev = 0, sms = 152;
     if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     return std::max(sms, 1);
 }
 
+// Register-resident RMSNorm launches.  Forward (dim <= 8192): CTAs of 256 threads, VPT = ceil(dim /
+// 2048) vectors per thread (measured faster at dim 4096 than 512 threads of one vector).  Backward
+// (dim <= 4096): one vector per thread in CTAs of 256 or 512 threads, persistent, as many CTAs as
+// the SMs hold at once.
+template <typename T, int VPT>
+cudaError_t norm_fwd_reg_launch(const NormArgs &a, cudaStream_t st) {
+    const size_t smem = sizeof(float) * 2 * (a.D / a.gs);
+    const int blocks = int(std::min<int64_t>(a.R, int64_t(num_sms()) * 16));
+    trace_begin("gated_rmsnorm_fwd", st);
+    rmsnorm_fwd_reg_kernel<T, VPT, 256><<<blocks, 256, smem, st>>>(a);
+    trace_end(st);
+    return cudaGetLastError();
+}
+
+template <typename T, int NT>
+cudaError_t norm_reg_launch(const NormArgs &a, bool bwd, cudaStream_t st) {
+    const int ng = a.D / a.gs;
+    if (!bwd) {
+        switch ((a.D + 2047) / 2048) {
+            case 1: return norm_fwd_reg_launch<T, 1>(a, st);
+            case 2: return norm_fwd_reg_launch<T, 2>(a, st);
+            case 3: return norm_fwd_reg_launch<T, 3>(a, st);
+            default: return norm_fwd_reg_launch<T, 4>(a, st);
+        }
+    }
+    const size_t smem = sizeof(float) * 4 * ng;
+    auto k = rmsnorm_bwd_reg_kernel<T, 1, NT>;
+    int per_sm = 0;
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, NT, smem);
+    if (e != cudaSuccess) return e;
+    const int blocks = int(std::min<int64_t>(a.R, int64_t(num_sms()) * std::max(per_sm, 1)));
+    trace_begin("gated_rmsnorm_bwd", st);
+    k<<<blocks, NT, smem, st>>>(a);
+    trace_end(st);
+    return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t norm_reg(const NormArgs &a, bool bwd, cudaStream_t st) {
+    if (a.D <= 8 * 256) return norm_reg_launch<T, 256>(a, bwd, st);
+    if (a.D <= 8 * 512) return norm_reg_launch<T, 512>(a, bwd, st);
+    return norm_reg_launch<T, 512>(a, false, st);  // forward only: the backward stops at 4096
+}
+constexpr int kNormRegMaxDim = 8192, kNormRegMaxDimBwd = 4096;
+
 template <typename T, int W>
-cudaError_t conv_launch_w(const ConvArgs &a, bool bwd, bool vec, cudaStream_t st) {
+cudaError_t conv_launch_w(const ConvArgs &a, bool bwd, bool vec, bool vec4, cudaStream_t st) {
     dim3 block(32, kRows);
     dim3 grid((a.C + 63) / 64, (a.L + kRows * kRun - 1) / (kRows * kRun), a.B);
     if (grid.y == 0) return cudaSuccess;
+    if (vec4 && (!bwd || W <= 4)) {  // four channels per thread: 128 channels per block column
+                                     // (the backward of wider filters keeps two channels)
+        grid.x = (a.C + 127) / 128;
+        trace_begin(bwd ? "conv1d_bwd" : "conv1d_fwd", st);
+        if constexpr (W <= 4) {
+            if (bwd) conv1d_bwd4_kernel<T, W><<<grid, block, 0, st>>>(a);
+        }
+        if (!bwd) conv1d_fwd4_kernel<T, W><<<grid, block, 0, st>>>(a);
+        trace_end(st);
+        return cudaGetLastError();
+    }
     if (!bwd) {
         trace_begin("conv1d_fwd", st);
         if (vec) conv1d_fwd_kernel<T, W, true><<<grid, block, 0, st>>>(a);
@@ -521,16 +1071,16 @@ cudaError_t conv_launch_w(const ConvArgs &a, bool bwd, bool vec, cudaStream_t st
 }
 
 template <typename T>
-cudaError_t conv_launch(const ConvArgs &a, bool bwd, bool vec, cudaStream_t st) {
+cudaError_t conv_launch(const ConvArgs &a, bool bwd, bool vec, bool vec4, cudaStream_t st) {
     switch (a.W) {
-        case 1: return conv_launch_w<T, 1>(a, bwd, vec, st);
-        case 2: return conv_launch_w<T, 2>(a, bwd, vec, st);
-        case 3: return conv_launch_w<T, 3>(a, bwd, vec, st);
-        case 4: return conv_launch_w<T, 4>(a, bwd, vec, st);
-        case 5: return conv_launch_w<T, 5>(a, bwd, vec, st);
-        case 6: return conv_launch_w<T, 6>(a, bwd, vec, st);
-        case 7: return conv_launch_w<T, 7>(a, bwd, vec, st);
-        default: return conv_launch_w<T, 8>(a, bwd, vec, st);
+        case 1: return conv_launch_w<T, 1>(a, bwd, vec, vec4, st);
+        case 2: return conv_launch_w<T, 2>(a, bwd, vec, vec4, st);
+        case 3: return conv_launch_w<T, 3>(a, bwd, vec, vec4, st);
+        case 4: return conv_launch_w<T, 4>(a, bwd, vec, vec4, st);
+        case 5: return conv_launch_w<T, 5>(a, bwd, vec, vec4, st);
+        case 6: return conv_launch_w<T, 6>(a, bwd, vec, vec4, st);
+        case 7: return conv_launch_w<T, 7>(a, bwd, vec, vec4, st);
+        default: return conv_launch_w<T, 8>(a, bwd, vec, vec4, st);
     }
 }
 
@@ -625,8 +1175,9 @@ frac_status frac_conv1d_fwd(const frac_conv_dims *dims, const void *x, const flo
                                "frac_conv1d_fwd");
     }
     const bool vec = a.C % 2 == 0 && frac::aligned(x, 2 * es) && frac::aligned(u, 2 * es);
-    return frac::glue_cuda(dims->dtype == FRAC_DTYPE_BF16 ? frac::conv_launch<__nv_bfloat16>(a, false, vec, st)
-                                                          : frac::conv_launch<float>(a, false, vec, st),
+    const bool vec4 = a.C % 4 == 0 && frac::aligned(x, 4 * es) && frac::aligned(u, 4 * es);
+    return frac::glue_cuda(dims->dtype == FRAC_DTYPE_BF16 ? frac::conv_launch<__nv_bfloat16>(a, false, vec, vec4, st)
+                                                          : frac::conv_launch<float>(a, false, vec, vec4, st),
                            "frac_conv1d_fwd");
 }
 
@@ -662,8 +1213,10 @@ frac_status frac_conv1d_bwd(const frac_conv_dims *dims, const void *x, const flo
     if (e == cudaSuccess && a.L > 0) {
         const bool vec = a.C % 2 == 0 && frac::aligned(x, 2 * es) && frac::aligned(du, 2 * es) &&
                          frac::aligned(dx, 2 * es);
-        e = dims->dtype == FRAC_DTYPE_BF16 ? frac::conv_launch<__nv_bfloat16>(a, true, vec, st)
-                                           : frac::conv_launch<float>(a, true, vec, st);
+        const bool vec4 = a.C % 4 == 0 && frac::aligned(x, 4 * es) && frac::aligned(du, 4 * es) &&
+                          frac::aligned(dx, 4 * es);
+        e = dims->dtype == FRAC_DTYPE_BF16 ? frac::conv_launch<__nv_bfloat16>(a, true, vec, vec4, st)
+                                           : frac::conv_launch<float>(a, true, vec, vec4, st);
     }
     return frac::glue_cuda(e, "frac_conv1d_bwd");
 }
@@ -711,6 +1264,10 @@ frac_status frac_gated_rmsnorm_fwd(const frac_norm_dims *dims, const void *y, co
     a.R = dims->rows; a.D = int(dims->dim); a.gs = int(dims->group_size); a.eps = dims->eps;
     a.y = y; a.z = z; a.weight = weight; a.out = out;
     cudaStream_t st = (cudaStream_t)stream;
+    if (a.D <= frac::kNormRegMaxDim)
+        return frac::glue_cuda(dims->dtype == FRAC_DTYPE_BF16 ? frac::norm_reg<__nv_bfloat16>(a, false, st)
+                                                              : frac::norm_reg<float>(a, false, st),
+                               "frac_gated_rmsnorm_fwd");
     const int blocks = int(std::min<int64_t>(a.R, int64_t(frac::num_sms()) * 16));
     const size_t smem = sizeof(float) * (a.D / a.gs);
     frac::trace_begin("gated_rmsnorm_fwd", st);
@@ -742,7 +1299,10 @@ frac_status frac_gated_rmsnorm_bwd(const frac_norm_dims *dims, const void *y, co
     a.y = y; a.z = z; a.dout = dout; a.weight = weight; a.dy = dy; a.dz = dz; a.dweight = dweight;
     cudaStream_t st = (cudaStream_t)stream;
     cudaError_t e = cudaMemsetAsync(dweight, 0, sizeof(float) * a.D, st);
-    if (e == cudaSuccess && a.R > 0) {
+    if (e == cudaSuccess && a.R > 0 && a.D <= frac::kNormRegMaxDimBwd) {
+        e = dims->dtype == FRAC_DTYPE_BF16 ? frac::norm_reg<__nv_bfloat16>(a, true, st)
+                                           : frac::norm_reg<float>(a, true, st);
+    } else if (e == cudaSuccess && a.R > 0) {
         const int blocks = int(std::min<int64_t>(a.R, int64_t(frac::num_sms()) * 4));
         const size_t smem = sizeof(float) * (a.D + 2 * (a.D / a.gs));
         auto k16 = frac::rmsnorm_bwd_kernel<__nv_bfloat16>;

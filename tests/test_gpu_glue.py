@@ -3,8 +3,9 @@ against the fp64 oracle (oracle/mixer_glue.py), through the C ABI.
 
 Tolerances as for the scan: relative L2 per output <= 1e-5 float32, <= 1e-2 bf16.  The conv
 cases cover lengths inside, at and across the 32-position runs of a thread (1, 31, 33, 300),
-widths 1 to 8, odd channel counts (the scalar path), the carried state and SiLU on and off; the
-norm cases cover gated and ungated rows and several group sizes.
+widths 1 to 8, channel counts that take two or four channels per thread or the scalar path, the
+carried state and SiLU on and off; the norm cases cover gated and ungated rows, several group
+sizes, and rows held in registers (dim <= 8192 forward, <= 4096 backward) or streamed.
 """
 import numpy as np
 import pytest
@@ -43,8 +44,9 @@ def _conv_case(B, L, C, W, dtype, silu, with_state, seed=0):
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("L", [1, 31, 33, 300])
-def test_conv_lengths(dtype, L):
-    _conv_case(2, L, 70, 4, dtype, silu=True, with_state=True, seed=L)
+@pytest.mark.parametrize("C", [70, 72])  # two channels per thread / four channels per thread
+def test_conv_lengths(dtype, L, C):
+    _conv_case(2, L, C, 4, dtype, silu=True, with_state=True, seed=L)
 
 
 @pytest.mark.parametrize("W", [1, 2, 3, 5, 8])
@@ -104,7 +106,7 @@ def _norm_case(R, D, gs, dtype, gated, seed=0):
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("gated", [False, True])
-@pytest.mark.parametrize("D,gs", [(64, 64), (256, 32), (1032, 8)])
+@pytest.mark.parametrize("D,gs", [(64, 64), (256, 32), (1032, 8), (4096, 512), (6000, 600), (8200, 1640)])
 def test_rmsnorm_shapes(dtype, gated, D, gs):
     _norm_case(37, D, gs, dtype, gated, seed=D + gs)
 
