@@ -167,6 +167,13 @@ def train_flops_per_token_head(s, q=128):
     return 14 * kpn(s) + 3 * q * s.headdim + 2 * q * s.dstate * s.ngroups / s.nheads
 
 
+def intra_pair_flops_per_token_head(s, q=128):
+    """FP32 work of the intra-chunk backward by its definition: for each pair k <= t of a chunk
+    ((q + 1) / 2 pairs per token) and each mode, the decay factor's contributions to Gamma,
+    Gamma', the read-weight gradient and the kappa gradient, one multiply-add (2 flops) each."""
+    return (q + 1) / 2 * s.nmodes * 8
+
+
 def fwd_bytes_per_token_head(s):
     """Algorithmic bytes of the forward per token-head: x and y, the three controls, the two
     weight rows, and B, C shared by the group's heads."""
@@ -175,19 +182,30 @@ def fwd_bytes_per_token_head(s):
 
 
 # DRAM bytes (read + write) per launch of each tensor-core kernel from one ncu capture of the
-# training shape at batch 2 (the ncu summary of these kernels kept under profiles/); the
-# per-chunk state traffic grows in proportion to the batch, so a run at batch B reports
-# bytes x B / 2.  A figure is used only while the kernel's sources hash to the digest they had
-# when they were profiled.
+# training shape at batch 2 (dram__bytes_read.sum + dram__bytes_write.sum of every launch of the
+# step, averaged; the summary is kept under profiles/); the per-chunk state traffic grows in
+# proportion to the batch, so a run at batch B reports bytes x B / 2.  A figure is used only while
+# the kernel's sources hash to the digest they had when they were profiled.
 PROFILED_TRAFFIC_BATCH = 2
 PROFILED_TRAFFIC = {
-    "coef_tc": ("scan_tc.cu", "900e85af153e741a", 23.101e6 + 41.631e6),
-    "state_pass_fwd_tc": ("scan_tc.cu", "900e85af153e741a", 138.760e6 + 481.840e6),
-    "chunk_fwd_tc": ("scan_tc.cu", "900e85af153e741a", 717.318e6 + 60.756e6),
-    "state_pass_rev_tc": ("scan_tc.cu", "900e85af153e741a", 139.129e6 + 482.585e6),
-    "bwd_intra_tc": ("scan_tc_bwd.cu", "a135ecad70d3c440", 182.952e6 + 126.667e6),
-    "bwd_state_tc": ("scan_tc_bwd.cu", "a135ecad70d3c440", 1464.175e6 + 165.234e6),
-    "bwd_final_tc": ("scan_tc_bwd.cu", "a135ecad70d3c440", 323.524e6 + 70.281e6),
+    "coef_tc": ("scan_tc.cu", "7389ea60990165f0", 23.10e6 + 38.92e6),
+    "state_pass_fwd_tc": ("scan_tc.cu", "7389ea60990165f0", 138.80e6 + 479.22e6),
+    "chunk_fwd_tc": ("scan_tc.cu", "7389ea60990165f0", 717.32e6 + 57.95e6),
+    "state_pass_rev_tc": ("scan_tc.cu", "7389ea60990165f0", 139.26e6 + 479.18e6),
+    "bwd_intra_tc": ("scan_tc_bwd.cu", "627544f5ba419d34", 182.99e6 + 123.75e6),
+    "bwd_state_tc": ("scan_tc_bwd.cu", "627544f5ba419d34", 1466.46e6 + 166.23e6),
+    "bwd_final_tc": ("scan_tc_bwd.cu", "627544f5ba419d34", 323.48e6 + 67.26e6),
+}
+
+# DRAM bytes (read + write) per launch of the scan-parameter and mixer-glue kernels at the
+# benchmark's training shape (B8 L4096), from one ncu capture of bench.py's mixer section.
+PROFILED_MIXER_TRAFFIC = {
+    "param_prep_fwd": ("param_prep.cu", "296e863496dae618", 92.31e6 + 43.92e6),
+    "param_prep_bwd": ("param_prep.cu", "296e863496dae618", 184.62e6 + 64.71e6),
+    "conv1d_fwd": ("mixer_glue.cu", "eca11e4487de8cc6", 285.37e6 + 236.23e6),
+    "conv1d_bwd": ("mixer_glue.cu", "eca11e4487de8cc6", 570.77e6 + 253.83e6),
+    "gated_rmsnorm_fwd": ("mixer_glue.cu", "eca11e4487de8cc6", 536.96e6 + 235.98e6),
+    "gated_rmsnorm_bwd": ("mixer_glue.cu", "eca11e4487de8cc6", 805.42e6 + 497.52e6),
 }
 
 # DRAM bytes (read + write) of one decode_step launch of the decode workload (B128 H64 P64 N128
@@ -487,6 +505,10 @@ def bench_train(args, ctx, rank, local):
                 "bf16_tflops_sustained", peaks.get("bf16_tflops"))
         elif kind == "bytes":
             kern[k]["achieved_gbs"] = work / (kern[k]["avg_ms"] / 1e3) / 1e9
+    if "bwd_intra_tc" in kern:  # its real bound: the per-pair FP32 work on the CUDA cores
+        kern["bwd_intra_tc"]["roofline_alu"] = roofline_of(
+            "bwd_intra_tc", "flops_alu", intra_pair_flops_per_token_head(s) * units,
+            kern["bwd_intra_tc"]["avg_ms"], peaks)
     dom = dominant(trace)
     roofline = None
     if dom:
@@ -767,9 +789,15 @@ def bench_mixer(ctx):
     rows = B * L * H
 
     def add(name, fn, nbytes):
+        # the call's time through the Python API, and the kernel's own device time (CUDA events
+        # around its launch on the stream), which the roofline takes
         ms, trace = ctx.time(fn, 10)
-        out[name] = {"ms": ms, "gpu_launches_per_call": sum(c for c, _ in trace.values()) / 10,
-                     "roofline": roofline_of(name, "bytes", nbytes, ms, ctx.peaks)}
+        entry = PROFILED_MIXER_TRAFFIC.get(name)
+        traffic = entry[2] if entry and source_digest(entry[0]) == entry[1] else None
+        kms = trace[name][1] / max(trace[name][0], 1) if name in trace else ms
+        out[name] = {"ms": ms, "kernel_ms": kms,
+                     "gpu_launches_per_call": sum(c for c, _ in trace.values()) / 10,
+                     "roofline": roofline_of(name, "bytes", nbytes, kms, ctx.peaks, traffic)}
 
     # prep: 3 float32 controls + 2 K bf16 logits in, 3 controls + 2 K weights out
     add("param_prep_fwd", lambda: param_prep_fwd(raw["dt_raw"], raw["alpha_raw"], raw["lam_raw"],
