@@ -211,7 +211,7 @@ PROFILED_MIXER_TRAFFIC = {
 # DRAM bytes (read + write) of one decode_step launch of the decode workload (B128 H64 P64 N128
 # K8, float32 state), from one ncu capture (summarised under profiles/); used only while
 # decode.cu hashes to the digest it had when profiled.
-PROFILED_DECODE_TRAFFIC = ("decode.cu", "5a6ee76a91d8f3d2", 2151.500e6 + 2097.820e6)
+PROFILED_DECODE_TRAFFIC = ("decode.cu", "7a02e3079579523a", 2151.60e6 + 2098.05e6)
 
 
 def source_digest(fname: str) -> str:

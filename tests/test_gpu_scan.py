@@ -238,6 +238,42 @@ def test_train_workload_fwd_bwd_sampled():
     assert torch.count_nonzero(g["dB"][other]) == 0
 
 
+def _heads_per_bwd_state_cta(B, L, H, G, sms, chunk=128):
+    """The host's choice of heads per CTA for the state-term backward: the largest divisor (at
+    most 16) of a group's heads that still leaves two waves of CTAs, else the largest divisor."""
+    hpg, nc = H // G, (L + chunk - 1) // chunk
+    divisors = [hg for hg in range(1, 17) if hpg % hg == 0]
+    fits = [hg for hg in divisors if (H // hg) * nc * B >= 2 * sms]
+    return (fits or divisors)[-1], divisors[-1]
+
+
+def test_bwd_state_fewer_heads_per_cta_sampled():
+    """B4 L2048 H16 P64 N64 K8 bf16 (the forward workload's shape) through the backward: here the
+    state-term backward takes fewer heads per CTA than the largest divisor of the group (two
+    instead of sixteen, so that at least two waves of CTAs remain).  Two (batch, head) streams are
+    compared with the oracle, dy zero elsewhere as in the training-shape test."""
+    s = synth.WORKLOADS["fwd_bf16_b4_l2048"]
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    hg, largest = _heads_per_bwd_state_cta(s.batch, s.seqlen, s.nheads, s.ngroups, sms)
+    assert hg < largest, (hg, largest)
+    host = synth.make_scan_inputs(s, seed=4, with_dy=True)
+    b, heads = 2, [3, 12]
+    mask = np.zeros((s.batch, 1, s.nheads, 1), dtype=bool)
+    mask[b, 0, heads] = True
+    host["dy"] = synth.f32_to_bf16_bits(synth.bf16_bits_to_f32(host["dy"]) * mask)
+    dv = dev_inputs(host)
+    g = _gpu_bwd(dv)
+    torch.cuda.synchronize()
+    sub = _slice_streams(host, b, heads)
+    gr = _ora_bwd(sub)
+    for k in ("dx", "dw_read", "dw_write", "ddt", "dalpha", "dlam"):
+        assert_close(k, to_host64(g[k][b:b + 1][:, :, heads]), gr[k], 1e-2)
+    assert_close("dh0", to_host64(g["dh0"][b:b + 1][:, heads]), gr["dh0"], 1e-2)
+    assert_close("dB", to_host64(g["dB"][b:b + 1]), gr["dB"], 1e-2)
+    assert_close("dC", to_host64(g["dC"][b:b + 1]), gr["dC"], 1e-2)
+    assert_close("dD", to_host64(g["dD"][heads]), gr["dD"], 1e-2)
+
+
 @pytest.mark.slow
 def test_long_prefill_workload_sampled():
     """B1 L65536 H64 P64 N128 K8 bf16, Delta skewed small: y and h_final of two heads."""
