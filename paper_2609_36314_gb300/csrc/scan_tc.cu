@@ -265,21 +265,17 @@ __global__ void __launch_bounds__(kSPThreads, 2)
                 tma_load_3d(sV + jb * 16384, &mapV, &bars[0], g * N + 64 * jb, c0, b);
         }
         // A[(m, p), k] = s_{k,m} x_{k,p} as bf16, MN-major: row k = this thread's position,
-        // 64-element M-atoms (64 / TPSK modes x TPSK p each), 128-byte swizzle; group g writes atom g
+        // 64-element M-atoms (64 / TPSK modes x TPSK p each), 128-byte swizzle; group g writes atom g.
+        // Packed bf16 products (one instruction per two elements; s rounded to bf16 first)
         {
             unsigned char *row = sA + grp * 16384 + t * 128;
 #pragma unroll
             for (int c8 = 0; c8 < 8; ++c8) {  // elements M = 64 grp + 8 c8 ..: mode M / TPSK
                 const float s = grp == 0 ? cv[(8 * c8) / TPSK] : cv[(64 + 8 * c8) / TPSK];
+                const __nv_bfloat162 s2 = __float2bfloat162_rn(s);
                 const uint4 xv = xr[c8 % NX];
-                const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
-                uint32_t r[4];
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const float2 f = bf16x2_to_float2(xw[i]);
-                    r[i] = pack_bf16x2(s * f.x, s * f.y);
-                }
-                *reinterpret_cast<uint4 *>(row + ((c8 ^ (t & 7)) * 16)) = make_uint4(r[0], r[1], r[2], r[3]);
+                *reinterpret_cast<uint4 *>(row + ((c8 ^ (t & 7)) * 16)) =
+                    make_uint4(bf16x2_mul(xv.x, s2), bf16x2_mul(xv.y, s2), bf16x2_mul(xv.z, s2), bf16x2_mul(xv.w, s2));
             }
         }
         // emit the entering state (bf16) and apply the chunk's decay in place (the TMEM load of

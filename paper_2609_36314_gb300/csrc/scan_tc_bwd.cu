@@ -795,15 +795,10 @@ __device__ __forceinline__ float dot_bf16x8(uint4 a, uint4 b, float acc) {
     return acc;
 }
 
+// eight bf16 values times s, as packed bf16 products (s rounded to bf16 first)
 __device__ __forceinline__ uint4 scale_bf16x8(uint4 a, float s) {
-    const uint32_t ra[4] = {a.x, a.y, a.z, a.w};
-    uint32_t r[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const float2 f = bf16x2_to_float2(ra[i]);
-        r[i] = pack_bf16x2(s * f.x, s * f.y);
-    }
-    return make_uint4(r[0], r[1], r[2], r[3]);
+    const __nv_bfloat162 s2 = __float2bfloat162_rn(s);
+    return make_uint4(bf16x2_mul(a.x, s2), bf16x2_mul(a.y, s2), bf16x2_mul(a.z, s2), bf16x2_mul(a.w, s2));
 }
 
 __global__ void __launch_bounds__(kStLaunch, 1)

@@ -23,6 +23,12 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
 __device__ __forceinline__ float2 bf16x2_to_float2(uint32_t v) {
     return make_float2(__uint_as_float(v << 16), __uint_as_float(v & 0xffff0000u));
 }
+// (x.lo * s.lo, x.hi * s.hi) in one packed bf16 multiply (round to nearest); x as raw bits
+__device__ __forceinline__ uint32_t bf16x2_mul(uint32_t x, __nv_bfloat162 s) {
+    __nv_bfloat162 v = *reinterpret_cast<const __nv_bfloat162 *>(&x);
+    v = __hmul2(v, s);
+    return *reinterpret_cast<const uint32_t *>(&v);
+}
 
 __device__ __forceinline__ size_t blh(const ScanDims &d, int b, int t, int h) {
     return (size_t(b) * d.L + t) * d.H + h;
