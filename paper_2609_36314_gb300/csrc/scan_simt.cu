@@ -142,14 +142,28 @@ __global__ void __launch_bounds__(512) simt_state_pass(
         const int c0 = c * d.Q, n = min(d.Q, d.L - c0);
         __syncthreads();  // the previous chunk's shared-memory reads are done
         chunk_rates(d, b, h, c0, n, log_cap, dt, alpha, lam, e_s, E_s, nullptr);
-        for (int idx = tid; idx < n * Ps; idx += blockDim.x) {
-            const int k = idx / Ps, pp = idx - k * Ps, p = pbase + pp;
-            u_s[k * Ps + pp] = p < P ? to_f(U[blh(d, b, c0 + k, h) * P + p]) : 0.f;
+        // the chunk's rows, four independent loads per thread in flight before their stores
+        for (int i0 = tid; i0 < n * Ps; i0 += 4 * blockDim.x) {
+            float v[4];
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                const int idx = i0 + r * int(blockDim.x), k = idx / Ps, pp = idx - k * Ps, p = pbase + pp;
+                v[r] = (idx < n * Ps && p < P) ? to_f(U[blh(d, b, c0 + k, h) * P + p]) : 0.f;
+            }
+#pragma unroll
+            for (int r = 0; r < 4; ++r)
+                if (i0 + r * int(blockDim.x) < n * Ps) u_s[i0 + r * blockDim.x] = v[r];
         }
-        for (int idx = tid; idx < n * Npad; idx += blockDim.x) {
-            const int k = idx / Npad, nn = idx - k * Npad;
-            v_s[k * Npad + nn] =
-                nn < N ? to_f(V[((size_t(b) * d.L + c0 + k) * d.G + g) * N + nn]) : 0.f;
+        for (int i0 = tid; i0 < n * Npad; i0 += 4 * blockDim.x) {
+            float v[4];
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                const int idx = i0 + r * int(blockDim.x), k = idx / Npad, nn = idx - k * Npad;
+                v[r] = (idx < n * Npad && nn < N) ? to_f(V[((size_t(b) * d.L + c0 + k) * d.G + g) * N + nn]) : 0.f;
+            }
+#pragma unroll
+            for (int r = 0; r < 4; ++r)
+                if (i0 + r * int(blockDim.x) < n * Npad) v_s[i0 + r * blockDim.x] = v[r];
         }
         __syncthreads();  // E_s, e_s ready
         const double Eend = E_s[n - 1];
@@ -248,15 +262,38 @@ __global__ void __launch_bounds__(kThreads) simt_chunk_fwd(
     if (tid < K) itau[tid] = 1.f / tau[h * K + tid];
     const float log_cap = head_log_cap(tau, h, K);
     chunk_rates(d, b, h, c0, n, log_cap, dt, alpha, lam, e_s, E_s, nullptr);
-    for (int idx = tid; idx < Q * P; idx += blockDim.x) {
-        const int t = idx / P, p = idx - t * P;
-        xs[t * P1 + p] = t < n ? to_f(x[blh(d, b, c0 + t, h) * P + p]) : 0.f;
+    // the chunk's rows, four independent loads per thread in flight before their stores
+    for (int i0 = tid; i0 < Q * P; i0 += 4 * blockDim.x) {
+        float v[4];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            const int idx = i0 + r * int(blockDim.x), t = idx / P, p = idx - t * P;
+            v[r] = (idx < Q * P && t < n) ? to_f(x[blh(d, b, c0 + t, h) * P + p]) : 0.f;
+        }
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            const int idx = i0 + r * int(blockDim.x), t = idx / P, p = idx - t * P;
+            if (idx < Q * P) xs[t * P1 + p] = v[r];
+        }
     }
-    for (int idx = tid; idx < Q * N; idx += blockDim.x) {
-        const int t = idx / N, nn = idx - t * N;
-        const size_t gi = ((size_t(b) * d.L + c0 + t) * d.G + g) * N + nn;
-        Cs[t * N1 + nn] = t < n ? to_f(Cm[gi]) : 0.f;
-        Bs[t * N1 + nn] = t < n ? to_f(Bm[gi]) : 0.f;
+    for (int i0 = tid; i0 < Q * N; i0 += 4 * blockDim.x) {
+        float vc[4], vb[4];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            const int idx = i0 + r * int(blockDim.x), t = idx / N, nn = idx - t * N;
+            const size_t gi = ((size_t(b) * d.L + c0 + t) * d.G + g) * N + nn;
+            const bool in = idx < Q * N && t < n;
+            vc[r] = in ? to_f(Cm[gi]) : 0.f;
+            vb[r] = in ? to_f(Bm[gi]) : 0.f;
+        }
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            const int idx = i0 + r * int(blockDim.x), t = idx / N, nn = idx - t * N;
+            if (idx < Q * N) {
+                Cs[t * N1 + nn] = vc[r];
+                Bs[t * N1 + nn] = vb[r];
+            }
+        }
     }
     __syncthreads();
     for (int idx = tid; idx < Q * K; idx += blockDim.x) {
@@ -852,7 +889,8 @@ cudaError_t run_state_pass(const ScanDims &d, bool rev, const void *U, const voi
                            float *fin, cudaStream_t st) {
     const int Ps = state_pass_ps(d);
     const int ntiles = d.K * (Ps / 8) * ((d.N + 3) >> 2);
-    const int threads = ((ntiles + 31) / 32) * 32;
+    // at least 256 threads: the ones beyond the register tiles only help stage each chunk's rows
+    const int threads = std::max(((ntiles + 31) / 32) * 32, 256);
     const size_t smem = state_pass_smem(d, Ps);
     dim3 grid((d.P + Ps - 1) / Ps, d.H, d.B);
     if (rev) {
