@@ -117,7 +117,8 @@ struct Row {
     float pre, sp_dt, dt, alpha, sp_lam, lam;
     float ltau[KP], wr[KP], b[KP];
 
-    __device__ __forceinline__ void compute(const PrepArgs &a, int64_t r, int h) {
+    // ltab: ln tau of every (head, mode) in shared memory, or null (then evaluated here)
+    __device__ __forceinline__ void compute(const PrepArgs &a, int64_t r, int h, const float *ltab = nullptr) {
         const int K = a.K;
         pre = a.dt_raw[r] + (a.dt_bias ? a.dt_bias[h] : 0.f);
         sp_dt = softplus_f(pre);
@@ -130,7 +131,7 @@ struct Row {
         const bool rp = !(a.flags & FRAC_PREP_NO_READ_PRIOR), wp = !(a.flags & FRAC_PREP_NO_WRITE_PRIOR);
 #pragma unroll
         for (int m = 0; m < KP; ++m) {
-            ltau[m] = m < K ? logf(__ldg(a.tau + h * K + m)) : 0.f;
+            ltau[m] = m < K ? (ltab ? ltab[h * K + m] : logf(__ldg(a.tau + h * K + m))) : 0.f;
             const float prior = -alpha * ltau[m];
             if (rp) wr[m] += prior;
             if (wp) b[m] += prior;
@@ -141,13 +142,23 @@ struct Row {
     }
 };
 
+// ln tau of every (head, mode) in shared memory when the table is at most kTauTab entries (the
+// logarithm is then evaluated once per block instead of K times per row)
+constexpr int kTauTab = 4096;
+
 template <typename T, int KP, bool VEC>
 __global__ void __launch_bounds__(256) param_prep_fwd_kernel(PrepArgs a) {
+    __shared__ float ltab_s[kTauTab];
+    const bool tab = a.H * a.K <= kTauTab;
+    if (tab) {
+        for (int i = threadIdx.x; i < a.H * a.K; i += blockDim.x) ltab_s[i] = logf(__ldg(a.tau + i));
+        __syncthreads();
+    }
     const int64_t stride = int64_t(gridDim.x) * blockDim.x;
     for (int64_t r = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; r < a.n; r += stride) {
         const int h = int(r % a.H);
         Row<T, KP, VEC> w;
-        w.compute(a, r, h);
+        w.compute(a, r, h, tab ? ltab_s : nullptr);
         a.dt[r] = w.dt;
         a.alpha[r] = w.alpha;
         a.lam[r] = w.lam;
@@ -176,14 +187,21 @@ __device__ __forceinline__ void softmax_bwd_row(const float *w, float *dw, int K
 template <typename T, int KP, bool VEC>
 __global__ void __launch_bounds__(256) param_prep_bwd_kernel(PrepArgs a, int64_t hstride) {
     extern __shared__ float red[];  // [min(H, blockDim)][KP + 1] when H <= blockDim
+    __shared__ float ltab_s[kTauTab], itab_s[kTauTab];  // ln tau and 1 / tau per (head, mode)
     const int K = a.K, H = a.H;
     const int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
     const bool reduce = a.dtau || a.ddt_bias;
     const bool shared_slots = reduce && H <= int(blockDim.x);
-    if (shared_slots) {
+    const bool tab = H * K <= kTauTab;
+    if (tab)
+        for (int q = threadIdx.x; q < H * K; q += blockDim.x) {
+            const float tv = __ldg(a.tau + q);
+            ltab_s[q] = logf(tv);
+            itab_s[q] = 1.f / tv;
+        }
+    if (shared_slots)
         for (int q = threadIdx.x; q < H * (KP + 1); q += blockDim.x) red[q] = 0.f;
-        __syncthreads();
-    }
+    if (tab || shared_slots) __syncthreads();
     const int h = int(i % H);  // every row this thread visits has this head
     float acc_bias = 0.f, acc_tau[KP];
 #pragma unroll
@@ -192,7 +210,7 @@ __global__ void __launch_bounds__(256) param_prep_bwd_kernel(PrepArgs a, int64_t
     const bool rp = !(a.flags & FRAC_PREP_NO_READ_PRIOR), wp = !(a.flags & FRAC_PREP_NO_WRITE_PRIOR);
     for (int64_t r = i; i < hstride && r < a.n; r += hstride) {
         Row<T, KP, VEC> w;
-        w.compute(a, r, h);
+        w.compute(a, r, h, tab ? ltab_s : nullptr);
         float dwr[KP], db[KP];
         load_row<T, KP, VEC>(a.dw_read, r, K, dwr);
         load_row<T, KP, VEC>(a.dw_write, r, K, db);
@@ -214,7 +232,8 @@ __global__ void __launch_bounds__(256) param_prep_bwd_kernel(PrepArgs a, int64_t
         for (int m = 0; m < KP; ++m) {
             const float dp = (rp ? dwr[m] : 0.f) + (wp ? db[m] : 0.f);  // d(-alpha ln tau_m)
             dal = fmaf(-dp, w.ltau[m], dal);
-            if (m < K) acc_tau[m] = fmaf(dp, -w.alpha / __ldg(a.tau + h * K + m), acc_tau[m]);
+            if (m < K)
+                acc_tau[m] = fmaf(dp, -w.alpha * (tab ? itab_s[h * K + m] : 1.f / __ldg(a.tau + h * K + m)), acc_tau[m]);
         }
         store_row<T, KP, VEC>(a.dg_read, r, K, dwr);
         store_row<T, KP, VEC>(a.dg_write, r, K, db);

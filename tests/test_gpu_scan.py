@@ -204,38 +204,73 @@ def _slice_streams(host, b, heads):
 
 @pytest.mark.slow
 def test_train_workload_fwd_bwd_sampled():
-    """B8 L4096 H64 P64 N128 K8 bf16 at full size, in the configuration the benchmark times.
-    y, h_final and every per-stream gradient are compared on two (batch, head) streams; dy is
-    zero outside those streams so that dB, dC (sums over all heads) and dD are exactly the
+    """B8 L4096 H64 P64 N128 K8 bf16 at full size, in the configuration the benchmark times: one
+    workspace for both calls, the backward reusing the forward's per-chunk states.  y, h_final and
+    every per-stream gradient are compared on four (batch, head) streams in two batch rows; dy is
+    zero outside those streams so that dB, dC (sums over a row's heads) and dD are exactly the
     sampled streams' contributions, which the oracle computes."""
+    from paper_2609_36314_gb300.api import bwd_workspace_size, fwd_workspace_size, make_dims
     s = synth.WORKLOADS["train_bf16_b8_l4096"]
     host = synth.make_scan_inputs(s, seed=0, with_dy=True)
-    b, heads = 3, [5, 37]
+    sample = {3: [5, 37], 6: [12, 60]}
     mask = np.zeros((s.batch, 1, s.nheads, 1), dtype=bool)
-    mask[b, 0, heads] = True
+    for b, heads in sample.items():
+        mask[b, 0, heads] = True
     dy = synth.bf16_bits_to_f32(host["dy"]) * mask
     host["dy"] = synth.f32_to_bf16_bits(dy)
     dv = dev_inputs(host)
-    y, hf = _gpu_fwd(dv)
-    g = _gpu_bwd(dv)
+    dims = make_dims(s.batch, s.seqlen, s.nheads, s.headdim, s.ngroups, s.dstate, s.nmodes,
+                     torch.bfloat16)
+    ws = torch.empty(max(bwd_workspace_size(dims), fwd_workspace_size(dims)), dtype=torch.uint8,
+                     device="cuda")
+    y, hf = _gpu_fwd(dv, workspace=ws)
+    g = _gpu_bwd(dv, workspace=ws, reuse_fwd_states=True)
     torch.cuda.synchronize()
-    sub = _slice_streams(host, b, heads)
-    yr, hfr = _ora_fwd(sub)
-    gr = _ora_bwd(sub)
-    assert_close("y", to_host64(y[b:b + 1][:, :, heads]), yr, 1e-2)
-    assert_close("h_final", to_host64(hf[b:b + 1][:, heads]), hfr, 1e-2)
-    for k in ("dx", "dw_read", "dw_write"):
-        assert_close(k, to_host64(g[k][b:b + 1][:, :, heads]), gr[k], 1e-2)
-    for k in ("ddt", "dalpha", "dlam"):
-        assert_close(k, to_host64(g[k][b:b + 1][:, :, heads]), gr[k], 1e-2)
-    assert_close("dh0", to_host64(g["dh0"][b:b + 1][:, heads]), gr["dh0"], 1e-2)
-    assert_close("dB", to_host64(g["dB"][b:b + 1]), gr["dB"], 1e-2)
-    assert_close("dC", to_host64(g["dC"][b:b + 1]), gr["dC"], 1e-2)
-    assert_close("dD", to_host64(g["dD"][heads]), gr["dD"], 1e-2)
-    # streams outside the sample got no upstream gradient
+    dD = np.zeros(s.nheads)
+    for b, heads in sample.items():
+        sub = _slice_streams(host, b, heads)
+        yr, hfr = _ora_fwd(sub)
+        gr = _ora_bwd(sub)
+        assert_close("y", to_host64(y[b:b + 1][:, :, heads]), yr, 1e-2)
+        assert_close("h_final", to_host64(hf[b:b + 1][:, heads]), hfr, 1e-2)
+        for k in ("dx", "dw_read", "dw_write", "ddt", "dalpha", "dlam"):
+            assert_close(k, to_host64(g[k][b:b + 1][:, :, heads]), gr[k], 1e-2)
+        assert_close("dh0", to_host64(g["dh0"][b:b + 1][:, heads]), gr["dh0"], 1e-2)
+        assert_close("dB", to_host64(g["dB"][b:b + 1]), gr["dB"], 1e-2)
+        assert_close("dC", to_host64(g["dC"][b:b + 1]), gr["dC"], 1e-2)
+        dD[heads] += gr["dD"]
+    hs = sorted({h for heads in sample.values() for h in heads})
+    assert_close("dD", to_host64(g["dD"][hs]), dD[hs], 1e-2)
+    # rows outside the sample got no upstream gradient
     other = torch.ones(s.batch, dtype=torch.bool)
-    other[b] = False
+    other[list(sample)] = False
     assert torch.count_nonzero(g["dB"][other]) == 0
+
+
+def test_nonfinite_input_stays_in_its_stream():
+    """A NaN in one element of x (batch 1, head 2, channel 5, position 300 of a ragged 3-chunk
+    sequence) on the tensor-core path: y of every other (batch, head) stream and of every other
+    channel of the stream stays finite, and so do the positions of the chunks before the NaN's
+    chunk; y of that channel is NaN from the NaN's position on.  Inside its chunk the NaN may also
+    reach the positions before it (the chunk's intra-chunk product multiplies the masked-out
+    coefficients by it), which the sequential recurrence would not do."""
+    s = synth.Shape(2, 330, 4, 64, 1, 128, 8, 0, "bf16")
+    host = synth.make_scan_inputs(s, seed=13)
+    x = synth.bf16_bits_to_f32(host["x"]).copy()
+    b, h, p, t = 1, 2, 5, 300
+    x[b, t, h, p] = np.nan
+    host["x"] = synth.f32_to_bf16_bits(x)
+    dv = dev_inputs(host)
+    y, hf = _gpu_fwd(dv)
+    torch.cuda.synchronize()
+    yy = to_host64(y)
+    bad = np.isnan(yy)
+    keep = np.ones_like(bad)
+    keep[b, :, h, p] = False
+    assert not bad[keep].any()
+    assert bad[b, t:, h, p].all()
+    c0 = (t // 128) * 128
+    assert not bad[b, :c0, h, p].any()
 
 
 def _heads_per_bwd_state_cta(B, L, H, G, sms, chunk=128):
