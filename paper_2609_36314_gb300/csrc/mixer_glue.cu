@@ -7,13 +7,14 @@
 //   gated RMS normalisation   out = v / sqrt(mean_group(v^2) + eps) * weight,  v = y * silu(z)
 //        (before the output projection), and its backward.
 //
-// conv1d: a thread owns four adjacent channels (channel counts a multiple of 4; else two, else
-// one) and a run of kRun consecutive positions; a warp covers 128 contiguous channels of one
-// position per access, and the next batch of positions is loaded while the current one is
-// convolved.  The filter window of the last W-1 inputs stays in registers.  The backward streams
-// g = du * act'(pre) through a register ring of the last W values (dx_t needs g at t .. t+W-1),
-// and reduces dw / dbias over the block's rows of runs in shared memory before one atomic per
-// channel and block.
+// conv1d, bf16 with channel counts a multiple of 8: a block stages a tile of 64 positions (plus
+// the filter's halo) x 256 channels in shared memory with cp.async, every piece in flight at once,
+// and convolves from there (kernels *_tile_kernel below).  Other shapes: a thread owns four
+// adjacent channels (a multiple of 4; else two, else one) and a run of kRun consecutive positions
+// read from global memory.  The filter window of the last W-1 inputs stays in registers.  The
+// backward streams g = du * act'(pre) through a register ring of the last W values (dx_t needs g
+// at t .. t+W-1), and reduces dw / dbias in shared memory before one atomic per channel, tap and
+// block.
 // RMSNorm (dim <= 8192 forward, <= 4096 backward): a CTA per row holds the row in registers,
 // 8-element vectors per thread, so each row is read from HBM once; per-group sums by
 // shared-memory atomics.  The backward is persistent over rows, loads the next row while it
@@ -592,6 +593,255 @@ __global__ void __launch_bounds__(32 * kRows, 2) conv1d_bwd4_kernel(ConvArgs a) 
     }
 }
 
+// Tile path of the forward (bf16, channels a multiple of 8, 16-byte aligned rows): a block stages
+// positions [t0 - kHalo, t0 + kTileT) x channels [c0, c0 + kTileC) in shared memory by cp.async
+// (every 16-byte piece of the tile in flight at once; zeros outside the sequence, the carried
+// state patched in before position 0), then convolves from shared memory: thread i owns the
+// channel pair c0 + 2 (i mod 128) and the 32 positions of half i / 128, a warp stores 128
+// contiguous bytes per position.  36 KB of shared memory per block, six blocks per SM.
+constexpr int kTileT = 64, kTileC = 256, kHalo = 8;  // kHalo >= W - 1 for every width
+
+__device__ __forceinline__ void cp_async16_zfill(void *dst, const void *src, bool in) {
+    const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst));
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(src), "r"(in ? 16 : 0) : "memory");
+}
+
+template <int W>
+__global__ void __launch_bounds__(256) conv1d_fwd_tile_kernel(ConvArgs a) {
+    using T = __nv_bfloat16;
+    __shared__ __align__(16) T tile[kTileT + kHalo][kTileC];
+    const int c0 = blockIdx.x * kTileC, t0 = blockIdx.y * kTileT, b = blockIdx.z;
+    const T *x = static_cast<const T *>(a.x);
+    for (int i = threadIdx.x; i < (kTileT + kHalo) * (kTileC / 8); i += blockDim.x) {
+        const int r = i / (kTileC / 8), q = i % (kTileC / 8);
+        const int t = t0 - kHalo + r, c = c0 + 8 * q;
+        const bool in = t >= 0 && t < a.L && c < a.C;
+        cp_async16_zfill(&tile[r][8 * q], in ? x + (size_t(b) * a.L + t) * a.C + c : x, in);
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    if (t0 == 0 && a.state_in && W > 1) {  // positions -(W-1) .. -1 from the carried state
+        __syncthreads();
+        const T *si = static_cast<const T *>(a.state_in);
+        for (int i = threadIdx.x; i < (W - 1) * kTileC; i += blockDim.x) {
+            const int j = i / kTileC, cc = i % kTileC, c = c0 + cc;
+            if (c < a.C) tile[kHalo - (W - 1) + j][cc] = si[(size_t(b) * a.C + c) * (W - 1) + j];
+        }
+    }
+    __syncthreads();
+    const int cp = threadIdx.x & 127, half = threadIdx.x >> 7;
+    const int c = c0 + 2 * cp;
+    if (c >= a.C) return;  // C is a multiple of 8: the pair is whole
+    float w0[W], w1[W], win0[W], win1[W];
+#pragma unroll
+    for (int j = 0; j < W; ++j) {
+        w0[j] = a.w[c * W + j];
+        w1[j] = a.w[(c + 1) * W + j];
+    }
+    const float b0 = a.bias ? a.bias[c] : 0.f, b1 = a.bias ? a.bias[c + 1] : 0.f;
+    const int r0 = kHalo + 32 * half;  // tile row of this thread's first position
+#pragma unroll
+    for (int j = 0; j < W - 1; ++j) {
+        const float2 v = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&tile[r0 - (W - 1) + j][2 * cp]));
+        win0[j] = v.x;
+        win1[j] = v.y;
+    }
+    T *u = static_cast<T *>(a.u);
+#pragma unroll 4
+    for (int i = 0; i < 32; ++i) {
+        const int t = t0 + 32 * half + i;
+        if (t >= a.L) break;
+        const float2 v = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&tile[r0 + i][2 * cp]));
+        win0[W - 1] = v.x;
+        win1[W - 1] = v.y;
+        float p0 = b0, p1 = b1;
+#pragma unroll
+        for (int j = 0; j < W; ++j) {
+            p0 = fmaf(w0[j], win0[j], p0);
+            p1 = fmaf(w1[j], win1[j], p1);
+        }
+        if (a.silu) {
+            p0 = silu_f(p0);
+            p1 = silu_f(p1);
+        }
+        *reinterpret_cast<__nv_bfloat162 *>(u + (size_t(b) * a.L + t) * a.C + c) = __floats2bfloat162_rn(p0, p1);
+        if (a.state_out && t >= a.L - (W - 1)) {  // the last W-1 inputs become the carried state
+            T *so = static_cast<T *>(a.state_out);
+            const int ks = t - (a.L - (W - 1));
+            so[(size_t(b) * a.C + c) * (W - 1) + ks] = __float2bfloat16_rn(v.x);
+            so[(size_t(b) * a.C + c + 1) * (W - 1) + ks] = __float2bfloat16_rn(v.y);
+        }
+#pragma unroll
+        for (int j = 0; j < W - 1; ++j) {
+            win0[j] = win0[j + 1];
+            win1[j] = win1[j + 1];
+        }
+    }
+    if (a.state_out && t0 == 0 && half == 0 && a.L < W - 1) {  // short sequence: part of the old state stays
+        T *so = static_cast<T *>(a.state_out);
+        for (int ks = 0; ks < W - 1 - a.L; ++ks) {
+            const int row = kHalo - (W - 1) + ks + a.L;  // position ks + L - (W-1) < 0: a state row
+            so[(size_t(b) * a.C + c) * (W - 1) + ks] = tile[row][2 * cp];
+            so[(size_t(b) * a.C + c + 1) * (W - 1) + ks] = tile[row][2 * cp + 1];
+        }
+    }
+}
+
+// Tile path of the backward (same conditions): a block stages x at positions [t0 - kHalo,
+// t0 + kTileT + kHalo) and du at [t0, t0 + kTileT + kHalo) (76 KB, two blocks per SM); thread i
+// owns the channel pair c0 + 2 (i mod 128) and the 32 positions s of half i / 128: it walks
+// tt = s .. s + 31 + W - 1, forming g = du act'(pre) into a register ring of the last W values
+// (dx_s needs g at s .. s + W - 1), accumulating dw and dbias over its own positions, and writing
+// dx_s once the ring holds g at s .. s + W - 1.  dw, dbias: both halves' partials summed in shared
+// memory, one atomic per (channel, tap) and block.
+constexpr int kXRows = kTileT + 2 * kHalo, kDRows = kTileT + kHalo;
+
+template <int W>
+__global__ void __launch_bounds__(256, 2) conv1d_bwd_tile_kernel(ConvArgs a) {
+    using T = __nv_bfloat16;
+    extern __shared__ __align__(16) unsigned char tile_raw[];
+    T (*xt)[kTileC] = reinterpret_cast<T (*)[kTileC]>(tile_raw);                          // [kXRows]
+    T (*dt)[kTileC] = reinterpret_cast<T (*)[kTileC]>(tile_raw + kXRows * kTileC * 2);  // [kDRows]
+    const int c0 = blockIdx.x * kTileC, t0 = blockIdx.y * kTileT, b = blockIdx.z;
+    const T *x = static_cast<const T *>(a.x), *du = static_cast<const T *>(a.du);
+    for (int i = threadIdx.x; i < (kXRows + kDRows) * (kTileC / 8); i += blockDim.x) {
+        const bool isx = i < kXRows * (kTileC / 8);
+        const int ii = isx ? i : i - kXRows * (kTileC / 8);
+        const int r = ii / (kTileC / 8), q = ii % (kTileC / 8);
+        const int t = isx ? t0 - kHalo + r : t0 + r, c = c0 + 8 * q;
+        const bool in = t >= 0 && t < a.L && c < a.C;
+        const T *src = isx ? x : du;
+        cp_async16_zfill(isx ? &xt[r][8 * q] : &dt[r][8 * q], in ? src + (size_t(b) * a.L + t) * a.C + c : src, in);
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    if (t0 == 0 && a.state_in && W > 1) {  // positions -(W-1) .. -1 from the carried state
+        __syncthreads();
+        const T *si = static_cast<const T *>(a.state_in);
+        for (int i = threadIdx.x; i < (W - 1) * kTileC; i += blockDim.x) {
+            const int j = i / kTileC, cc = i % kTileC, c = c0 + cc;
+            if (c < a.C) xt[kHalo - (W - 1) + j][cc] = si[(size_t(b) * a.C + c) * (W - 1) + j];
+        }
+    }
+    __syncthreads();
+    const int cp = threadIdx.x & 127, half = threadIdx.x >> 7;
+    const int c = c0 + 2 * cp;
+    const bool active = c < a.C;
+    float acc0[W + 1], acc1[W + 1];  // dw taps, then dbias
+#pragma unroll
+    for (int j = 0; j <= W; ++j) acc0[j] = acc1[j] = 0.f;
+    if (active) {
+        float w0[W], w1[W], win0[W], win1[W], g0[W], g1[W], gf0[kMaxW], gf1[kMaxW];
+#pragma unroll
+        for (int j = 0; j < W; ++j) {
+            w0[j] = a.w[c * W + j];
+            w1[j] = a.w[(c + 1) * W + j];
+            g0[j] = g1[j] = 0.f;
+        }
+        const float b0 = a.bias ? a.bias[c] : 0.f, b1 = a.bias ? a.bias[c + 1] : 0.f;
+        const int s0 = t0 + 32 * half;  // this thread's first own position
+        // x window before s0: positions s0 - (W-1) .. s0 - 1 at rows s0 - t0 + kHalo - (W-1) ..
+#pragma unroll
+        for (int j = 0; j < W - 1; ++j) {
+            const float2 v = __bfloat1622float2(
+                *reinterpret_cast<const __nv_bfloat162 *>(&xt[s0 - t0 + kHalo - (W - 1) + j][2 * cp]));
+            win0[j] = v.x;
+            win1[j] = v.y;
+        }
+        T *dx = static_cast<T *>(a.dx);
+#pragma unroll 4
+        for (int i = 0; i < 32 + W - 1; ++i) {
+            const int tt = s0 + i;
+            const float2 xv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&xt[tt - t0 + kHalo][2 * cp]));
+            const float2 dv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&dt[tt - t0][2 * cp]));
+            win0[W - 1] = xv.x;
+            win1[W - 1] = xv.y;
+            float p0 = b0, p1 = b1;
+#pragma unroll
+            for (int j = 0; j < W; ++j) {
+                p0 = fmaf(w0[j], win0[j], p0);
+                p1 = fmaf(w1[j], win1[j], p1);
+            }
+            const float gg0 = a.silu ? dv.x * silu_grad_f(p0) : dv.x;  // du is 0 past the end
+            const float gg1 = a.silu ? dv.y * silu_grad_f(p1) : dv.y;
+#pragma unroll
+            for (int j = 0; j < W - 1; ++j) {
+                g0[j] = g0[j + 1];
+                g1[j] = g1[j + 1];
+            }
+            g0[W - 1] = gg0;
+            g1[W - 1] = gg1;
+            if (i < 32 && tt < a.L) {  // own positions: dw and dbias terms
+#pragma unroll
+                for (int j = 0; j < W; ++j) {
+                    acc0[j] = fmaf(gg0, win0[j], acc0[j]);
+                    acc1[j] = fmaf(gg1, win1[j], acc1[j]);
+                }
+                acc0[W] += gg0;
+                acc1[W] += gg1;
+            }
+#pragma unroll
+            for (int j = 0; j < W - 1; ++j)  // g at positions 0 .. W-2, for the carried-state gradient
+                if (tt == j) {
+                    gf0[j] = gg0;
+                    gf1[j] = gg1;
+                }
+            const int s = tt - (W - 1);  // the ring now holds g at s .. s + W - 1
+            if (i >= W - 1 && s < a.L) {
+                float d0 = 0.f, d1 = 0.f;
+#pragma unroll
+                for (int j = 0; j < W; ++j) {
+                    d0 = fmaf(w0[j], g0[W - 1 - j], d0);
+                    d1 = fmaf(w1[j], g1[W - 1 - j], d1);
+                }
+                *reinterpret_cast<__nv_bfloat162 *>(dx + (size_t(b) * a.L + s) * a.C + c) = __floats2bfloat162_rn(d0, d1);
+            }
+#pragma unroll
+            for (int j = 0; j < W - 1; ++j) {
+                win0[j] = win0[j + 1];
+                win1[j] = win1[j + 1];
+            }
+        }
+        if (a.dstate && t0 == 0 && half == 0) {
+            // gradient of the carried inputs i = 0 .. W-2 (position i - (W-1)): taps j <= i of
+            // w_j g[i - j] over the positions that exist
+            T *ds = static_cast<T *>(a.dstate);
+#pragma unroll
+            for (int ii = 0; ii < W - 1; ++ii) {
+                float d0 = 0.f, d1 = 0.f;
+#pragma unroll
+                for (int j = 0; j < W; ++j) {
+                    const int tt = ii - j;
+                    if (j <= ii && tt < a.L) {
+                        d0 = fmaf(w0[j], gf0[tt], d0);
+                        d1 = fmaf(w1[j], gf1[tt], d1);
+                    }
+                }
+                ds[(size_t(b) * a.C + c) * (W - 1) + ii] = __float2bfloat16_rn(d0);
+                ds[(size_t(b) * a.C + c + 1) * (W - 1) + ii] = __float2bfloat16_rn(d1);
+            }
+        }
+    }
+    __syncthreads();  // the tiles are dead: their space sums dw, dbias
+    float *red = reinterpret_cast<float *>(tile_raw);  // [2 halves][W + 1][kTileC]
+#pragma unroll
+    for (int j = 0; j <= W; ++j) {
+        red[(half * (W + 1) + j) * kTileC + 2 * cp] = acc0[j];
+        red[(half * (W + 1) + j) * kTileC + 2 * cp + 1] = acc1[j];
+    }
+    __syncthreads();
+    for (int q = threadIdx.x; q < (W + 1) * kTileC; q += blockDim.x) {
+        const int j = q / kTileC, cc = q % kTileC, ch = c0 + cc;
+        if (ch >= a.C) continue;
+        const float sum = red[j * kTileC + cc] + red[((W + 1) + j) * kTileC + cc];
+        if (j < W)
+            atomicAdd(a.dw + ch * W + j, sum);
+        else if (a.dbias)
+            atomicAdd(a.dbias + ch, sum);
+    }
+}
+constexpr size_t kConvBwdTileSmem = size_t(kXRows + kDRows) * kTileC * 2;
+
 // one decode step: window = carried state (W-1 inputs) then x_t; the state shifts by one
 template <typename T>
 __global__ void __launch_bounds__(256) conv1d_step_kernel(ConvArgs a, const T *__restrict__ xt, T *__restrict__ ut) {
@@ -1042,7 +1292,23 @@ cudaError_t norm_reg(const NormArgs &a, bool bwd, cudaStream_t st) {
 constexpr int kNormRegMaxDim = 8192, kNormRegMaxDimBwd = 4096;
 
 template <typename T, int W>
-cudaError_t conv_launch_w(const ConvArgs &a, bool bwd, bool vec, bool vec4, cudaStream_t st) {
+cudaError_t conv_launch_w(const ConvArgs &a, bool bwd, bool vec, bool vec4, bool tile, cudaStream_t st) {
+    if constexpr (sizeof(T) == 2) {
+        if (tile) {  // bf16 through shared-memory tiles
+            const dim3 tgrid((a.C + kTileC - 1) / kTileC, (a.L + kTileT - 1) / kTileT, a.B);
+            if (!bwd) {
+                trace_begin("conv1d_fwd", st);
+                conv1d_fwd_tile_kernel<W><<<tgrid, 256, 0, st>>>(a);
+            } else {
+                auto k = conv1d_bwd_tile_kernel<W>;
+                cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kConvBwdTileSmem));
+                trace_begin("conv1d_bwd", st);
+                k<<<tgrid, 256, kConvBwdTileSmem, st>>>(a);
+            }
+            trace_end(st);
+            return cudaGetLastError();
+        }
+    }
     dim3 block(32, kRows);
     dim3 grid((a.C + 63) / 64, (a.L + kRows * kRun - 1) / (kRows * kRun), a.B);
     if (grid.y == 0) return cudaSuccess;
@@ -1071,16 +1337,16 @@ cudaError_t conv_launch_w(const ConvArgs &a, bool bwd, bool vec, bool vec4, cuda
 }
 
 template <typename T>
-cudaError_t conv_launch(const ConvArgs &a, bool bwd, bool vec, bool vec4, cudaStream_t st) {
+cudaError_t conv_launch(const ConvArgs &a, bool bwd, bool vec, bool vec4, bool tile, cudaStream_t st) {
     switch (a.W) {
-        case 1: return conv_launch_w<T, 1>(a, bwd, vec, vec4, st);
-        case 2: return conv_launch_w<T, 2>(a, bwd, vec, vec4, st);
-        case 3: return conv_launch_w<T, 3>(a, bwd, vec, vec4, st);
-        case 4: return conv_launch_w<T, 4>(a, bwd, vec, vec4, st);
-        case 5: return conv_launch_w<T, 5>(a, bwd, vec, vec4, st);
-        case 6: return conv_launch_w<T, 6>(a, bwd, vec, vec4, st);
-        case 7: return conv_launch_w<T, 7>(a, bwd, vec, vec4, st);
-        default: return conv_launch_w<T, 8>(a, bwd, vec, vec4, st);
+        case 1: return conv_launch_w<T, 1>(a, bwd, vec, vec4, tile, st);
+        case 2: return conv_launch_w<T, 2>(a, bwd, vec, vec4, tile, st);
+        case 3: return conv_launch_w<T, 3>(a, bwd, vec, vec4, tile, st);
+        case 4: return conv_launch_w<T, 4>(a, bwd, vec, vec4, tile, st);
+        case 5: return conv_launch_w<T, 5>(a, bwd, vec, vec4, tile, st);
+        case 6: return conv_launch_w<T, 6>(a, bwd, vec, vec4, tile, st);
+        case 7: return conv_launch_w<T, 7>(a, bwd, vec, vec4, tile, st);
+        default: return conv_launch_w<T, 8>(a, bwd, vec, vec4, tile, st);
     }
 }
 
@@ -1176,8 +1442,10 @@ frac_status frac_conv1d_fwd(const frac_conv_dims *dims, const void *x, const flo
     }
     const bool vec = a.C % 2 == 0 && frac::aligned(x, 2 * es) && frac::aligned(u, 2 * es);
     const bool vec4 = a.C % 4 == 0 && frac::aligned(x, 4 * es) && frac::aligned(u, 4 * es);
-    return frac::glue_cuda(dims->dtype == FRAC_DTYPE_BF16 ? frac::conv_launch<__nv_bfloat16>(a, false, vec, vec4, st)
-                                                          : frac::conv_launch<float>(a, false, vec, vec4, st),
+    const bool tile = a.C % 8 == 0 && frac::aligned(x, 16) && frac::aligned(u, 4);
+    return frac::glue_cuda(dims->dtype == FRAC_DTYPE_BF16
+                               ? frac::conv_launch<__nv_bfloat16>(a, false, vec, vec4, tile, st)
+                               : frac::conv_launch<float>(a, false, vec, vec4, false, st),
                            "frac_conv1d_fwd");
 }
 
@@ -1215,8 +1483,9 @@ frac_status frac_conv1d_bwd(const frac_conv_dims *dims, const void *x, const flo
                          frac::aligned(dx, 2 * es);
         const bool vec4 = a.C % 4 == 0 && frac::aligned(x, 4 * es) && frac::aligned(du, 4 * es) &&
                           frac::aligned(dx, 4 * es);
-        e = dims->dtype == FRAC_DTYPE_BF16 ? frac::conv_launch<__nv_bfloat16>(a, true, vec, vec4, st)
-                                           : frac::conv_launch<float>(a, true, vec, vec4, st);
+        const bool tile = a.C % 8 == 0 && frac::aligned(x, 16) && frac::aligned(du, 16) && frac::aligned(dx, 4);
+        e = dims->dtype == FRAC_DTYPE_BF16 ? frac::conv_launch<__nv_bfloat16>(a, true, vec, vec4, tile, st)
+                                           : frac::conv_launch<float>(a, true, vec, vec4, false, st);
     }
     return frac::glue_cuda(e, "frac_conv1d_bwd");
 }

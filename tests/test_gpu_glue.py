@@ -3,7 +3,8 @@ against the fp64 oracle (oracle/mixer_glue.py), through the C ABI.
 
 Tolerances as for the scan: relative L2 per output <= 1e-5 float32, <= 1e-2 bf16.  The conv
 cases cover lengths inside, at and across the 32-position runs of a thread (1, 31, 33, 300),
-widths 1 to 8, channel counts that take two or four channels per thread or the scalar path, the
+widths 1 to 8, channel counts that take the shared-memory tiles (bf16, a multiple of 8), four or
+two channels per thread or the scalar path, the
 carried state and SiLU on and off; the norm cases cover gated and ungated rows, several group
 sizes, and rows held in registers (dim <= 8192 forward, <= 4096 backward) or streamed.
 """
@@ -44,7 +45,7 @@ def _conv_case(B, L, C, W, dtype, silu, with_state, seed=0):
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("L", [1, 31, 33, 300])
-@pytest.mark.parametrize("C", [70, 72])  # two channels per thread / four channels per thread
+@pytest.mark.parametrize("C", [68, 70, 72])  # four / two channels per thread / shared-memory tiles (bf16)
 def test_conv_lengths(dtype, L, C):
     _conv_case(2, L, C, 4, dtype, silu=True, with_state=True, seed=L)
 
