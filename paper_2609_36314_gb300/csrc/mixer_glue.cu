@@ -15,11 +15,12 @@
 // backward streams g = du * act'(pre) through a register ring of the last W values (dx_t needs g
 // at t .. t+W-1), and reduces dw / dbias in shared memory before one atomic per channel, tap and
 // block.
-// RMSNorm (dim <= 8192 forward, <= 4096 backward): a CTA per row holds the row in registers,
-// 8-element vectors per thread, so each row is read from HBM once; per-group sums by
-// shared-memory atomics.  The backward is persistent over rows, loads the next row while it
-// processes the current one, and keeps each thread's dweight partials in registers until one
-// global atomic per feature and CTA.  Wider rows take streaming kernels that re-read the row.
+// RMSNorm (dim <= 8192 forward, <= 4096 backward): a CTA per row holds the row in registers (or,
+// bf16 backward, in a ring of shared-memory row buffers filled by cp.async), 8-element vectors
+// per thread, so each row is read from HBM once; per-group sums by shared-memory atomics.  The
+// backward is persistent over rows, loads the next rows while it processes the current one, and
+// keeps each thread's dweight partials in registers until one global atomic per feature and CTA.
+// Wider rows take streaming kernels that re-read the row.
 #include <algorithm>
 #include <cstdio>
 
@@ -1240,6 +1241,147 @@ __global__ void __launch_bounds__(NT, NT <= 256 ? 2 : 1) rmsnorm_bwd_reg_kernel(
     }
 }
 
+// bf16 backward with rows staged in shared memory (dim <= 4096): persistent over rows, y, z and
+// dout of the next two rows (up to 24 KB each) loaded by cp.async into a ring of three buffers
+// while the current row is processed from its buffer, three CTAs per SM; thread i owns the
+// 8-feature vectors at 8 (i + 256 j), j < VPT, and keeps their dweight partials in registers until
+// one global atomic per feature and CTA.  Both row sums come from one pass: sum(v^2) and
+// sum(dout w v), since sum(dn n) = (1 / rms) sum(dout w v).
+template <int VPT>
+__global__ void __launch_bounds__(256, 3) rmsnorm_bwd_tile_kernel(NormArgs a) {
+    using T = __nv_bfloat16;
+    extern __shared__ __align__(16) unsigned char nsm[];
+    const int ng = a.D / a.gs, D8 = a.D / 8;
+    const bool gated = a.z != nullptr;
+    float *sums = reinterpret_cast<float *>(nsm);  // [2][2 ng]: sum(v^2), then sum(dn n), per row parity
+    uint4 *rows = reinterpret_cast<uint4 *>(nsm + ((sizeof(float) * 4 * ng + 15) / 16) * 16);  // [3][3][D8]
+    auto stage = [&](int64_t row, int slot) {
+        uint4 *dst = rows + size_t(slot) * 3 * D8;
+        for (int i = threadIdx.x; i < 3 * D8; i += blockDim.x) {
+            const int which = i / D8, v = i - which * D8;
+            if (which == 1 && !gated) continue;
+            const T *src = static_cast<const T *>(which == 0 ? a.y : which == 1 ? a.z : a.dout);
+            cp_async16_zfill(dst + i, src + size_t(row) * a.D + 8 * v, true);
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+    float dwp[VPT][8];
+#pragma unroll
+    for (int j = 0; j < VPT; ++j)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) dwp[j][i] = 0.f;
+    if (blockIdx.x < a.R) stage(blockIdx.x, 0);
+    if (blockIdx.x + gridDim.x < a.R) stage(blockIdx.x + gridDim.x, 1);
+    int k = 0;
+    for (int64_t r = blockIdx.x; r < a.R; r += gridDim.x, ++k) {
+        const int slot = k % 3;
+        float *ssq = sums + (k & 1) * 2 * ng, *dot = ssq + ng;
+        if (r + 2 * int64_t(gridDim.x) < a.R) stage(r + 2 * int64_t(gridDim.x), (k + 2) % 3);
+        // this row's group is complete once at most the groups of the rows after it are pending
+        const int later = int(r + gridDim.x < a.R) + int(r + 2 * int64_t(gridDim.x) < a.R);
+        if (later == 2)
+            asm volatile("cp.async.wait_group 2;" ::: "memory");
+        else if (later == 1)
+            asm volatile("cp.async.wait_group 1;" ::: "memory");
+        else
+            asm volatile("cp.async.wait_group 0;" ::: "memory");
+        for (int g = threadIdx.x; g < 2 * ng; g += blockDim.x) ssq[g] = 0.f;
+        __syncthreads();
+        const uint4 *ry = rows + size_t(slot) * 3 * D8, *rz = ry + D8, *rg = rz + D8;
+        auto unpack = [](uint4 u, float *v) {
+            const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&u);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float2 f = __bfloat1622float2(h[i]);
+                v[2 * i] = f.x;
+                v[2 * i + 1] = f.y;
+            }
+        };
+        // one pass for both row sums: sum(v^2) and sum(dout w v) (= rms sum(dn n))
+        float sg[VPT][8];  // sigmoid(z) of the gate; the gate factor is silu(z) = z sg (1 without the gate)
+#pragma unroll
+        for (int j = 0; j < VPT; ++j) {
+            const int v = threadIdx.x + 256 * j, f = 8 * v;
+            const bool valid = f < a.D;
+            float sq = 0.f, sd = 0.f;
+            if (valid) {
+                float y[8], z[8], go[8];
+                unpack(ry[v], y);
+                unpack(rg[v], go);
+                if (gated) unpack(rz[v], z);
+                const float4 w0 = reinterpret_cast<const float4 *>(a.weight + f)[0];
+                const float4 w1 = reinterpret_cast<const float4 *>(a.weight + f)[1];
+                const float wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    sg[j][i] = gated ? sigm(z[i]) : 1.f;
+                    const float vv = y[i] * (gated ? z[i] * sg[j][i] : 1.f);
+                    sq = fmaf(vv, vv, sq);
+                    sd = fmaf(go[i] * wv[i], vv, sd);
+                }
+            }
+            if (8 * 256 * j < a.D) {  // whole warps take part
+                group_add(ssq, f, a.gs, valid, sq);
+                group_add(dot, f, a.gs, valid, sd);
+            }
+        }
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < VPT; ++j) {
+            const int v = threadIdx.x + 256 * j, f = 8 * v;
+            if (f < a.D) {
+                const float iv = rsqrtf(ssq[f / a.gs] / a.gs + a.eps);
+                const float m = iv * dot[f / a.gs] / a.gs;  // mean(dn n)
+                float y[8], go[8], z[8], dyv[8], dzv[8];
+                unpack(ry[v], y);
+                unpack(rg[v], go);
+                if (gated) unpack(rz[v], z);
+                const float4 w0 = reinterpret_cast<const float4 *>(a.weight + f)[0];
+                const float4 w1 = reinterpret_cast<const float4 *>(a.weight + f)[1];
+                const float wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const float gz = gated ? z[i] * sg[j][i] : 1.f;
+                    const float n = y[i] * gz * iv;
+                    dwp[j][i] = fmaf(go[i], n, dwp[j][i]);
+                    const float dv = (go[i] * wv[i] - n * m) * iv;  // (dn - n mean(dn n)) / rms
+                    dyv[i] = dv * gz;
+                    dzv[i] = gated ? dv * y[i] * (sg[j][i] * (1.f + z[i] * (1.f - sg[j][i]))) : 0.f;
+                }
+                const size_t o = size_t(r) * a.D + f;
+                st8<T>(static_cast<T *>(a.dy) + o, dyv);
+                if (gated) st8<T>(static_cast<T *>(a.dz) + o, dzv);
+            }
+        }
+        __syncthreads();  // this slot's rows and sums are read: the next stage may overwrite them
+    }
+#pragma unroll
+    for (int j = 0; j < VPT; ++j) {
+        const int f = 8 * (threadIdx.x + 256 * j);
+        if (f < a.D)
+#pragma unroll
+            for (int i = 0; i < 8; ++i) atomicAdd(a.dweight + f + i, dwp[j][i]);
+    }
+}
+
+int num_sms();
+
+template <int VPT>
+cudaError_t norm_bwd_tile_launch(const NormArgs &a, cudaStream_t st) {
+    const int ng = a.D / a.gs;
+    const size_t smem = ((sizeof(float) * 4 * ng + 15) / 16) * 16 + size_t(3) * 3 * a.D * 2;
+    auto k = rmsnorm_bwd_tile_kernel<VPT>;
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    int per_sm = 0;
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, 256, smem);
+    if (e != cudaSuccess) return e;
+    const int blocks = int(std::min<int64_t>(a.R, int64_t(num_sms()) * std::max(per_sm, 1)));
+    trace_begin("gated_rmsnorm_bwd", st);
+    k<<<blocks, 256, smem, st>>>(a);
+    trace_end(st);
+    return cudaGetLastError();
+}
+
 int num_sms() {
     int dev = 0, sms = 152;
     if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -1569,8 +1711,12 @@ frac_status frac_gated_rmsnorm_bwd(const frac_norm_dims *dims, const void *y, co
     cudaStream_t st = (cudaStream_t)stream;
     cudaError_t e = cudaMemsetAsync(dweight, 0, sizeof(float) * a.D, st);
     if (e == cudaSuccess && a.R > 0 && a.D <= frac::kNormRegMaxDimBwd) {
-        e = dims->dtype == FRAC_DTYPE_BF16 ? frac::norm_reg<__nv_bfloat16>(a, true, st)
-                                           : frac::norm_reg<float>(a, true, st);
+        const bool al16 = frac::aligned(y, 16) && frac::aligned(dout, 16) && (!z || frac::aligned(z, 16));
+        if (dims->dtype == FRAC_DTYPE_BF16 && al16)  // rows staged in shared memory
+            e = a.D <= 2048 ? frac::norm_bwd_tile_launch<1>(a, st) : frac::norm_bwd_tile_launch<2>(a, st);
+        else
+            e = dims->dtype == FRAC_DTYPE_BF16 ? frac::norm_reg<__nv_bfloat16>(a, true, st)
+                                               : frac::norm_reg<float>(a, true, st);
     } else if (e == cudaSuccess && a.R > 0) {
         const int blocks = int(std::min<int64_t>(a.R, int64_t(frac::num_sms()) * 4));
         const size_t smem = sizeof(float) * (a.D + 2 * (a.D / a.gs));
