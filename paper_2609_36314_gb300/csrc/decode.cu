@@ -112,6 +112,47 @@ __global__ void __launch_bounds__(256, 4) decode_step_kernel(
     if (lane == 0) y[bh * a.P + p] = from_f<T>(acc + a.D[h] * xp);
 }
 
+// N = 1 (the paper's own layer: scalar B, C per position): one thread per (b, h, p), all K mode
+// states of the row loaded before any arithmetic (for each mode a warp reads 32 consecutive p: one
+// 128-byte line), then S_m <- rho_m S_m + kappa_m x B and y = sum_m w_read,m C S_m + D x with no
+// cross-lane reduction.
+constexpr int kDecodeN1Modes = 32;  // nmodes <= 32 (checked at the boundary)
+
+template <typename T>
+__global__ void __launch_bounds__(256) decode_step_n1_kernel(
+    DecodeArgs a, const T *__restrict__ x, const T *__restrict__ Bt, const T *__restrict__ Ct,
+    const T *__restrict__ wr, const T *__restrict__ ww, T *__restrict__ y) {
+    const int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (i >= int64_t(a.B) * a.H * a.P) return;
+    const int p = int(i % a.P);
+    const int64_t bh = i / a.P;
+    const int h = int(bh % a.H), b = int(bh / a.H), g = h / (a.H / a.G);
+    const int K = a.K;
+    float *srow = a.state + bh * K * a.P + p;  // mode m at srow[m P]
+    float sv[kDecodeN1Modes];
+#pragma unroll
+    for (int m = 0; m < kDecodeN1Modes; ++m)
+        if (m < K) sv[m] = __ldcs(srow + int64_t(m) * a.P);
+    float tmax = 0.f;
+    for (int m = 0; m < K; ++m) tmax = fmaxf(tmax, a.tau[h * K + m]);
+    bool clamped;
+    const float e = token_rate(a.dt[bh], a.alpha[bh], a.lam[bh], logf(64.f * tmax), &clamped);
+    const float xp = to_f(x[bh * a.P + p]);
+    const float kb = xp * to_f(Bt[int64_t(b) * a.G + g]), cv = to_f(Ct[int64_t(b) * a.G + g]);
+    float acc = 0.f;
+#pragma unroll
+    for (int m = 0; m < kDecodeN1Modes; ++m) {
+        if (m < K) {
+            const float z = e / a.tau[h * K + m];
+            const float kap = -expm1f(-z) * to_f(ww[bh * K + m]);
+            const float v = fmaf(expf(-z), sv[m], kap * kb);
+            acc = fmaf(to_f(wr[bh * K + m]), v * cv, acc);
+            __stcs(srow + int64_t(m) * a.P, v);
+        }
+    }
+    y[bh * a.P + p] = from_f<T>(acc + a.D[h] * xp);
+}
+
 template <typename T>
 cudaError_t launch_decode_t(const DecodeArgs &a, const void *x, const void *Bt, const void *Ct,
                             const void *wr, const void *ww, void *y, cudaStream_t st) {
@@ -124,7 +165,11 @@ cudaError_t launch_decode_t(const DecodeArgs &a, const void *x, const void *Bt, 
                      (reinterpret_cast<uintptr_t>(Bt) % (4 * sizeof(T))) == 0 &&
                      (reinterpret_cast<uintptr_t>(Ct) % (4 * sizeof(T))) == 0;
     trace_begin("decode_step", st);
-    if (vec)
+    if (a.N == 1) {
+        const int64_t nthreads = rows;
+        decode_step_n1_kernel<T><<<dim3(unsigned((nthreads + 255) / 256)), 256, 0, st>>>(
+            a, (const T *)x, (const T *)Bt, (const T *)Ct, (const T *)wr, (const T *)ww, (T *)y);
+    } else if (vec)
         decode_step_kernel<T, true><<<dim3(unsigned(blocks)), 256, 0, st>>>(
             a, (const T *)x, (const T *)Bt, (const T *)Ct, (const T *)wr, (const T *)ww, (T *)y);
     else
