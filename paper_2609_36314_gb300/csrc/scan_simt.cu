@@ -1028,17 +1028,22 @@ __global__ void __launch_bounds__(kN1P) n1_local(ScanDims d, const T *__restrict
 #pragma unroll 4
     for (int t = 0; t < n; ++t) {
         const float xv = to_f(x_s[t * kN1P + threadIdx.x]);
-        if ((K & 3) == 0) {
+        if ((K & 3) == 0) {  // rows of 16-byte pieces; packed float32 pairs (the same IEEE operations)
             const float4 *r4 = reinterpret_cast<const float4 *>(rho_s + t * K);
             const float4 *k4 = reinterpret_cast<const float4 *>(kb_s + t * K);
+            const float2 xx = make_float2(xv, xv);
 #pragma unroll
             for (int q = 0; q < KP / 4; ++q) {
                 if (4 * q < K) {
                     const float4 r = r4[q], kv = k4[q];
-                    S[4 * q] = fmaf(r.x, S[4 * q], kv.x * xv);
-                    S[4 * q + 1] = fmaf(r.y, S[4 * q + 1], kv.y * xv);
-                    S[4 * q + 2] = fmaf(r.z, S[4 * q + 2], kv.z * xv);
-                    S[4 * q + 3] = fmaf(r.w, S[4 * q + 3], kv.w * xv);
+                    const float2 a = __ffma2_rn(make_float2(r.x, r.y), make_float2(S[4 * q], S[4 * q + 1]),
+                                                __fmul2_rn(make_float2(kv.x, kv.y), xx));
+                    const float2 c2 = __ffma2_rn(make_float2(r.z, r.w), make_float2(S[4 * q + 2], S[4 * q + 3]),
+                                                 __fmul2_rn(make_float2(kv.z, kv.w), xx));
+                    S[4 * q] = a.x;
+                    S[4 * q + 1] = a.y;
+                    S[4 * q + 2] = c2.x;
+                    S[4 * q + 3] = c2.y;
                 }
             }
         } else {
@@ -1128,24 +1133,32 @@ __global__ void __launch_bounds__(kN1P) n1_chunk_fwd(ScanDims d, const T *__rest
     for (int t = 0; t < n; ++t) {
         const float xv = to_f(x_s[t * kN1P + threadIdx.x]);
         float ya[4] = {Dh * xv, 0.f, 0.f, 0.f};  // four independent partial readout sums
-        if ((K & 3) == 0) {  // rows of 16-byte pieces
+        if ((K & 3) == 0) {  // rows of 16-byte pieces; packed float32 pairs (the same IEEE operations)
             const float4 *r4 = reinterpret_cast<const float4 *>(rho_s + t * K);
             const float4 *k4 = reinterpret_cast<const float4 *>(kb_s + t * K);
             const float4 *w4 = reinterpret_cast<const float4 *>(wc_s + t * K);
+            const float2 xx = make_float2(xv, xv);
+            float2 y01 = make_float2(ya[0], ya[1]), y23 = make_float2(ya[2], ya[3]);
 #pragma unroll
             for (int q = 0; q < KP / 4; ++q) {
                 if (4 * q < K) {
                     const float4 r = r4[q], kv = k4[q], wv = w4[q];
-                    S[4 * q] = fmaf(r.x, S[4 * q], kv.x * xv);
-                    S[4 * q + 1] = fmaf(r.y, S[4 * q + 1], kv.y * xv);
-                    S[4 * q + 2] = fmaf(r.z, S[4 * q + 2], kv.z * xv);
-                    S[4 * q + 3] = fmaf(r.w, S[4 * q + 3], kv.w * xv);
-                    ya[0] = fmaf(wv.x, S[4 * q], ya[0]);
-                    ya[1] = fmaf(wv.y, S[4 * q + 1], ya[1]);
-                    ya[2] = fmaf(wv.z, S[4 * q + 2], ya[2]);
-                    ya[3] = fmaf(wv.w, S[4 * q + 3], ya[3]);
+                    const float2 a = __ffma2_rn(make_float2(r.x, r.y), make_float2(S[4 * q], S[4 * q + 1]),
+                                                __fmul2_rn(make_float2(kv.x, kv.y), xx));
+                    const float2 c2 = __ffma2_rn(make_float2(r.z, r.w), make_float2(S[4 * q + 2], S[4 * q + 3]),
+                                                 __fmul2_rn(make_float2(kv.z, kv.w), xx));
+                    S[4 * q] = a.x;
+                    S[4 * q + 1] = a.y;
+                    S[4 * q + 2] = c2.x;
+                    S[4 * q + 3] = c2.y;
+                    y01 = __ffma2_rn(make_float2(wv.x, wv.y), a, y01);
+                    y23 = __ffma2_rn(make_float2(wv.z, wv.w), c2, y23);
                 }
             }
+            ya[0] = y01.x;
+            ya[1] = y01.y;
+            ya[2] = y23.x;
+            ya[3] = y23.y;
         } else {
 #pragma unroll
             for (int m = 0; m < KP; ++m) {
@@ -1284,14 +1297,19 @@ __global__ void __launch_bounds__(kN1P) n1_rev_local(ScanDims d, const T *__rest
         if ((K & 3) == 0) {
             const float4 *r4 = reinterpret_cast<const float4 *>(rho_s + (t + 1) * K);
             const float4 *w4 = reinterpret_cast<const float4 *>(wc_s + t * K);
+            const float2 dd = make_float2(dv, dv);
 #pragma unroll
-            for (int q = 0; q < KP / 4; ++q) {
+            for (int q = 0; q < KP / 4; ++q) {  // packed float32 pairs (the same IEEE operations)
                 if (4 * q < K) {
                     const float4 r = r4[q], wv = w4[q];
-                    g[4 * q] = fmaf(r.x, g[4 * q], wv.x * dv);
-                    g[4 * q + 1] = fmaf(r.y, g[4 * q + 1], wv.y * dv);
-                    g[4 * q + 2] = fmaf(r.z, g[4 * q + 2], wv.z * dv);
-                    g[4 * q + 3] = fmaf(r.w, g[4 * q + 3], wv.w * dv);
+                    const float2 a = __ffma2_rn(make_float2(r.x, r.y), make_float2(g[4 * q], g[4 * q + 1]),
+                                                __fmul2_rn(make_float2(wv.x, wv.y), dd));
+                    const float2 c2 = __ffma2_rn(make_float2(r.z, r.w), make_float2(g[4 * q + 2], g[4 * q + 3]),
+                                                 __fmul2_rn(make_float2(wv.z, wv.w), dd));
+                    g[4 * q] = a.x;
+                    g[4 * q + 1] = a.y;
+                    g[4 * q + 2] = c2.x;
+                    g[4 * q + 3] = c2.y;
                 }
             }
         } else {
