@@ -942,7 +942,9 @@ __global__ void __launch_bounds__(kStLaunch, 1)
         if (!*abort_s) {
             const uint32_t zu = lane_base + colZU;  // Z at +0, U at +64
             const float sj = my_coef[2 * KMAX + mj], aj = my_coef[mj], bj = my_coef[KMAX + mj];
-            float dp[4] = {0.f, 0.f, 0.f, 0.f};  // independent partial sums
+            float2 dp[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                            make_float2(0.f, 0.f)};  // independent partial sums (packed float32 pairs)
+            const float2 sj2 = make_float2(sj, sj);
             // 16-column chunks, the next one loading while the current one is used: group 0 reads
             // Z (4 chunks, against dY) and U's first half (2, dx); group 1 reads U (4, against X,
             // the second half also for dx)
@@ -964,23 +966,27 @@ __global__ void __launch_bounds__(kStLaunch, 1)
                             const uint4 rv = row[2 * ch + q];
                             const uint32_t rr[4] = {rv.x, rv.y, rv.z, rv.w};
 #pragma unroll
-                            for (int k = 0; k < 4; ++k) {
-                                const float2 f = bf16x2_to_float2(rr[k]);
-                                dp[k] = fmaf(f.x, cur[8 * q + 2 * k], fmaf(f.y, cur[8 * q + 2 * k + 1], dp[k]));
-                            }
+                            for (int k = 0; k < 4; ++k)
+                                dp[k] = __ffma2_rn(bf16x2_to_float2(rr[k]),
+                                                   make_float2(cur[8 * q + 2 * k], cur[8 * q + 2 * k + 1]), dp[k]);
                         }
                     }
                     if (ch >= 2 && (grp == 1 || ch >= 4)) {  // dx: U columns [0, 32) (group 0) / [32, 64)
                         const int o = 16 * ((ch - 2) & 1);
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) dxr[o + i] = fmaf(sj, cur[i], dxr[o + i]);
+                        for (int i = 0; i < 16; i += 2) {
+                            const float2 v = __ffma2_rn(sj2, make_float2(cur[i], cur[i + 1]),
+                                                        make_float2(dxr[o + i], dxr[o + i + 1]));
+                            dxr[o + i] = v.x;
+                            dxr[o + i + 1] = v.y;
+                        }
                     }
                     if (ch + 1 < nch) tmem_ld_wait16(nxt);
                 }
             }
             tc_fence_before();
             mbar_arrive(&bars[12]);  // the Z / U columns may take step j + 1
-            const float dotv = (dp[0] + dp[1]) + (dp[2] + dp[3]);
+            const float dotv = ((dp[0].x + dp[0].y) + (dp[1].x + dp[1].y)) + ((dp[2].x + dp[2].y) + (dp[3].x + dp[3].y));
 #pragma unroll
             for (int m = 0; m < KMAX; ++m) {
                 if (m == mj) acc_h[m] = bj * dotv;  // group 0: dw_read (inter); group 1: dkappa (inter)
