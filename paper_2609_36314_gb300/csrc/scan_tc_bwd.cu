@@ -440,18 +440,26 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
                         const float4 ka = *reinterpret_cast<const float4 *>(kap_s + k * KMAX);
                         const float4 kb = *reinterpret_cast<const float4 *>(kap_s + k * KMAX + 4);
                         const float kpv[8] = {ka.x, ka.y, ka.z, ka.w, kb.x, kb.y, kb.z, kb.w};
-                        float gam = 0.f, gamt = 0.f;
+                        // modes in packed float32 pairs (K is even)
+                        float2 gam2 = make_float2(0.f, 0.f), gamt2 = make_float2(0.f, 0.f);
+                        const float2 ndE = make_float2(-dE, -dE), gh2 = make_float2(gh, gh);
 #pragma unroll
-                        for (int m = 0; m < KMAX; ++m) {
+                        for (int m = 0; m < KMAX; m += 2) {
                             if (m < K) {
-                                const float W = ex2_approx(-dE * l2r[m]);
-                                const float kp = kpv[m];
-                                const float aa = wr_t[m] * kp * W;
-                                gam += aa;
-                                gamt = fmaf(aa, l2r[m], gamt);  // times log2(e) / tau
-                                dwr_i[m] = fmaf(kp * W, gh, dwr_i[m]);
+                                const float2 l2 = make_float2(l2r[m], l2r[m + 1]);
+                                const float2 x2 = __fmul2_rn(ndE, l2);
+                                const float2 kpW = __fmul2_rn(make_float2(kpv[m], kpv[m + 1]),
+                                                              make_float2(ex2_approx(x2.x), ex2_approx(x2.y)));
+                                const float2 aa = __fmul2_rn(make_float2(wr_t[m], wr_t[m + 1]), kpW);
+                                gam2 = __fadd2_rn(gam2, aa);
+                                gamt2 = __ffma2_rn(aa, l2, gamt2);  // times log2(e) / tau
+                                const float2 dw = __ffma2_rn(kpW, gh2, make_float2(dwr_i[m], dwr_i[m + 1]));
+                                dwr_i[m] = dw.x;
+                                dwr_i[m + 1] = dw.y;
                             }
                         }
+                        float gam = gam2.x + gam2.y;
+                        const float gamt = gamt2.x + gamt2.y;
                         gam = valid ? gam : 0.f;
                         gv[kk] = gam * gv[kk];
                         hv[kk] = gam * hv[kk];
@@ -475,13 +483,18 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
                         const float4 p1 = *reinterpret_cast<const float4 *>(V16ps + j16 * KMAX + 4);
                         const float vk[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
                         const float pk[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
-                        float gam = 0.f, gamp = 0.f;
+                        float2 g2 = make_float2(0.f, 0.f), gp2 = make_float2(0.f, 0.f);
+                        const float2 gh2 = make_float2(gh, gh);
 #pragma unroll
-                        for (int m = 0; m < KMAX; ++m) {
-                            gam = fmaf(uu[m], vk[m], gam);
-                            gamp = fmaf(uu[m], pk[m], gamp);
-                            a16[m] = fmaf(vk[m], gh, a16[m]);
+                        for (int m = 0; m < KMAX; m += 2) {  // packed float32 pairs of modes
+                            const float2 u2 = make_float2(uu[m], uu[m + 1]), v2 = make_float2(vk[m], vk[m + 1]);
+                            g2 = __ffma2_rn(u2, v2, g2);
+                            gp2 = __ffma2_rn(u2, make_float2(pk[m], pk[m + 1]), gp2);
+                            const float2 a2 = __ffma2_rn(v2, gh2, make_float2(a16[m], a16[m + 1]));
+                            a16[m] = a2.x;
+                            a16[m + 1] = a2.y;
                         }
+                        const float gam = g2.x + g2.y, gamp = gp2.x + gp2.y;
                         XX[t * XS + k] = gamp * gh;
                         GHs[t * XS + k] = gh;
                         gv[kk] *= gam;
@@ -533,8 +546,13 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
                         const float4 v0 = *reinterpret_cast<const float4 *>(Vs + k * KMAX);
                         const float4 v1 = *reinterpret_cast<const float4 *>(Vs + k * KMAX + 4);
                         const float vk[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+                        const float2 gh2 = make_float2(gh, gh);
 #pragma unroll
-                        for (int m = 0; m < KMAX; ++m) acc[m] = fmaf(vk[m], gh, acc[m]);
+                        for (int m = 0; m < KMAX; m += 2) {
+                            const float2 s2 = __ffma2_rn(make_float2(vk[m], vk[m + 1]), gh2, make_float2(acc[m], acc[m + 1]));
+                            acc[m] = s2.x;
+                            acc[m + 1] = s2.y;
+                        }
                         gv[kk] *= gm[kk];  // Gamma o G
                         hv[kk] *= gm[kk];  // Gamma o H
                     }
@@ -600,14 +618,17 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
                 const float4 w0 = *reinterpret_cast<const float4 *>(wr_s + tt * KMAX);
                 const float4 w1 = *reinterpret_cast<const float4 *>(wr_s + tt * KMAX + 4);
                 const float wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+                const float2 ndE = make_float2(-dE, -dE), gh2 = make_float2(gh, gh);
 #pragma unroll
-                for (int m = 0; m < KMAX; ++m) {
+                for (int m = 0; m < KMAX; m += 2) {  // packed float32 pairs of modes (K is even)
                     if (m < K) {
-                        const float v = wv[m] * ex2_approx(-dE * l2r[m]);
-                        if (i & 1)
-                            dk2[m] = fmaf(v, gh, dk2[m]);
-                        else
-                            dk[m] = fmaf(v, gh, dk[m]);
+                        const float2 x2 = __fmul2_rn(ndE, make_float2(l2r[m], l2r[m + 1]));
+                        const float2 v = __fmul2_rn(make_float2(wv[m], wv[m + 1]),
+                                                    make_float2(ex2_approx(x2.x), ex2_approx(x2.y)));
+                        float *dst = (i & 1) ? dk2 : dk;
+                        const float2 r2 = __ffma2_rn(v, gh2, make_float2(dst[m], dst[m + 1]));
+                        dst[m] = r2.x;
+                        dst[m + 1] = r2.y;
                     }
                 }
             }
@@ -622,8 +643,13 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
                     const float4 u0 = *reinterpret_cast<const float4 *>(u16);
                     const float4 u1 = *reinterpret_cast<const float4 *>(u16 + 4);
                     const float uu[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+                    const float2 gh2 = make_float2(gh, gh);
 #pragma unroll
-                    for (int m = 0; m < KMAX; ++m) a16[m] = fmaf(uu[m], gh, a16[m]);
+                    for (int m = 0; m < KMAX; m += 2) {  // packed float32 pairs of modes
+                        const float2 a2 = __ffma2_rn(make_float2(uu[m], uu[m + 1]), gh2, make_float2(a16[m], a16[m + 1]));
+                        a16[m] = a2.x;
+                        a16[m + 1] = a2.y;
+                    }
                 }
                 const float dE16 = diff_f2(E_s[32 * J + 15], Ek);
 #pragma unroll
@@ -642,12 +668,13 @@ __global__ void __launch_bounds__(kIntraLaunch, 1)
                         const float4 u0 = *reinterpret_cast<const float4 *>(Ufp + tt * 32 + 8 * J);
                         const float4 u1 = *reinterpret_cast<const float4 *>(Ufp + tt * 32 + 8 * J + 4);
                         const float uu[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+                        const float2 gh2 = make_float2(gh, gh);
+                        float *sd = (u & 1) ? s1 : s0;
 #pragma unroll
-                        for (int m = 0; m < KMAX; ++m) {
-                            if (u & 1)
-                                s1[m] = fmaf(uu[m], gh, s1[m]);
-                            else
-                                s0[m] = fmaf(uu[m], gh, s0[m]);
+                        for (int m = 0; m < KMAX; m += 2) {  // packed float32 pairs of modes
+                            const float2 r2 = __ffma2_rn(make_float2(uu[m], uu[m + 1]), gh2, make_float2(sd[m], sd[m + 1]));
+                            sd[m] = r2.x;
+                            sd[m + 1] = r2.y;
                         }
                     }
                 }
