@@ -683,19 +683,28 @@ __global__ void __launch_bounds__(kOutLaunch, 2)
                     for (int kk = 0; kk < 8; ++kk) gv[kk] = q8 == grp ? ga[kk] : gb[kk];
                 }
                 if (dstep) {
+                    // branch-free over the eight columns (a pair above the diagonal runs with its
+                    // decay exponent clamped to zero and is masked after), modes in packed float32
+                    // pairs (K is even)
 #pragma unroll
                     for (int kk = 0; kk < 8; ++kk) {
                         const int k = k0 + kk;
-                        float v = 0.f;
-                        if (k <= t && t < n) {
-                            const float dE = diff_f2(Et2, E_s[k]);
-                            float gam = 0.f;
+                        const bool valid = k <= t && t < n;
+                        const float dE = fmaxf(diff_f2(Et2, E_s[k]), 0.f);
+                        const float4 ka = *reinterpret_cast<const float4 *>(kap_s + k * KMAX);
+                        const float4 kb = *reinterpret_cast<const float4 *>(kap_s + k * KMAX + 4);
+                        const float kpv[8] = {ka.x, ka.y, ka.z, ka.w, kb.x, kb.y, kb.z, kb.w};
+                        const float2 ndE = make_float2(-dE, -dE);
+                        float2 g2 = make_float2(0.f, 0.f);
 #pragma unroll
-                            for (int m = 0; m < KMAX; ++m)
-                                if (m < K) gam = fmaf(wr_t[m] * kap_s[k * KMAX + m], ex2_approx(-dE * l2t[m]), gam);
-                            v = gam * gv[kk];
+                        for (int m = 0; m < KMAX; m += 2) {
+                            if (m < K) {
+                                const float2 x2 = __fmul2_rn(ndE, make_float2(l2t[m], l2t[m + 1]));
+                                g2 = __ffma2_rn(__fmul2_rn(make_float2(wr_t[m], wr_t[m + 1]), make_float2(kpv[m], kpv[m + 1])),
+                                                make_float2(ex2_approx(x2.x), ex2_approx(x2.y)), g2);
+                            }
                         }
-                        gv[kk] = v;
+                        gv[kk] = valid ? (g2.x + g2.y) * gv[kk] : 0.f;
                     }
                 } else if (!upper) {
                     const float dE = diff_f2(Et2, E_s[32 * kc + 15]);
