@@ -1476,7 +1476,20 @@ __device__ __forceinline__ int warp_halving_sum(float (&v)[NV], int lane) {
 // kappa B_k exp(-(E_t - E_k)/tau_m) to put(t, k, .), Gamma' o H to XR, and the intra dw_read-like
 // sums over k (a halving-exchange sum across the warp).  Column pass, one warp per column k with
 // the lanes on the rows t: the intra dkappa B-like sums over t.  Every entry has one writer.
-template <int KP, typename PutGamma>
+// exp(-x tau^-1) as 2^(-x tau^-1 log2 e) by the approximate hardware exp2 (relative error ~1e-6 over
+// the arguments of the pair decays, inside the bf16 tolerance); FAST = false keeps expf
+template <bool FAST>
+__device__ __forceinline__ float pair_decay(float dE, float it) {
+    if constexpr (FAST) {
+        float y;
+        asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(-dE * (it * 1.4426950408889634f)));
+        return y;
+    } else {
+        return expf(-dE * it);
+    }
+}
+
+template <int KP, bool FAST, typename PutGamma>
 __device__ __forceinline__ void n1_pair_passes(int n, int K, const float *itau, const float2 *Ef_s,
                                                const N1Arrays &a, const float *H, float *XR, PutGamma put) {
     constexpr int Q1 = kN1BQ + 1;
@@ -1496,7 +1509,7 @@ __device__ __forceinline__ void n1_pair_passes(int n, int K, const float *itau, 
         for (int m = 0; m < KP; ++m) {
             float av = 0.f, kw = 0.f;
             if (m < K && ok) {
-                kw = a.kbT[m * kN1BQ + lane] * expf(-dE * it[m]);
+                kw = a.kbT[m * kN1BQ + lane] * pair_decay<FAST>(dE, it[m]);
                 av = a.wc[t * K + m] * kw;
             }
             gam += av;
@@ -1518,7 +1531,7 @@ __device__ __forceinline__ void n1_pair_passes(int n, int K, const float *itau, 
         float dk[KP];
 #pragma unroll
         for (int m = 0; m < KP; ++m)
-            dk[m] = (m < K && ok) ? a.wcT[m * kN1BQ + lane] * expf(-dE * it[m]) * hv : 0.f;
+            dk[m] = (m < K && ok) ? a.wcT[m * kN1BQ + lane] * pair_decay<FAST>(dE, it[m]) * hv : 0.f;
         const int m0 = warp_halving_sum<KP>(dk, lane);
         if ((lane & kDup) == 0 && m0 < K) a.dkbi[k * K + m0] = dk[0];
     }
@@ -1835,7 +1848,7 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd(
     for (int idx = tid; idx < kN1BQ * kGS; idx += blockDim.x) Gm[idx] = 0.f;
     for (int idx = tid; idx < kN1BQ * Q1; idx += blockDim.x) XR[idx] = 0.f;
     __syncthreads();
-    n1_pair_passes<KP>(n, K, itau, Ef_s, a, H, XR, [&](int t, int k, float v) { Gm[t * kGS + k] = v; });
+    n1_pair_passes<KP, false>(n, K, itau, Ef_s, a, H, XR, [&](int t, int k, float v) { Gm[t * kGS + k] = v; });
     __syncthreads();
 
     // ---- P3: rectangle sums of Gamma' o H over pairs k < t <= t' (row prefix, column suffix)
@@ -2080,7 +2093,7 @@ __global__ void __launch_bounds__(kThreads) n1_chunk_bwd_tc(
     // ---- P2: pair passes; Gamma (hi, lo) into rows t and 32 + KS + t of P4's B, column k, and
     // s = kappa B u into rows 32 + m and 64 + KS + m
     if (!bad) {
-        n1_pair_passes<KP>(n, K, itau, Ef_s, a, H, XR, [&](int t, int k, float v) {
+        n1_pair_passes<KP, true>(n, K, itau, Ef_s, a, H, XR, [&](int t, int k, float v) {
             st_bf16_pair(img, uint32_t(t), uint32_t(32 + KS + t), uint32_t(k), v);
         });
         for (int idx = tid; idx < K * kN1BQ; idx += blockDim.x) {

@@ -712,13 +712,15 @@ __global__ void __launch_bounds__(kOutLaunch, 2)
 #pragma unroll
                     for (int m = 0; m < KMAX; ++m) u16[m] = m < K ? wr_t[m] * ex2_approx(-dE * l2t[m]) : 0.f;
 #pragma unroll
-                    for (int kk = 0; kk < 8; ++kk) {
+                    for (int kk = 0; kk < 8; ++kk) {  // the K = 8 mode sum in packed float32 pairs
                         const float *v16 = V16s + (16 * kc + ((k0 + kk) & 15)) * KMAX;
                         const float4 v0 = *reinterpret_cast<const float4 *>(v16);
                         const float4 v1 = *reinterpret_cast<const float4 *>(v16 + 4);
-                        const float gam = u16[0] * v0.x + u16[1] * v0.y + u16[2] * v0.z + u16[3] * v0.w +
-                                          u16[4] * v1.x + u16[5] * v1.y + u16[6] * v1.z + u16[7] * v1.w;
-                        gv[kk] = t < n ? gam * gv[kk] : 0.f;
+                        float2 g2 = __fmul2_rn(make_float2(u16[0], u16[1]), make_float2(v0.x, v0.y));
+                        g2 = __ffma2_rn(make_float2(u16[2], u16[3]), make_float2(v0.z, v0.w), g2);
+                        g2 = __ffma2_rn(make_float2(u16[4], u16[5]), make_float2(v1.x, v1.y), g2);
+                        g2 = __ffma2_rn(make_float2(u16[6], u16[7]), make_float2(v1.z, v1.w), g2);
+                        gv[kk] = t < n ? (g2.x + g2.y) * gv[kk] : 0.f;
                     }
                 } else {
 #pragma unroll
