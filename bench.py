@@ -188,30 +188,30 @@ def fwd_bytes_per_token_head(s):
 # the kernel's sources hash to the digest they had when they were profiled.
 PROFILED_TRAFFIC_BATCH = 2
 PROFILED_TRAFFIC = {
-    "coef_tc": ("scan_tc.cu", "7389ea60990165f0", 23.10e6 + 38.92e6),
-    "state_pass_fwd_tc": ("scan_tc.cu", "7389ea60990165f0", 138.80e6 + 479.22e6),
-    "chunk_fwd_tc": ("scan_tc.cu", "7389ea60990165f0", 717.32e6 + 57.95e6),
-    "state_pass_rev_tc": ("scan_tc.cu", "7389ea60990165f0", 139.26e6 + 479.18e6),
-    "bwd_intra_tc": ("scan_tc_bwd.cu", "627544f5ba419d34", 182.99e6 + 123.75e6),
-    "bwd_state_tc": ("scan_tc_bwd.cu", "627544f5ba419d34", 1466.46e6 + 166.23e6),
-    "bwd_final_tc": ("scan_tc_bwd.cu", "627544f5ba419d34", 323.48e6 + 67.26e6),
+    "coef_tc": ("scan_tc.cu", "6165989fffff61ad", 23.10e6 + 38.93e6),
+    "state_pass_fwd_tc": ("scan_tc.cu", "6165989fffff61ad", 138.87e6 + 479.23e6),
+    "chunk_fwd_tc": ("scan_tc.cu", "6165989fffff61ad", 717.33e6 + 57.85e6),
+    "state_pass_rev_tc": ("scan_tc.cu", "6165989fffff61ad", 139.00e6 + 479.77e6),
+    "bwd_intra_tc": ("scan_tc_bwd.cu", "0352bc18c55c4601", 183.02e6 + 122.53e6),
+    "bwd_state_tc": ("scan_tc_bwd.cu", "0352bc18c55c4601", 1467.70e6 + 167.03e6),
+    "bwd_final_tc": ("scan_tc_bwd.cu", "0352bc18c55c4601", 323.47e6 + 67.30e6),
 }
 
 # DRAM bytes (read + write) per launch of the scan-parameter and mixer-glue kernels at the
 # benchmark's training shape (B8 L4096), from one ncu capture of bench.py's mixer section.
 PROFILED_MIXER_TRAFFIC = {
-    "param_prep_fwd": ("param_prep.cu", "296e863496dae618", 92.31e6 + 43.92e6),
-    "param_prep_bwd": ("param_prep.cu", "296e863496dae618", 184.62e6 + 64.71e6),
-    "conv1d_fwd": ("mixer_glue.cu", "eca11e4487de8cc6", 285.37e6 + 236.23e6),
-    "conv1d_bwd": ("mixer_glue.cu", "eca11e4487de8cc6", 570.77e6 + 253.83e6),
-    "gated_rmsnorm_fwd": ("mixer_glue.cu", "eca11e4487de8cc6", 536.96e6 + 235.98e6),
-    "gated_rmsnorm_bwd": ("mixer_glue.cu", "eca11e4487de8cc6", 805.42e6 + 497.52e6),
+    "param_prep_fwd": ("param_prep.cu", "a42db5452b48d9ca", 92.31e6 + 43.86e6),
+    "param_prep_bwd": ("param_prep.cu", "a42db5452b48d9ca", 184.63e6 + 64.66e6),
+    "conv1d_fwd": ("mixer_glue.cu", "c05c49b825953b57", 285.36e6 + 233.22e6),
+    "conv1d_bwd": ("mixer_glue.cu", "c05c49b825953b57", 570.67e6 + 252.29e6),
+    "gated_rmsnorm_fwd": ("mixer_glue.cu", "c05c49b825953b57", 536.95e6 + 235.98e6),
+    "gated_rmsnorm_bwd": ("mixer_glue.cu", "c05c49b825953b57", 805.43e6 + 491.07e6),
 }
 
 # DRAM bytes (read + write) of one decode_step launch of the decode workload (B128 H64 P64 N128
 # K8, float32 state), from one ncu capture (summarised under profiles/); used only while
 # decode.cu hashes to the digest it had when profiled.
-PROFILED_DECODE_TRAFFIC = ("decode.cu", "7a02e3079579523a", 2151.60e6 + 2098.05e6)
+PROFILED_DECODE_TRAFFIC = ("decode.cu", "853bdd0b44e394c4", 2151.50e6 + 2098.02e6)
 
 
 def source_digest(fname: str) -> str:
