@@ -513,7 +513,9 @@ def bench_train(args, ctx, rank, local):
     roofline = None
     if dom:
         kind, work = algorithmic_work(dom, s, units)
-        if kind == "flops":
+        if dom == "bwd_intra_tc":  # bound by its per-pair FP32 work, not by its small tensor-core products
+            roofline = dict(kern[dom]["roofline_alu"], traffic=profiled_traffic(dom, s.batch))
+        elif kind == "flops":
             roofline = roofline_of(dom, "flops_tc" if dom.endswith("_tc") else "flops_alu", work,
                                    kern[dom]["avg_ms"], peaks, profiled_traffic(dom, s.batch))
         elif kind == "bytes":
