@@ -135,3 +135,21 @@ def test_decode_paper_layer_shape(dtype):
     yr, str_ = _oracle_decode(dec, h_or, 16)
     assert_close("y", to_host64(y), yr, tol(dtype))
     assert_close("state", to_host64(st), str_, tol(dtype))
+
+
+@pytest.mark.parametrize("K,P,G", [(5, 40, 1), (1, 33, 1), (4, 64, 2)])
+def test_decode_n1_shapes(K, P, G):
+    """N = 1 decode (one thread per (b, h, p)) off the paper's shape: odd mode counts, a single
+    mode, head dims that are not a multiple of 32, B/C groups; float32 and 8 steps."""
+    s = synth.Shape(3, 40, 4, P, G, 1, K, 0, "f32")
+    host = synth.make_scan_inputs(s, seed=60 + K)
+    dv = dev_inputs(host)
+    _, hf = scan_fwd(dv["x"], dv["dt"], dv["alpha"], dv["lam"], dv["tau"], dv["B"], dv["C"],
+                     dv["w_read"], dv["w_write"], dv["D"])
+    dec, y, st = _run_decode(s, 8, 61 + K, to_host64(hf))
+    o = f64_inputs(host)
+    _, h_or = oracle.fwd(o["x"], o["dt"], o["alpha"], o["lam"], o["tau"], o["B"], o["C"],
+                         o["w_read"], o["w_write"], o["D"])
+    yr, str_ = _oracle_decode(dec, h_or, 8)
+    assert_close("y", to_host64(y), yr, tol("f32"))
+    assert_close("state", to_host64(st), str_, tol("f32"))

@@ -55,6 +55,14 @@ def test_conv_widths(W):
     _conv_case(2, 97, 64, W, "f32", silu=False, with_state=True, seed=W)
 
 
+@pytest.mark.parametrize("W", [1, 2, 3, 5, 8])
+def test_conv_widths_bf16_tiles(W):
+    """bf16 with 8-divisible channels takes the shared-memory tile kernels (forward and backward):
+    every width, a sequence across two 64-position tiles and the carried state."""
+    _conv_case(2, 150, 72, W, "bf16", silu=True, with_state=True, seed=40 + W)
+    _conv_case(1, W // 2 + 1, 16, W, "bf16", silu=False, with_state=True, seed=50 + W)  # L < W possible
+
+
 @pytest.mark.parametrize("C", [1, 33, 129])
 def test_conv_odd_channels(C):
     _conv_case(3, 70, C, 4, "bf16", silu=True, with_state=True, seed=C)
