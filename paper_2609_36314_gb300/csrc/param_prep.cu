@@ -185,7 +185,7 @@ __device__ __forceinline__ void softmax_bwd_row(const float *w, float *dw, int K
 }
 
 template <typename T, int KP, bool VEC>
-__global__ void __launch_bounds__(256) param_prep_bwd_kernel(PrepArgs a, int64_t hstride) {
+__global__ void __launch_bounds__(256, KP <= 8 ? 3 : 1) param_prep_bwd_kernel(PrepArgs a, int64_t hstride) {
     extern __shared__ float red[];  // [min(H, blockDim)][KP + 1] when H <= blockDim
     __shared__ float ltab_s[kTauTab], itab_s[kTauTab];  // ln tau and 1 / tau per (head, mode)
     const int K = a.K, H = a.H;
@@ -249,8 +249,11 @@ __global__ void __launch_bounds__(256) param_prep_bwd_kernel(PrepArgs a, int64_t
     if (shared_slots) {
         if (i < hstride) {
             if (a.ddt_bias) atomicAdd(&red[h * (KP + 1) + KP], acc_bias);
-            if (a.dtau)
-                for (int m = 0; m < K; ++m) atomicAdd(&red[h * (KP + 1) + m], acc_tau[m]);
+            if (a.dtau) {
+#pragma unroll
+                for (int m = 0; m < KP; ++m)  // unrolled: the sums stay in registers
+                    if (m < K) atomicAdd(&red[h * (KP + 1) + m], acc_tau[m]);
+            }
         }
         __syncthreads();
         for (int q = threadIdx.x; q < H * (KP + 1); q += blockDim.x) {
@@ -263,8 +266,11 @@ __global__ void __launch_bounds__(256) param_prep_bwd_kernel(PrepArgs a, int64_t
         }
     } else if (i < hstride) {  // H > blockDim: the block's threads all have different heads
         if (a.ddt_bias) atomicAdd(a.ddt_bias + h, acc_bias);
-        if (a.dtau)
-            for (int m = 0; m < K; ++m) atomicAdd(a.dtau + h * K + m, acc_tau[m]);
+        if (a.dtau) {
+#pragma unroll
+            for (int m = 0; m < KP; ++m)
+                if (m < K) atomicAdd(a.dtau + h * K + m, acc_tau[m]);
+        }
     }
 }
 
@@ -276,10 +282,8 @@ cudaError_t launch_kp(const PrepArgs &a, bool backward, bool vec, cudaStream_t s
     int dev = 0, sms = 152;
     if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int64_t want = (a.n + threads - 1) / threads;
-    // the forward has no sums: one row per thread; the backward caps its grid (its per-block
-    // reductions end in global atomics)
-    const int blocks = int(std::max<int64_t>(1, std::min<int64_t>(want, backward ? int64_t(sms) * 8 : int64_t(1) << 30)));
-    if (!backward) {
+    if (!backward) {  // no sums: one row per thread
+        const int blocks = int(std::max<int64_t>(1, std::min<int64_t>(want, int64_t(1) << 30)));
         trace_begin("param_prep_fwd", st);
         if (vec)
             param_prep_fwd_kernel<T, KP, true><<<blocks, threads, 0, st>>>(a);
@@ -288,9 +292,19 @@ cudaError_t launch_kp(const PrepArgs &a, bool backward, bool vec, cudaStream_t s
         trace_end(st);
         return cudaGetLastError();
     }
-    const int64_t total = int64_t(blocks) * threads;
-    const int64_t hstride = (total / a.H) * a.H;  // >= H: blocks >= ceil(n / 256) >= ceil(H / 256)
+    // the backward's per-block sums end in global atomics: one resident wave of blocks, each
+    // walking its rows with a stride of whole head cycles
     const size_t smem = (a.H <= threads) ? size_t(a.H) * (KP + 1) * sizeof(float) : 0;
+    int occ = 0;
+    if (vec)
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, param_prep_bwd_kernel<T, KP, true>, threads, smem);
+    else
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, param_prep_bwd_kernel<T, KP, false>, threads, smem);
+    // at least ceil(H / 256) blocks, so that the stride holds one whole head cycle (n >= H rows)
+    const int64_t cap = std::max<int64_t>(int64_t(sms) * std::max(occ, 1), (a.H + threads - 1) / threads);
+    const int blocks = int(std::max<int64_t>(1, std::min<int64_t>(want, cap)));
+    const int64_t total = int64_t(blocks) * threads;
+    const int64_t hstride = (total / a.H) * a.H;  // >= H
     trace_begin("param_prep_bwd", st);
     if (vec)
         param_prep_bwd_kernel<T, KP, true><<<blocks, threads, smem, st>>>(a, hstride);

@@ -78,6 +78,13 @@ def test_prep_many_heads_and_no_bias():
     _check(synth.Shape(1, 9, 300, 1, 1, 1, 8, 0, "f32"), bias=False, seed=3)
 
 
+@pytest.mark.parametrize("K", [8, 16])
+def test_prep_more_heads_than_one_wave_of_threads(K):
+    """More heads than the backward's resident threads (its row stride must still hold whole
+    head cycles), and per-head sums across only a couple of positions."""
+    _check(synth.Shape(1, 2, 45000, 1, 1, 1, K, 0, "f32"), seed=11 + K)
+
+
 def test_prep_empty_sequence():
     _check(synth.Shape(2, 0, 4, 1, 1, 1, 8, 0, "bf16"))
 
