@@ -200,8 +200,8 @@ PROFILED_TRAFFIC = {
 # DRAM bytes (read + write) per launch of the scan-parameter and mixer-glue kernels at the
 # benchmark's training shape (B8 L4096), from one ncu capture of bench.py's mixer section.
 PROFILED_MIXER_TRAFFIC = {
-    "param_prep_fwd": ("param_prep.cu", "a42db5452b48d9ca", 92.31e6 + 43.86e6),
-    "param_prep_bwd": ("param_prep.cu", "a42db5452b48d9ca", 184.63e6 + 64.66e6),
+    "param_prep_fwd": ("param_prep.cu", "60ecfacdc7d4a027", 92.31e6 + 43.81e6),
+    "param_prep_bwd": ("param_prep.cu", "60ecfacdc7d4a027", 184.63e6 + 60.37e6),
     "conv1d_fwd": ("mixer_glue.cu", "c05c49b825953b57", 285.36e6 + 233.22e6),
     "conv1d_bwd": ("mixer_glue.cu", "c05c49b825953b57", 570.67e6 + 252.29e6),
     "gated_rmsnorm_fwd": ("mixer_glue.cu", "c05c49b825953b57", 536.95e6 + 235.98e6),
