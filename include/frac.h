@@ -19,8 +19,10 @@
  *     aligned at least to their element size, and must not alias each other (except where
  *     stated).  16-byte alignment of every tensor lets the library pick its vectorised and
  *     TMA-fed kernels; otherwise it uses kernels with scalar accesses.  The library
- *     never allocates device memory and keeps no state between calls apart from a
- *     thread-local error message.
+ *     allocates no device memory in any call; the only device memory it owns is the fixed
+ *     scratch array of frac_scan_fwd_static (a static device array of the module).  Between
+ *     calls it keeps a thread-local error message, the launch trace when tracing is on, and
+ *     the cached address of that array.
  *   - `stream` is a cudaStream_t (NULL = the legacy default stream).  Every call only
  *     enqueues work on `stream`; results are valid once the stream has completed.
  *   - Element types: x, B, C, w_read, w_write, y and their gradients use `dims->dtype`

@@ -127,3 +127,23 @@ def test_param_prep_rejects_bad_arguments(bad):
     assert st == 1
     st = lib.frac_param_prep_bwd(ctypes.byref(dims), cfg_ref, *([p] * 19), None)
     assert st == 1
+
+
+def test_plain_c_caller(tmp_path):
+    """tests/abi_check.c includes the header as C99, links libfrac.so and checks the calls that
+    need no GPU (status strings, workspace queries, rejection before anything is enqueued)."""
+    import shutil
+    import subprocess
+    from paper_2609_36314_gb300 import build
+    if shutil.which("gcc") is None:
+        pytest.skip("gcc not found")
+    lib = _lib.load()  # builds the library if needed
+    del lib
+    libdir = os.path.dirname(build.LIB_PATH)
+    exe = str(tmp_path / "abi_check")
+    subprocess.run(["gcc", "-std=c99", "-Wall", "-Wextra", "-Werror", "-I", os.path.join(ROOT, "include"),
+                    os.path.join(ROOT, "tests", "abi_check.c"), "-L", libdir, "-lfrac",
+                    "-Wl,-rpath," + libdir, "-o", exe], check=True, capture_output=True, text=True)
+    out = subprocess.run([exe], capture_output=True, text=True, timeout=120)
+    assert out.returncode == 0, out.stderr
+    assert out.stdout.strip() == "ok"
