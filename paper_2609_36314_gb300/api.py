@@ -47,6 +47,29 @@ def _need(t, name, dtype, shape=None):
     return t
 
 
+def _need_out(t, name, dtype, shape):
+    """An output the caller supplied: the kernels write exactly `shape` elements of `dtype`."""
+    if t is not None:
+        _need(t, name, dtype, shape)
+    return t
+
+
+def _need_scan_inputs(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, h0, dims):
+    Bz, L, H, P, G, N, K = dims
+    dt_, f32 = x.dtype, torch.float32
+    _need(x, "x", dt_, (Bz, L, H, P))
+    for name, t in (("dt", dt), ("alpha", alpha), ("lam", lam)):
+        _need(t, name, f32, (Bz, L, H))
+    _need(tau, "tau", f32, (H, K))
+    _need(B, "B", dt_, (Bz, L, G, N))
+    _need(C, "C", dt_, (Bz, L, G, N))
+    _need(w_read, "w_read", dt_, (Bz, L, H, K))
+    _need(w_write, "w_write", dt_, (Bz, L, H, K))
+    _need(D, "D", f32, (H,))
+    if h0 is not None:
+        _need(h0, "h0", f32, (Bz, H, K, P, N))
+
+
 def _scan_dims(x, B, tau, chunk, force_simt, reuse_fwd_states=False):
     if x.dim() != 4 or B.dim() != 4 or tau.dim() != 2:
         raise ValueError("x [B,L,H,P], B/C [B,L,G,N], tau [H,K] expected")
@@ -83,20 +106,13 @@ def scan_fwd(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, h0=None, *, chunk
              force_simt=False, want_final_state=True, y=None, h_final=None, workspace=None,
              stream=None):
     """Chunked forward scan.  Returns (y [B,L,H,P], h_final [B,H,K,P,N] or None)."""
-    dims, (Bz, L, H, P, G, N, K) = _scan_dims(x, B, tau, chunk, force_simt)
-    dt_ = x.dtype
+    dims, shp = _scan_dims(x, B, tau, chunk, force_simt)
+    Bz, L, H, P, G, N, K = shp
     f32 = torch.float32
-    _need(x, "x", dt_, (Bz, L, H, P))
-    for name, t in (("dt", dt), ("alpha", alpha), ("lam", lam)):
-        _need(t, name, f32, (Bz, L, H))
-    _need(tau, "tau", f32, (H, K))
-    _need(B, "B", dt_, (Bz, L, G, N))
-    _need(C, "C", dt_, (Bz, L, G, N))
-    _need(w_read, "w_read", dt_, (Bz, L, H, K))
-    _need(w_write, "w_write", dt_, (Bz, L, H, K))
-    _need(D, "D", f32, (H,))
-    if h0 is not None:
-        _need(h0, "h0", f32, (Bz, H, K, P, N))
+    _need_scan_inputs(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, h0, shp)
+    _need_out(y, "y", x.dtype, (Bz, L, H, P))
+    if want_final_state:
+        _need_out(h_final, "h_final", f32, (Bz, H, K, P, N))
     if y is None:
         y = torch.empty_like(x)
     if want_final_state and h_final is None:
@@ -116,7 +132,12 @@ def scan_fwd_static(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, h0=None, *
     array (FRAC_SCAN_FWD_STATIC_SCRATCH_BYTES) holds the per-chunk states, so this call
     allocates nothing besides the outputs it is not given.  Calls that overlap on the GPU
     race on that array."""
-    dims, (Bz, L, H, P, G, N, K) = _scan_dims(x, B, tau, chunk, force_simt)
+    dims, shp = _scan_dims(x, B, tau, chunk, force_simt)
+    Bz, L, H, P, G, N, K = shp
+    _need_scan_inputs(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, h0, shp)
+    _need_out(y, "y", x.dtype, (Bz, L, H, P))
+    if want_final_state:
+        _need_out(h_final, "h_final", torch.float32, (Bz, H, K, P, N))
     if y is None:
         y = torch.empty_like(x)
     if want_final_state and h_final is None:
@@ -137,18 +158,23 @@ def scan_bwd(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, dy, h0=None, dh_f
     bwd_workspace_size)."""
     if reuse_fwd_states and workspace is None:
         raise ValueError("reuse_fwd_states needs the workspace of the forward call")
-    dims, (Bz, L, H, P, G, N, K) = _scan_dims(x, B, tau, chunk, force_simt, reuse_fwd_states)
+    dims, shp = _scan_dims(x, B, tau, chunk, force_simt, reuse_fwd_states)
+    Bz, L, H, P, G, N, K = shp
     dt_ = x.dtype
     f32 = torch.float32
+    _need_scan_inputs(x, dt, alpha, lam, tau, B, C, w_read, w_write, D, h0, shp)
     _need(dy, "dy", dt_, (Bz, L, H, P))
     if dh_final is not None:
         _need(dh_final, "dh_final", f32, (Bz, H, K, P, N))
-    if h0 is not None:
-        _need(h0, "h0", f32, (Bz, H, K, P, N))
-    for name, t in (("x", x), ("B", B), ("C", C), ("w_read", w_read), ("w_write", w_write)):
-        _need(t, name, dt_)
-    for name, t in (("dt", dt), ("alpha", alpha), ("lam", lam), ("tau", tau), ("D", D)):
-        _need(t, name, f32)
+    if out is not None:
+        for name, dtype, shape in (("dx", dt_, (Bz, L, H, P)), ("ddt", f32, (Bz, L, H)),
+                                   ("dalpha", f32, (Bz, L, H)), ("dlam", f32, (Bz, L, H)),
+                                   ("dB", dt_, (Bz, L, G, N)), ("dC", dt_, (Bz, L, G, N)),
+                                   ("dw_read", dt_, (Bz, L, H, K)), ("dw_write", dt_, (Bz, L, H, K)),
+                                   ("dD", f32, (H,))):
+            _need(out.get(name), name, dtype, shape)
+        _need_out(out.get("dh0"), "dh0", f32, (Bz, H, K, P, N))
+        _need_out(out.get("dtau"), "dtau", f32, (H, K))
     g = out if out is not None else dict(
         dx=torch.empty_like(x), ddt=torch.empty_like(dt), dalpha=torch.empty_like(alpha),
         dlam=torch.empty_like(lam), dB=torch.empty_like(B), dC=torch.empty_like(C),
@@ -187,6 +213,7 @@ def decode_step(x_t, dt, alpha, lam, tau, B_t, C_t, w_read, w_write, D, state, y
     _need(tau, "tau", f32, (H, K))
     _need(D, "D", f32, (H,))
     _need(state, "state", f32, (Bz, H, K, P, N))
+    _need_out(y_t, "y_t", dt_, (Bz, H, P))
     if y_t is None:
         y_t = torch.empty_like(x_t)
     dims = make_dims(Bz, 1, H, P, G, N, K, dt_)
@@ -236,6 +263,11 @@ def param_prep_fwd(dt_raw, alpha_raw, lam_raw, g_read, g_write, tau, dt_bias=Non
     _need(g_read, "g_read", g_read.dtype)
     if dt_bias is not None:
         _need(dt_bias, "dt_bias", f32, (tau.shape[0],))
+    if out is not None:
+        for name in ("dt", "alpha", "lam"):
+            _need(out.get(name), name, f32, dt_raw.shape)
+        for name in ("w_read", "w_write"):
+            _need(out.get(name), name, g_read.dtype, g_read.shape)
     o = out if out is not None else dict(
         dt=torch.empty_like(dt_raw), alpha=torch.empty_like(dt_raw), lam=torch.empty_like(dt_raw),
         w_read=torch.empty_like(g_read), w_write=torch.empty_like(g_read))
