@@ -314,18 +314,23 @@ def _conv_dims(x, w, silu):
                              _lib.FRAC_CONV_SILU if silu else 0)
 
 
-def conv1d_fwd(x, w, bias=None, state=None, *, silu=False, want_state=False, stream=None):
-    """Depthwise causal conv1d over [B, L, C] (optionally SiLU).  Returns (u, final state
-    [B, C, W-1] or None)."""
-    dims = _conv_dims(x, w, silu)
-    _need(x, "x", x.dtype)
-    _need(w, "w", torch.float32)
+def _need_conv_inputs(x, w, bias, state):
     B, L, C = x.shape
     W = w.shape[1]
+    _need(x, "x", x.dtype)
+    _need(w, "w", torch.float32, (C, W))
     if bias is not None:
         _need(bias, "bias", torch.float32, (C,))
     if state is not None:
         _need(state, "state", x.dtype, (B, C, W - 1))
+    return B, L, C, W
+
+
+def conv1d_fwd(x, w, bias=None, state=None, *, silu=False, want_state=False, stream=None):
+    """Depthwise causal conv1d over [B, L, C] (optionally SiLU).  Returns (u, final state
+    [B, C, W-1] or None)."""
+    dims = _conv_dims(x, w, silu)
+    B, L, C, W = _need_conv_inputs(x, w, bias, state)
     u = torch.empty_like(x)
     fin = torch.empty((B, C, W - 1), dtype=x.dtype, device=x.device) if want_state else None
     _lib.check(_lib.load().frac_conv1d_fwd(ctypes.byref(dims), _ptr(x), _ptr(w), _ptr(bias),
@@ -337,8 +342,7 @@ def conv1d_fwd(x, w, bias=None, state=None, *, silu=False, want_state=False, str
 def conv1d_bwd(x, w, du, bias=None, state=None, *, silu=False, want_dstate=False, stream=None):
     """Backward of conv1d_fwd.  Returns dict(dx, dw, dbias, dstate)."""
     dims = _conv_dims(x, w, silu)
-    B, L, C = x.shape
-    W = w.shape[1]
+    B, L, C, W = _need_conv_inputs(x, w, bias, state)
     _need(du, "du", x.dtype, x.shape)
     g = dict(dx=torch.empty_like(x), dw=torch.empty_like(w),
              dbias=torch.empty(C, dtype=torch.float32, device=x.device) if bias is not None else None,
@@ -351,10 +355,16 @@ def conv1d_bwd(x, w, du, bias=None, state=None, *, silu=False, want_dstate=False
 
 def conv1d_step(x_t, w, state, bias=None, *, silu=False, u_t=None, stream=None):
     """One decode step of the conv: x_t [B, C]; state [B, C, W-1] shifts in place."""
+    if x_t.dim() != 2 or w.dim() != 2:
+        raise ValueError("x_t [B, C], w [C, W] expected")
     B, C = x_t.shape
     W = w.shape[1]
     _need(x_t, "x_t", x_t.dtype)
+    _need(w, "w", torch.float32, (C, W))
+    if bias is not None:
+        _need(bias, "bias", torch.float32, (C,))
     _need(state, "state", x_t.dtype, (B, C, W - 1))
+    _need_out(u_t, "u_t", x_t.dtype, (B, C))
     dims = _lib.FracConvDims(B, 1, C, W, _DT[x_t.dtype], _lib.FRAC_CONV_SILU if silu else 0)
     if u_t is None:
         u_t = torch.empty_like(x_t)
@@ -388,6 +398,10 @@ def gated_rmsnorm_fwd(y, z, weight, group_size=0, eps=1e-5, stream=None):
 def gated_rmsnorm_bwd(y, z, weight, dout, group_size=0, eps=1e-5, stream=None):
     """Backward of gated_rmsnorm_fwd.  Returns dict(dy, dz, dweight)."""
     dims = _norm_dims(y, group_size, eps)
+    _need(y, "y", y.dtype)
+    if z is not None:
+        _need(z, "z", y.dtype, y.shape)
+    _need(weight, "weight", torch.float32, (y.shape[1],))
     _need(dout, "dout", y.dtype, y.shape)
     g = dict(dy=torch.empty_like(y), dz=torch.empty_like(y) if z is not None else None,
              dweight=torch.empty_like(weight))

@@ -123,3 +123,26 @@ def test_decode_output_is_checked():
             Fake((H,), F32), Fake((BZ, H, K, P, N), F32))
     with pytest.raises(ValueError, match="y_t"):
         api.decode_step(*args, y_t=Fake((BZ, H, P + 1), BF))
+
+
+def test_glue_arguments_are_checked():
+    Bz, Lc, C, W = 2, 30, 72, 4
+    x = Fake((Bz, Lc, C), BF)
+    w = Fake((C, W), F32)
+    with pytest.raises(ValueError, match="w"):
+        api.conv1d_fwd(x, Fake((C, W), BF))
+    with pytest.raises(ValueError, match="bias"):
+        api.conv1d_fwd(x, w, Fake((C + 1,), F32))
+    with pytest.raises(ValueError, match="state"):
+        api.conv1d_bwd(x, w, Fake((Bz, Lc, C), BF), state=Fake((Bz, C, W), BF))
+    with pytest.raises(ValueError, match="du"):
+        api.conv1d_bwd(x, w, Fake((Bz, Lc - 1, C), BF))
+    with pytest.raises(ValueError, match="u_t"):
+        api.conv1d_step(Fake((Bz, C), BF), w, Fake((Bz, C, W - 1), BF), u_t=Fake((Bz, C + 8), BF))
+    with pytest.raises(ValueError, match="w"):
+        api.conv1d_step(Fake((Bz, C), BF), Fake((C - 8, W), F32), Fake((Bz, C, W - 1), BF))
+    y = Fake((16, 256), BF)
+    with pytest.raises(ValueError, match="weight"):
+        api.gated_rmsnorm_bwd(y, None, Fake((255,), F32), Fake((16, 256), BF))
+    with pytest.raises(ValueError, match="z"):
+        api.gated_rmsnorm_bwd(y, Fake((16, 256), F32), Fake((256,), F32), Fake((16, 256), BF))
