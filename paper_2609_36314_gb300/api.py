@@ -241,10 +241,23 @@ def _prep_dims(dt_raw, g_read, tau):
     if dt_raw.dim() < 1 or g_read.dim() != dt_raw.dim() + 1 or tau.dim() != 2:
         raise ValueError("dt_raw [..., H], g_read [..., H, K], tau [H, K] expected")
     H, K = tau.shape
-    if dt_raw.shape[-1] != H or g_read.shape[-1] != K:
-        raise ValueError("head / mode counts of dt_raw, g_read and tau differ")
+    if dt_raw.shape[-1] != H or g_read.shape[-1] != K or tuple(g_read.shape[:-1]) != tuple(dt_raw.shape):
+        raise ValueError("dt_raw [..., H], g_read [..., H, K] (the same leading dims) and tau [H, K] expected")
     rows = dt_raw.numel() // H
     return make_dims(1, rows, H, 1, 1, 1, K, g_read.dtype)
+
+
+def _need_prep_inputs(dt_raw, alpha_raw, lam_raw, g_read, g_write, tau, dt_bias):
+    f32 = torch.float32
+    _need(dt_raw, "dt_raw", f32)
+    _need(tau, "tau", f32)
+    if alpha_raw is not None:
+        _need(alpha_raw, "alpha_raw", f32, dt_raw.shape)
+    _need(lam_raw, "lam_raw", f32, dt_raw.shape)
+    _need(g_read, "g_read", g_read.dtype)
+    _need(g_write, "g_write", g_read.dtype, g_read.shape)
+    if dt_bias is not None:
+        _need(dt_bias, "dt_bias", f32, (tau.shape[0],))
 
 
 def param_prep_fwd(dt_raw, alpha_raw, lam_raw, g_read, g_write, tau, dt_bias=None, cfg=None,
@@ -254,15 +267,7 @@ def param_prep_fwd(dt_raw, alpha_raw, lam_raw, g_read, g_write, tau, dt_bias=Non
     cfg = cfg or prep_config()
     dims = _prep_dims(dt_raw, g_read, tau)
     f32 = torch.float32
-    for name, t in (("dt_raw", dt_raw), ("lam_raw", lam_raw), ("tau", tau)):
-        _need(t, name, f32)
-    if alpha_raw is not None:
-        _need(alpha_raw, "alpha_raw", f32, dt_raw.shape)
-    _need(lam_raw, "lam_raw", f32, dt_raw.shape)
-    _need(g_write, "g_write", g_read.dtype, g_read.shape)
-    _need(g_read, "g_read", g_read.dtype)
-    if dt_bias is not None:
-        _need(dt_bias, "dt_bias", f32, (tau.shape[0],))
+    _need_prep_inputs(dt_raw, alpha_raw, lam_raw, g_read, g_write, tau, dt_bias)
     if out is not None:
         for name in ("dt", "alpha", "lam"):
             _need(out.get(name), name, f32, dt_raw.shape)
@@ -287,6 +292,7 @@ def param_prep_bwd(dt_raw, alpha_raw, lam_raw, g_read, g_write, tau, ddt, dalpha
     cfg = cfg or prep_config()
     dims = _prep_dims(dt_raw, g_read, tau)
     f32 = torch.float32
+    _need_prep_inputs(dt_raw, alpha_raw, lam_raw, g_read, g_write, tau, dt_bias)
     for name, t in (("ddt", ddt), ("dalpha", dalpha), ("dlam", dlam)):
         _need(t, name, f32, dt_raw.shape)
     for name, t in (("dw_read", dw_read), ("dw_write", dw_write)):

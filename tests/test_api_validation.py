@@ -24,6 +24,12 @@ class Fake:
     def dim(self):
         return len(self.shape)
 
+    def numel(self):
+        n = 1
+        for v in self.shape:
+            n *= v
+        return n
+
 
 BZ, L, H, P, G, N, K = 2, 40, 4, 64, 1, 128, 8
 BF, F32 = torch.bfloat16, torch.float32
@@ -146,3 +152,29 @@ def test_glue_arguments_are_checked():
         api.gated_rmsnorm_bwd(y, None, Fake((255,), F32), Fake((16, 256), BF))
     with pytest.raises(ValueError, match="z"):
         api.gated_rmsnorm_bwd(y, Fake((16, 256), F32), Fake((256,), F32), Fake((16, 256), BF))
+
+
+def test_prep_arguments_are_checked():
+    Bz, Lp, Hp, Kp = 2, 9, 4, 8
+    dt_raw = Fake((Bz, Lp, Hp), F32)
+    g = Fake((Bz, Lp, Hp, Kp), BF)
+    tau = Fake((Hp, Kp), F32)
+    ok = dict(dt_raw=dt_raw, alpha_raw=Fake((Bz, Lp, Hp), F32), lam_raw=Fake((Bz, Lp, Hp), F32),
+              g_read=g, g_write=Fake((Bz, Lp, Hp, Kp), BF), tau=tau)
+    up = (Fake((Bz, Lp, Hp), F32), Fake((Bz, Lp, Hp), F32), Fake((Bz, Lp, Hp), F32),
+          Fake((Bz, Lp, Hp, Kp), BF), Fake((Bz, Lp, Hp, Kp), BF))
+    for name, bad in (("lam_raw", Fake((Bz, Lp + 1, Hp), F32)), ("g_write", Fake((Bz, Lp, Hp, Kp), F32)),
+                      ("g_read", Fake((Bz, Lp - 1, Hp, Kp), BF)), ("alpha_raw", Fake((Bz, Lp, Hp), BF))):
+        a = dict(ok, **{name: bad})
+        args = (a["dt_raw"], a["alpha_raw"], a["lam_raw"], a["g_read"], a["g_write"], a["tau"])
+        with pytest.raises(ValueError, match=name):
+            api.param_prep_fwd(*args)
+        with pytest.raises(ValueError, match=name):
+            api.param_prep_bwd(*args, *up)
+    args = (ok["dt_raw"], ok["alpha_raw"], ok["lam_raw"], ok["g_read"], ok["g_write"], ok["tau"])
+    with pytest.raises(ValueError, match="dt_bias"):
+        api.param_prep_bwd(*args, *up, dt_bias=Fake((Hp + 1,), F32))
+    with pytest.raises(ValueError, match="w_read"):
+        api.param_prep_fwd(*args, out=dict(dt=Fake((Bz, Lp, Hp), F32), alpha=Fake((Bz, Lp, Hp), F32),
+                                            lam=Fake((Bz, Lp, Hp), F32), w_read=Fake((Bz, Lp, Hp, 4), BF),
+                                            w_write=Fake((Bz, Lp, Hp, Kp), BF)))
