@@ -147,3 +147,48 @@ def test_plain_c_caller(tmp_path):
     out = subprocess.run([exe], capture_output=True, text=True, timeout=120)
     assert out.returncode == 0, out.stderr
     assert out.stdout.strip() == "ok"
+
+
+@pytest.mark.parametrize("case", ["conv_wide", "conv_zero_width", "conv_flag", "conv_null_x",
+                                  "conv_alias", "conv_bwd_null_dims", "step_null_state",
+                                  "norm_group", "norm_split", "norm_big", "norm_null_weight",
+                                  "norm_bwd_null_dz"])
+def test_glue_rejects_bad_arguments(case):
+    """The conv1d and gated RMSNorm calls check dims, flags, pointers and aliasing before
+    touching the device (each case fails validation, so nothing is launched)."""
+    lib = _lib.load()
+    p, q = ctypes.c_void_p(0x1000), ctypes.c_void_p(0x2000)
+    cd = _lib.FracConvDims(2, 16, 64, 4, 1, 0)
+    nd = _lib.FracNormDims(4, 64, 64, 1e-5, 1, 0)
+    if case == "conv_wide":
+        cd.width = 9
+        st, want = lib.frac_conv1d_fwd(ctypes.byref(cd), p, p, None, None, q, None, None), 2
+    elif case == "conv_zero_width":
+        cd.width = 0
+        st, want = lib.frac_conv1d_fwd(ctypes.byref(cd), p, p, None, None, q, None, None), 1
+    elif case == "conv_flag":
+        cd.flags = 2
+        st, want = lib.frac_conv1d_fwd(ctypes.byref(cd), p, p, None, None, q, None, None), 1
+    elif case == "conv_null_x":
+        st, want = lib.frac_conv1d_fwd(ctypes.byref(cd), None, p, None, None, q, None, None), 1
+    elif case == "conv_alias":
+        st, want = lib.frac_conv1d_fwd(ctypes.byref(cd), p, p, None, q, p, q, None), 1
+    elif case == "conv_bwd_null_dims":
+        st, want = lib.frac_conv1d_bwd(None, p, p, None, None, p, q, p, None, None, None), 1
+    elif case == "step_null_state":
+        st, want = lib.frac_conv1d_step(ctypes.byref(cd), p, p, None, None, q, None), 1
+    elif case == "norm_group":
+        nd.group_size = 12
+        st, want = lib.frac_gated_rmsnorm_fwd(ctypes.byref(nd), p, None, p, q, None), 1
+    elif case == "norm_split":
+        nd.dim, nd.group_size = 40, 16
+        st, want = lib.frac_gated_rmsnorm_fwd(ctypes.byref(nd), p, None, p, q, None), 1
+    elif case == "norm_big":
+        nd.dim, nd.group_size = 40000, 40000
+        st, want = lib.frac_gated_rmsnorm_fwd(ctypes.byref(nd), p, None, p, q, None), 2
+    elif case == "norm_null_weight":
+        st, want = lib.frac_gated_rmsnorm_fwd(ctypes.byref(nd), p, None, None, q, None), 1
+    else:  # a gate without its gradient
+        st, want = lib.frac_gated_rmsnorm_bwd(ctypes.byref(nd), p, p, p, p, q, None, p, None), 1
+    assert st == want
+    assert lib.frac_last_error()
